@@ -1,0 +1,276 @@
+/*
+ * tqfx4.h -- C ABI of libtqfx4, the GB300 (sm_103a) implementation of the
+ * tq2_0_fx4 integer dot pass and of the mixture-of-experts layers built on it.
+ *
+ * Paper: "Tied Trit-Planes: Constraining PTQTP to a Uniform Nine-Level
+ * Quantizer, with a Persistent Folded Format for Disk-Streamed
+ * Mixture-of-Experts Serving" (arXiv 2608.08910).
+ *
+ *   Sec. 2.1  Tying the two PTQTP scales at alpha = (3s, s) turns the pair of
+ *             trit planes t1, t2 in {-1, 0, 1} into one uniform nine-level
+ *             code c = 3 t1 + t2 in {-4, ..., 4}, with W_hat = s * c.
+ *   Sec. 2.2  tq2_0_fx4 stores c directly: one 520-byte block covers four
+ *             columns x 256 elements (512 code bytes, two codes per byte, plus
+ *             four f16 column scales), 4.0625 bits/weight. Codes decode by
+ *             arithmetic, are dotted against block-quantized activations with
+ *             integer arithmetic, and get one float multiply-add per block.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - W is a logical [N][K] fp32 weight (out x in, row-major); y = W x.
+ *    N must be a multiple of 4 (TQFX4_ROWS), K a multiple of 256 (TQFX4_QK).
+ *  - Block layout (the paper names the parts, not their order; this is the
+ *    library's reading): bytes 0..7 are the f16 scales d[0..3] of the block's
+ *    four rows, little endian; bytes 8 + 128 r .. 8 + 128 r + 127 hold row r's
+ *    codes, byte j carrying element j in its low nibble and element j + 128
+ *    in its high nibble. A nibble holds u = c + 4 in 0..8 (9..15 invalid).
+ *    A matrix is [N/4 row groups][K/256 blocks] of such blocks, contiguous.
+ *  - Activations are quantized per 256-element block: da = absmax / 127,
+ *    q = clamp(round(x / da), -127, 127) (x times the binary32 reciprocal of
+ *    da, rounded half away from zero), bsum = sum(q).
+ *  - The dot pass computes, per row n and block b, the exact integer
+ *    S[n][b] = sum_j c[n][256 b + j] q[256 b + j], then
+ *    y[n] = sum over b ascending of float(S) * (d[n][b] * da[b]) in binary32
+ *    with no fused multiply-add (a fixed float schedule).
+ *  - Memory: every pointer argument named as device memory must be device
+ *    memory (cudaMalloc or equivalent) owned by the caller. The library
+ *    allocates no device memory and keeps no state between calls. Host
+ *    structs passed by pointer (tqfx4_experts, tqfx4_router) are read during
+ *    the call only.
+ *  - Alignment: block arrays 16 bytes; fp32/int32 arrays 4 bytes; int8
+ *    activation arrays 16 bytes; the workspace 256 bytes.
+ *  - Streams: `stream` is a cudaStream_t (NULL = the legacy default stream).
+ *    Every call enqueues its kernels asynchronously on that stream and
+ *    returns. Argument errors are detected on the host before anything is
+ *    enqueued. Errors found by a kernel (invalid data, a bounded wait that
+ *    ran out) are recorded in the status word at the start of the workspace
+ *    `ws`; tqfx4_check() synchronizes the stream and reports them.
+ *  - Workspace: each call takes `ws`/`ws_bytes`, device memory of at least
+ *    the size its *_workspace_bytes query returns (TQFX4_STATUS_BYTES at
+ *    least). Zero it once (cudaMemset) before its first use; the library
+ *    keeps the status word and its counters consistent after that. Calls
+ *    that share a workspace must be ordered on one stream.
+ *  - Determinism: no output is produced with atomics; repeated calls on the
+ *    same inputs give bit-identical outputs, wherever the data sits in
+ *    memory (the "same bytes, same result" property of Sec. 2.2).
+ */
+#ifndef TQFX4_H
+#define TQFX4_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum tqfx4_status {
+    TQFX4_OK = 0,
+    TQFX4_EINVAL = 1,     /* null pointer, unknown enum value, negative size */
+    TQFX4_ESHAPE = 2,     /* N % 4, K % 256, top_k or expert count out of range */
+    TQFX4_EALIGN = 3,     /* a pointer violates its alignment rule */
+    TQFX4_EWORKSPACE = 4, /* ws smaller than the size query returned */
+    TQFX4_ECUDA = 5,      /* a CUDA runtime call or launch failed */
+    TQFX4_ETIMEOUT = 6,   /* a kernel's bounded wait ran out (from tqfx4_check) */
+    TQFX4_EDATA = 7       /* invalid data seen by a kernel: a trit outside
+                             {-1,0,1}, a non-finite weight or activation */
+} tqfx4_status;
+
+#define TQFX4_QK 256           /* elements per block along K (Sec. 2.2) */
+#define TQFX4_ROWS 4           /* rows ("columns") per block (Sec. 2.2) */
+#define TQFX4_BLOCK_BYTES 520  /* 8 scale bytes + 512 code bytes (Sec. 2.2) */
+#define TQFX4_STATUS_BYTES 256 /* status area at the start of every workspace */
+#define TQFX4_MAX_K 16384      /* largest K (hidden or intermediate size) */
+#define TQFX4_MAX_EXPERTS 1024
+#define TQFX4_MAX_TOP_K 16
+
+/* Sources for tqfx4_pack. */
+#define TQFX4_SRC_TRITS 0   /* fold two trit planes with given f16 scales */
+#define TQFX4_SRC_F32_RTN 1 /* round-to-nearest codes from fp32 weights */
+
+/* Paths for tqfx4_moe_grouped. */
+#define TQFX4_PATH_AUTO 0    /* DECODE for small token counts, else PREFILL */
+#define TQFX4_PATH_DECODE 1  /* per-expert grouped GEMV (weights read once) */
+#define TQFX4_PATH_PREFILL 2 /* per-expert grouped GEMM on tensor cores */
+
+/* Bytes of one N x K matrix: (N/4) * (K/256) * 520 (Sec. 2.2: 4.0625
+ * bits/weight). Returns -1 if N % 4 or K % 256 or a size is negative. */
+int64_t tqfx4_matrix_bytes(int64_t n, int64_t k);
+
+/* Workspace bytes for tqfx4_pack, tqfx4_quantize_act and tqfx4_gemv
+ * (the status area only). */
+size_t tqfx4_basic_workspace_bytes(void);
+
+/*
+ * tqfx4_pack -- write blocks for an N x K matrix (Sec. 2.1 fold, Sec. 2.2
+ * layout).
+ *   src == TQFX4_SRC_TRITS: a = t1 (int8 [n][k], device), t2 = int8 [n][k]
+ *     (device), scales_f16 = f16 bit patterns [n][k/256] (device). Each code
+ *     is c = 3 t1 + t2. A trit outside {-1, 0, 1} sets TQFX4_EDATA.
+ *   src == TQFX4_SRC_F32_RTN: a = W (fp32 [n][k], device); t2 and
+ *     scales_f16 must be NULL. Per (row, block): d = f16(absmax / 4)
+ *     (round to nearest even, saturated at 65504), c = clamp(round(w /
+ *     float(d)), -4, 4) computed as w times the binary32 reciprocal of the
+ *     f16-rounded scale, rounded half away from zero; d = 0 gives c = 0. A
+ *     non-finite weight sets TQFX4_EDATA.
+ *   blocks: device, tqfx4_matrix_bytes(n, k) bytes, 16-byte aligned, written
+ *     completely. n == 0 or k == 0 writes nothing.
+ */
+tqfx4_status tqfx4_pack(int src, const void *a, const int8_t *t2, const uint16_t *scales_f16,
+                        int64_t n, int64_t k, void *blocks,
+                        void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * tqfx4_quantize_act -- per-256-block int8 activation quantization (Sec. 2.2,
+ * "block-quantized activations"). x: fp32 [m][k] (device). Outputs (device):
+ * q int8 [m][k] (16-byte aligned), da fp32 [m][k/256], bsum int32
+ * [m][k/256]. A non-finite input sets TQFX4_EDATA.
+ */
+tqfx4_status tqfx4_quantize_act(const float *x, int64_t m, int64_t k,
+                                int8_t *q, float *da, int32_t *bsum,
+                                void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * tqfx4_gemv -- the integer dot pass (Sec. 2.2): y = W x for one activation
+ * vector already quantized by tqfx4_quantize_act.
+ *   blocks: device, the N x K matrix. q, da, bsum: device, one vector
+ *   (k, k/256, k/256 entries). y: fp32 [n] (device).
+ *   block_sums: nullable; if given, int32 [n][k/256] (device) receives the
+ *   exact integer block sums S[n][b].
+ *   k == 0 gives y = 0; n == 0 does nothing.
+ */
+tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k,
+                        const int8_t *q, const float *da, const int32_t *bsum,
+                        float *y, int32_t *block_sums,
+                        void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * Routed experts: gate and up are [n_experts] stacked matrices of shape
+ * inter x hidden, down is [n_experts] stacked matrices of shape hidden x
+ * inter, each expert's matrix at base + e * tqfx4_matrix_bytes(...) (one
+ * expert-projection is one contiguous byte range, Sec. 1 and 2.2). Device
+ * pointers, 16-byte aligned.
+ */
+typedef struct tqfx4_experts {
+    const void *gate;
+    const void *up;
+    const void *down;
+    int64_t n_experts; /* 1 .. TQFX4_MAX_EXPERTS */
+    int64_t hidden;    /* multiple of 256, <= TQFX4_MAX_K */
+    int64_t inter;     /* multiple of 256, <= TQFX4_MAX_K */
+} tqfx4_experts;
+
+/*
+ * Router: logits = W_r x + bias in fp32; the top_k experts by logit (ties
+ * go to the lower expert index) in descending order; weights = softmax over
+ * the selected logits (the renormalized top-k of the full softmax). The
+ * paper does not describe the router; this is the standard top-k router.
+ */
+typedef struct tqfx4_router {
+    const float *weight; /* [n_experts][hidden] fp32, device */
+    const float *bias;   /* nullable [n_experts] fp32, device; added before selection */
+    int32_t top_k;       /* 1 .. min(n_experts, TQFX4_MAX_TOP_K) */
+} tqfx4_router;
+
+/* Workspace bytes for tqfx4_moe_ffn (tokens == 1, path ignored) or
+ * tqfx4_moe_grouped with `tokens` tokens on `path`. Returns 0 if the shapes
+ * are invalid. */
+size_t tqfx4_moe_workspace_bytes(const tqfx4_experts *ex, const tqfx4_router *rt,
+                                 int64_t tokens, int path);
+
+/*
+ * tqfx4_moe_ffn -- one token through a routed-expert MoE layer:
+ *   route x (fp32 logits, top-k, renormalized weights); quantize x once;
+ *   for each selected expert j: g = gate_j x, u = up_j x (dot pass),
+ *   h = silu(g) * u, quantize h, o_j = down_j h (dot pass);
+ *   out = sum over j in rank order of w_j * o_j (binary32, fixed order).
+ * SwiGLU is evaluated in binary32 as g / (1 + exp(-g)) * u with exp computed
+ * by Cody-Waite reduction and a degree-7 Taylor polynomial, so that the int8
+ * re-quantization of h is reproducible bit for bit.
+ * Only the selected experts' blocks are read.
+ *   x, out: fp32 [hidden] (device). sel_idx int32 [top_k], sel_w fp32
+ *   [top_k] (device) receive the routing decision.
+ */
+tqfx4_status tqfx4_moe_ffn(const tqfx4_experts *ex, const tqfx4_router *rt,
+                           const float *x, float *out, int32_t *sel_idx, float *sel_w,
+                           void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * tqfx4_moe_grouped -- T tokens through the same MoE layer, grouped by
+ * expert: route all tokens, count (token, slot) pairs per expert, exclusive
+ * scan, stable gather (ascending token order within each expert), run each
+ * touched expert once over all of its tokens (its weights are read once),
+ * then combine each token's expert outputs in rank order. Results equal
+ * tqfx4_moe_ffn applied to each token.
+ *   X, OUT: fp32 [T][hidden] (device). sel_idx int32 [T][top_k], sel_w fp32
+ *   [T][top_k] (device). T == 0 does nothing.
+ */
+tqfx4_status tqfx4_moe_grouped(const tqfx4_experts *ex, const tqfx4_router *rt,
+                               const float *X, int64_t T, float *OUT,
+                               int32_t *sel_idx, float *sel_w, int path,
+                               void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * Profiling variants: identical to the calls above, and additionally record
+ * `events[i]` (cudaEvent_t, created by the caller) on the stream before
+ * stage i, and events[n_stages] after the last stage, where n_stages is
+ * given by tqfx4_moe_stage_count. Stage names come from
+ * tqfx4_moe_stage_name.
+ */
+int tqfx4_moe_stage_count(int grouped, int path);
+const char *tqfx4_moe_stage_name(int grouped, int path, int stage);
+tqfx4_status tqfx4_moe_ffn_traced(const tqfx4_experts *ex, const tqfx4_router *rt,
+                                  const float *x, float *out, int32_t *sel_idx, float *sel_w,
+                                  void *ws, size_t ws_bytes, void *stream, void *const *events);
+tqfx4_status tqfx4_moe_grouped_traced(const tqfx4_experts *ex, const tqfx4_router *rt,
+                                      const float *X, int64_t T, float *OUT,
+                                      int32_t *sel_idx, float *sel_w, int path,
+                                      void *ws, size_t ws_bytes, void *stream,
+                                      void *const *events);
+
+/*
+ * Byte offsets, from the start of the workspace, of the intermediates a MoE
+ * call leaves there (for inspection and tests; valid after the call's
+ * stream work completes). Entries that a path does not produce are
+ * SIZE_MAX. P = T * top_k (token, slot) pairs; pairs are ordered by expert
+ * then token for the grouped call, by rank for tqfx4_moe_ffn.
+ */
+typedef struct tqfx4_moe_views {
+    size_t logits;     /* fp32 [T][n_experts] */
+    size_t qx;         /* int8 [T][hidden] */
+    size_t dx;         /* fp32 [T][hidden/256] */
+    size_t bx;         /* int32 [T][hidden/256] */
+    size_t g;          /* fp32 [P][inter] */
+    size_t u;          /* fp32 [P][inter] */
+    size_t h;          /* fp32 [P][inter] */
+    size_t qh;         /* int8 [P][inter] */
+    size_t dh;         /* fp32 [P][inter/256] */
+    size_t bh;         /* int32 [P][inter/256] */
+    size_t o;          /* fp32 [P][hidden]: each pair's expert output */
+    size_t counts;     /* int32 [n_experts] (grouped only) */
+    size_t offsets;    /* int32 [n_experts + 1] (grouped only) */
+    size_t pair_token; /* int32 [P] (grouped only) */
+    size_t pair_slot;  /* int32 [P] (grouped only) */
+} tqfx4_moe_views;
+
+tqfx4_status tqfx4_moe_workspace_views(const tqfx4_experts *ex, const tqfx4_router *rt,
+                                       int64_t tokens, int grouped, int path,
+                                       tqfx4_moe_views *views);
+
+/*
+ * tqfx4_check -- synchronize `stream`, read the status word in `ws` and
+ * clear it. Returns TQFX4_OK, the first device-side error recorded since
+ * the last check (TQFX4_EDATA, TQFX4_ETIMEOUT), or TQFX4_ECUDA if the
+ * stream reports a CUDA error.
+ */
+tqfx4_status tqfx4_check(void *ws, void *stream);
+
+/* Message for the last error returned on the calling host thread. */
+const char *tqfx4_last_error(void);
+const char *tqfx4_status_string(tqfx4_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TQFX4_H */

@@ -1,0 +1,542 @@
+/*
+ * tqfx4 oracle: a plain, slow, single-threaded CPU restatement of the
+ * tied trit-plane (tq2_0_fx4) integer dot pass and of the mixture-of-experts
+ * decode math built on it.
+ *
+ * THIS IS TEST INFRASTRUCTURE. Only the test suite, the smoke check and the
+ * benchmark's CPU-baseline leg load it. The product path (the CUDA library)
+ * neither links nor calls it, and shares no header, table or helper with it.
+ *
+ * Build: gcc -std=c11 -O2 -ffp-contract=off -fPIC -shared (no intrinsics,
+ * no SIMD, no OpenMP). Every float operation is a single IEEE binary32
+ * operation with round-to-nearest-even; no fused multiply-add is allowed, so
+ * the results are identical on x86-64 and aarch64.
+ *
+ * Paper references are to "Tied Trit-Planes" (arXiv 2608.08910):
+ *   Sec. 2.1  the tie alpha = (3s, s): W_hat = s * c, c = 3 t1 + t2 in {-4..4}
+ *   Sec. 2.2  the persistent folded format: a 520-byte block covers four
+ *             columns x 256 elements, 512 code bytes (two codes per byte) plus
+ *             four f16 column scales, 4.0625 bits/weight; codes decode by
+ *             arithmetic; integer dot against block-quantized activations;
+ *             one float multiply-add per block; a shared float schedule.
+ * Readings where the paper is silent (byte order inside the block, nibble
+ * encoding, activation block size and scale type, the router and SwiGLU
+ * arithmetic) are stated at each function.
+ *
+ * Parity status: every function here is pinned by the CPU test suite
+ * (closed forms, brute force, library routines); none is "parity unpinned".
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define QK 256          /* elements per block along K (Sec. 2.2) */
+#define ROWS 4          /* output rows ("columns") per block (Sec. 2.2) */
+#define BLOCK_BYTES 520 /* 8 scale bytes + 512 code bytes (Sec. 2.2) */
+#define CODE_OFS 8      /* reading: the four f16 scales come first */
+#define ROW_CODE_BYTES 128
+
+/* ------------------------------------------------------------------ */
+/* Sec. 2.1: the fold. c = 3 t1 + t2, t1, t2 in {-1, 0, 1}.            */
+/* ------------------------------------------------------------------ */
+
+/* Returns c in -4..4, or -100 if a trit is outside {-1, 0, 1}. */
+int tqo_fold(int t1, int t2) {
+    if (t1 < -1 || t1 > 1 || t2 < -1 || t2 > 1) return -100;
+    return 3 * t1 + t2;
+}
+
+/* Inverse of the fold (balanced ternary, two digits): t2 is the balanced
+ * residue of c modulo 3, t1 the remaining digit. Returns 0, or -1 if c is
+ * outside -4..4. */
+int tqo_unfold(int c, int *t1, int *t2) {
+    if (c < -4 || c > 4) return -1;
+    int r = ((c % 3) + 3) % 3;   /* 0, 1, 2 */
+    int d2 = (r == 2) ? -1 : r;  /* balanced digit -1, 0, 1 */
+    *t2 = d2;
+    *t1 = (c - d2) / 3;
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* IEEE 754 binary16, written out from the format definition.           */
+/* ------------------------------------------------------------------ */
+
+/* float -> binary16, round to nearest, ties to even; overflow gives inf. */
+uint16_t tqo_f32_to_f16(float f) {
+    uint32_t x;
+    memcpy(&x, &f, 4);
+    uint32_t sign = (x >> 16) & 0x8000u;
+    uint32_t ex = (x >> 23) & 0xffu;
+    uint32_t man = x & 0x7fffffu;
+    if (ex == 0xffu) return (uint16_t)(sign | 0x7c00u | (man ? 0x200u : 0u));
+    int e = (int)ex - 127 + 15;
+    if (e >= 31) return (uint16_t)(sign | 0x7c00u);
+    if (e <= 0) {
+        if (e < -10) return (uint16_t)sign;
+        uint32_t m = man | 0x800000u;
+        int shift = 14 - e;
+        uint32_t h = m >> shift;
+        uint32_t rem = m & ((1u << shift) - 1u);
+        uint32_t half = 1u << (shift - 1);
+        if (rem > half || (rem == half && (h & 1u))) h++;
+        return (uint16_t)(sign | h);
+    }
+    uint32_t h = ((uint32_t)e << 10) | (man >> 13);
+    uint32_t rem = man & 0x1fffu;
+    if (rem > 0x1000u || (rem == 0x1000u && (h & 1u))) h++;
+    return (uint16_t)(sign | h);
+}
+
+float tqo_f16_to_f32(uint16_t h) {
+    int sign = (h >> 15) & 1;
+    int ex = (h >> 10) & 0x1f;
+    int man = h & 0x3ff;
+    double v;
+    if (ex == 0) v = ldexp((double)man, -24);
+    else if (ex == 31) v = man ? NAN : INFINITY;
+    else v = ldexp((double)(1024 + man), ex - 25);
+    return (float)(sign ? -v : v);
+}
+
+/* ------------------------------------------------------------------ */
+/* Sec. 2.2: the 520-byte block.                                        */
+/* Reading of the byte order (the paper names the parts but not their   */
+/* order): bytes 0..7 hold the four f16 scales d[r] of rows r = 0..3    */
+/* (little endian); bytes 8 + 128 r .. 8 + 128 r + 127 hold row r's 256  */
+/* codes, byte j carrying element j in its low nibble and element       */
+/* j + 128 in its high nibble. A nibble stores u = c + 4 in 0..8          */
+/* (values 9..15 are invalid). Blocks of a matrix W[N][K] are ordered    */
+/* [N/4 row groups][K/256 blocks].                                       */
+/* ------------------------------------------------------------------ */
+
+int64_t tqo_matrix_bytes(int64_t n, int64_t k) {
+    if (n < 0 || k < 0 || n % ROWS || k % QK) return -1;
+    return (n / ROWS) * (k / QK) * BLOCK_BYTES;
+}
+
+static uint8_t *block_at(uint8_t *blocks, int64_t k, int64_t n, int64_t kk) {
+    int64_t nb = k / QK;
+    return blocks + ((n / ROWS) * nb + kk / QK) * BLOCK_BYTES;
+}
+
+static const uint8_t *cblock_at(const uint8_t *blocks, int64_t k, int64_t n, int64_t kk) {
+    int64_t nb = k / QK;
+    return blocks + ((n / ROWS) * nb + kk / QK) * BLOCK_BYTES;
+}
+
+static void put_scale(uint8_t *blk, int r, uint16_t d) {
+    blk[2 * r] = (uint8_t)(d & 0xff);
+    blk[2 * r + 1] = (uint8_t)(d >> 8);
+}
+
+static uint16_t get_scale(const uint8_t *blk, int r) {
+    return (uint16_t)(blk[2 * r] | (blk[2 * r + 1] << 8));
+}
+
+static void put_code(uint8_t *blk, int r, int j, int c) {
+    uint8_t *p = blk + CODE_OFS + ROW_CODE_BYTES * r + (j % ROW_CODE_BYTES);
+    uint8_t u = (uint8_t)(c + 4);
+    if (j < ROW_CODE_BYTES) *p = (uint8_t)((*p & 0xf0) | u);
+    else *p = (uint8_t)((*p & 0x0f) | (u << 4));
+}
+
+/* Returns the nibble u (0..15); the caller maps it to c = u - 4. */
+static int get_nibble(const uint8_t *blk, int r, int j) {
+    const uint8_t *p = blk + CODE_OFS + ROW_CODE_BYTES * r + (j % ROW_CODE_BYTES);
+    return (j < ROW_CODE_BYTES) ? (*p & 0x0f) : (*p >> 4);
+}
+
+/* Fold two trit planes into blocks (Sec. 2.1 and 2.2): c = 3 t1 + t2 with the
+ * given f16 scale per (row, 256-block). t1, t2: int8 [n][k]; d: [n][k/256].
+ * Returns 0, -1 on a bad shape, -2 on a trit outside {-1, 0, 1}. */
+int tqo_pack_trits(const int8_t *t1, const int8_t *t2, const uint16_t *d,
+                   int64_t n, int64_t k, uint8_t *out) {
+    if (tqo_matrix_bytes(n, k) < 0) return -1;
+    int64_t nb = k / QK;
+    memset(out, 0, (size_t)tqo_matrix_bytes(n, k));
+    for (int64_t row = 0; row < n; row++) {
+        for (int64_t b = 0; b < nb; b++) {
+            uint8_t *blk = block_at(out, k, row, b * QK);
+            put_scale(blk, (int)(row % ROWS), d[row * nb + b]);
+            for (int j = 0; j < QK; j++) {
+                int64_t i = row * k + b * QK + j;
+                int c = tqo_fold(t1[i], t2[i]);
+                if (c == -100) return -2;
+                put_code(blk, (int)(row % ROWS), j, c);
+            }
+        }
+    }
+    return 0;
+}
+
+/* Round-to-nearest codes from fp32 weights. Per (row, 256-block):
+ *   d  = f16(absmax / 4)           (saturated to the largest finite f16)
+ *   dq = float(d)                   (codes use the stored, f16-rounded scale)
+ *   c  = clamp(round(w * (1/dq)), -4, 4), round = half away from zero,
+ * with dq = 0 giving every code 0. W_hat = dq * c is the tied quantizer of
+ * Sec. 2.1 fitted in one step. Returns 0, -1 on a bad shape, -3 on a
+ * non-finite weight. */
+int tqo_pack_rtn(const float *w, int64_t n, int64_t k, uint8_t *out) {
+    if (tqo_matrix_bytes(n, k) < 0) return -1;
+    int64_t nb = k / QK;
+    memset(out, 0, (size_t)tqo_matrix_bytes(n, k));
+    for (int64_t row = 0; row < n; row++) {
+        for (int64_t b = 0; b < nb; b++) {
+            const float *src = w + row * k + b * QK;
+            float amax = 0.0f;
+            for (int j = 0; j < QK; j++) {
+                if (!isfinite(src[j])) return -3;
+                float a = fabsf(src[j]);
+                if (a > amax) amax = a;
+            }
+            uint16_t d = tqo_f32_to_f16(amax / 4.0f);
+            if ((d & 0x7c00u) == 0x7c00u) d = 0x7bffu; /* saturate */
+            float dq = tqo_f16_to_f32(d);
+            float id = (dq != 0.0f) ? 1.0f / dq : 0.0f;
+            uint8_t *blk = block_at(out, k, row, b * QK);
+            put_scale(blk, (int)(row % ROWS), d);
+            for (int j = 0; j < QK; j++) {
+                float v = roundf(src[j] * id);
+                if (v > 4.0f) v = 4.0f;
+                if (v < -4.0f) v = -4.0f;
+                put_code(blk, (int)(row % ROWS), j, (int)v);
+            }
+        }
+    }
+    return 0;
+}
+
+/* Decode blocks back to codes c[n][k] (c = u - 4, "by arithmetic") and
+ * scales d[n][k/256]. Returns 0, -1 on a bad shape, -4 on a nibble > 8. */
+int tqo_unpack(const uint8_t *blocks, int64_t n, int64_t k, int8_t *c, uint16_t *d) {
+    if (tqo_matrix_bytes(n, k) < 0) return -1;
+    int64_t nb = k / QK;
+    for (int64_t row = 0; row < n; row++) {
+        for (int64_t b = 0; b < nb; b++) {
+            const uint8_t *blk = cblock_at(blocks, k, row, b * QK);
+            if (d) d[row * nb + b] = get_scale(blk, (int)(row % ROWS));
+            for (int j = 0; j < QK; j++) {
+                int u = get_nibble(blk, (int)(row % ROWS), j);
+                if (u > 8) return -4;
+                c[row * k + b * QK + j] = (int8_t)(u - 4);
+            }
+        }
+    }
+    return 0;
+}
+
+/* Dequantized weights W_hat = s * c (Sec. 2.1), in fp64. */
+int tqo_dequant(const uint8_t *blocks, int64_t n, int64_t k, double *w_hat) {
+    if (tqo_matrix_bytes(n, k) < 0) return -1;
+    int64_t nb = k / QK;
+    for (int64_t row = 0; row < n; row++) {
+        for (int64_t b = 0; b < nb; b++) {
+            const uint8_t *blk = cblock_at(blocks, k, row, b * QK);
+            double s = (double)tqo_f16_to_f32(get_scale(blk, (int)(row % ROWS)));
+            for (int j = 0; j < QK; j++) {
+                int u = get_nibble(blk, (int)(row % ROWS), j);
+                if (u > 8) return -4;
+                w_hat[row * k + b * QK + j] = s * (double)(u - 4);
+            }
+        }
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* Sec. 2.2: block-quantized activations. Reading: 256-element blocks    */
+/* aligned with the weight blocks, symmetric int8 in -127..127, one fp32 */
+/* scale per block:                                                      */
+/*   da = absmax / 127, q = clamp(round(x * (1/da)), -127, 127),          */
+/*   bsum = sum(q) (the offset-binary dot needs it).                      */
+/* x: [m][k]; q: [m][k]; da, bsum: [m][k/256].                          */
+/* Returns 0, -1 on a bad shape, -3 on a non-finite input.               */
+/* ------------------------------------------------------------------ */
+int tqo_quantize_act(const float *x, int64_t m, int64_t k, int8_t *q, float *da, int32_t *bsum) {
+    if (m < 0 || k < 0 || k % QK) return -1;
+    int64_t nb = k / QK;
+    for (int64_t t = 0; t < m; t++) {
+        for (int64_t b = 0; b < nb; b++) {
+            const float *src = x + t * k + b * QK;
+            float amax = 0.0f;
+            for (int j = 0; j < QK; j++) {
+                if (!isfinite(src[j])) return -3;
+                float a = fabsf(src[j]);
+                if (a > amax) amax = a;
+            }
+            float s = amax / 127.0f;
+            float id = (s != 0.0f) ? 1.0f / s : 0.0f;
+            int32_t sum = 0;
+            for (int j = 0; j < QK; j++) {
+                float v = roundf(src[j] * id);
+                if (v > 127.0f) v = 127.0f;
+                if (v < -127.0f) v = -127.0f;
+                q[t * k + b * QK + j] = (int8_t)v;
+                sum += (int32_t)v;
+            }
+            da[t * nb + b] = s;
+            bsum[t * nb + b] = sum;
+        }
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* Sec. 2.2: the integer dot pass.                                       */
+/*   S[n][b] = sum_{j<256} c[n][256 b + j] * q[256 b + j]   (exact int)   */
+/*   y[n]    = sum over b ascending of float(S) * (d[n][b] * da[b])       */
+/* The float schedule is fixed: acc starts at +0.0f and, for b = 0, 1,    */
+/* ..., acc = acc + float(S) * (dq * da) with each operation rounded to   */
+/* binary32 (no fused multiply-add). Returns 0, -1 on a bad shape, -4 on  */
+/* an invalid nibble.                                                     */
+/* ------------------------------------------------------------------ */
+int tqo_block_sums(const uint8_t *blocks, int64_t n, int64_t k, const int8_t *q, int32_t *S) {
+    if (tqo_matrix_bytes(n, k) < 0) return -1;
+    int64_t nb = k / QK;
+    for (int64_t row = 0; row < n; row++) {
+        for (int64_t b = 0; b < nb; b++) {
+            const uint8_t *blk = cblock_at(blocks, k, row, b * QK);
+            int32_t s = 0;
+            for (int j = 0; j < QK; j++) {
+                int u = get_nibble(blk, (int)(row % ROWS), j);
+                if (u > 8) return -4;
+                s += (int32_t)(u - 4) * (int32_t)q[b * QK + j];
+            }
+            S[row * nb + b] = s;
+        }
+    }
+    return 0;
+}
+
+int tqo_gemv(const uint8_t *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
+             float *y, int32_t *S_out) {
+    if (tqo_matrix_bytes(n, k) < 0) return -1;
+    int64_t nb = k / QK;
+    int32_t *S = S_out ? S_out : (int32_t *)malloc(sizeof(int32_t) * (size_t)(n * nb + 1));
+    if (!S) return -5;
+    int rc = tqo_block_sums(blocks, n, k, q, S);
+    if (rc == 0) {
+        for (int64_t row = 0; row < n; row++) {
+            float acc = 0.0f;
+            for (int64_t b = 0; b < nb; b++) {
+                const uint8_t *blk = cblock_at(blocks, k, row, b * QK);
+                float dq = tqo_f16_to_f32(get_scale(blk, (int)(row % ROWS)));
+                float sc = dq * da[b];
+                float t = (float)S[row * nb + b] * sc;
+                acc = acc + t;
+            }
+            y[row] = acc;
+        }
+    }
+    if (!S_out) free(S);
+    return rc;
+}
+
+/* ------------------------------------------------------------------ */
+/* exp in binary32 (used by SwiGLU). The paper does not fix how SwiGLU   */
+/* is evaluated; because its output is re-quantized to int8 (a rounding  */
+/* decision), both this oracle and the kernel evaluate it with the same  */
+/* fully specified binary32 method, each from its own source:            */
+/* Cody-Waite range reduction z = n ln2 + r with ln2 split into          */
+/* 0.693359375 + (-2.12194440e-4) (the Cephes split), |r| <= ln2/2, then */
+/* the degree-7 Taylor polynomial of e^r in Horner form, scaled by 2^n.  */
+/* Inputs are clamped to [-87, 88] so the result stays a normal number.  */
+/* ------------------------------------------------------------------ */
+float tqo_expf(float z) {
+    if (z != z) return z;
+    if (z > 88.0f) z = 88.0f;
+    if (z < -87.0f) z = -87.0f;
+    float t = z * 1.44269502f; /* log2(e) rounded to binary32 */
+    float nf = rintf(t);
+    float r = z - nf * 0.693359375f;
+    r = r - nf * -2.12194440e-4f;
+    float p = 1.98412698e-4f;        /* 1/7! */
+    p = p * r + 1.38888889e-3f;      /* 1/6! */
+    p = p * r + 8.33333333e-3f;      /* 1/5! */
+    p = p * r + 4.16666667e-2f;      /* 1/4! */
+    p = p * r + 1.66666667e-1f;      /* 1/3! */
+    p = p * r + 0.5f;                /* 1/2! */
+    p = p * r + 1.0f;
+    p = p * r + 1.0f;
+    return ldexpf(p, (int)nf);
+}
+
+/* SwiGLU: h = silu(g) * u with silu(g) = g / (1 + exp(-g)), binary32. */
+void tqo_swiglu(const float *g, const float *u, int64_t n, float *h) {
+    for (int64_t i = 0; i < n; i++) {
+        float e = tqo_expf(-g[i]);
+        float den = 1.0f + e;
+        float s = g[i] / den;
+        h[i] = s * u[i];
+    }
+}
+
+/* ------------------------------------------------------------------ */
+/* One routed expert (gate/up/down SwiGLU FFN, the projections the paper */
+/* stores in tq2_0_fx4): x [hidden] -> out [hidden].                       */
+/*   qx = quant(x); g = gemv(gate, qx); u = gemv(up, qx);                  */
+/*   h = swiglu(g, u); qh = quant(h); out = gemv(down, qh).                */
+/* gate, up: [inter][hidden]; down: [hidden][inter]. Optional debug        */
+/* outputs (nullable): g, u, h [inter]; qh [inter]; dh, bh [inter/256].    */
+/* ------------------------------------------------------------------ */
+int tqo_expert_ffn(const uint8_t *gate, const uint8_t *up, const uint8_t *down,
+                   int64_t hidden, int64_t inter, const float *x, float *out,
+                   float *g_dbg, float *u_dbg, float *h_dbg, int8_t *qh_dbg,
+                   float *dh_dbg, int32_t *bh_dbg) {
+    if (hidden % QK || inter % QK || hidden <= 0 || inter <= 0) return -1;
+    int64_t nbh = hidden / QK, nbi = inter / QK;
+    int8_t *qx = (int8_t *)malloc((size_t)hidden);
+    float *dx = (float *)malloc(sizeof(float) * (size_t)nbh);
+    int32_t *bx = (int32_t *)malloc(sizeof(int32_t) * (size_t)nbh);
+    float *g = (float *)malloc(sizeof(float) * (size_t)inter);
+    float *u = (float *)malloc(sizeof(float) * (size_t)inter);
+    float *h = (float *)malloc(sizeof(float) * (size_t)inter);
+    int8_t *qh = (int8_t *)malloc((size_t)inter);
+    float *dh = (float *)malloc(sizeof(float) * (size_t)nbi);
+    int32_t *bh = (int32_t *)malloc(sizeof(int32_t) * (size_t)nbi);
+    int rc = -5;
+    if (qx && dx && bx && g && u && h && qh && dh && bh) {
+        rc = tqo_quantize_act(x, 1, hidden, qx, dx, bx);
+        if (!rc) rc = tqo_gemv(gate, inter, hidden, qx, dx, g, NULL);
+        if (!rc) rc = tqo_gemv(up, inter, hidden, qx, dx, u, NULL);
+        if (!rc) {
+            tqo_swiglu(g, u, inter, h);
+            rc = tqo_quantize_act(h, 1, inter, qh, dh, bh);
+        }
+        if (!rc) rc = tqo_gemv(down, hidden, inter, qh, dh, out, NULL);
+        if (!rc) {
+            if (g_dbg) memcpy(g_dbg, g, sizeof(float) * (size_t)inter);
+            if (u_dbg) memcpy(u_dbg, u, sizeof(float) * (size_t)inter);
+            if (h_dbg) memcpy(h_dbg, h, sizeof(float) * (size_t)inter);
+            if (qh_dbg) memcpy(qh_dbg, qh, (size_t)inter);
+            if (dh_dbg) memcpy(dh_dbg, dh, sizeof(float) * (size_t)nbi);
+            if (bh_dbg) memcpy(bh_dbg, bh, sizeof(int32_t) * (size_t)nbi);
+        }
+    }
+    free(qx); free(dx); free(bx); free(g); free(u); free(h); free(qh); free(dh); free(bh);
+    return rc;
+}
+
+/* ------------------------------------------------------------------ */
+/* Router (the paper does not describe it; this is the standard MoE      */
+/* router that the workload names): logits in fp64,                       */
+/*   l[e] = sum_k W_r[e][k] x[k] + bias[e],                               */
+/* the top_k experts by logit (ties to the lower index), in rank order,   */
+/* and w_j = exp(l_j - l_0) / sum_i exp(l_i - l_0) over the selected ones */
+/* (equal to renormalizing the top-k of a full softmax), rounded to fp32. */
+/* W_r: [E][H]; bias nullable [E]; logits (nullable) [E]; idx, w [top_k]. */
+/* ------------------------------------------------------------------ */
+int tqo_router(const float *Wr, const float *bias, int64_t E, int64_t H, const float *x,
+               int top_k, double *logits_out, int32_t *idx, float *w) {
+    if (E <= 0 || H <= 0 || top_k <= 0 || top_k > E) return -1;
+    double *l = (double *)malloc(sizeof(double) * (size_t)E);
+    char *taken = (char *)calloc((size_t)E, 1);
+    if (!l || !taken) { free(l); free(taken); return -5; }
+    for (int64_t e = 0; e < E; e++) {
+        double acc = 0.0;
+        for (int64_t kk = 0; kk < H; kk++) acc += (double)Wr[e * H + kk] * (double)x[kk];
+        if (bias) acc += (double)bias[e];
+        l[e] = acc;
+    }
+    for (int j = 0; j < top_k; j++) {
+        int64_t best = -1;
+        for (int64_t e = 0; e < E; e++) {
+            if (taken[e]) continue;
+            if (best < 0 || l[e] > l[best]) best = e; /* strict: ties keep the lower index */
+        }
+        taken[best] = 1;
+        idx[j] = (int32_t)best;
+    }
+    double m = l[idx[0]], sum = 0.0;
+    for (int j = 0; j < top_k; j++) sum += exp(l[idx[j]] - m);
+    for (int j = 0; j < top_k; j++) w[j] = (float)(exp(l[idx[j]] - m) / sum);
+    if (logits_out) memcpy(logits_out, l, sizeof(double) * (size_t)E);
+    free(l); free(taken);
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* MoE layer for one token: route, run each selected expert, combine in  */
+/* rank order: out[n] = sum over j = 0..top_k-1 of w_j * o_j[n], fp32,    */
+/* acc starting at +0.0f, acc = acc + w_j * o_j[n] (no fused multiply-add).*/
+/* Experts are given as per-expert pointer arrays; an entry may be NULL   */
+/* for an expert the token does not select (returns -6 if it does).       */
+/* ------------------------------------------------------------------ */
+int tqo_moe_token(const uint8_t *const *gate, const uint8_t *const *up, const uint8_t *const *down,
+                  int64_t E, int64_t hidden, int64_t inter, const float *Wr, const float *bias,
+                  int top_k, const float *x, float *out, int32_t *idx, float *w) {
+    int rc = tqo_router(Wr, bias, E, hidden, x, top_k, NULL, idx, w);
+    if (rc) return rc;
+    float *o = (float *)malloc(sizeof(float) * (size_t)hidden);
+    if (!o) return -5;
+    for (int64_t n = 0; n < hidden; n++) out[n] = 0.0f;
+    for (int j = 0; j < top_k; j++) {
+        int32_t e = idx[j];
+        if (!gate[e] || !up[e] || !down[e]) { free(o); return -6; }
+        rc = tqo_expert_ffn(gate[e], up[e], down[e], hidden, inter, x, o,
+                            NULL, NULL, NULL, NULL, NULL, NULL);
+        if (rc) { free(o); return rc; }
+        for (int64_t n = 0; n < hidden; n++) {
+            float t = w[j] * o[n];
+            out[n] = out[n] + t;
+        }
+    }
+    free(o);
+    return 0;
+}
+
+/* Batched MoE: by definition, each of the T tokens independently through
+ * tqo_moe_token. X, OUT: [T][hidden]; idx, w: [T][top_k]. */
+int tqo_moe_tokens(const uint8_t *const *gate, const uint8_t *const *up, const uint8_t *const *down,
+                   int64_t E, int64_t hidden, int64_t inter, const float *Wr, const float *bias,
+                   int top_k, const float *X, int64_t T, float *OUT, int32_t *idx, float *w) {
+    for (int64_t t = 0; t < T; t++) {
+        int rc = tqo_moe_token(gate, up, down, E, hidden, inter, Wr, bias, top_k,
+                               X + t * hidden, OUT + t * hidden, idx + t * top_k, w + t * top_k);
+        if (rc) return rc;
+    }
+    return 0;
+}
+
+/* Token gather per expert (the grouping step of batched decode/prefill):
+ * counts[e] = number of (token, slot) pairs routed to e; offsets = exclusive
+ * prefix sum of counts; pairs are listed expert by expert, and within an
+ * expert by ascending token (then slot). pair_token, pair_slot: [T*top_k];
+ * offsets: [E+1]. Returns 0, or -1 on an index outside 0..E-1. */
+int tqo_group_by_expert(const int32_t *idx, int64_t T, int top_k, int64_t E,
+                        int32_t *counts, int32_t *offsets, int32_t *pair_token, int32_t *pair_slot) {
+    for (int64_t e = 0; e < E; e++) counts[e] = 0;
+    for (int64_t i = 0; i < T * top_k; i++) {
+        if (idx[i] < 0 || idx[i] >= E) return -1;
+        counts[idx[i]]++;
+    }
+    offsets[0] = 0;
+    for (int64_t e = 0; e < E; e++) offsets[e + 1] = offsets[e] + counts[e];
+    int64_t p = 0;
+    for (int64_t e = 0; e < E; e++)
+        for (int64_t t = 0; t < T; t++)
+            for (int j = 0; j < top_k; j++)
+                if (idx[t * top_k + j] == e) {
+                    pair_token[p] = (int32_t)t;
+                    pair_slot[p] = j;
+                    p++;
+                }
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* Array helpers for the test harness (element-wise, no new arithmetic). */
+/* ------------------------------------------------------------------ */
+void tqo_f32_to_f16_n(const float *x, int64_t n, uint16_t *h) {
+    for (int64_t i = 0; i < n; i++) h[i] = tqo_f32_to_f16(x[i]);
+}
+
+void tqo_f16_to_f32_n(const uint16_t *h, int64_t n, float *x) {
+    for (int64_t i = 0; i < n; i++) x[i] = tqo_f16_to_f32(h[i]);
+}
+
+void tqo_expf_n(const float *z, int64_t n, float *y) {
+    for (int64_t i = 0; i < n; i++) y[i] = tqo_expf(z[i]);
+}
