@@ -1,0 +1,253 @@
+// Device-side building blocks shared by the tqfx4 kernels (sm_103a only):
+// the block geometry of tq2_0_fx4 (Tied Trit-Planes, Sec. 2.2), the device
+// status word, mbarrier + cp.async.bulk staging, and the integer dot step.
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "tqfx4.h"
+
+#if defined(__CUDA_ARCH__) && (__CUDA_ARCH__ < 1000)
+#error "libtqfx4 targets Blackwell (sm_103a) only"
+#endif
+
+namespace tq {
+
+constexpr int QK = 256;           // elements per block along K
+constexpr int ROWS = 4;           // rows per block
+constexpr int BLOCK_BYTES = 520;  // 8 scale bytes + 4 x 128 code bytes
+constexpr int CODE_OFS = 8;       // codes follow the four f16 scales
+constexpr int ROW_BYTES = 128;    // code bytes per row (256 nibbles)
+constexpr int QS_STRIDE = 264;    // shared-memory stride of one 256-byte activation block
+                                  // (33 x 8 bytes: consecutive blocks land on distinct banks)
+
+// Kernel ids recorded with a device error (status word slot 1).
+enum KernelId : int {
+    K_PACK = 1, K_QUANT = 2, K_GEMV = 3, K_ROUTER = 4, K_GATEUP = 5, K_DOWN = 6,
+    K_TOPK = 7, K_GROUP = 8, K_GGATEUP = 9, K_GDOWN = 10, K_COMBINE = 11, K_PREFILL = 12,
+};
+
+// Roughly two seconds at the GB300's 2 GHz clock: any mbarrier wait longer
+// than this is treated as lost, reported, and abandoned.
+constexpr long long kWaitBudgetCycles = 4000000000LL;
+
+__host__ __device__ __forceinline__ int64_t imin64(int64_t a, int64_t b) { return a < b ? a : b; }
+__host__ __device__ __forceinline__ int64_t imax64(int64_t a, int64_t b) { return a > b ? a : b; }
+
+__device__ __forceinline__ void report(int *status, int code, int kernel, int detail) {
+    if (atomicCAS(status, 0, code) == 0) {
+        atomicExch(status + 1, kernel);
+        atomicExch(status + 2, detail);
+    }
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// ---- mbarrier ---------------------------------------------------------------
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ uint32_t mbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok;
+}
+
+// Waits for phase `parity` of `bar` to complete; gives up after
+// kWaitBudgetCycles and returns false.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const long long t0 = clock64();
+    while (true) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (clock64() - t0 > kWaitBudgetCycles) return false;
+    }
+}
+
+// One-dimensional bulk copy global -> shared, completing on `bar`
+// (dst and src 16-byte aligned, bytes a multiple of 16).
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// Stage `bytes` (a multiple of 8) of global memory starting at the 8-byte
+// aligned `src` into the 16-byte aligned shared buffer `dst`, on barrier
+// `bar`, issued by one warp. The data lands at dst + (src & 15): its 16-byte
+// aligned interior goes by one cp.async.bulk, a leading or trailing 8-byte
+// piece by ordinary loads (visible to the warp after the wait plus
+// __syncwarp). Returns the offset of the data inside `dst`.
+__device__ __forceinline__ uint32_t stage_range(int lane, uint8_t *dst, const uint8_t *src, uint32_t bytes,
+                                                uint64_t *bar) {
+    const uint32_t o = static_cast<uint32_t>(reinterpret_cast<uintptr_t>(src) & 15u);
+    const uint32_t head = (o != 0u && bytes >= 8u) ? 8u : 0u;
+    const uint32_t body = ((bytes - head) / 16u) * 16u;
+    const uint32_t tail = bytes - head - body;
+    if (lane == 0) {
+        mbar_arrive_expect_tx(bar, body);
+        if (body) bulk_g2s(dst + o + head, src + head, body, bar);
+    } else if (lane == 1 && head) {
+        *reinterpret_cast<uint2 *>(dst + o) = __ldg(reinterpret_cast<const uint2 *>(src));
+    } else if (lane == 2 && tail) {
+        *reinterpret_cast<uint2 *>(dst + o + head + body) =
+            __ldg(reinterpret_cast<const uint2 *>(src + head + body));
+    }
+    return o;
+}
+
+// ---- integer dot step ----------------------------------------------------------
+
+// d = c + dot(bytes of a as unsigned, bytes of b as signed)
+__device__ __forceinline__ int dp4a_us(uint32_t a, uint32_t b, int c) {
+    int d;
+    asm("dp4a.u32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+
+// Exact block sums S[r] = sum_j c[r][j] q[j] of one 520-byte block whose code
+// bytes start at `codes` (8-byte aligned, shared memory) against one 256-byte
+// activation block `qb` (8-byte aligned, shared memory) with sum `bsum`.
+// Nibbles hold u = c + 4, so S = sum u q - 4 bsum. Low nibbles (elements
+// j) are taken in place; high nibbles (elements j + 128) are kept at 16 u
+// and divided out at the end (the sum is an exact multiple of 16).
+__device__ __forceinline__ void block_dot(const uint8_t *codes, const uint8_t *qb, int bsum, int S[4]) {
+    const uint2 *c2 = reinterpret_cast<const uint2 *>(codes);
+    const uint2 *q2 = reinterpret_cast<const uint2 *>(qb);
+    int lo[4] = {0, 0, 0, 0}, hi[4] = {0, 0, 0, 0};
+#pragma unroll 4
+    for (int w = 0; w < 16; ++w) {
+        const uint2 qa = q2[w];
+        const uint2 qh = q2[16 + w];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const uint2 c = c2[r * 16 + w];
+            lo[r] = dp4a_us(c.x & 0x0f0f0f0fu, qa.x, lo[r]);
+            lo[r] = dp4a_us(c.y & 0x0f0f0f0fu, qa.y, lo[r]);
+            hi[r] = dp4a_us(c.x & 0xf0f0f0f0u, qh.x, hi[r]);
+            hi[r] = dp4a_us(c.y & 0xf0f0f0f0u, qh.y, hi[r]);
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < 4; ++r) S[r] = lo[r] + (hi[r] >> 4) - 4 * bsum;
+}
+
+// Scale of row r (0..3) of the block at `blk` (shared memory), as fp32.
+__device__ __forceinline__ float block_scale(const uint8_t *blk, int r) {
+    const __half h = *reinterpret_cast<const __half *>(blk + 2 * r);
+    return __half2float(h);
+}
+
+// Copy one quantized activation vector (q: k bytes, 16-byte aligned; da,
+// bsum: k/256 entries) into shared memory with the padded block stride,
+// cooperatively by the whole thread block.
+__device__ __forceinline__ void load_act_smem(const int8_t *q, const float *da, const int32_t *bsum, int nb,
+                                              uint8_t *qs, float *das, int *bss) {
+    const int chunks = nb * 16;  // 16-byte chunks
+    for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
+        const int b = c >> 4, w = c & 15;
+        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(q) + c);
+        uint2 *dst = reinterpret_cast<uint2 *>(qs + b * QS_STRIDE + w * 16);
+        dst[0] = make_uint2(v.x, v.y);
+        dst[1] = make_uint2(v.z, v.w);
+    }
+    for (int b = threadIdx.x; b < nb; b += blockDim.x) {
+        das[b] = __ldg(da + b);
+        bss[b] = __ldg(bsum + b);
+    }
+}
+
+// ---- binary32 helpers with a fixed operation order ------------------------------
+
+// exp in binary32: Cody-Waite reduction z = n ln2 + r (ln2 split as
+// 0.693359375 + -2.12194440e-4, the Cephes split), degree-7 Taylor polynomial
+// of e^r in Horner form, scaled by 2^n; inputs clamped to [-87, 88]. Every
+// step is one correctly rounded binary32 operation (no contraction), so the
+// result is reproducible on any IEEE binary32 machine.
+__device__ __forceinline__ float tq_expf(float z) {
+    if (z != z) return z;
+    z = fminf(fmaxf(z, -87.0f), 88.0f);
+    const float t = __fmul_rn(z, 1.44269502f);
+    const float nf = rintf(t);
+    float r = __fsub_rn(z, __fmul_rn(nf, 0.693359375f));
+    r = __fsub_rn(r, __fmul_rn(nf, -2.12194440e-4f));
+    float p = 1.98412698e-4f;
+    p = __fadd_rn(__fmul_rn(p, r), 1.38888889e-3f);
+    p = __fadd_rn(__fmul_rn(p, r), 8.33333333e-3f);
+    p = __fadd_rn(__fmul_rn(p, r), 4.16666667e-2f);
+    p = __fadd_rn(__fmul_rn(p, r), 1.66666667e-1f);
+    p = __fadd_rn(__fmul_rn(p, r), 0.5f);
+    p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+    p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+    return ldexpf(p, static_cast<int>(nf));
+}
+
+// h = silu(g) * u = g / (1 + exp(-g)) * u in binary32.
+__device__ __forceinline__ float tq_swiglu(float g, float u) {
+    const float e = tq_expf(-g);
+    const float s = __fdiv_rn(g, __fadd_rn(1.0f, e));
+    return __fmul_rn(s, u);
+}
+
+// Quantization of one 256-element activation block held by a warp, 8
+// consecutive elements per lane (lane l holds elements 8l .. 8l+7):
+// da = absmax / 127, q = clamp(round(x * (1/da)), -127, 127), bsum = sum q.
+// Returns false if an element is not finite.
+__device__ __forceinline__ bool quant_block_warp(const float v[8], uint2 &packed, float &da_out, int &bsum_out) {
+    bool finite = true;
+    float amax = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        finite &= isfinite(v[i]);
+        amax = fmaxf(amax, fabsf(v[i]));
+    }
+#pragma unroll
+    for (int s = 16; s > 0; s >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, s));
+    const float da = __fdiv_rn(amax, 127.0f);
+    const float id = (da != 0.0f) ? __fdiv_rn(1.0f, da) : 0.0f;
+    int sum = 0;
+    uint32_t w[2] = {0u, 0u};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        float t = roundf(__fmul_rn(v[i], id));
+        t = fminf(fmaxf(t, -127.0f), 127.0f);
+        const int qi = finite ? static_cast<int>(t) : 0;
+        sum += qi;
+        w[i >> 2] |= (static_cast<uint32_t>(qi) & 0xffu) << (8 * (i & 3));
+    }
+#pragma unroll
+    for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+    packed = make_uint2(w[0], w[1]);
+    da_out = da;
+    bsum_out = sum;
+    return __all_sync(0xffffffffu, finite);
+}
+
+}  // namespace tq

@@ -1,0 +1,54 @@
+"""Tensor-allocating conveniences over the C ABI (binding.py).
+
+Each helper allocates its outputs with torch on the inputs' device and makes
+exactly one library call; none computes anything itself.
+"""
+import torch
+
+from . import binding as B
+
+
+def workspace(nbytes: int, device="cuda") -> torch.Tensor:
+    """Zeroed device workspace (torch allocations are 256-byte aligned)."""
+    n = max(int(nbytes), B.TQFX4_STATUS_BYTES)
+    return torch.zeros(((n + 255) // 256) * 256, dtype=torch.uint8, device=device)
+
+
+def empty_blocks(n: int, k: int, device="cuda", count: int = 1) -> torch.Tensor:
+    nbytes = B.tqfx4_matrix_bytes(n, k)
+    if nbytes < 0:
+        raise ValueError("bad shape %dx%d" % (n, k))
+    return torch.empty(count * nbytes, dtype=torch.uint8, device=device)
+
+
+def pack_rtn(w: torch.Tensor, ws: torch.Tensor, out: torch.Tensor = None) -> torch.Tensor:
+    n, k = w.shape
+    blocks = empty_blocks(n, k, w.device) if out is None else out
+    B.tqfx4_pack(B.TQFX4_SRC_F32_RTN, w, None, None, n, k, blocks, ws)
+    return blocks
+
+
+def pack_trits(t1, t2, scales_f16, ws) -> torch.Tensor:
+    n, k = t1.shape
+    blocks = empty_blocks(n, k, t1.device)
+    B.tqfx4_pack(B.TQFX4_SRC_TRITS, t1, t2, scales_f16, n, k, blocks, ws)
+    return blocks
+
+
+def quantize_act(x: torch.Tensor, ws: torch.Tensor):
+    x2 = x.reshape(-1, x.shape[-1])
+    m, k = x2.shape
+    q = torch.empty((m, k), dtype=torch.int8, device=x.device)
+    da = torch.empty((m, k // 256), dtype=torch.float32, device=x.device)
+    bs = torch.empty((m, k // 256), dtype=torch.int32, device=x.device)
+    B.tqfx4_quantize_act(x2, m, k, q, da, bs, ws)
+    if x.dim() == 1:
+        return q[0], da[0], bs[0]
+    return q, da, bs
+
+
+def gemv(blocks, n: int, k: int, q, da, bsum, ws, block_sums: bool = False):
+    y = torch.empty(n, dtype=torch.float32, device=blocks.device)
+    S = torch.empty((n, k // 256), dtype=torch.int32, device=blocks.device) if block_sums else None
+    B.tqfx4_gemv(blocks, n, k, q, da, bsum, y, S, ws)
+    return (y, S) if block_sums else y
