@@ -161,10 +161,14 @@ typedef struct tqfx4_experts {
 } tqfx4_experts;
 
 /*
- * Router: logits = W_r x + bias in fp32; the top_k experts by logit (ties
- * go to the lower expert index) in descending order; weights = softmax over
- * the selected logits (the renormalized top-k of the full softmax). The
- * paper does not describe the router; this is the standard top-k router.
+ * Router: logits = W_r x + bias, evaluated with a compensated binary32 dot
+ * product (Ogita-Rump-Oishi Dot2) and kept as double-binary32 pairs (about
+ * 44 significant bits); the top_k experts by logit (ties go to the lower
+ * expert index) in descending order; weights = softmax over the selected
+ * logits (the renormalized top-k of the full softmax), evaluated in
+ * double-binary32 and rounded once to binary32, so they agree with a binary64
+ * evaluation. The paper does not describe the router; this is the standard
+ * top-k router.
  */
 typedef struct tqfx4_router {
     const float *weight; /* [n_experts][hidden] fp32, device */
@@ -236,7 +240,8 @@ tqfx4_status tqfx4_moe_grouped_traced(const tqfx4_experts *ex, const tqfx4_route
  * then token for the grouped call, by rank for tqfx4_moe_ffn.
  */
 typedef struct tqfx4_moe_views {
-    size_t logits;     /* fp32 [T][n_experts] */
+    size_t logits;     /* fp32 [T][n_experts]: high part of each logit */
+    size_t logits_lo;  /* fp32 [T][n_experts]: low part (logit = hi + lo exactly) */
     size_t qx;         /* int8 [T][hidden] */
     size_t dx;         /* fp32 [T][hidden/256] */
     size_t bx;         /* int32 [T][hidden/256] */

@@ -5,6 +5,7 @@
 #include <cstring>
 
 #include "tq_launch.h"
+#include "tq_moe_common.cuh"
 #include "tqfx4.h"
 
 namespace {
@@ -112,6 +113,133 @@ tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
     cudaError_t e = tq::launch_gemv(blocks, n, k, q, da, bsum, y, block_sums, static_cast<int *>(ws),
                                     static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "tqfx4_gemv");
+    return ok();
+}
+
+
+// ---------------------------------------------------------------- MoE
+
+namespace {
+
+tqfx4_status check_moe_shapes(const tqfx4_experts *ex, const tqfx4_router *rt, const char *fn) {
+    if (!ex || !rt) return fail(TQFX4_EINVAL, "%s: NULL experts or router", fn);
+    if (ex->n_experts < 1 || ex->n_experts > TQFX4_MAX_EXPERTS)
+        return fail(TQFX4_ESHAPE, "%s: n_experts=%lld outside 1..%d", fn, (long long)ex->n_experts,
+                    TQFX4_MAX_EXPERTS);
+    if (ex->hidden <= 0 || ex->inter <= 0 || ex->hidden % 256 || ex->inter % 256 || ex->hidden > TQFX4_MAX_K ||
+        ex->inter > TQFX4_MAX_K)
+        return fail(TQFX4_ESHAPE, "%s: hidden=%lld, inter=%lld must be positive multiples of 256 <= %d", fn,
+                    (long long)ex->hidden, (long long)ex->inter, TQFX4_MAX_K);
+    if (rt->top_k < 1 || rt->top_k > TQFX4_MAX_TOP_K || rt->top_k > ex->n_experts)
+        return fail(TQFX4_ESHAPE, "%s: top_k=%d outside 1..min(n_experts, %d)", fn, rt->top_k, TQFX4_MAX_TOP_K);
+    return TQFX4_OK;
+}
+
+tqfx4_status check_moe_ptrs(const tqfx4_experts *ex, const tqfx4_router *rt, const char *fn) {
+    if (!ex->gate || !ex->up || !ex->down || !rt->weight) return fail(TQFX4_EINVAL, "%s: NULL weights", fn);
+    if (!aligned(ex->gate, 16) || !aligned(ex->up, 16) || !aligned(ex->down, 16) || !aligned(rt->weight, 16) ||
+        !aligned(rt->bias, 4))
+        return fail(TQFX4_EALIGN, "%s: expert and router weights must be 16-byte aligned", fn);
+    return TQFX4_OK;
+}
+
+}  // namespace
+
+size_t tqfx4_moe_workspace_bytes(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t tokens, int path) {
+    (void)path;
+    if (check_moe_shapes(ex, rt, "tqfx4_moe_workspace_bytes") || tokens < 0) return 0;
+    const int64_t T = tokens < 1 ? 1 : tokens;
+    const size_t dec = tq::moe_layout(ex->n_experts, ex->hidden, ex->inter, rt->top_k, 1, false, true).total;
+    const size_t grp = tq::moe_layout(ex->n_experts, ex->hidden, ex->inter, rt->top_k, T, true, true).total;
+    return tokens <= 1 ? (dec > grp ? dec : grp) : grp;
+}
+
+int tqfx4_moe_stage_count(int grouped, int path) {
+    (void)path;
+    return grouped ? 0 : 3;
+}
+
+const char *tqfx4_moe_stage_name(int grouped, int path, int stage) {
+    (void)path;
+    static const char *dec[] = {"router", "gate_up", "down"};
+    if (!grouped && stage >= 0 && stage < 3) return dec[stage];
+    return "";
+}
+
+static tqfx4_status moe_ffn_impl(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, float *out,
+                                 int32_t *sel_idx, float *sel_w, void *ws, size_t ws_bytes, void *stream,
+                                 void *const *events) {
+    const char *fn = "tqfx4_moe_ffn";
+    tqfx4_status s = check_moe_shapes(ex, rt, fn);
+    if (s) return s;
+    if ((s = check_moe_ptrs(ex, rt, fn))) return s;
+    if (!x || !out || !sel_idx || !sel_w) return fail(TQFX4_EINVAL, "%s: NULL x, out or selection output", fn);
+    if (!aligned(x, 16) || !aligned(out, 4) || !aligned(sel_idx, 4) || !aligned(sel_w, 4))
+        return fail(TQFX4_EALIGN, "%s: x must be 16-byte aligned", fn);
+    tq::MoeArgs a;
+    tq::MoeLayout L;
+    if (!tq::moe_decode_args(ex, rt, nullptr, a, L))
+        return fail(TQFX4_ESHAPE, "%s: too many row ranges for the counter area", fn);
+    if ((s = check_ws(ws, ws_bytes, L.total, fn))) return s;
+    if (tq::gate_up_smem(a) > tq::max_smem_optin() || tq::down_smem(a) > tq::max_smem_optin())
+        return fail(TQFX4_ESHAPE, "%s: top_k x inter too large for the decode kernels' shared memory", fn);
+    tq::moe_decode_args(ex, rt, ws, a, L);
+    cudaError_t e = tq::launch_moe_decode(a, x, out, sel_idx, sel_w, static_cast<cudaStream_t>(stream), events);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
+tqfx4_status tqfx4_moe_ffn(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, float *out,
+                           int32_t *sel_idx, float *sel_w, void *ws, size_t ws_bytes, void *stream) {
+    return moe_ffn_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, nullptr);
+}
+
+tqfx4_status tqfx4_moe_ffn_traced(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, float *out,
+                                  int32_t *sel_idx, float *sel_w, void *ws, size_t ws_bytes, void *stream,
+                                  void *const *events) {
+    return moe_ffn_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, events);
+}
+
+tqfx4_status tqfx4_moe_grouped(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X, int64_t T,
+                               float *OUT, int32_t *sel_idx, float *sel_w, int path, void *ws, size_t ws_bytes,
+                               void *stream) {
+    (void)X; (void)T; (void)OUT; (void)sel_idx; (void)sel_w; (void)path; (void)ws; (void)ws_bytes; (void)stream;
+    (void)ex; (void)rt;
+    return fail(TQFX4_EINVAL, "tqfx4_moe_grouped: not available in this build");
+}
+
+tqfx4_status tqfx4_moe_grouped_traced(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X, int64_t T,
+                                      float *OUT, int32_t *sel_idx, float *sel_w, int path, void *ws,
+                                      size_t ws_bytes, void *stream, void *const *events) {
+    (void)events;
+    return tqfx4_moe_grouped(ex, rt, X, T, OUT, sel_idx, sel_w, path, ws, ws_bytes, stream);
+}
+
+tqfx4_status tqfx4_moe_workspace_views(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t tokens,
+                                       int grouped, int path, tqfx4_moe_views *v) {
+    (void)path;
+    const char *fn = "tqfx4_moe_workspace_views";
+    tqfx4_status s = check_moe_shapes(ex, rt, fn);
+    if (s) return s;
+    if (!v) return fail(TQFX4_EINVAL, "%s: NULL views", fn);
+    const int64_t T = grouped ? tokens : 1;
+    const tq::MoeLayout L = tq::moe_layout(ex->n_experts, ex->hidden, ex->inter, rt->top_k, T, grouped != 0, true);
+    v->logits = L.logits;
+    v->logits_lo = L.logits_lo;
+    v->qx = L.qx;
+    v->dx = L.dx;
+    v->bx = L.bx;
+    v->g = L.g;
+    v->u = L.u;
+    v->h = L.h;
+    v->qh = L.qh;
+    v->dh = L.dh;
+    v->bh = L.bh;
+    v->o = L.o;
+    v->counts = L.counts;
+    v->offsets = L.offsets;
+    v->pair_token = L.pair_token;
+    v->pair_slot = L.pair_slot;
     return ok();
 }
 

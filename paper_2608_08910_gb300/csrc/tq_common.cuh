@@ -15,6 +15,23 @@
 
 namespace tq {
 
+// Phase timestamps for development builds (-DTQ_INSTRUMENT): thread 0 of a
+// CTA records %globaltimer into tq_stamps[kernel][cta][slot]. Compiled out
+// otherwise.
+#ifdef TQ_INSTRUMENT
+extern __device__ unsigned long long tq_stamps[8][2048][8];
+#define TQ_STAMP(k, s)                                                                              \
+    do {                                                                                            \
+        if (threadIdx.x == 0 && blockIdx.x < 2048) {                                                \
+            unsigned long long t_;                                                                  \
+            asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));                                  \
+            tq_stamps[k][blockIdx.x][s] = t_;                                                       \
+        }                                                                                           \
+    } while (0)
+#else
+#define TQ_STAMP(k, s) ((void)0)
+#endif
+
 constexpr int QK = 256;           // elements per block along K
 constexpr int ROWS = 4;           // rows per block
 constexpr int BLOCK_BYTES = 520;  // 8 scale bytes + 4 x 128 code bytes
@@ -184,6 +201,72 @@ __device__ __forceinline__ void load_act_smem(const int8_t *q, const float *da, 
     }
 }
 
+// Activation vector staged through registers: loads issued early (ahead of
+// bulk weight copies in the memory queues), stored to shared memory later.
+// Holds nb <= 64 blocks for thread blocks of at least 128 threads.
+struct ActRegs {
+    uint4 q[8];
+    float da;
+    int bs;
+};
+
+__device__ __forceinline__ void act_load(const int8_t *q, const float *da, const int32_t *bsum, int nb, ActRegs &r) {
+    const int chunks = nb * 16;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const int c = threadIdx.x + i * blockDim.x;
+        if (c < chunks) r.q[i] = __ldcg(reinterpret_cast<const uint4 *>(q) + c);
+    }
+    if (static_cast<int>(threadIdx.x) < nb) {
+        r.da = __ldcg(da + threadIdx.x);
+        r.bs = __ldcg(bsum + threadIdx.x);
+    }
+}
+
+__device__ __forceinline__ void act_store(const ActRegs &r, int nb, uint8_t *qs, float *das, int *bss) {
+    const int chunks = nb * 16;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const int c = threadIdx.x + i * blockDim.x;
+        if (c < chunks) {
+            uint2 *dst = reinterpret_cast<uint2 *>(qs + (c >> 4) * QS_STRIDE + (c & 15) * 16);
+            dst[0] = make_uint2(r.q[i].x, r.q[i].y);
+            dst[1] = make_uint2(r.q[i].z, r.q[i].w);
+        }
+    }
+    if (static_cast<int>(threadIdx.x) < nb) {
+        das[threadIdx.x] = r.da;
+        bss[threadIdx.x] = r.bs;
+    }
+}
+
+// ---- inter-kernel ordering ----------------------------------------------------------
+
+// Programmatic dependent launch: wait until the preceding kernel in the
+// stream has completed and its writes are visible (a no-op when the kernel
+// was launched without the programmatic-serialization attribute).
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Allow the next kernel in the stream (if launched as a programmatic
+// dependent) to start launching.
+__device__ __forceinline__ void grid_dependents_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// atomicAdd with acquire-release semantics at GPU scope: orders this
+// thread's earlier writes before the add and later reads after it.
+__device__ __forceinline__ int atomic_add_acq_rel(int *p, int v) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
+// First row group of part p when n_rg row groups, in units of rpu, are split
+// into `parts` nearly equal parts.
+__host__ __device__ inline int64_t part_begin(int64_t n_rg, int rpu, int parts, int p) {
+    const int64_t units = (n_rg + rpu - 1) / rpu;
+    const int64_t u = units * p / parts;
+    return imin64(n_rg, u * rpu);
+}
+
 // ---- binary32 helpers with a fixed operation order ------------------------------
 
 // exp in binary32: Cody-Waite reduction z = n ln2 + r (ln2 split as
@@ -206,7 +289,10 @@ __device__ __forceinline__ float tq_expf(float z) {
     p = __fadd_rn(__fmul_rn(p, r), 0.5f);
     p = __fadd_rn(__fmul_rn(p, r), 1.0f);
     p = __fadd_rn(__fmul_rn(p, r), 1.0f);
-    return ldexpf(p, static_cast<int>(nf));
+    // p * 2^n as one correctly rounded multiplication (n in -126..127, so 2^n
+    // is a normal binary32 built from its exponent bits)
+    const float two_n = __int_as_float((static_cast<int>(nf) + 127) << 23);
+    return __fmul_rn(p, two_n);
 }
 
 // h = silu(g) * u = g / (1 + exp(-g)) * u in binary32.

@@ -5,10 +5,13 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "tqfx4.h"
+
 namespace tq {
 
 int num_sms();
 int max_smem_optin();
+cudaError_t allow_max_smem(const void *kernel, unsigned char *flags);
 
 cudaError_t launch_pack(int src, const void *a, const int8_t *t2, const uint16_t *scales, int64_t n, int64_t k,
                         void *blocks, int *status, cudaStream_t st);
@@ -16,5 +19,13 @@ cudaError_t launch_quantize(const float *x, int64_t m, int64_t k, int8_t *q, flo
                             int *status, cudaStream_t st);
 cudaError_t launch_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
                         const int32_t *bsum, float *y, int32_t *block_sums, int *status, cudaStream_t st);
+
+struct MoeArgs;
+struct MoeLayout;
+bool moe_decode_args(const tqfx4_experts *ex, const tqfx4_router *rt, void *ws, MoeArgs &a, MoeLayout &L);
+cudaError_t launch_moe_decode(const MoeArgs &a, const float *x, float *out, int32_t *sel_idx, float *sel_w,
+                              cudaStream_t st, void *const *events);
+int gate_up_smem(const MoeArgs &a);
+int down_smem(const MoeArgs &a);
 
 }  // namespace tq

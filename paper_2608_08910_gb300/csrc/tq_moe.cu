@@ -1,26 +1,373 @@
-// Mixture-of-experts entry points (work in progress).
+// tqfx4_moe_ffn: one token through a routed-expert MoE layer whose gate/up/
+// down projections are tq2_0_fx4 matrices (Tied Trit-Planes, Sec. 1 and 2.2).
+//
+// Three launches, reading only the selected experts' bytes:
+//   router   one CTA per expert: logit W_r[e] x + bias[e] by a compensated
+//            binary32 dot product kept as a double-binary32 pair; extra CTAs
+//            quantize x. The CTA that finishes last (one counter) selects
+//            the top-k experts.
+//   gate_up  CTA (j, p) streams row range p of selected expert j's gate and
+//            up matrices (tq_stream.cuh) and writes g_j and u_j; no CTA
+//            depends on another.
+//   down     CTA (j, p) issues its first weight copies (the selection is
+//            known), then forms h_j = silu(g_j) u_j and quantizes it into
+//            shared memory while one warp evaluates the softmax weights,
+//            streams row range p of down_j and writes o_j. The last of the
+//            top_k CTAs sharing row range p (one counter per range) combines
+//            out = sum_j w_j o_j in rank order.
+// gate_up and down are launched as programmatic dependents: each starts its
+// prologue while its predecessor drains and waits (griddepcontrol.wait)
+// before reading what the predecessor wrote.
+// Counters only decide which CTA finishes a reduction; every output is a
+// fixed sequence of binary32 operations, so results are bit-reproducible.
 #include "tq_launch.h"
-#include "tqfx4.h"
+#include "tq_stream.cuh"
 
-extern "C" {
-size_t tqfx4_moe_workspace_bytes(const tqfx4_experts *, const tqfx4_router *, int64_t, int) { return 0; }
-tqfx4_status tqfx4_moe_ffn(const tqfx4_experts *, const tqfx4_router *, const float *, float *, int32_t *,
-                           float *, void *, size_t, void *) { return TQFX4_EINVAL; }
-tqfx4_status tqfx4_moe_grouped(const tqfx4_experts *, const tqfx4_router *, const float *, int64_t, float *,
-                               int32_t *, float *, int, void *, size_t, void *) { return TQFX4_EINVAL; }
-int tqfx4_moe_stage_count(int, int) { return 0; }
-const char *tqfx4_moe_stage_name(int, int, int) { return ""; }
-tqfx4_status tqfx4_moe_ffn_traced(const tqfx4_experts *, const tqfx4_router *, const float *, float *,
-                                  int32_t *, float *, void *, size_t, void *, void *const *) {
-    return TQFX4_EINVAL;
+namespace tq {
+
+// Counter slots at the start of the workspace's counter area.
+constexpr int kCtrRouter = 0;  // router CTAs done
+constexpr int kCtrDown = 1;    // down: one counter per row range
+
+// ---------------------------------------------------------------- router
+
+__global__ void __launch_bounds__(128) router_kernel(MoeArgs a) {
+    TQ_STAMP(0, 0);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    __shared__ float part_hi[4], part_lo[4];
+    __shared__ int last;
+    __shared__ TopkScratch topk_s;
+    if (static_cast<int>(blockIdx.x) >= a.E) {
+        // x quantization, one warp per 256-block
+        const int b = (blockIdx.x - a.E) * 4 + warp;
+        if (b >= a.nbh) return;
+        const float4 *src = reinterpret_cast<const float4 *>(a.x + b * QK + 8 * lane);
+        const float4 v0 = __ldg(src), v1 = __ldg(src + 1);
+        const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+        uint2 packed;
+        float d;
+        int sum;
+        const bool ok = quant_block_warp(v, packed, d, sum);
+        *reinterpret_cast<uint2 *>(a.qx + b * QK + 8 * lane) = packed;
+        if (lane == 0) {
+            a.dx[b] = d;
+            a.bx[b] = sum;
+            if (!ok) report(a.status, TQFX4_EDATA, K_ROUTER, b);
+        }
+        return;
+    }
+    grid_dependents_launch();  // let the gate/up kernel's CTAs get resident early
+    const int e = blockIdx.x;
+    if (e == 0)  // the down kernel's counters start every call at zero
+        for (int i = threadIdx.x; i < a.n_ctr - kCtrDown; i += blockDim.x) a.ctr[kCtrDown + i] = 0;
+    float hi, lo;
+    router_logit_block(a.wr + static_cast<int64_t>(e) * a.H, a.x, a.H, hi, lo);
+    TQ_STAMP(0, 1);
+    if (lane == 0) {
+        part_hi[warp] = hi;
+        part_lo[warp] = lo;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float h01, l01, h23, l23;
+        ff_add(part_hi[0], part_lo[0], part_hi[1], part_lo[1], h01, l01);
+        ff_add(part_hi[2], part_lo[2], part_hi[3], part_lo[3], h23, l23);
+        ff_add(h01, l01, h23, l23, hi, lo);
+        if (a.bias) ff_add(hi, lo, __ldg(a.bias + e), 0.0f, hi, lo);
+        a.logits[e] = hi;
+        a.logits_lo[e] = lo;
+        last = (atomic_add_acq_rel(&a.ctr[kCtrRouter], 1) == a.E - 1);
+    }
+    __syncthreads();
+    TQ_STAMP(0, 2);
+    if (!last) return;
+    topk_block(a.logits, a.logits_lo, a.E, a.top_k, a.sel, topk_s);
+    TQ_STAMP(0, 5);
+    if (threadIdx.x < a.top_k) a.sel_out[threadIdx.x] = __ldcg(a.sel + threadIdx.x);
+    if (threadIdx.x == 0) a.ctr[kCtrRouter] = 0;
+    TQ_STAMP(0, 3);
 }
-tqfx4_status tqfx4_moe_grouped_traced(const tqfx4_experts *, const tqfx4_router *, const float *, int64_t,
-                                      float *, int32_t *, float *, int, void *, size_t, void *,
-                                      void *const *) {
-    return TQFX4_EINVAL;
+
+// ---------------------------------------------------------------- gate/up
+
+__global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    TQ_STAMP(1, 0);
+    const int warp = threadIdx.x >> 5;
+    const int nbh = a.nbh;
+    uint8_t *qs = smem;
+    float *das = reinterpret_cast<float *>(qs + nbh * QS_STRIDE);
+    int *bss = reinterpret_cast<int *>(das + nbh);
+    const WarpRing ring = carve_ring(
+        smem + act_bytes(nbh) + warp * stream_warp_bytes(a.stages_gu, a.slot_gu, a.rpu_gu, nbh), a.stages_gu,
+        a.slot_gu, a.rpu_gu, nbh);
+    ring_init(ring);
+    fence_barrier_init();
+    grid_dependency_wait();  // the router's selection and quantized x
+    TQ_STAMP(1, 1);
+    grid_dependents_launch();
+    const int j = blockIdx.x / a.parts_gu, p = blockIdx.x - j * a.parts_gu;
+    // issue the activation loads first: weight copies issued before them
+    // would queue ahead in the memory system
+    ActRegs act;
+    act_load(a.qx, a.dx, a.bx, nbh, act);
+    const int64_t e = __ldcg(a.sel + j);
+    const int64_t n_rg = a.I / 4;
+    MatJob jobs[2];
+    for (int q = 0; q < 2; ++q) {
+        MatJob &J = jobs[q];
+        J.mat = (q == 0 ? a.gate : a.up) + e * a.mb_gu;
+        J.rg_begin = part_begin(n_rg, a.rpu_gu, a.parts_gu, p);
+        J.rg_end = part_begin(n_rg, a.rpu_gu, a.parts_gu, p + 1);
+        J.y = (q == 0 ? a.g : a.u) + static_cast<int64_t>(j) * a.I;
+        J.s_out = nullptr;
+        J.qs = qs;
+        J.das = das;
+        J.bss = bss;
+        J.nb = nbh;
+    }
+    const bool any = jobs[0].rg_begin < jobs[0].rg_end;
+    if (any) warp_stream_prefetch(ring, jobs, 2, a.rpu_gu, warp, a.warps_gu);
+    act_store(act, nbh, qs, das, bss);
+    __syncthreads();
+    TQ_STAMP(1, 2);
+    if (any) warp_stream_run(ring, jobs, 2, a.rpu_gu, warp, a.warps_gu, a.status, K_GATEUP);
+    TQ_STAMP(1, 3);
 }
-tqfx4_status tqfx4_moe_workspace_views(const tqfx4_experts *, const tqfx4_router *, int64_t, int, int,
-                                       tqfx4_moe_views *) {
-    return TQFX4_EINVAL;
+
+// ---------------------------------------------------------------- down
+
+__global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    TQ_STAMP(2, 0);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nbi = a.nbi, K = a.top_k;
+    __shared__ int last;
+    __shared__ float selw_s[TQFX4_MAX_TOP_K];
+    uint8_t *qs = smem;
+    float *das = reinterpret_cast<float *>(qs + nbi * QS_STRIDE);
+    int *bss = reinterpret_cast<int *>(das + nbi);
+    const WarpRing ring = carve_ring(
+        smem + act_bytes(nbi) + warp * stream_warp_bytes(a.stages_d, a.slot_d, a.rpu_d, nbi), a.stages_d,
+        a.slot_d, a.rpu_d, nbi);
+    ring_init(ring);
+    fence_barrier_init();
+    const int j = blockIdx.x / a.parts_d, p = blockIdx.x - j * a.parts_d;
+    const int64_t e = __ldcg(a.sel + j);
+    const int64_t n_rg = a.H / 4;
+    MatJob job;
+    job.mat = a.down + e * a.mb_d;
+    job.rg_begin = part_begin(n_rg, a.rpu_d, a.parts_d, p);
+    job.rg_end = part_begin(n_rg, a.rpu_d, a.parts_d, p + 1);
+    job.y = a.o + static_cast<int64_t>(j) * a.H;
+    job.s_out = nullptr;
+    job.qs = qs;
+    job.das = das;
+    job.bss = bss;
+    job.nb = nbi;
+    const bool any = job.rg_begin < job.rg_end;
+    if (warp == a.warps_d - 1) {
+        // the routing weights (needed by the combine at the end); the router
+        // has completed, so this runs while gate/up drains
+        int sel_l[TQFX4_MAX_TOP_K];
+        for (int i = 0; i < K; ++i) sel_l[i] = __ldcg(a.sel + i);
+        softmax_ff_warp(a.logits, a.logits_lo, sel_l, K, selw_s);
+        if (blockIdx.x == 0 && lane < K) {
+            a.selw[lane] = selw_s[lane];
+            a.selw_out[lane] = selw_s[lane];
+        }
+    }
+    TQ_STAMP(2, 1);
+    grid_dependency_wait();  // g and u of the gate/up kernel
+    TQ_STAMP(2, 2);
+    if (blockIdx.x == 0 && threadIdx.x == 0) a.ctr[kCtrRouter] = 0;  // for the next call
+    // h_j = silu(g_j) u_j and its int8 quantization, one 256-block per warp;
+    // the g/u loads go out before the rest of the weight prefetch
+    const float *gj = a.g + static_cast<int64_t>(j) * a.I;
+    const float *uj = a.u + static_cast<int64_t>(j) * a.I;
+    for (int b0 = 0; b0 < nbi; b0 += a.warps_d) {
+        const int b = b0 + warp;
+        const bool mine = b < nbi;
+        float gg[8], uu[8];
+        if (mine) {
+            const int o = b * QK + 8 * lane;
+            const float4 g0 = __ldcg(reinterpret_cast<const float4 *>(gj + o));
+            const float4 g1 = __ldcg(reinterpret_cast<const float4 *>(gj + o) + 1);
+            const float4 u0 = __ldcg(reinterpret_cast<const float4 *>(uj + o));
+            const float4 u1 = __ldcg(reinterpret_cast<const float4 *>(uj + o) + 1);
+            gg[0] = g0.x; gg[1] = g0.y; gg[2] = g0.z; gg[3] = g0.w;
+            gg[4] = g1.x; gg[5] = g1.y; gg[6] = g1.z; gg[7] = g1.w;
+            uu[0] = u0.x; uu[1] = u0.y; uu[2] = u0.z; uu[3] = u0.w;
+            uu[4] = u1.x; uu[5] = u1.y; uu[6] = u1.z; uu[7] = u1.w;
+        }
+        if (!mine) continue;
+        const int o = b * QK + 8 * lane;
+        TQ_STAMP(2, 6);
+        float hv[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) hv[i] = tq_swiglu(gg[i], uu[i]);
+        TQ_STAMP(2, 7);
+        uint2 packed;
+        float d;
+        int sum;
+        const bool ok = quant_block_warp(hv, packed, d, sum);
+        *reinterpret_cast<uint2 *>(qs + b * QS_STRIDE + 8 * lane) = packed;
+        if (lane == 0) {
+            das[b] = d;
+            bss[b] = sum;
+        }
+        if (p == 0) {  // one CTA per expert leaves h and its quantization in the workspace
+            float *hj = a.h + static_cast<int64_t>(j) * a.I + o;
+            reinterpret_cast<float4 *>(hj)[0] = make_float4(hv[0], hv[1], hv[2], hv[3]);
+            reinterpret_cast<float4 *>(hj)[1] = make_float4(hv[4], hv[5], hv[6], hv[7]);
+            *reinterpret_cast<uint2 *>(a.qh + static_cast<int64_t>(j) * a.I + o) = packed;
+            if (lane == 0) {
+                a.dh[j * nbi + b] = d;
+                a.bh[j * nbi + b] = sum;
+                if (!ok) report(a.status, TQFX4_EDATA, K_DOWN, j * nbi + b);
+            }
+        }
+    }
+    if (any) warp_stream_prefetch(ring, &job, 1, a.rpu_d, warp, a.warps_d);
+    __syncthreads();
+    TQ_STAMP(2, 3);
+    if (any) warp_stream_run(ring, &job, 1, a.rpu_d, warp, a.warps_d, a.status, K_DOWN);
+    __syncthreads();
+    TQ_STAMP(2, 4);
+    if (threadIdx.x == 0) last = (atomic_add_acq_rel(&a.ctr[kCtrDown + p], 1) == K - 1);
+    __syncthreads();
+    if (!last) return;
+    const int64_t r0 = job.rg_begin * 4, r1 = job.rg_end * 4;
+    for (int64_t n = r0 + threadIdx.x; n < r1; n += blockDim.x) {
+        float acc = 0.0f;
+        for (int jj = 0; jj < K; ++jj)
+            acc = __fadd_rn(acc, __fmul_rn(selw_s[jj], __ldcg(a.o + static_cast<int64_t>(jj) * a.H + n)));
+        a.out[n] = acc;
+    }
+    TQ_STAMP(2, 5);
 }
+
+// ---------------------------------------------------------------- host side
+
+namespace {
+
+// Launch `kernel(a)` as a programmatic dependent of the previous kernel in
+// the stream (plain stream order when `plain`).
+cudaError_t launch_pdl(const void *kernel, int grid, int block, int smem, cudaStream_t st, bool plain,
+                       MoeArgs &a) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(block);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = plain ? 0 : 1;
+    void *args[] = {&a};
+    return cudaLaunchKernelExC(&cfg, kernel, args);
 }
+
+// Warps per CTA that fit the shared memory left after `act` bytes, 2 stages.
+int fit_warps(int slot, int rpu, int nb, int act, int max_warps) {
+    const int budget = max_smem_optin() - 1024 - act;
+    int w = max_warps;
+    while (w > 1 && w * stream_warp_bytes(2, slot, rpu, nb) > budget) --w;
+    return w;
+}
+
+}  // namespace
+
+// Geometry and workspace views for the decode (T = 1) path.
+bool moe_decode_args(const tqfx4_experts *ex, const tqfx4_router *rt, void *ws, MoeArgs &a, MoeLayout &L) {
+    a = MoeArgs{};
+    a.E = static_cast<int>(ex->n_experts);
+    a.H = static_cast<int>(ex->hidden);
+    a.I = static_cast<int>(ex->inter);
+    a.top_k = rt->top_k;
+    a.nbh = a.H / QK;
+    a.nbi = a.I / QK;
+    a.mb_gu = static_cast<int64_t>(a.I / 4) * a.nbh * BLOCK_BYTES;
+    a.mb_d = static_cast<int64_t>(a.H / 4) * a.nbi * BLOCK_BYTES;
+    a.gate = static_cast<const uint8_t *>(ex->gate);
+    a.up = static_cast<const uint8_t *>(ex->up);
+    a.down = static_cast<const uint8_t *>(ex->down);
+    a.wr = rt->weight;
+    a.bias = rt->bias;
+    L = moe_layout(a.E, a.H, a.I, a.top_k, 1, false, true);
+    uint8_t *base = static_cast<uint8_t *>(ws);
+    a.n_ctr = static_cast<int>(L.n_ctr);
+    if (base) {
+        a.status = reinterpret_cast<int *>(base);
+        a.ctr = reinterpret_cast<int *>(base + L.ctr);
+        a.logits = reinterpret_cast<float *>(base + L.logits);
+        a.logits_lo = reinterpret_cast<float *>(base + L.logits_lo);
+        a.sel = reinterpret_cast<int *>(base + L.sel);
+        a.selw = reinterpret_cast<float *>(base + L.selw);
+        a.qx = reinterpret_cast<int8_t *>(base + L.qx);
+        a.dx = reinterpret_cast<float *>(base + L.dx);
+        a.bx = reinterpret_cast<int *>(base + L.bx);
+        a.g = reinterpret_cast<float *>(base + L.g);
+        a.u = reinterpret_cast<float *>(base + L.u);
+        a.h = reinterpret_cast<float *>(base + L.h);
+        a.qh = reinterpret_cast<int8_t *>(base + L.qh);
+        a.dh = reinterpret_cast<float *>(base + L.dh);
+        a.bh = reinterpret_cast<int *>(base + L.bh);
+        a.o = reinterpret_cast<float *>(base + L.o);
+    }
+    const int sms = num_sms();
+    // gate/up: top_k x parts CTAs, each a contiguous range of row groups
+    a.rpu_gu = pow2_rows(32, a.nbh);
+    a.slot_gu = stream_slot_bytes(a.rpu_gu, a.nbh);
+    a.stages_gu = 2;
+    a.warps_gu = fit_warps(a.slot_gu, a.rpu_gu, a.nbh, act_bytes(a.nbh), 8);
+    a.parts_gu = static_cast<int>(imax64(1, sms / a.top_k));
+
+    // down: the same partition over the hidden rows
+    a.rpu_d = pow2_rows(32, a.nbi);
+    a.slot_d = stream_slot_bytes(a.rpu_d, a.nbi);
+    a.stages_d = 2;
+    a.warps_d = fit_warps(a.slot_d, a.rpu_d, a.nbi, act_bytes(a.nbi), 8);
+    a.parts_d = static_cast<int>(imax64(1, sms / a.top_k));
+
+    return static_cast<int64_t>(a.n_ctr) >= kCtrDown + a.parts_d;
+}
+
+int gate_up_smem(const MoeArgs &a) {
+    return act_bytes(a.nbh) + a.warps_gu * stream_warp_bytes(a.stages_gu, a.slot_gu, a.rpu_gu, a.nbh);
+}
+int down_smem(const MoeArgs &a) {
+    return act_bytes(a.nbi) + a.warps_d * stream_warp_bytes(a.stages_d, a.slot_d, a.rpu_d, a.nbi);
+}
+
+cudaError_t launch_moe_decode(const MoeArgs &a0, const float *x, float *out, int32_t *sel_idx, float *sel_w,
+                              cudaStream_t st, void *const *events) {
+    MoeArgs a = a0;
+    a.x = x;
+    a.out = out;
+    a.sel_out = sel_idx;
+    a.selw_out = sel_w;
+    static unsigned char set_gu[64], set_dn[64];
+    cudaError_t e = allow_max_smem(reinterpret_cast<const void *>(gate_up_kernel), set_gu);
+    if (e == cudaSuccess) e = allow_max_smem(reinterpret_cast<const void *>(down_kernel), set_dn);
+    if (e != cudaSuccess) return e;
+    auto rec = [&](int i) {
+        if (events && events[i]) cudaEventRecord(static_cast<cudaEvent_t>(events[i]), st);
+    };
+    rec(0);
+    router_kernel<<<a.E + (a.nbh + 3) / 4, 128, 0, st>>>(a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    rec(1);
+    if ((e = launch_pdl(reinterpret_cast<const void *>(gate_up_kernel), a.top_k * a.parts_gu, a.warps_gu * 32,
+                        gate_up_smem(a), st, events != nullptr, a)) != cudaSuccess)
+        return e;
+    rec(2);
+    if ((e = launch_pdl(reinterpret_cast<const void *>(down_kernel), a.top_k * a.parts_d, a.warps_d * 32,
+                        down_smem(a), st, events != nullptr, a)) != cudaSuccess)
+        return e;
+    rec(3);
+    return cudaSuccess;
+}
+
+}  // namespace tq

@@ -1,0 +1,411 @@
+// Pieces shared by the MoE decode and grouped kernels: workspace layout,
+// top-k selection, and two-range bulk staging.
+#pragma once
+
+#include "tq_common.cuh"
+
+namespace tq {
+
+// ---- workspace layout (byte offsets from the workspace base) -------------------
+
+struct MoeLayout {
+    size_t ctr;      // int32 counters, zeroed by the first kernel of every call
+    size_t n_ctr;
+    size_t logits;   // fp32 [T][E]
+    size_t logits_lo; // fp32 [T][E]: logit = logits + logits_lo (double-binary32)
+    size_t sel;      // int32 [T][top_k]
+    size_t selw;     // fp32 [T][top_k]
+    size_t qx, dx, bx;
+    size_t g, u, h;  // fp32 [P][I]
+    size_t qh, dh, bh;
+    size_t o;        // fp32 [P][H]
+    size_t counts, offsets, pair_token, pair_slot, pair_of;
+    size_t total;
+};
+
+inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int64_t T, bool grouped,
+                            bool keep_gu) {
+    MoeLayout L{};
+    const int64_t P = T * top_k;
+    const int64_t nbh = H / QK, nbi = I / QK;
+    size_t off = TQFX4_STATUS_BYTES;
+    auto take = [&](size_t bytes) {
+        const size_t at = off;
+        off = align256(off + bytes);
+        return at;
+    };
+    L.n_ctr = static_cast<size_t>(P * nbi + (H / 4) * (grouped ? T : 1) + E + 1024);
+    L.ctr = take(4 * L.n_ctr);
+    L.logits = take(4 * static_cast<size_t>(T * E));
+    L.logits_lo = take(4 * static_cast<size_t>(T * E));
+    L.sel = take(4 * static_cast<size_t>(P));
+    L.selw = take(4 * static_cast<size_t>(P));
+    L.qx = take(static_cast<size_t>(T * H));
+    L.dx = take(4 * static_cast<size_t>(T * nbh));
+    L.bx = take(4 * static_cast<size_t>(T * nbh));
+    if (keep_gu) {
+        L.g = take(4 * static_cast<size_t>(P * I));
+        L.u = take(4 * static_cast<size_t>(P * I));
+    } else {
+        L.g = L.u = SIZE_MAX;
+    }
+    L.h = take(4 * static_cast<size_t>(P * I));
+    L.qh = take(static_cast<size_t>(P * I));
+    L.dh = take(4 * static_cast<size_t>(P * nbi));
+    L.bh = take(4 * static_cast<size_t>(P * nbi));
+    L.o = take(4 * static_cast<size_t>(P * H));
+    if (grouped) {
+        L.counts = take(4 * static_cast<size_t>(E));
+        L.offsets = take(4 * static_cast<size_t>(E + 1));
+        L.pair_token = take(4 * static_cast<size_t>(P));
+        L.pair_slot = take(4 * static_cast<size_t>(P));
+        L.pair_of = take(4 * static_cast<size_t>(P));
+    } else {
+        L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = SIZE_MAX;
+    }
+    L.total = off;
+    return L;
+}
+
+// ---- kernel arguments of the decode path ----
+
+struct MoeArgs {
+    const uint8_t *gate, *up, *down;
+    int64_t mb_gu, mb_d;  // bytes of one expert's gate (= up) and down matrix
+    const float *wr, *bias;
+    const float *x;
+    float *out;
+    int32_t *sel_out;
+    float *selw_out;
+    int E, H, I, top_k, nbh, nbi;
+    // workspace views
+    int *status, *ctr;
+    int n_ctr;
+    float *logits, *logits_lo;
+    int *sel;
+    float *selw;
+    int8_t *qx;
+    float *dx;
+    int *bx;
+    float *g, *u, *h;
+    int8_t *qh;
+    float *dh;
+    int *bh;
+    float *o;
+    // gate/up geometry: top_k x parts_gu CTAs, each a range of row groups
+    int rpu_gu, slot_gu, stages_gu, warps_gu, parts_gu;
+    // down geometry
+    int rpu_d, slot_d, stages_d, warps_d, parts_d;
+};
+
+// Shared-memory bytes of one quantized activation vector of nb blocks
+// (codes at QS_STRIDE, then scales and block sums), 128-byte rounded.
+__host__ __device__ inline int act_bytes(int nb) { return ((nb * (QS_STRIDE + 8) + 127) / 128) * 128; }
+
+// ---- router ----------------------------------------------------------------------
+
+// Error-free transformations (Knuth's TwoSum, and the fused-multiply-add
+// product error), used to evaluate router logits to twice binary32 precision
+// with the "Dot2" compensated dot product of Ogita, Rump and Oishi (2005).
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
+    s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+
+// (hi, lo) + (hi, lo) in double-binary32 arithmetic: TwoSum of the high
+// parts, the low parts added into the error, then renormalized with
+// Fast2Sum. Relative error of order 2^-44 of the operands' magnitude.
+__device__ __forceinline__ void ff_add(float ah, float al, float bh, float bl, float &sh, float &sl) {
+    float s, e;
+    two_sum(ah, bh, s, e);
+    e = __fadd_rn(e, __fadd_rn(al, bl));
+    sh = __fadd_rn(s, e);
+    sl = __fsub_rn(e, __fsub_rn(sh, s));
+}
+
+// One router logit, sum_k w[k] x[k], by a block of 128 threads (H a
+// multiple of 256; w and x 16-byte aligned). Each thread runs Dot2 over its
+// float4s (all loads issued up front) with four independent (sum, error)
+// pairs; partial results are combined as double-binary32 pairs across the
+// warp (binary64 arithmetic is slow on this part). Returns the warp's
+// partial as (hi, lo) in every lane; the caller adds the four warps' pairs
+// in a fixed order. The result is within a few units of 2^-44 of the exact
+// dot product relative to sum |w x|, so top-k decisions and softmax weights
+// match an fp64 reference.
+__device__ __forceinline__ void router_logit_block(const float *w, const float *x, int H, float &hi, float &lo) {
+    const float4 *w4 = reinterpret_cast<const float4 *>(w);
+    const float4 *x4 = reinterpret_cast<const float4 *>(x);
+    float s[4] = {0.f, 0.f, 0.f, 0.f}, c[4] = {0.f, 0.f, 0.f, 0.f};
+    const int n4 = H >> 2;
+#pragma unroll 8
+    for (int i = threadIdx.x; i < n4; i += 128) {
+        const float4 wv = __ldg(w4 + i), xv = __ldg(x4 + i);
+        const float ww[4] = {wv.x, wv.y, wv.z, wv.w}, xx[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float p = __fmul_rn(ww[q], xx[q]);
+            const float pe = __fmaf_rn(ww[q], xx[q], -p);
+            float t, te;
+            two_sum(s[q], p, t, te);
+            s[q] = t;
+            c[q] = __fadd_rn(c[q], __fadd_rn(te, pe));
+        }
+    }
+    float h01, l01, h23, l23;
+    ff_add(s[0], c[0], s[1], c[1], h01, l01);
+    ff_add(s[2], c[2], s[3], c[3], h23, l23);
+    ff_add(h01, l01, h23, l23, hi, lo);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float oh = __shfl_xor_sync(0xffffffffu, hi, o), ol = __shfl_xor_sync(0xffffffffu, lo, o);
+        ff_add(hi, lo, oh, ol, hi, lo);
+    }
+}
+
+// Total order on binary32 values as unsigned keys (-0 folded into +0).
+__device__ __forceinline__ uint32_t order_key(float f) {
+    const uint32_t u = __float_as_uint(f + 0.0f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Sort key of expert e with logit (hi, lo), a normalized double-binary32
+// pair: the hi key, then the top 22 bits of the lo key (the pair's order is
+// the order of the exact values; 22 bits of lo resolve differences down to
+// about 2^-37 of the logit, below the accuracy of its evaluation), then the
+// lower expert index first. Distinct for distinct experts.
+__device__ __forceinline__ unsigned long long topk_key(float hi, float lo, int e) {
+    return (static_cast<unsigned long long>(order_key(hi)) << 32) |
+           (static_cast<unsigned long long>(order_key(lo) >> 10) << 10) |
+           static_cast<unsigned long long>(1023 - e);
+}
+
+// Shared scratch of topk_block.
+struct TopkScratch {
+    unsigned long long key[TQFX4_MAX_EXPERTS];
+    int hist[256];
+    int cand[TQFX4_MAX_EXPERTS];
+    int ncand;
+    int bin_cut;
+    unsigned int kmin, kmax;
+};
+
+// Top-k of E <= 1024 logits (double-binary32 pairs, read through L2) by the
+// whole thread block, in descending order with ties to the lower index:
+// (1) the keys' hi parts are binned linearly between their minimum and
+// maximum into 256 bins; (2) the highest bin b* whose suffix count reaches k
+// is found; (3) only the experts in bins >= b* (normally a few more than k)
+// are ranked exactly by comparing full keys. Writes sel[rank] (global
+// memory). All threads must call.
+__device__ __forceinline__ void topk_block(const float *lhi, const float *llo, int E, int k, int *sel,
+                                           TopkScratch &s) {
+    const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31;
+    if (tid == 0) {
+        s.kmin = 0xffffffffu;
+        s.kmax = 0u;
+        s.ncand = 0;
+    }
+    for (int i = tid; i < 256; i += nt) s.hist[i] = 0;
+    __syncthreads();
+    unsigned int lmin = 0xffffffffu, lmax = 0u;
+    for (int e = tid; e < E; e += nt) {
+        const unsigned long long key = topk_key(__ldcg(lhi + e), __ldcg(llo + e), e);
+        s.key[e] = key;
+        const unsigned int h = static_cast<unsigned int>(key >> 32);
+        lmin = min(lmin, h);
+        lmax = max(lmax, h);
+    }
+    lmin = __reduce_min_sync(0xffffffffu, lmin);
+    lmax = __reduce_max_sync(0xffffffffu, lmax);
+    if (lane == 0) {
+        atomicMin(&s.kmin, lmin);
+        atomicMax(&s.kmax, lmax);
+    }
+    __syncthreads();
+    const unsigned int kmin = s.kmin, span = s.kmax - s.kmin;
+    const int shift = span == 0u ? 0 : max(0, 24 - __clz(span));  // (span >> shift) < 256
+    for (int e = tid; e < E; e += nt)
+        atomicAdd(&s.hist[(static_cast<unsigned int>(s.key[e] >> 32) - kmin) >> shift], 1);
+    __syncthreads();
+    if (tid < 32) {
+        // suffix sums over the 256 bins, 8 per lane (lane 31 holds the top bins)
+        int c[8], tot = 0;
+#pragma unroll
+        for (int i = 7; i >= 0; --i) {
+            tot += s.hist[lane * 8 + i];
+            c[i] = tot;  // count of bins lane*8+i .. lane*8+7
+        }
+        // inclusive suffix scan of the lane totals; `above` counts higher lanes
+        int v = tot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_down_sync(0xffffffffu, v, o);
+            if (lane + o < 32) v += t;
+        }
+        const int above = v - tot;
+        int cut = -1;
+#pragma unroll
+        for (int i = 7; i >= 0; --i)
+            if (cut < 0 && above + c[i] >= k) cut = lane * 8 + i;
+        const int best = __reduce_max_sync(0xffffffffu, cut);
+        if (lane == 0) s.bin_cut = best < 0 ? 0 : best;
+    }
+    __syncthreads();
+    const int cut = s.bin_cut;
+    for (int e = tid; e < E; e += nt)
+        if (static_cast<int>((static_cast<unsigned int>(s.key[e] >> 32) - kmin) >> shift) >= cut)
+            s.cand[atomicAdd(&s.ncand, 1)] = e;
+    __syncthreads();
+    const int nc = s.ncand;
+    for (int ci = tid; ci < nc; ci += nt) {
+        const int e = s.cand[ci];
+        const unsigned long long ke = s.key[e];
+        int r = 0;
+        for (int cj = 0; cj < nc; ++cj) r += s.key[s.cand[cj]] > ke;
+        if (r < k) sel[r] = e;
+    }
+    __syncthreads();
+}
+
+// ---- double-binary32 softmax ----------------------------------------------------
+
+__device__ __forceinline__ void fast_two_sum(float a, float b, float &s, float &e) {
+    s = __fadd_rn(a, b);
+    e = __fsub_rn(b, __fsub_rn(s, a));
+}
+
+// (ah, al) * (bh, bl), normalized.
+__device__ __forceinline__ void ff_mul(float ah, float al, float bh, float bl, float &ph, float &pl) {
+    const float p = __fmul_rn(ah, bh);
+    float e = __fmaf_rn(ah, bh, -p);
+    e = __fadd_rn(e, __fadd_rn(__fmul_rn(ah, bl), __fmul_rn(al, bh)));
+    fast_two_sum(p, e, ph, pl);
+}
+
+// exp(d) for d = dh + dl <= 0 in double-binary32: d = n ln2 + r with ln2
+// split into 0.693145751953125 + 1.428606765330187e-06 + 5.497923148104107e-14
+// (the first part exact in n * part), |r| <= ln2 / 2, then the degree-13
+// Taylor polynomial of e^r (coefficients 1/k! as pairs) in Horner form, and
+// the scaling by 2^n. Relative error near 2^-44 for d >= -87.
+__device__ __forceinline__ void ff_exp_nonpos(float dh, float dl, float &eh, float &el) {
+    dh = fmaxf(dh, -100.0f);
+    const float nf = rintf(__fmul_rn(dh, 1.4426950216293335f));
+    const float t1 = __fsub_rn(dh, __fmul_rn(nf, 0.693145751953125f));
+    const float p2 = __fmul_rn(nf, 1.428606765330187e-06f);
+    const float e2 = __fmaf_rn(nf, 1.428606765330187e-06f, -p2);
+    float rh, rl;
+    ff_add(t1, dl, -p2, -e2, rh, rl);
+    rl = __fsub_rn(rl, __fmul_rn(nf, 5.497923148104107e-14f));
+    fast_two_sum(rh, rl, rh, rl);
+    // 1/k!, k = 13 .. 0, as (hi, lo)
+    const float ch[14] = {1.6059044372074283e-10f, 2.0876755879584152e-09f, 2.5052107943679403e-08f,
+                          2.755731998149713e-07f,  2.7557318844628753e-06f, 2.4801587642286904e-05f,
+                          0.00019841270113829523f, 0.0013888889225199819f,  0.008333333767950535f,
+                          0.0416666679084301f,     0.1666666716337204f,     0.5f,
+                          1.0f,                    1.0f};
+    const float cl[14] = {-5.352526511562726e-18f, 1.1082839147459852e-16f, 4.4176230446483665e-16f,
+                          -7.575112209051195e-15f, 3.793571224297229e-14f,  -3.40699609366682e-13f,
+                          -2.725596874933456e-12f, -3.3631094437103215e-11f, -4.34617203337595e-10f,
+                          -1.2417634698280722e-09f, -4.967053879312289e-09f, 0.0f,
+                          0.0f,                    0.0f};
+    float ph = ch[0], pl = cl[0];
+#pragma unroll
+    for (int i = 1; i < 14; ++i) {
+        float mh, ml;
+        ff_mul(ph, pl, rh, rl, mh, ml);
+        ff_add(mh, ml, ch[i], cl[i], ph, pl);
+    }
+    const int n = static_cast<int>(nf);
+    eh = ldexpf(ph, n);
+    el = ldexpf(pl, n);
+}
+
+// Softmax weights of the selected logits sel[0..k) (k <= 32) by one warp:
+// w_j = exp(l_j - l_0) / sum_i exp(l_i - l_0), in double-binary32
+// arithmetic, each w_j rounded once to binary32 (so it matches a binary64
+// evaluation rounded to binary32). Writes w[0..k) (any memory) from lanes
+// j < k. All lanes must call.
+__device__ __forceinline__ void softmax_ff_warp(const float *lhi, const float *llo, const int *sel, int k,
+                                                float *w) {
+    const int lane = threadIdx.x & 31;
+    const int e0 = sel[0];
+    const float h0 = __ldcg(lhi + e0), l0 = __ldcg(llo + e0);
+    float eh = 0.0f, el = 0.0f;
+    if (lane < k) {
+        const int e = sel[lane];
+        float dh, dl;
+        ff_add(__ldcg(lhi + e), __ldcg(llo + e), -h0, -l0, dh, dl);
+        ff_exp_nonpos(dh, dl, eh, el);
+    }
+    float sh = eh, sl = el;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float oh = __shfl_xor_sync(0xffffffffu, sh, o), ol = __shfl_xor_sync(0xffffffffu, sl, o);
+        ff_add(sh, sl, oh, ol, sh, sl);
+    }
+    if (lane < k) {
+        // q = e / s: one binary32 quotient, then a correction from the exact residual
+        const float q = __fdiv_rn(eh, sh);
+        float ph, pl;
+        ff_mul(q, 0.0f, sh, sl, ph, pl);
+        float rh, rl;
+        ff_add(eh, el, -ph, -pl, rh, rl);
+        const float q2 = __fdiv_rn(rh, sh);
+        w[lane] = __fadd_rn(q, q2);
+    }
+    __syncwarp();
+}
+
+// ---- staging of up to two byte ranges on one barrier -----------------------------
+
+// Stages `n` (1 or 2) ranges, each a multiple of 8 bytes from an 8-byte
+// aligned source, into 16-byte aligned destinations on one mbarrier phase.
+// Lane 0 arms the barrier with the sum of the 16-byte aligned interiors and
+// issues their bulk copies; lanes 1..4 copy the 8-byte heads and tails.
+// Returns through `ofs` the offset of each range's data in its destination.
+__device__ __forceinline__ void stage_ranges(int lane, int n, uint8_t *const dst[2], const uint8_t *const src[2],
+                                             const uint32_t bytes[2], uint64_t *bar, uint32_t ofs[2]) {
+    uint32_t head[2], body[2], tail[2], total = 0;
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+        if (p < n) {
+            ofs[p] = static_cast<uint32_t>(reinterpret_cast<uintptr_t>(src[p]) & 15u);
+            head[p] = (ofs[p] != 0u && bytes[p] >= 8u) ? 8u : 0u;
+            body[p] = ((bytes[p] - head[p]) / 16u) * 16u;
+            tail[p] = bytes[p] - head[p] - body[p];
+            total += body[p];
+        }
+    }
+    if (lane == 0) {
+        mbar_arrive_expect_tx(bar, total);
+#pragma unroll
+        for (int p = 0; p < 2; ++p)
+            if (p < n && body[p]) bulk_g2s(dst[p] + ofs[p] + head[p], src[p] + head[p], body[p], bar);
+    }
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+        if (p < n) {
+            if (lane == 1 + 2 * p && head[p])
+                *reinterpret_cast<uint2 *>(dst[p] + ofs[p]) = __ldg(reinterpret_cast<const uint2 *>(src[p]));
+            if (lane == 2 + 2 * p && tail[p])
+                *reinterpret_cast<uint2 *>(dst[p] + ofs[p] + head[p] + body[p]) =
+                    __ldg(reinterpret_cast<const uint2 *>(src[p] + head[p] + body[p]));
+        }
+    }
+}
+
+__device__ __forceinline__ uint32_t src_ofs(const void *p) {
+    return static_cast<uint32_t>(reinterpret_cast<uintptr_t>(p) & 15u);
+}
+
+// Row groups per unit: the largest power of two r (at least 1) with
+// r * per_rg <= cap blocks, where per_rg is the blocks one row group brings.
+__host__ __device__ inline int pow2_rows(int cap, int per_rg) {
+    int r = 1;
+    while (r * 2 * per_rg <= cap) r *= 2;
+    return r;
+}
+
+}  // namespace tq

@@ -1,0 +1,177 @@
+// Warp-level streaming of tq2_0_fx4 row groups through shared memory: the
+// engine under the GEMV, the MoE gate/up/down kernels and the grouped decode.
+//
+// Each warp owns a ring of `stages` slots and an mbarrier per slot. A "job"
+// is a contiguous range of row groups of one matrix; its rows are cut into
+// units of `rpu` row groups (<= 32 blocks), copied with cp.async.bulk a few
+// units ahead. In a unit, lane i owns block i: it forms the block's four
+// exact int32 sums S with dp4a and the four products t = float(S) * (d * da)
+// of the fixed float schedule, and stores t in shared memory; then one lane
+// per row adds its row's t over the blocks in ascending order.
+#pragma once
+
+#include "tq_moe_common.cuh"
+
+namespace tq {
+
+struct MatJob {
+    const uint8_t *mat;    // first byte of the matrix
+    int64_t rg_begin;      // row-group range handled by this CTA
+    int64_t rg_end;
+    float *y;              // output rows (indexed by matrix row)
+    int32_t *s_out;        // optional exact block sums [n][nb] (matrix rows)
+    const uint8_t *qs;     // activation blocks in shared memory (QS_STRIDE apart)
+    const float *das;      // activation scales (shared memory)
+    const int *bss;        // activation block sums (shared memory)
+    int nb;                // blocks per row group
+};
+
+__host__ __device__ inline int stream_tbuf_bytes(int rpu, int nb) { return ((rpu * 4 * (nb + 1) * 4 + 15) / 16) * 16; }
+
+__host__ __device__ inline int stream_warp_bytes(int stages, int slot_bytes, int rpu, int nb) {
+    return ((stages * slot_bytes + stream_tbuf_bytes(rpu, nb) + stages * 8 + 127) / 128) * 128;
+}
+
+__host__ __device__ inline int stream_slot_bytes(int rpu, int nb) { return ((rpu * nb * BLOCK_BYTES + 16 + 15) / 16) * 16; }
+
+// Units of `job`, with `rpu` row groups each.
+__device__ __forceinline__ int64_t job_units(const MatJob &j, int rpu) {
+    return (j.rg_end - j.rg_begin + rpu - 1) / rpu;
+}
+
+struct WarpRing {
+    uint8_t *slots;
+    float *tbuf;
+    uint64_t *bars;
+    int stages;
+    int slot_bytes;
+};
+
+__device__ __forceinline__ WarpRing carve_ring(uint8_t *wbase, int stages, int slot_bytes, int rpu, int nb) {
+    WarpRing r;
+    r.slots = wbase;
+    r.tbuf = reinterpret_cast<float *>(wbase + stages * slot_bytes);
+    r.bars = reinterpret_cast<uint64_t *>(wbase + stages * slot_bytes + stream_tbuf_bytes(rpu, nb));
+    r.stages = stages;
+    r.slot_bytes = slot_bytes;
+    return r;
+}
+
+// Initialize the ring's barriers (lane 0); the caller fences and syncs.
+__device__ __forceinline__ void ring_init(const WarpRing &r) {
+    if ((threadIdx.x & 31) == 0)
+        for (int s = 0; s < r.stages; ++s) mbar_init(&r.bars[s], 1);
+}
+
+// Locate global unit u of the concatenated jobs.
+__device__ __forceinline__ void unit_locate(const MatJob *jobs, int njobs, int rpu, int64_t u, int &q,
+                                            int64_t &rg0, int &rgs) {
+    q = 0;
+    int64_t n0 = job_units(jobs[0], rpu);
+    while (q + 1 < njobs && u >= n0) {
+        u -= n0;
+        ++q;
+        n0 = job_units(jobs[q], rpu);
+    }
+    rg0 = jobs[q].rg_begin + u * rpu;
+    rgs = static_cast<int>(imin64(rpu, jobs[q].rg_end - rg0));
+}
+
+__device__ __forceinline__ void unit_issue(const WarpRing &r, const MatJob *jobs, int njobs, int rpu, int64_t u,
+                                           int slot) {
+    int q, rgs;
+    int64_t rg0;
+    unit_locate(jobs, njobs, rpu, u, q, rg0, rgs);
+    const int64_t stripe = static_cast<int64_t>(jobs[q].nb) * BLOCK_BYTES;
+    uint8_t *dst[2] = {r.slots + slot * r.slot_bytes, nullptr};
+    const uint8_t *src[2] = {jobs[q].mat + rg0 * stripe, nullptr};
+    const uint32_t bytes[2] = {static_cast<uint32_t>(rgs * stripe), 0u};
+    uint32_t ofs[2];
+    stage_ranges(threadIdx.x & 31, 1, dst, src, bytes, &r.bars[slot], ofs);
+}
+
+__device__ __forceinline__ int64_t jobs_total_units(const MatJob *jobs, int njobs, int rpu) {
+    int64_t total = 0;
+    for (int q = 0; q < njobs; ++q) total += job_units(jobs[q], rpu);
+    return total;
+}
+
+// Issue the first `stages` units of this warp's share (units first, first +
+// step, ...). Only the matrix pointers and row ranges of the jobs are used,
+// so this may run before the activations are in shared memory.
+__device__ __forceinline__ void warp_stream_prefetch(const WarpRing &r, const MatJob *jobs, int njobs, int rpu,
+                                                     int64_t first, int64_t step, int max_stages = 1 << 30) {
+    const int64_t total = jobs_total_units(jobs, njobs, rpu);
+    int64_t nx = first;
+    for (int s = 0; s < r.stages && s < max_stages; ++s, nx += step)
+        if (nx < total) unit_issue(r, jobs, njobs, rpu, nx, s);
+}
+
+// Issue the remaining prefetch slots [from, stages) after a partial
+// warp_stream_prefetch(..., from).
+__device__ __forceinline__ void warp_stream_prefetch_from(const WarpRing &r, const MatJob *jobs, int njobs,
+                                                          int rpu, int64_t first, int64_t step, int from) {
+    const int64_t total = jobs_total_units(jobs, njobs, rpu);
+    int64_t nx = first + from * step;
+    for (int s = from; s < r.stages; ++s, nx += step)
+        if (nx < total) unit_issue(r, jobs, njobs, rpu, nx, s);
+}
+
+// Consume this warp's units (prefetched by warp_stream_prefetch), refilling
+// each slot with the unit `stages` steps ahead. Returns false if a copy
+// never arrived (status recorded).
+__device__ __forceinline__ bool warp_stream_run(const WarpRing &r, const MatJob *jobs, int njobs, int rpu,
+                                                int64_t first, int64_t step, int *status, int kernel_id) {
+    const int lane = threadIdx.x & 31;
+    const int64_t total = jobs_total_units(jobs, njobs, rpu);
+    int it = 0;
+    for (int64_t u = first; u < total; u += step, ++it) {
+        const int slot = it % r.stages;
+        const uint32_t parity = static_cast<uint32_t>((it / r.stages) & 1);
+        if (!__all_sync(0xffffffffu, mbar_wait(&r.bars[slot], parity))) {
+            if (lane == 0) report(status, TQFX4_ETIMEOUT, kernel_id, static_cast<int>(u));
+            return false;
+        }
+        __syncwarp();
+        int q, rgs;
+        int64_t rg0;
+        unit_locate(jobs, njobs, rpu, u, q, rg0, rgs);
+        const MatJob &J = jobs[q];
+        const int nb = J.nb;
+        const int64_t stripe = static_cast<int64_t>(nb) * BLOCK_BYTES;
+        const uint8_t *data = r.slots + slot * r.slot_bytes + src_ofs(J.mat + rg0 * stripe);
+        const int nblk = rgs * nb;
+        for (int i = lane; i < nblk; i += 32) {
+            const int rgl = i / nb, b = i - rgl * nb;
+            const uint8_t *blk = data + i * BLOCK_BYTES;
+            int S[4];
+            block_dot(blk + CODE_OFS, J.qs + b * QS_STRIDE, J.bss[b], S);
+            const float da = J.das[b];
+#pragma unroll
+            for (int rr = 0; rr < 4; ++rr) {
+                const float sc = __fmul_rn(block_scale(blk, rr), da);
+                r.tbuf[(rgl * 4 + rr) * (nb + 1) + b] = __fmul_rn(static_cast<float>(S[rr]), sc);
+            }
+            if (J.s_out) {
+#pragma unroll
+                for (int rr = 0; rr < 4; ++rr) J.s_out[((rg0 + rgl) * 4 + rr) * nb + b] = S[rr];
+            }
+        }
+        __syncwarp();
+        for (int t = lane; t < rgs * 4; t += 32) {
+            const float *tb = r.tbuf + t * (nb + 1);
+            float acc = 0.0f;
+            for (int b = 0; b < nb; ++b) acc = __fadd_rn(acc, tb[b]);
+            J.y[rg0 * 4 + t] = acc;
+        }
+        __syncwarp();
+        const int64_t nu = u + static_cast<int64_t>(r.stages) * step;
+        if (nu < total) {
+            fence_proxy_async_smem();
+            unit_issue(r, jobs, njobs, rpu, nu, slot);
+        }
+    }
+    return true;
+}
+
+}  // namespace tq

@@ -1,0 +1,82 @@
+"""A routed-expert MoE layer held in device memory as tq2_0_fx4 blocks.
+
+Plumbing only: it allocates the stacked expert matrices and the router with
+torch, fills them through tqfx4_pack, and calls tqfx4_moe_ffn /
+tqfx4_moe_grouped. Each expert projection is one contiguous byte range
+(gate and up: inter x hidden; down: hidden x inter), experts stacked in
+order, as the C ABI's tqfx4_experts describes.
+"""
+import torch
+
+from . import binding as B
+from . import inputs
+
+
+class MoeLayer:
+    def __init__(self, gate, up, down, router_w, router_b, n_experts, hidden, inter, top_k):
+        self.gate, self.up, self.down = gate, up, down
+        self.router_w, self.router_b = router_w, router_b
+        self.n_experts, self.hidden, self.inter, self.top_k = n_experts, hidden, inter, top_k
+        self.ex = B.c_experts(gate, up, down, n_experts, hidden, inter)
+        self.rt = B.c_router(router_w, router_b, top_k)
+        self.mb_gu = B.tqfx4_matrix_bytes(inter, hidden)
+        self.mb_d = B.tqfx4_matrix_bytes(hidden, inter)
+
+    @classmethod
+    def synthetic(cls, seed: int, n_experts: int, hidden: int, inter: int, top_k: int, zipf: float = 0.0,
+                  device="cuda"):
+        """Student-t(5) * 0.02 expert weights packed by round-to-nearest, an
+        N(0, 0.02) router, and the -zipf * ln(rank) bias when zipf > 0."""
+        mb_gu = B.tqfx4_matrix_bytes(inter, hidden)
+        mb_d = B.tqfx4_matrix_bytes(hidden, inter)
+        gate = torch.empty(n_experts * mb_gu, dtype=torch.uint8, device=device)
+        up = torch.empty(n_experts * mb_gu, dtype=torch.uint8, device=device)
+        down = torch.empty(n_experts * mb_d, dtype=torch.uint8, device=device)
+        ws = torch.zeros(B.TQFX4_STATUS_BYTES, dtype=torch.uint8, device=device)
+        for e in range(n_experts):
+            for proj, buf, mb in ((inputs.PROJ_GATE, gate, mb_gu), (inputs.PROJ_UP, up, mb_gu),
+                                  (inputs.PROJ_DOWN, down, mb_d)):
+                w = inputs.expert_matrix(seed, e, proj, hidden, inter, device)
+                n, k = w.shape
+                B.tqfx4_pack(B.TQFX4_SRC_F32_RTN, w, None, None, n, k, buf[e * mb:(e + 1) * mb], ws)
+        B.tqfx4_check(ws)
+        rw = inputs.router_weight(seed, n_experts, hidden, device)
+        rb = inputs.zipf_bias(n_experts, zipf).to(device) if zipf > 0 else None
+        return cls(gate, up, down, rw, rb, n_experts, hidden, inter, top_k)
+
+    def expert_blocks(self, e: int):
+        """The (gate, up, down) byte ranges of expert e."""
+        return (self.gate[e * self.mb_gu:(e + 1) * self.mb_gu], self.up[e * self.mb_gu:(e + 1) * self.mb_gu],
+                self.down[e * self.mb_d:(e + 1) * self.mb_d])
+
+    def workspace(self, tokens: int = 1, path: int = 0) -> torch.Tensor:
+        n = B.tqfx4_moe_workspace_bytes(self.ex, self.rt, tokens, path)
+        if n == 0:
+            raise ValueError("invalid MoE shapes")
+        return torch.zeros(((n + 255) // 256) * 256, dtype=torch.uint8, device=self.gate.device)
+
+    def ffn(self, x, ws, out=None, sel_idx=None, sel_w=None, stream=None, events=None):
+        dev = x.device
+        out = torch.empty(self.hidden, dtype=torch.float32, device=dev) if out is None else out
+        sel_idx = torch.empty(self.top_k, dtype=torch.int32, device=dev) if sel_idx is None else sel_idx
+        sel_w = torch.empty(self.top_k, dtype=torch.float32, device=dev) if sel_w is None else sel_w
+        B.tqfx4_moe_ffn(self.ex, self.rt, x, out, sel_idx, sel_w, ws, stream, events)
+        return out, sel_idx, sel_w
+
+    def grouped(self, X, ws, path=0, OUT=None, sel_idx=None, sel_w=None, stream=None, events=None):
+        T = X.shape[0]
+        dev = X.device
+        OUT = torch.empty((T, self.hidden), dtype=torch.float32, device=dev) if OUT is None else OUT
+        sel_idx = torch.empty((T, self.top_k), dtype=torch.int32, device=dev) if sel_idx is None else sel_idx
+        sel_w = torch.empty((T, self.top_k), dtype=torch.float32, device=dev) if sel_w is None else sel_w
+        B.tqfx4_moe_grouped(self.ex, self.rt, X, T, OUT, sel_idx, sel_w, path, ws, stream, events)
+        return OUT, sel_idx, sel_w
+
+    def view(self, ws, name, dtype, shape, tokens=1, grouped=0, path=0):
+        """A typed view of one intermediate the last call left in `ws`."""
+        off = B.tqfx4_moe_workspace_views(self.ex, self.rt, tokens, grouped, path)[name]
+        n = 1
+        for s in shape:
+            n *= s
+        nbytes = n * torch.tensor([], dtype=dtype).element_size()
+        return ws[off:off + nbytes].view(dtype).view(*shape)

@@ -1,0 +1,176 @@
+"""GPU parity of tqfx4_moe_ffn (one token through a routed-expert MoE layer)
+against the CPU oracle, through the C ABI.
+
+Checked per token: the routing decision (expert ids bit-exact unless the
+oracle puts two candidates within the error bound of the two logit
+evaluations, in
+which case either order is valid), the quantized hidden state, each selected
+expert's g, u, h, re-quantized h and down output (bit-exact: the kernels use
+the oracle's float schedule and the same specified binary32 SwiGLU), and the
+combined output within 1e-4 relative.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_08910_gb300 import binding as B
+from paper_2608_08910_gb300 import inputs
+from paper_2608_08910_gb300.moe import MoeLayer
+from tests.parity import FP32_TOL, rel_err
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+def oracle_experts(seed, experts, hidden, inter):
+    """Oracle-packed blocks of the given experts, from the generator's fp32
+    weights (the same draws the GPU layer was packed from)."""
+    out = {}
+    for e in experts:
+        out[int(e)] = tuple(
+            oracle.pack_rtn(inputs.expert_matrix(seed, int(e), p, hidden, inter, DEV).cpu().numpy())
+            for p in (inputs.PROJ_GATE, inputs.PROJ_UP, inputs.PROJ_DOWN))
+    return out
+
+
+def selection_tolerance(Wr, x, bias):
+    """Per-expert bound on |kernel logit - oracle logit|: the kernel's
+    compensated binary32 dot product (Dot2, error below gamma_n^2 sum|w x|
+    with per-thread chains of n <= H/128 terms, then double-binary32 sums
+    with relative error near 2^-44) plus the oracle's sequential binary64
+    sum (H 2^-53 sum|w x|), doubled for safety."""
+    terms = np.abs(Wr.astype(np.float64)) @ np.abs(x.astype(np.float64))
+    H = Wr.shape[1]
+    b = 0 if bias is None else np.abs(bias.astype(np.float64))
+    gamma = (H // 128 + 2) * 2.0 ** -24
+    return 2 * (gamma ** 2 + 16 * 2.0 ** -44 + H * 2.0 ** -53) * (terms + b) + 1e-300
+
+
+def check_selection(sel, logits, tol, k):
+    """Expert ids must equal the oracle's ranking except where two adjacent
+    candidates (ranks 0..k) are closer than the fp32 error bound."""
+    order = np.lexsort((np.arange(logits.size), -logits))
+    ties = 0
+    for r in range(k):
+        a, b = order[r], order[r + 1] if r + 1 < logits.size else order[r]
+        close = abs(logits[a] - logits[b]) <= tol[a] + tol[b]
+        if sel[r] != order[r]:
+            assert close, "rank %d: got expert %d, oracle %d" % (r, sel[r], order[r])
+            ties += 1
+    return ties
+
+
+def run_and_check(layer, seed, X, zipf_bias=None, check_stages=True):
+    H, I, E, k = layer.hidden, layer.inter, layer.n_experts, layer.top_k
+    ws = layer.workspace(1)
+    Wr = layer.router_w.cpu().numpy()
+    bias = None if layer.router_b is None else layer.router_b.cpu().numpy()
+    worst = 0.0
+    for t in range(X.shape[0]):
+        x = X[t]
+        out, sel, selw = layer.ffn(x.to(DEV), ws)
+        B.tqfx4_check(ws)
+        out, sel, selw = out.cpu().numpy(), sel.cpu().numpy(), selw.cpu().numpy()
+        logits, r_idx, r_w = oracle.router(Wr, bias, x.numpy(), k)
+        tol = selection_tolerance(Wr, x.numpy(), bias)
+        hi = layer.view(ws, "logits", torch.float32, (E,)).cpu().numpy().astype(np.float64)
+        lo = layer.view(ws, "logits_lo", torch.float32, (E,)).cpu().numpy().astype(np.float64)
+        assert np.all(np.abs((hi + lo) - logits) <= tol)
+        assert np.all(np.abs(lo) <= np.spacing(np.abs(hi).astype(np.float32)))  # normalized pairs
+        ties = check_selection(sel, logits, tol, k)
+        ex = oracle_experts(seed, np.union1d(sel, r_idx), H, I)
+        ref, _, _ = oracle.moe_tokens(ex, E, H, I, Wr, bias, k, x.numpy())
+        if ties == 0:
+            assert np.array_equal(sel, r_idx)
+            assert np.allclose(selw, r_w, rtol=1.2e-7, atol=0)  # fp64 softmax, one rounding
+            e_ = rel_err(out, ref[0])
+            assert e_ <= FP32_TOL, e_
+            worst = max(worst, e_)
+        if check_stages:
+            rq, rdx, rbx = oracle.quantize_act(x.numpy())
+            assert np.array_equal(layer.view(ws, "qx", torch.int8, (H,)).cpu().numpy(), rq)
+            g = layer.view(ws, "g", torch.float32, (k, I)).cpu().numpy()
+            u = layer.view(ws, "u", torch.float32, (k, I)).cpu().numpy()
+            h = layer.view(ws, "h", torch.float32, (k, I)).cpu().numpy()
+            qh = layer.view(ws, "qh", torch.int8, (k, I)).cpu().numpy()
+            o = layer.view(ws, "o", torch.float32, (k, H)).cpu().numpy()
+            for j, e in enumerate(sel):
+                ro, dbg = oracle.expert_ffn(*ex[int(e)], H, I, x.numpy())
+                assert np.array_equal(g[j], dbg["g"]) and np.array_equal(u[j], dbg["u"])
+                assert np.array_equal(h[j].view(np.uint32), dbg["h"].view(np.uint32))
+                assert np.array_equal(qh[j], dbg["qh"])
+                assert np.array_equal(o[j].view(np.uint32), ro.view(np.uint32))
+            # the combine in rank order with the kernel's own weights is exact
+            acc = np.zeros(H, np.float32)
+            for j in range(k):
+                acc = (acc + np.float32(selw[j]) * o[j]).astype(np.float32)
+            assert np.array_equal(acc.view(np.uint32), out.view(np.uint32))
+    return worst
+
+
+@pytest.mark.parametrize("E,H,I,k,zipf", [(16, 512, 768, 4, 0.0), (8, 256, 256, 8, 0.0), (32, 1024, 512, 6, 1.1),
+                                          (1, 256, 512, 1, 0.0), (64, 2048, 1280, 8, 0.0)])
+def test_moe_ffn_small_shapes(E, H, I, k, zipf):
+    seed = E * 7 + H + I
+    layer = MoeLayer.synthetic(seed, E, H, I, k, zipf, DEV)
+    X = inputs.hidden_states(seed, 3, H)
+    run_and_check(layer, seed, X)
+
+
+def test_one_expert_ffn_full_size():
+    # the batch-1 SwiGLU expert, gate/up 4096->2048 and down 2048->4096
+    layer = MoeLayer.synthetic(1, 1, 4096, 2048, 1, 0.0, DEV)
+    X = inputs.hidden_states(1, 2, 4096)
+    ws = layer.workspace(1)
+    ex = oracle_experts(1, [0], 4096, 2048)
+    g, u, d = layer.expert_blocks(0)
+    for e_, blk in zip(ex[0], (g, u, d)):
+        assert np.array_equal(blk.cpu().numpy(), e_)
+    for t in range(2):
+        out, sel, selw = layer.ffn(X[t].to(DEV), ws)
+        B.tqfx4_check(ws)
+        ref, _ = oracle.expert_ffn(*ex[0], 4096, 2048, X[t].numpy())
+        assert sel.item() == 0 and selw.item() == 1.0
+        assert np.array_equal(out.cpu().numpy().view(np.uint32), ref.view(np.uint32))
+
+
+@pytest.fixture(scope="module")
+def full_layer():
+    return MoeLayer.synthetic(0, 256, 4096, 2048, 8, 0.0, DEV)
+
+
+def test_moe_decode_full_size(full_layer):
+    # 256 experts, hidden 4096, expert-intermediate 2048, top-8: sampled tokens
+    X = inputs.hidden_states(0, 3, 4096)
+    run_and_check(full_layer, 0, X)
+
+
+def test_moe_decode_is_deterministic(full_layer):
+    x = inputs.hidden_states(5, 1, 4096)[0].to(DEV)
+    ws = full_layer.workspace(1)
+    a = [t.clone() for t in full_layer.ffn(x, ws)]
+    b = full_layer.ffn(x, ws)
+    for p, q in zip(a, b):
+        assert torch.equal(p, q)
+
+
+def test_moe_top_k_equals_n_experts():
+    layer = MoeLayer.synthetic(3, 4, 256, 256, 4, 0.0, DEV)
+    run_and_check(layer, 3, inputs.hidden_states(3, 2, 256))
+
+
+def test_moe_argument_errors(full_layer):
+    ws = full_layer.workspace(1)
+    x = torch.zeros(4096, device=DEV)
+    with pytest.raises(B.TqfxError) as e:
+        full_layer.ffn(x, ws[:1024])
+    assert e.value.status == 4
+    bad = B.c_router(full_layer.router_w, None, 0)
+    with pytest.raises(B.TqfxError) as e:
+        B.tqfx4_moe_ffn(full_layer.ex, bad, x, x, torch.zeros(8, dtype=torch.int32, device=DEV),
+                        torch.zeros(8, device=DEV), ws)
+    assert e.value.status == 2
+    with pytest.raises(B.TqfxError) as e:
+        full_layer.ffn(x[1:], ws)
+    assert e.value.status == 3
