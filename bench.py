@@ -1,0 +1,354 @@
+"""Benchmark of the tq2_0_fx4 MoE decode hot path on GB300.
+
+Workload (one "step" = one token through one routed-expert MoE layer): 256
+experts with gate/up 4096 -> 2048 and down 2048 -> 4096 projections in
+tq2_0_fx4 (Student-t(5) * 0.02 synthetic weights, 3.27 GB of blocks), an
+N(0, 0.02) fp32 router, top-8 with renormalized weights, N(0, 1) hidden
+states. Every step routes a different hidden state, so the experts it reads
+are (almost always) not the previous step's: the 3.27 GB expert pool is
+larger than the 129 MB L2.
+
+Metric: effective tq2_0_fx4 GB/s = (bytes of the 8 selected experts' blocks +
+router weights) per token / time per token; tokens/s per MoE layer is the
+same number divided by the bytes per token, reported beside it.
+
+    python bench.py [--steps K] [--warmup W] [--gpus N] [--impl ours|reference]
+
+Under torchrun (N > 1) every rank runs its own replica on its own GPU (the
+path has no exchange step here: replicas only) and rank 0 reports the
+aggregate.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+E, H, I, TOPK = 256, 4096, 2048, 8
+SEED = 0
+POOL = 256  # distinct hidden states cycled through the steps
+WORKLOAD = "moe_decode_t1_e256_h4096_i2048_top8"
+METRIC = "effective tq2_0_fx4 GB/s (MoE-layer decode)"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def bytes_per_token():
+    from paper_2608_08910_gb300 import binding as B
+    mb = B.tqfx4_matrix_bytes(I, H)  # gate = up = down size
+    return TOPK * 3 * mb + E * H * 4, TOPK * 2 * mb, TOPK * mb
+
+
+class ClockSampler:
+    """nvidia-smi clock and throttle-reason samples while the timed region runs."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.samples = []
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.QUERY, "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append([x.strip() for x in line.split(",")])
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(s[1]) for s in self.samples if s[1].replace(".", "", 1).isdigit()]
+        mx = [float(s[2]) for s in self.samples if s[2].replace(".", "", 1).isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for s in self.samples:
+            for n, v in zip(names, s[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(self.samples)}
+
+
+def cpu_baseline(seconds_budget=20.0, tokens=None):
+    """The oracle (plain single-threaded C) on a bounded sample of the same
+    workload: whole tokens through the MoE layer, packing of the experts they
+    select excluded from the time. Returns (GB/s, tokens, seconds)."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2608_08910_gb300 import inputs
+
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    Wr = inputs.router_weight(SEED, E, H, dev).cpu().numpy()
+    X = inputs.hidden_states(SEED, POOL, H, dev).cpu().numpy()
+    per_token, _, _ = bytes_per_token()
+    total_t, done = 0.0, 0
+    n_max = tokens if tokens else 64
+    for t in range(n_max):
+        _, idx, _ = oracle.router(Wr, None, X[t], TOPK)
+        ex = {int(e): tuple(oracle.pack_rtn(inputs.expert_matrix(SEED, int(e), p, H, I, dev).cpu().numpy())
+                            for p in (0, 1, 2)) for e in idx}
+        t0 = time.perf_counter()
+        oracle.moe_tokens(ex, E, H, I, Wr, None, TOPK, X[t])
+        total_t += time.perf_counter() - t0
+        done += 1
+        if tokens is None and total_t >= seconds_budget:
+            break
+    return per_token * done / total_t / 1e9, done, total_t
+
+
+def run_reference(args, rank, world):
+    """--impl reference: the CPU oracle, as it stands, on this machine's host
+    cores; each step is one expert FFN of a routed token (1/8 of a token)."""
+    if rank != 0:
+        return
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2608_08910_gb300 import binding as B
+    from paper_2608_08910_gb300 import inputs
+
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    Wr = inputs.router_weight(SEED, E, H, dev).cpu().numpy()
+    X = inputs.hidden_states(SEED, POOL, H, dev).cpu().numpy()
+    mb = B.tqfx4_matrix_bytes(I, H)
+    cache = {}
+
+    def expert(e):
+        if e not in cache:
+            cache.clear()
+            cache[e] = tuple(oracle.pack_rtn(inputs.expert_matrix(SEED, e, p, H, I, dev).cpu().numpy())
+                             for p in (0, 1, 2))
+        return cache[e]
+
+    def step(s):
+        t = s // TOPK
+        _, idx, _ = oracle.router(Wr, None, X[t % POOL], TOPK)
+        g, u, d = expert(int(idx[s % TOPK]))
+        t0 = time.perf_counter()
+        oracle.expert_ffn(g, u, d, H, I, X[t % POOL])
+        return time.perf_counter() - t0
+
+    for s in range(args.warmup):
+        step(s)
+    el = sum(step(args.warmup + s) for s in range(args.steps))
+    bytes_step = 3 * mb
+    value = bytes_step * args.steps / el / 1e9
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "i8xi4-i32,f32",
+        "data": "synthetic", "config": {"workload": WORKLOAD, "sample": "one expert FFN per step (1/8 token)"},
+        "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": "%d expert FFNs of routed tokens, packing excluded" % args.steps},
+        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+
+    import torch
+    import torch.distributed as dist
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    from paper_2608_08910_gb300 import binding as B
+    from paper_2608_08910_gb300 import inputs
+    from paper_2608_08910_gb300.moe import MoeLayer
+
+    assert args.warmup >= 3, "at least 3 warm-up steps"
+    dev = torch.device("cuda", local)
+    layer = MoeLayer.synthetic(SEED, E, H, I, TOPK, 0.0, dev)
+    ws = layer.workspace(1)
+    X = inputs.hidden_states(SEED + rank, POOL, H, dev)
+    out = torch.empty(H, device=dev)
+    sel = torch.empty(TOPK, dtype=torch.int32, device=dev)
+    selw = torch.empty(TOPK, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    per_token, gu_bytes, dn_bytes = bytes_per_token()
+
+    def step(i, events=None, st=stream):
+        layer.ffn(X[i % POOL], ws, out, sel, selw, stream=st, events=events)
+
+    for i in range(args.warmup):
+        step(i)
+    B.tqfx4_check(ws)
+
+    # The K steps are captured once into a CUDA graph (the launches keep their
+    # programmatic-dependency edges) so that host launch cost stays out of the
+    # device timing; each step routes a different hidden state.
+    cap_stream = torch.cuda.Stream(dev)
+    cap_stream.wait_stream(stream)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(cap_stream):
+        with torch.cuda.graph(graph, stream=cap_stream):
+            for i in range(args.steps):
+                step(args.warmup + i, st=cap_stream)
+    stream.wait_stream(cap_stream)
+    graph.replay()  # untimed
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
+
+    # ---- timed region: K steps, device time, max over ranks ----
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        graph.replay()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+    B.tqfx4_check(ws)
+    t = ev0.elapsed_time(ev1) / 1e3
+    if world > 1:
+        tt = torch.tensor([t], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t = float(tt.item())
+    tokens = args.steps * world
+    value = per_token * tokens / t / 1e9
+
+    # ---- dominant kernel: CUDA events around every stage of every step, on
+    # the launching stream (a second graph of the same K steps; the stage
+    # launches are plain stream-ordered here) ----
+    n_st = B.tqfx4_moe_stage_count(0, 0)
+    names = [B.tqfx4_moe_stage_name(0, 0, s) for s in range(n_st)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_st + 1)] for _ in range(args.steps)]
+    for row in evs:
+        for e_ in row:
+            e_.record(stream)
+    torch.cuda.synchronize()
+    graph2 = torch.cuda.CUDAGraph()
+    cap_stream.wait_stream(stream)
+    with torch.cuda.stream(cap_stream):
+        with torch.cuda.graph(graph2, stream=cap_stream):
+            for i in range(args.steps):
+                step(args.warmup + i, events=evs[i], st=cap_stream)
+    stream.wait_stream(cap_stream)
+    graph2.replay()
+    torch.cuda.synchronize()
+    acc = [0.0] * n_st
+    for row in evs:
+        for s in range(n_st):
+            acc[s] += row[s].elapsed_time(row[s + 1]) / 1e3
+    stage_s = {names[s]: acc[s] / args.steps for s in range(n_st)}
+    dom = "gate_up"
+    peak, peak_kind = _peaks()
+    achieved = gu_bytes / stage_s[dom] / 1e9
+
+    # ---- end to end through the public API with host buffers ----
+    Xh = X.cpu().pin_memory()
+    xin = torch.empty(H, device=dev)
+    outh = torch.empty(H, pin_memory=True)
+    selh = torch.empty(TOPK, dtype=torch.int32, pin_memory=True)
+    for i in range(3):
+        xin.copy_(Xh[i], non_blocking=True)
+        layer.ffn(xin, ws, out, sel, selw, stream=stream)
+        outh.copy_(out, non_blocking=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for i in range(args.steps):
+        xin.copy_(Xh[i % POOL], non_blocking=True)
+        layer.ffn(xin, ws, out, sel, selw, stream=stream)
+        outh.copy_(out, non_blocking=True)
+        selh.copy_(sel, non_blocking=True)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
+    te = ev0.elapsed_time(ev1) / 1e3
+    if world > 1:
+        tt = torch.tensor([te], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        te = float(tt.item())
+    e2e = per_token * tokens / te / 1e9
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "i8xi4-i32,f32", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "experts": E, "hidden": H, "inter": I, "top_k": TOPK,
+                   "tokens_per_step": 1, "bytes_per_token": per_token,
+                   "l2": "inputs larger than L2: 3.27 GB expert pool, a different hidden state per step",
+                   "parallelism": "replicas" if world > 1 else "single"},
+        "tokens_per_s": tokens / t,
+        "pct_of_hbm_peak": 100.0 * value / peak,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None, "kernel": dom,
+                     "peak_source": peak_kind + " (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
+                     else "fallback 6.8 TB/s",
+                     "stage_us": {k: v * 1e6 for k, v in stage_s.items()}},
+        "e2e": {"value": e2e, "unit": "GB/s", "h2d_bytes_per_step": H * 4,
+                "d2h_bytes_per_step": H * 4 + TOPK * 4},
+        "gpu_launches": 3 * args.steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        v, n, secs = cpu_baseline()
+        line["cpu_baseline"] = {"value": v, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                "sample": "%d tokens through the layer (%.1f s), expert packing excluded" % (n, secs)}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

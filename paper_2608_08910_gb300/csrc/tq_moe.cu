@@ -352,8 +352,14 @@ cudaError_t launch_moe_decode(const MoeArgs &a0, const float *x, float *out, int
     cudaError_t e = allow_max_smem(reinterpret_cast<const void *>(gate_up_kernel), set_gu);
     if (e == cudaSuccess) e = allow_max_smem(reinterpret_cast<const void *>(down_kernel), set_dn);
     if (e != cudaSuccess) return e;
+    // under stream capture the records become event nodes of the graph
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (events) cudaStreamIsCapturing(st, &cap);
     auto rec = [&](int i) {
-        if (events && events[i]) cudaEventRecord(static_cast<cudaEvent_t>(events[i]), st);
+        if (events && events[i])
+            cudaEventRecordWithFlags(static_cast<cudaEvent_t>(events[i]), st,
+                                     cap == cudaStreamCaptureStatusActive ? cudaEventRecordExternal
+                                                                          : cudaEventRecordDefault);
     };
     rec(0);
     router_kernel<<<a.E + (a.nbh + 3) / 4, 128, 0, st>>>(a);
