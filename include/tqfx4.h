@@ -215,6 +215,36 @@ tqfx4_status tqfx4_moe_grouped(const tqfx4_experts *ex, const tqfx4_router *rt,
                                void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * tqfx4_moe_ffn_noalloc -- tqfx4_moe_ffn without a caller workspace, for
+ * callers that cannot allocate device memory: for example a plug-in whose
+ * host application owns all device memory through its own allocator and
+ * hands it no workspace, or a real-time serving loop in which an allocation
+ * (which may block and synchronize the device) is not allowed. The paper
+ * has no counterpart; it is a convenience of this library.
+ *   Inputs, outputs and their rules are those of tqfx4_moe_ffn. The scratch
+ *   is a device array of TQFX4_NOALLOC_SCRATCH_BYTES (1 MiB) inside the
+ *   library, which every GPU that loads the library keeps until the process
+ *   exits. Shapes whose tqfx4_moe_workspace_bytes exceeds that size are
+ *   rejected with TQFX4_EWORKSPACE before anything is enqueued (the
+ *   256-expert, hidden 4096, intermediate 2048, top-8 layer needs about
+ *   0.35 MiB). The call allocates nothing: no cudaMalloc, no cudaFree.
+ *   The first call on a device looks up the scratch's device address
+ *   (cudaGetSymbolAddress) with that device current; make that first call
+ *   before any stream capture. Each call clears the scratch's status word
+ *   and counters on `stream` before its kernels; device-side error reports
+ *   therefore are not kept between calls (use tqfx4_moe_ffn with a workspace
+ *   and tqfx4_check to read them).
+ *   All calls share the one scratch array, which keeps the last call's
+ *   contents: calls whose work overlaps on the GPU (different streams, or
+ *   different host threads without ordering) race on it and must not be
+ *   issued.
+ */
+#define TQFX4_NOALLOC_SCRATCH_BYTES (1 << 20)
+tqfx4_status tqfx4_moe_ffn_noalloc(const tqfx4_experts *ex, const tqfx4_router *rt,
+                                   const float *x, float *out, int32_t *sel_idx, float *sel_w,
+                                   void *stream);
+
+/*
  * Profiling variants: identical to the calls above, and additionally record
  * `events[i]` (cudaEvent_t, created by the caller) on the stream before
  * stage i, and events[n_stages] after the last stage, where n_stages is

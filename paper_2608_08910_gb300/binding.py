@@ -17,6 +17,7 @@ TQFX4_QK = 256
 TQFX4_ROWS = 4
 TQFX4_BLOCK_BYTES = 520
 TQFX4_STATUS_BYTES = 256
+TQFX4_NOALLOC_SCRATCH_BYTES = 1 << 20
 TQFX4_SRC_TRITS = 0
 TQFX4_SRC_F32_RTN = 1
 TQFX4_PATH_AUTO = 0
@@ -67,6 +68,7 @@ _SIGS = {
                                         _int, _vp, _sz, _vp, C.POINTER(_vp)]),
     "tqfx4_moe_workspace_views": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int, _int,
                                          C.POINTER(CMoeViews)]),
+    "tqfx4_moe_ffn_noalloc": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp]),
     "tqfx4_check": (_int, [_vp, _vp]),
     "tqfx4_last_error": (C.c_char_p, []),
     "tqfx4_status_string": (C.c_char_p, [_int]),
@@ -164,6 +166,13 @@ def tqfx4_moe_ffn(ex, rt, x, out, sel_idx, sel_w, ws, stream=None, events=None):
         rc = lib().tqfx4_moe_ffn_traced(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w),
                                         _p(ws), _nbytes(ws), _s(stream), arr)
     _check(rc, "tqfx4_moe_ffn")
+
+
+def tqfx4_moe_ffn_noalloc(ex, rt, x, out, sel_idx, sel_w, stream=None):
+    """tqfx4_moe_ffn on the library's own scratch (for callers that cannot
+    allocate device memory; see include/tqfx4.h)."""
+    _check(lib().tqfx4_moe_ffn_noalloc(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w),
+                                       _s(stream)), "tqfx4_moe_ffn_noalloc")
 
 
 def tqfx4_moe_grouped(ex, rt, X, T, OUT, sel_idx, sel_w, path, ws, stream=None, events=None):

@@ -48,6 +48,12 @@ tqfx4_status check_nk(int64_t n, int64_t k, const char *fn) {
 
 }  // namespace
 
+namespace tq {
+// Record a failure message for tqfx4_last_error() from other translation
+// units of the library.
+tqfx4_status api_fail(tqfx4_status s, const char *msg) { return fail(s, "%s", msg); }
+}  // namespace tq
+
 extern "C" {
 
 int64_t tqfx4_matrix_bytes(int64_t n, int64_t k) {

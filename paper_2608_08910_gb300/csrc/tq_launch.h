@@ -20,6 +20,8 @@ cudaError_t launch_quantize(const float *x, int64_t m, int64_t k, int8_t *q, flo
 cudaError_t launch_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
                         const int32_t *bsum, float *y, int32_t *block_sums, int *status, cudaStream_t st);
 
+tqfx4_status api_fail(tqfx4_status s, const char *msg);
+
 struct MoeArgs;
 struct MoeLayout;
 bool moe_decode_args(const tqfx4_experts *ex, const tqfx4_router *rt, void *ws, MoeArgs &a, MoeLayout &L);
