@@ -206,8 +206,9 @@ tqfx4_status tqfx4_moe_ffn(const tqfx4_experts *ex, const tqfx4_router *rt,
  * touched expert once over all of its tokens (its weights are read once),
  * then combine each token's expert outputs in rank order. Results equal
  * tqfx4_moe_ffn applied to each token.
- *   X, OUT: fp32 [T][hidden] (device). sel_idx int32 [T][top_k], sel_w fp32
- *   [T][top_k] (device). T == 0 does nothing.
+ *   X, OUT: fp32 [T][hidden] (device, 16-byte aligned). sel_idx int32
+ *   [T][top_k], sel_w fp32 [T][top_k] (device). T == 0 does nothing. hidden
+ *   and inter must be multiples of 512 on this path.
  */
 tqfx4_status tqfx4_moe_grouped(const tqfx4_experts *ex, const tqfx4_router *rt,
                                const float *X, int64_t T, float *OUT,
@@ -286,6 +287,7 @@ typedef struct tqfx4_moe_views {
     size_t offsets;    /* int32 [n_experts + 1] (grouped only) */
     size_t pair_token; /* int32 [P] (grouped only) */
     size_t pair_slot;  /* int32 [P] (grouped only) */
+    size_t pair_of;    /* int32 [T][top_k]: position of each (token, slot) pair (grouped only) */
 } tqfx4_moe_views;
 
 tqfx4_status tqfx4_moe_workspace_views(const tqfx4_experts *ex, const tqfx4_router *rt,

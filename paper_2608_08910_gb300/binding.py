@@ -47,7 +47,7 @@ class CRouter(C.Structure):
 
 class CMoeViews(C.Structure):
     _fields_ = [(n, _sz) for n in ("logits", "logits_lo", "qx", "dx", "bx", "g", "u", "h", "qh", "dh", "bh", "o",
-                                   "counts", "offsets", "pair_token", "pair_slot")]
+                                   "counts", "offsets", "pair_token", "pair_slot", "pair_of")]
 
 
 _SIGS = {

@@ -162,13 +162,14 @@ size_t tqfx4_moe_workspace_bytes(const tqfx4_experts *ex, const tqfx4_router *rt
 
 int tqfx4_moe_stage_count(int grouped, int path) {
     (void)path;
-    return grouped ? 0 : 3;
+    return grouped ? tq::grouped_stage_count() : 3;
 }
 
 const char *tqfx4_moe_stage_name(int grouped, int path, int stage) {
     (void)path;
     static const char *dec[] = {"router", "gate_up", "down"};
-    if (!grouped && stage >= 0 && stage < 3) return dec[stage];
+    if (grouped) return tq::grouped_stage_name(stage);
+    if (stage >= 0 && stage < 3) return dec[stage];
     return "";
 }
 
@@ -206,19 +207,42 @@ tqfx4_status tqfx4_moe_ffn_traced(const tqfx4_experts *ex, const tqfx4_router *r
     return moe_ffn_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, events);
 }
 
+static tqfx4_status moe_grouped_impl(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X, int64_t T,
+                                     float *OUT, int32_t *sel_idx, float *sel_w, int path, void *ws,
+                                     size_t ws_bytes, void *stream, void *const *events) {
+    const char *fn = "tqfx4_moe_grouped";
+    tqfx4_status s = check_moe_shapes(ex, rt, fn);
+    if (s) return s;
+    if (T < 0) return fail(TQFX4_EINVAL, "%s: negative token count", fn);
+    if (path < TQFX4_PATH_AUTO || path > TQFX4_PATH_PREFILL) return fail(TQFX4_EINVAL, "%s: unknown path %d", fn, path);
+    if (ex->hidden % 512 || ex->inter % 512)
+        return fail(TQFX4_ESHAPE, "%s: hidden and inter must be multiples of 512 for the grouped path", fn);
+    if (T * rt->top_k > (int64_t(1) << 30)) return fail(TQFX4_ESHAPE, "%s: too many tokens", fn);
+    if ((s = check_moe_ptrs(ex, rt, fn))) return s;
+    if (T == 0) return ok();
+    if (!X || !OUT || !sel_idx || !sel_w) return fail(TQFX4_EINVAL, "%s: NULL X, OUT or selection output", fn);
+    if (!aligned(X, 16) || !aligned(OUT, 16) || !aligned(sel_idx, 4) || !aligned(sel_w, 4))
+        return fail(TQFX4_EALIGN, "%s: X and OUT must be 16-byte aligned", fn);
+    tq::GroupedArgs a;
+    tq::MoeLayout L;
+    tq::grouped_args(ex, rt, T, nullptr, a, L);
+    if ((s = check_ws(ws, ws_bytes, L.total, fn))) return s;
+    tq::grouped_args(ex, rt, T, ws, a, L);
+    cudaError_t e = tq::launch_moe_grouped(a, X, OUT, sel_idx, sel_w, static_cast<cudaStream_t>(stream), events);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
 tqfx4_status tqfx4_moe_grouped(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X, int64_t T,
                                float *OUT, int32_t *sel_idx, float *sel_w, int path, void *ws, size_t ws_bytes,
                                void *stream) {
-    (void)X; (void)T; (void)OUT; (void)sel_idx; (void)sel_w; (void)path; (void)ws; (void)ws_bytes; (void)stream;
-    (void)ex; (void)rt;
-    return fail(TQFX4_EINVAL, "tqfx4_moe_grouped: not available in this build");
+    return moe_grouped_impl(ex, rt, X, T, OUT, sel_idx, sel_w, path, ws, ws_bytes, stream, nullptr);
 }
 
 tqfx4_status tqfx4_moe_grouped_traced(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X, int64_t T,
                                       float *OUT, int32_t *sel_idx, float *sel_w, int path, void *ws,
                                       size_t ws_bytes, void *stream, void *const *events) {
-    (void)events;
-    return tqfx4_moe_grouped(ex, rt, X, T, OUT, sel_idx, sel_w, path, ws, ws_bytes, stream);
+    return moe_grouped_impl(ex, rt, X, T, OUT, sel_idx, sel_w, path, ws, ws_bytes, stream, events);
 }
 
 tqfx4_status tqfx4_moe_workspace_views(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t tokens,
@@ -246,6 +270,7 @@ tqfx4_status tqfx4_moe_workspace_views(const tqfx4_experts *ex, const tqfx4_rout
     v->offsets = L.offsets;
     v->pair_token = L.pair_token;
     v->pair_slot = L.pair_slot;
+    v->pair_of = L.pair_of;
     return ok();
 }
 

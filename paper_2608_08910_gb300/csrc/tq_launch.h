@@ -28,6 +28,14 @@ bool moe_decode_args(const tqfx4_experts *ex, const tqfx4_router *rt, void *ws, 
 cudaError_t launch_moe_decode(const MoeArgs &a, const float *x, float *out, int32_t *sel_idx, float *sel_w,
                               cudaStream_t st, void *const *events);
 int gate_up_smem(const MoeArgs &a);
+
+struct GroupedArgs;
+bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, void *ws, GroupedArgs &a,
+                  MoeLayout &L);
+cudaError_t launch_moe_grouped(const GroupedArgs &a, const float *X, float *OUT, int32_t *sel_idx, float *sel_w,
+                               cudaStream_t st, void *const *events);
+int grouped_stage_count();
+const char *grouped_stage_name(int s);
 int down_smem(const MoeArgs &a);
 
 }  // namespace tq

@@ -83,7 +83,7 @@ __global__ void __launch_bounds__(128) router_kernel(MoeArgs a) {
     if (!last) return;
     topk_block(a.logits, a.logits_lo, a.E, a.top_k, a.sel, topk_s);
     TQ_STAMP(0, 5);
-    if (threadIdx.x < a.top_k) a.sel_out[threadIdx.x] = __ldcg(a.sel + threadIdx.x);
+    if (threadIdx.x < a.top_k) a.sel_out[threadIdx.x] = topk_s.res[threadIdx.x];
     if (threadIdx.x == 0) a.ctr[kCtrRouter] = 0;
     TQ_STAMP(0, 3);
 }

@@ -20,8 +20,13 @@ struct MoeLayout {
     size_t qh, dh, bh;
     size_t o;        // fp32 [P][H]
     size_t counts, offsets, pair_token, pair_slot, pair_of;
+    size_t chunk_expert, chunk_begin, chunk_len, n_chunks;  // grouped GEMM work list
+    int64_t max_chunks;
     size_t total;
 };
+
+// Tokens (pairs) per chunk of the grouped GEMM.
+constexpr int GG_TOK = 64;
 
 inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
@@ -62,8 +67,15 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.pair_token = take(4 * static_cast<size_t>(P));
         L.pair_slot = take(4 * static_cast<size_t>(P));
         L.pair_of = take(4 * static_cast<size_t>(P));
+        L.max_chunks = P / GG_TOK + E + 1;
+        L.chunk_expert = take(4 * static_cast<size_t>(L.max_chunks));
+        L.chunk_begin = take(4 * static_cast<size_t>(L.max_chunks));
+        L.chunk_len = take(4 * static_cast<size_t>(L.max_chunks));
+        L.n_chunks = take(4);
     } else {
         L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = SIZE_MAX;
+        L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
+        L.max_chunks = 0;
     }
     L.total = off;
     return L;
@@ -98,6 +110,33 @@ struct MoeArgs {
     int rpu_gu, slot_gu, stages_gu, warps_gu, parts_gu;
     // down geometry
     int rpu_d, slot_d, stages_d, warps_d, parts_d;
+};
+
+// Arguments of the grouped (T-token) kernels.
+struct GroupedArgs {
+    int E, H, I, top_k, T, P, nbh, nbi;
+    const uint8_t *gate, *up, *down;
+    int64_t mb_gu, mb_d;
+    const float *wr, *bias;
+    const float *X;
+    float *OUT;
+    int32_t *sel_out;
+    float *selw_out;
+    int *status;
+    float *logits, *logits_lo;
+    int *sel;
+    float *selw;
+    int8_t *qx;
+    float *dx;
+    int *bx;
+    float *g, *u, *h;
+    int8_t *qh;
+    float *dh;
+    int *bh;
+    float *o;
+    int *counts, *offsets, *pair_token, *pair_slot, *pair_of;
+    int *chunk_expert, *chunk_begin, *chunk_len, *n_chunks;
+    int keep_h;
 };
 
 // Shared-memory bytes of one quantized activation vector of nb blocks
@@ -165,6 +204,40 @@ __device__ __forceinline__ void router_logit_block(const float *w, const float *
     }
 }
 
+// One router logit by one warp (H a multiple of 128): Dot2 over the lane's
+// float4s with four (sum, error) pairs, then double-binary32 sums across the
+// warp. Every lane receives (hi, lo).
+__device__ __forceinline__ void router_logit_warp(const float *w, const float *x, int H, float &hi, float &lo) {
+    const int lane = threadIdx.x & 31;
+    const float4 *w4 = reinterpret_cast<const float4 *>(w);
+    const float4 *x4 = reinterpret_cast<const float4 *>(x);
+    float s[4] = {0.f, 0.f, 0.f, 0.f}, c[4] = {0.f, 0.f, 0.f, 0.f};
+    const int n4 = H >> 2;
+#pragma unroll 4
+    for (int i = lane; i < n4; i += 32) {
+        const float4 wv = __ldg(w4 + i), xv = __ldg(x4 + i);
+        const float ww[4] = {wv.x, wv.y, wv.z, wv.w}, xx[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float p = __fmul_rn(ww[q], xx[q]);
+            const float pe = __fmaf_rn(ww[q], xx[q], -p);
+            float t, te;
+            two_sum(s[q], p, t, te);
+            s[q] = t;
+            c[q] = __fadd_rn(c[q], __fadd_rn(te, pe));
+        }
+    }
+    float h01, l01, h23, l23;
+    ff_add(s[0], c[0], s[1], c[1], h01, l01);
+    ff_add(s[2], c[2], s[3], c[3], h23, l23);
+    ff_add(h01, l01, h23, l23, hi, lo);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float oh = __shfl_xor_sync(0xffffffffu, hi, o), ol = __shfl_xor_sync(0xffffffffu, lo, o);
+        ff_add(hi, lo, oh, ol, hi, lo);
+    }
+}
+
 // Total order on binary32 values as unsigned keys (-0 folded into +0).
 __device__ __forceinline__ uint32_t order_key(float f) {
     const uint32_t u = __float_as_uint(f + 0.0f);
@@ -184,6 +257,7 @@ __device__ __forceinline__ unsigned long long topk_key(float hi, float lo, int e
 
 // Shared scratch of topk_block.
 struct TopkScratch {
+    int res[TQFX4_MAX_TOP_K];  // the selection, in rank order
     unsigned long long key[TQFX4_MAX_EXPERTS];
     int hist[256];
     int cand[TQFX4_MAX_EXPERTS];
@@ -197,8 +271,8 @@ struct TopkScratch {
 // (1) the keys' hi parts are binned linearly between their minimum and
 // maximum into 256 bins; (2) the highest bin b* whose suffix count reaches k
 // is found; (3) only the experts in bins >= b* (normally a few more than k)
-// are ranked exactly by comparing full keys. Writes sel[rank] (global
-// memory). All threads must call.
+// are ranked exactly by comparing full keys. Leaves the selection in s.res
+// (shared) and writes it to sel (global). All threads must call.
 __device__ __forceinline__ void topk_block(const float *lhi, const float *llo, int E, int k, int *sel,
                                            TopkScratch &s) {
     const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31;
@@ -264,9 +338,10 @@ __device__ __forceinline__ void topk_block(const float *lhi, const float *llo, i
         const unsigned long long ke = s.key[e];
         int r = 0;
         for (int cj = 0; cj < nc; ++cj) r += s.key[s.cand[cj]] > ke;
-        if (r < k) sel[r] = e;
+        if (r < k) s.res[r] = e;
     }
     __syncthreads();
+    if (tid < k) sel[tid] = s.res[tid];
 }
 
 // ---- double-binary32 softmax ----------------------------------------------------
@@ -326,7 +401,7 @@ __device__ __forceinline__ void ff_exp_nonpos(float dh, float dl, float &eh, flo
 // w_j = exp(l_j - l_0) / sum_i exp(l_i - l_0), in double-binary32
 // arithmetic, each w_j rounded once to binary32 (so it matches a binary64
 // evaluation rounded to binary32). Writes w[0..k) (any memory) from lanes
-// j < k. All lanes must call.
+// j < k (followed by __syncwarp). All lanes must call.
 __device__ __forceinline__ void softmax_ff_warp(const float *lhi, const float *llo, const int *sel, int k,
                                                 float *w) {
     const int lane = threadIdx.x & 31;

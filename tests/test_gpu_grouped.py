@@ -1,0 +1,141 @@
+"""GPU parity of tqfx4_moe_grouped (T tokens grouped by expert: batched
+decode and prefill) against the CPU oracle, through the C ABI.
+
+Per call: the routing of every token (bit-exact up to accepted near-ties),
+the grouping (counts, offsets and the stable expert-then-token order,
+bit-exact against the oracle's counting sort), and for sampled tokens the
+per-pair g, u, quantized h and expert outputs (bit-exact) and the combined
+output (within 1e-4 relative; equal to tqfx4_moe_ffn on the same token).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_08910_gb300 import binding as B
+from paper_2608_08910_gb300 import inputs
+from paper_2608_08910_gb300.moe import MoeLayer
+from tests.parity import FP32_TOL, check_selection, oracle_experts, rel_err, selection_tolerance
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+def run_grouped(layer, X, path=0):
+    T = X.shape[0]
+    ws = layer.workspace(T, path)
+    OUT, sel, selw = layer.grouped(X.to(DEV), ws, path)
+    B.tqfx4_check(ws)
+    return ws, OUT.cpu().numpy(), sel.cpu().numpy(), selw.cpu().numpy()
+
+
+def check_grouped(layer, seed, X, sample, path=0, check_stages=True):
+    H, I, E, k = layer.hidden, layer.inter, layer.n_experts, layer.top_k
+    T = X.shape[0]
+    P = T * k
+    ws, OUT, sel, selw = run_grouped(layer, X, path)
+    Wr = layer.router_w.cpu().numpy()
+    bias = None if layer.router_b is None else layer.router_b.cpu().numpy()
+    Xn = X.numpy()
+    ties = 0
+    for t in range(T):
+        logits, r_idx, r_w = oracle.router(Wr, bias, Xn[t], k)
+        n = check_selection(sel[t], logits, selection_tolerance(Wr, Xn[t], bias), k)
+        ties += n
+        if n == 0:
+            assert np.allclose(selw[t], r_w, rtol=1.2e-7, atol=0)
+    # grouping: the oracle's stable counting sort of the kernel's own selection
+    counts, offsets, pt, ps = oracle.group_by_expert(sel, E)
+    g = lambda name, dt, shape: layer.view(ws, name, dt, shape, tokens=T, grouped=1, path=path).cpu().numpy()
+    assert np.array_equal(g("counts", torch.int32, (E,)), counts)
+    assert np.array_equal(g("offsets", torch.int32, (E + 1,)), offsets)
+    assert np.array_equal(g("pair_token", torch.int32, (P,)), pt)
+    assert np.array_equal(g("pair_slot", torch.int32, (P,)), ps)
+    pair_of = g("pair_of", torch.int32, (T, k))
+    assert np.array_equal(pt[pair_of], np.repeat(np.arange(T), k).reshape(T, k))
+    if check_stages:
+        gv, uv = g("g", torch.float32, (P, I)), g("u", torch.float32, (P, I))
+        qh, ov = g("qh", torch.int8, (P, I)), g("o", torch.float32, (P, H))
+    for t in sample:
+        ex = oracle_experts(seed, sel[t], H, I)
+        ref, ridx, _ = oracle.moe_tokens(ex, E, H, I, Wr, bias, k, Xn[t])
+        if np.array_equal(ridx[0], sel[t]):
+            e_ = rel_err(OUT[t], ref[0])
+            assert e_ <= FP32_TOL, (t, e_)
+        if check_stages:
+            for j in range(k):
+                pos = pair_of[t, j]
+                ro, dbg = oracle.expert_ffn(*ex[int(sel[t, j])], H, I, Xn[t])
+                assert np.array_equal(gv[pos].view(np.uint32), dbg["g"].view(np.uint32))
+                assert np.array_equal(uv[pos].view(np.uint32), dbg["u"].view(np.uint32))
+                assert np.array_equal(qh[pos], dbg["qh"])
+                assert np.array_equal(ov[pos].view(np.uint32), ro.view(np.uint32))
+    return OUT, sel, selw, ties
+
+
+@pytest.mark.parametrize("E,H,I,k,T,zipf", [
+    (16, 512, 1024, 4, 20, 0.0),     # ragged counts, one chunk per expert
+    (8, 512, 512, 4, 200, 0.0),      # ~100 pairs per expert: two chunks, ragged tail
+    (32, 1024, 512, 6, 33, 1.1),     # skewed routing
+    (4, 512, 512, 4, 3, 0.0),        # top_k = n_experts
+    (64, 2048, 1536, 8, 1, 0.0),     # a single token; inter not a multiple of 1024
+])
+def test_grouped_small(E, H, I, k, T, zipf):
+    seed = 100 + E + T
+    layer = MoeLayer.synthetic(seed, E, H, I, k, zipf, DEV)
+    X = inputs.hidden_states(seed, T, H)
+    check_grouped(layer, seed, X, sample=range(min(T, 6)))
+
+
+def test_grouped_equals_per_token_moe_ffn():
+    layer = MoeLayer.synthetic(5, 32, 1024, 1024, 8, 0.0, DEV)
+    X = inputs.hidden_states(5, 24, 1024)
+    ws, OUT, sel, selw = run_grouped(layer, X)
+    wsd = layer.workspace(1)
+    for t in range(24):
+        out, s, w = layer.ffn(X[t].to(DEV), wsd)
+        assert np.array_equal(s.cpu().numpy(), sel[t])
+        assert np.array_equal(w.cpu().numpy(), selw[t])
+        assert np.array_equal(out.cpu().numpy().view(np.uint32), OUT[t].view(np.uint32))
+
+
+def test_grouped_empty_batch():
+    layer = MoeLayer.synthetic(6, 8, 512, 512, 2, 0.0, DEV)
+    ws = layer.workspace(1)
+    X = torch.zeros((0, 512), device=DEV)
+    OUT = torch.zeros((0, 512), device=DEV)
+    B.tqfx4_moe_grouped(layer.ex, layer.rt, X, 0, OUT, torch.zeros(0, dtype=torch.int32, device=DEV),
+                        torch.zeros(0, device=DEV), 0, ws)
+    B.tqfx4_check(ws)
+
+
+def test_grouped_rejects_odd_block_counts():
+    layer = MoeLayer.synthetic(6, 8, 768, 512, 2, 0.0, DEV)  # hidden = 3 blocks
+    X = inputs.hidden_states(6, 2, 768).to(DEV)
+    ws = torch.zeros(1 << 20, dtype=torch.uint8, device=DEV)
+    with pytest.raises(B.TqfxError) as e:
+        layer.grouped(X, ws)
+    assert e.value.status == 2
+
+
+@pytest.fixture(scope="module")
+def zipf_layer():
+    return MoeLayer.synthetic(0, 256, 4096, 2048, 8, 1.1, DEV)
+
+
+def test_grouped_decode_64_tokens_zipf_full_size(zipf_layer):
+    # batched decode: 64 tokens, 256 experts, top-8, Zipf(1.1) router bias
+    X = inputs.hidden_states(0, 64, 4096)
+    OUT, sel, selw, ties = check_grouped(zipf_layer, 0, X, sample=[0, 17, 63], path=B.TQFX4_PATH_DECODE)
+    hits = np.bincount(sel.ravel(), minlength=256)
+    assert hits.max() > 8 and (hits > 0).sum() < 256  # the skew is visible
+
+
+@pytest.fixture(scope="module")
+def prefill_layer():
+    return MoeLayer.synthetic(0, 256, 4096, 2048, 8, 0.0, DEV)
+
+
+def test_grouped_prefill_2048_tokens_full_size(prefill_layer):
+    X = inputs.hidden_states(1, 2048, 4096)
+    check_grouped(prefill_layer, 0, X, sample=[0, 1023, 2047], path=B.TQFX4_PATH_PREFILL, check_stages=False)

@@ -17,48 +17,10 @@ import oracle
 from paper_2608_08910_gb300 import binding as B
 from paper_2608_08910_gb300 import inputs
 from paper_2608_08910_gb300.moe import MoeLayer
-from tests.parity import FP32_TOL, rel_err
+from tests.parity import FP32_TOL, check_selection, oracle_experts, rel_err, selection_tolerance
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
-
-
-def oracle_experts(seed, experts, hidden, inter):
-    """Oracle-packed blocks of the given experts, from the generator's fp32
-    weights (the same draws the GPU layer was packed from)."""
-    out = {}
-    for e in experts:
-        out[int(e)] = tuple(
-            oracle.pack_rtn(inputs.expert_matrix(seed, int(e), p, hidden, inter, DEV).cpu().numpy())
-            for p in (inputs.PROJ_GATE, inputs.PROJ_UP, inputs.PROJ_DOWN))
-    return out
-
-
-def selection_tolerance(Wr, x, bias):
-    """Per-expert bound on |kernel logit - oracle logit|: the kernel's
-    compensated binary32 dot product (Dot2, error below gamma_n^2 sum|w x|
-    with per-thread chains of n <= H/128 terms, then double-binary32 sums
-    with relative error near 2^-44) plus the oracle's sequential binary64
-    sum (H 2^-53 sum|w x|), doubled for safety."""
-    terms = np.abs(Wr.astype(np.float64)) @ np.abs(x.astype(np.float64))
-    H = Wr.shape[1]
-    b = 0 if bias is None else np.abs(bias.astype(np.float64))
-    gamma = (H // 128 + 2) * 2.0 ** -24
-    return 2 * (gamma ** 2 + 16 * 2.0 ** -44 + H * 2.0 ** -53) * (terms + b) + 1e-300
-
-
-def check_selection(sel, logits, tol, k):
-    """Expert ids must equal the oracle's ranking except where two adjacent
-    candidates (ranks 0..k) are closer than the fp32 error bound."""
-    order = np.lexsort((np.arange(logits.size), -logits))
-    ties = 0
-    for r in range(k):
-        a, b = order[r], order[r + 1] if r + 1 < logits.size else order[r]
-        close = abs(logits[a] - logits[b]) <= tol[a] + tol[b]
-        if sel[r] != order[r]:
-            assert close, "rank %d: got expert %d, oracle %d" % (r, sel[r], order[r])
-            ties += 1
-    return ties
 
 
 def run_and_check(layer, seed, X, zipf_bias=None, check_stages=True):
