@@ -184,6 +184,99 @@ def run_reference(args, rank, world):
     print(json.dumps(line), flush=True)
 
 
+def run_grouped(args, rank, world, local):
+    """Batched decode (64 tokens, Zipf(1.1) router bias) or prefill (2048
+    tokens) through tqfx4_moe_grouped; one step = one call over the batch.
+    Metric: tokens/s, with the effective GB/s of the touched experts' blocks
+    and, for prefill, the dense-equivalent TFLOP/s of the expert GEMMs."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_08910_gb300 import binding as B
+    from paper_2608_08910_gb300 import inputs
+    from paper_2608_08910_gb300.moe import MoeLayer
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    T, zipf, path = (64, 1.1, B.TQFX4_PATH_DECODE) if args.workload == "grouped_decode_64" else \
+        (2048, 0.0, B.TQFX4_PATH_PREFILL)
+    dev = torch.device("cuda", local)
+    layer = MoeLayer.synthetic(SEED, E, H, I, TOPK, zipf, dev)
+    ws = layer.workspace(T, path)
+    n_batches = 4
+    Xs = [inputs.hidden_states(SEED + 97 * b + rank, T, H, dev) for b in range(n_batches)]
+    OUT = torch.empty((T, H), device=dev)
+    sel = torch.empty((T, TOPK), dtype=torch.int32, device=dev)
+    selw = torch.empty((T, TOPK), device=dev)
+    stream = torch.cuda.current_stream(dev)
+    for i in range(args.warmup):
+        layer.grouped(Xs[i % n_batches], ws, path, OUT, sel, selw, stream=stream)
+    B.tqfx4_check(ws)
+    mb = B.tqfx4_matrix_bytes(I, H)
+    touched = 0
+    for X in Xs:
+        layer.grouped(X, ws, path, OUT, sel, selw, stream=stream)
+        touched += int((torch.bincount(sel.flatten().long(), minlength=E) > 0).sum())
+    bytes_per_step = touched / n_batches * 3 * mb + E * H * 4
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for i in range(args.steps):
+            layer.grouped(Xs[i % n_batches], ws, path, OUT, sel, selw, stream=stream)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+    B.tqfx4_check(ws)
+    t = ev0.elapsed_time(ev1) / 1e3
+    if world > 1:
+        tt = torch.tensor([t], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t = float(tt.item())
+    tokens = T * args.steps * world
+    # per-stage device times (CUDA events on the launching stream)
+    n_st = B.tqfx4_moe_stage_count(1, path)
+    names = [B.tqfx4_moe_stage_name(1, path, s) for s in range(n_st)]
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(n_st + 1)]
+    for e_ in evs:
+        e_.record(stream)
+    acc = [0.0] * n_st
+    reps = min(args.steps, 10)
+    for i in range(reps):
+        layer.grouped(Xs[i % n_batches], ws, path, OUT, sel, selw, stream=stream, events=evs)
+        evs[-1].synchronize()
+        for s in range(n_st):
+            acc[s] += evs[s].elapsed_time(evs[s + 1]) / 1e3
+    stage_s = {names[s]: acc[s] / reps for s in range(n_st)}
+    peak_hbm, peak_kind = _peaks()
+    flops_gu = 2.0 * T * TOPK * 2 * I * H
+    line = {
+        "metric": "MoE-layer tokens/s (%s)" % args.workload, "value": tokens / t, "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "i8xi4-i32,f32",
+        "data": "synthetic",
+        "config": {"workload": args.workload, "tokens": T, "experts": E, "hidden": H, "inter": I, "top_k": TOPK,
+                   "zipf": zipf, "touched_experts_avg": touched / n_batches,
+                   "l2": "inputs larger than L2 (3.27 GB expert pool); 4 batches cycled"},
+        "effective_gbs": bytes_per_step * args.steps * world / t / 1e9,
+        "roofline": {"bound": "hbm", "achieved": bytes_per_step / (t / args.steps) / 1e9, "peak": peak_hbm,
+                     "unit": "GB/s", "frac": bytes_per_step / (t / args.steps) / 1e9 / peak_hbm,
+                     "traffic": None, "kernel": "whole step",
+                     "gate_up_tflops": flops_gu / stage_s["gate_up"] / 1e12,
+                     "stage_us": {k: v * 1e6 for k, v in stage_s.items()}},
+        "gpu_launches": 10 * args.steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -191,6 +284,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default="moe_decode",
+                    choices=["moe_decode", "grouped_decode_64", "prefill_2048"],
+                    help="moe_decode (default): 1 token; grouped_decode_64: 64 tokens with Zipf(1.1) "
+                         "routing; prefill_2048: 2048 tokens")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
@@ -199,6 +296,9 @@ def main():
 
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.workload != "moe_decode":
+        run_grouped(args, rank, world, local)
         return
 
     import torch

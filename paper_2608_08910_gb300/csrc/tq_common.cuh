@@ -28,8 +28,14 @@ extern __device__ unsigned long long tq_stamps[8][2048][8];
             tq_stamps[k][blockIdx.x][s] = t_;                                                       \
         }                                                                                           \
     } while (0)
+// Accumulate `v` into tq_stamps[k][cta][slot] (lane 0 of the calling warp).
+#define TQ_ADD(k, s, v)                                                                             \
+    do {                                                                                            \
+        if ((threadIdx.x & 31) == 0 && blockIdx.x < 2048) atomicAdd(&tq_stamps[k][blockIdx.x][s], (unsigned long long)(v)); \
+    } while (0)
 #else
 #define TQ_STAMP(k, s) ((void)0)
+#define TQ_ADD(k, s, v) ((void)0)
 #endif
 
 constexpr int QK = 256;           // elements per block along K

@@ -8,7 +8,8 @@
 //   group    counts per expert, exclusive scan, stable gather of the
 //            (token, slot) pairs (expert, then ascending token), and the
 //            work list of <= 64-pair chunks per expert
-//   quant_x  int8 quantization of the T hidden states
+//   quant_x  int8 quantization of the T hidden states, then a gather of
+//            each pair's token row into pair order
 //   gate_up  grouped GEMM of the gate and up projections over the chunks
 //   swiglu   h = silu(g) u per pair and its int8 quantization
 //   down     grouped GEMM of the down projection
@@ -19,9 +20,12 @@
 // (mma.sync m16n8k32, s8 x s8 -> s32; the nibbles u = c + 4 are the A
 // operand, S = U - 4 bsum), then applies the fixed float schedule
 // y = y + float(S) * (d * da) block by block, so its outputs are the
-// oracle's, bit for bit. One producer warp streams each stage (two blocks of
-// 32 row groups plus the chunk's activation rows) with cp.async.bulk; eight
-// consumer warps each own 16 weight rows.
+// oracle's, bit for bit. A producer warp streams each stage with TMA tensor
+// copies (one box of weight blocks, four swizzled boxes of pair-ordered
+// activations); four consumer warps each own 8 row groups (32 rows).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include "tq_launch.h"
 #include "tq_moe_common.cuh"
 
@@ -162,27 +166,28 @@ __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
 
 // ---------------------------------------------------------------- grouped GEMM
 
-constexpr int GG_CW = 8;                       // consumer warps, 16 weight rows each
-constexpr int GG_RG = GG_CW * 16 / 4;          // 32 row groups per tile
+// Tile: 128 weight rows (32 row groups) x one chunk of <= 64 pairs. Four
+// consumer warps own 8 row groups (32 rows) each and all 64 pairs; a fifth
+// warp produces. A stage is two 256-blocks: the 32 row groups' blocks (one
+// 2-D tensor copy, 1040 bytes per row group) and the chunk's 512 activation
+// bytes per pair (four 2-D tensor copies of one 128-byte line x 64 pairs,
+// 128-byte swizzled so that ldmatrix reads are conflict-free).
+constexpr int GG_CW = 4;
+constexpr int GG_RG = GG_CW * 8;               // 32 row groups per tile
 constexpr int GG_KB = 2;                       // 256-blocks per stage
 constexpr int GG_STAGES = 3;
 constexpr int GG_WROW = GG_KB * BLOCK_BYTES;   // 1040 bytes per row group per stage
-constexpr int GG_TSTRIDE = GG_KB * QK + 32;    // 544: activation row stride in shared memory
-constexpr int GG_W_BYTES = GG_RG * GG_WROW;    // 33280
-constexpr int GG_T_BYTES = GG_TOK * GG_TSTRIDE;  // 34816
-constexpr int GG_S_BYTES = GG_TOK * GG_KB * 8;   // da and bsum
+constexpr int GG_W_BYTES = 33 * 1024;          // 32 x 1040 = 33280, padded to 1 KB
+constexpr int GG_LINE_BYTES = GG_TOK * 128;    // one 128-byte line of 64 pairs
+constexpr int GG_T_BYTES = 4 * GG_LINE_BYTES;  // 32768
+constexpr int GG_S_BYTES = 2048;               // da and bsum boxes: 64 pairs x 4 blocks each
 constexpr int GG_STAGE_BYTES = GG_W_BYTES + GG_T_BYTES + GG_S_BYTES;
-constexpr int GG_SMEM = GG_STAGES * GG_STAGE_BYTES + 2 * GG_STAGES * 8;
+constexpr int GG_SMEM = GG_STAGES * GG_STAGE_BYTES + 1024 + 2 * GG_STAGES * 8;
 
 struct GemmJob {
-    const uint8_t *mat0;  // expert 0's matrix; expert e at mat0 + e * mb
-    int64_t mb;
-    int N, nb;            // rows and 256-blocks per row of one expert matrix
-    const int8_t *act;    // activation rows (K = 256 nb bytes each)
-    const float *act_da;  // [rows][nb]
-    const int *act_bs;
-    int by_token;         // activation row of pair p: pair_token[p] (1) or p (0)
-    float *Y;             // [P][N]
+    int64_t mb;  // bytes of one expert matrix
+    int N, nb;   // rows and 256-blocks per row of one expert matrix
+    float *Y;    // [P][N]
 };
 
 __device__ __forceinline__ uint32_t nib(uint32_t w, int hi) {
@@ -198,9 +203,102 @@ __device__ __forceinline__ void mma_s8(int (&d)[4], uint32_t a0, uint32_t a1, ui
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-__global__ void __launch_bounds__((GG_CW + 1) * 32, 1) grouped_gemm_kernel(GroupedArgs a, GemmJob j0, GemmJob j1,
-                                                                           int njobs) {
-    extern __shared__ __align__(128) uint8_t smem[];
+__device__ __forceinline__ void ldmatrix_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int c0, int c1, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// One stage (GG_KB blocks) of a consumer warp for NT token tiles of 8.
+template <int NT>
+__device__ __forceinline__ void gg_stage(const uint8_t *st, uint32_t stt, const float *sda, const int *sbs, int cofs,
+                                         int rgl, bool vr, int lane, float (&y)[2][8][4]) {
+    const int tig = lane & 3;
+#pragma unroll 1
+    for (int bl = 0; bl < GG_KB; ++bl) {
+                    // this thread's code words of the 4 rows of its row group in this block
+                    const uint8_t *blk = st + rgl * GG_WROW + bl * BLOCK_BYTES;
+                    uint32_t W[4][8];
+#pragma unroll
+                    for (int r = 0; r < 4; ++r)
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            W[r][j] = *reinterpret_cast<const uint32_t *>(blk + CODE_OFS + ROW_BYTES * r + 4 * tig +
+                                                                           16 * j);
+                    int acc[2][8][4];
+#pragma unroll
+                    for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+                        for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) acc[mt][nt][q] = 0;
+#pragma unroll
+                    for (int s = 0; s < 8; ++s) {
+                        const int q = s & 3, hh = s >> 2;
+                        const int E0 = bl * QK + 32 * s;  // first element of this k-step in the stage
+                        const int L = E0 >> 7, c0 = (E0 & 127) >> 4;
+                        uint32_t bf[8][2];
+#pragma unroll
+                        for (int np = 0; np < 4; ++np) {
+                            if (2 * np < NT) {
+                                const int mi = lane >> 3;  // matrix supplied by this lane's address
+                                const int t = (2 * np + (mi >> 1)) * 8 + (lane & 7);
+                                const int c = c0 + (mi & 1);
+                                const uint32_t addr = stt + L * GG_LINE_BYTES + t * 128 + ((c ^ (t & 7)) << 4);
+                                ldmatrix_x4(addr, bf[2 * np][0], bf[2 * np][1], bf[2 * np + 1][0],
+                                            bf[2 * np + 1][1]);
+                            }
+                        }
+#pragma unroll
+                        for (int mt = 0; mt < 2; ++mt) {
+                            const uint32_t a0 = nib(W[2 * mt][2 * q], hh), a2 = nib(W[2 * mt][2 * q + 1], hh);
+                            const uint32_t a1 = nib(W[2 * mt + 1][2 * q], hh), a3 = nib(W[2 * mt + 1][2 * q + 1], hh);
+#pragma unroll
+                            for (int nt = 0; nt < 8; ++nt)
+                                if (nt < NT) mma_s8(acc[mt][nt], a0, a1, a2, a3, bf[nt][0], bf[nt][1]);
+                        }
+                    }
+                    // fixed float schedule for this block
+                    float dw[4];
+#pragma unroll
+                    for (int r = 0; r < 4; ++r) dw[r] = vr ? block_scale(blk, r) : 0.0f;
+#pragma unroll
+                    for (int nt = 0; nt < 8; ++nt) {
+                        if (nt < NT) {
+                            const int t0 = nt * 8 + 2 * tig, t1 = t0 + 1;
+                            const float da0 = sda[t0 * 4 + cofs + bl], da1 = sda[t1 * 4 + cofs + bl];
+                            const int bs0 = sbs[t0 * 4 + cofs + bl], bs1 = sbs[t1 * 4 + cofs + bl];
+#pragma unroll
+                            for (int mt = 0; mt < 2; ++mt) {
+                                const float dlo = dw[2 * mt], dhi = dw[2 * mt + 1];
+                                y[mt][nt][0] = __fadd_rn(y[mt][nt][0], __fmul_rn(static_cast<float>(acc[mt][nt][0] - 4 * bs0),
+                                                                                 __fmul_rn(dlo, da0)));
+                                y[mt][nt][1] = __fadd_rn(y[mt][nt][1], __fmul_rn(static_cast<float>(acc[mt][nt][1] - 4 * bs1),
+                                                                                 __fmul_rn(dlo, da1)));
+                                y[mt][nt][2] = __fadd_rn(y[mt][nt][2], __fmul_rn(static_cast<float>(acc[mt][nt][2] - 4 * bs0),
+                                                                                 __fmul_rn(dhi, da0)));
+                                y[mt][nt][3] = __fadd_rn(y[mt][nt][3], __fmul_rn(static_cast<float>(acc[mt][nt][3] - 4 * bs1),
+                                                                                 __fmul_rn(dhi, da1)));
+                            }
+                        }
+                    }
+                }
+}
+
+__global__ void __launch_bounds__((GG_CW + 1) * 32, 1)
+    grouped_gemm_kernel(GroupedArgs a, GemmJob j0, GemmJob j1, int njobs, const __grid_constant__ CUtensorMap w0,
+                        const __grid_constant__ CUtensorMap w1, const __grid_constant__ CUtensorMap xmap,
+                        const __grid_constant__ CUtensorMap damap, const __grid_constant__ CUtensorMap bsmap) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + GG_STAGES * GG_STAGE_BYTES);
     uint64_t *empty = full + GG_STAGES;
@@ -216,151 +314,146 @@ __global__ void __launch_bounds__((GG_CW + 1) * 32, 1) grouped_gemm_kernel(Group
     int64_t it = 0;  // stage counter, identical in every warp
     const int64_t tiles0 = (j0.N / 4 + GG_RG - 1) / GG_RG;
     const int64_t tiles1 = njobs > 1 ? (j1.N / 4 + GG_RG - 1) / GG_RG : 0;
-    const int64_t items = static_cast<int64_t>(n_chunks) * (tiles0 + tiles1);
+    const int64_t per_chunk = tiles0 + tiles1;
+    const int64_t items = static_cast<int64_t>(n_chunks) * per_chunk;
+    // the chunk descriptor of the next item is loaded one item ahead
+    auto chunk_of = [&](int64_t w) { return static_cast<int>(w / per_chunk); };
+    int ce = 0, cb = 0, cl = 0;
+    if (blockIdx.x < items) {
+        const int c = chunk_of(blockIdx.x);
+        ce = __ldcg(a.chunk_expert + c);
+        cb = __ldcg(a.chunk_begin + c);
+        cl = __ldcg(a.chunk_len + c);
+    }
     for (int64_t w = blockIdx.x; w < items; w += gridDim.x) {
-        const int64_t per_chunk = tiles0 + tiles1;
-        const int chunk = static_cast<int>(w / per_chunk);
+        const int chunk = chunk_of(w);
         int64_t tl = w - chunk * per_chunk;
         const bool second = tl >= tiles0;
         if (second) tl -= tiles0;
         const GemmJob &J = second ? j1 : j0;
-        const int e = __ldcg(a.chunk_expert + chunk);
-        const int pb = __ldcg(a.chunk_begin + chunk);
-        const int m = __ldcg(a.chunk_len + chunk);
+        const CUtensorMap *wmap = second ? &w1 : &w0;
+        const int e = ce, pb = cb, m = cl;
+        if (w + gridDim.x < items) {
+            const int c = chunk_of(w + gridDim.x);
+            ce = __ldcg(a.chunk_expert + c);
+            cb = __ldcg(a.chunk_begin + c);
+            cl = __ldcg(a.chunk_len + c);
+        }
         const int n_rg = J.N / 4;
         const int rg0 = static_cast<int>(tl) * GG_RG;
-        const int rgs = min(GG_RG, n_rg - rg0);
-        const uint8_t *mat = J.mat0 + static_cast<int64_t>(e) * J.mb;
-        const int64_t stripe = static_cast<int64_t>(J.nb) * BLOCK_BYTES;
-        const int K = J.nb * QK;
         const int n_st = J.nb / GG_KB;
         if (warp == GG_CW) {
             // ---- producer ----
             for (int kc = 0; kc < n_st; ++kc, ++it) {
                 const int slot = static_cast<int>(it % GG_STAGES);
                 const uint32_t par = static_cast<uint32_t>(((it / GG_STAGES) & 1) ^ 1);
+#ifdef TQ_INSTRUMENT
+                const long long tw0 = clock64();
+#endif
                 if (!__all_sync(0xffffffffu, mbar_wait(&empty[slot], par))) {
                     if (lane == 0) report(a.status, TQFX4_ETIMEOUT, K_GGATEUP, static_cast<int>(w));
                     return;
                 }
+                TQ_ADD(3, 0, clock64() - tw0);
                 uint8_t *st = smem + slot * GG_STAGE_BYTES;
-                float *sda = reinterpret_cast<float *>(st + GG_W_BYTES + GG_T_BYTES);
-                int *sbs = reinterpret_cast<int *>(sda + GG_TOK * GG_KB);
-                for (int i = lane; i < m * GG_KB; i += 32) {
-                    const int ti = i / GG_KB, bl = i - ti * GG_KB;
-                    const int p = pb + ti;
-                    const int64_t r = J.by_token ? __ldcg(a.pair_token + p) : p;
-                    sda[ti * GG_KB + bl] = __ldcg(J.act_da + r * J.nb + kc * GG_KB + bl);
-                    sbs[ti * GG_KB + bl] = __ldcg(J.act_bs + r * J.nb + kc * GG_KB + bl);
-                }
-                __syncwarp();
+#ifdef TQ_INSTRUMENT
+                const long long ti0 = clock64();
+#endif
                 if (lane == 0) {
-                    mbar_arrive_expect_tx(&full[slot],
-                                          static_cast<uint32_t>(rgs * GG_WROW + m * GG_KB * QK));
-                    for (int r = 0; r < rgs; ++r)
-                        bulk_g2s(st + r * GG_WROW, mat + (rg0 + r) * stripe + kc * GG_WROW, GG_WROW, &full[slot]);
-                    for (int ti = 0; ti < m; ++ti) {
-                        const int p = pb + ti;
-                        const int64_t row = J.by_token ? __ldcg(a.pair_token + p) : p;
-                        bulk_g2s(st + GG_W_BYTES + ti * GG_TSTRIDE, J.act + row * K + kc * GG_KB * QK, GG_KB * QK,
-                                 &full[slot]);
-                    }
+                    mbar_arrive_expect_tx(&full[slot], static_cast<uint32_t>(GG_RG * GG_WROW + GG_T_BYTES + GG_S_BYTES));
+                    // weights: rows e * n_rg + rg0 .. + 31 of the stacked matrix, bytes kc * 1040 ..
+                    tma_load_2d(st, wmap, kc * (GG_WROW / 8), e * n_rg + rg0, &full[slot]);
+                    // activations: four 128-byte lines of 64 pair rows starting at pb
+                    for (int L = 0; L < 4; ++L)
+                        tma_load_2d(st + GG_W_BYTES + L * GG_LINE_BYTES, &xmap, (kc * GG_KB * QK + L * 128) / 8, pb,
+                                    &full[slot]);
+                    // scales and block sums of blocks 4 (kc / 2) .. + 3 of the 64 pairs
+                    tma_load_2d(st + GG_W_BYTES + GG_T_BYTES, &damap, 4 * (kc >> 1), pb, &full[slot]);
+                    tma_load_2d(st + GG_W_BYTES + GG_T_BYTES + 1024, &bsmap, 4 * (kc >> 1), pb, &full[slot]);
                 }
+                TQ_ADD(3, 1, clock64() - ti0);
+                TQ_ADD(3, 2, 1);
                 __syncwarp();
             }
         } else {
-            // ---- consumers: warp owns rows 16 warp .. 16 warp + 15 of the tile ----
+            // ---- consumers: warp owns row groups rg0 + 8 warp + (lane >> 2) ----
             const int g = lane >> 2, tig = lane & 3;
-            const int row_a = warp * 16 + g, row_b = row_a + 8;  // rows within the tile
-            const int rga = row_a >> 2, rgb = row_b >> 2, r4 = g & 3;
-            const bool va = rga < rgs, vb = rgb < rgs;
+            const int rgl = warp * 8 + g;  // row group within the tile
+            const bool vr = rg0 + rgl < n_rg;
             const int ntiles = (m + 7) >> 3;
-            float y[8][4];
+            float y[2][8][4];
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt)
+            for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
-                for (int q = 0; q < 4; ++q) y[nt][q] = 0.0f;
+                for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) y[mt][nt][q] = 0.0f;
             for (int kc = 0; kc < n_st; ++kc, ++it) {
                 const int slot = static_cast<int>(it % GG_STAGES);
                 const uint32_t par = static_cast<uint32_t>((it / GG_STAGES) & 1);
+#ifdef TQ_INSTRUMENT
+                const long long tf0 = clock64();
+#endif
                 if (!__all_sync(0xffffffffu, mbar_wait(&full[slot], par))) {
                     if (lane == 0) report(a.status, TQFX4_ETIMEOUT, K_GGATEUP, static_cast<int>(w));
                     return;
                 }
+#ifdef TQ_INSTRUMENT
+                const long long tc0 = clock64();
+                if (warp == 0) TQ_ADD(3, 3, tc0 - tf0);
+#endif
                 const uint8_t *st = smem + slot * GG_STAGE_BYTES;
-                const uint8_t *stt = st + GG_W_BYTES;
+                const uint32_t stt = smem_u32(st + GG_W_BYTES);
                 const float *sda = reinterpret_cast<const float *>(st + GG_W_BYTES + GG_T_BYTES);
-                const int *sbs = reinterpret_cast<const int *>(sda + GG_TOK * GG_KB);
-#pragma unroll 1
-                for (int bl = 0; bl < GG_KB; ++bl) {
-                    // this thread's 32 code bytes of rows a and b in this block
-                    uint32_t wa[8], wb[8];
-                    const uint8_t *ba = st + rga * GG_WROW + bl * BLOCK_BYTES + CODE_OFS + ROW_BYTES * r4;
-                    const uint8_t *bb = st + rgb * GG_WROW + bl * BLOCK_BYTES + CODE_OFS + ROW_BYTES * r4;
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const int o = (q < 2 ? 16 * tig + 8 * q : 64 + 16 * tig + 8 * (q - 2));
-                        uint2 v = va ? *reinterpret_cast<const uint2 *>(ba + o) : make_uint2(0u, 0u);
-                        wa[2 * q] = v.x;
-                        wa[2 * q + 1] = v.y;
-                        v = vb ? *reinterpret_cast<const uint2 *>(bb + o) : make_uint2(0u, 0u);
-                        wb[2 * q] = v.x;
-                        wb[2 * q + 1] = v.y;
-                    }
-                    int acc[8][4];
-#pragma unroll
-                    for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) acc[nt][q] = 0;
-#pragma unroll
-                    for (int s = 0; s < 8; ++s) {
-                        const int q = s & 3, hh = s >> 2;
-                        const int koff = (q < 2 ? 16 * tig + 8 * q : 64 + 16 * tig + 8 * (q - 2)) + 128 * hh;
-                        const uint32_t a0 = nib(wa[2 * q], hh), a2 = nib(wa[2 * q + 1], hh);
-                        const uint32_t a1 = nib(wb[2 * q], hh), a3 = nib(wb[2 * q + 1], hh);
-#pragma unroll
-                        for (int nt = 0; nt < 8; ++nt) {
-                            if (nt < ntiles) {
-                                const uint2 bw = *reinterpret_cast<const uint2 *>(
-                                    stt + (nt * 8 + g) * GG_TSTRIDE + bl * QK + koff);
-                                mma_s8(acc[nt], a0, a1, a2, a3, bw.x, bw.y);
-                            }
-                        }
-                    }
-                    // fixed float schedule for this block
-                    const float dwa = va ? block_scale(st + rga * GG_WROW + bl * BLOCK_BYTES, r4) : 0.0f;
-                    const float dwb = vb ? block_scale(st + rgb * GG_WROW + bl * BLOCK_BYTES, r4) : 0.0f;
-#pragma unroll
-                    for (int nt = 0; nt < 8; ++nt) {
-                        if (nt < ntiles) {
-                            const int t0 = nt * 8 + 2 * tig, t1 = t0 + 1;
-                            const float da0 = sda[t0 * GG_KB + bl], da1 = sda[t1 * GG_KB + bl];
-                            const int bs0 = sbs[t0 * GG_KB + bl], bs1 = sbs[t1 * GG_KB + bl];
-                            y[nt][0] = __fadd_rn(y[nt][0], __fmul_rn(static_cast<float>(acc[nt][0] - 4 * bs0),
-                                                                     __fmul_rn(dwa, da0)));
-                            y[nt][1] = __fadd_rn(y[nt][1], __fmul_rn(static_cast<float>(acc[nt][1] - 4 * bs1),
-                                                                     __fmul_rn(dwa, da1)));
-                            y[nt][2] = __fadd_rn(y[nt][2], __fmul_rn(static_cast<float>(acc[nt][2] - 4 * bs0),
-                                                                     __fmul_rn(dwb, da0)));
-                            y[nt][3] = __fadd_rn(y[nt][3], __fmul_rn(static_cast<float>(acc[nt][3] - 4 * bs1),
-                                                                     __fmul_rn(dwb, da1)));
-                        }
-                    }
+                const int *sbs = reinterpret_cast<const int *>(st + GG_W_BYTES + GG_T_BYTES + 1024);
+                const int cofs = (kc & 1) * GG_KB;  // this stage's blocks inside the 4-block scale box
+                switch (ntiles) {
+                    case 1: gg_stage<1>(st, stt, sda, sbs, cofs, rgl, vr, lane, y); break;
+                    case 2: gg_stage<2>(st, stt, sda, sbs, cofs, rgl, vr, lane, y); break;
+                    case 3: gg_stage<3>(st, stt, sda, sbs, cofs, rgl, vr, lane, y); break;
+                    case 4: gg_stage<4>(st, stt, sda, sbs, cofs, rgl, vr, lane, y); break;
+                    case 5: gg_stage<5>(st, stt, sda, sbs, cofs, rgl, vr, lane, y); break;
+                    case 6: gg_stage<6>(st, stt, sda, sbs, cofs, rgl, vr, lane, y); break;
+                    case 7: gg_stage<7>(st, stt, sda, sbs, cofs, rgl, vr, lane, y); break;
+                    default: gg_stage<8>(st, stt, sda, sbs, cofs, rgl, vr, lane, y); break;
                 }
                 __syncwarp();
+#ifdef TQ_INSTRUMENT
+                if (warp == 0) TQ_ADD(3, 4, clock64() - tc0);
+#endif
                 if (lane == 0) mbar_arrive(&empty[slot]);
             }
-            // write the outputs of valid rows and pairs
-            const int gra = rg0 * 4 + row_a, grb = rg0 * 4 + row_b;
+            if (vr) {
+                const int64_t row0 = static_cast<int64_t>(rg0 + rgl) * 4;
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                const int t0 = nt * 8 + 2 * tig, t1 = t0 + 1;
-                if (va && t0 < m) J.Y[static_cast<int64_t>(pb + t0) * J.N + gra] = y[nt][0];
-                if (va && t1 < m) J.Y[static_cast<int64_t>(pb + t1) * J.N + gra] = y[nt][1];
-                if (vb && t0 < m) J.Y[static_cast<int64_t>(pb + t0) * J.N + grb] = y[nt][2];
-                if (vb && t1 < m) J.Y[static_cast<int64_t>(pb + t1) * J.N + grb] = y[nt][3];
+                for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+                    for (int nt = 0; nt < 8; ++nt) {
+                        const int t0 = nt * 8 + 2 * tig, t1 = t0 + 1;
+                        if (t0 < m) {
+                            J.Y[static_cast<int64_t>(pb + t0) * J.N + row0 + 2 * mt] = y[mt][nt][0];
+                            J.Y[static_cast<int64_t>(pb + t0) * J.N + row0 + 2 * mt + 1] = y[mt][nt][2];
+                        }
+                        if (t1 < m) {
+                            J.Y[static_cast<int64_t>(pb + t1) * J.N + row0 + 2 * mt] = y[mt][nt][1];
+                            J.Y[static_cast<int64_t>(pb + t1) * J.N + row0 + 2 * mt + 1] = y[mt][nt][3];
+                        }
+                    }
             }
         }
+    }
+}
+
+// Gather the quantized hidden state of each pair's token into pair order.
+__global__ void __launch_bounds__(256) gather_rows_kernel(GroupedArgs a) {
+    const int64_t pos = blockIdx.x;
+    const int64_t t = __ldcg(a.pair_token + pos);
+    const uint4 *src = reinterpret_cast<const uint4 *>(a.qx + t * a.H);
+    uint4 *dst = reinterpret_cast<uint4 *>(a.xg + pos * a.H);
+    for (int i = threadIdx.x; i < a.H / 16; i += blockDim.x) dst[i] = __ldcg(src + i);
+    for (int b = threadIdx.x; b < a.nbhp; b += blockDim.x) {
+        a.dxg[pos * a.nbhp + b] = b < a.nbh ? __ldcg(a.dx + t * a.nbh + b) : 0.0f;
+        a.bxg[pos * a.nbhp + b] = b < a.nbh ? __ldcg(a.bx + t * a.nbh + b) : 0;
     }
 }
 
@@ -394,6 +487,13 @@ __global__ void __launch_bounds__(256) swiglu_quant_kernel(GroupedArgs a) {
     if (lane == 0) {
         a.dh[unit] = d;
         a.bh[unit] = sum;
+        a.dhp[p * a.nbip + b] = d;
+        a.bhp[p * a.nbip + b] = sum;
+        if (b == a.nbi - 1)
+            for (int i = a.nbi; i < a.nbip; ++i) {
+                a.dhp[p * a.nbip + i] = 0.0f;
+                a.bhp[p * a.nbip + i] = 0;
+            }
         if (!ok) report(a.status, TQFX4_EDATA, K_GDOWN, static_cast<int>(unit));
     }
 }
@@ -425,6 +525,70 @@ __global__ void __launch_bounds__(256) combine_kernel(GroupedArgs a) {
 
 // ---------------------------------------------------------------- host side
 
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+cudaError_t encoder() {
+    if (g_encode) return cudaSuccess;
+    cudaDriverEntryPointQueryResult q;
+    void *fn = nullptr;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess) return e;
+    if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    return cudaSuccess;
+}
+
+// The stacked matrices of one projection as a 2-D tensor of 8-byte elements:
+// one row per row group (E * n_rg rows, stride nb * 520 bytes), boxes of
+// GG_KB blocks (130 elements) x GG_RG row groups.
+cudaError_t weight_map(CUtensorMap *m, const void *base, int64_t E, int64_t n_rg, int nb) {
+    cudaError_t e = encoder();
+    if (e != cudaSuccess) return e;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(nb) * BLOCK_BYTES / 8, static_cast<cuuint64_t>(E * n_rg)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(nb) * BLOCK_BYTES};
+    const cuuint32_t box[2] = {GG_WROW / 8, GG_RG};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_UINT64, 2, const_cast<void *>(base), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+// Activation rows [rows][K] int8 as 8-byte elements; boxes of one 128-byte
+// line x GG_TOK rows, 128-byte swizzled.
+cudaError_t act_map(CUtensorMap *m, const void *base, int64_t rows, int64_t K) {
+    cudaError_t e = encoder();
+    if (e != cudaSuccess) return e;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(K / 8), static_cast<cuuint64_t>(rows)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
+    const cuuint32_t box[2] = {16, GG_TOK};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_UINT64, 2, const_cast<void *>(base), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+// Per-pair block scales (fp32) or block sums (int32) [rows][nbp] with nbp a
+// multiple of 4; boxes of 4 blocks x GG_TOK rows.
+cudaError_t scale_map(CUtensorMap *m, const void *base, int64_t rows, int nbp, bool is_float) {
+    cudaError_t e = encoder();
+    if (e != cudaSuccess) return e;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(nbp), static_cast<cuuint64_t>(rows)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(nbp) * 4};
+    const cuuint32_t box[2] = {4, GG_TOK};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode(m, is_float ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_INT32, 2,
+                          const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+}  // namespace
+
 bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, void *ws, GroupedArgs &a,
                   MoeLayout &L) {
     a = GroupedArgs{};
@@ -444,6 +608,8 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
     a.wr = rt->weight;
     a.bias = rt->bias;
     a.keep_h = 1;
+    a.nbhp = (a.nbh + 3) / 4 * 4;
+    a.nbip = (a.nbi + 3) / 4 * 4;
     L = moe_layout(a.E, a.H, a.I, a.top_k, T, true, true);
     uint8_t *base = static_cast<uint8_t *>(ws);
     if (base) {
@@ -455,6 +621,11 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
         a.qx = reinterpret_cast<int8_t *>(base + L.qx);
         a.dx = reinterpret_cast<float *>(base + L.dx);
         a.bx = reinterpret_cast<int *>(base + L.bx);
+        a.xg = reinterpret_cast<int8_t *>(base + L.xg);
+        a.dxg = reinterpret_cast<float *>(base + L.dxg);
+        a.bxg = reinterpret_cast<int *>(base + L.bxg);
+        a.dhp = reinterpret_cast<float *>(base + L.dhp);
+        a.bhp = reinterpret_cast<int *>(base + L.bhp);
         a.g = reinterpret_cast<float *>(base + L.g);
         a.u = reinterpret_cast<float *>(base + L.u);
         a.h = reinterpret_cast<float *>(base + L.h);
@@ -478,7 +649,8 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
 int grouped_stage_count() { return 8; }
 
 const char *grouped_stage_name(int s) {
-    static const char *names[] = {"router", "topk", "group", "quant_x", "gate_up", "swiglu", "down", "combine"};
+    static const char *names[] = {"router", "topk", "group", "quant_gather", "gate_up", "swiglu", "down",
+                                  "combine"};
     return (s >= 0 && s < 8) ? names[s] : "";
 }
 
@@ -512,18 +684,30 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(3);
     if ((e = launch_quantize(a.X, a.T, a.H, a.qx, a.dx, a.bx, a.status, st)) != cudaSuccess) return e;
+    gather_rows_kernel<<<a.P, 256, 0, st>>>(a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(4);
-    GemmJob jg{a.gate, a.mb_gu, a.I, a.nbh, a.qx, a.dx, a.bx, 1, a.g};
-    GemmJob ju{a.up, a.mb_gu, a.I, a.nbh, a.qx, a.dx, a.bx, 1, a.u};
-    grouped_gemm_kernel<<<sms, (GG_CW + 1) * 32, GG_SMEM, st>>>(a, jg, ju, 2);
+    CUtensorMap mg, mu, md, mx, mh, sdx, sbx, sdh, sbh;
+    if ((e = scale_map(&sdx, a.dxg, a.P, a.nbhp, true)) != cudaSuccess) return e;
+    if ((e = scale_map(&sbx, a.bxg, a.P, a.nbhp, false)) != cudaSuccess) return e;
+    if ((e = scale_map(&sdh, a.dhp, a.P, a.nbip, true)) != cudaSuccess) return e;
+    if ((e = scale_map(&sbh, a.bhp, a.P, a.nbip, false)) != cudaSuccess) return e;
+    if ((e = weight_map(&mg, a.gate, a.E, a.I / 4, a.nbh)) != cudaSuccess) return e;
+    if ((e = weight_map(&mu, a.up, a.E, a.I / 4, a.nbh)) != cudaSuccess) return e;
+    if ((e = weight_map(&md, a.down, a.E, a.H / 4, a.nbi)) != cudaSuccess) return e;
+    if ((e = act_map(&mx, a.xg, a.P, a.H)) != cudaSuccess) return e;
+    if ((e = act_map(&mh, a.qh, a.P, a.I)) != cudaSuccess) return e;
+    GemmJob jg{a.mb_gu, a.I, a.nbh, a.g};
+    GemmJob ju{a.mb_gu, a.I, a.nbh, a.u};
+    grouped_gemm_kernel<<<sms, (GG_CW + 1) * 32, GG_SMEM, st>>>(a, jg, ju, 2, mg, mu, mx, sdx, sbx);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(5);
     const int64_t units = static_cast<int64_t>(a.P) * a.nbi;
     swiglu_quant_kernel<<<static_cast<unsigned>((units * 32 + 255) / 256), 256, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(6);
-    GemmJob jd{a.down, a.mb_d, a.H, a.nbi, a.qh, a.dh, a.bh, 0, a.o};
-    grouped_gemm_kernel<<<sms, (GG_CW + 1) * 32, GG_SMEM, st>>>(a, jd, jd, 1);
+    GemmJob jd{a.mb_d, a.H, a.nbi, a.o};
+    grouped_gemm_kernel<<<sms, (GG_CW + 1) * 32, GG_SMEM, st>>>(a, jd, jd, 1, md, md, mh, sdh, sbh);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(7);
     combine_kernel<<<a.T, 256, 0, st>>>(a);

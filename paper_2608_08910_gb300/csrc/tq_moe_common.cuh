@@ -20,6 +20,8 @@ struct MoeLayout {
     size_t qh, dh, bh;
     size_t o;        // fp32 [P][H]
     size_t counts, offsets, pair_token, pair_slot, pair_of;
+    size_t xg;  // int8 [P][H] (grouped only)
+    size_t dxg, bxg, dhp, bhp;  // [P][round4(nb)] (grouped only)
     size_t chunk_expert, chunk_begin, chunk_len, n_chunks;  // grouped GEMM work list
     int64_t max_chunks;
     size_t total;
@@ -67,13 +69,20 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.pair_token = take(4 * static_cast<size_t>(P));
         L.pair_slot = take(4 * static_cast<size_t>(P));
         L.pair_of = take(4 * static_cast<size_t>(P));
+        L.xg = take(static_cast<size_t>(P * H));
+        const int64_t nbhp = (nbh + 3) / 4 * 4, nbip = (nbi + 3) / 4 * 4;
+        L.dxg = take(4 * static_cast<size_t>(P * nbhp));
+        L.bxg = take(4 * static_cast<size_t>(P * nbhp));
+        L.dhp = take(4 * static_cast<size_t>(P * nbip));
+        L.bhp = take(4 * static_cast<size_t>(P * nbip));
         L.max_chunks = P / GG_TOK + E + 1;
         L.chunk_expert = take(4 * static_cast<size_t>(L.max_chunks));
         L.chunk_begin = take(4 * static_cast<size_t>(L.max_chunks));
         L.chunk_len = take(4 * static_cast<size_t>(L.max_chunks));
         L.n_chunks = take(4);
     } else {
-        L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = SIZE_MAX;
+        L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = L.xg = SIZE_MAX;
+        L.dxg = L.bxg = L.dhp = L.bhp = SIZE_MAX;
         L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
         L.max_chunks = 0;
     }
@@ -129,6 +138,10 @@ struct GroupedArgs {
     int8_t *qx;
     float *dx;
     int *bx;
+    int8_t *xg;  // [P][H] quantized hidden state of each pair, in pair order
+    float *dxg, *dhp;  // [P][nbp] scales in pair order, rows padded to a multiple of 4 blocks
+    int *bxg, *bhp;
+    int nbhp, nbip;
     float *g, *u, *h;
     int8_t *qh;
     float *dh;
