@@ -228,6 +228,8 @@ static tqfx4_status moe_grouped_impl(const tqfx4_experts *ex, const tqfx4_router
     tq::grouped_args(ex, rt, T, nullptr, a, L);
     if ((s = check_ws(ws, ws_bytes, L.total, fn))) return s;
     tq::grouped_args(ex, rt, T, ws, a, L);
+    // The tensor-core contraction pays off once the chunks are mostly full.
+    a.tc = path == TQFX4_PATH_PREFILL || (path == TQFX4_PATH_AUTO && T * rt->top_k >= tq::kTcMinPairs);
     cudaError_t e = tq::launch_moe_grouped(a, X, OUT, sel_idx, sel_w, static_cast<cudaStream_t>(stream), events);
     if (e != cudaSuccess) return cuda_fail(e, fn);
     return ok();

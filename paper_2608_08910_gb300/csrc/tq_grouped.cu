@@ -24,6 +24,7 @@
 // copies (one box of weight blocks, four swizzled boxes of pair-ordered
 // activations); four consumer warps each own 8 row groups (32 rows).
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
 #include "tq_launch.h"
@@ -444,13 +445,34 @@ __global__ void __launch_bounds__((GG_CW + 1) * 32, 1)
     }
 }
 
+// Eight int8 values as eight bf16 values (exact: |q| <= 127 needs 7 bits).
+__device__ __forceinline__ uint4 i8x8_to_bf16x8(uint2 v) {
+    const int8_t *b = reinterpret_cast<const int8_t *>(&v);
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const __nv_bfloat162 h = __floats2bfloat162_rn(static_cast<float>(b[2 * i]), static_cast<float>(b[2 * i + 1]));
+        w[i] = *reinterpret_cast<const uint32_t *>(&h);
+    }
+    return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 // Gather the quantized hidden state of each pair's token into pair order.
 __global__ void __launch_bounds__(256) gather_rows_kernel(GroupedArgs a) {
     const int64_t pos = blockIdx.x;
     const int64_t t = __ldcg(a.pair_token + pos);
     const uint4 *src = reinterpret_cast<const uint4 *>(a.qx + t * a.H);
-    uint4 *dst = reinterpret_cast<uint4 *>(a.xg + pos * a.H);
-    for (int i = threadIdx.x; i < a.H / 16; i += blockDim.x) dst[i] = __ldcg(src + i);
+    if (a.tc) {
+        // bf16 copy for the tensor-core contraction (int8 values are exact in bf16)
+        uint4 *dst = reinterpret_cast<uint4 *>(a.xgb + pos * a.H);
+        for (int i = threadIdx.x; i < a.H / 8; i += blockDim.x) {
+            const uint2 v = __ldcg(reinterpret_cast<const uint2 *>(a.qx + t * a.H) + i);
+            dst[i] = i8x8_to_bf16x8(v);
+        }
+    } else {
+        uint4 *dst = reinterpret_cast<uint4 *>(a.xg + pos * a.H);
+        for (int i = threadIdx.x; i < a.H / 16; i += blockDim.x) dst[i] = __ldcg(src + i);
+    }
     for (int b = threadIdx.x; b < a.nbhp; b += blockDim.x) {
         a.dxg[pos * a.nbhp + b] = b < a.nbh ? __ldcg(a.dx + t * a.nbh + b) : 0.0f;
         a.bxg[pos * a.nbhp + b] = b < a.nbh ? __ldcg(a.bx + t * a.nbh + b) : 0;
@@ -480,6 +502,7 @@ __global__ void __launch_bounds__(256) swiglu_quant_kernel(GroupedArgs a) {
     int sum;
     const bool ok = quant_block_warp(hv, packed, d, sum);
     *reinterpret_cast<uint2 *>(a.qh + o) = packed;
+    if (a.tc) *reinterpret_cast<uint4 *>(a.qhb + o) = i8x8_to_bf16x8(packed);
     if (a.keep_h) {
         reinterpret_cast<float4 *>(a.h + o)[0] = make_float4(hv[0], hv[1], hv[2], hv[3]);
         reinterpret_cast<float4 *>(a.h + o)[1] = make_float4(hv[4], hv[5], hv[6], hv[7]);
@@ -642,6 +665,8 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
         a.chunk_begin = reinterpret_cast<int *>(base + L.chunk_begin);
         a.chunk_len = reinterpret_cast<int *>(base + L.chunk_len);
         a.n_chunks = reinterpret_cast<int *>(base + L.n_chunks);
+        a.xgb = reinterpret_cast<uint16_t *>(base + L.xgb);
+        a.qhb = reinterpret_cast<uint16_t *>(base + L.qhb);
     }
     return true;
 }
@@ -687,28 +712,37 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
     gather_rows_kernel<<<a.P, 256, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(4);
-    CUtensorMap mg, mu, md, mx, mh, sdx, sbx, sdh, sbh;
-    if ((e = scale_map(&sdx, a.dxg, a.P, a.nbhp, true)) != cudaSuccess) return e;
-    if ((e = scale_map(&sbx, a.bxg, a.P, a.nbhp, false)) != cudaSuccess) return e;
-    if ((e = scale_map(&sdh, a.dhp, a.P, a.nbip, true)) != cudaSuccess) return e;
-    if ((e = scale_map(&sbh, a.bhp, a.P, a.nbip, false)) != cudaSuccess) return e;
-    if ((e = weight_map(&mg, a.gate, a.E, a.I / 4, a.nbh)) != cudaSuccess) return e;
-    if ((e = weight_map(&mu, a.up, a.E, a.I / 4, a.nbh)) != cudaSuccess) return e;
-    if ((e = weight_map(&md, a.down, a.E, a.H / 4, a.nbi)) != cudaSuccess) return e;
-    if ((e = act_map(&mx, a.xg, a.P, a.H)) != cudaSuccess) return e;
-    if ((e = act_map(&mh, a.qh, a.P, a.I)) != cudaSuccess) return e;
-    GemmJob jg{a.mb_gu, a.I, a.nbh, a.g};
-    GemmJob ju{a.mb_gu, a.I, a.nbh, a.u};
-    grouped_gemm_kernel<<<sms, (GG_CW + 1) * 32, GG_SMEM, st>>>(a, jg, ju, 2, mg, mu, mx, sdx, sbx);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    rec(5);
     const int64_t units = static_cast<int64_t>(a.P) * a.nbi;
-    swiglu_quant_kernel<<<static_cast<unsigned>((units * 32 + 255) / 256), 256, 0, st>>>(a);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    rec(6);
-    GemmJob jd{a.mb_d, a.H, a.nbi, a.o};
-    grouped_gemm_kernel<<<sms, (GG_CW + 1) * 32, GG_SMEM, st>>>(a, jd, jd, 1, md, md, mh, sdh, sbh);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (a.tc) {
+        if ((e = launch_tc_gemm(a, false, st)) != cudaSuccess) return e;
+        rec(5);
+        swiglu_quant_kernel<<<static_cast<unsigned>((units * 32 + 255) / 256), 256, 0, st>>>(a);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        rec(6);
+        if ((e = launch_tc_gemm(a, true, st)) != cudaSuccess) return e;
+    } else {
+        CUtensorMap mg, mu, md, mx, mh, sdx, sbx, sdh, sbh;
+        if ((e = scale_map(&sdx, a.dxg, a.P, a.nbhp, true)) != cudaSuccess) return e;
+        if ((e = scale_map(&sbx, a.bxg, a.P, a.nbhp, false)) != cudaSuccess) return e;
+        if ((e = scale_map(&sdh, a.dhp, a.P, a.nbip, true)) != cudaSuccess) return e;
+        if ((e = scale_map(&sbh, a.bhp, a.P, a.nbip, false)) != cudaSuccess) return e;
+        if ((e = weight_map(&mg, a.gate, a.E, a.I / 4, a.nbh)) != cudaSuccess) return e;
+        if ((e = weight_map(&mu, a.up, a.E, a.I / 4, a.nbh)) != cudaSuccess) return e;
+        if ((e = weight_map(&md, a.down, a.E, a.H / 4, a.nbi)) != cudaSuccess) return e;
+        if ((e = act_map(&mx, a.xg, a.P, a.H)) != cudaSuccess) return e;
+        if ((e = act_map(&mh, a.qh, a.P, a.I)) != cudaSuccess) return e;
+        GemmJob jg{a.mb_gu, a.I, a.nbh, a.g};
+        GemmJob ju{a.mb_gu, a.I, a.nbh, a.u};
+        grouped_gemm_kernel<<<sms, (GG_CW + 1) * 32, GG_SMEM, st>>>(a, jg, ju, 2, mg, mu, mx, sdx, sbx);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        rec(5);
+        swiglu_quant_kernel<<<static_cast<unsigned>((units * 32 + 255) / 256), 256, 0, st>>>(a);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        rec(6);
+        GemmJob jd{a.mb_d, a.H, a.nbi, a.o};
+        grouped_gemm_kernel<<<sms, (GG_CW + 1) * 32, GG_SMEM, st>>>(a, jd, jd, 1, md, md, mh, sdh, sbh);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
     rec(7);
     combine_kernel<<<a.T, 256, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;

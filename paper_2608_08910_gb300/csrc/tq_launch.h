@@ -34,6 +34,7 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
                   MoeLayout &L);
 cudaError_t launch_moe_grouped(const GroupedArgs &a, const float *X, float *OUT, int32_t *sel_idx, float *sel_w,
                                cudaStream_t st, void *const *events);
+cudaError_t launch_tc_gemm(const GroupedArgs &a, bool down, cudaStream_t st);
 int grouped_stage_count();
 const char *grouped_stage_name(int s);
 int down_smem(const MoeArgs &a);

@@ -23,12 +23,15 @@ struct MoeLayout {
     size_t xg;  // int8 [P][H] (grouped only)
     size_t dxg, bxg, dhp, bhp;  // [P][round4(nb)] (grouped only)
     size_t chunk_expert, chunk_begin, chunk_len, n_chunks;  // grouped GEMM work list
+    size_t xgb, qhb;  // bf16 [P][H], [P][I] activation rows for the tensor-core contraction (grouped only)
     int64_t max_chunks;
     size_t total;
 };
 
 // Tokens (pairs) per chunk of the grouped GEMM.
 constexpr int GG_TOK = 64;
+// Pairs from which the automatic path choice takes the tensor-core contraction.
+constexpr int64_t kTcMinPairs = 4096;
 
 inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
@@ -80,10 +83,13 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.chunk_begin = take(4 * static_cast<size_t>(L.max_chunks));
         L.chunk_len = take(4 * static_cast<size_t>(L.max_chunks));
         L.n_chunks = take(4);
+        L.xgb = take(2 * static_cast<size_t>(P * H));
+        L.qhb = take(2 * static_cast<size_t>(P * I));
     } else {
         L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = L.xg = SIZE_MAX;
         L.dxg = L.bxg = L.dhp = L.bhp = SIZE_MAX;
         L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
+        L.xgb = L.qhb = SIZE_MAX;
         L.max_chunks = 0;
     }
     L.total = off;
@@ -150,6 +156,8 @@ struct GroupedArgs {
     int *counts, *offsets, *pair_token, *pair_slot, *pair_of;
     int *chunk_expert, *chunk_begin, *chunk_len, *n_chunks;
     int keep_h;
+    int tc;              // contraction on tcgen05 tensor cores (bf16 activation rows below)
+    uint16_t *xgb, *qhb;  // bf16 copies of xg [P][H] and qh [P][I]
 };
 
 // Shared-memory bytes of one quantized activation vector of nb blocks

@@ -1,0 +1,493 @@
+// Grouped expert GEMM on the 5th-generation tensor cores (tcgen05), the
+// contraction of the prefill path: one work item is 128 weight rows of one
+// expert times one chunk of <= 64 (token, slot) pairs of that expert.
+//
+// tcgen05.mma has no integer kind on sm_103a, so the integer block sums
+// S = sum_j c_j q_j (Eq. 5) are formed with kind::f16 on bf16 operands: the
+// codes c in -4..4 and the int8 activations q are exact in bf16, every
+// product is an exact integer, and the fp32 accumulator of one 256-element
+// block stays below 2^17 in magnitude, so it holds S exactly whatever the
+// order of the additions. The accumulator restarts at every block (the
+// block's first MMA does not accumulate) and the epilogue applies the fixed
+// float schedule y = y + float(S) * (d * da) block by block, the same
+// operations in the same order as the streaming kernels and the oracle.
+//
+// Warp roles (320 threads, one CTA per SM):
+//   warps 0-7  math: unpack the tile's nibbles into bf16 A tiles (K-major,
+//              128-byte swizzled canonical layout), and one block behind,
+//              read the block's accumulator from TMEM and update y. Warps w
+//              and w + 4 share TMEM lanes 32 (w % 4) .. + 31 (the rows of
+//              the tile) and split the 64 columns (the pairs) in halves;
+//   warp 8     producer: TMA copies of the raw weight blocks (one box per two
+//              blocks of 32 row groups), of the bf16 activation tiles (four
+//              64 x 64 boxes per block, 128-byte swizzled) and of the
+//              activation scales (4 blocks x 64 pairs);
+//   warp 9     TMEM allocation; one elected thread issues the MMAs
+//              (M = 128, N = 64, K = 16; 16 per block) and the commits.
+// Every wait is bounded. On a timeout the CTA records the error, all roles
+// leave their loops, the producer waits (bounded) for its copies in flight,
+// the MMA thread for its MMAs, and TMEM is freed before the CTA exits.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "tq_launch.h"
+#include "tq_moe_common.cuh"
+
+namespace tq {
+
+namespace {
+
+constexpr int TC_ROWS = 128;                   // weight rows per tile = TMEM lanes
+constexpr int TC_RG = TC_ROWS / 4;             // row groups per tile
+constexpr int TC_N = GG_TOK;                   // pairs per chunk = MMA N
+constexpr int TC_MATH_WARPS = 8;
+constexpr int TC_THREADS = (TC_MATH_WARPS + 2) * 32;
+constexpr int TC_RAW_ROW = 2 * BLOCK_BYTES;    // two blocks of one row group: 1040 bytes
+constexpr int TC_RAW_BYTES = 33 * 1024;        // 32 x 1040 bytes, padded
+constexpr int TC_A_BYTES = TC_ROWS * 128;      // one 64-element k-stage of A (bf16): 16 KB
+constexpr int TC_B_KS_BYTES = TC_N * 128;      // one k-stage of B: 8 KB
+constexpr int TC_B_BYTES = 4 * TC_B_KS_BYTES;  // one block of B: 32 KB
+constexpr int TC_DA_BYTES = 4 * TC_N * 4;      // scales of 64 pairs x 4 blocks: 1 KB
+constexpr int TC_OFF_RAW = 0;
+constexpr int TC_OFF_A = TC_OFF_RAW + 2 * TC_RAW_BYTES;
+constexpr int TC_OFF_B = TC_OFF_A + 4 * TC_A_BYTES;
+constexpr int TC_OFF_DA = TC_OFF_B + 2 * TC_B_BYTES;
+constexpr int TC_OFF_BAR = TC_OFF_DA + 2 * TC_DA_BYTES;
+constexpr int TC_NBAR = 25;  // barriers; the TMEM address and abort flag follow
+constexpr int TC_SMEM = TC_OFF_BAR + TC_NBAR * 8 + 16 + 1024;  // + alignment slack
+constexpr int TC_TMEM_COLS = 2 * TC_N;         // two accumulators (double buffer)
+
+static_assert(TC_OFF_A % 1024 == 0 && TC_OFF_B % 1024 == 0, "swizzled tiles need 1024-byte alignment");
+static_assert(TC_RG * TC_RAW_ROW <= TC_RAW_BYTES, "raw stage too small");
+
+// Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1),
+// A and B bf16 (bits 7-9 = 1, 10-12 = 1), both K-major (bits 15, 16 = 0),
+// N >> 3 at bits 17-22, M >> 4 at bits 24-28.
+constexpr uint32_t TC_IDESC = (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(TC_N >> 3) << 17) |
+                              (static_cast<uint32_t>(TC_ROWS >> 4) << 24);
+
+// Shared-memory matrix descriptor of a K-major operand in the 128-byte
+// swizzle canonical layout: rows of 128 bytes, 8-row atoms of 1024 bytes
+// (stride byte offset), start address advanced by 32 bytes per K = 16 step.
+__device__ __forceinline__ uint64_t umma_desc(uint32_t saddr) {
+    uint64_t d = static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);  // bits 0-13: start address >> 4
+    d |= static_cast<uint64_t>(1) << 16;                           // bits 16-29: leading byte offset (unused)
+    d |= static_cast<uint64_t>(1024 >> 4) << 32;                   // bits 32-45: stride byte offset >> 4
+    d |= static_cast<uint64_t>(1) << 46;                           // bits 46-47: descriptor version 1
+    d |= static_cast<uint64_t>(2) << 61;                           // bits 61-63: 128-byte swizzle
+    return d;
+}
+
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(TC_IDESC), "r"(accumulate)
+        : "memory");
+}
+
+// Arrives on `bar` once every tcgen05 operation issued so far by this thread
+// has completed.
+__device__ __forceinline__ void tc_commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// 32 TMEM lanes x 32 columns of 32 bits: the calling thread's lane, columns
+// taddr .. taddr + 31.
+__device__ __forceinline__ void tc_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,"
+        "%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int c0, int c1, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// Two nibble codes u0, u1 (bytes `sel` picks from x) as bf16x2 of c = u - 4:
+// the bytes [u0, 0x43, u1, 0x43] are the bf16 values 128 + u0 and 128 + u1,
+// and adding -132 (bf16 0xC304) to each half is exact.
+__device__ __forceinline__ uint32_t nib2bf16x2(uint32_t x, uint32_t sel) {
+    uint32_t w, r;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(w) : "r"(x), "r"(0x43u), "r"(sel));
+    asm("add.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(w), "r"(0xC304C304u));
+    return r;
+}
+
+struct TcJob {
+    int N, nb;   // rows and 256-blocks per row of one expert matrix
+    float *Y;    // [P][N] output in pair order
+};
+
+// Single-thread bounded wait (producer and MMA threads).
+__device__ __forceinline__ bool tc_wait(uint64_t *bar, uint32_t parity, int *abort, int *status, int where) {
+    if (*reinterpret_cast<volatile int *>(abort)) return false;
+    if (mbar_wait(bar, parity)) return true;
+    *reinterpret_cast<volatile int *>(abort) = 1;
+    report(status, TQFX4_ETIMEOUT, K_PREFILL, where);
+    return false;
+}
+
+// Warp-uniform bounded wait (math warps): all lanes observe the phase, and
+// all agree on the outcome so that the .sync.aligned TMEM loads that follow
+// are executed by the whole warp or by none of it.
+__device__ __forceinline__ bool tc_warp_wait(uint64_t *bar, uint32_t parity, int *abort, int *status, int where) {
+    const int lane = threadIdx.x & 31;
+    int ab = lane == 0 ? *reinterpret_cast<volatile int *>(abort) : 0;
+    ab = __shfl_sync(0xffffffffu, ab, 0);
+    if (ab) return false;
+    const bool ok = __all_sync(0xffffffffu, mbar_wait(bar, parity));
+    if (!ok && lane == 0) {
+        *reinterpret_cast<volatile int *>(abort) = 1;
+        report(status, TQFX4_ETIMEOUT, K_PREFILL, where);
+    }
+    return ok;
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    tc_gemm_kernel(GroupedArgs a, TcJob j0, TcJob j1, int njobs, const __grid_constant__ CUtensorMap wmap0,
+                   const __grid_constant__ CUtensorMap wmap1, const __grid_constant__ CUtensorMap bmap,
+                   const __grid_constant__ CUtensorMap damap) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + TC_OFF_BAR);
+    uint64_t *raw_full = bars, *raw_empty = bars + 2;
+    uint64_t *a_full = bars + 4, *a_empty = bars + 8;
+    uint64_t *b_full = bars + 12, *b_empty = bars + 14;
+    uint64_t *da_full = bars + 16, *da_empty = bars + 18;
+    uint64_t *d_full = bars + 20, *d_empty = bars + 22;
+    uint64_t *fin = bars + 24;  // MMA drain at exit
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + TC_NBAR);
+    int *abort = reinterpret_cast<int *>(tmem_slot + 1);
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&raw_full[i], 1);
+            mbar_init(&raw_empty[i], TC_MATH_WARPS);
+            mbar_init(&b_full[i], 1);
+            mbar_init(&b_empty[i], 1);
+            mbar_init(&da_full[i], 1);
+            mbar_init(&da_empty[i], TC_MATH_WARPS);
+            mbar_init(&d_full[i], 1);
+            mbar_init(&d_empty[i], TC_MATH_WARPS);
+        }
+        for (int i = 0; i < 4; ++i) {
+            mbar_init(&a_full[i], TC_MATH_WARPS);
+            mbar_init(&a_empty[i], 1);
+        }
+        mbar_init(fin, 1);
+        *abort = 0;
+    }
+    if (warp == TC_MATH_WARPS + 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(TC_TMEM_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    fence_barrier_init();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(tmem_slot);
+
+    const int n_chunks = __ldcg(a.n_chunks);
+    const int64_t tiles0 = (j0.N / 4 + TC_RG - 1) / TC_RG;
+    const int64_t tiles1 = njobs > 1 ? (j1.N / 4 + TC_RG - 1) / TC_RG : 0;
+    const int64_t per_chunk = tiles0 + tiles1;
+    const int64_t items = static_cast<int64_t>(n_chunks) * per_chunk;
+
+    // All roles walk the same items and blocks, so each keeps identical
+    // counts of raw stages and blocks used so far (the ring positions).
+    int64_t nraw = 0, nblk = 0;
+    // Producer: uses issued on each stage's full barriers (for the drain).
+    int64_t n_rf[2] = {0, 0}, n_bf[2] = {0, 0};
+    for (int64_t w = blockIdx.x; w < items; w += gridDim.x) {
+        if (*reinterpret_cast<volatile int *>(abort)) break;
+        const int chunk = static_cast<int>(w / per_chunk);
+        int64_t tl = w - chunk * per_chunk;
+        const bool second = tl >= tiles0;
+        if (second) tl -= tiles0;
+        const TcJob &J = second ? j1 : j0;
+        const int e = __ldcg(a.chunk_expert + chunk);
+        const int pb = __ldcg(a.chunk_begin + chunk);
+        const int m = __ldcg(a.chunk_len + chunk);
+        const int n_rg = J.N / 4;
+        const int rg0 = static_cast<int>(tl) * TC_RG;
+        const int nb = J.nb;
+
+        if (warp == TC_MATH_WARPS) {
+            // ---------------- producer ----------------
+            if (lane == 0) {
+                const CUtensorMap *wmap = second ? &wmap1 : &wmap0;
+                for (int b = 0; b < nb; ++b) {
+                    const int64_t bb = nblk + b;
+                    if ((b & 1) == 0) {
+                        const int64_t rb = nraw + b / 2;
+                        const int rs = static_cast<int>(rb & 1);
+                        if (!tc_wait(&raw_empty[rs], static_cast<uint32_t>(((rb >> 1) & 1) ^ 1), abort, a.status, 1))
+                            break;
+                        mbar_arrive_expect_tx(&raw_full[rs], TC_RG * TC_RAW_ROW);
+                        tma_2d(smem + TC_OFF_RAW + rs * TC_RAW_BYTES, wmap, (b / 2) * (TC_RAW_ROW / 8),
+                               e * n_rg + rg0, &raw_full[rs]);
+                        ++n_rf[rs];
+                    }
+                    const int bs = static_cast<int>(bb & 1);
+                    const uint32_t par = static_cast<uint32_t>(((bb >> 1) & 1) ^ 1);
+                    if (!tc_wait(&b_empty[bs], par, abort, a.status, 2)) break;
+                    mbar_arrive_expect_tx(&b_full[bs], TC_B_BYTES);
+                    for (int ks = 0; ks < 4; ++ks)
+                        tma_2d(smem + TC_OFF_B + bs * TC_B_BYTES + ks * TC_B_KS_BYTES, &bmap, b * QK + ks * 64, pb,
+                               &b_full[bs]);
+                    if (!tc_wait(&da_empty[bs], par, abort, a.status, 3)) break;
+                    mbar_arrive_expect_tx(&da_full[bs], TC_DA_BYTES);
+                    tma_2d(smem + TC_OFF_DA + bs * TC_DA_BYTES, &damap, 4 * (b >> 2), pb, &da_full[bs]);
+                    ++n_bf[bs];
+                }
+            }
+            __syncwarp();
+        } else if (warp == TC_MATH_WARPS + 1) {
+            // ---------------- MMA issuer ----------------
+            if (lane == 0) {
+                for (int b = 0; b < nb; ++b) {
+                    const int64_t bb = nblk + b;
+                    const int bs = static_cast<int>(bb & 1);
+                    const uint32_t par = static_cast<uint32_t>((bb >> 1) & 1);
+                    if (!tc_wait(&d_empty[bs], par ^ 1, abort, a.status, 4)) break;
+                    if (!tc_wait(&b_full[bs], par, abort, a.status, 5)) break;
+                    tc_fence_after();
+                    const uint32_t d_tmem = tmem + bs * TC_N;
+                    bool ok = true;
+                    for (int ks = 0; ks < 4; ++ks) {
+                        const int64_t kidx = bb * 4 + ks;  // A stage uses so far
+                        const int as = static_cast<int>(kidx & 3);
+                        if (!tc_wait(&a_full[as], static_cast<uint32_t>((kidx >> 2) & 1), abort, a.status, 6)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t abase = smem_u32(smem + TC_OFF_A + as * TC_A_BYTES);
+                        const uint32_t bbase = smem_u32(smem + TC_OFF_B + bs * TC_B_BYTES + ks * TC_B_KS_BYTES);
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk)
+                            tc_mma(d_tmem, umma_desc(abase + kk * 32), umma_desc(bbase + kk * 32),
+                                   (ks | kk) != 0 ? 1u : 0u);
+                        tc_commit(&a_empty[as]);
+                    }
+                    if (!ok) break;
+                    tc_commit(&b_empty[bs]);
+                    tc_commit(&d_full[bs]);
+                }
+            }
+            __syncwarp();
+        } else {
+            // ---------------- math warps ----------------
+            const int t = threadIdx.x;             // 0 .. 255
+            const int row = (warp & 3) * 32 + lane;  // this thread's tile row = TMEM lane (epilogue)
+            const int half = warp >> 2;              // columns 32 half .. 32 half + 31
+            // Unpacking map: 8 threads per 128-byte A row (one 16-byte chunk
+            // each); the two rows of a half-warp are 4 row groups apart, so
+            // their 64-byte source ranges fall in disjoint banks.
+            const int q = t >> 3, cq = t & 7;
+            const int rgl_u = 8 * (q >> 3) + 4 * (q & 1) + ((q >> 1) & 3);
+            float y[32];
+#pragma unroll
+            for (int n = 0; n < 32; ++n) y[n] = 0.0f;
+            float dw_prev = 0.0f;
+            bool ok = true;
+            for (int b = 0; b <= nb && ok; ++b) {
+                float dw_cur = 0.0f;
+                if (b < nb) {
+                    const int64_t rb = nraw + b / 2;
+                    const int rs = static_cast<int>(rb & 1);
+                    if ((b & 1) == 0 &&
+                        !tc_warp_wait(&raw_full[rs], static_cast<uint32_t>((rb >> 1) & 1), abort, a.status, 7)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint8_t *raw = smem + TC_OFF_RAW + rs * TC_RAW_BYTES + (b & 1) * BLOCK_BYTES;
+                    dw_cur = block_scale(raw + (row >> 2) * TC_RAW_ROW, row & 3);
+                    for (int ks = 0; ks < 4; ++ks) {
+                        const int64_t kidx = (nblk + b) * 4 + ks;
+                        const int as = static_cast<int>(kidx & 3);
+                        if (!tc_warp_wait(&a_empty[as], static_cast<uint32_t>(((kidx >> 2) & 1) ^ 1), abort,
+                                          a.status, 8)) {
+                            ok = false;
+                            break;
+                        }
+                        // elements 64 ks .. 64 ks + 63 of a row: code bytes
+                        // 64 (ks & 1) .. + 63, low nibbles for ks < 2
+                        uint8_t *atile = smem + TC_OFF_A + as * TC_A_BYTES;
+                        const int hi = ks >> 1;
+#pragma unroll
+                        for (int it = 0; it < 4; ++it) {
+                            const int r = 4 * rgl_u + it;  // tile row
+                            const uint2 wv = *reinterpret_cast<const uint2 *>(
+                                raw + rgl_u * TC_RAW_ROW + CODE_OFS + ROW_BYTES * it + 64 * (ks & 1) + 8 * cq);
+                            const uint32_t x0 = (hi ? (wv.x >> 4) : wv.x) & 0x0f0f0f0fu;
+                            const uint32_t x1 = (hi ? (wv.y >> 4) : wv.y) & 0x0f0f0f0fu;
+                            uint4 o;
+                            o.x = nib2bf16x2(x0, 0x4140u);
+                            o.y = nib2bf16x2(x0, 0x4342u);
+                            o.z = nib2bf16x2(x1, 0x4140u);
+                            o.w = nib2bf16x2(x1, 0x4342u);
+                            *reinterpret_cast<uint4 *>(atile + (r >> 3) * 1024 + (r & 7) * 128 +
+                                                       ((cq ^ (r & 7)) << 4)) = o;
+                        }
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&a_full[as]);
+                    }
+                    if (!ok) break;
+                    if (b & 1) {
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&raw_empty[rs]);
+                    }
+                }
+                if (b > 0) {
+                    // epilogue of block b - 1
+                    const int64_t bb = nblk + b - 1;
+                    const int bs = static_cast<int>(bb & 1);
+                    const uint32_t par = static_cast<uint32_t>((bb >> 1) & 1);
+                    if (!tc_warp_wait(&d_full[bs], par, abort, a.status, 9) ||
+                        !tc_warp_wait(&da_full[bs], par, abort, a.status, 10)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    uint32_t d[32];
+                    tc_ld32(tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + bs * TC_N + 32 * half, d);
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&d_empty[bs]);
+                    const float *da = reinterpret_cast<const float *>(smem + TC_OFF_DA + bs * TC_DA_BYTES);
+                    const int col = (b - 1) & 3;  // the block's column in the 4-block scale box
+#pragma unroll
+                    for (int n = 0; n < 32; ++n)
+                        y[n] = __fadd_rn(y[n], __fmul_rn(__uint_as_float(d[n]),
+                                                         __fmul_rn(dw_prev, da[(32 * half + n) * 4 + col])));
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&da_empty[bs]);
+                }
+                dw_prev = dw_cur;
+            }
+            if (ok && rg0 + (row >> 2) < n_rg) {
+                const int64_t grow = static_cast<int64_t>(rg0) * 4 + row;
+#pragma unroll
+                for (int n = 0; n < 32; ++n)
+                    if (32 * half + n < m) J.Y[static_cast<int64_t>(pb + 32 * half + n) * J.N + grow] = y[n];
+            }
+        }
+        nraw += (nb + 1) / 2;
+        nblk += nb;
+    }
+
+    // Drain: nothing asynchronous may still target this CTA's shared memory
+    // or TMEM when it exits. After a normal run these waits return at once.
+    if (warp == TC_MATH_WARPS && lane == 0) {
+        for (int s = 0; s < 2; ++s) {
+            if (n_rf[s] > 0) mbar_wait(&raw_full[s], static_cast<uint32_t>((n_rf[s] - 1) & 1));
+            if (n_bf[s] > 0) {
+                mbar_wait(&b_full[s], static_cast<uint32_t>((n_bf[s] - 1) & 1));
+                mbar_wait(&da_full[s], static_cast<uint32_t>((n_bf[s] - 1) & 1));
+            }
+        }
+    }
+    if (warp == TC_MATH_WARPS + 1 && lane == 0) {
+        tc_commit(fin);
+        mbar_wait(fin, 0);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == TC_MATH_WARPS + 1)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TC_TMEM_COLS) : "memory");
+}
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode_tc = nullptr;
+
+cudaError_t encode_2d(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t d0, uint64_t d1,
+                      uint64_t stride1, uint32_t b0, uint32_t b1, CUtensorMapSwizzle sw) {
+    if (!g_encode_tc) {
+        cudaDriverEntryPointQueryResult q;
+        void *fn = nullptr;
+        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e != cudaSuccess) return e;
+        if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+        g_encode_tc = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    const cuuint64_t dims[2] = {d0, d1};
+    const cuuint64_t strides[1] = {stride1};
+    const cuuint32_t box[2] = {b0, b1};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode_tc(m, dt, 2, const_cast<void *>(base), dims, strides, box, estr,
+                             CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+int tc_gemm_smem() { return TC_SMEM; }
+
+// One grouped projection pass on tensor cores: gate and up into g and u
+// (down = false), or down into o (down = true). Needs the bf16 activation
+// rows (xgb or qhb) and the padded per-pair scales (dxg or dhp).
+cudaError_t launch_tc_gemm(const GroupedArgs &a, bool down, cudaStream_t st) {
+    static unsigned char set_tc[64];
+    cudaError_t e = allow_max_smem(reinterpret_cast<const void *>(tc_gemm_kernel), set_tc);
+    if (e != cudaSuccess) return e;
+    const int nb = down ? a.nbi : a.nbh;
+    const int N = down ? a.H : a.I;
+    const int K = nb * QK;
+    const int nbp = down ? a.nbip : a.nbhp;
+    const uint8_t *m0 = down ? a.down : a.gate;
+    const uint8_t *m1 = down ? a.down : a.up;
+    // weights: one row per row group (E * N / 4 rows of nb * 520 bytes) as
+    // 8-byte elements; boxes of two blocks x 32 row groups
+    const uint64_t wd0 = static_cast<uint64_t>(nb) * BLOCK_BYTES / 8;
+    const uint64_t wd1 = static_cast<uint64_t>(a.E) * (N / 4);
+    const uint64_t wstride = static_cast<uint64_t>(nb) * BLOCK_BYTES;
+    CUtensorMap w0, w1, bm, dm;
+    if ((e = encode_2d(&w0, CU_TENSOR_MAP_DATA_TYPE_UINT64, m0, wd0, wd1, wstride, TC_RAW_ROW / 8, TC_RG,
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) != cudaSuccess)
+        return e;
+    if ((e = encode_2d(&w1, CU_TENSOR_MAP_DATA_TYPE_UINT64, m1, wd0, wd1, wstride, TC_RAW_ROW / 8, TC_RG,
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) != cudaSuccess)
+        return e;
+    // activations: [P][K] bf16; boxes of 64 elements (128 bytes) x 64 pairs
+    const void *act = down ? static_cast<const void *>(a.qhb) : static_cast<const void *>(a.xgb);
+    if ((e = encode_2d(&bm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, act, K, a.P, static_cast<uint64_t>(K) * 2, 64, TC_N,
+                       CU_TENSOR_MAP_SWIZZLE_128B)) != cudaSuccess)
+        return e;
+    // activation scales: [P][nbp] fp32; boxes of 4 blocks x 64 pairs
+    const void *da = down ? static_cast<const void *>(a.dhp) : static_cast<const void *>(a.dxg);
+    if ((e = encode_2d(&dm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, da, nbp, a.P, static_cast<uint64_t>(nbp) * 4, 4, TC_N,
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) != cudaSuccess)
+        return e;
+    const TcJob j0{N, nb, down ? a.o : a.g};
+    const TcJob j1{N, nb, down ? a.o : a.u};
+    tc_gemm_kernel<<<num_sms(), TC_THREADS, TC_SMEM, st>>>(a, j0, j1, down ? 1 : 2, w0, w1, bm, dm);
+    return cudaGetLastError();
+}
+
+}  // namespace tq

@@ -1,5 +1,7 @@
 """GPU parity of tqfx4_moe_grouped (T tokens grouped by expert: batched
-decode and prefill) against the CPU oracle, through the C ABI.
+decode and prefill) against the CPU oracle, through the C ABI, on both
+contractions: the decode path (legacy integer MMA) and the prefill path
+(tcgen05 tensor cores on exact bf16 operands).
 
 Per call: the routing of every token (bit-exact up to accepted near-ties),
 the grouping (counts, offsets and the stable expert-then-token order,
@@ -80,23 +82,43 @@ def check_grouped(layer, seed, X, sample, path=0, check_stages=True):
     (4, 512, 512, 4, 3, 0.0),        # top_k = n_experts
     (64, 2048, 1536, 8, 1, 0.0),     # a single token; inter not a multiple of 1024
 ])
-def test_grouped_small(E, H, I, k, T, zipf):
+@pytest.mark.parametrize("path", [B.TQFX4_PATH_DECODE, B.TQFX4_PATH_PREFILL])
+def test_grouped_small(E, H, I, k, T, zipf, path):
     seed = 100 + E + T
     layer = MoeLayer.synthetic(seed, E, H, I, k, zipf, DEV)
     X = inputs.hidden_states(seed, T, H)
-    check_grouped(layer, seed, X, sample=range(min(T, 6)))
+    check_grouped(layer, seed, X, sample=range(min(T, 6)), path=path)
 
 
-def test_grouped_equals_per_token_moe_ffn():
+@pytest.mark.parametrize("path", [B.TQFX4_PATH_DECODE, B.TQFX4_PATH_PREFILL])
+def test_grouped_equals_per_token_moe_ffn(path):
     layer = MoeLayer.synthetic(5, 32, 1024, 1024, 8, 0.0, DEV)
     X = inputs.hidden_states(5, 24, 1024)
-    ws, OUT, sel, selw = run_grouped(layer, X)
+    ws, OUT, sel, selw = run_grouped(layer, X, path)
     wsd = layer.workspace(1)
     for t in range(24):
         out, s, w = layer.ffn(X[t].to(DEV), wsd)
         assert np.array_equal(s.cpu().numpy(), sel[t])
         assert np.array_equal(w.cpu().numpy(), selw[t])
         assert np.array_equal(out.cpu().numpy().view(np.uint32), OUT[t].view(np.uint32))
+
+
+def test_tensor_core_path_equals_integer_mma_path():
+    # every pair's g, u, quantized h and expert output, and the combined
+    # output, bit-identical between the two contractions: ~150 pairs per
+    # expert (three chunks, ragged), 8 row tiles of 128 rows, ragged tiles
+    E, H, I, k, T = 16, 1536, 1024, 4, 600
+    layer = MoeLayer.synthetic(8, E, H, I, k, 0.5, DEV)
+    X = inputs.hidden_states(8, T, H)
+    P = T * k
+    res = []
+    for path in (B.TQFX4_PATH_DECODE, B.TQFX4_PATH_PREFILL):
+        ws, OUT, sel, selw = run_grouped(layer, X, path)
+        g = lambda name, dt, shape: layer.view(ws, name, dt, shape, tokens=T, grouped=1, path=path).cpu().numpy()
+        res.append([OUT, sel, g("g", torch.float32, (P, I)), g("u", torch.float32, (P, I)),
+                    g("qh", torch.int8, (P, I)), g("o", torch.float32, (P, H))])
+    for a, b in zip(*res):
+        assert np.array_equal(a.view(np.uint8), b.view(np.uint8))
 
 
 def test_grouped_empty_batch():
