@@ -103,14 +103,15 @@ __device__ __forceinline__ int block_scan_1024(int v, int *warp_tot) {
 }
 
 __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
-    __shared__ int cnt[TQFX4_MAX_EXPERTS], off[TQFX4_MAX_EXPERTS + 1], run[TQFX4_MAX_EXPERTS];
+    // counts, offsets, the chunk list and the stable (token, slot) order of
+    // the pairs inside each expert's range
+    constexpr int HIST = 8192;  // per-warp counts: warps x experts
+    __shared__ int cnt[TQFX4_MAX_EXPERTS], off[TQFX4_MAX_EXPERTS + 1];
+    __shared__ int hist[HIST];
     __shared__ int warp_tot[32];
-    const int tid = threadIdx.x, lane = tid & 31;
-    const int E = a.E, P = a.P, k = a.top_k;
-    if (tid < E) {
-        cnt[tid] = 0;
-        run[tid] = 0;
-    }
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int E = a.E, P = a.P, k = a.top_k, CH = a.chunk;
+    if (tid < E) cnt[tid] = 0;
     __syncthreads();
     for (int p = tid; p < P; p += blockDim.x) atomicAdd(&cnt[__ldcg(a.sel + p)], 1);
     __syncthreads();
@@ -125,42 +126,67 @@ __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
         off[0] = 0;
         a.offsets[0] = 0;
     }
-    // chunk list: ceil(count / GG_TOK) chunks per expert
-    const int nc = (c + GG_TOK - 1) / GG_TOK;
+    // chunk list: ceil(count / CH) chunks per expert
+    const int nc = (c + CH - 1) / CH;
     const int cincl = block_scan_1024(nc, warp_tot);
     if (tid < E) {
         const int base = cincl - nc;
         for (int i = 0; i < nc; ++i) {
             a.chunk_expert[base + i] = tid;
-            a.chunk_begin[base + i] = incl - c + i * GG_TOK;
-            a.chunk_len[base + i] = min(GG_TOK, c - i * GG_TOK);
+            a.chunk_begin[base + i] = incl - c + i * CH;
+            a.chunk_len[base + i] = min(CH, c - i * CH);
         }
     }
     if (tid == blockDim.x - 1) *a.n_chunks = cincl;
+    // Stable placement: W warps take consecutive ranges of the pairs; each
+    // counts its hits per expert, the counts are turned into per-warp start
+    // positions (expert offset + hits of the earlier ranges), and each warp
+    // places its pairs in order, ranking equal experts by lane.
+    const int W = min(32, HIST / E);
+    const int R = (P + W - 1) / W;
+    for (int i = tid; i < W * E; i += blockDim.x) hist[i] = 0;
     __syncthreads();
-    // stable placement by one warp: pairs visited in (token, slot) order
-    if (tid < 32) {
-        const unsigned lt = (1u << lane) - 1u;
-        for (int base = 0; base < P; base += 32) {
+    const unsigned lt = (1u << lane) - 1u;
+    if (warp < W) {
+        const int p0 = warp * R, p1 = min(P, p0 + R);
+        for (int base = p0; base < p1; base += 32) {
             const int p = base + lane;
-            const bool valid = p < P;
+            const bool valid = p < p1;
             const int e = valid ? __ldcg(a.sel + p) : -1 - lane;
             const unsigned peers = __match_any_sync(0xffffffffu, e);
-            const int rank = __popc(peers & lt);
+            if (valid && lane == __ffs(peers) - 1) hist[warp * E + e] += __popc(peers);
+        }
+    }
+    __syncthreads();
+    if (tid < E) {
+        int run = off[tid];
+        for (int w = 0; w < W; ++w) {
+            const int h = hist[w * E + tid];
+            hist[w * E + tid] = run;
+            run += h;
+        }
+    }
+    __syncthreads();
+    if (warp < W) {
+        const int p0 = warp * R, p1 = min(P, p0 + R);
+        for (int base = p0; base < p1; base += 32) {
+            const int p = base + lane;
+            const bool valid = p < p1;
+            const int e = valid ? __ldcg(a.sel + p) : -1 - lane;
+            const unsigned peers = __match_any_sync(0xffffffffu, e);
             const int leader = __ffs(peers) - 1;
             int b = 0;
             if (valid && lane == leader) {
-                b = run[e];
-                run[e] = b + __popc(peers);
+                b = hist[warp * E + e];
+                hist[warp * E + e] = b + __popc(peers);
             }
             b = __shfl_sync(0xffffffffu, b, leader);
             if (valid) {
-                const int pos = off[e] + b + rank;
+                const int pos = b + __popc(peers & lt);
                 a.pair_token[pos] = p / k;
                 a.pair_slot[pos] = p - (p / k) * k;
                 a.pair_of[p] = pos;
             }
-            __syncwarp();
         }
     }
 }
@@ -462,20 +488,33 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(GroupedArgs a) {
     const int64_t pos = blockIdx.x;
     const int64_t t = __ldcg(a.pair_token + pos);
     const uint4 *src = reinterpret_cast<const uint4 *>(a.qx + t * a.H);
-    if (a.tc) {
-        // bf16 copy for the tensor-core contraction (int8 values are exact in bf16)
-        uint4 *dst = reinterpret_cast<uint4 *>(a.xgb + pos * a.H);
-        for (int i = threadIdx.x; i < a.H / 8; i += blockDim.x) {
-            const uint2 v = __ldcg(reinterpret_cast<const uint2 *>(a.qx + t * a.H) + i);
-            dst[i] = i8x8_to_bf16x8(v);
-        }
-    } else {
-        uint4 *dst = reinterpret_cast<uint4 *>(a.xg + pos * a.H);
-        for (int i = threadIdx.x; i < a.H / 16; i += blockDim.x) dst[i] = __ldcg(src + i);
-    }
+    uint4 *dst = reinterpret_cast<uint4 *>(a.xg + pos * a.H);
+    for (int i = threadIdx.x; i < a.H / 16; i += blockDim.x) dst[i] = __ldcg(src + i);
     for (int b = threadIdx.x; b < a.nbhp; b += blockDim.x) {
         a.dxg[pos * a.nbhp + b] = b < a.nbh ? __ldcg(a.dx + t * a.nbh + b) : 0.0f;
         a.bxg[pos * a.nbhp + b] = b < a.nbh ? __ldcg(a.bx + t * a.nbh + b) : 0;
+    }
+}
+
+// Tensor-core path: per chunk, the bf16 rows of its pairs' quantized hidden
+// states, and per block the pairs' scales da in the chunk-aligned layout
+// the contraction stages with one bulk copy.
+__global__ void __launch_bounds__(256) gather_tc_kernel(GroupedArgs a) {
+    const int c = blockIdx.x;
+    if (c >= __ldcg(a.n_chunks)) return;
+    const int pb = __ldcg(a.chunk_begin + c), m = __ldcg(a.chunk_len + c);
+    for (int n = threadIdx.x >> 5; n < m; n += blockDim.x >> 5) {
+        const int64_t pos = pb + n;
+        const int64_t t = __ldcg(a.pair_token + pos);
+        const uint2 *src = reinterpret_cast<const uint2 *>(a.qx + t * a.H);
+        uint4 *dst = reinterpret_cast<uint4 *>(a.xgb + pos * a.H);
+        for (int i = threadIdx.x & 31; i < a.H / 8; i += 32) dst[i] = i8x8_to_bf16x8(__ldcg(src + i));
+        if ((threadIdx.x & 31) == 0) a.pair_chunk[pos] = c;
+    }
+    for (int i = threadIdx.x; i < a.nbh * TC_CHUNK; i += blockDim.x) {
+        const int b = i / TC_CHUNK, n = i - b * TC_CHUNK;
+        const float d = n < m ? __ldcg(a.dx + __ldcg(a.pair_token + pb + n) * static_cast<int64_t>(a.nbh) + b) : 0.0f;
+        a.xs[(static_cast<int64_t>(c) * a.nbh + b) * TC_CHUNK + n] = d;
     }
 }
 
@@ -502,7 +541,14 @@ __global__ void __launch_bounds__(256) swiglu_quant_kernel(GroupedArgs a) {
     int sum;
     const bool ok = quant_block_warp(hv, packed, d, sum);
     *reinterpret_cast<uint2 *>(a.qh + o) = packed;
-    if (a.tc) *reinterpret_cast<uint4 *>(a.qhb + o) = i8x8_to_bf16x8(packed);
+    if (a.tc) {
+        *reinterpret_cast<uint4 *>(a.qhb + o) = i8x8_to_bf16x8(packed);
+        if (lane == 0) {
+            const int c = __ldcg(a.pair_chunk + p);
+            const int n = static_cast<int>(p - __ldcg(a.chunk_begin + c));
+            a.hs[(static_cast<int64_t>(c) * a.nbi + b) * TC_CHUNK + n] = d;
+        }
+    }
     if (a.keep_h) {
         reinterpret_cast<float4 *>(a.h + o)[0] = make_float4(hv[0], hv[1], hv[2], hv[3]);
         reinterpret_cast<float4 *>(a.h + o)[1] = make_float4(hv[4], hv[5], hv[6], hv[7]);
@@ -634,6 +680,8 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
     a.nbhp = (a.nbh + 3) / 4 * 4;
     a.nbip = (a.nbi + 3) / 4 * 4;
     L = moe_layout(a.E, a.H, a.I, a.top_k, T, true, true);
+    a.max_chunks = static_cast<int>(L.max_chunks);
+    a.chunk = GG_TOK;
     uint8_t *base = static_cast<uint8_t *>(ws);
     if (base) {
         a.status = reinterpret_cast<int *>(base);
@@ -667,6 +715,9 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
         a.n_chunks = reinterpret_cast<int *>(base + L.n_chunks);
         a.xgb = reinterpret_cast<uint16_t *>(base + L.xgb);
         a.qhb = reinterpret_cast<uint16_t *>(base + L.qhb);
+        a.pair_chunk = reinterpret_cast<int *>(base + L.pair_chunk);
+        a.xs = reinterpret_cast<float *>(base + L.xs);
+        a.hs = reinterpret_cast<float *>(base + L.hs);
     }
     return true;
 }
@@ -682,6 +733,7 @@ const char *grouped_stage_name(int s) {
 cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT, int32_t *sel_idx, float *sel_w,
                                cudaStream_t st, void *const *events) {
     GroupedArgs a = a0;
+    a.chunk = a.tc ? TC_CHUNK : GG_TOK;
     a.X = X;
     a.OUT = OUT;
     a.sel_out = sel_idx;
@@ -709,7 +761,10 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(3);
     if ((e = launch_quantize(a.X, a.T, a.H, a.qx, a.dx, a.bx, a.status, st)) != cudaSuccess) return e;
-    gather_rows_kernel<<<a.P, 256, 0, st>>>(a);
+    if (a.tc)
+        gather_tc_kernel<<<a.max_chunks, 256, 0, st>>>(a);
+    else
+        gather_rows_kernel<<<a.P, 256, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(4);
     const int64_t units = static_cast<int64_t>(a.P) * a.nbi;

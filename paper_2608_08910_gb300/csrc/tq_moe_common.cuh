@@ -24,6 +24,7 @@ struct MoeLayout {
     size_t dxg, bxg, dhp, bhp;  // [P][round4(nb)] (grouped only)
     size_t chunk_expert, chunk_begin, chunk_len, n_chunks;  // grouped GEMM work list
     size_t xgb, qhb;  // bf16 [P][H], [P][I] activation rows for the tensor-core contraction (grouped only)
+    size_t pair_chunk, xs, hs;  // tensor-core work list helpers (grouped only)
     int64_t max_chunks;
     size_t total;
 };
@@ -32,6 +33,8 @@ struct MoeLayout {
 constexpr int GG_TOK = 64;
 // Pairs from which the automatic path choice takes the tensor-core contraction.
 constexpr int64_t kTcMinPairs = 4096;
+// Pairs per chunk on the tensor-core path (the largest MMA N used).
+constexpr int TC_CHUNK = 128;
 
 inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
@@ -85,11 +88,14 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.n_chunks = take(4);
         L.xgb = take(2 * static_cast<size_t>(P * H));
         L.qhb = take(2 * static_cast<size_t>(P * I));
+        L.pair_chunk = take(4 * static_cast<size_t>(P));
+        L.xs = take(static_cast<size_t>(L.max_chunks) * nbh * TC_CHUNK * 4);
+        L.hs = take(static_cast<size_t>(L.max_chunks) * nbi * TC_CHUNK * 4);
     } else {
         L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = L.xg = SIZE_MAX;
         L.dxg = L.bxg = L.dhp = L.bhp = SIZE_MAX;
         L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
-        L.xgb = L.qhb = SIZE_MAX;
+        L.xgb = L.qhb = L.pair_chunk = L.xs = L.hs = SIZE_MAX;
         L.max_chunks = 0;
     }
     L.total = off;
@@ -156,8 +162,13 @@ struct GroupedArgs {
     int *counts, *offsets, *pair_token, *pair_slot, *pair_of;
     int *chunk_expert, *chunk_begin, *chunk_len, *n_chunks;
     int keep_h;
-    int tc;              // contraction on tcgen05 tensor cores (bf16 activation rows below)
-    uint16_t *xgb, *qhb;  // bf16 copies of xg [P][H] and qh [P][I]
+    int tc;               // contraction on tcgen05 tensor cores
+    int chunk;            // pairs per chunk of the work list (GG_TOK, or TC_CHUNK on tensor cores)
+    int max_chunks;       // capacity of the work list
+    uint16_t *xgb, *qhb;  // bf16 copies of xg [P][H] and qh [P][I] (tensor-core path)
+    int *pair_chunk;      // [P] chunk of each pair (tensor-core path)
+    float *xs, *hs;       // [chunks][nb][TC_CHUNK]: per chunk and block, the pairs' scales da
+                          // (tensor-core path)
 };
 
 // Shared-memory bytes of one quantized activation vector of nb blocks

@@ -1,29 +1,44 @@
 // Grouped expert GEMM on the 5th-generation tensor cores (tcgen05), the
-// contraction of the prefill path: one work item is 128 weight rows of one
-// expert times one chunk of <= 64 (token, slot) pairs of that expert.
+// contraction of the prefill path: one work item is 128 weight rows (32 row
+// groups) of one expert times one chunk of <= 128 (token, slot) pairs of
+// that expert.
 //
 // tcgen05.mma has no integer kind on sm_103a, so the integer block sums
-// S = sum_j c_j q_j (Eq. 5) are formed with kind::f16 on bf16 operands: the
-// codes c in -4..4 and the int8 activations q are exact in bf16, every
-// product is an exact integer, and the fp32 accumulator of one 256-element
-// block stays below 2^17 in magnitude, so it holds S exactly whatever the
-// order of the additions. The accumulator restarts at every block (the
-// block's first MMA does not accumulate) and the epilogue applies the fixed
-// float schedule y = y + float(S) * (d * da) block by block, the same
+// S = sum_j c_j q_j (Eq. 5) are formed with kind::f16 on bf16 operands that
+// hold small integers exactly: the codes c in -4..4 (A) and the int8
+// activations q (B). Every product is an exact integer and |S| < 2^17, so
+// the fp32 accumulator of one 256-element block holds S exactly. (Operands
+// with an offset, such as 128 + u, make the block sums reach 2^22, and
+// there the tensor core's sums are no longer exact: the codes are centred.)
+// The accumulator restarts at every block and the epilogue applies the
+// fixed float schedule y = y + float(S) * (d * da) block by block, the same
 // operations in the same order as the streaming kernels and the oracle.
 //
+// Operands: A (the unpacked weights) is written by the math warps straight
+// into tensor memory with tcgen05.st (thread = row = TMEM lane), so it never
+// passes through shared memory; B (bf16 activation rows of the chunk) is
+// staged by TMA in the 128-byte swizzled K-major layout.
+// Tile rows are ordered r4-major (tile row = 32 * r4 + row group), so that a
+// warp (one TMEM lane quadrant) reads the codes of one row of 32 row groups,
+// 1040 bytes apart: the 16-byte loads of odd blocks are conflict-free and
+// the 8-byte loads of even blocks (codes 8 bytes off 16-byte alignment)
+// two-way.
+//
 // Warp roles (320 threads, one CTA per SM):
-//   warps 0-7  math: unpack the tile's nibbles into bf16 A tiles (K-major,
-//              128-byte swizzled canonical layout), and one block behind,
-//              read the block's accumulator from TMEM and update y. Warps w
-//              and w + 4 share TMEM lanes 32 (w % 4) .. + 31 (the rows of
-//              the tile) and split the 64 columns (the pairs) in halves;
+//   warps 0-7  math. Warp w serves TMEM lanes 32 (w % 4) .. + 31 (rows with
+//              r4 = w % 4) and half h = w / 4: it unpacks code bytes
+//              64 h .. 64 h + 63 of its rows (elements 64 h + j and
+//              128 + 64 h + j) into A, and in the epilogue, one block behind,
+//              reads accumulator columns (pairs) 64 h .. 64 h + 63;
 //   warp 8     producer: TMA copies of the raw weight blocks (one box per two
-//              blocks of 32 row groups), of the bf16 activation tiles (four
-//              64 x 64 boxes per block, 128-byte swizzled) and of the
-//              activation scales (4 blocks x 64 pairs);
-//   warp 9     TMEM allocation; one elected thread issues the MMAs
-//              (M = 128, N = 64, K = 16; 16 per block) and the commits.
+//              blocks of the tile), of the activation tiles (64-element x
+//              64-pair boxes) and a bulk copy of the chunk's block scales;
+//   warp 9     TMEM allocation; one thread issues the MMAs (M = 128,
+//              N = the chunk's pairs rounded up to 16, K = 16; 16 per block)
+//              and the commits.
+// TMEM: A in columns [0, 256) (two blocks), accumulators in [256, 512).
+// The epilogue uses scalar fp32 multiplies and adds: the packed f32x2 forms
+// were measured to give results that differ from them.
 // Every wait is bounded. On a timeout the CTA records the error, all roles
 // leave their loops, the producer waits (bounded) for its copies in flight,
 // the MMA thread for its MMAs, and TMEM is freed before the CTA exits.
@@ -39,32 +54,34 @@ namespace {
 
 constexpr int TC_ROWS = 128;                   // weight rows per tile = TMEM lanes
 constexpr int TC_RG = TC_ROWS / 4;             // row groups per tile
-constexpr int TC_N = GG_TOK;                   // pairs per chunk = MMA N
 constexpr int TC_MATH_WARPS = 8;
 constexpr int TC_THREADS = (TC_MATH_WARPS + 2) * 32;
 constexpr int TC_RAW_ROW = 2 * BLOCK_BYTES;    // two blocks of one row group: 1040 bytes
 constexpr int TC_RAW_BYTES = 33 * 1024;        // 32 x 1040 bytes, padded
-constexpr int TC_A_BYTES = TC_ROWS * 128;      // one 64-element k-stage of A (bf16): 16 KB
-constexpr int TC_B_KS_BYTES = TC_N * 128;      // one k-stage of B: 8 KB
-constexpr int TC_B_BYTES = 4 * TC_B_KS_BYTES;  // one block of B: 32 KB
-constexpr int TC_DA_BYTES = 4 * TC_N * 4;      // scales of 64 pairs x 4 blocks: 1 KB
+constexpr int TC_BOX_BYTES = 64 * 128;         // one 64-element x 64-pair bf16 box: 8 KB
+constexpr int TC_KS_BYTES = 2 * TC_BOX_BYTES;  // one k-stage (64 elements) of up to 128 pairs
+constexpr int TC_B_BYTES = 4 * TC_KS_BYTES;    // one block of B: 64 KB
+constexpr int TC_SC_BYTES = TC_CHUNK * 4;      // da of the chunk's pairs: 512 bytes
 constexpr int TC_OFF_RAW = 0;
-constexpr int TC_OFF_A = TC_OFF_RAW + 2 * TC_RAW_BYTES;
-constexpr int TC_OFF_B = TC_OFF_A + 4 * TC_A_BYTES;
-constexpr int TC_OFF_DA = TC_OFF_B + 2 * TC_B_BYTES;
-constexpr int TC_OFF_BAR = TC_OFF_DA + 2 * TC_DA_BYTES;
-constexpr int TC_NBAR = 25;  // barriers; the TMEM address and abort flag follow
+constexpr int TC_OFF_B = TC_OFF_RAW + 2 * TC_RAW_BYTES;
+constexpr int TC_OFF_SC = TC_OFF_B + 2 * TC_B_BYTES;
+constexpr int TC_OFF_BAR = TC_OFF_SC + 2 * TC_SC_BYTES;
+constexpr int TC_NBAR = 21;  // barriers; the TMEM address and abort flag follow
 constexpr int TC_SMEM = TC_OFF_BAR + TC_NBAR * 8 + 16 + 1024;  // + alignment slack
-constexpr int TC_TMEM_COLS = 2 * TC_N;         // two accumulators (double buffer)
+constexpr int TC_TMEM_COLS = 512;
+constexpr uint32_t TC_TMEM_D = 256;            // first accumulator column
 
-static_assert(TC_OFF_A % 1024 == 0 && TC_OFF_B % 1024 == 0, "swizzled tiles need 1024-byte alignment");
+static_assert(TC_OFF_B % 1024 == 0, "swizzled tiles need 1024-byte alignment");
 static_assert(TC_RG * TC_RAW_ROW <= TC_RAW_BYTES, "raw stage too small");
+static_assert(TC_CHUNK == 128, "two 64-pair boxes and two 64-column epilogue halves");
 
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1),
 // A and B bf16 (bits 7-9 = 1, 10-12 = 1), both K-major (bits 15, 16 = 0),
 // N >> 3 at bits 17-22, M >> 4 at bits 24-28.
-constexpr uint32_t TC_IDESC = (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(TC_N >> 3) << 17) |
-                              (static_cast<uint32_t>(TC_ROWS >> 4) << 24);
+__device__ __forceinline__ uint32_t tc_idesc(int n) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
+           (static_cast<uint32_t>(TC_ROWS >> 4) << 24);
+}
 
 // Shared-memory matrix descriptor of a K-major operand in the 128-byte
 // swizzle canonical layout: rows of 128 bytes, 8-row atoms of 1024 bytes
@@ -78,11 +95,13 @@ __device__ __forceinline__ uint64_t umma_desc(uint32_t saddr) {
     return d;
 }
 
-__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+// D (tmem) [+]= A (tmem) x B (smem descriptor)
+__device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
     asm volatile(
         "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(TC_IDESC), "r"(accumulate)
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
 
@@ -96,20 +115,30 @@ __device__ __forceinline__ void tc_commit(uint64_t *bar) {
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
+#define TC_R32(r)                                                                                                    \
+    "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),    \
+        "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]),   \
+        "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]),   \
+        "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+#define TC_W32(r)                                                                                                    \
+    "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),      \
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),       \
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),      \
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+#define TC_LIST32                                                                                                    \
+    "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,"  \
+    "%30,%31}"
+
 // 32 TMEM lanes x 32 columns of 32 bits: the calling thread's lane, columns
 // taddr .. taddr + 31.
 __device__ __forceinline__ void tc_ld32(uint32_t taddr, uint32_t (&r)[32]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,"
-        "%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 " TC_LIST32 ", [%32];" : TC_W32(r) : "r"(taddr));
 }
+__device__ __forceinline__ void tc_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%32], " TC_LIST32 ";" ::TC_R32(r), "r"(taddr) : "memory");
+}
+__device__ __forceinline__ void tc_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 __device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int c0, int c1, uint64_t *bar) {
     asm volatile(
@@ -117,16 +146,6 @@ __device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int c0
             smem_u32(dst)),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
         : "memory");
-}
-
-// Two nibble codes u0, u1 (bytes `sel` picks from x) as bf16x2 of c = u - 4:
-// the bytes [u0, 0x43, u1, 0x43] are the bf16 values 128 + u0 and 128 + u1,
-// and adding -132 (bf16 0xC304) to each half is exact.
-__device__ __forceinline__ uint32_t nib2bf16x2(uint32_t x, uint32_t sel) {
-    uint32_t w, r;
-    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(w) : "r"(x), "r"(0x43u), "r"(sel));
-    asm("add.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(w), "r"(0xC304C304u));
-    return r;
 }
 
 struct TcJob {
@@ -144,8 +163,8 @@ __device__ __forceinline__ bool tc_wait(uint64_t *bar, uint32_t parity, int *abo
 }
 
 // Warp-uniform bounded wait (math warps): all lanes observe the phase, and
-// all agree on the outcome so that the .sync.aligned TMEM loads that follow
-// are executed by the whole warp or by none of it.
+// all agree on the outcome so that the .sync.aligned TMEM accesses that
+// follow are executed by the whole warp or by none of it.
 __device__ __forceinline__ bool tc_warp_wait(uint64_t *bar, uint32_t parity, int *abort, int *status, int where) {
     const int lane = threadIdx.x & 31;
     int ab = lane == 0 ? *reinterpret_cast<volatile int *>(abort) : 0;
@@ -159,22 +178,43 @@ __device__ __forceinline__ bool tc_warp_wait(uint64_t *bar, uint32_t parity, int
     return ok;
 }
 
+// Two nibbles u0, u1 (the bytes of x that `sel` picks, next to the byte
+// 0x43) as bf16x2 of c = u - 4: the bytes [u0, 0x43, u1, 0x43] are the bf16
+// values 128 + u, and adding -132 (bf16 0xC304) to each half is exact.
+__device__ __forceinline__ uint32_t nib_pair(uint32_t x, uint32_t sel) {
+    uint32_t w, r;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(w) : "r"(x), "r"(0x43434343u), "r"(sel));
+    asm("add.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(w), "r"(0xC304C304u));
+    return r;
+}
+
+// One 32-bit word of code bytes (4 bytes of one row) -> four A columns:
+// lo0, lo1 = elements j .. j+3 (low nibbles), hi0, hi1 = elements
+// 128 + j .. 131 + j (high nibbles).
+__device__ __forceinline__ void unpack_word(uint32_t x, uint32_t &lo0, uint32_t &lo1, uint32_t &hi0, uint32_t &hi1) {
+    const uint32_t l = x & 0x0f0f0f0fu, h = (x >> 4) & 0x0f0f0f0fu;
+    lo0 = nib_pair(l, 0x5140u);
+    lo1 = nib_pair(l, 0x5342u);
+    hi0 = nib_pair(h, 0x5140u);
+    hi1 = nib_pair(h, 0x5342u);
+}
+
 }  // namespace
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
-    tc_gemm_kernel(GroupedArgs a, TcJob j0, TcJob j1, int njobs, const __grid_constant__ CUtensorMap wmap0,
-                   const __grid_constant__ CUtensorMap wmap1, const __grid_constant__ CUtensorMap bmap,
-                   const __grid_constant__ CUtensorMap damap) {
+    tc_gemm_kernel(GroupedArgs a, TcJob j0, TcJob j1, int njobs, const float *__restrict__ scales,
+                   const __grid_constant__ CUtensorMap wmap0, const __grid_constant__ CUtensorMap wmap1,
+                   const __grid_constant__ CUtensorMap bmap) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + TC_OFF_BAR);
     uint64_t *raw_full = bars, *raw_empty = bars + 2;
-    uint64_t *a_full = bars + 4, *a_empty = bars + 8;
-    uint64_t *b_full = bars + 12, *b_empty = bars + 14;
-    uint64_t *da_full = bars + 16, *da_empty = bars + 18;
-    uint64_t *d_full = bars + 20, *d_empty = bars + 22;
-    uint64_t *fin = bars + 24;  // MMA drain at exit
+    uint64_t *a_full = bars + 4, *a_empty = bars + 6;
+    uint64_t *b_full = bars + 8, *b_empty = bars + 10;
+    uint64_t *sc_full = bars + 12, *sc_empty = bars + 14;
+    uint64_t *d_full = bars + 16, *d_empty = bars + 18;
+    uint64_t *fin = bars + 20;  // MMA drain at exit
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + TC_NBAR);
     int *abort = reinterpret_cast<int *>(tmem_slot + 1);
 
@@ -182,16 +222,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(&raw_full[i], 1);
             mbar_init(&raw_empty[i], TC_MATH_WARPS);
-            mbar_init(&b_full[i], 1);
-            mbar_init(&b_empty[i], 1);
-            mbar_init(&da_full[i], 1);
-            mbar_init(&da_empty[i], TC_MATH_WARPS);
-            mbar_init(&d_full[i], 1);
-            mbar_init(&d_empty[i], TC_MATH_WARPS);
-        }
-        for (int i = 0; i < 4; ++i) {
             mbar_init(&a_full[i], TC_MATH_WARPS);
             mbar_init(&a_empty[i], 1);
+            mbar_init(&b_full[i], 1);
+            mbar_init(&b_empty[i], 1);
+            mbar_init(&sc_full[i], 1);
+            mbar_init(&sc_empty[i], TC_MATH_WARPS);
+            mbar_init(&d_full[i], 1);
+            mbar_init(&d_empty[i], TC_MATH_WARPS);
         }
         mbar_init(fin, 1);
         *abort = 0;
@@ -218,7 +256,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     // counts of raw stages and blocks used so far (the ring positions).
     int64_t nraw = 0, nblk = 0;
     // Producer: uses issued on each stage's full barriers (for the drain).
-    int64_t n_rf[2] = {0, 0}, n_bf[2] = {0, 0};
+    int64_t n_rf0 = 0, n_rf1 = 0, n_bf0 = 0, n_bf1 = 0;
     for (int64_t w = blockIdx.x; w < items; w += gridDim.x) {
         if (*reinterpret_cast<volatile int *>(abort)) break;
         const int chunk = static_cast<int>(w / per_chunk);
@@ -232,11 +270,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         const int n_rg = J.N / 4;
         const int rg0 = static_cast<int>(tl) * TC_RG;
         const int nb = J.nb;
+        const int nbox = m > 64 ? 2 : 1;          // 64-pair boxes of B per k-stage
+        const int nmma = (m + 15) & ~15;          // MMA N
 
         if (warp == TC_MATH_WARPS) {
             // ---------------- producer ----------------
             if (lane == 0) {
                 const CUtensorMap *wmap = second ? &wmap1 : &wmap0;
+                const float *sc = scales + static_cast<int64_t>(chunk) * nb * TC_CHUNK;
                 for (int b = 0; b < nb; ++b) {
                     const int64_t bb = nblk + b;
                     if ((b & 1) == 0) {
@@ -247,51 +288,44 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         mbar_arrive_expect_tx(&raw_full[rs], TC_RG * TC_RAW_ROW);
                         tma_2d(smem + TC_OFF_RAW + rs * TC_RAW_BYTES, wmap, (b / 2) * (TC_RAW_ROW / 8),
                                e * n_rg + rg0, &raw_full[rs]);
-                        ++n_rf[rs];
+                        if (rs) ++n_rf1; else ++n_rf0;
                     }
                     const int bs = static_cast<int>(bb & 1);
                     const uint32_t par = static_cast<uint32_t>(((bb >> 1) & 1) ^ 1);
                     if (!tc_wait(&b_empty[bs], par, abort, a.status, 2)) break;
-                    mbar_arrive_expect_tx(&b_full[bs], TC_B_BYTES);
+                    mbar_arrive_expect_tx(&b_full[bs], 4 * nbox * TC_BOX_BYTES);
                     for (int ks = 0; ks < 4; ++ks)
-                        tma_2d(smem + TC_OFF_B + bs * TC_B_BYTES + ks * TC_B_KS_BYTES, &bmap, b * QK + ks * 64, pb,
-                               &b_full[bs]);
-                    if (!tc_wait(&da_empty[bs], par, abort, a.status, 3)) break;
-                    mbar_arrive_expect_tx(&da_full[bs], TC_DA_BYTES);
-                    tma_2d(smem + TC_OFF_DA + bs * TC_DA_BYTES, &damap, 4 * (b >> 2), pb, &da_full[bs]);
-                    ++n_bf[bs];
+                        for (int x = 0; x < nbox; ++x)
+                            tma_2d(smem + TC_OFF_B + bs * TC_B_BYTES + ks * TC_KS_BYTES + x * TC_BOX_BYTES, &bmap,
+                                   b * QK + ks * 64, pb + 64 * x, &b_full[bs]);
+                    if (!tc_wait(&sc_empty[bs], par, abort, a.status, 3)) break;
+                    mbar_arrive_expect_tx(&sc_full[bs], TC_SC_BYTES);
+                    bulk_g2s(smem + TC_OFF_SC + bs * TC_SC_BYTES, sc + b * TC_CHUNK, TC_SC_BYTES, &sc_full[bs]);
+                    if (bs) ++n_bf1; else ++n_bf0;
                 }
             }
             __syncwarp();
         } else if (warp == TC_MATH_WARPS + 1) {
             // ---------------- MMA issuer ----------------
             if (lane == 0) {
+                const uint32_t idesc = tc_idesc(nmma);
                 for (int b = 0; b < nb; ++b) {
                     const int64_t bb = nblk + b;
                     const int bs = static_cast<int>(bb & 1);
                     const uint32_t par = static_cast<uint32_t>((bb >> 1) & 1);
                     if (!tc_wait(&d_empty[bs], par ^ 1, abort, a.status, 4)) break;
                     if (!tc_wait(&b_full[bs], par, abort, a.status, 5)) break;
+                    if (!tc_wait(&a_full[bs], par, abort, a.status, 6)) break;
                     tc_fence_after();
-                    const uint32_t d_tmem = tmem + bs * TC_N;
-                    bool ok = true;
-                    for (int ks = 0; ks < 4; ++ks) {
-                        const int64_t kidx = bb * 4 + ks;  // A stage uses so far
-                        const int as = static_cast<int>(kidx & 3);
-                        if (!tc_wait(&a_full[as], static_cast<uint32_t>((kidx >> 2) & 1), abort, a.status, 6)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        const uint32_t abase = smem_u32(smem + TC_OFF_A + as * TC_A_BYTES);
-                        const uint32_t bbase = smem_u32(smem + TC_OFF_B + bs * TC_B_BYTES + ks * TC_B_KS_BYTES);
+                    const uint32_t d_tmem = tmem + TC_TMEM_D + bs * TC_CHUNK;
+                    const uint32_t a_tmem = tmem + bs * 128;
+                    const uint32_t bbase = smem_u32(smem + TC_OFF_B + bs * TC_B_BYTES);
 #pragma unroll
-                        for (int kk = 0; kk < 4; ++kk)
-                            tc_mma(d_tmem, umma_desc(abase + kk * 32), umma_desc(bbase + kk * 32),
-                                   (ks | kk) != 0 ? 1u : 0u);
-                        tc_commit(&a_empty[as]);
-                    }
-                    if (!ok) break;
+                    for (int kk = 0; kk < 16; ++kk)
+                        tc_mma_ts(d_tmem, a_tmem + 8 * kk,
+                                  umma_desc(bbase + (kk >> 2) * TC_KS_BYTES + (kk & 3) * 32), idesc,
+                                  kk != 0 ? 1u : 0u);
+                    tc_commit(&a_empty[bs]);
                     tc_commit(&b_empty[bs]);
                     tc_commit(&d_full[bs]);
                 }
@@ -299,22 +333,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             __syncwarp();
         } else {
             // ---------------- math warps ----------------
-            const int t = threadIdx.x;             // 0 .. 255
-            const int row = (warp & 3) * 32 + lane;  // this thread's tile row = TMEM lane (epilogue)
-            const int half = warp >> 2;              // columns 32 half .. 32 half + 31
-            // Unpacking map: 8 threads per 128-byte A row (one 16-byte chunk
-            // each); the two rows of a half-warp are 4 row groups apart, so
-            // their 64-byte source ranges fall in disjoint banks.
-            const int q = t >> 3, cq = t & 7;
-            const int rgl_u = 8 * (q >> 3) + 4 * (q & 1) + ((q >> 1) & 3);
-            float y[32];
+            const int r4 = warp & 3, h = warp >> 2;
+            const int rgl = lane;                      // row group within the tile
+            const uint32_t lane_base = static_cast<uint32_t>(r4 * 32) << 16;
+            const bool active = 64 * h < m;            // this half has pairs to finish
+            float y[64];
 #pragma unroll
-            for (int n = 0; n < 32; ++n) y[n] = 0.0f;
+            for (int n = 0; n < 64; ++n) y[n] = 0.0f;
             float dw_prev = 0.0f;
             bool ok = true;
             for (int b = 0; b <= nb && ok; ++b) {
                 float dw_cur = 0.0f;
                 if (b < nb) {
+                    const int64_t bb = nblk + b;
+                    const int as = static_cast<int>(bb & 1);
                     const int64_t rb = nraw + b / 2;
                     const int rs = static_cast<int>(rb & 1);
                     if ((b & 1) == 0 &&
@@ -322,42 +354,42 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         ok = false;
                         break;
                     }
-                    const uint8_t *raw = smem + TC_OFF_RAW + rs * TC_RAW_BYTES + (b & 1) * BLOCK_BYTES;
-                    dw_cur = block_scale(raw + (row >> 2) * TC_RAW_ROW, row & 3);
-                    for (int ks = 0; ks < 4; ++ks) {
-                        const int64_t kidx = (nblk + b) * 4 + ks;
-                        const int as = static_cast<int>(kidx & 3);
-                        if (!tc_warp_wait(&a_empty[as], static_cast<uint32_t>(((kidx >> 2) & 1) ^ 1), abort,
-                                          a.status, 8)) {
-                            ok = false;
-                            break;
-                        }
-                        // elements 64 ks .. 64 ks + 63 of a row: code bytes
-                        // 64 (ks & 1) .. + 63, low nibbles for ks < 2
-                        uint8_t *atile = smem + TC_OFF_A + as * TC_A_BYTES;
-                        const int hi = ks >> 1;
-#pragma unroll
-                        for (int it = 0; it < 4; ++it) {
-                            const int r = 4 * rgl_u + it;  // tile row
-                            const uint2 wv = *reinterpret_cast<const uint2 *>(
-                                raw + rgl_u * TC_RAW_ROW + CODE_OFS + ROW_BYTES * it + 64 * (ks & 1) + 8 * cq);
-                            const uint32_t x0 = (hi ? (wv.x >> 4) : wv.x) & 0x0f0f0f0fu;
-                            const uint32_t x1 = (hi ? (wv.y >> 4) : wv.y) & 0x0f0f0f0fu;
-                            uint4 o;
-                            o.x = nib2bf16x2(x0, 0x4140u);
-                            o.y = nib2bf16x2(x0, 0x4342u);
-                            o.z = nib2bf16x2(x1, 0x4140u);
-                            o.w = nib2bf16x2(x1, 0x4342u);
-                            *reinterpret_cast<uint4 *>(atile + (r >> 3) * 1024 + (r & 7) * 128 +
-                                                       ((cq ^ (r & 7)) << 4)) = o;
-                        }
-                        fence_proxy_async_smem();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&a_full[as]);
-                    }
-                    if (!ok) break;
+                    const uint8_t *blk = smem + TC_OFF_RAW + rs * TC_RAW_BYTES + rgl * TC_RAW_ROW + (b & 1) * BLOCK_BYTES;
+                    dw_cur = block_scale(blk, r4);
+                    const uint8_t *codes = blk + CODE_OFS + ROW_BYTES * r4 + 64 * h;
+                    uint32_t x[16];
                     if (b & 1) {
-                        __syncwarp();
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const uint4 v = *reinterpret_cast<const uint4 *>(codes + 16 * i);
+                            x[4 * i] = v.x, x[4 * i + 1] = v.y, x[4 * i + 2] = v.z, x[4 * i + 3] = v.w;
+                        }
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const uint2 v = *reinterpret_cast<const uint2 *>(codes + 8 * i);
+                            x[2 * i] = v.x, x[2 * i + 1] = v.y;
+                        }
+                    }
+                    if (!tc_warp_wait(&a_empty[as], static_cast<uint32_t>(((bb >> 1) & 1) ^ 1), abort, a.status, 8)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    {
+                        uint32_t lo[32], hi[32];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) unpack_word(x[i], lo[2 * i], lo[2 * i + 1], hi[2 * i], hi[2 * i + 1]);
+                        // element j (< 128) sits in column j / 2 of the block's A
+                        const uint32_t acol = tmem + lane_base + as * 128 + 32 * h;
+                        tc_st32(acol, lo);
+                        tc_st32(acol + 64, hi);
+                    }
+                    tc_wait_st();
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&a_full[as]);
+                    if (b & 1) {
                         if (lane == 0) mbar_arrive(&raw_empty[rs]);
                     }
                 }
@@ -367,32 +399,45 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     const int bs = static_cast<int>(bb & 1);
                     const uint32_t par = static_cast<uint32_t>((bb >> 1) & 1);
                     if (!tc_warp_wait(&d_full[bs], par, abort, a.status, 9) ||
-                        !tc_warp_wait(&da_full[bs], par, abort, a.status, 10)) {
+                        !tc_warp_wait(&sc_full[bs], par, abort, a.status, 10)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    uint32_t d[32];
-                    tc_ld32(tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + bs * TC_N + 32 * half, d);
+                    if (active) {
+                        const float *sc = reinterpret_cast<const float *>(smem + TC_OFF_SC + bs * TC_SC_BYTES) + 64 * h;
+                        const uint32_t dcol = tmem + lane_base + TC_TMEM_D + bs * TC_CHUNK + 64 * h;
+#pragma unroll
+                        for (int half = 0; half < 2; ++half) {
+                            uint32_t d[32];
+                            tc_ld32(dcol + 32 * half, d);
+                            tc_wait_ld();
+#pragma unroll
+                            for (int n4 = 0; n4 < 8; ++n4) {
+                                const float4 da = *reinterpret_cast<const float4 *>(sc + 32 * half + 4 * n4);
+                                const float dav[4] = {da.x, da.y, da.z, da.w};
+#pragma unroll
+                                for (int q = 0; q < 4; ++q) {
+                                    const int n = 32 * half + 4 * n4 + q;
+                                    y[n] = __fadd_rn(y[n], __fmul_rn(__uint_as_float(d[4 * n4 + q]), __fmul_rn(dw_prev, dav[q])));
+                                }
+                            }
+                        }
+                    }
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(&d_empty[bs]);
-                    const float *da = reinterpret_cast<const float *>(smem + TC_OFF_DA + bs * TC_DA_BYTES);
-                    const int col = (b - 1) & 3;  // the block's column in the 4-block scale box
-#pragma unroll
-                    for (int n = 0; n < 32; ++n)
-                        y[n] = __fadd_rn(y[n], __fmul_rn(__uint_as_float(d[n]),
-                                                         __fmul_rn(dw_prev, da[(32 * half + n) * 4 + col])));
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&da_empty[bs]);
+                    if (lane == 0) {
+                        mbar_arrive(&d_empty[bs]);
+                        mbar_arrive(&sc_empty[bs]);
+                    }
                 }
                 dw_prev = dw_cur;
             }
-            if (ok && rg0 + (row >> 2) < n_rg) {
-                const int64_t grow = static_cast<int64_t>(rg0) * 4 + row;
+            if (ok && active && rg0 + rgl < n_rg) {
+                const int64_t grow = static_cast<int64_t>(rg0 + rgl) * 4 + r4;
 #pragma unroll
-                for (int n = 0; n < 32; ++n)
-                    if (32 * half + n < m) J.Y[static_cast<int64_t>(pb + 32 * half + n) * J.N + grow] = y[n];
+                for (int n = 0; n < 64; ++n)
+                    if (64 * h + n < m) J.Y[static_cast<int64_t>(pb + 64 * h + n) * J.N + grow] = y[n];
             }
         }
         nraw += (nb + 1) / 2;
@@ -402,12 +447,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     // Drain: nothing asynchronous may still target this CTA's shared memory
     // or TMEM when it exits. After a normal run these waits return at once.
     if (warp == TC_MATH_WARPS && lane == 0) {
-        for (int s = 0; s < 2; ++s) {
-            if (n_rf[s] > 0) mbar_wait(&raw_full[s], static_cast<uint32_t>((n_rf[s] - 1) & 1));
-            if (n_bf[s] > 0) {
-                mbar_wait(&b_full[s], static_cast<uint32_t>((n_bf[s] - 1) & 1));
-                mbar_wait(&da_full[s], static_cast<uint32_t>((n_bf[s] - 1) & 1));
-            }
+        if (n_rf0 > 0) mbar_wait(&raw_full[0], static_cast<uint32_t>((n_rf0 - 1) & 1));
+        if (n_rf1 > 0) mbar_wait(&raw_full[1], static_cast<uint32_t>((n_rf1 - 1) & 1));
+        if (n_bf0 > 0) {
+            mbar_wait(&b_full[0], static_cast<uint32_t>((n_bf0 - 1) & 1));
+            mbar_wait(&sc_full[0], static_cast<uint32_t>((n_bf0 - 1) & 1));
+        }
+        if (n_bf1 > 0) {
+            mbar_wait(&b_full[1], static_cast<uint32_t>((n_bf1 - 1) & 1));
+            mbar_wait(&sc_full[1], static_cast<uint32_t>((n_bf1 - 1) & 1));
         }
     }
     if (warp == TC_MATH_WARPS + 1 && lane == 0) {
@@ -451,7 +499,7 @@ int tc_gemm_smem() { return TC_SMEM; }
 
 // One grouped projection pass on tensor cores: gate and up into g and u
 // (down = false), or down into o (down = true). Needs the bf16 activation
-// rows (xgb or qhb) and the padded per-pair scales (dxg or dhp).
+// rows (xgb or qhb) and the chunk-aligned scales (xs or hs).
 cudaError_t launch_tc_gemm(const GroupedArgs &a, bool down, cudaStream_t st) {
     static unsigned char set_tc[64];
     cudaError_t e = allow_max_smem(reinterpret_cast<const void *>(tc_gemm_kernel), set_tc);
@@ -459,7 +507,6 @@ cudaError_t launch_tc_gemm(const GroupedArgs &a, bool down, cudaStream_t st) {
     const int nb = down ? a.nbi : a.nbh;
     const int N = down ? a.H : a.I;
     const int K = nb * QK;
-    const int nbp = down ? a.nbip : a.nbhp;
     const uint8_t *m0 = down ? a.down : a.gate;
     const uint8_t *m1 = down ? a.down : a.up;
     // weights: one row per row group (E * N / 4 rows of nb * 520 bytes) as
@@ -467,7 +514,7 @@ cudaError_t launch_tc_gemm(const GroupedArgs &a, bool down, cudaStream_t st) {
     const uint64_t wd0 = static_cast<uint64_t>(nb) * BLOCK_BYTES / 8;
     const uint64_t wd1 = static_cast<uint64_t>(a.E) * (N / 4);
     const uint64_t wstride = static_cast<uint64_t>(nb) * BLOCK_BYTES;
-    CUtensorMap w0, w1, bm, dm;
+    CUtensorMap w0, w1, bm;
     if ((e = encode_2d(&w0, CU_TENSOR_MAP_DATA_TYPE_UINT64, m0, wd0, wd1, wstride, TC_RAW_ROW / 8, TC_RG,
                        CU_TENSOR_MAP_SWIZZLE_NONE)) != cudaSuccess)
         return e;
@@ -476,17 +523,12 @@ cudaError_t launch_tc_gemm(const GroupedArgs &a, bool down, cudaStream_t st) {
         return e;
     // activations: [P][K] bf16; boxes of 64 elements (128 bytes) x 64 pairs
     const void *act = down ? static_cast<const void *>(a.qhb) : static_cast<const void *>(a.xgb);
-    if ((e = encode_2d(&bm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, act, K, a.P, static_cast<uint64_t>(K) * 2, 64, TC_N,
+    if ((e = encode_2d(&bm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, act, K, a.P, static_cast<uint64_t>(K) * 2, 64, 64,
                        CU_TENSOR_MAP_SWIZZLE_128B)) != cudaSuccess)
-        return e;
-    // activation scales: [P][nbp] fp32; boxes of 4 blocks x 64 pairs
-    const void *da = down ? static_cast<const void *>(a.dhp) : static_cast<const void *>(a.dxg);
-    if ((e = encode_2d(&dm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, da, nbp, a.P, static_cast<uint64_t>(nbp) * 4, 4, TC_N,
-                       CU_TENSOR_MAP_SWIZZLE_NONE)) != cudaSuccess)
         return e;
     const TcJob j0{N, nb, down ? a.o : a.g};
     const TcJob j1{N, nb, down ? a.o : a.u};
-    tc_gemm_kernel<<<num_sms(), TC_THREADS, TC_SMEM, st>>>(a, j0, j1, down ? 1 : 2, w0, w1, bm, dm);
+    tc_gemm_kernel<<<num_sms(), TC_THREADS, TC_SMEM, st>>>(a, j0, j1, down ? 1 : 2, down ? a.hs : a.xs, w0, w1, bm);
     return cudaGetLastError();
 }
 
