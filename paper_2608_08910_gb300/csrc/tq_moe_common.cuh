@@ -25,6 +25,7 @@ struct MoeLayout {
     size_t chunk_expert, chunk_begin, chunk_len, n_chunks;  // grouped GEMM work list
     size_t xgb, qhb;  // bf16 [P][H], [P][I] activation rows for the tensor-core contraction (grouped only)
     size_t pair_chunk, xs, hs;  // tensor-core work list helpers (grouped only)
+    size_t rnorm;     // fp32 [T + E]: Euclidean norms of the hidden states and router rows (grouped only)
     int64_t max_chunks;
     size_t total;
 };
@@ -89,13 +90,14 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.xgb = take(2 * static_cast<size_t>(P * H));
         L.qhb = take(2 * static_cast<size_t>(P * I));
         L.pair_chunk = take(4 * static_cast<size_t>(P));
+        L.rnorm = take(4 * static_cast<size_t>(T + E));
         L.xs = take(static_cast<size_t>(L.max_chunks) * nbh * TC_CHUNK * 4);
         L.hs = take(static_cast<size_t>(L.max_chunks) * nbi * TC_CHUNK * 4);
     } else {
         L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = L.xg = SIZE_MAX;
         L.dxg = L.bxg = L.dhp = L.bhp = SIZE_MAX;
         L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
-        L.xgb = L.qhb = L.pair_chunk = L.xs = L.hs = SIZE_MAX;
+        L.xgb = L.qhb = L.pair_chunk = L.xs = L.hs = L.rnorm = SIZE_MAX;
         L.max_chunks = 0;
     }
     L.total = off;
@@ -169,6 +171,7 @@ struct GroupedArgs {
     int *pair_chunk;      // [P] chunk of each pair (tensor-core path)
     float *xs, *hs;       // [chunks][nb][TC_CHUNK]: per chunk and block, the pairs' scales da
                           // (tensor-core path)
+    float *rnorm;         // [T + E] norms for the screened router
 };
 
 // Shared-memory bytes of one quantized activation vector of nb blocks
