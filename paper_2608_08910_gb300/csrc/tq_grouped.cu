@@ -65,12 +65,15 @@ __global__ void __launch_bounds__(128) router_batch_kernel(GroupedArgs a) {
 // evaluated candidates, so the top-k selection and the softmax weights are
 // those of the exact path.
 //
-// Bound: one thread sums the H products of a logit in ascending order with
-// fused multiply-adds, so |fl(g) - g| <= gamma_H * sum_h |x_h w_h|
-// <= gamma_H * ||x|| * ||w|| (Higham, Accuracy and Stability of Numerical
-// Algorithms, section 3.1; Cauchy-Schwarz), gamma_H = H u / (1 - H u),
-// u = 2^-24. The bias add and the bound arithmetic add a few units of
-// roundoff relative to |logit|; the bound below covers them with margin.
+// Bound: the H products of a logit are summed in kScreenSplit slices, each
+// in ascending order with fused multiply-adds by one thread, and the slice
+// sums are then added in slice order: every product passes through at most
+// H / kScreenSplit + kScreenSplit - 1 <= H roundings, so
+// |fl(g) - g| <= gamma_H * sum_h |x_h w_h| <= gamma_H * ||x|| * ||w||
+// (Higham, Accuracy and Stability of Numerical Algorithms, section 3.1;
+// Cauchy-Schwarz), gamma_H = H u / (1 - H u), u = 2^-24. The bias add and
+// the bound arithmetic add a few units of roundoff relative to |logit|; the
+// bound below covers them with margin.
 constexpr int RG_T = 64, RG_E = 64, RG_BK = 32;
 
 __global__ void __launch_bounds__(256) router_norm_kernel(GroupedArgs a) {
@@ -87,109 +90,140 @@ __global__ void __launch_bounds__(256) router_norm_kernel(GroupedArgs a) {
     if (lane == 0) a.rnorm[w] = sqrtf(s);
 }
 
-// approx[t][e] = fl(sum_h x[t][h] w[e][h]), h ascending, one thread per
-// output; tiles of 64 tokens x 64 experts, 4 x 4 outputs per thread.
+// part[s][t][e] = fl(sum over slice s of x[t][h] w[e][h]), h ascending, one
+// thread per output; tiles of 64 tokens x 64 experts, 4 x 4 outputs per
+// thread, grid z = slice.
 __global__ void __launch_bounds__(256) router_gemm_kernel(GroupedArgs a) {
-    __shared__ __align__(16) float xs[RG_BK][RG_T + 4];
-    __shared__ __align__(16) float wsm[RG_BK][RG_E + 4];
+    __shared__ __align__(16) float xs[2][RG_BK][RG_T + 4];
+    __shared__ __align__(16) float wsm[2][RG_BK][RG_E + 4];
     const int e0 = blockIdx.x * RG_E, t0 = blockIdx.y * RG_T;
+    const int hs = a.H / kScreenSplit, h0 = blockIdx.z * hs;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     float acc[4][4];
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
-    for (int k0 = 0; k0 < a.H; k0 += RG_BK) {
-        for (int i = threadIdx.x; i < RG_T * RG_BK / 4; i += blockDim.x) {
-            const int r = i >> 3, c4 = i & 7;
-            float4 xv = make_float4(0.f, 0.f, 0.f, 0.f), wv = xv;
-            if (t0 + r < a.T) xv = __ldg(reinterpret_cast<const float4 *>(a.X + static_cast<int64_t>(t0 + r) * a.H + k0) + c4);
-            if (e0 + r < a.E) wv = __ldg(reinterpret_cast<const float4 *>(a.wr + static_cast<int64_t>(e0 + r) * a.H + k0) + c4);
-            xs[4 * c4][r] = xv.x, xs[4 * c4 + 1][r] = xv.y, xs[4 * c4 + 2][r] = xv.z, xs[4 * c4 + 3][r] = xv.w;
-            wsm[4 * c4][r] = wv.x, wsm[4 * c4 + 1][r] = wv.y, wsm[4 * c4 + 2][r] = wv.z, wsm[4 * c4 + 3][r] = wv.w;
+    float4 xr[2], wr[2];
+    auto fetch = [&](int k0) {
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int i = threadIdx.x + 256 * u, r = i >> 3, c4 = i & 7;
+            xr[u] = t0 + r < a.T ? __ldg(reinterpret_cast<const float4 *>(a.X + static_cast<int64_t>(t0 + r) * a.H + k0) + c4)
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+            wr[u] = e0 + r < a.E ? __ldg(reinterpret_cast<const float4 *>(a.wr + static_cast<int64_t>(e0 + r) * a.H + k0) + c4)
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        __syncthreads();
+    };
+    auto stash = [&](int buf) {
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int i = threadIdx.x + 256 * u, r = i >> 3, c4 = i & 7;
+            xs[buf][4 * c4][r] = xr[u].x, xs[buf][4 * c4 + 1][r] = xr[u].y;
+            xs[buf][4 * c4 + 2][r] = xr[u].z, xs[buf][4 * c4 + 3][r] = xr[u].w;
+            wsm[buf][4 * c4][r] = wr[u].x, wsm[buf][4 * c4 + 1][r] = wr[u].y;
+            wsm[buf][4 * c4 + 2][r] = wr[u].z, wsm[buf][4 * c4 + 3][r] = wr[u].w;
+        }
+    };
+    fetch(h0);
+    stash(0);
+    __syncthreads();
+    const int nk = hs / RG_BK;
+    for (int it = 0; it < nk; ++it) {
+        const int buf = it & 1;
+        if (it + 1 < nk) fetch(h0 + (it + 1) * RG_BK);
 #pragma unroll 8
         for (int k = 0; k < RG_BK; ++k) {
-            const float4 xv = *reinterpret_cast<const float4 *>(&xs[k][4 * ty]);
-            const float4 wv = *reinterpret_cast<const float4 *>(&wsm[k][4 * tx]);
+            const float4 xv = *reinterpret_cast<const float4 *>(&xs[buf][k][4 * ty]);
+            const float4 wv = *reinterpret_cast<const float4 *>(&wsm[buf][k][4 * tx]);
             const float xx[4] = {xv.x, xv.y, xv.z, xv.w}, ww[4] = {wv.x, wv.y, wv.z, wv.w};
 #pragma unroll
             for (int i = 0; i < 4; ++i)
 #pragma unroll
                 for (int j = 0; j < 4; ++j) acc[i][j] = __fmaf_rn(xx[i], ww[j], acc[i][j]);
         }
+        if (it + 1 < nk) stash(buf ^ 1);
         __syncthreads();
     }
+    float *part = a.rpart + static_cast<int64_t>(blockIdx.z) * a.T * a.E;
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const int t = t0 + 4 * ty + i, e = e0 + 4 * tx + j;
-            if (t < a.T && e < a.E) a.logits[static_cast<int64_t>(t) * a.E + e] = acc[i][j];
+            if (t < a.T && e < a.E) part[static_cast<int64_t>(t) * a.E + e] = acc[i][j];
         }
 }
 
-// One warp per token: bounds, the k-th largest lower bound, and the exact
-// logit of every expert whose upper bound reaches it.
-__global__ void __launch_bounds__(256) router_refine_kernel(GroupedArgs a) {
-    extern __shared__ float lower_all[];
+// One CTA per token: the slice sums and the bounds, the k-th largest lower
+// bound (warp 0), then the compensated logits of the candidates, spread over
+// the CTA's warps.
+constexpr int RF_WARPS = 4;
+
+__global__ void __launch_bounds__(RF_WARPS * 32) router_refine_kernel(GroupedArgs a) {
+    extern __shared__ float lower[];  // [E]
+    __shared__ int cand[TQFX4_MAX_EXPERTS];
+    __shared__ int n_cand;
+    __shared__ float kth_s;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int t = blockIdx.x * 8 + warp;
-    if (t >= a.T) return;
-    float *lower = lower_all + warp * a.E;
+    const int t = blockIdx.x;
     float *lg = a.logits + static_cast<int64_t>(t) * a.E;
     float *ll = a.logits_lo + static_cast<int64_t>(t) * a.E;
+    const int64_t TE = static_cast<int64_t>(a.T) * a.E;
     // gamma_H ||x|| with 1% margin for gamma's denominator and the norms' own roundoff
     const float cx = 1.01f * static_cast<float>(a.H) * 5.9604645e-8f * __ldcg(a.rnorm + t);
     auto bound = [&](int e, float v) { return cx * __ldcg(a.rnorm + a.T + e) + 4.0e-7f * fabsf(v); };
-    for (int e = lane; e < a.E; e += 32) {
-        float v = lg[e];
+    if (threadIdx.x == 0) n_cand = 0;
+    for (int e = threadIdx.x; e < a.E; e += blockDim.x) {
+        const float *p = a.rpart + static_cast<int64_t>(t) * a.E + e;
+        float v = __ldcg(p);
+#pragma unroll
+        for (int s = 1; s < kScreenSplit; ++s) v = __fadd_rn(v, __ldcg(p + s * TE));
         if (a.bias) v = __fadd_rn(v, __ldg(a.bias + e));
         lg[e] = v;
+        ll[e] = 0.0f;
         lower[e] = v - bound(e, v);
     }
-    __syncwarp();
-    // k-th largest lower bound: k rounds of a warp maximum, taking one entry per round
-    float kth = 0.0f;
-    for (int r = 0; r < a.top_k; ++r) {
-        float best = -INFINITY;
-        int bi = 0x7fffffff;
-        for (int e = lane; e < a.E; e += 32) {
-            const float v = lower[e];
-            if (v > best || (v == best && e < bi)) best = v, bi = e;
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float ob = __shfl_xor_sync(0xffffffffu, best, o);
-            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-            if (ob > best || (ob == best && oi < bi)) best = ob, bi = oi;
-        }
-        kth = best;
-        __syncwarp();
-        if (lane == 0) lower[bi] = -INFINITY;
-        __syncwarp();
-    }
-    const float *x = a.X + static_cast<int64_t>(t) * a.H;
-    for (int e0 = 0; e0 < a.E; e0 += 32) {
-        const int e = e0 + lane;
-        bool cand = false;
-        if (e < a.E) {
-            const float v = lg[e];
-            cand = v + bound(e, v) >= kth;
-            if (!cand) ll[e] = 0.0f;
-        }
-        unsigned m = __ballot_sync(0xffffffffu, cand);
-        while (m) {
-            const int c = e0 + __ffs(m) - 1;
-            m &= m - 1;
-            float hi, lo;
-            router_logit_warp(a.wr + static_cast<int64_t>(c) * a.H, x, a.H, hi, lo);
-            if (lane == 0) {
-                if (a.bias) ff_add(hi, lo, __ldg(a.bias + c), 0.0f, hi, lo);
-                lg[c] = hi;
-                ll[c] = lo;
+    __syncthreads();
+    if (warp == 0) {
+        // k-th largest lower bound: k rounds of a warp maximum, taking one entry per round
+        float kth = 0.0f;
+        for (int r = 0; r < a.top_k; ++r) {
+            float best = -INFINITY;
+            int bi = 0x7fffffff;
+            for (int e = lane; e < a.E; e += 32) {
+                const float v = lower[e];
+                if (v > best || (v == best && e < bi)) best = v, bi = e;
             }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+                const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+                if (ob > best || (ob == best && oi < bi)) best = ob, bi = oi;
+            }
+            kth = best;
+            __syncwarp();
+            if (lane == 0) lower[bi] = -INFINITY;
+            __syncwarp();
+        }
+        if (lane == 0) kth_s = kth;
+    }
+    __syncthreads();
+    const float kth = kth_s;
+    for (int e = threadIdx.x; e < a.E; e += blockDim.x) {
+        const float v = lg[e];
+        if (v + bound(e, v) >= kth) cand[atomicAdd(&n_cand, 1)] = e;
+    }
+    __syncthreads();
+    const float *x = a.X + static_cast<int64_t>(t) * a.H;
+    for (int i = warp; i < n_cand; i += RF_WARPS) {
+        const int c = cand[i];
+        float hi, lo;
+        router_logit_warp(a.wr + static_cast<int64_t>(c) * a.H, x, a.H, hi, lo);
+        if (lane == 0) {
+            if (a.bias) ff_add(hi, lo, __ldg(a.bias + c), 0.0f, hi, lo);
+            lg[c] = hi;
+            ll[c] = lo;
         }
     }
 }
@@ -858,6 +892,7 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
         a.xs = reinterpret_cast<float *>(base + L.xs);
         a.hs = reinterpret_cast<float *>(base + L.hs);
         a.rnorm = reinterpret_cast<float *>(base + L.rnorm);
+        a.rpart = reinterpret_cast<float *>(base + L.rpart);
     }
     return true;
 }
@@ -893,8 +928,8 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
     rec(0);
     if (a.T >= kScreenMinTokens) {
         router_norm_kernel<<<(a.T + a.E + 7) / 8, 256, 0, st>>>(a);
-        router_gemm_kernel<<<dim3((a.E + RG_E - 1) / RG_E, (a.T + RG_T - 1) / RG_T), 256, 0, st>>>(a);
-        router_refine_kernel<<<(a.T + 7) / 8, 256, 8 * a.E * sizeof(float), st>>>(a);
+        router_gemm_kernel<<<dim3((a.E + RG_E - 1) / RG_E, (a.T + RG_T - 1) / RG_T, kScreenSplit), 256, 0, st>>>(a);
+        router_refine_kernel<<<a.T, RF_WARPS * 32, a.E * sizeof(float), st>>>(a);
     } else {
         router_batch_kernel<<<dim3(a.E, (a.T + RB_TOK - 1) / RB_TOK), 128, 0, st>>>(a);
     }

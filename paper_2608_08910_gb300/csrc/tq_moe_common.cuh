@@ -26,6 +26,7 @@ struct MoeLayout {
     size_t xgb, qhb;  // bf16 [P][H], [P][I] activation rows for the tensor-core contraction (grouped only)
     size_t pair_chunk, xs, hs;  // tensor-core work list helpers (grouped only)
     size_t rnorm;     // fp32 [T + E]: Euclidean norms of the hidden states and router rows (grouped only)
+    size_t rpart;     // fp32 [kScreenSplit][T][E]: partial router logits of the screening GEMM (grouped only)
     int64_t max_chunks;
     size_t total;
 };
@@ -34,6 +35,8 @@ struct MoeLayout {
 constexpr int GG_TOK = 64;
 // Pairs from which the automatic path choice takes the tensor-core contraction.
 constexpr int64_t kTcMinPairs = 4096;
+// Slices of the hidden dimension the router's screening GEMM sums separately.
+constexpr int kScreenSplit = 4;
 // Pairs per chunk on the tensor-core path (the largest MMA N used).
 constexpr int TC_CHUNK = 128;
 
@@ -91,13 +94,14 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.qhb = take(2 * static_cast<size_t>(P * I));
         L.pair_chunk = take(4 * static_cast<size_t>(P));
         L.rnorm = take(4 * static_cast<size_t>(T + E));
+        L.rpart = take(4 * static_cast<size_t>(kScreenSplit) * T * E);
         L.xs = take(static_cast<size_t>(L.max_chunks) * nbh * TC_CHUNK * 4);
         L.hs = take(static_cast<size_t>(L.max_chunks) * nbi * TC_CHUNK * 4);
     } else {
         L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = L.xg = SIZE_MAX;
         L.dxg = L.bxg = L.dhp = L.bhp = SIZE_MAX;
         L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
-        L.xgb = L.qhb = L.pair_chunk = L.xs = L.hs = L.rnorm = SIZE_MAX;
+        L.xgb = L.qhb = L.pair_chunk = L.xs = L.hs = L.rnorm = L.rpart = SIZE_MAX;
         L.max_chunks = 0;
     }
     L.total = off;
@@ -172,6 +176,7 @@ struct GroupedArgs {
     float *xs, *hs;       // [chunks][nb][TC_CHUNK]: per chunk and block, the pairs' scales da
                           // (tensor-core path)
     float *rnorm;         // [T + E] norms for the screened router
+    float *rpart;         // [kScreenSplit][T][E] partial logits of the screening GEMM
 };
 
 // Shared-memory bytes of one quantized activation vector of nb blocks
