@@ -230,21 +230,25 @@ __global__ void __launch_bounds__(RF_WARPS * 32) router_refine_kernel(GroupedArg
 
 // ---------------------------------------------------------------- top-k
 
+// One warp per token: the top-k selection and its softmax weights.
 __global__ void __launch_bounds__(128) topk_batch_kernel(GroupedArgs a) {
-    __shared__ TopkScratch s;
-    const int t = blockIdx.x, lane = threadIdx.x & 31;
+    __shared__ int sel_s[4][TQFX4_MAX_TOP_K];
+    __shared__ float w_s[4][TQFX4_MAX_TOP_K];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int t = blockIdx.x * 4 + warp;
+    if (t >= a.T) return;
     const int k = a.top_k;
     const float *lh = a.logits + static_cast<int64_t>(t) * a.E;
     const float *ll = a.logits_lo + static_cast<int64_t>(t) * a.E;
-    int *sel = a.sel + static_cast<int64_t>(t) * k;
-    __shared__ float w[TQFX4_MAX_TOP_K];
-    topk_block(lh, ll, a.E, k, sel, s);
-    if (threadIdx.x >= 32) return;
-    softmax_ff_warp(lh, ll, s.res, k, w);
+    topk_warp(lh, ll, a.E, k, sel_s[warp]);
+    softmax_ff_warp(lh, ll, sel_s[warp], k, w_s[warp]);
+    __syncwarp();
     if (lane < k) {
-        a.selw[static_cast<int64_t>(t) * k + lane] = w[lane];
-        a.sel_out[static_cast<int64_t>(t) * k + lane] = s.res[lane];
-        a.selw_out[static_cast<int64_t>(t) * k + lane] = w[lane];
+        const int64_t o = static_cast<int64_t>(t) * k + lane;
+        a.sel[o] = sel_s[warp][lane];
+        a.sel_out[o] = sel_s[warp][lane];
+        a.selw[o] = w_s[warp][lane];
+        a.selw_out[o] = w_s[warp][lane];
     }
 }
 
@@ -935,7 +939,7 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
     }
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(1);
-    topk_batch_kernel<<<a.T, 128, 0, st>>>(a);
+    topk_batch_kernel<<<(a.T + 3) / 4, 128, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(2);
     group_kernel<<<1, 1024, 0, st>>>(a);

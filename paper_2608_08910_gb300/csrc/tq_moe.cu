@@ -5,7 +5,7 @@
 //   router   one CTA per expert: logit W_r[e] x + bias[e] by a compensated
 //            binary32 dot product kept as a double-binary32 pair; extra CTAs
 //            quantize x. The CTA that finishes last (one counter) selects
-//            the top-k experts.
+//            the top-k experts (one warp, registers and warp reductions).
 //   gate_up  CTA (j, p) streams row range p of selected expert j's gate and
 //            up matrices (tq_stream.cuh) and writes g_j and u_j; no CTA
 //            depends on another.
@@ -36,7 +36,7 @@ __global__ void __launch_bounds__(128) router_kernel(MoeArgs a) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     __shared__ float part_hi[4], part_lo[4];
     __shared__ int last;
-    __shared__ TopkScratch topk_s;
+    __shared__ int sel_s[TQFX4_MAX_TOP_K];
     if (static_cast<int>(blockIdx.x) >= a.E) {
         // x quantization, one warp per 256-block
         const int b = (blockIdx.x - a.E) * 4 + warp;
@@ -81,9 +81,13 @@ __global__ void __launch_bounds__(128) router_kernel(MoeArgs a) {
     __syncthreads();
     TQ_STAMP(0, 2);
     if (!last) return;
-    topk_block(a.logits, a.logits_lo, a.E, a.top_k, a.sel, topk_s);
+    if (warp == 0) topk_warp(a.logits, a.logits_lo, a.E, a.top_k, sel_s);
+    __syncthreads();
     TQ_STAMP(0, 5);
-    if (threadIdx.x < a.top_k) a.sel_out[threadIdx.x] = topk_s.res[threadIdx.x];
+    if (threadIdx.x < a.top_k) {
+        a.sel[threadIdx.x] = sel_s[threadIdx.x];
+        a.sel_out[threadIdx.x] = sel_s[threadIdx.x];
+    }
     if (threadIdx.x == 0) a.ctr[kCtrRouter] = 0;
     TQ_STAMP(0, 3);
 }
@@ -166,6 +170,7 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
     job.bss = bss;
     job.nb = nbi;
     const bool any = job.rg_begin < job.rg_end;
+    if (any) warp_stream_prefetch(ring, &job, 1, a.rpu_d, warp, a.warps_d);
     if (warp == a.warps_d - 1) {
         // the routing weights (needed by the combine at the end); the router
         // has completed, so this runs while gate/up drains
@@ -228,7 +233,6 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
             }
         }
     }
-    if (any) warp_stream_prefetch(ring, &job, 1, a.rpu_d, warp, a.warps_d);
     __syncthreads();
     TQ_STAMP(2, 3);
     if (any) warp_stream_run(ring, &job, 1, a.rpu_d, warp, a.warps_d, a.status, K_DOWN);

@@ -85,7 +85,8 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.bxg = take(4 * static_cast<size_t>(P * nbhp));
         L.dhp = take(4 * static_cast<size_t>(P * nbip));
         L.bhp = take(4 * static_cast<size_t>(P * nbip));
-        L.max_chunks = P / GG_TOK + E + 1;
+        // every chunk holds at least one pair, and an expert adds at most one partial chunk
+        L.max_chunks = (P < P / GG_TOK + E ? P : P / GG_TOK + E) + 1;
         L.chunk_expert = take(4 * static_cast<size_t>(L.max_chunks));
         L.chunk_begin = take(4 * static_cast<size_t>(L.max_chunks));
         L.chunk_len = take(4 * static_cast<size_t>(L.max_chunks));
@@ -295,93 +296,74 @@ __device__ __forceinline__ unsigned long long topk_key(float hi, float lo, int e
            static_cast<unsigned long long>(1023 - e);
 }
 
-// Shared scratch of topk_block.
-struct TopkScratch {
-    int res[TQFX4_MAX_TOP_K];  // the selection, in rank order
-    unsigned long long key[TQFX4_MAX_EXPERTS];
-    int hist[256];
-    int cand[TQFX4_MAX_EXPERTS];
-    int ncand;
-    int bin_cut;
-    unsigned int kmin, kmax;
-};
+// Top-k of E <= 32 * KPL logits (double-binary32 pairs, read through L2) by
+// one warp, descending by key, ties to the lower index. Lane l holds the keys
+// of experts l, l + 32, ... as (high, low) 32-bit words, sorted in
+// descending order in registers by a bitonic network; each of the k rounds
+// takes the largest head with two warp reductions (the high words, then the
+// low words of the lanes whose head has that high word), and the owning lane
+// shifts its list. Keys are distinct (their low bits are the expert index),
+// so exactly one lane owns the maximum. Writes the selection, in rank order,
+// to res. All lanes of the warp must call.
+template <int KPL>
+__device__ __forceinline__ void topk_warp_kpl(const float *lhi, const float *llo, int E, int k, int *res) {
+    const int lane = threadIdx.x & 31;
+    uint32_t kh[KPL], kl[KPL];  // (0, 0) is below every key
+    float h[KPL], l[KPL];
+#pragma unroll
+    for (int i = 0; i < KPL; ++i) {  // all loads in flight before the first use
+        const int e = lane + 32 * i;
+        h[i] = e < E ? __ldcg(lhi + e) : 0.0f;
+        l[i] = e < E ? __ldcg(llo + e) : 0.0f;
+    }
+#pragma unroll
+    for (int i = 0; i < KPL; ++i) {
+        const int e = lane + 32 * i;
+        const unsigned long long key = e < E ? topk_key(h[i], l[i], e) : 0ull;
+        kh[i] = static_cast<uint32_t>(key >> 32);
+        kl[i] = static_cast<uint32_t>(key);
+    }
+    // bitonic sort, descending
+#pragma unroll
+    for (int size = 2; size <= KPL; size <<= 1) {
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+#pragma unroll
+            for (int i = 0; i < KPL; ++i) {
+                const int j = i ^ stride;
+                if (j > i) {
+                    const bool desc = (i & size) == 0;
+                    const bool gt = kh[i] > kh[j] || (kh[i] == kh[j] && kl[i] > kl[j]);
+                    if (gt != desc) {
+                        const uint32_t th = kh[i], tl = kl[i];
+                        kh[i] = kh[j], kl[i] = kl[j];
+                        kh[j] = th, kl[j] = tl;
+                    }
+                }
+            }
+        }
+    }
+    for (int r = 0; r < k; ++r) {
+        const uint32_t mh = __reduce_max_sync(0xffffffffu, kh[0]);
+        const uint32_t ml = __reduce_max_sync(0xffffffffu, kh[0] == mh ? kl[0] : 0u);
+        if (kh[0] == mh && kl[0] == ml) {
+#pragma unroll
+            for (int i = 0; i + 1 < KPL; ++i) kh[i] = kh[i + 1], kl[i] = kl[i + 1];
+            kh[KPL - 1] = kl[KPL - 1] = 0u;
+        }
+        if (lane == 0) res[r] = 1023 - static_cast<int>(ml & 1023u);
+    }
+    __syncwarp();
+}
 
-// Top-k of E <= 1024 logits (double-binary32 pairs, read through L2) by the
-// whole thread block, in descending order with ties to the lower index:
-// (1) the keys' hi parts are binned linearly between their minimum and
-// maximum into 256 bins; (2) the highest bin b* whose suffix count reaches k
-// is found; (3) only the experts in bins >= b* (normally a few more than k)
-// are ranked exactly by comparing full keys. Leaves the selection in s.res
-// (shared) and writes it to sel (global). All threads must call.
-__device__ __forceinline__ void topk_block(const float *lhi, const float *llo, int E, int k, int *sel,
-                                           TopkScratch &s) {
-    const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31;
-    if (tid == 0) {
-        s.kmin = 0xffffffffu;
-        s.kmax = 0u;
-        s.ncand = 0;
-    }
-    for (int i = tid; i < 256; i += nt) s.hist[i] = 0;
-    __syncthreads();
-    unsigned int lmin = 0xffffffffu, lmax = 0u;
-    for (int e = tid; e < E; e += nt) {
-        const unsigned long long key = topk_key(__ldcg(lhi + e), __ldcg(llo + e), e);
-        s.key[e] = key;
-        const unsigned int h = static_cast<unsigned int>(key >> 32);
-        lmin = min(lmin, h);
-        lmax = max(lmax, h);
-    }
-    lmin = __reduce_min_sync(0xffffffffu, lmin);
-    lmax = __reduce_max_sync(0xffffffffu, lmax);
-    if (lane == 0) {
-        atomicMin(&s.kmin, lmin);
-        atomicMax(&s.kmax, lmax);
-    }
-    __syncthreads();
-    const unsigned int kmin = s.kmin, span = s.kmax - s.kmin;
-    const int shift = span == 0u ? 0 : max(0, 24 - __clz(span));  // (span >> shift) < 256
-    for (int e = tid; e < E; e += nt)
-        atomicAdd(&s.hist[(static_cast<unsigned int>(s.key[e] >> 32) - kmin) >> shift], 1);
-    __syncthreads();
-    if (tid < 32) {
-        // suffix sums over the 256 bins, 8 per lane (lane 31 holds the top bins)
-        int c[8], tot = 0;
-#pragma unroll
-        for (int i = 7; i >= 0; --i) {
-            tot += s.hist[lane * 8 + i];
-            c[i] = tot;  // count of bins lane*8+i .. lane*8+7
-        }
-        // inclusive suffix scan of the lane totals; `above` counts higher lanes
-        int v = tot;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int t = __shfl_down_sync(0xffffffffu, v, o);
-            if (lane + o < 32) v += t;
-        }
-        const int above = v - tot;
-        int cut = -1;
-#pragma unroll
-        for (int i = 7; i >= 0; --i)
-            if (cut < 0 && above + c[i] >= k) cut = lane * 8 + i;
-        const int best = __reduce_max_sync(0xffffffffu, cut);
-        if (lane == 0) s.bin_cut = best < 0 ? 0 : best;
-    }
-    __syncthreads();
-    const int cut = s.bin_cut;
-    for (int e = tid; e < E; e += nt)
-        if (static_cast<int>((static_cast<unsigned int>(s.key[e] >> 32) - kmin) >> shift) >= cut)
-            s.cand[atomicAdd(&s.ncand, 1)] = e;
-    __syncthreads();
-    const int nc = s.ncand;
-    for (int ci = tid; ci < nc; ci += nt) {
-        const int e = s.cand[ci];
-        const unsigned long long ke = s.key[e];
-        int r = 0;
-        for (int cj = 0; cj < nc; ++cj) r += s.key[s.cand[cj]] > ke;
-        if (r < k) s.res[r] = e;
-    }
-    __syncthreads();
-    if (tid < k) sel[tid] = s.res[tid];
+// topk_warp_kpl with the register capacity chosen for E (<= 1024).
+__device__ __forceinline__ void topk_warp(const float *lhi, const float *llo, int E, int k, int *res) {
+    if (E <= 256)
+        topk_warp_kpl<8>(lhi, llo, E, k, res);
+    else if (E <= 512)
+        topk_warp_kpl<16>(lhi, llo, E, k, res);
+    else
+        topk_warp_kpl<32>(lhi, llo, E, k, res);
 }
 
 // ---- double-binary32 softmax ----------------------------------------------------

@@ -72,7 +72,9 @@ def run_and_check(layer, seed, X, zipf_bias=None, check_stages=True):
 
 
 @pytest.mark.parametrize("E,H,I,k,zipf", [(16, 512, 768, 4, 0.0), (8, 256, 256, 8, 0.0), (32, 1024, 512, 6, 1.1),
-                                          (1, 256, 512, 1, 0.0), (64, 2048, 1280, 8, 0.0)])
+                                          (1, 256, 512, 1, 0.0), (64, 2048, 1280, 8, 0.0),
+                                          (300, 256, 256, 16, 0.5),    # 16 keys per lane in the top-k, k at its maximum
+                                          (1024, 256, 256, 12, 1.1)])  # 32 keys per lane, the largest expert count
 def test_moe_ffn_small_shapes(E, H, I, k, zipf):
     seed = E * 7 + H + I
     layer = MoeLayer.synthetic(seed, E, H, I, k, zipf, DEV)
