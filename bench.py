@@ -47,6 +47,25 @@ def _peaks():
         return 6800.0, "fallback"
 
 
+# DRAM bytes (read + write) of one gate_up_kernel launch, from an ncu --set full capture of the
+# 64-expert layer (one launch reads the 8 selected experts whatever the expert count). Set to None
+# when the kernel changes until it is captured again.
+GATE_UP_TRAFFIC = 68207360 + 1805056
+# The same for one tc_gemm_kernel gate/up launch of the 2048-token prefill: an ncu capture at 64
+# experts and 512 tokens (one chunk per expert, as in the full workload) scaled by the full
+# workload's 4x weight bytes and pairs.
+TC_GATE_UP_TRAFFIC = 4 * (579433728 + 58311680)
+
+
+def _tensor_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops_sustained"]), "measured (MEASURED_PEAKS.json bf16_tflops_sustained)"
+    except Exception:
+        return 1700.0, "fallback 1.7 PFLOP/s sustained"
+
+
 def bytes_per_token():
     from paper_2608_08910_gb300 import binding as B
     mb = B.tqfx4_matrix_bytes(I, H)  # gate = up = down size
@@ -120,7 +139,7 @@ def cpu_baseline(seconds_budget=20.0, tokens=None):
     X = inputs.hidden_states(SEED, POOL, H, dev).cpu().numpy()
     per_token, _, _ = bytes_per_token()
     total_t, done = 0.0, 0
-    n_max = tokens if tokens else 64
+    n_max = tokens if tokens else POOL
     for t in range(n_max):
         _, idx, _ = oracle.router(Wr, None, X[t], TOPK)
         ex = {int(e): tuple(oracle.pack_rtn(inputs.expert_matrix(SEED, int(e), p, H, I, dev).cpu().numpy())
@@ -201,6 +220,8 @@ def run_grouped(args, rank, world, local):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     T, zipf, path = (64, 1.1, B.TQFX4_PATH_DECODE) if args.workload == "grouped_decode_64" else \
         (2048, 0.0, B.TQFX4_PATH_PREFILL)
+    if args.tokens:
+        T = args.tokens
     dev = torch.device("cuda", local)
     layer = MoeLayer.synthetic(SEED, E, H, I, TOPK, zipf, dev)
     ws = layer.workspace(T, path)
@@ -254,6 +275,48 @@ def run_grouped(args, rank, world, local):
     stage_s = {names[s]: acc[s] / reps for s in range(n_st)}
     peak_hbm, peak_kind = _peaks()
     flops_gu = 2.0 * T * TOPK * 2 * I * H
+    # end to end through the public API: the batch's hidden states copied in
+    # from pinned host memory and the outputs and expert ids copied back
+    Xh = [x.cpu().pin_memory() for x in Xs]
+    xin = torch.empty((T, H), device=dev)
+    outh = torch.empty((T, H), pin_memory=True)
+    selh = torch.empty((T, TOPK), dtype=torch.int32, pin_memory=True)
+    for i in range(2):
+        xin.copy_(Xh[i % n_batches], non_blocking=True)
+        layer.grouped(xin, ws, path, OUT, sel, selw, stream=stream)
+        outh.copy_(OUT, non_blocking=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for i in range(args.steps):
+        xin.copy_(Xh[i % n_batches], non_blocking=True)
+        layer.grouped(xin, ws, path, OUT, sel, selw, stream=stream)
+        outh.copy_(OUT, non_blocking=True)
+        selh.copy_(sel, non_blocking=True)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
+    te = ev0.elapsed_time(ev1) / 1e3
+    if world > 1:
+        tt = torch.tensor([te], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        te = float(tt.item())
+    if path == B.TQFX4_PATH_PREFILL:
+        # the dominant kernel is the tensor-core contraction of gate and up:
+        # dense-equivalent flops over its time, against the measured bf16 peak
+        peak_tc, tc_kind = _tensor_peak()
+        achieved = flops_gu / stage_s["gate_up"] / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peak_tc, "unit": "TFLOP/s",
+                "frac": achieved / peak_tc, "kernel": "tc_gemm_kernel (gate_up)",
+                "traffic": TC_GATE_UP_TRAFFIC if (T == 2048 and E == 256) else None,
+                "traffic_source": "ncu capture at 64 experts / 512 tokens, scaled x4",
+                "peak_source": tc_kind}
+    else:
+        gu_bytes = touched / n_batches * 2 * mb
+        achieved = gu_bytes / stage_s["gate_up"] / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peak_hbm, "unit": "GB/s",
+                "frac": achieved / peak_hbm, "traffic": None, "kernel": "grouped_gemm_kernel (gate_up)",
+                "peak_source": peak_kind}
+    roof["stage_us"] = {k: v * 1e6 for k, v in stage_s.items()}
     line = {
         "metric": "MoE-layer tokens/s (%s)" % args.workload, "value": tokens / t, "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3,
@@ -263,12 +326,12 @@ def run_grouped(args, rank, world, local):
                    "zipf": zipf, "touched_experts_avg": touched / n_batches,
                    "l2": "inputs larger than L2 (3.27 GB expert pool); 4 batches cycled"},
         "effective_gbs": bytes_per_step * args.steps * world / t / 1e9,
-        "roofline": {"bound": "hbm", "achieved": bytes_per_step / (t / args.steps) / 1e9, "peak": peak_hbm,
-                     "unit": "GB/s", "frac": bytes_per_step / (t / args.steps) / 1e9 / peak_hbm,
-                     "traffic": None, "kernel": "whole step",
-                     "gate_up_tflops": flops_gu / stage_s["gate_up"] / 1e12,
-                     "stage_us": {k: v * 1e6 for k, v in stage_s.items()}},
-        "gpu_launches": 10 * args.steps,
+        "roofline": roof,
+        "e2e": {"value": tokens / te, "unit": "tokens/s", "h2d_bytes_per_step": T * H * 4,
+                "d2h_bytes_per_step": T * H * 4 + T * TOPK * 4},
+        # router (screening GEMM, norms and refinement from 256 tokens, else one kernel), top-k, group,
+        # quantize, gather, gate/up, SwiGLU, down, combine
+        "gpu_launches": ((3 if T >= 256 else 1) + 8) * args.steps,
         "clocks": clk.summary(),
     }
     if rank == 0:
@@ -284,11 +347,16 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--experts", type=int, default=E,
+                    help="routed experts in the layer (default 256; smaller only for profiling captures)")
+    ap.add_argument("--tokens", type=int, default=0,
+                    help="tokens per step of the grouped workloads (default: 64 or 2048; profiling only)")
     ap.add_argument("--workload", default="moe_decode",
                     choices=["moe_decode", "grouped_decode_64", "prefill_2048"],
                     help="moe_decode (default): 1 token; grouped_decode_64: 64 tokens with Zipf(1.1) "
                          "routing; prefill_2048: 2048 tokens")
     args = ap.parse_args()
+    globals()["E"] = args.experts
 
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -431,7 +499,8 @@ def main():
         "tokens_per_s": tokens / t,
         "pct_of_hbm_peak": 100.0 * value / peak,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": None, "kernel": dom,
+                     "frac": achieved / peak, "traffic": GATE_UP_TRAFFIC, "kernel": dom,
+                     "traffic_source": "ncu capture (dram__bytes_read + write) of one gate_up_kernel launch",
                      "peak_source": peak_kind + " (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
                      else "fallback 6.8 TB/s",
                      "stage_us": {k: v * 1e6 for k, v in stage_s.items()}},
