@@ -220,9 +220,11 @@ __device__ __forceinline__ void router_logit_block(const float *w, const float *
     const float4 *x4 = reinterpret_cast<const float4 *>(x);
     float s[4] = {0.f, 0.f, 0.f, 0.f}, c[4] = {0.f, 0.f, 0.f, 0.f};
     const int n4 = H >> 2;
+    // the router is read by every call: keep it in L2 ahead of the streamed experts
+    const uint64_t pol = l2_policy_evict_last();
 #pragma unroll 8
     for (int i = threadIdx.x; i < n4; i += 128) {
-        const float4 wv = __ldg(w4 + i), xv = __ldg(x4 + i);
+        const float4 wv = ldg_f4_hint(w4 + i, pol), xv = __ldg(x4 + i);
         const float ww[4] = {wv.x, wv.y, wv.z, wv.w}, xx[4] = {xv.x, xv.y, xv.z, xv.w};
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
@@ -477,9 +479,11 @@ __device__ __forceinline__ void stage_ranges(int lane, int n, uint8_t *const dst
     }
     if (lane == 0) {
         mbar_arrive_expect_tx(bar, total);
+        // weight blocks are read once per call: evict-first keeps L2 for reused data
+        const uint64_t pol = l2_policy_evict_first();
 #pragma unroll
         for (int p = 0; p < 2; ++p)
-            if (p < n && body[p]) bulk_g2s(dst[p] + ofs[p] + head[p], src[p] + head[p], body[p], bar);
+            if (p < n && body[p]) bulk_g2s_hint(dst[p] + ofs[p] + head[p], src[p] + head[p], body[p], bar, pol);
     }
 #pragma unroll
     for (int p = 0; p < 2; ++p) {
