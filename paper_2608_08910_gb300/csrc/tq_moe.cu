@@ -6,15 +6,17 @@
 //            binary32 dot product kept as a double-binary32 pair; extra CTAs
 //            quantize x. The CTA that finishes last (one counter) selects
 //            the top-k experts (one warp, registers and warp reductions).
-//   gate_up  CTA (j, p) streams row range p of selected expert j's gate and
-//            up matrices (tq_stream.cuh) and writes g_j and u_j; no CTA
-//            depends on another.
+//   gate_up  the CTAs stream the units (row-group ranges) of the selected
+//            experts' gate and up matrices (tq_stream.cuh) and write g_j and
+//            u_j.
 //   down     CTA (j, p) issues its first weight copies (the selection is
 //            known), then forms h_j = silu(g_j) u_j and quantizes it into
 //            shared memory while one warp evaluates the softmax weights,
 //            streams row range p of down_j and writes o_j. The last of the
 //            top_k CTAs sharing row range p (one counter per range) combines
 //            out = sum_j w_j o_j in rank order.
+// gate/up hands out three quarters of its units statically and the rest
+// through a shared counter, so that its CTAs finish together.
 // gate_up and down are launched as programmatic dependents: each starts its
 // prologue while its predecessor drains and waits (griddepcontrol.wait)
 // before reading what the predecessor wrote.
@@ -25,9 +27,13 @@
 
 namespace tq {
 
-// Counter slots at the start of the workspace's counter area.
-constexpr int kCtrRouter = 0;  // router CTAs done
-constexpr int kCtrDown = 1;    // down: one counter per row range
+// Counter slots at the start of the workspace's counter area (all but the
+// first are zeroed by the router at every call).
+constexpr int kCtrRouter = 0;   // router CTAs done
+constexpr int kCtrZero = 1;     // first slot the router zeroes at every call
+constexpr int kCtrGateUp = 1;   // gate/up: shared unit counter
+constexpr int kCtrDown = 2;     // down: one counter per row range
+constexpr int kMaxStages = 2;   // ring depth of the gate/up kernel
 
 // ---------------------------------------------------------------- router
 
@@ -59,7 +65,7 @@ __global__ void __launch_bounds__(128) router_kernel(MoeArgs a) {
     grid_dependents_launch();  // let the gate/up kernel's CTAs get resident early
     const int e = blockIdx.x;
     if (e == 0)  // the down kernel's counters start every call at zero
-        for (int i = threadIdx.x; i < a.n_ctr - kCtrDown; i += blockDim.x) a.ctr[kCtrDown + i] = 0;
+        for (int i = threadIdx.x; i < a.n_ctr - kCtrZero; i += blockDim.x) a.ctr[kCtrZero + i] = 0;
     float hi, lo;
     router_logit_block(a.wr + static_cast<int64_t>(e) * a.H, a.x, a.H, hi, lo);
     TQ_STAMP(0, 1);
@@ -94,11 +100,15 @@ __global__ void __launch_bounds__(128) router_kernel(MoeArgs a) {
 
 // ---------------------------------------------------------------- gate/up
 
+// Work of gate_up: the units (rpu_gu row groups) of every selected expert's
+// gate and up matrices, numbered u = (j * 2 + q) * upm + r. Each CTA streams
+// a static contiguous share, then takes units from one shared counter.
 __global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     TQ_STAMP(1, 0);
     const int warp = threadIdx.x >> 5;
     const int nbh = a.nbh;
+    __shared__ int sel_s[TQFX4_MAX_TOP_K];
     uint8_t *qs = smem;
     float *das = reinterpret_cast<float *>(qs + nbh * QS_STRIDE);
     int *bss = reinterpret_cast<int *>(das + nbh);
@@ -110,32 +120,40 @@ __global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
     grid_dependency_wait();  // the router's selection and quantized x
     TQ_STAMP(1, 1);
     grid_dependents_launch();
-    const int j = blockIdx.x / a.parts_gu, p = blockIdx.x - j * a.parts_gu;
     // issue the activation loads first: weight copies issued before them
     // would queue ahead in the memory system
     ActRegs act;
     act_load(a.qx, a.dx, a.bx, nbh, act);
-    const int64_t e = __ldcg(a.sel + j);
+    if (threadIdx.x < a.top_k) sel_s[threadIdx.x] = __ldcg(a.sel + threadIdx.x);
+    __syncthreads();
     const int64_t n_rg = a.I / 4;
-    MatJob jobs[2];
-    for (int q = 0; q < 2; ++q) {
-        MatJob &J = jobs[q];
-        J.mat = (q == 0 ? a.gate : a.up) + e * a.mb_gu;
-        J.rg_begin = part_begin(n_rg, a.rpu_gu, a.parts_gu, p);
-        J.rg_end = part_begin(n_rg, a.rpu_gu, a.parts_gu, p + 1);
-        J.y = (q == 0 ? a.g : a.u) + static_cast<int64_t>(j) * a.I;
-        J.s_out = nullptr;
-        J.qs = qs;
-        J.das = das;
-        J.bss = bss;
-        J.nb = nbh;
-    }
-    const bool any = jobs[0].rg_begin < jobs[0].rg_end;
-    if (any) warp_stream_prefetch(ring, jobs, 2, a.rpu_gu, warp, a.warps_gu);
+    const int64_t upm = (n_rg + a.rpu_gu - 1) / a.rpu_gu;
+    const int64_t total = static_cast<int64_t>(a.top_k) * 2 * upm;
+    UnitQueue q;
+    q.next = static_cast<int64_t>(blockIdx.x) * a.static_gu + warp;
+    q.end = static_cast<int64_t>(blockIdx.x + 1) * a.static_gu;
+    q.step = a.warps_gu;
+    q.dyn_ctr = a.ctr + kCtrGateUp;
+    q.dyn_base = static_cast<int64_t>(gridDim.x) * a.static_gu;
+    q.total = total;
+    auto map = [&](int64_t u) {
+        const int j = static_cast<int>(u / (2 * upm));
+        const int64_t rem = u - static_cast<int64_t>(j) * 2 * upm;
+        const int qq = rem >= upm;
+        const int64_t r = rem - qq * upm;
+        UnitRef U;
+        U.mat = (qq ? a.up : a.gate) + static_cast<int64_t>(sel_s[j]) * a.mb_gu;
+        U.rg0 = r * a.rpu_gu;
+        U.rgs = static_cast<int>(imin64(a.rpu_gu, n_rg - U.rg0));
+        U.y = (qq ? a.u : a.g) + static_cast<int64_t>(j) * a.I;
+        return U;
+    };
+    int64_t slot_u[kMaxStages];
+    warp_units_prefetch(ring, q, nbh, map, slot_u);
     act_store(act, nbh, qs, das, bss);
     __syncthreads();
     TQ_STAMP(1, 2);
-    if (any) warp_stream_run(ring, jobs, 2, a.rpu_gu, warp, a.warps_gu, a.status, K_GATEUP);
+    warp_units_run(ring, q, nbh, qs, das, bss, map, [](int64_t) {}, slot_u, a.status, K_GATEUP);
     TQ_STAMP(1, 3);
 }
 
@@ -335,6 +353,10 @@ bool moe_decode_args(const tqfx4_experts *ex, const tqfx4_router *rt, void *ws, 
     a.warps_d = fit_warps(a.slot_d, a.rpu_d, a.nbi, act_bytes(a.nbi), 8);
     a.parts_d = static_cast<int>(imax64(1, sms / a.top_k));
 
+    // gate/up's static share: three quarters of the units, split evenly; the
+    // rest is handed out by the shared counter
+    const int64_t upm_gu = (a.I / 4 + a.rpu_gu - 1) / a.rpu_gu;
+    a.static_gu = static_cast<int>((static_cast<int64_t>(a.top_k) * 2 * upm_gu * 3 / 4) / (a.top_k * a.parts_gu));
     return static_cast<int64_t>(a.n_ctr) >= kCtrDown + a.parts_d;
 }
 

@@ -134,9 +134,9 @@ struct MoeArgs {
     float *dh;
     int *bh;
     float *o;
-    // gate/up geometry: top_k x parts_gu CTAs, each a range of row groups
-    int rpu_gu, slot_gu, stages_gu, warps_gu, parts_gu;
-    // down geometry
+    // gate/up geometry: top_k x parts_gu CTAs; static_gu units per CTA before the shared counter
+    int rpu_gu, slot_gu, stages_gu, warps_gu, parts_gu, static_gu;
+    // down geometry: top_k x parts_d CTAs, each a range of row groups
     int rpu_d, slot_d, stages_d, warps_d, parts_d;
 };
 

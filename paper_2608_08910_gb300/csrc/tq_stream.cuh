@@ -175,3 +175,130 @@ __device__ __forceinline__ bool warp_stream_run(const WarpRing &r, const MatJob 
 }
 
 }  // namespace tq
+
+namespace tq {
+
+// ---- units handed out partly statically, partly by a shared counter ----
+//
+// A warp first takes its static units (first, first + step, ... < end), then
+// units dyn_base + atomicAdd(dyn_ctr, 1) while they are below total. The
+// static share lets every warp prefetch before anything is known about its
+// peers; the shared tail lets the CTAs that stream faster take more, so that
+// all finish together.
+struct UnitQueue {
+    int64_t next, end, step;  // remaining static units of this warp
+    int *dyn_ctr;
+    int64_t dyn_base, total;
+
+    // The warp's next unit, or -1 (warp-uniform; lane 0 takes dynamic units).
+    __device__ __forceinline__ int64_t take() {
+        if (next < end) {
+            const int64_t u = next;
+            next += step;
+            return u;
+        }
+        int v = 0;
+        if ((threadIdx.x & 31) == 0) v = atomicAdd(dyn_ctr, 1);
+        v = __shfl_sync(0xffffffffu, v, 0);
+        const int64_t u = dyn_base + v;
+        return u < total ? u : -1;
+    }
+};
+
+// A unit of streamed work: rgs row groups of a matrix starting at row group
+// rg0, results to y (indexed by matrix row).
+struct UnitRef {
+    const uint8_t *mat;
+    int64_t rg0;
+    int rgs;
+    float *y;
+};
+
+// Prefetch the first ring.stages units of the queue into the ring; the unit
+// ids go to slot_u (register array of the caller). `map(u)` gives the
+// UnitRef of unit u (matrix pointer and rows only are used here).
+template <int MAXST, class Map>
+__device__ __forceinline__ void warp_units_prefetch(const WarpRing &r, UnitQueue &q, int nb, Map map,
+                                                    int64_t (&slot_u)[MAXST]) {
+    const int64_t stripe = static_cast<int64_t>(nb) * BLOCK_BYTES;
+#pragma unroll
+    for (int s = 0; s < MAXST; ++s) {
+        slot_u[s] = -1;
+        if (s >= r.stages) continue;
+        slot_u[s] = q.take();
+        if (slot_u[s] < 0) continue;
+        const UnitRef U = map(slot_u[s]);
+        uint8_t *dst[2] = {r.slots + s * r.slot_bytes, nullptr};
+        const uint8_t *src[2] = {U.mat + U.rg0 * stripe, nullptr};
+        const uint32_t bytes[2] = {static_cast<uint32_t>(U.rgs * stripe), 0u};
+        uint32_t ofs[2];
+        stage_ranges(threadIdx.x & 31, 1, dst, src, bytes, &r.bars[s], ofs);
+    }
+}
+
+// Consume the prefetched units and the rest of the queue, refilling each
+// slot as it frees; after a unit's rows are written, done(u) runs on the
+// whole warp. Activations: qs / das / bss in shared memory. Returns false
+// if a copy never arrived (status recorded).
+template <int MAXST, class Map, class Done>
+__device__ __forceinline__ bool warp_units_run(const WarpRing &r, UnitQueue &q, int nb, const uint8_t *qs,
+                                               const float *das, const int *bss, Map map, Done done,
+                                               int64_t (&slot_u)[MAXST], int *status, int kernel_id) {
+    const int lane = threadIdx.x & 31;
+    const int64_t stripe = static_cast<int64_t>(nb) * BLOCK_BYTES;
+    for (int it = 0;; ++it) {
+        const int slot = it % r.stages;
+        int64_t u = -1;
+#pragma unroll
+        for (int s = 0; s < MAXST; ++s)
+            if (s == slot) u = slot_u[s];
+        if (u < 0) break;
+        const uint32_t parity = static_cast<uint32_t>((it / r.stages) & 1);
+        if (!__all_sync(0xffffffffu, mbar_wait(&r.bars[slot], parity))) {
+            if (lane == 0) report(status, TQFX4_ETIMEOUT, kernel_id, static_cast<int>(u));
+            return false;
+        }
+        __syncwarp();
+        const UnitRef U = map(u);
+        const uint8_t *data = r.slots + slot * r.slot_bytes + src_ofs(U.mat + U.rg0 * stripe);
+        const int nblk = U.rgs * nb;
+        for (int i = lane; i < nblk; i += 32) {
+            const int rgl = i / nb, b = i - rgl * nb;
+            const uint8_t *blk = data + i * BLOCK_BYTES;
+            int S[4];
+            block_dot(blk + CODE_OFS, qs + b * QS_STRIDE, bss[b], S);
+            const float da = das[b];
+#pragma unroll
+            for (int rr = 0; rr < 4; ++rr) {
+                const float sc = __fmul_rn(block_scale(blk, rr), da);
+                r.tbuf[(rgl * 4 + rr) * (nb + 1) + b] = __fmul_rn(static_cast<float>(S[rr]), sc);
+            }
+        }
+        __syncwarp();
+        for (int t = lane; t < U.rgs * 4; t += 32) {
+            const float *tb = r.tbuf + t * (nb + 1);
+            float acc = 0.0f;
+            for (int b = 0; b < nb; ++b) acc = __fadd_rn(acc, tb[b]);
+            U.y[U.rg0 * 4 + t] = acc;
+        }
+        __syncwarp();
+        // refill this slot before the callback, so the copy is in flight meanwhile
+        const int64_t nu = q.take();
+#pragma unroll
+        for (int s = 0; s < MAXST; ++s)
+            if (s == slot) slot_u[s] = nu;
+        if (nu >= 0) {
+            fence_proxy_async_smem();
+            const UnitRef N = map(nu);
+            uint8_t *dst[2] = {r.slots + slot * r.slot_bytes, nullptr};
+            const uint8_t *src[2] = {N.mat + N.rg0 * stripe, nullptr};
+            const uint32_t bytes[2] = {static_cast<uint32_t>(N.rgs * stripe), 0u};
+            uint32_t ofs[2];
+            stage_ranges(lane, 1, dst, src, bytes, &r.bars[slot], ofs);
+        }
+        done(u);
+    }
+    return true;
+}
+
+}  // namespace tq
