@@ -57,6 +57,23 @@ GATE_UP_TRAFFIC = None
 TC_GATE_UP_TRAFFIC = 4 * (579433728 + 58311680)
 
 
+def max_over_ranks(t, world, device):
+    """The job's time: the largest of the ranks' times (the job ends with its
+    slowest replica). All ranks must call it when world > 1."""
+    if world <= 1:
+        return t
+    import torch
+    import torch.distributed as dist
+    tt = torch.tensor([float(t)], device=device, dtype=torch.float64)
+    dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+    return float(tt.item())
+
+
+def job_rate(units_per_rank, world, t):
+    """Whole-job throughput: the units all ranks processed over the job's time."""
+    return units_per_rank * world / t
+
+
 def _tensor_peak():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -254,11 +271,8 @@ def run_grouped(args, rank, world, local):
             dist.barrier()
     B.tqfx4_check(ws)
     t = ev0.elapsed_time(ev1) / 1e3
-    if world > 1:
-        tt = torch.tensor([t], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t = float(tt.item())
-    tokens = T * args.steps * world
+    t = max_over_ranks(t, world, dev)
+    tokens = T * args.steps * world  # tokens of the whole job
     # per-stage device times (CUDA events on the launching stream)
     n_st = B.tqfx4_moe_stage_count(1, path)
     names = [B.tqfx4_moe_stage_name(1, path, s) for s in range(n_st)]
@@ -296,10 +310,7 @@ def run_grouped(args, rank, world, local):
     torch.cuda.synchronize()
     B.tqfx4_check(ws)
     te = ev0.elapsed_time(ev1) / 1e3
-    if world > 1:
-        tt = torch.tensor([te], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        te = float(tt.item())
+    te = max_over_ranks(te, world, dev)
     if path == B.TQFX4_PATH_PREFILL:
         # the dominant kernel is the tensor-core contraction of gate and up:
         # dense-equivalent flops over its time, against the measured bf16 peak
@@ -318,7 +329,8 @@ def run_grouped(args, rank, world, local):
                 "peak_source": peak_kind}
     roof["stage_us"] = {k: v * 1e6 for k, v in stage_s.items()}
     line = {
-        "metric": "MoE-layer tokens/s (%s)" % args.workload, "value": tokens / t, "unit": "tokens/s",
+        "metric": "MoE-layer tokens/s (%s)" % args.workload, "value": job_rate(T * args.steps, world, t),
+        "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "i8xi4-i32,f32",
         "data": "synthetic",
@@ -427,12 +439,9 @@ def main():
             dist.barrier()
     B.tqfx4_check(ws)
     t = ev0.elapsed_time(ev1) / 1e3
-    if world > 1:
-        tt = torch.tensor([t], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t = float(tt.item())
-    tokens = args.steps * world
-    value = per_token * tokens / t / 1e9
+    t = max_over_ranks(t, world, dev)
+    tokens = args.steps * world  # tokens of the whole job
+    value = job_rate(per_token * args.steps, world, t) / 1e9
 
     # ---- dominant kernel: CUDA events around every stage of every step, on
     # the launching stream (a second graph of the same K steps; the stage
@@ -482,10 +491,7 @@ def main():
     torch.cuda.synchronize()
     B.tqfx4_check(ws)
     te = ev0.elapsed_time(ev1) / 1e3
-    if world > 1:
-        tt = torch.tensor([te], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        te = float(tt.item())
+    te = max_over_ranks(te, world, dev)
     e2e = per_token * tokens / te / 1e9
 
     line = {
