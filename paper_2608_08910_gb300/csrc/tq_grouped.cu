@@ -24,7 +24,6 @@
 // copies (one box of weight blocks, four swizzled boxes of pair-ordered
 // activations); four consumer warps each own 8 row groups (32 rows).
 #include <cuda.h>
-#include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
 #include "tq_launch.h"
@@ -648,16 +647,32 @@ __global__ void __launch_bounds__((GG_CW + 1) * 32, 1)
     }
 }
 
-// Eight int8 values as eight bf16 values (exact: |q| <= 127 needs 7 bits).
-__device__ __forceinline__ uint4 i8x8_to_bf16x8(uint2 v) {
+// e4m3 byte of a small integer v, |v| <= 8 (exact: at most 4 significant
+// bits): 1 -> 0x38 (2^0), 2 -> 0x40, 3 -> 0x44, ..., 8 -> 0x50.
+__device__ __forceinline__ uint32_t e4m3_small(int v) {
+    const int a = v < 0 ? -v : v;
+    if (a == 0) return 0u;
+    const int e = 31 - __clz(a);
+    const uint32_t m = static_cast<uint32_t>((a << 3 >> e) - 8);
+    return (v < 0 ? 0x80u : 0u) | (static_cast<uint32_t>(e + 7) << 3) | m;
+}
+
+// Eight int8 activations q as the two e4m3 planes of q = 16 h + l, with
+// h = floor((q + 8) / 16) in -8..8 and l in -8..7: bytes of 16 h and of l.
+__device__ __forceinline__ void q_planes8(uint2 v, uint2 &hi, uint2 &lo) {
     const int8_t *b = reinterpret_cast<const int8_t *>(&v);
-    uint32_t w[4];
+    uint32_t hw[2] = {0u, 0u}, lw[2] = {0u, 0u};
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const __nv_bfloat162 h = __floats2bfloat162_rn(static_cast<float>(b[2 * i]), static_cast<float>(b[2 * i + 1]));
-        w[i] = *reinterpret_cast<const uint32_t *>(&h);
+    for (int i = 0; i < 8; ++i) {
+        const int q = b[i];
+        const int h = (q + 8) >> 4;  // arithmetic shift: floor
+        const int l = q - 16 * h;
+        const uint32_t hb = h ? e4m3_small(h) + 0x20u : 0u;  // 16 h: four more in the exponent
+        hw[i >> 2] |= hb << (8 * (i & 3));
+        lw[i >> 2] |= e4m3_small(l) << (8 * (i & 3));
     }
-    return make_uint4(w[0], w[1], w[2], w[3]);
+    hi = make_uint2(hw[0], hw[1]);
+    lo = make_uint2(lw[0], lw[1]);
 }
 
 // Gather the quantized hidden state of each pair's token into pair order.
@@ -673,25 +688,39 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(GroupedArgs a) {
     }
 }
 
-// Tensor-core path: per chunk, the bf16 rows of its pairs' quantized hidden
-// states, and per block the pairs' scales da in the chunk-aligned layout
-// the contraction stages with one bulk copy.
+// Tensor-core path: per chunk, its pairs' quantized hidden states as the two
+// e4m3 planes, and per block the pairs' scales da and -4 bsum (as float) in
+// the chunk-aligned layout the contraction stages with one bulk copy.
 __global__ void __launch_bounds__(256) gather_tc_kernel(GroupedArgs a) {
     const int c = blockIdx.x;
     if (c >= __ldcg(a.n_chunks)) return;
     const int pb = __ldcg(a.chunk_begin + c), m = __ldcg(a.chunk_len + c);
+    const int64_t plane = static_cast<int64_t>(a.P) * a.H;
     for (int n = threadIdx.x >> 5; n < m; n += blockDim.x >> 5) {
         const int64_t pos = pb + n;
         const int64_t t = __ldcg(a.pair_token + pos);
         const uint2 *src = reinterpret_cast<const uint2 *>(a.qx + t * a.H);
-        uint4 *dst = reinterpret_cast<uint4 *>(a.xgb + pos * a.H);
-        for (int i = threadIdx.x & 31; i < a.H / 8; i += 32) dst[i] = i8x8_to_bf16x8(__ldcg(src + i));
+        uint2 *dh = reinterpret_cast<uint2 *>(a.xq + pos * a.H);
+        uint2 *dl = reinterpret_cast<uint2 *>(a.xq + plane + pos * a.H);
+        for (int i = threadIdx.x & 31; i < a.H / 8; i += 32) {
+            uint2 hi, lo;
+            q_planes8(__ldcg(src + i), hi, lo);
+            dh[i] = hi;
+            dl[i] = lo;
+        }
         if ((threadIdx.x & 31) == 0) a.pair_chunk[pos] = c;
     }
     for (int i = threadIdx.x; i < a.nbh * TC_CHUNK; i += blockDim.x) {
         const int b = i / TC_CHUNK, n = i - b * TC_CHUNK;
-        const float d = n < m ? __ldcg(a.dx + __ldcg(a.pair_token + pb + n) * static_cast<int64_t>(a.nbh) + b) : 0.0f;
-        a.xs[(static_cast<int64_t>(c) * a.nbh + b) * TC_CHUNK + n] = d;
+        float d = 0.0f, nb4 = 0.0f;
+        if (n < m) {
+            const int64_t t = __ldcg(a.pair_token + pb + n);
+            d = __ldcg(a.dx + t * a.nbh + b);
+            nb4 = static_cast<float>(-4 * __ldcg(a.bx + t * a.nbh + b));
+        }
+        float *o = a.xs + (static_cast<int64_t>(c) * a.nbh + b) * 2 * TC_CHUNK;
+        o[n] = d;
+        o[TC_CHUNK + n] = nb4;
     }
 }
 
@@ -719,11 +748,16 @@ __global__ void __launch_bounds__(256) swiglu_quant_kernel(GroupedArgs a) {
     const bool ok = quant_block_warp(hv, packed, d, sum);
     *reinterpret_cast<uint2 *>(a.qh + o) = packed;
     if (a.tc) {
-        *reinterpret_cast<uint4 *>(a.qhb + o) = i8x8_to_bf16x8(packed);
+        uint2 hi, lo;
+        q_planes8(packed, hi, lo);
+        *reinterpret_cast<uint2 *>(a.hq + o) = hi;
+        *reinterpret_cast<uint2 *>(a.hq + static_cast<int64_t>(a.P) * a.I + o) = lo;
         if (lane == 0) {
             const int c = __ldcg(a.pair_chunk + p);
             const int n = static_cast<int>(p - __ldcg(a.chunk_begin + c));
-            a.hs[(static_cast<int64_t>(c) * a.nbi + b) * TC_CHUNK + n] = d;
+            float *hs = a.hs + (static_cast<int64_t>(c) * a.nbi + b) * 2 * TC_CHUNK;
+            hs[n] = d;
+            hs[TC_CHUNK + n] = static_cast<float>(-4 * sum);
         }
     }
     if (a.keep_h) {
@@ -890,8 +924,8 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
         a.chunk_begin = reinterpret_cast<int *>(base + L.chunk_begin);
         a.chunk_len = reinterpret_cast<int *>(base + L.chunk_len);
         a.n_chunks = reinterpret_cast<int *>(base + L.n_chunks);
-        a.xgb = reinterpret_cast<uint16_t *>(base + L.xgb);
-        a.qhb = reinterpret_cast<uint16_t *>(base + L.qhb);
+        a.xq = base + L.xq;
+        a.hq = base + L.hq;
         a.pair_chunk = reinterpret_cast<int *>(base + L.pair_chunk);
         a.xs = reinterpret_cast<float *>(base + L.xs);
         a.hs = reinterpret_cast<float *>(base + L.hs);

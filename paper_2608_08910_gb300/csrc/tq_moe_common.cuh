@@ -23,7 +23,7 @@ struct MoeLayout {
     size_t xg;  // int8 [P][H] (grouped only)
     size_t dxg, bxg, dhp, bhp;  // [P][round4(nb)] (grouped only)
     size_t chunk_expert, chunk_begin, chunk_len, n_chunks;  // grouped GEMM work list
-    size_t xgb, qhb;  // bf16 [P][H], [P][I] activation rows for the tensor-core contraction (grouped only)
+    size_t xq, hq;    // e4m3 activation planes [2][P][H], [2][P][I] for the tensor-core contraction (grouped only)
     size_t pair_chunk, xs, hs;  // tensor-core work list helpers (grouped only)
     size_t rnorm;     // fp32 [T + E]: Euclidean norms of the hidden states and router rows (grouped only)
     size_t rpart;     // fp32 [kScreenSplit][T][E]: partial router logits of the screening GEMM (grouped only)
@@ -91,18 +91,18 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.chunk_begin = take(4 * static_cast<size_t>(L.max_chunks));
         L.chunk_len = take(4 * static_cast<size_t>(L.max_chunks));
         L.n_chunks = take(4);
-        L.xgb = take(2 * static_cast<size_t>(P * H));
-        L.qhb = take(2 * static_cast<size_t>(P * I));
+        L.xq = take(2 * static_cast<size_t>(P * H));
+        L.hq = take(2 * static_cast<size_t>(P * I));
         L.pair_chunk = take(4 * static_cast<size_t>(P));
         L.rnorm = take(4 * static_cast<size_t>(T + E));
         L.rpart = take(4 * static_cast<size_t>(kScreenSplit) * T * E);
-        L.xs = take(static_cast<size_t>(L.max_chunks) * nbh * TC_CHUNK * 4);
-        L.hs = take(static_cast<size_t>(L.max_chunks) * nbi * TC_CHUNK * 4);
+        L.xs = take(static_cast<size_t>(L.max_chunks) * nbh * 2 * TC_CHUNK * 4);
+        L.hs = take(static_cast<size_t>(L.max_chunks) * nbi * 2 * TC_CHUNK * 4);
     } else {
         L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = L.xg = SIZE_MAX;
         L.dxg = L.bxg = L.dhp = L.bhp = SIZE_MAX;
         L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
-        L.xgb = L.qhb = L.pair_chunk = L.xs = L.hs = L.rnorm = L.rpart = SIZE_MAX;
+        L.xq = L.hq = L.pair_chunk = L.xs = L.hs = L.rnorm = L.rpart = SIZE_MAX;
         L.max_chunks = 0;
     }
     L.total = off;
@@ -172,10 +172,10 @@ struct GroupedArgs {
     int tc;               // contraction on tcgen05 tensor cores
     int chunk;            // pairs per chunk of the work list (GG_TOK, or TC_CHUNK on tensor cores)
     int max_chunks;       // capacity of the work list
-    uint16_t *xgb, *qhb;  // bf16 copies of xg [P][H] and qh [P][I] (tensor-core path)
+    uint8_t *xq, *hq;     // [2][P][H], [2][P][I]: e4m3 planes 16 h and l of q = 16 h + l (tensor-core path)
     int *pair_chunk;      // [P] chunk of each pair (tensor-core path)
-    float *xs, *hs;       // [chunks][nb][TC_CHUNK]: per chunk and block, the pairs' scales da
-                          // (tensor-core path)
+    float *xs, *hs;       // [chunks][nb][2][TC_CHUNK]: per chunk and block, the pairs' scales da,
+                          // then -4 bsum as float (tensor-core path)
     float *rnorm;         // [T + E] norms for the screened router
     float *rpart;         // [kScreenSplit][T][E] partial logits of the screening GEMM
 };

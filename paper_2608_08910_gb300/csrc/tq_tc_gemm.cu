@@ -4,19 +4,26 @@
 // that expert.
 //
 // tcgen05.mma has no integer kind on sm_103a, so the integer block sums
-// S = sum_j c_j q_j (Eq. 5) are formed with kind::f16 on bf16 operands that
-// hold small integers exactly: the codes c in -4..4 (A) and the int8
-// activations q (B). Every product is an exact integer and |S| < 2^17, so
-// the fp32 accumulator of one 256-element block holds S exactly. (Operands
-// with an offset, such as 128 + u, make the block sums reach 2^22, and
-// there the tensor core's sums are no longer exact: the codes are centred.)
+// S = sum_j c_j q_j (Eq. 5) are formed with kind::f8f6f4 on e4m3 operands
+// that hold small dyadic numbers exactly:
+//   A  the nibble u = c + 4 (0..8) as the e4m3 byte 0x0u, which is exactly
+//      u * 2^-9 (subnormals, and 0x08 = 2^-6), so unpacking a 32-bit word of
+//      codes is one mask (four low nibbles) or a shift and a mask (four high
+//      nibbles);
+//   B  q = 16 h + l with h = floor((q + 8) / 16) in -8..8 and l in -8..7, as
+//      two e4m3 planes 16 h and l (both exact).
+// Each 256-element block takes 8 K-steps of 32 x 2 planes, accumulated in
+// fp32: every product is a multiple of 2^-9 below 2 in magnitude and the
+// block sum D = 2^-9 sum u q stays below 2^9, so the accumulator holds it
+// exactly (checked against exact integer sums at the extremes); the
+// epilogue recovers S = 512 D - 4 bsum with one exact fused multiply-add.
 // The accumulator restarts at every block and the epilogue applies the
 // fixed float schedule y = y + float(S) * (d * da) block by block, the same
 // operations in the same order as the streaming kernels and the oracle.
 //
 // Operands: A (the unpacked weights) is written by the math warps straight
 // into tensor memory with tcgen05.st (thread = row = TMEM lane), so it never
-// passes through shared memory; B (bf16 activation rows of the chunk) is
+// passes through shared memory; B (the activation planes of the chunk) is
 // staged by TMA in the 128-byte swizzled K-major layout.
 // Tile rows are ordered r4-major (tile row = 32 * r4 + row group), so that a
 // warp (one TMEM lane quadrant) reads the codes of one row of 32 row groups,
@@ -27,18 +34,19 @@
 // Warp roles (320 threads, one CTA per SM):
 //   warps 0-7  math. Warp w serves TMEM lanes 32 (w % 4) .. + 31 (rows with
 //              r4 = w % 4) and half h = w / 4: it unpacks code bytes
-//              64 h .. 64 h + 63 of its rows (elements 64 h + j and
+//              64 h .. 64 h + 63 of its rows (elements 64 h + j, then
 //              128 + 64 h + j) into A, and in the epilogue, one block behind,
 //              reads accumulator columns (pairs) 64 h .. 64 h + 63;
 //   warp 8     producer: TMA copies of the raw weight blocks (one box per two
-//              blocks of the tile), of the activation tiles (64-element x
+//              blocks of the tile), of the activation planes (128-element x
 //              64-pair boxes) and a bulk copy of the chunk's block scales;
 //   warp 9     TMEM allocation; one thread issues the MMAs (M = 128,
-//              N = the chunk's pairs rounded up to 16, K = 16; 16 per block)
-//              and the commits.
-// TMEM: A in columns [0, 256) (two blocks), accumulators in [256, 512).
-// The epilogue uses scalar fp32 multiplies and adds: the packed f32x2 forms
-// were measured to give results that differ from them.
+//              N = the chunk's pairs rounded up to 16, K = 32; 16 per block,
+//              the first 8 as soon as the low nibbles are in place) and the
+//              commits.
+// TMEM: A in columns [0, 128) (two blocks of 64), accumulators in [256, 512).
+// The epilogue uses scalar fp32 operations: the packed f32x2 forms were
+// measured to give results that differ from them.
 // Every wait is bounded. On a timeout the CTA records the error, all roles
 // leave their loops, the producer waits (bounded) for its copies in flight,
 // the MMA thread for its MMAs, and TMEM is freed before the CTA exits.
@@ -58,29 +66,30 @@ constexpr int TC_MATH_WARPS = 8;
 constexpr int TC_THREADS = (TC_MATH_WARPS + 2) * 32;
 constexpr int TC_RAW_ROW = 2 * BLOCK_BYTES;    // two blocks of one row group: 1040 bytes
 constexpr int TC_RAW_BYTES = 33 * 1024;        // 32 x 1040 bytes, padded
-constexpr int TC_BOX_BYTES = 64 * 128;         // one 64-element x 64-pair bf16 box: 8 KB
-constexpr int TC_KS_BYTES = 2 * TC_BOX_BYTES;  // one k-stage (64 elements) of up to 128 pairs
-constexpr int TC_B_BYTES = 4 * TC_KS_BYTES;    // one block of B: 64 KB
-constexpr int TC_SC_BYTES = TC_CHUNK * 4;      // da of the chunk's pairs: 512 bytes
+constexpr int TC_BOX_BYTES = 64 * 128;         // one 128-element x 64-pair e4m3 box: 8 KB
+constexpr int TC_PLANE_BYTES = 2 * TC_BOX_BYTES;  // one k-stage (128 elements) of one plane, <= 128 pairs
+constexpr int TC_KS_BYTES = 2 * TC_PLANE_BYTES;   // one k-stage of both planes
+constexpr int TC_B_BYTES = 2 * TC_KS_BYTES;    // one block of B: 64 KB
+constexpr int TC_SC_BYTES = 2 * TC_CHUNK * 4;  // da and -4 bsum of the chunk's pairs: 1 KB
 constexpr int TC_OFF_RAW = 0;
 constexpr int TC_OFF_B = TC_OFF_RAW + 2 * TC_RAW_BYTES;
 constexpr int TC_OFF_SC = TC_OFF_B + 2 * TC_B_BYTES;
 constexpr int TC_OFF_BAR = TC_OFF_SC + 2 * TC_SC_BYTES;
-constexpr int TC_NBAR = 21;  // barriers; the TMEM address and abort flag follow
+constexpr int TC_NBAR = 23;  // barriers; the TMEM address and abort flag follow
 constexpr int TC_SMEM = TC_OFF_BAR + TC_NBAR * 8 + 16 + 1024;  // + alignment slack
 constexpr int TC_TMEM_COLS = 512;
 constexpr uint32_t TC_TMEM_D = 256;            // first accumulator column
+constexpr int TC_A_COLS = 64;                  // TMEM columns of one block of A (256 bytes per row)
 
 static_assert(TC_OFF_B % 1024 == 0, "swizzled tiles need 1024-byte alignment");
 static_assert(TC_RG * TC_RAW_ROW <= TC_RAW_BYTES, "raw stage too small");
 static_assert(TC_CHUNK == 128, "two 64-pair boxes and two 64-column epilogue halves");
 
-// Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1),
-// A and B bf16 (bits 7-9 = 1, 10-12 = 1), both K-major (bits 15, 16 = 0),
+// Instruction descriptor of tcgen05.mma kind::f8f6f4: D fp32 (bits 4-5 = 1),
+// A and B e4m3 (bits 7-9 = 0, 10-12 = 0), both K-major (bits 15, 16 = 0),
 // N >> 3 at bits 17-22, M >> 4 at bits 24-28.
 __device__ __forceinline__ uint32_t tc_idesc(int n) {
-    return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
-           (static_cast<uint32_t>(TC_ROWS >> 4) << 24);
+    return (1u << 4) | (static_cast<uint32_t>(n >> 3) << 17) | (static_cast<uint32_t>(TC_ROWS >> 4) << 24);
 }
 
 // Shared-memory matrix descriptor of a K-major operand in the 128-byte
@@ -100,7 +109,7 @@ __device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint
                                           uint32_t accumulate) {
     asm volatile(
         "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
         "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
@@ -136,6 +145,14 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, uint32_t (&r)[32]) {
 }
 __device__ __forceinline__ void tc_st32(uint32_t taddr, const uint32_t (&r)[32]) {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%32], " TC_LIST32 ";" ::TC_R32(r), "r"(taddr) : "memory");
+}
+__device__ __forceinline__ void tc_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%16], "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15};" ::"r"(r[0]),
+        "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]),
+        "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(taddr)
+        : "memory");
 }
 __device__ __forceinline__ void tc_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
@@ -178,33 +195,12 @@ __device__ __forceinline__ bool tc_warp_wait(uint64_t *bar, uint32_t parity, int
     return ok;
 }
 
-// Two nibbles u0, u1 (the bytes of x that `sel` picks, next to the byte
-// 0x43) as bf16x2 of c = u - 4: the bytes [u0, 0x43, u1, 0x43] are the bf16
-// values 128 + u, and adding -132 (bf16 0xC304) to each half is exact.
-__device__ __forceinline__ uint32_t nib_pair(uint32_t x, uint32_t sel) {
-    uint32_t w, r;
-    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(w) : "r"(x), "r"(0x43434343u), "r"(sel));
-    asm("add.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(w), "r"(0xC304C304u));
-    return r;
-}
-
-// One 32-bit word of code bytes (4 bytes of one row) -> four A columns:
-// lo0, lo1 = elements j .. j+3 (low nibbles), hi0, hi1 = elements
-// 128 + j .. 131 + j (high nibbles).
-__device__ __forceinline__ void unpack_word(uint32_t x, uint32_t &lo0, uint32_t &lo1, uint32_t &hi0, uint32_t &hi1) {
-    const uint32_t l = x & 0x0f0f0f0fu, h = (x >> 4) & 0x0f0f0f0fu;
-    lo0 = nib_pair(l, 0x5140u);
-    lo1 = nib_pair(l, 0x5342u);
-    hi0 = nib_pair(h, 0x5140u);
-    hi1 = nib_pair(h, 0x5342u);
-}
-
 }  // namespace
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
     tc_gemm_kernel(GroupedArgs a, TcJob j0, TcJob j1, int njobs, const float *__restrict__ scales,
                    const __grid_constant__ CUtensorMap wmap0, const __grid_constant__ CUtensorMap wmap1,
-                   const __grid_constant__ CUtensorMap bmap) {
+                   const __grid_constant__ CUtensorMap bmap_hi, const __grid_constant__ CUtensorMap bmap_lo) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -214,7 +210,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     uint64_t *b_full = bars + 8, *b_empty = bars + 10;
     uint64_t *sc_full = bars + 12, *sc_empty = bars + 14;
     uint64_t *d_full = bars + 16, *d_empty = bars + 18;
-    uint64_t *fin = bars + 20;  // MMA drain at exit
+    uint64_t *fin = bars + 20;        // MMA drain at exit
+    uint64_t *a_full_hi = bars + 21;  // [2]: elements 128..255 of the block in A (a_full: 0..127)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + TC_NBAR);
     int *abort = reinterpret_cast<int *>(tmem_slot + 1);
 
@@ -223,6 +220,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             mbar_init(&raw_full[i], 1);
             mbar_init(&raw_empty[i], TC_MATH_WARPS);
             mbar_init(&a_full[i], TC_MATH_WARPS);
+            mbar_init(&a_full_hi[i], TC_MATH_WARPS);
             mbar_init(&a_empty[i], 1);
             mbar_init(&b_full[i], 1);
             mbar_init(&b_empty[i], 1);
@@ -277,7 +275,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             // ---------------- producer ----------------
             if (lane == 0) {
                 const CUtensorMap *wmap = second ? &wmap1 : &wmap0;
-                const float *sc = scales + static_cast<int64_t>(chunk) * nb * TC_CHUNK;
+                const float *sc = scales + static_cast<int64_t>(chunk) * nb * (2 * TC_CHUNK);
                 for (int b = 0; b < nb; ++b) {
                     const int64_t bb = nblk + b;
                     if ((b & 1) == 0) {
@@ -294,13 +292,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     const uint32_t par = static_cast<uint32_t>(((bb >> 1) & 1) ^ 1);
                     if (!tc_wait(&b_empty[bs], par, abort, a.status, 2)) break;
                     mbar_arrive_expect_tx(&b_full[bs], 4 * nbox * TC_BOX_BYTES);
-                    for (int ks = 0; ks < 4; ++ks)
-                        for (int x = 0; x < nbox; ++x)
-                            tma_2d(smem + TC_OFF_B + bs * TC_B_BYTES + ks * TC_KS_BYTES + x * TC_BOX_BYTES, &bmap,
-                                   b * QK + ks * 64, pb + 64 * x, &b_full[bs]);
+                    for (int ks = 0; ks < 2; ++ks)
+                        for (int pl = 0; pl < 2; ++pl)
+                            for (int x = 0; x < nbox; ++x)
+                                tma_2d(smem + TC_OFF_B + bs * TC_B_BYTES + ks * TC_KS_BYTES + pl * TC_PLANE_BYTES +
+                                           x * TC_BOX_BYTES,
+                                       pl ? &bmap_lo : &bmap_hi, b * QK + ks * 128, pb + 64 * x, &b_full[bs]);
                     if (!tc_wait(&sc_empty[bs], par, abort, a.status, 3)) break;
                     mbar_arrive_expect_tx(&sc_full[bs], TC_SC_BYTES);
-                    bulk_g2s(smem + TC_OFF_SC + bs * TC_SC_BYTES, sc + b * TC_CHUNK, TC_SC_BYTES, &sc_full[bs]);
+                    bulk_g2s(smem + TC_OFF_SC + bs * TC_SC_BYTES, sc + b * (2 * TC_CHUNK), TC_SC_BYTES, &sc_full[bs]);
                     if (bs) ++n_bf1; else ++n_bf0;
                 }
             }
@@ -309,22 +309,37 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             // ---------------- MMA issuer ----------------
             if (lane == 0) {
                 const uint32_t idesc = tc_idesc(nmma);
+                // B descriptors: stage 0, k-step 0, plane 0; the others differ by
+                // constant byte offsets (>> 4) in the start-address field
+                const uint64_t bdesc0 = umma_desc(smem_u32(smem + TC_OFF_B));
                 for (int b = 0; b < nb; ++b) {
                     const int64_t bb = nblk + b;
                     const int bs = static_cast<int>(bb & 1);
                     const uint32_t par = static_cast<uint32_t>((bb >> 1) & 1);
                     if (!tc_wait(&d_empty[bs], par ^ 1, abort, a.status, 4)) break;
                     if (!tc_wait(&b_full[bs], par, abort, a.status, 5)) break;
-                    if (!tc_wait(&a_full[bs], par, abort, a.status, 6)) break;
-                    tc_fence_after();
                     const uint32_t d_tmem = tmem + TC_TMEM_D + bs * TC_CHUNK;
-                    const uint32_t a_tmem = tmem + bs * 128;
-                    const uint32_t bbase = smem_u32(smem + TC_OFF_B + bs * TC_B_BYTES);
+                    const uint32_t a_tmem = tmem + bs * TC_A_COLS;
+                    const uint64_t bd = bdesc0 + static_cast<uint64_t>((bs * TC_B_BYTES) >> 4);
+                    bool ok = true;
 #pragma unroll
-                    for (int kk = 0; kk < 16; ++kk)
-                        tc_mma_ts(d_tmem, a_tmem + 8 * kk,
-                                  umma_desc(bbase + (kk >> 2) * TC_KS_BYTES + (kk & 3) * 32), idesc,
-                                  kk != 0 ? 1u : 0u);
+                    for (int half = 0; half < 2; ++half) {
+                        if (!tc_wait(half ? &a_full_hi[bs] : &a_full[bs], par, abort, a.status, half ? 11 : 6)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+#pragma unroll
+                        for (int k4 = 0; k4 < 4; ++k4) {
+                            const int kk = 4 * half + k4;  // 32-element step: A columns 8 kk .. 8 kk + 7
+#pragma unroll
+                            for (int pl = 0; pl < 2; ++pl)
+                                tc_mma_ts(d_tmem, a_tmem + 8 * kk,
+                                          bd + ((half * TC_KS_BYTES + pl * TC_PLANE_BYTES + k4 * 32) >> 4), idesc,
+                                          (kk | pl) != 0 ? 1u : 0u);
+                        }
+                    }
+                    if (!ok) break;
                     tc_commit(&a_empty[bs]);
                     tc_commit(&b_empty[bs]);
                     tc_commit(&d_full[bs]);
@@ -376,19 +391,31 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         break;
                     }
                     tc_fence_after();
+                    // A columns: element j (< 128) is byte j % 4 of column j / 4;
+                    // element 128 + j of column 32 + j / 4. A code word of bytes
+                    // 64 h + 4 i .. + 3 gives column 16 h + i (its low nibbles)
+                    // and column 32 + 16 h + i (its high nibbles).
+                    const uint32_t acol = tmem + lane_base + as * TC_A_COLS + 16 * h;
                     {
-                        uint32_t lo[32], hi[32];
+                        uint32_t lo[16];
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) unpack_word(x[i], lo[2 * i], lo[2 * i + 1], hi[2 * i], hi[2 * i + 1]);
-                        // element j (< 128) sits in column j / 2 of the block's A
-                        const uint32_t acol = tmem + lane_base + as * 128 + 32 * h;
-                        tc_st32(acol, lo);
-                        tc_st32(acol + 64, hi);
+                        for (int i = 0; i < 16; ++i) lo[i] = x[i] & 0x0f0f0f0fu;
+                        tc_st16(acol, lo);
+                    }
+                    {
+                        uint32_t hi[16];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) hi[i] = (x[i] >> 4) & 0x0f0f0f0fu;
+                        tc_wait_st();
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&a_full[as]);
+                        tc_st16(acol + 32, hi);
                     }
                     tc_wait_st();
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(&a_full[as]);
+                    if (lane == 0) mbar_arrive(&a_full_hi[as]);
                     if (b & 1) {
                         if (lane == 0) mbar_arrive(&raw_empty[rs]);
                     }
@@ -415,11 +442,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 #pragma unroll
                             for (int n4 = 0; n4 < 8; ++n4) {
                                 const float4 da = *reinterpret_cast<const float4 *>(sc + 32 * half + 4 * n4);
-                                const float dav[4] = {da.x, da.y, da.z, da.w};
+                                const float4 bi = *reinterpret_cast<const float4 *>(sc + TC_CHUNK + 32 * half + 4 * n4);
+                                const float dav[4] = {da.x, da.y, da.z, da.w}, biv[4] = {bi.x, bi.y, bi.z, bi.w};
 #pragma unroll
                                 for (int q = 0; q < 4; ++q) {
                                     const int n = 32 * half + 4 * n4 + q;
-                                    y[n] = __fadd_rn(y[n], __fmul_rn(__uint_as_float(d[4 * n4 + q]), __fmul_rn(dw_prev, dav[q])));
+                                    // S = 512 D - 4 bsum, exact (integers below 2^18)
+                                    const float S = __fmaf_rn(512.0f, __uint_as_float(d[4 * n4 + q]), biv[q]);
+                                    y[n] = __fadd_rn(y[n], __fmul_rn(S, __fmul_rn(dw_prev, dav[q])));
                                 }
                             }
                         }
@@ -498,8 +528,8 @@ cudaError_t encode_2d(CUtensorMap *m, CUtensorMapDataType dt, const void *base, 
 int tc_gemm_smem() { return TC_SMEM; }
 
 // One grouped projection pass on tensor cores: gate and up into g and u
-// (down = false), or down into o (down = true). Needs the bf16 activation
-// rows (xgb or qhb) and the chunk-aligned scales (xs or hs).
+// (down = false), or down into o (down = true). Needs the e4m3 activation
+// planes (xq or hq) and the chunk-aligned scales (xs or hs).
 cudaError_t launch_tc_gemm(const GroupedArgs &a, bool down, cudaStream_t st) {
     static unsigned char set_tc[64];
     cudaError_t e = allow_max_smem(reinterpret_cast<const void *>(tc_gemm_kernel), set_tc);
@@ -514,21 +544,27 @@ cudaError_t launch_tc_gemm(const GroupedArgs &a, bool down, cudaStream_t st) {
     const uint64_t wd0 = static_cast<uint64_t>(nb) * BLOCK_BYTES / 8;
     const uint64_t wd1 = static_cast<uint64_t>(a.E) * (N / 4);
     const uint64_t wstride = static_cast<uint64_t>(nb) * BLOCK_BYTES;
-    CUtensorMap w0, w1, bm;
+    CUtensorMap w0, w1, bh, bl;
     if ((e = encode_2d(&w0, CU_TENSOR_MAP_DATA_TYPE_UINT64, m0, wd0, wd1, wstride, TC_RAW_ROW / 8, TC_RG,
                        CU_TENSOR_MAP_SWIZZLE_NONE)) != cudaSuccess)
         return e;
     if ((e = encode_2d(&w1, CU_TENSOR_MAP_DATA_TYPE_UINT64, m1, wd0, wd1, wstride, TC_RAW_ROW / 8, TC_RG,
                        CU_TENSOR_MAP_SWIZZLE_NONE)) != cudaSuccess)
         return e;
-    // activations: [P][K] bf16; boxes of 64 elements (128 bytes) x 64 pairs
-    const void *act = down ? static_cast<const void *>(a.qhb) : static_cast<const void *>(a.xgb);
-    if ((e = encode_2d(&bm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, act, K, a.P, static_cast<uint64_t>(K) * 2, 64, 64,
+    // activation planes: [P][K] bytes each (16 h, then l, as e4m3); boxes of
+    // 128 elements x 64 pairs, 128-byte swizzled
+    const uint8_t *act = down ? a.hq : a.xq;
+    const int64_t plane = static_cast<int64_t>(a.P) * K;
+    if ((e = encode_2d(&bh, CU_TENSOR_MAP_DATA_TYPE_UINT8, act, K, a.P, static_cast<uint64_t>(K), 128, 64,
+                       CU_TENSOR_MAP_SWIZZLE_128B)) != cudaSuccess)
+        return e;
+    if ((e = encode_2d(&bl, CU_TENSOR_MAP_DATA_TYPE_UINT8, act + plane, K, a.P, static_cast<uint64_t>(K), 128, 64,
                        CU_TENSOR_MAP_SWIZZLE_128B)) != cudaSuccess)
         return e;
     const TcJob j0{N, nb, down ? a.o : a.g};
     const TcJob j1{N, nb, down ? a.o : a.u};
-    tc_gemm_kernel<<<num_sms(), TC_THREADS, TC_SMEM, st>>>(a, j0, j1, down ? 1 : 2, down ? a.hs : a.xs, w0, w1, bm);
+    tc_gemm_kernel<<<num_sms(), TC_THREADS, TC_SMEM, st>>>(a, j0, j1, down ? 1 : 2, down ? a.hs : a.xs, w0, w1, bh,
+                                                           bl);
     return cudaGetLastError();
 }
 
