@@ -32,11 +32,14 @@
 // two-way.
 //
 // Warp roles (320 threads, one CTA per SM):
-//   warps 0-7  math. Warp w serves TMEM lanes 32 (w % 4) .. + 31 (rows with
-//              r4 = w % 4) and half h = w / 4: it unpacks code bytes
-//              64 h .. 64 h + 63 of its rows (elements 64 h + j, then
-//              128 + 64 h + j) into A, and in the epilogue, one block behind,
-//              reads accumulator columns (pairs) 64 h .. 64 h + 63;
+//   warps 0-3  unpacking. Warp w serves TMEM lanes 32 w .. + 31 (rows with
+//              r4 = w) and writes their codes into A, up to two blocks ahead
+//              of the MMAs;
+//   warps 4-7  epilogue. Warp w serves TMEM lanes 32 (w - 4) .. + 31: per
+//              block it reads the accumulator and the running output y
+//              (kept in TMEM), adds float(S) * (d * da) and writes y back,
+//              trailing the MMAs by up to two blocks; at the end of the
+//              item it stores y;
 //   warp 8     producer: TMA copies of the raw weight blocks (one box per two
 //              blocks of the tile), of the activation planes (128-element x
 //              64-pair boxes) and a bulk copy of the chunk's block scales;
@@ -44,7 +47,8 @@
 //              N = the chunk's pairs rounded up to 16, K = 32; 16 per block,
 //              the first 8 as soon as the low nibbles are in place) and the
 //              commits.
-// TMEM: A in columns [0, 128) (two blocks of 64), accumulators in [256, 512).
+// TMEM: A in columns [0, 128) (two blocks of 64), y in [128, 256),
+// accumulators in [256, 512).
 // The epilogue uses scalar fp32 operations: the packed f32x2 forms were
 // measured to give results that differ from them.
 // Every wait is bounded. On a timeout the CTA records the error, all roles
@@ -62,7 +66,9 @@ namespace {
 
 constexpr int TC_ROWS = 128;                   // weight rows per tile = TMEM lanes
 constexpr int TC_RG = TC_ROWS / 4;             // row groups per tile
-constexpr int TC_MATH_WARPS = 8;
+constexpr int TC_MATH_WARPS = 8;              // warps 0-3 unpack A, warps 4-7 run the epilogue
+constexpr int TC_CONV_WARPS = 4, TC_EPI_WARPS = 4;
+constexpr int TC_SC_STAGES = 4;                // scale ring: runs ahead of the epilogue
 constexpr int TC_THREADS = (TC_MATH_WARPS + 2) * 32;
 constexpr int TC_RAW_ROW = 2 * BLOCK_BYTES;    // two blocks of one row group: 1040 bytes
 constexpr int TC_RAW_BYTES = 33 * 1024;        // 32 x 1040 bytes, padded
@@ -74,10 +80,11 @@ constexpr int TC_SC_BYTES = 2 * TC_CHUNK * 4;  // da and -4 bsum of the chunk's 
 constexpr int TC_OFF_RAW = 0;
 constexpr int TC_OFF_B = TC_OFF_RAW + 2 * TC_RAW_BYTES;
 constexpr int TC_OFF_SC = TC_OFF_B + 2 * TC_B_BYTES;
-constexpr int TC_OFF_BAR = TC_OFF_SC + 2 * TC_SC_BYTES;
-constexpr int TC_NBAR = 23;  // barriers; the TMEM address and abort flag follow
+constexpr int TC_OFF_BAR = TC_OFF_SC + TC_SC_STAGES * TC_SC_BYTES;
+constexpr int TC_NBAR = 19 + 2 * TC_SC_STAGES;  // barriers; the TMEM address and abort flag follow
 constexpr int TC_SMEM = TC_OFF_BAR + TC_NBAR * 8 + 16 + 1024;  // + alignment slack
 constexpr int TC_TMEM_COLS = 512;
+constexpr uint32_t TC_TMEM_Y = 128;            // the running output y (128 columns: pairs)
 constexpr uint32_t TC_TMEM_D = 256;            // first accumulator column
 constexpr int TC_A_COLS = 64;                  // TMEM columns of one block of A (256 bytes per row)
 
@@ -206,28 +213,30 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + TC_OFF_BAR);
     uint64_t *raw_full = bars, *raw_empty = bars + 2;
-    uint64_t *a_full = bars + 4, *a_empty = bars + 6;
+    uint64_t *a_full = bars + 4, *a_empty = bars + 6;  // a_full: elements 0..127 of the block in A
     uint64_t *b_full = bars + 8, *b_empty = bars + 10;
-    uint64_t *sc_full = bars + 12, *sc_empty = bars + 14;
-    uint64_t *d_full = bars + 16, *d_empty = bars + 18;
-    uint64_t *fin = bars + 20;        // MMA drain at exit
-    uint64_t *a_full_hi = bars + 21;  // [2]: elements 128..255 of the block in A (a_full: 0..127)
+    uint64_t *d_full = bars + 12, *d_empty = bars + 14;
+    uint64_t *fin = bars + 16;                          // MMA drain at exit
+    uint64_t *a_full_hi = bars + 17;                    // [2]: elements 128..255
+    uint64_t *sc_full = bars + 19, *sc_empty = bars + 19 + TC_SC_STAGES;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + TC_NBAR);
     int *abort = reinterpret_cast<int *>(tmem_slot + 1);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < 2; ++i) {
             mbar_init(&raw_full[i], 1);
-            mbar_init(&raw_empty[i], TC_MATH_WARPS);
-            mbar_init(&a_full[i], TC_MATH_WARPS);
-            mbar_init(&a_full_hi[i], TC_MATH_WARPS);
+            mbar_init(&raw_empty[i], TC_CONV_WARPS + TC_EPI_WARPS);  // the epilogue reads the row scales
+            mbar_init(&a_full[i], TC_CONV_WARPS);
+            mbar_init(&a_full_hi[i], TC_CONV_WARPS);
             mbar_init(&a_empty[i], 1);
             mbar_init(&b_full[i], 1);
             mbar_init(&b_empty[i], 1);
-            mbar_init(&sc_full[i], 1);
-            mbar_init(&sc_empty[i], TC_MATH_WARPS);
             mbar_init(&d_full[i], 1);
-            mbar_init(&d_empty[i], TC_MATH_WARPS);
+            mbar_init(&d_empty[i], TC_EPI_WARPS);
+        }
+        for (int i = 0; i < TC_SC_STAGES; ++i) {
+            mbar_init(&sc_full[i], 1);
+            mbar_init(&sc_empty[i], TC_EPI_WARPS);
         }
         mbar_init(fin, 1);
         *abort = 0;
@@ -254,7 +263,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     // counts of raw stages and blocks used so far (the ring positions).
     int64_t nraw = 0, nblk = 0;
     // Producer: uses issued on each stage's full barriers (for the drain).
-    int64_t n_rf0 = 0, n_rf1 = 0, n_bf0 = 0, n_bf1 = 0;
+    int64_t n_rf0 = 0, n_rf1 = 0, n_bf0 = 0, n_bf1 = 0, last_sc = -1;
     for (int64_t w = blockIdx.x; w < items; w += gridDim.x) {
         if (*reinterpret_cast<volatile int *>(abort)) break;
         const int chunk = static_cast<int>(w / per_chunk);
@@ -298,9 +307,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                                 tma_2d(smem + TC_OFF_B + bs * TC_B_BYTES + ks * TC_KS_BYTES + pl * TC_PLANE_BYTES +
                                            x * TC_BOX_BYTES,
                                        pl ? &bmap_lo : &bmap_hi, b * QK + ks * 128, pb + 64 * x, &b_full[bs]);
-                    if (!tc_wait(&sc_empty[bs], par, abort, a.status, 3)) break;
-                    mbar_arrive_expect_tx(&sc_full[bs], TC_SC_BYTES);
-                    bulk_g2s(smem + TC_OFF_SC + bs * TC_SC_BYTES, sc + b * (2 * TC_CHUNK), TC_SC_BYTES, &sc_full[bs]);
+                    const int ss = static_cast<int>(bb % TC_SC_STAGES);
+                    if (!tc_wait(&sc_empty[ss], static_cast<uint32_t>(((bb / TC_SC_STAGES) & 1) ^ 1), abort, a.status, 3))
+                        break;
+                    mbar_arrive_expect_tx(&sc_full[ss], TC_SC_BYTES);
+                    bulk_g2s(smem + TC_OFF_SC + ss * TC_SC_BYTES, sc + b * (2 * TC_CHUNK), TC_SC_BYTES, &sc_full[ss]);
+                    last_sc = bb;
                     if (bs) ++n_bf1; else ++n_bf0;
                 }
             }
@@ -348,18 +360,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             __syncwarp();
         } else {
             // ---------------- math warps ----------------
-            const int r4 = warp & 3, h = warp >> 2;
+            const int r4 = warp & 3;                   // TMEM lane quadrant = row r4 of each row group
             const int rgl = lane;                      // row group within the tile
             const uint32_t lane_base = static_cast<uint32_t>(r4 * 32) << 16;
-            const bool active = 64 * h < m;            // this half has pairs to finish
-            float y[64];
-#pragma unroll
-            for (int n = 0; n < 64; ++n) y[n] = 0.0f;
-            float dw_prev = 0.0f;
             bool ok = true;
-            for (int b = 0; b <= nb && ok; ++b) {
-                float dw_cur = 0.0f;
-                if (b < nb) {
+            if (warp < TC_CONV_WARPS) {
+                // ---- unpacking: codes of row (rgl, r4) into A, one block at a time
+                for (int b = 0; b < nb && ok; ++b) {
                     const int64_t bb = nblk + b;
                     const int as = static_cast<int>(bb & 1);
                     const int64_t rb = nraw + b / 2;
@@ -369,19 +376,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         ok = false;
                         break;
                     }
-                    const uint8_t *blk = smem + TC_OFF_RAW + rs * TC_RAW_BYTES + rgl * TC_RAW_ROW + (b & 1) * BLOCK_BYTES;
-                    dw_cur = block_scale(blk, r4);
-                    const uint8_t *codes = blk + CODE_OFS + ROW_BYTES * r4 + 64 * h;
-                    uint32_t x[16];
-                    if (b & 1) {
+                    const uint8_t *codes = smem + TC_OFF_RAW + rs * TC_RAW_BYTES + rgl * TC_RAW_ROW +
+                                           (b & 1) * BLOCK_BYTES + CODE_OFS + ROW_BYTES * r4;
+                    uint32_t x[32];
+                    if (b & 1) {  // 16-byte aligned codes
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) {
+                        for (int i = 0; i < 8; ++i) {
                             const uint4 v = *reinterpret_cast<const uint4 *>(codes + 16 * i);
                             x[4 * i] = v.x, x[4 * i + 1] = v.y, x[4 * i + 2] = v.z, x[4 * i + 3] = v.w;
                         }
                     } else {
 #pragma unroll
-                        for (int i = 0; i < 8; ++i) {
+                        for (int i = 0; i < 16; ++i) {
                             const uint2 v = *reinterpret_cast<const uint2 *>(codes + 8 * i);
                             x[2 * i] = v.x, x[2 * i + 1] = v.y;
                         }
@@ -391,83 +397,101 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         break;
                     }
                     tc_fence_after();
-                    // A columns: element j (< 128) is byte j % 4 of column j / 4;
-                    // element 128 + j of column 32 + j / 4. A code word of bytes
-                    // 64 h + 4 i .. + 3 gives column 16 h + i (its low nibbles)
-                    // and column 32 + 16 h + i (its high nibbles).
-                    const uint32_t acol = tmem + lane_base + as * TC_A_COLS + 16 * h;
+                    // A columns: element j (< 128) is byte j % 4 of column j / 4,
+                    // element 128 + j of column 32 + j / 4: code word i gives
+                    // column i (its low nibbles) and column 32 + i (its high ones)
+                    const uint32_t acol = tmem + lane_base + as * TC_A_COLS;
                     {
-                        uint32_t lo[16];
+                        uint32_t lo[32];
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) lo[i] = x[i] & 0x0f0f0f0fu;
-                        tc_st16(acol, lo);
+                        for (int i = 0; i < 32; ++i) lo[i] = x[i] & 0x0f0f0f0fu;
+                        tc_st32(acol, lo);
                     }
                     {
-                        uint32_t hi[16];
+                        uint32_t hi[32];
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) hi[i] = (x[i] >> 4) & 0x0f0f0f0fu;
+                        for (int i = 0; i < 32; ++i) hi[i] = (x[i] >> 4) & 0x0f0f0f0fu;
                         tc_wait_st();
                         tc_fence_before();
                         __syncwarp();
                         if (lane == 0) mbar_arrive(&a_full[as]);
-                        tc_st16(acol + 32, hi);
+                        tc_st32(acol + 32, hi);
                     }
                     tc_wait_st();
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(&a_full_hi[as]);
-                    if (b & 1) {
-                        if (lane == 0) mbar_arrive(&raw_empty[rs]);
+                    if (lane == 0) {
+                        mbar_arrive(&a_full_hi[as]);
+                        if (b & 1) mbar_arrive(&raw_empty[rs]);
                     }
                 }
-                if (b > 0) {
-                    // epilogue of block b - 1
-                    const int64_t bb = nblk + b - 1;
+            } else {
+                // ---- epilogue: y (in TMEM) += float(S) * (d * da), block after block
+                const uint32_t ycol = tmem + lane_base + TC_TMEM_Y;
+                for (int b = 0; b < nb && ok; ++b) {
+                    const int64_t bb = nblk + b;
                     const int bs = static_cast<int>(bb & 1);
-                    const uint32_t par = static_cast<uint32_t>((bb >> 1) & 1);
-                    if (!tc_warp_wait(&d_full[bs], par, abort, a.status, 9) ||
-                        !tc_warp_wait(&sc_full[bs], par, abort, a.status, 10)) {
+                    const int ss = static_cast<int>(bb % TC_SC_STAGES);
+                    const int64_t rb = nraw + b / 2;
+                    const int rs = static_cast<int>(rb & 1);
+                    if (!tc_warp_wait(&d_full[bs], static_cast<uint32_t>((bb >> 1) & 1), abort, a.status, 9) ||
+                        !tc_warp_wait(&sc_full[ss], static_cast<uint32_t>((bb / TC_SC_STAGES) & 1), abort, a.status,
+                                      10)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    if (active) {
-                        const float *sc = reinterpret_cast<const float *>(smem + TC_OFF_SC + bs * TC_SC_BYTES) + 64 * h;
-                        const uint32_t dcol = tmem + lane_base + TC_TMEM_D + bs * TC_CHUNK + 64 * h;
+                    // this row's weight scale (the raw stage is held until the epilogue is done with it)
+                    const float dw = block_scale(
+                        smem + TC_OFF_RAW + rs * TC_RAW_BYTES + rgl * TC_RAW_ROW + (b & 1) * BLOCK_BYTES, r4);
+                    const float *sc = reinterpret_cast<const float *>(smem + TC_OFF_SC + ss * TC_SC_BYTES);
+                    const uint32_t dcol = tmem + lane_base + TC_TMEM_D + bs * TC_CHUNK;
+#pragma unroll 1
+                    for (int c = 0; c < TC_CHUNK / 32; ++c) {
+                        if (32 * c >= m) break;
+                        uint32_t d[32], yv[32];
+                        tc_ld32(dcol + 32 * c, d);
+                        if (b > 0) tc_ld32(ycol + 32 * c, yv);
+                        tc_wait_ld();
 #pragma unroll
-                        for (int half = 0; half < 2; ++half) {
-                            uint32_t d[32];
-                            tc_ld32(dcol + 32 * half, d);
-                            tc_wait_ld();
+                        for (int n4 = 0; n4 < 8; ++n4) {
+                            const float4 da = *reinterpret_cast<const float4 *>(sc + 32 * c + 4 * n4);
+                            const float4 bi = *reinterpret_cast<const float4 *>(sc + TC_CHUNK + 32 * c + 4 * n4);
+                            const float dav[4] = {da.x, da.y, da.z, da.w}, biv[4] = {bi.x, bi.y, bi.z, bi.w};
 #pragma unroll
-                            for (int n4 = 0; n4 < 8; ++n4) {
-                                const float4 da = *reinterpret_cast<const float4 *>(sc + 32 * half + 4 * n4);
-                                const float4 bi = *reinterpret_cast<const float4 *>(sc + TC_CHUNK + 32 * half + 4 * n4);
-                                const float dav[4] = {da.x, da.y, da.z, da.w}, biv[4] = {bi.x, bi.y, bi.z, bi.w};
-#pragma unroll
-                                for (int q = 0; q < 4; ++q) {
-                                    const int n = 32 * half + 4 * n4 + q;
-                                    // S = 512 D - 4 bsum, exact (integers below 2^18)
-                                    const float S = __fmaf_rn(512.0f, __uint_as_float(d[4 * n4 + q]), biv[q]);
-                                    y[n] = __fadd_rn(y[n], __fmul_rn(S, __fmul_rn(dw_prev, dav[q])));
-                                }
+                            for (int q = 0; q < 4; ++q) {
+                                const int i = 4 * n4 + q;
+                                // S = 512 D - 4 bsum, exact (integers below 2^18)
+                                const float S = __fmaf_rn(512.0f, __uint_as_float(d[i]), biv[q]);
+                                const float yo = b > 0 ? __uint_as_float(yv[i]) : 0.0f;
+                                yv[i] = __float_as_uint(__fadd_rn(yo, __fmul_rn(S, __fmul_rn(dw, dav[q]))));
                             }
                         }
+                        tc_st32(ycol + 32 * c, yv);
                     }
+                    tc_wait_st();
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) {
                         mbar_arrive(&d_empty[bs]);
-                        mbar_arrive(&sc_empty[bs]);
+                        mbar_arrive(&sc_empty[ss]);
+                        if (b & 1) mbar_arrive(&raw_empty[rs]);
                     }
                 }
-                dw_prev = dw_cur;
-            }
-            if (ok && active && rg0 + rgl < n_rg) {
-                const int64_t grow = static_cast<int64_t>(rg0 + rgl) * 4 + r4;
+                if (ok && rg0 + rgl < n_rg) {
+                    const int64_t grow = static_cast<int64_t>(rg0 + rgl) * 4 + r4;
+#pragma unroll 1
+                    for (int c = 0; c < TC_CHUNK / 32; ++c) {
+                        if (32 * c >= m) break;
+                        uint32_t yv[32];
+                        tc_ld32(ycol + 32 * c, yv);
+                        tc_wait_ld();
 #pragma unroll
-                for (int n = 0; n < 64; ++n)
-                    if (64 * h + n < m) J.Y[static_cast<int64_t>(pb + 64 * h + n) * J.N + grow] = y[n];
+                        for (int i = 0; i < 32; ++i)
+                            if (32 * c + i < m)
+                                J.Y[static_cast<int64_t>(pb + 32 * c + i) * J.N + grow] = __uint_as_float(yv[i]);
+                    }
+                }
             }
         }
         nraw += (nb + 1) / 2;
@@ -479,14 +503,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     if (warp == TC_MATH_WARPS && lane == 0) {
         if (n_rf0 > 0) mbar_wait(&raw_full[0], static_cast<uint32_t>((n_rf0 - 1) & 1));
         if (n_rf1 > 0) mbar_wait(&raw_full[1], static_cast<uint32_t>((n_rf1 - 1) & 1));
-        if (n_bf0 > 0) {
-            mbar_wait(&b_full[0], static_cast<uint32_t>((n_bf0 - 1) & 1));
-            mbar_wait(&sc_full[0], static_cast<uint32_t>((n_bf0 - 1) & 1));
-        }
-        if (n_bf1 > 0) {
-            mbar_wait(&b_full[1], static_cast<uint32_t>((n_bf1 - 1) & 1));
-            mbar_wait(&sc_full[1], static_cast<uint32_t>((n_bf1 - 1) & 1));
-        }
+        if (n_bf0 > 0) mbar_wait(&b_full[0], static_cast<uint32_t>((n_bf0 - 1) & 1));
+        if (n_bf1 > 0) mbar_wait(&b_full[1], static_cast<uint32_t>((n_bf1 - 1) & 1));
+        // the last TC_SC_STAGES scale copies, oldest first
+        for (int64_t u = imax64(0, last_sc - TC_SC_STAGES + 1); u <= last_sc; ++u)
+            mbar_wait(&sc_full[u % TC_SC_STAGES], static_cast<uint32_t>((u / TC_SC_STAGES) & 1));
     }
     if (warp == TC_MATH_WARPS + 1 && lane == 0) {
         tc_commit(fin);
