@@ -31,22 +31,29 @@
 // the 8-byte loads of even blocks (codes 8 bytes off 16-byte alignment)
 // two-way.
 //
-// Warp roles (320 threads, one CTA per SM):
+// Warp roles (448 threads, one CTA per SM):
 //   warps 0-3  unpacking. Warp w serves TMEM lanes 32 w .. + 31 (rows with
-//              r4 = w) and writes their codes into A, up to two blocks ahead
-//              of the MMAs;
-//   warps 4-7  epilogue. Warp w serves TMEM lanes 32 (w - 4) .. + 31: per
+//              r4 = w) and writes their codes into A, into the buffer of
+//              block b - 2 once that block's MMAs are complete;
+//   warps 4-11 epilogue. Warp w serves TMEM lanes 32 (w % 4) .. + 31 and
+//              the 32-column chunks (pairs) e and e + 2, e = (w - 4) / 4: per
 //              block it reads the accumulator and the running output y
 //              (kept in TMEM), adds float(S) * (d * da) and writes y back,
 //              trailing the MMAs by up to two blocks; at the end of the
 //              item it stores y;
-//   warp 8     producer: TMA copies of the raw weight blocks (one box per two
-//              blocks of the tile), of the activation planes (128-element x
-//              64-pair boxes) and a bulk copy of the chunk's block scales;
-//   warp 9     TMEM allocation; one thread issues the MMAs (M = 128,
-//              N = the chunk's pairs rounded up to 16, K = 32; 16 per block,
-//              the first 8 as soon as the low nibbles are in place) and the
-//              commits.
+//   warp 12    producer: TMA copies of the raw weight blocks (one box per
+//              two blocks of the tile), of the activation planes (one 4-D
+//              box per block, into a byte ring where a block takes the
+//              chunk's pairs rounded up to 16, times 512 bytes) and a bulk
+//              copy of the chunk's block scales;
+//   warp 13    TMEM allocation; one thread issues the MMAs (M = 128, K = 32)
+//              and two commits per block. Chunks of up to 64 pairs take one
+//              MMA of N = 128 per K-step with both planes side by side (the
+//              two 64-column halves of the accumulator are added by the
+//              epilogue, exactly); larger chunks one MMA per plane, N = the
+//              pairs rounded up to 16. Each shared-memory access the thread
+//              makes stalls its issue, and the tensor pipe with it, so it
+//              reads the abort flag only when it actually has to wait.
 // TMEM: A in columns [0, 128) (two blocks of 64), y in [128, 256),
 // accumulators in [256, 512).
 // The epilogue uses scalar fp32 operations: the packed f32x2 forms were
@@ -66,31 +73,41 @@ namespace {
 
 constexpr int TC_ROWS = 128;                   // weight rows per tile = TMEM lanes
 constexpr int TC_RG = TC_ROWS / 4;             // row groups per tile
-constexpr int TC_MATH_WARPS = 8;              // warps 0-3 unpack A, warps 4-7 run the epilogue
-constexpr int TC_CONV_WARPS = 4, TC_EPI_WARPS = 4;
+constexpr int TC_CONV_WARPS = 4, TC_EPI_WARPS = 8;
+constexpr int TC_MATH_WARPS = TC_CONV_WARPS + TC_EPI_WARPS;  // warps 0-3 unpack A, 4-11 the epilogue
 constexpr int TC_SC_STAGES = 4;                // scale ring: runs ahead of the epilogue
+constexpr int TC_DW_STAGES = 4;                // weight-scale ring: unpacking -> epilogue
 constexpr int TC_THREADS = (TC_MATH_WARPS + 2) * 32;
 constexpr int TC_RAW_ROW = 2 * BLOCK_BYTES;    // two blocks of one row group: 1040 bytes
 constexpr int TC_RAW_BYTES = 33 * 1024;        // 32 x 1040 bytes, padded
-constexpr int TC_BOX_BYTES = 64 * 128;         // one 128-element x 64-pair e4m3 box: 8 KB
-constexpr int TC_PLANE_BYTES = 2 * TC_BOX_BYTES;  // one k-stage (128 elements) of one plane, <= 128 pairs
-constexpr int TC_KS_BYTES = 2 * TC_PLANE_BYTES;   // one k-stage of both planes
-constexpr int TC_B_BYTES = 2 * TC_KS_BYTES;    // one block of B: 64 KB
+// B, the activation planes of a block: four regions (k-stage ks, plane pl)
+// of R rows (pairs) x 128 bytes, R = 64 for chunks of up to 64 pairs, else
+// the pairs rounded up to 16, so a block takes R * 512 bytes (32 KB for 64
+// pairs, 64 KB for 128), loaded by one 4-D TMA copy. Blocks are placed one after another in a byte ring
+// (never split at its end), which keeps more small blocks in flight than
+// fixed slots sized for 128 pairs.
+constexpr int TC_B_ROW = 128;                  // one pair's 128 elements of one plane
+constexpr int TC_B_RING = 144 * 1024;          // ring bytes
+constexpr int TC_B_SLOTS = 8;                  // full / empty barrier pairs: blocks in flight at most
 constexpr int TC_SC_BYTES = 2 * TC_CHUNK * 4;  // da and -4 bsum of the chunk's pairs: 1 KB
 constexpr int TC_OFF_RAW = 0;
 constexpr int TC_OFF_B = TC_OFF_RAW + 2 * TC_RAW_BYTES;
-constexpr int TC_OFF_SC = TC_OFF_B + 2 * TC_B_BYTES;
-constexpr int TC_OFF_BAR = TC_OFF_SC + TC_SC_STAGES * TC_SC_BYTES;
-constexpr int TC_NBAR = 19 + 2 * TC_SC_STAGES;  // barriers; the TMEM address and abort flag follow
-constexpr int TC_SMEM = TC_OFF_BAR + TC_NBAR * 8 + 16 + 1024;  // + alignment slack
+constexpr int TC_OFF_SC = TC_OFF_B + TC_B_RING;
+constexpr int TC_OFF_DW = TC_OFF_SC + TC_SC_STAGES * TC_SC_BYTES;  // [TC_DW_STAGES][128] fp32
+constexpr int TC_OFF_BAR = TC_OFF_DW + TC_DW_STAGES * TC_ROWS * 4;
+constexpr int TC_NBAR = 11 + 2 * TC_B_SLOTS + 2 * TC_SC_STAGES + 2 * TC_DW_STAGES;  // barriers
+constexpr int TC_OFF_BSTART = TC_OFF_BAR + TC_NBAR * 8;  // [TC_B_SLOTS] int64: producer's ring history
+constexpr int TC_SMEM = TC_OFF_BSTART + TC_B_SLOTS * 8 + 16 + 1024;  // + TMEM address, abort flag, alignment slack
 constexpr int TC_TMEM_COLS = 512;
 constexpr uint32_t TC_TMEM_Y = 128;            // the running output y (128 columns: pairs)
 constexpr uint32_t TC_TMEM_D = 256;            // first accumulator column
 constexpr int TC_A_COLS = 64;                  // TMEM columns of one block of A (256 bytes per row)
 
 static_assert(TC_OFF_B % 1024 == 0, "swizzled tiles need 1024-byte alignment");
+static_assert(TC_B_RING % 2048 == 0 && TC_B_RING >= 2 * TC_CHUNK * 4 * TC_B_ROW, "ring: two blocks of 128 pairs");
+static_assert(TC_SMEM <= 227 * 1024, "shared memory per CTA");
 static_assert(TC_RG * TC_RAW_ROW <= TC_RAW_BYTES, "raw stage too small");
-static_assert(TC_CHUNK == 128, "two 64-pair boxes and two 64-column epilogue halves");
+static_assert(TC_CHUNK == 128, "four 32-column epilogue chunks");
 
 // Instruction descriptor of tcgen05.mma kind::f8f6f4: D fp32 (bits 4-5 = 1),
 // A and B e4m3 (bits 7-9 = 0, 10-12 = 0), both K-major (bits 15, 16 = 0),
@@ -164,6 +181,25 @@ __device__ __forceinline__ void tc_st16(uint32_t taddr, const uint32_t (&r)[16])
 __device__ __forceinline__ void tc_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
+__device__ __forceinline__ void tma_4d(void *dst, const CUtensorMap *map, int c0, int c1, int c2, int c3,
+                                       uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], "
+        "[%6];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_map(const CUtensorMap *map) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// Activation-plane tensor maps: dims (128 elements, pairs, plane, K / 128),
+// map i copies boxes of 16 (i + 1) pairs.
+struct TcBMaps {
+    CUtensorMap m[TC_CHUNK / 16];
+};
+
 __device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int c0, int c1, uint64_t *bar) {
     asm volatile(
         "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
@@ -172,15 +208,56 @@ __device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int c0
         : "memory");
 }
 
+// Placement of the blocks of B in the ring. The producer and the MMA thread
+// walk the same blocks with the same sizes, so they compute the same offsets.
+struct BRing {
+    int64_t pos = 0;  // virtual byte position (grows without wrapping)
+    // virtual start of the next block of `bytes` (ring offset = start % ring)
+    __device__ __forceinline__ int64_t place(int bytes) {
+        const int64_t r = pos % TC_B_RING;
+        if (r + bytes > TC_B_RING) pos += TC_B_RING - r;  // do not straddle the end
+        const int64_t v = pos;
+        pos += bytes;
+        return v;
+    }
+};
+
 struct TcJob {
     int N, nb;   // rows and 256-blocks per row of one expert matrix
     float *Y;    // [P][N] output in pair order
 };
 
 // Single-thread bounded wait (producer and MMA threads).
+// Polling wait with a suspend-time hint: a thread whose phase is not yet
+// complete sleeps in the barrier unit (until the phase completes or the hint
+// runs out) instead of re-issuing shared-memory requests, which slow every
+// other warp's barrier and shared-memory traffic. Bounded like mbar_wait.
+__device__ __forceinline__ uint32_t tc_try_wait_sleep(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(1000000u)  // hint: 1 ms
+        : "memory");
+    return ok;
+}
+__device__ __forceinline__ bool tc_poll(uint64_t *bar, uint32_t parity) {
+    const long long t0 = clock64();
+    while (true) {
+        if (tc_try_wait_sleep(bar, parity)) return true;
+        if (clock64() - t0 > kWaitBudgetCycles) return false;
+    }
+}
+
+// A phase that is already complete costs one try_wait: shared-memory
+// accesses of the MMA thread stall it (and with it the tensor pipe), so the
+// abort flag is read only when the thread has to wait.
 __device__ __forceinline__ bool tc_wait(uint64_t *bar, uint32_t parity, int *abort, int *status, int where) {
+    if (mbar_try_wait(bar, parity)) return true;
     if (*reinterpret_cast<volatile int *>(abort)) return false;
-    if (mbar_wait(bar, parity)) return true;
+    if (tc_poll(bar, parity)) return true;
     *reinterpret_cast<volatile int *>(abort) = 1;
     report(status, TQFX4_ETIMEOUT, K_PREFILL, where);
     return false;
@@ -188,13 +265,15 @@ __device__ __forceinline__ bool tc_wait(uint64_t *bar, uint32_t parity, int *abo
 
 // Warp-uniform bounded wait (math warps): all lanes observe the phase, and
 // all agree on the outcome so that the .sync.aligned TMEM accesses that
-// follow are executed by the whole warp or by none of it.
+// follow are executed by the whole warp or by none of it. (Every lane polls:
+// a single polling lane followed by a confirming wait measured slower.)
 __device__ __forceinline__ bool tc_warp_wait(uint64_t *bar, uint32_t parity, int *abort, int *status, int where) {
     const int lane = threadIdx.x & 31;
+    if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;  // already complete
     int ab = lane == 0 ? *reinterpret_cast<volatile int *>(abort) : 0;
     ab = __shfl_sync(0xffffffffu, ab, 0);
     if (ab) return false;
-    const bool ok = __all_sync(0xffffffffu, mbar_wait(bar, parity));
+    const bool ok = __all_sync(0xffffffffu, tc_poll(bar, parity));
     if (!ok && lane == 0) {
         *reinterpret_cast<volatile int *>(abort) = 1;
         report(status, TQFX4_ETIMEOUT, K_PREFILL, where);
@@ -207,39 +286,50 @@ __device__ __forceinline__ bool tc_warp_wait(uint64_t *bar, uint32_t parity, int
 __global__ void __launch_bounds__(TC_THREADS, 1)
     tc_gemm_kernel(GroupedArgs a, TcJob j0, TcJob j1, int njobs, const float *__restrict__ scales,
                    const __grid_constant__ CUtensorMap wmap0, const __grid_constant__ CUtensorMap wmap1,
-                   const __grid_constant__ CUtensorMap bmap_hi, const __grid_constant__ CUtensorMap bmap_lo) {
+                   const __grid_constant__ TcBMaps bmaps) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + TC_OFF_BAR);
     uint64_t *raw_full = bars, *raw_empty = bars + 2;
-    uint64_t *a_full = bars + 4, *a_empty = bars + 6;  // a_full: elements 0..127 of the block in A
-    uint64_t *b_full = bars + 8, *b_empty = bars + 10;
-    uint64_t *d_full = bars + 12, *d_empty = bars + 14;
-    uint64_t *fin = bars + 16;                          // MMA drain at exit
-    uint64_t *a_full_hi = bars + 17;                    // [2]: elements 128..255
-    uint64_t *sc_full = bars + 19, *sc_empty = bars + 19 + TC_SC_STAGES;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + TC_NBAR);
+    uint64_t *a_full = bars + 4;                        // [2]: the block's codes are in A
+    uint64_t *d_full = bars + 6, *d_empty = bars + 8;   // accumulator written / read out
+    uint64_t *fin = bars + 10;                          // MMA drain at exit
+    uint64_t *b_full = bars + 11, *b_empty = b_full + TC_B_SLOTS;
+    uint64_t *sc_full = b_empty + TC_B_SLOTS, *sc_empty = sc_full + TC_SC_STAGES;
+    uint64_t *dw_full = sc_empty + TC_SC_STAGES, *dw_empty = dw_full + TC_DW_STAGES;
+    float *dw_ring = reinterpret_cast<float *>(smem + TC_OFF_DW);
+    int64_t *b_start = reinterpret_cast<int64_t *>(smem + TC_OFF_BSTART);  // virtual starts of the last blocks of B
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(b_start + TC_B_SLOTS);
     int *abort = reinterpret_cast<int *>(tmem_slot + 1);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < 2; ++i) {
             mbar_init(&raw_full[i], 1);
-            mbar_init(&raw_empty[i], TC_CONV_WARPS + TC_EPI_WARPS);  // the epilogue reads the row scales
+            mbar_init(&raw_empty[i], TC_CONV_WARPS);
             mbar_init(&a_full[i], TC_CONV_WARPS);
-            mbar_init(&a_full_hi[i], TC_CONV_WARPS);
-            mbar_init(&a_empty[i], 1);
-            mbar_init(&b_full[i], 1);
-            mbar_init(&b_empty[i], 1);
             mbar_init(&d_full[i], 1);
             mbar_init(&d_empty[i], TC_EPI_WARPS);
+        }
+        for (int i = 0; i < TC_B_SLOTS; ++i) {
+            mbar_init(&b_full[i], 1);
+            mbar_init(&b_empty[i], 1);
         }
         for (int i = 0; i < TC_SC_STAGES; ++i) {
             mbar_init(&sc_full[i], 1);
             mbar_init(&sc_empty[i], TC_EPI_WARPS);
         }
+        for (int i = 0; i < TC_DW_STAGES; ++i) {
+            mbar_init(&dw_full[i], TC_CONV_WARPS);
+            mbar_init(&dw_empty[i], TC_EPI_WARPS);
+        }
         mbar_init(fin, 1);
         *abort = 0;
+    }
+    if (warp == TC_MATH_WARPS && lane == 0) {
+        tma_prefetch_map(&wmap0);
+        tma_prefetch_map(&wmap1);
+        for (int i = 0; i < TC_CHUNK / 16; ++i) tma_prefetch_map(&bmaps.m[i]);
     }
     if (warp == TC_MATH_WARPS + 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
@@ -262,8 +352,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     // All roles walk the same items and blocks, so each keeps identical
     // counts of raw stages and blocks used so far (the ring positions).
     int64_t nraw = 0, nblk = 0;
-    // Producer: uses issued on each stage's full barriers (for the drain).
-    int64_t n_rf0 = 0, n_rf1 = 0, n_bf0 = 0, n_bf1 = 0, last_sc = -1;
+    BRing bring;
+    // Producer: uses issued on each raw stage's full barrier, and the last
+    // block of B and of scales issued (for the drain).
+    int64_t n_rf0 = 0, n_rf1 = 0, last_b = -1, last_sc = -1;
     for (int64_t w = blockIdx.x; w < items; w += gridDim.x) {
         if (*reinterpret_cast<volatile int *>(abort)) break;
         const int chunk = static_cast<int>(w / per_chunk);
@@ -277,8 +369,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         const int n_rg = J.N / 4;
         const int rg0 = static_cast<int>(tl) * TC_RG;
         const int nb = J.nb;
-        const int nbox = m > 64 ? 2 : 1;          // 64-pair boxes of B per k-stage
-        const int nmma = (m + 15) & ~15;          // MMA N
+        const int nmma = (m + 15) & ~15;          // pairs rounded up to 16
+        // Up to 64 pairs: both planes side by side in one MMA of N = 128
+        // (B rows 0..63 the high plane, 64..127 the low one; the epilogue adds
+        // the two halves of the accumulator), else one MMA per plane, N = nmma.
+        const bool side = nmma <= 64;
+        const int brows = side ? 64 : nmma;       // B rows per (k-stage, plane)
+        const int bbytes = 4 * brows * TC_B_ROW;  // one block of B
 
         if (warp == TC_MATH_WARPS) {
             // ---------------- producer ----------------
@@ -297,63 +394,74 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                                e * n_rg + rg0, &raw_full[rs]);
                         if (rs) ++n_rf1; else ++n_rf0;
                     }
-                    const int bs = static_cast<int>(bb & 1);
-                    const uint32_t par = static_cast<uint32_t>(((bb >> 1) & 1) ^ 1);
-                    if (!tc_wait(&b_empty[bs], par, abort, a.status, 2)) break;
-                    mbar_arrive_expect_tx(&b_full[bs], 4 * nbox * TC_BOX_BYTES);
-                    for (int ks = 0; ks < 2; ++ks)
-                        for (int pl = 0; pl < 2; ++pl)
-                            for (int x = 0; x < nbox; ++x)
-                                tma_2d(smem + TC_OFF_B + bs * TC_B_BYTES + ks * TC_KS_BYTES + pl * TC_PLANE_BYTES +
-                                           x * TC_BOX_BYTES,
-                                       pl ? &bmap_lo : &bmap_hi, b * QK + ks * 128, pb + 64 * x, &b_full[bs]);
+                    // B: first wait until the blocks whose bytes this one reuses
+                    // are consumed: the latest block that starts less than one
+                    // ring before this block's end, and at least the previous
+                    // user of this barrier pair (in-order consumption makes
+                    // the latest of them sufficient)
+                    const int64_t v = bring.place(bbytes);
+                    int64_t need = bb - TC_B_SLOTS;
+                    for (int64_t j = bb - 1; j > need && j >= 0; --j)
+                        if (b_start[j % TC_B_SLOTS] < v + bbytes - TC_B_RING) {
+                            need = j;
+                            break;
+                        }
+                    if (need >= 0 && !tc_wait(&b_empty[need % TC_B_SLOTS],
+                                              static_cast<uint32_t>((need / TC_B_SLOTS) & 1), abort, a.status, 2))
+                        break;
+                    const int bs = static_cast<int>(bb % TC_B_SLOTS);
+                    b_start[bs] = v;
+                    mbar_arrive_expect_tx(&b_full[bs], bbytes);
+                    // both k-stages, both planes, brows pairs: [ks][pl][pair][128]
+                    tma_4d(smem + TC_OFF_B + v % TC_B_RING, &bmaps.m[brows / 16 - 1], 0, pb, 0, 2 * b, &b_full[bs]);
+                    last_b = bb;
                     const int ss = static_cast<int>(bb % TC_SC_STAGES);
                     if (!tc_wait(&sc_empty[ss], static_cast<uint32_t>(((bb / TC_SC_STAGES) & 1) ^ 1), abort, a.status, 3))
                         break;
                     mbar_arrive_expect_tx(&sc_full[ss], TC_SC_BYTES);
                     bulk_g2s(smem + TC_OFF_SC + ss * TC_SC_BYTES, sc + b * (2 * TC_CHUNK), TC_SC_BYTES, &sc_full[ss]);
                     last_sc = bb;
-                    if (bs) ++n_bf1; else ++n_bf0;
                 }
             }
             __syncwarp();
         } else if (warp == TC_MATH_WARPS + 1) {
             // ---------------- MMA issuer ----------------
             if (lane == 0) {
-                const uint32_t idesc = tc_idesc(nmma);
-                // B descriptors: stage 0, k-step 0, plane 0; the others differ by
-                // constant byte offsets (>> 4) in the start-address field
+                const uint32_t idesc = tc_idesc(side ? 128 : nmma);
+                // B descriptors: ring start; the others differ by constant
+                // byte offsets (>> 4) in the start-address field
                 const uint64_t bdesc0 = umma_desc(smem_u32(smem + TC_OFF_B));
+                const int region = brows * TC_B_ROW;  // one (k-stage, plane) of B
                 for (int b = 0; b < nb; ++b) {
                     const int64_t bb = nblk + b;
                     const int bs = static_cast<int>(bb & 1);
-                    const uint32_t par = static_cast<uint32_t>((bb >> 1) & 1);
-                    if (!tc_wait(&d_empty[bs], par ^ 1, abort, a.status, 4)) break;
-                    if (!tc_wait(&b_full[bs], par, abort, a.status, 5)) break;
+                    const int64_t v = bring.place(bbytes);
+                    const int slot = static_cast<int>(bb % TC_B_SLOTS);
+                    // the epilogue has read out block bb - 2 (this accumulator
+                    // buffer), the codes are in A and B has landed
+                    if (!tc_wait(&d_empty[bs], static_cast<uint32_t>(((bb >> 1) & 1) ^ 1), abort, a.status, 4)) break;
+                    if (!tc_wait(&a_full[bs], static_cast<uint32_t>((bb >> 1) & 1), abort, a.status, 6)) break;
+                    if (!tc_wait(&b_full[slot], static_cast<uint32_t>((bb / TC_B_SLOTS) & 1), abort, a.status, 5))
+                        break;
+                    tc_fence_after();
                     const uint32_t d_tmem = tmem + TC_TMEM_D + bs * TC_CHUNK;
                     const uint32_t a_tmem = tmem + bs * TC_A_COLS;
-                    const uint64_t bd = bdesc0 + static_cast<uint64_t>((bs * TC_B_BYTES) >> 4);
-                    bool ok = true;
+                    const uint64_t bd = bdesc0 + static_cast<uint64_t>((v % TC_B_RING) >> 4);
+                    if (side) {
 #pragma unroll
-                    for (int half = 0; half < 2; ++half) {
-                        if (!tc_wait(half ? &a_full_hi[bs] : &a_full[bs], par, abort, a.status, half ? 11 : 6)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
+                        for (int kk = 0; kk < 8; ++kk)  // 32-element step: A columns 8 kk .. 8 kk + 7
+                            tc_mma_ts(d_tmem, a_tmem + 8 * kk, bd + (((kk >> 2) * 2 * region + (kk & 3) * 32) >> 4),
+                                      idesc, kk != 0 ? 1u : 0u);
+                    } else {
 #pragma unroll
-                        for (int k4 = 0; k4 < 4; ++k4) {
-                            const int kk = 4 * half + k4;  // 32-element step: A columns 8 kk .. 8 kk + 7
+                        for (int kk = 0; kk < 8; ++kk)
 #pragma unroll
                             for (int pl = 0; pl < 2; ++pl)
                                 tc_mma_ts(d_tmem, a_tmem + 8 * kk,
-                                          bd + ((half * TC_KS_BYTES + pl * TC_PLANE_BYTES + k4 * 32) >> 4), idesc,
+                                          bd + ((((kk >> 2) * 2 + pl) * region + (kk & 3) * 32) >> 4), idesc,
                                           (kk | pl) != 0 ? 1u : 0u);
-                        }
                     }
-                    if (!ok) break;
-                    tc_commit(&a_empty[bs]);
-                    tc_commit(&b_empty[bs]);
+                    tc_commit(&b_empty[slot]);
                     tc_commit(&d_full[bs]);
                 }
             }
@@ -376,81 +484,99 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         ok = false;
                         break;
                     }
-                    const uint8_t *codes = smem + TC_OFF_RAW + rs * TC_RAW_BYTES + rgl * TC_RAW_ROW +
-                                           (b & 1) * BLOCK_BYTES + CODE_OFS + ROW_BYTES * r4;
-                    uint32_t x[32];
-                    if (b & 1) {  // 16-byte aligned codes
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            const uint4 v = *reinterpret_cast<const uint4 *>(codes + 16 * i);
-                            x[4 * i] = v.x, x[4 * i + 1] = v.y, x[4 * i + 2] = v.z, x[4 * i + 3] = v.w;
-                        }
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const uint2 v = *reinterpret_cast<const uint2 *>(codes + 8 * i);
-                            x[2 * i] = v.x, x[2 * i + 1] = v.y;
-                        }
+                    const uint8_t *blk = smem + TC_OFF_RAW + rs * TC_RAW_BYTES + rgl * TC_RAW_ROW + (b & 1) * BLOCK_BYTES;
+                    const uint8_t *codes = blk + CODE_OFS + ROW_BYTES * r4;
+                    // this row's weight scale, handed to the epilogue
+                    const int ds = static_cast<int>(bb % TC_DW_STAGES);
+                    if (!tc_warp_wait(&dw_empty[ds], static_cast<uint32_t>(((bb / TC_DW_STAGES) & 1) ^ 1), abort,
+                                      a.status, 12)) {
+                        ok = false;
+                        break;
                     }
-                    if (!tc_warp_wait(&a_empty[as], static_cast<uint32_t>(((bb >> 1) & 1) ^ 1), abort, a.status, 8)) {
+                    dw_ring[ds * TC_ROWS + r4 * 32 + rgl] = block_scale(blk, r4);
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&dw_full[ds]);
+                    // A buffer `as` is free once the MMAs of block bb - 2 are
+                    // complete (d_full of that block; block bb's own MMAs need
+                    // this block's codes, so the phase cannot have moved on)
+                    if (!tc_warp_wait(&d_full[as], static_cast<uint32_t>(((bb >> 1) & 1) ^ 1), abort, a.status, 8)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
                     // A columns: element j (< 128) is byte j % 4 of column j / 4,
                     // element 128 + j of column 32 + j / 4: code word i gives
-                    // column i (its low nibbles) and column 32 + i (its high ones)
+                    // column i (its low nibbles) and column 32 + i (its high
+                    // ones). Two passes of 16 words keep the registers low.
                     const uint32_t acol = tmem + lane_base + as * TC_A_COLS;
-                    {
-                        uint32_t lo[32];
+                    uint32_t hi[32];
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) lo[i] = x[i] & 0x0f0f0f0fu;
-                        tc_st32(acol, lo);
-                    }
-                    {
-                        uint32_t hi[32];
+                    for (int pass = 0; pass < 2; ++pass) {
+                        uint32_t x[16];
+                        if (b & 1) {  // 16-byte aligned codes
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) hi[i] = (x[i] >> 4) & 0x0f0f0f0fu;
-                        tc_wait_st();
-                        tc_fence_before();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&a_full[as]);
-                        tc_st32(acol + 32, hi);
+                            for (int i = 0; i < 4; ++i) {
+                                const uint4 v = *reinterpret_cast<const uint4 *>(codes + 64 * pass + 16 * i);
+                                x[4 * i] = v.x, x[4 * i + 1] = v.y, x[4 * i + 2] = v.z, x[4 * i + 3] = v.w;
+                            }
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) {
+                                const uint2 v = *reinterpret_cast<const uint2 *>(codes + 64 * pass + 8 * i);
+                                x[2 * i] = v.x, x[2 * i + 1] = v.y;
+                            }
+                        }
+                        uint32_t lo[16];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            lo[i] = x[i] & 0x0f0f0f0fu;
+                            hi[16 * pass + i] = (x[i] >> 4) & 0x0f0f0f0fu;
+                        }
+                        tc_st16(acol + 16 * pass, lo);
                     }
+                    tc_st32(acol + 32, hi);
                     tc_wait_st();
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) {
-                        mbar_arrive(&a_full_hi[as]);
+                        mbar_arrive(&a_full[as]);
                         if (b & 1) mbar_arrive(&raw_empty[rs]);
                     }
                 }
             } else {
-                // ---- epilogue: y (in TMEM) += float(S) * (d * da), block after block
+                // ---- epilogue: y (in TMEM) += float(S) * (d * da), block after block;
+                // two warps per lane quadrant, 32-column chunks (pairs) eh and eh + 2
+                const int eh = (warp - TC_CONV_WARPS) >> 2;
                 const uint32_t ycol = tmem + lane_base + TC_TMEM_Y;
                 for (int b = 0; b < nb && ok; ++b) {
                     const int64_t bb = nblk + b;
                     const int bs = static_cast<int>(bb & 1);
                     const int ss = static_cast<int>(bb % TC_SC_STAGES);
-                    const int64_t rb = nraw + b / 2;
-                    const int rs = static_cast<int>(rb & 1);
+                    const int ds = static_cast<int>(bb % TC_DW_STAGES);
                     if (!tc_warp_wait(&d_full[bs], static_cast<uint32_t>((bb >> 1) & 1), abort, a.status, 9) ||
                         !tc_warp_wait(&sc_full[ss], static_cast<uint32_t>((bb / TC_SC_STAGES) & 1), abort, a.status,
-                                      10)) {
+                                      10) ||
+                        !tc_warp_wait(&dw_full[ds], static_cast<uint32_t>((bb / TC_DW_STAGES) & 1), abort, a.status,
+                                      13)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    // this row's weight scale (the raw stage is held until the epilogue is done with it)
-                    const float dw = block_scale(
-                        smem + TC_OFF_RAW + rs * TC_RAW_BYTES + rgl * TC_RAW_ROW + (b & 1) * BLOCK_BYTES, r4);
+                    const float dw = dw_ring[ds * TC_ROWS + r4 * 32 + rgl];
                     const float *sc = reinterpret_cast<const float *>(smem + TC_OFF_SC + ss * TC_SC_BYTES);
                     const uint32_t dcol = tmem + lane_base + TC_TMEM_D + bs * TC_CHUNK;
 #pragma unroll 1
-                    for (int c = 0; c < TC_CHUNK / 32; ++c) {
+                    for (int c = eh; c < TC_CHUNK / 32; c += 2) {
                         if (32 * c >= m) break;
                         uint32_t d[32], yv[32];
                         tc_ld32(dcol + 32 * c, d);
+                        if (side) {  // D = high-plane half + low-plane half (exact)
+                            tc_ld32(dcol + 64 + 32 * c, yv);
+                            tc_wait_ld();
+#pragma unroll
+                            for (int i = 0; i < 32; ++i)
+                                d[i] = __float_as_uint(__fadd_rn(__uint_as_float(d[i]), __uint_as_float(yv[i])));
+                        }
                         if (b > 0) tc_ld32(ycol + 32 * c, yv);
                         tc_wait_ld();
 #pragma unroll
@@ -475,21 +601,22 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     if (lane == 0) {
                         mbar_arrive(&d_empty[bs]);
                         mbar_arrive(&sc_empty[ss]);
-                        if (b & 1) mbar_arrive(&raw_empty[rs]);
+                        mbar_arrive(&dw_empty[ds]);
                     }
                 }
                 if (ok && rg0 + rgl < n_rg) {
                     const int64_t grow = static_cast<int64_t>(rg0 + rgl) * 4 + r4;
 #pragma unroll 1
-                    for (int c = 0; c < TC_CHUNK / 32; ++c) {
-                        if (32 * c >= m) break;
+                    for (int c = eh; c < TC_CHUNK / 32; c += 2) {
+                        const int n0 = 32 * c;
+                        if (n0 >= m) break;
                         uint32_t yv[32];
                         tc_ld32(ycol + 32 * c, yv);
                         tc_wait_ld();
 #pragma unroll
                         for (int i = 0; i < 32; ++i)
-                            if (32 * c + i < m)
-                                J.Y[static_cast<int64_t>(pb + 32 * c + i) * J.N + grow] = __uint_as_float(yv[i]);
+                            if (n0 + i < m)
+                                J.Y[static_cast<int64_t>(pb + n0 + i) * J.N + grow] = __uint_as_float(yv[i]);
                     }
                 }
             }
@@ -503,8 +630,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     if (warp == TC_MATH_WARPS && lane == 0) {
         if (n_rf0 > 0) mbar_wait(&raw_full[0], static_cast<uint32_t>((n_rf0 - 1) & 1));
         if (n_rf1 > 0) mbar_wait(&raw_full[1], static_cast<uint32_t>((n_rf1 - 1) & 1));
-        if (n_bf0 > 0) mbar_wait(&b_full[0], static_cast<uint32_t>((n_bf0 - 1) & 1));
-        if (n_bf1 > 0) mbar_wait(&b_full[1], static_cast<uint32_t>((n_bf1 - 1) & 1));
+        // the last TC_B_SLOTS blocks of B, oldest first
+        for (int64_t u = imax64(0, last_b - TC_B_SLOTS + 1); u <= last_b; ++u)
+            mbar_wait(&b_full[u % TC_B_SLOTS], static_cast<uint32_t>((u / TC_B_SLOTS) & 1));
         // the last TC_SC_STAGES scale copies, oldest first
         for (int64_t u = imax64(0, last_sc - TC_SC_STAGES + 1); u <= last_sc; ++u)
             mbar_wait(&sc_full[u % TC_SC_STAGES], static_cast<uint32_t>((u / TC_SC_STAGES) & 1));
@@ -524,8 +652,8 @@ namespace {
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode_tc = nullptr;
 
-cudaError_t encode_2d(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t d0, uint64_t d1,
-                      uint64_t stride1, uint32_t b0, uint32_t b1, CUtensorMapSwizzle sw) {
+cudaError_t encode_tiled(CUtensorMap *m, CUtensorMapDataType dt, int rank, const void *base, const cuuint64_t *dims,
+                         const cuuint64_t *strides, const cuuint32_t *box, CUtensorMapSwizzle sw) {
     if (!g_encode_tc) {
         cudaDriverEntryPointQueryResult q;
         void *fn = nullptr;
@@ -534,14 +662,19 @@ cudaError_t encode_2d(CUtensorMap *m, CUtensorMapDataType dt, const void *base, 
         if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
         g_encode_tc = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     }
-    const cuuint64_t dims[2] = {d0, d1};
-    const cuuint64_t strides[1] = {stride1};
-    const cuuint32_t box[2] = {b0, b1};
-    const cuuint32_t estr[2] = {1, 1};
-    CUresult r = g_encode_tc(m, dt, 2, const_cast<void *>(base), dims, strides, box, estr,
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = g_encode_tc(m, dt, rank, const_cast<void *>(base), dims, strides, box, estr,
                              CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+cudaError_t encode_2d(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t d0, uint64_t d1,
+                      uint64_t stride1, uint32_t b0, uint32_t b1, CUtensorMapSwizzle sw) {
+    const cuuint64_t dims[2] = {d0, d1};
+    const cuuint64_t strides[1] = {stride1};
+    const cuuint32_t box[2] = {b0, b1};
+    return encode_tiled(m, dt, 2, base, dims, strides, box, sw);
 }
 
 }  // namespace
@@ -565,27 +698,30 @@ cudaError_t launch_tc_gemm(const GroupedArgs &a, bool down, cudaStream_t st) {
     const uint64_t wd0 = static_cast<uint64_t>(nb) * BLOCK_BYTES / 8;
     const uint64_t wd1 = static_cast<uint64_t>(a.E) * (N / 4);
     const uint64_t wstride = static_cast<uint64_t>(nb) * BLOCK_BYTES;
-    CUtensorMap w0, w1, bh, bl;
+    CUtensorMap w0, w1;
     if ((e = encode_2d(&w0, CU_TENSOR_MAP_DATA_TYPE_UINT64, m0, wd0, wd1, wstride, TC_RAW_ROW / 8, TC_RG,
                        CU_TENSOR_MAP_SWIZZLE_NONE)) != cudaSuccess)
         return e;
     if ((e = encode_2d(&w1, CU_TENSOR_MAP_DATA_TYPE_UINT64, m1, wd0, wd1, wstride, TC_RAW_ROW / 8, TC_RG,
                        CU_TENSOR_MAP_SWIZZLE_NONE)) != cudaSuccess)
         return e;
-    // activation planes: [P][K] bytes each (16 h, then l, as e4m3); boxes of
-    // 128 elements x 64 pairs, 128-byte swizzled
+    // activation planes: [2][P][K] bytes (16 h, then l, as e4m3), seen as
+    // (128 elements, P pairs, 2 planes, K / 128); boxes of (128, 16 (i + 1),
+    // 2, 2): one block of both planes for up to 16 (i + 1) pairs, laid out
+    // [k-stage][plane][pair][128 bytes], 128-byte swizzled
     const uint8_t *act = down ? a.hq : a.xq;
-    const int64_t plane = static_cast<int64_t>(a.P) * K;
-    if ((e = encode_2d(&bh, CU_TENSOR_MAP_DATA_TYPE_UINT8, act, K, a.P, static_cast<uint64_t>(K), 128, 64,
-                       CU_TENSOR_MAP_SWIZZLE_128B)) != cudaSuccess)
-        return e;
-    if ((e = encode_2d(&bl, CU_TENSOR_MAP_DATA_TYPE_UINT8, act + plane, K, a.P, static_cast<uint64_t>(K), 128, 64,
-                       CU_TENSOR_MAP_SWIZZLE_128B)) != cudaSuccess)
-        return e;
+    TcBMaps bm;
+    for (int i = 0; i < TC_CHUNK / 16; ++i) {
+        const cuuint64_t dims[4] = {128, static_cast<cuuint64_t>(a.P), 2, static_cast<cuuint64_t>(K / 128)};
+        const cuuint64_t strides[3] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(a.P) * K, 128};
+        const cuuint32_t box[4] = {128, static_cast<cuuint32_t>(16 * (i + 1)), 2, 2};
+        if ((e = encode_tiled(&bm.m[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, act, dims, strides, box,
+                              CU_TENSOR_MAP_SWIZZLE_128B)) != cudaSuccess)
+            return e;
+    }
     const TcJob j0{N, nb, down ? a.o : a.g};
     const TcJob j1{N, nb, down ? a.o : a.u};
-    tc_gemm_kernel<<<num_sms(), TC_THREADS, TC_SMEM, st>>>(a, j0, j1, down ? 1 : 2, down ? a.hs : a.xs, w0, w1, bh,
-                                                           bl);
+    tc_gemm_kernel<<<num_sms(), TC_THREADS, TC_SMEM, st>>>(a, j0, j1, down ? 1 : 2, down ? a.hs : a.xs, w0, w1, bm);
     return cudaGetLastError();
 }
 
