@@ -188,7 +188,7 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
     job.bss = bss;
     job.nb = nbi;
     const bool any = job.rg_begin < job.rg_end;
-    if (any) warp_stream_prefetch(ring, &job, 1, a.rpu_d, warp, a.warps_d);
+    if (any) warp_stream_prefetch(ring, &job, 1, a.rpu_d, warp, a.warps_d, 1);
     if (warp == a.warps_d - 1) {
         // the routing weights (needed by the combine at the end); the router
         // has completed, so this runs while gate/up drains
@@ -251,6 +251,7 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
             }
         }
     }
+    if (any) warp_stream_prefetch_from(ring, &job, 1, a.rpu_d, warp, a.warps_d, 1);
     __syncthreads();
     TQ_STAMP(2, 3);
     if (any) warp_stream_run(ring, &job, 1, a.rpu_d, warp, a.warps_d, a.status, K_DOWN);
