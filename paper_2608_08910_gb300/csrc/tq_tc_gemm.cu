@@ -281,6 +281,24 @@ __device__ __forceinline__ bool tc_warp_wait(uint64_t *bar, uint32_t parity, int
     return ok;
 }
 
+// Waits on three barriers: the three try_waits go out back to back, so a set
+// of phases that is already complete costs one round trip instead of three;
+// otherwise the bounded waits run one after another.
+__device__ __forceinline__ bool tc_wait3(uint64_t *b0, uint32_t p0, uint64_t *b1, uint32_t p1, uint64_t *b2,
+                                         uint32_t p2, int *abort, int *status, int where) {
+    const uint32_t ok = mbar_try_wait(b0, p0) & mbar_try_wait(b1, p1) & mbar_try_wait(b2, p2);
+    if (ok) return true;
+    return tc_wait(b0, p0, abort, status, where) && tc_wait(b1, p1, abort, status, where) &&
+           tc_wait(b2, p2, abort, status, where);
+}
+__device__ __forceinline__ bool tc_warp_wait3(uint64_t *b0, uint32_t p0, uint64_t *b1, uint32_t p1, uint64_t *b2,
+                                              uint32_t p2, int *abort, int *status, int where) {
+    const uint32_t ok = mbar_try_wait(b0, p0) & mbar_try_wait(b1, p1) & mbar_try_wait(b2, p2);
+    if (__all_sync(0xffffffffu, ok)) return true;
+    return tc_warp_wait(b0, p0, abort, status, where) && tc_warp_wait(b1, p1, abort, status, where) &&
+           tc_warp_wait(b2, p2, abort, status, where);
+}
+
 }  // namespace
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
@@ -439,9 +457,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     const int slot = static_cast<int>(bb % TC_B_SLOTS);
                     // the epilogue has read out block bb - 2 (this accumulator
                     // buffer), the codes are in A and B has landed
-                    if (!tc_wait(&d_empty[bs], static_cast<uint32_t>(((bb >> 1) & 1) ^ 1), abort, a.status, 4)) break;
-                    if (!tc_wait(&a_full[bs], static_cast<uint32_t>((bb >> 1) & 1), abort, a.status, 6)) break;
-                    if (!tc_wait(&b_full[slot], static_cast<uint32_t>((bb / TC_B_SLOTS) & 1), abort, a.status, 5))
+                    if (!tc_wait3(&d_empty[bs], static_cast<uint32_t>(((bb >> 1) & 1) ^ 1), &a_full[bs],
+                                  static_cast<uint32_t>((bb >> 1) & 1), &b_full[slot],
+                                  static_cast<uint32_t>((bb / TC_B_SLOTS) & 1), abort, a.status, 4))
                         break;
                     tc_fence_after();
                     const uint32_t d_tmem = tmem + TC_TMEM_D + bs * TC_CHUNK;
@@ -479,30 +497,24 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     const int as = static_cast<int>(bb & 1);
                     const int64_t rb = nraw + b / 2;
                     const int rs = static_cast<int>(rb & 1);
-                    if ((b & 1) == 0 &&
-                        !tc_warp_wait(&raw_full[rs], static_cast<uint32_t>((rb >> 1) & 1), abort, a.status, 7)) {
+                    // the raw blocks (for odd b the phase its even partner already
+                    // waited for), a free slot of the weight-scale ring, and the A
+                    // buffer, free once the MMAs of block bb - 2 are complete
+                    // (d_full of that block; block bb's own MMAs need this block's
+                    // codes, so the phase cannot have moved on)
+                    const int ds = static_cast<int>(bb % TC_DW_STAGES);
+                    if (!tc_warp_wait3(&raw_full[rs], static_cast<uint32_t>((rb >> 1) & 1), &dw_empty[ds],
+                                       static_cast<uint32_t>(((bb / TC_DW_STAGES) & 1) ^ 1), &d_full[as],
+                                       static_cast<uint32_t>(((bb >> 1) & 1) ^ 1), abort, a.status, 7)) {
                         ok = false;
                         break;
                     }
                     const uint8_t *blk = smem + TC_OFF_RAW + rs * TC_RAW_BYTES + rgl * TC_RAW_ROW + (b & 1) * BLOCK_BYTES;
                     const uint8_t *codes = blk + CODE_OFS + ROW_BYTES * r4;
                     // this row's weight scale, handed to the epilogue
-                    const int ds = static_cast<int>(bb % TC_DW_STAGES);
-                    if (!tc_warp_wait(&dw_empty[ds], static_cast<uint32_t>(((bb / TC_DW_STAGES) & 1) ^ 1), abort,
-                                      a.status, 12)) {
-                        ok = false;
-                        break;
-                    }
                     dw_ring[ds * TC_ROWS + r4 * 32 + rgl] = block_scale(blk, r4);
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&dw_full[ds]);
-                    // A buffer `as` is free once the MMAs of block bb - 2 are
-                    // complete (d_full of that block; block bb's own MMAs need
-                    // this block's codes, so the phase cannot have moved on)
-                    if (!tc_warp_wait(&d_full[as], static_cast<uint32_t>(((bb >> 1) & 1) ^ 1), abort, a.status, 8)) {
-                        ok = false;
-                        break;
-                    }
                     tc_fence_after();
                     // A columns: element j (< 128) is byte j % 4 of column j / 4,
                     // element 128 + j of column 32 + j / 4: code word i gives
@@ -553,11 +565,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     const int bs = static_cast<int>(bb & 1);
                     const int ss = static_cast<int>(bb % TC_SC_STAGES);
                     const int ds = static_cast<int>(bb % TC_DW_STAGES);
-                    if (!tc_warp_wait(&d_full[bs], static_cast<uint32_t>((bb >> 1) & 1), abort, a.status, 9) ||
-                        !tc_warp_wait(&sc_full[ss], static_cast<uint32_t>((bb / TC_SC_STAGES) & 1), abort, a.status,
-                                      10) ||
-                        !tc_warp_wait(&dw_full[ds], static_cast<uint32_t>((bb / TC_DW_STAGES) & 1), abort, a.status,
-                                      13)) {
+                    if (!tc_warp_wait3(&d_full[bs], static_cast<uint32_t>((bb >> 1) & 1), &sc_full[ss],
+                                       static_cast<uint32_t>((bb / TC_SC_STAGES) & 1), &dw_full[ds],
+                                       static_cast<uint32_t>((bb / TC_DW_STAGES) & 1), abort, a.status, 9)) {
                         ok = false;
                         break;
                     }
