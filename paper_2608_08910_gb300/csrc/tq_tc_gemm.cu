@@ -37,10 +37,11 @@
 //              block b - 2 once that block's MMAs are complete;
 //   warps 4-11 epilogue. Warp w serves TMEM lanes 32 (w % 4) .. + 31 and
 //              the 32-column chunks (pairs) e and e + 2, e = (w - 4) / 4: per
-//              block it reads the accumulator and the running output y
-//              (kept in TMEM), adds float(S) * (d * da) and writes y back,
-//              trailing the MMAs by up to two blocks; at the end of the
-//              item it stores y;
+//              block it reads the accumulator (with the planes side by side:
+//              both halves, then hands the buffer back to the MMAs at once)
+//              and the running output y (kept in TMEM), adds
+//              float(S) * (d * da) and writes y back; at the end of the item
+//              it stores y;
 //   warp 12    producer: TMA copies of the raw weight blocks (one box per
 //              two blocks of the tile), of the activation planes (one 4-D
 //              box per block, into a byte ring where a block takes the
@@ -575,6 +576,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     const float dw = dw_ring[ds * TC_ROWS + r4 * 32 + rgl];
                     const float *sc = reinterpret_cast<const float *>(smem + TC_OFF_SC + ss * TC_SC_BYTES);
                     const uint32_t dcol = tmem + lane_base + TC_TMEM_D + bs * TC_CHUNK;
+                    // With the planes side by side a warp has one chunk: once both
+                    // accumulator halves are in registers the buffer goes back to
+                    // the MMAs, before the y update.
+                    bool released = false;
 #pragma unroll 1
                     for (int c = eh; c < TC_CHUNK / 32; c += 2) {
                         if (32 * c >= m) break;
@@ -583,6 +588,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         if (side) {  // D = high-plane half + low-plane half (exact)
                             tc_ld32(dcol + 64 + 32 * c, yv);
                             tc_wait_ld();
+                            tc_fence_before();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(&d_empty[bs]);
+                            released = true;
 #pragma unroll
                             for (int i = 0; i < 32; ++i)
                                 d[i] = __float_as_uint(__fadd_rn(__uint_as_float(d[i]), __uint_as_float(yv[i])));
@@ -609,7 +618,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) {
-                        mbar_arrive(&d_empty[bs]);
+                        if (!released) mbar_arrive(&d_empty[bs]);
                         mbar_arrive(&sc_empty[ss]);
                         mbar_arrive(&dw_empty[ds]);
                     }
