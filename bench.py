@@ -235,7 +235,7 @@ def run_grouped(args, rank, world, local):
     torch.cuda.set_device(local)
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    T, zipf, path = (64, 1.1, B.TQFX4_PATH_DECODE) if args.workload == "grouped_decode_64" else \
+    T, zipf, path = (64, 1.1, B.TQFX4_PATH_AUTO) if args.workload == "grouped_decode_64" else \
         (2048, 0.0, B.TQFX4_PATH_PREFILL)
     if args.tokens:
         T = args.tokens
@@ -325,7 +325,7 @@ def run_grouped(args, rank, world, local):
         gu_bytes = touched / n_batches * 2 * mb
         achieved = gu_bytes / stage_s["gate_up"] / 1e9
         roof = {"bound": "hbm", "achieved": achieved, "peak": peak_hbm, "unit": "GB/s",
-                "frac": achieved / peak_hbm, "traffic": None, "kernel": "grouped_gemm_kernel (gate_up)",
+                "frac": achieved / peak_hbm, "traffic": None, "kernel": "tc_gemm_kernel (gate_up)",
                 "peak_source": peak_kind}
     roof["stage_us"] = {k: v * 1e6 for k, v in stage_s.items()}
     line = {

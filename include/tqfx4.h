@@ -89,9 +89,9 @@ typedef enum tqfx4_status {
 #define TQFX4_SRC_F32_RTN 1 /* round-to-nearest codes from fp32 weights */
 
 /* Paths for tqfx4_moe_grouped. */
-#define TQFX4_PATH_AUTO 0    /* DECODE for small token counts, else PREFILL */
-#define TQFX4_PATH_DECODE 1  /* per-expert grouped GEMV (weights read once) */
-#define TQFX4_PATH_PREFILL 2 /* per-expert grouped GEMM on tensor cores */
+#define TQFX4_PATH_AUTO 0    /* the library's choice: PREFILL (measured faster at every batch size) */
+#define TQFX4_PATH_DECODE 1  /* per-expert grouped GEMM on integer MMA (weights read once) */
+#define TQFX4_PATH_PREFILL 2 /* per-expert grouped GEMM on tensor cores (tcgen05) */
 
 /* Bytes of one N x K matrix: (N/4) * (K/256) * 520 (Sec. 2.2: 4.0625
  * bits/weight). Returns -1 if N % 4 or K % 256 or a size is negative. */

@@ -35,7 +35,7 @@ namespace tq {
 
 // ---------------------------------------------------------------- router
 
-constexpr int RB_TOK = 16;  // tokens per CTA (4 per warp)
+constexpr int RB_TOK = 4;  // tokens per CTA, one per warp (each logit is a latency-bound 16 KB dot product)
 // Batches from which the router screens with an fp32 GEMM first.
 constexpr int kScreenMinTokens = 256;
 
@@ -696,12 +696,18 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(GroupedArgs a) {
 // Tensor-core path: per chunk, its pairs' quantized hidden states as the two
 // e4m3 planes, and per block the pairs' scales da and -4 bsum (as float) in
 // the chunk-aligned layout the contraction stages with one bulk copy.
+// CTA (c, y) handles pair columns 16 y .. 16 y + 15 of chunk c (chunks hold
+// 1..128 pairs, so a chunk is spread over several CTAs).
+constexpr int GT_PAIRS = 16;
+static_assert(TC_CHUNK % GT_PAIRS == 0, "whole CTAs per chunk");
+
 __global__ void __launch_bounds__(256) gather_tc_kernel(GroupedArgs a) {
     const int c = blockIdx.x;
     if (c >= __ldcg(a.n_chunks)) return;
     const int pb = __ldcg(a.chunk_begin + c), m = __ldcg(a.chunk_len + c);
+    const int n0 = blockIdx.y * GT_PAIRS;
     const int64_t plane = static_cast<int64_t>(a.P) * a.H;
-    for (int n = threadIdx.x >> 5; n < m; n += blockDim.x >> 5) {
+    for (int n = n0 + (threadIdx.x >> 5); n < m && n < n0 + GT_PAIRS; n += blockDim.x >> 5) {
         const int64_t pos = pb + n;
         const int64_t t = __ldcg(a.pair_token + pos);
         const uint2 *src = reinterpret_cast<const uint2 *>(a.qx + t * a.H);
@@ -715,8 +721,8 @@ __global__ void __launch_bounds__(256) gather_tc_kernel(GroupedArgs a) {
         }
         if ((threadIdx.x & 31) == 0) a.pair_chunk[pos] = c;
     }
-    for (int i = threadIdx.x; i < a.nbh * TC_CHUNK; i += blockDim.x) {
-        const int b = i / TC_CHUNK, n = i - b * TC_CHUNK;
+    for (int i = threadIdx.x; i < a.nbh * GT_PAIRS; i += blockDim.x) {
+        const int b = i / GT_PAIRS, n = n0 + (i - b * GT_PAIRS);
         float d = 0.0f, nb4 = 0.0f;
         if (n < m) {
             const int64_t t = __ldcg(a.pair_token + pb + n);
@@ -986,7 +992,7 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
     rec(3);
     if ((e = launch_quantize(a.X, a.T, a.H, a.qx, a.dx, a.bx, a.status, st)) != cudaSuccess) return e;
     if (a.tc)
-        gather_tc_kernel<<<a.max_chunks, 256, 0, st>>>(a);
+        gather_tc_kernel<<<dim3(static_cast<unsigned>(a.max_chunks), TC_CHUNK / GT_PAIRS), 256, 0, st>>>(a);
     else
         gather_rows_kernel<<<a.P, 256, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;

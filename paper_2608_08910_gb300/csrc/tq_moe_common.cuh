@@ -33,8 +33,10 @@ struct MoeLayout {
 
 // Tokens (pairs) per chunk of the grouped GEMM.
 constexpr int GG_TOK = 64;
-// Pairs from which the automatic path choice takes the tensor-core contraction.
-constexpr int64_t kTcMinPairs = 4096;
+// Pairs from which the automatic path choice takes the tensor-core
+// contraction: it measured faster than the integer-MMA one at every batch
+// from 4 tokens (top-8) up, so the automatic choice always takes it.
+constexpr int64_t kTcMinPairs = 1;
 // Slices of the hidden dimension the router's screening GEMM sums separately.
 constexpr int kScreenSplit = 4;
 // Pairs per chunk on the tensor-core path (the largest MMA N used).
