@@ -13,6 +13,12 @@ router weights) per token / time per token; tokens/s per MoE layer is the
 same number divided by the bytes per token, reported beside it.
 
     python bench.py [--steps K] [--warmup W] [--gpus N] [--impl ours|reference]
+                    [--workload moe_decode|grouped_decode_64|prefill_2048]
+
+The K timed steps are captured once into a CUDA graph and replayed inside
+the timed region (no host launch work in it); the other workloads time
+tqfx4_moe_grouped on a batch of 64 tokens with Zipf(1.1) routing or 2048
+tokens with uniform routing (tokens/s).
 
 Under torchrun (N > 1) every rank runs its own replica on its own GPU (the
 path has no exchange step here: replicas only) and rank 0 reports the
@@ -257,14 +263,26 @@ def run_grouped(args, rank, world, local):
         layer.grouped(X, ws, path, OUT, sel, selw, stream=stream)
         touched += int((torch.bincount(sel.flatten().long(), minlength=E) > 0).sum())
     bytes_per_step = touched / n_batches * 3 * mb + E * H * 4
+    # The K steps are captured once into a CUDA graph (as a serving loop
+    # would run them), so the timed region holds no host launch work.
+    cap_stream = torch.cuda.Stream(dev)
+    cap_stream.wait_stream(stream)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(cap_stream):
+        with torch.cuda.graph(graph, stream=cap_stream):
+            for i in range(args.steps):
+                layer.grouped(Xs[i % n_batches], ws, path, OUT, sel, selw, stream=cap_stream)
+    stream.wait_stream(cap_stream)
+    graph.replay()  # untimed
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize()
         ev0.record(stream)
-        for i in range(args.steps):
-            layer.grouped(Xs[i % n_batches], ws, path, OUT, sel, selw, stream=stream)
+        graph.replay()
         ev1.record(stream)
         torch.cuda.synchronize()
         if world > 1:
