@@ -40,6 +40,7 @@ def lib():
             "tqo_matrix_bytes": (i64, [i64, i64]),
             "tqo_pack_trits": (i32, [vp, vp, vp, i64, i64, vp]),
             "tqo_pack_rtn": (i32, [vp, i64, i64, vp]),
+            "tqo_pack_tied": (i32, [vp, i64, i64, i32, vp, vp]),
             "tqo_unpack": (i32, [vp, i64, i64, vp, vp]),
             "tqo_dequant": (i32, [vp, i64, i64, vp]),
             "tqo_quantize_act": (i32, [vp, i64, i64, vp, vp, vp]),
@@ -121,6 +122,21 @@ def pack_rtn(w) -> np.ndarray:
     out = np.empty(nbytes, np.uint8)
     _check(lib().tqo_pack_rtn(_p(w), n, k, _p(out)), "pack_rtn")
     return out
+
+
+def pack_tied(w, max_iter=64, with_iters=False):
+    """The tied alternating solver (Sec. 2.1), see tqo_pack_tied: blocks, and
+    with with_iters the scale updates per (row, block) (negated where
+    max_iter stopped a block before its fixed point)."""
+    w = _c(w, np.float32)
+    n, k = w.shape
+    nbytes = matrix_bytes(n, k)
+    if nbytes < 0:
+        raise OracleError("bad shape %r" % (w.shape,))
+    out = np.empty(nbytes, np.uint8)
+    iters = np.empty((n, k // 256), np.int32)
+    _check(lib().tqo_pack_tied(_p(w), n, k, int(max_iter), _p(out), _p(iters)), "pack_tied")
+    return (out, iters) if with_iters else out
 
 
 def pack_trits(t1, t2, d_bits) -> np.ndarray:

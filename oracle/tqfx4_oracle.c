@@ -208,6 +208,92 @@ int tqo_pack_rtn(const float *w, int64_t n, int64_t k, uint8_t *out) {
     return 0;
 }
 
+/* The tied alternating solver (Sec. 2.1: the solver alternates plane
+ * updates against the single scale s, which is the same as fitting the
+ * uniform quantizer W_hat = s * c, c in -4..4; scales serialize to f16).
+ * Readings where the paper gives no details (initialisation, iteration
+ * count, the group, the arithmetic): per (row, 256-block),
+ *   start:  the round-to-nearest fit (tqo_pack_rtn): s = f16(absmax / 4),
+ *           c = clamp(round(w * (1/s)), -4, 4);
+ *   repeat: s' = f16(<w, c> / <c, c>)   (least-squares scale of the codes,
+ *                                        rounded to the nearest f16);
+ *           stop if s' == s (a fixed point) or after max_iter updates;
+ *           s = s', c = clamp(round(w * (1/s)), -4, 4).
+ * Each step minimises the block's squared error over its own variable (the
+ * nearest level for each weight; and, the error being a parabola in s, the
+ * f16 value nearest the least-squares optimum is the best f16 value for the
+ * codes), so the error never exceeds the round-to-nearest fit's, and the
+ * stored block is a pair (s, c) whose codes are nearest to their own scale.
+ * Arithmetic: binary32, no fused operations. <c, c> is an exact integer;
+ * <w, c> is summed in one fixed order: 32 groups of 8 consecutive elements,
+ * each summed in index order, then the 32 partial sums combined pairwise
+ * with the partner whose index differs in bit 4, 3, 2, 1, 0 in turn (every
+ * partial of a level becomes p[l] + p[l ^ o]). iters (nullable, [n][k/256])
+ * receives the number of scale updates, negated when max_iter stopped the
+ * block before a fixed point. Returns 0, -1 on a bad shape or max_iter < 0,
+ * -3 on a non-finite weight. */
+static float tied_dot_wc(const float *w, const float *c) {
+    float p[32], q[32];
+    for (int l = 0; l < 32; l++) {
+        float a = 0.0f;
+        for (int i = 0; i < 8; i++) a = a + w[8 * l + i] * c[8 * l + i];
+        p[l] = a;
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        for (int l = 0; l < 32; l++) q[l] = p[l] + p[l ^ o];
+        memcpy(p, q, sizeof(p));
+    }
+    return p[0];
+}
+
+static void tied_codes(const float *w, float dq, float *c) {
+    float id = (dq != 0.0f) ? 1.0f / dq : 0.0f;
+    for (int j = 0; j < QK; j++) {
+        float v = roundf(w[j] * id);
+        if (v > 4.0f) v = 4.0f;
+        if (v < -4.0f) v = -4.0f;
+        c[j] = v;
+    }
+}
+
+int tqo_pack_tied(const float *w, int64_t n, int64_t k, int max_iter, uint8_t *out, int32_t *iters) {
+    if (tqo_matrix_bytes(n, k) < 0 || max_iter < 0) return -1;
+    int64_t nb = k / QK;
+    memset(out, 0, (size_t)tqo_matrix_bytes(n, k));
+    for (int64_t row = 0; row < n; row++) {
+        for (int64_t b = 0; b < nb; b++) {
+            const float *src = w + row * k + b * QK;
+            float amax = 0.0f;
+            for (int j = 0; j < QK; j++) {
+                if (!isfinite(src[j])) return -3;
+                float a = fabsf(src[j]);
+                if (a > amax) amax = a;
+            }
+            uint16_t d = tqo_f32_to_f16(amax / 4.0f);
+            if ((d & 0x7c00u) == 0x7c00u) d = 0x7bffu; /* saturate */
+            float c[QK];
+            tied_codes(src, tqo_f16_to_f32(d), c);
+            int updates = 0, fixed = 0;
+            while (!fixed && updates < max_iter) {
+                float cc = 0.0f;
+                for (int j = 0; j < QK; j++) cc = cc + c[j] * c[j];
+                if (cc == 0.0f) { fixed = 1; break; } /* all codes zero: absmax = 0 */
+                uint16_t d2 = tqo_f32_to_f16(tied_dot_wc(src, c) / cc);
+                if ((d2 & 0x7c00u) == 0x7c00u) d2 = 0x7bffu;
+                if (d2 == d) { fixed = 1; break; }
+                d = d2;
+                tied_codes(src, tqo_f16_to_f32(d), c);
+                updates++;
+            }
+            if (iters) iters[row * nb + b] = fixed ? updates : -updates;
+            uint8_t *blk = block_at(out, k, row, b * QK);
+            put_scale(blk, (int)(row % ROWS), d);
+            for (int j = 0; j < QK; j++) put_code(blk, (int)(row % ROWS), j, (int)c[j]);
+        }
+    }
+    return 0;
+}
+
 /* Decode blocks back to codes c[n][k] (c = u - 4, "by arithmetic") and
  * scales d[n][k/256]. Returns 0, -1 on a bad shape, -4 on a nibble > 8. */
 int tqo_unpack(const uint8_t *blocks, int64_t n, int64_t k, int8_t *c, uint16_t *d) {
