@@ -87,6 +87,8 @@ typedef enum tqfx4_status {
 /* Sources for tqfx4_pack. */
 #define TQFX4_SRC_TRITS 0   /* fold two trit planes with given f16 scales */
 #define TQFX4_SRC_F32_RTN 1 /* round-to-nearest codes from fp32 weights */
+#define TQFX4_SRC_F32_TIED 2 /* the tied alternating solver from fp32 weights */
+#define TQFX4_TIED_MAX_ITER 64 /* scale updates per block of the tied solver, at most */
 
 /* Paths for tqfx4_moe_grouped. */
 #define TQFX4_PATH_AUTO 0    /* the library's choice: PREFILL (measured faster at every batch size) */
@@ -113,6 +115,16 @@ size_t tqfx4_basic_workspace_bytes(void);
  *     float(d)), -4, 4) computed as w times the binary32 reciprocal of the
  *     f16-rounded scale, rounded half away from zero; d = 0 gives c = 0. A
  *     non-finite weight sets TQFX4_EDATA.
+ *   src == TQFX4_SRC_F32_TIED: a = W as for F32_RTN (t2, scales_f16 NULL).
+ *     The tied alternating solver of Sec. 2.1 (the two planes fitted against
+ *     one scale s, i.e. W_hat = s * c): per (row, block), starting from the
+ *     F32_RTN fit, the scale becomes f16(<w, c> / <c, c>) (binary32; <w, c>
+ *     summed as 32 groups of 8 consecutive elements in index order, then the
+ *     partials combined pairwise by index XOR 16, 8, 4, 2, 1) and the codes
+ *     are recomputed against it as in F32_RTN, until the scale repeats (a
+ *     fixed point: the codes are nearest to their own scale, the scale is
+ *     the best f16 value for the codes) or TQFX4_TIED_MAX_ITER updates. The
+ *     squared error of every block is at most the F32_RTN fit's.
  *   blocks: device, tqfx4_matrix_bytes(n, k) bytes, 16-byte aligned, written
  *     completely. n == 0 or k == 0 writes nothing.
  */

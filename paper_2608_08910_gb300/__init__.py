@@ -7,7 +7,7 @@ seeded synthetic input generators; `workloads` the named benchmark shapes.
 """
 from .binding import (  # noqa: F401
     TQFX4_BLOCK_BYTES, TQFX4_PATH_AUTO, TQFX4_PATH_DECODE, TQFX4_PATH_PREFILL, TQFX4_QK, TQFX4_ROWS,
-    TQFX4_SRC_F32_RTN, TQFX4_SRC_TRITS, TQFX4_STATUS_BYTES, TqfxError, c_experts, c_router, lib,
+    TQFX4_SRC_F32_RTN, TQFX4_SRC_F32_TIED, TQFX4_SRC_TRITS, TQFX4_STATUS_BYTES, TqfxError, c_experts, c_router, lib,
     tqfx4_basic_workspace_bytes, tqfx4_check, tqfx4_gemv, tqfx4_last_error, tqfx4_matrix_bytes,
     tqfx4_moe_ffn, tqfx4_moe_grouped, tqfx4_moe_stage_count, tqfx4_moe_stage_name,
     tqfx4_moe_workspace_bytes, tqfx4_moe_workspace_views, tqfx4_pack, tqfx4_quantize_act)

@@ -20,6 +20,8 @@ TQFX4_STATUS_BYTES = 256
 TQFX4_NOALLOC_SCRATCH_BYTES = 1 << 20
 TQFX4_SRC_TRITS = 0
 TQFX4_SRC_F32_RTN = 1
+TQFX4_SRC_F32_TIED = 2
+TQFX4_TIED_MAX_ITER = 64
 TQFX4_PATH_AUTO = 0
 TQFX4_PATH_DECODE = 1
 TQFX4_PATH_PREFILL = 2

@@ -71,8 +71,8 @@ tqfx4_status tqfx4_pack(int src, const void *a, const int8_t *t2, const uint16_t
     if (n == 0 || k == 0) return ok();
     if (!a || !blocks) return fail(TQFX4_EINVAL, "tqfx4_pack: NULL input or output");
     if (!aligned(blocks, 16)) return fail(TQFX4_EALIGN, "tqfx4_pack: blocks must be 16-byte aligned");
-    if (src == TQFX4_SRC_F32_RTN) {
-        if (t2 || scales_f16) return fail(TQFX4_EINVAL, "tqfx4_pack: t2/scales must be NULL for F32_RTN");
+    if (src == TQFX4_SRC_F32_RTN || src == TQFX4_SRC_F32_TIED) {
+        if (t2 || scales_f16) return fail(TQFX4_EINVAL, "tqfx4_pack: t2/scales must be NULL for F32 sources");
         if (!aligned(a, 16)) return fail(TQFX4_EALIGN, "tqfx4_pack: W must be 16-byte aligned");
     } else if (src == TQFX4_SRC_TRITS) {
         if (!t2 || !scales_f16) return fail(TQFX4_EINVAL, "tqfx4_pack: TRITS needs t2 and scales");

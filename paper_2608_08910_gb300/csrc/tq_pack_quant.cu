@@ -1,6 +1,7 @@
 // tqfx4_pack and tqfx4_quantize_act kernels (Tied Trit-Planes, Sec. 2.1 and
-// 2.2): writing 520-byte tq2_0_fx4 blocks from trit planes or fp32 weights,
-// and per-256-block int8 activation quantization.
+// 2.2): writing 520-byte tq2_0_fx4 blocks from trit planes or fp32 weights
+// (round-to-nearest, or the tied alternating solver), and per-256-block int8
+// activation quantization.
 #include "tq_common.cuh"
 #include "tq_launch.h"
 
@@ -27,7 +28,7 @@ __global__ void __launch_bounds__(256) pack_kernel(const void *a, const int8_t *
         const int64_t row = rg * 4 + r;
         const int64_t e0 = row * k + static_cast<int64_t>(b) * QK + 8 * lane;
         uint32_t u[2] = {0u, 0u};
-        if (SRC == TQFX4_SRC_F32_RTN) {
+        if (SRC == TQFX4_SRC_F32_RTN || SRC == TQFX4_SRC_F32_TIED) {
             const float4 *src = reinterpret_cast<const float4 *>(static_cast<const float *>(a) + e0);
             const float4 v0 = __ldg(src), v1 = __ldg(src + 1);
             const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
@@ -44,13 +45,43 @@ __global__ void __launch_bounds__(256) pack_kernel(const void *a, const int8_t *
             __half d = __float2half_rn(__fdiv_rn(amax, 4.0f));
             uint16_t db = __half_as_ushort(d);
             if ((db & 0x7c00u) == 0x7c00u) db = 0x7bffu;  // saturate at 65504
-            const float dq = __half2float(__ushort_as_half(db));
-            const float id = (dq != 0.0f) ? __fdiv_rn(1.0f, dq) : 0.0f;
+            float cf[8];
+            auto codes = [&](uint16_t bits) {
+                const float dq = __half2float(__ushort_as_half(bits));
+                const float id = (dq != 0.0f) ? __fdiv_rn(1.0f, dq) : 0.0f;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) cf[i] = fminf(fmaxf(roundf(__fmul_rn(v[i], id)), -4.0f), 4.0f);
+            };
+            codes(db);
+            if (SRC == TQFX4_SRC_F32_TIED && __all_sync(0xffffffffu, finite)) {
+                // the tied alternating solver: least-squares scale of the
+                // codes, rounded to f16, then the nearest codes to it, until
+                // the scale repeats. <w, c>: each lane sums its 8 products in
+                // index order, then partners at XOR 16, 8, 4, 2, 1 add (every
+                // lane ends with the same value); <c, c> is exact.
+                for (int it = 0; it < TQFX4_TIED_MAX_ITER; ++it) {
+                    float pw = 0.0f, pc = 0.0f;
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        pw = __fadd_rn(pw, __fmul_rn(v[i], cf[i]));
+                        pc = __fadd_rn(pc, __fmul_rn(cf[i], cf[i]));
+                    }
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1) {
+                        pw = __fadd_rn(pw, __shfl_xor_sync(0xffffffffu, pw, o));
+                        pc = __fadd_rn(pc, __shfl_xor_sync(0xffffffffu, pc, o));
+                    }
+                    if (pc == 0.0f) break;  // all codes zero (absmax = 0)
+                    uint16_t nbits = __half_as_ushort(__float2half_rn(__fdiv_rn(pw, pc)));
+                    if ((nbits & 0x7c00u) == 0x7c00u) nbits = 0x7bffu;
+                    if (nbits == db) break;  // a fixed point
+                    db = nbits;
+                    codes(db);
+                }
+            }
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
-                float c = roundf(__fmul_rn(v[i], id));
-                c = fminf(fmaxf(c, -4.0f), 4.0f);
-                const uint32_t uu = finite ? static_cast<uint32_t>(static_cast<int>(c) + 4) : 4u;
+                const uint32_t uu = finite ? static_cast<uint32_t>(static_cast<int>(cf[i]) + 4) : 4u;
                 u[i >> 2] |= uu << (8 * (i & 3));
             }
             dbits[r] = db;
@@ -122,6 +153,9 @@ cudaError_t launch_pack(int src, const void *a, const int8_t *t2, const uint16_t
     const int64_t grid = (units * 32 + 255) / 256;
     if (src == TQFX4_SRC_F32_RTN)
         pack_kernel<TQFX4_SRC_F32_RTN><<<static_cast<unsigned>(grid), 256, 0, st>>>(
+            a, t2, scales, n_rg, nb, k, static_cast<uint8_t *>(blocks), status);
+    else if (src == TQFX4_SRC_F32_TIED)
+        pack_kernel<TQFX4_SRC_F32_TIED><<<static_cast<unsigned>(grid), 256, 0, st>>>(
             a, t2, scales, n_rg, nb, k, static_cast<uint8_t *>(blocks), status);
     else
         pack_kernel<TQFX4_SRC_TRITS><<<static_cast<unsigned>(grid), 256, 0, st>>>(

@@ -28,6 +28,13 @@ def pack_rtn(w: torch.Tensor, ws: torch.Tensor, out: torch.Tensor = None) -> tor
     return blocks
 
 
+def pack_tied(w: torch.Tensor, ws: torch.Tensor, out: torch.Tensor = None) -> torch.Tensor:
+    n, k = w.shape
+    blocks = empty_blocks(n, k, w.device) if out is None else out
+    B.tqfx4_pack(B.TQFX4_SRC_F32_TIED, w, None, None, n, k, blocks, ws)
+    return blocks
+
+
 def pack_trits(t1, t2, scales_f16, ws) -> torch.Tensor:
     n, k = t1.shape
     blocks = empty_blocks(n, k, t1.device)
