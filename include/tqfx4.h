@@ -212,6 +212,35 @@ tqfx4_status tqfx4_moe_ffn(const tqfx4_experts *ex, const tqfx4_router *rt,
                            void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * tqfx4_moe_route and tqfx4_moe_experts -- tqfx4_moe_ffn in two calls, for
+ * callers that place the selected experts' blocks themselves between the
+ * routing decision and the expert projections: an expert tier that keeps
+ * experts in host memory and copies a missing expert projection, one
+ * contiguous range of bytes, into a device slot (the GPU counterpart of the
+ * paper's streamed expert store, Sec. 2.2: the same bytes and the same
+ * kernels wherever an expert is cached, so the outputs are bitwise the same).
+ *   tqfx4_moe_route: routes x as tqfx4_moe_ffn does and writes sel_idx and
+ *     sel_w (device, [top_k]); ex->gate/up/down are not read. It also
+ *     quantizes x into the workspace for the next call.
+ *   tqfx4_moe_experts: the rest of tqfx4_moe_ffn for the token last routed
+ *     on this workspace (the two calls must be ordered on one stream, with
+ *     no other MoE call on the workspace between them). ptrs: device array
+ *     of 3 x top_k device pointers, the gate blocks of the selected experts
+ *     in rank order, then their up blocks, then their down blocks, each
+ *     16-byte aligned and holding one expert projection
+ *     (tqfx4_matrix_bytes of its shape); ex->gate/up/down are not read.
+ *   Workspace and out: as for tqfx4_moe_ffn (tqfx4_moe_workspace_bytes with
+ *   tokens == 1). The results equal tqfx4_moe_ffn's bit for bit when ptrs
+ *   point at bytes equal to the selected experts' blocks.
+ */
+tqfx4_status tqfx4_moe_route(const tqfx4_experts *ex, const tqfx4_router *rt,
+                             const float *x, int32_t *sel_idx, float *sel_w,
+                             void *ws, size_t ws_bytes, void *stream);
+tqfx4_status tqfx4_moe_experts(const tqfx4_experts *ex, const tqfx4_router *rt,
+                               const void *const *ptrs, float *out,
+                               void *ws, size_t ws_bytes, void *stream);
+
+/*
  * tqfx4_moe_grouped -- T tokens through the same MoE layer, grouped by
  * expert: route all tokens, count (token, slot) pairs per expert, exclusive
  * scan, stable gather (ascending token order within each expert), run each

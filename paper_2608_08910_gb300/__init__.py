@@ -10,4 +10,5 @@ from .binding import (  # noqa: F401
     TQFX4_SRC_F32_RTN, TQFX4_SRC_F32_TIED, TQFX4_SRC_TRITS, TQFX4_STATUS_BYTES, TqfxError, c_experts, c_router, lib,
     tqfx4_basic_workspace_bytes, tqfx4_check, tqfx4_gemv, tqfx4_last_error, tqfx4_matrix_bytes,
     tqfx4_moe_ffn, tqfx4_moe_grouped, tqfx4_moe_stage_count, tqfx4_moe_stage_name,
-    tqfx4_moe_workspace_bytes, tqfx4_moe_workspace_views, tqfx4_pack, tqfx4_quantize_act)
+    tqfx4_moe_workspace_bytes, tqfx4_moe_workspace_views, tqfx4_pack, tqfx4_quantize_act, tqfx4_moe_route,
+    tqfx4_moe_experts)

@@ -71,6 +71,8 @@ _SIGS = {
     "tqfx4_moe_workspace_views": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int, _int,
                                          C.POINTER(CMoeViews)]),
     "tqfx4_moe_ffn_noalloc": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp]),
+    "tqfx4_moe_route": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_moe_experts": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_check": (_int, [_vp, _vp]),
     "tqfx4_last_error": (C.c_char_p, []),
     "tqfx4_status_string": (C.c_char_p, [_int]),
@@ -175,6 +177,18 @@ def tqfx4_moe_ffn_noalloc(ex, rt, x, out, sel_idx, sel_w, stream=None):
     allocate device memory; see include/tqfx4.h)."""
     _check(lib().tqfx4_moe_ffn_noalloc(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w),
                                        _s(stream)), "tqfx4_moe_ffn_noalloc")
+
+
+def tqfx4_moe_route(ex, rt, x, sel_idx, sel_w, ws, stream=None):
+    _check(lib().tqfx4_moe_route(C.byref(ex), C.byref(rt), _p(x), _p(sel_idx), _p(sel_w), _p(ws), _nbytes(ws),
+                                 _s(stream)), "tqfx4_moe_route")
+
+
+def tqfx4_moe_experts(ex, rt, ptrs, out, ws, stream=None):
+    """ptrs: a device int64 tensor of 3 x top_k block addresses (gate, up,
+    down of the selected experts in rank order)."""
+    _check(lib().tqfx4_moe_experts(C.byref(ex), C.byref(rt), _p(ptrs), _p(out), _p(ws), _nbytes(ws), _s(stream)),
+           "tqfx4_moe_experts")
 
 
 def tqfx4_moe_grouped(ex, rt, X, T, OUT, sel_idx, sel_w, path, ws, stream=None, events=None):

@@ -207,6 +207,48 @@ tqfx4_status tqfx4_moe_ffn_traced(const tqfx4_experts *ex, const tqfx4_router *r
     return moe_ffn_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, events);
 }
 
+tqfx4_status tqfx4_moe_route(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, int32_t *sel_idx,
+                             float *sel_w, void *ws, size_t ws_bytes, void *stream) {
+    const char *fn = "tqfx4_moe_route";
+    tqfx4_status s = check_moe_shapes(ex, rt, fn);
+    if (s) return s;
+    if (!rt->weight) return fail(TQFX4_EINVAL, "%s: NULL router weights", fn);
+    if (!aligned(rt->weight, 16) || !aligned(rt->bias, 4))
+        return fail(TQFX4_EALIGN, "%s: router weights must be 16-byte aligned", fn);
+    if (!x || !sel_idx || !sel_w) return fail(TQFX4_EINVAL, "%s: NULL x or selection output", fn);
+    if (!aligned(x, 16) || !aligned(sel_idx, 4) || !aligned(sel_w, 4))
+        return fail(TQFX4_EALIGN, "%s: x must be 16-byte aligned", fn);
+    tq::MoeArgs a;
+    tq::MoeLayout L;
+    if (!tq::moe_decode_args(ex, rt, nullptr, a, L))
+        return fail(TQFX4_ESHAPE, "%s: too many row ranges for the counter area", fn);
+    if ((s = check_ws(ws, ws_bytes, L.total, fn))) return s;
+    tq::moe_decode_args(ex, rt, ws, a, L);
+    cudaError_t e = tq::launch_moe_route(a, x, sel_idx, sel_w, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
+tqfx4_status tqfx4_moe_experts(const tqfx4_experts *ex, const tqfx4_router *rt, const void *const *ptrs, float *out,
+                               void *ws, size_t ws_bytes, void *stream) {
+    const char *fn = "tqfx4_moe_experts";
+    tqfx4_status s = check_moe_shapes(ex, rt, fn);
+    if (s) return s;
+    if (!ptrs || !out) return fail(TQFX4_EINVAL, "%s: NULL pointer table or output", fn);
+    if (!aligned(ptrs, 8) || !aligned(out, 4)) return fail(TQFX4_EALIGN, "%s: misaligned pointer table", fn);
+    tq::MoeArgs a;
+    tq::MoeLayout L;
+    if (!tq::moe_decode_args(ex, rt, nullptr, a, L))
+        return fail(TQFX4_ESHAPE, "%s: too many row ranges for the counter area", fn);
+    if ((s = check_ws(ws, ws_bytes, L.total, fn))) return s;
+    if (tq::gate_up_smem(a) > tq::max_smem_optin() || tq::down_smem(a) > tq::max_smem_optin())
+        return fail(TQFX4_ESHAPE, "%s: top_k x inter too large for the decode kernels' shared memory", fn);
+    tq::moe_decode_args(ex, rt, ws, a, L);
+    cudaError_t e = tq::launch_moe_experts(a, ptrs, out, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
 static tqfx4_status moe_grouped_impl(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X, int64_t T,
                                      float *OUT, int32_t *sel_idx, float *sel_w, int path, void *ws,
                                      size_t ws_bytes, void *stream, void *const *events) {

@@ -28,6 +28,8 @@ bool moe_decode_args(const tqfx4_experts *ex, const tqfx4_router *rt, void *ws, 
 cudaError_t launch_moe_decode(const MoeArgs &a, const float *x, float *out, int32_t *sel_idx, float *sel_w,
                               cudaStream_t st, void *const *events);
 int gate_up_smem(const MoeArgs &a);
+cudaError_t launch_moe_route(const MoeArgs &a, const float *x, int32_t *sel_idx, float *sel_w, cudaStream_t st);
+cudaError_t launch_moe_experts(const MoeArgs &a, const void *const *ptrs, float *out, cudaStream_t st);
 
 struct GroupedArgs;
 bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, void *ws, GroupedArgs &a,

@@ -94,6 +94,14 @@ __global__ void __launch_bounds__(128) router_kernel(MoeArgs a) {
         a.sel[threadIdx.x] = sel_s[threadIdx.x];
         a.sel_out[threadIdx.x] = sel_s[threadIdx.x];
     }
+    if (a.route_only && warp == 1) {  // the routing weights (else the down kernel forms them)
+        float w_s[TQFX4_MAX_TOP_K];
+        softmax_ff_warp(a.logits, a.logits_lo, sel_s, a.top_k, w_s);
+        if (lane < a.top_k) {
+            a.selw[lane] = w_s[lane];
+            a.selw_out[lane] = w_s[lane];
+        }
+    }
     if (threadIdx.x == 0) a.ctr[kCtrRouter] = 0;
     TQ_STAMP(0, 3);
 }
@@ -109,6 +117,7 @@ __global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
     const int warp = threadIdx.x >> 5;
     const int nbh = a.nbh;
     __shared__ int sel_s[TQFX4_MAX_TOP_K];
+    __shared__ const uint8_t *ptr_s[2 * TQFX4_MAX_TOP_K];
     uint8_t *qs = smem;
     float *das = reinterpret_cast<float *>(qs + nbh * QS_STRIDE);
     int *bss = reinterpret_cast<int *>(das + nbh);
@@ -125,6 +134,7 @@ __global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
     ActRegs act;
     act_load(a.qx, a.dx, a.bx, nbh, act);
     if (threadIdx.x < a.top_k) sel_s[threadIdx.x] = __ldcg(a.sel + threadIdx.x);
+    if (a.ptrs && threadIdx.x < 2 * a.top_k) ptr_s[threadIdx.x] = a.ptrs[threadIdx.x];
     __syncthreads();
     const int64_t n_rg = a.I / 4;
     const int64_t upm = (n_rg + a.rpu_gu - 1) / a.rpu_gu;
@@ -142,7 +152,7 @@ __global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
         const int qq = rem >= upm;
         const int64_t r = rem - qq * upm;
         UnitRef U;
-        U.mat = (qq ? a.up : a.gate) + static_cast<int64_t>(sel_s[j]) * a.mb_gu;
+        U.mat = a.ptrs ? ptr_s[qq * a.top_k + j] : (qq ? a.up : a.gate) + static_cast<int64_t>(sel_s[j]) * a.mb_gu;
         U.rg0 = r * a.rpu_gu;
         U.rgs = static_cast<int>(imin64(a.rpu_gu, n_rg - U.rg0));
         U.y = (qq ? a.u : a.g) + static_cast<int64_t>(j) * a.I;
@@ -175,10 +185,10 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
     ring_init(ring);
     fence_barrier_init();
     const int j = blockIdx.x / a.parts_d, p = blockIdx.x - j * a.parts_d;
-    const int64_t e = __ldcg(a.sel + j);
+    const int64_t e = a.ptrs ? 0 : __ldcg(a.sel + j);
     const int64_t n_rg = a.H / 4;
     MatJob job;
-    job.mat = a.down + e * a.mb_d;
+    job.mat = a.ptrs ? a.ptrs[2 * K + j] : a.down + e * a.mb_d;
     job.rg_begin = part_begin(n_rg, a.rpu_d, a.parts_d, p);
     job.rg_end = part_begin(n_rg, a.rpu_d, a.parts_d, p + 1);
     job.y = a.o + static_cast<int64_t>(j) * a.H;
@@ -197,7 +207,7 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
         softmax_ff_warp(a.logits, a.logits_lo, sel_l, K, selw_s);
         if (blockIdx.x == 0 && lane < K) {
             a.selw[lane] = selw_s[lane];
-            a.selw_out[lane] = selw_s[lane];
+            if (a.selw_out) a.selw_out[lane] = selw_s[lane];
         }
     }
     TQ_STAMP(2, 1);
@@ -401,6 +411,37 @@ cudaError_t launch_moe_decode(const MoeArgs &a0, const float *x, float *out, int
         return e;
     rec(3);
     return cudaSuccess;
+}
+
+// The two halves of launch_moe_decode for callers that place the selected
+// experts' blocks themselves between routing and the expert projections
+// (an expert tier): the router alone (selection and routing weights), then
+// gate/up and down over the given pointers.
+cudaError_t launch_moe_route(const MoeArgs &a0, const float *x, int32_t *sel_idx, float *sel_w, cudaStream_t st) {
+    MoeArgs a = a0;
+    a.x = x;
+    a.sel_out = sel_idx;
+    a.selw_out = sel_w;
+    a.route_only = 1;
+    router_kernel<<<a.E + (a.nbh + 3) / 4, 128, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_moe_experts(const MoeArgs &a0, const void *const *ptrs, float *out, cudaStream_t st) {
+    MoeArgs a = a0;
+    a.out = out;
+    a.ptrs = reinterpret_cast<const uint8_t *const *>(ptrs);
+    a.sel_out = nullptr;
+    a.selw_out = nullptr;
+    static unsigned char set_gu[64], set_dn[64];
+    cudaError_t e = allow_max_smem(reinterpret_cast<const void *>(gate_up_kernel), set_gu);
+    if (e == cudaSuccess) e = allow_max_smem(reinterpret_cast<const void *>(down_kernel), set_dn);
+    if (e != cudaSuccess) return e;
+    if ((e = launch_pdl(reinterpret_cast<const void *>(gate_up_kernel), a.top_k * a.parts_gu, a.warps_gu * 32,
+                        gate_up_smem(a), st, false, a)) != cudaSuccess)
+        return e;
+    return launch_pdl(reinterpret_cast<const void *>(down_kernel), a.top_k * a.parts_d, a.warps_d * 32, down_smem(a),
+                      st, false, a);
 }
 
 }  // namespace tq

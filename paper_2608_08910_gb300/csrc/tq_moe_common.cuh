@@ -140,6 +140,11 @@ struct MoeArgs {
     int rpu_gu, slot_gu, stages_gu, warps_gu, parts_gu, static_gu;
     // down geometry: top_k x parts_d CTAs, each a range of row groups
     int rpu_d, slot_d, stages_d, warps_d, parts_d;
+    // the selected experts' blocks given by the caller (device array of
+    // 3 x top_k pointers: gate, then up, then down, in rank order), or null
+    // for the stacked layout (base + expert * matrix bytes)
+    const uint8_t *const *ptrs;
+    int route_only;  // the router also forms the routing weights, and no expert kernels follow
 };
 
 // Arguments of the grouped (T-token) kernels.
