@@ -370,6 +370,114 @@ def run_grouped(args, rank, world, local):
         dist.destroy_process_group()
 
 
+def run_tiered(args, rank, world, local):
+    """One token per step through the 256-expert layer with every expert in
+    pinned host memory and a device slab of --slots experts (the expert tier):
+    route on the GPU, read the selection on the host, copy each missing
+    expert's blocks into a slot (one contiguous range per projection), then
+    the expert projections. Uniform routing over 256 experts with 8 slots
+    misses on almost every lookup, so this is the miss-bound rate of the
+    paper's streamed store, with the host link in the place of its SSD. The
+    host reads the selection every token, so the steps are not graph-captured."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_08910_gb300 import binding as B
+    from paper_2608_08910_gb300 import inputs
+    from paper_2608_08910_gb300.moe import MoeLayer
+    from paper_2608_08910_gb300.tier import ExpertTier
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    assert args.warmup >= 3, "at least 3 warm-up steps"
+    dev = torch.device("cuda", local)
+    layer = MoeLayer.synthetic(SEED, E, H, I, TOPK, 0.0, dev)
+    tier = ExpertTier(layer, args.slots)
+    ws = layer.workspace(1)
+    X = inputs.hidden_states(SEED + rank, POOL, H, dev)
+    Xh = X.cpu().pin_memory()
+    xin = torch.empty(H, device=dev)
+    out = torch.empty(H, device=dev)
+    outh = torch.empty(H, pin_memory=True)
+    sel = torch.empty(TOPK, dtype=torch.int32, device=dev)
+    selw = torch.empty(TOPK, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i):
+        xin.copy_(Xh[i % POOL], non_blocking=True)
+        tier.ffn(xin, ws, out, sel, selw, stream)
+        outh.copy_(out, non_blocking=True)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(first):
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for i in range(args.steps):
+            step(first + i)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        return ev0.elapsed_time(ev1) / 1e3
+
+    # The host waits for the selection every token, and nvidia-smi queries
+    # stall such host-synchronous loops (measured: a quarter of the rate), so
+    # the clocks are sampled over an adjacent run of the same steps and the
+    # reported time is the run without the sampler.
+    with ClockSampler(local) as clk:
+        t_sampled = timed(args.warmup)
+    m0, l0 = tier.misses, tier.lookups
+    t = max_over_ranks(timed(args.warmup + args.steps), world, dev)
+    B.tqfx4_check(ws)
+    misses, lookups = tier.misses - m0, tier.lookups - l0
+    expert_bytes = 2 * layer.mb_gu + layer.mb_d
+    miss_bytes = misses * expert_bytes
+    # the link's copy rate: one pinned host -> device copy of top_k experts'
+    # bytes (a token's misses), timed alone
+    probe_h = tier.host[:TOPK].reshape(-1)  # top_k experts' bytes
+    probe_d = torch.empty_like(probe_h, device=dev)
+    for _ in range(3):
+        probe_d.copy_(probe_h, non_blocking=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for _ in range(10):
+        probe_d.copy_(probe_h, non_blocking=True)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    link_gbs = 10 * probe_h.numel() / (ev0.elapsed_time(ev1) / 1e3) / 1e9
+    achieved = miss_bytes / t / 1e9
+    line = {
+        "metric": "MoE-layer tokens/s, experts in host memory (tiered_decode)",
+        "value": job_rate(args.steps, world, t), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "i8xi4-i32,f32", "data": "synthetic",
+        "config": {"workload": "tiered_decode", "experts": E, "hidden": H, "inter": I, "top_k": TOPK,
+                   "slots": args.slots, "routing": "uniform", "tokens_per_step": 1,
+                   "l2": "experts streamed from host memory; 3.27 GB pool"},
+        "miss_rate": misses / max(1, lookups),
+        "roofline": {"bound": "host-link", "achieved": achieved, "peak": link_gbs, "unit": "GB/s",
+                     "frac": achieved / link_gbs, "traffic": None, "kernel": "expert misses (cudaMemcpyAsync)",
+                     "peak_source": "measured in this run: pinned host -> device copy of %d bytes" % probe_h.numel()},
+        "e2e": {"value": job_rate(args.steps, world, t), "unit": "tokens/s", "h2d_bytes_per_step": H * 4,
+                "d2h_bytes_per_step": H * 4 + TOPK * 4},
+        "gpu_launches": 3 * args.steps,
+        "clocks": dict(clk.summary(), note="sampled over an adjacent run of the same steps (%.3f ms per step "
+                                           "with the sampler running)" % (t_sampled / args.steps * 1e3)),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -382,9 +490,11 @@ def main():
     ap.add_argument("--tokens", type=int, default=0,
                     help="tokens per step of the grouped workloads (default: 64 or 2048; profiling only)")
     ap.add_argument("--workload", default="moe_decode",
-                    choices=["moe_decode", "grouped_decode_64", "prefill_2048"],
+                    choices=["moe_decode", "grouped_decode_64", "prefill_2048", "tiered_decode"],
                     help="moe_decode (default): 1 token; grouped_decode_64: 64 tokens with Zipf(1.1) "
-                         "routing; prefill_2048: 2048 tokens")
+                         "routing; prefill_2048: 2048 tokens; tiered_decode: 1 token with the experts in "
+                         "host memory")
+    ap.add_argument("--slots", type=int, default=TOPK, help="device expert slots of tiered_decode")
     args = ap.parse_args()
     globals()["E"] = args.experts
 
@@ -394,6 +504,9 @@ def main():
 
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.workload == "tiered_decode":
+        run_tiered(args, rank, world, local)
         return
     if args.workload != "moe_decode":
         run_grouped(args, rank, world, local)
