@@ -323,14 +323,26 @@ __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
     for (int i = tid; i < W * E; i += blockDim.x) hist[i] = 0;
     __syncthreads();
     const unsigned lt = (1u << lane) - 1u;
+    // the selections are read 8 rounds of 32 at a time (all loads in flight
+    // before the first use), then processed round by round in order
+    constexpr int GB = 8;
     if (warp < W) {
         const int p0 = warp * R, p1 = min(P, p0 + R);
-        for (int base = p0; base < p1; base += 32) {
-            const int p = base + lane;
-            const bool valid = p < p1;
-            const int e = valid ? __ldcg(a.sel + p) : -1 - lane;
-            const unsigned peers = __match_any_sync(0xffffffffu, e);
-            if (valid && lane == __ffs(peers) - 1) hist[warp * E + e] += __popc(peers);
+        for (int base0 = p0; base0 < p1; base0 += 32 * GB) {
+            int ev[GB];
+#pragma unroll
+            for (int u = 0; u < GB; ++u) {
+                const int p = base0 + 32 * u + lane;
+                ev[u] = p < p1 ? __ldcg(a.sel + p) : -1 - lane;
+            }
+#pragma unroll
+            for (int u = 0; u < GB; ++u) {
+                if (base0 + 32 * u >= p1) break;
+                const int e = ev[u];
+                const bool valid = base0 + 32 * u + lane < p1;
+                const unsigned peers = __match_any_sync(0xffffffffu, e);
+                if (valid && lane == __ffs(peers) - 1) hist[warp * E + e] += __popc(peers);
+            }
         }
     }
     __syncthreads();
@@ -345,23 +357,33 @@ __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
     __syncthreads();
     if (warp < W) {
         const int p0 = warp * R, p1 = min(P, p0 + R);
-        for (int base = p0; base < p1; base += 32) {
-            const int p = base + lane;
-            const bool valid = p < p1;
-            const int e = valid ? __ldcg(a.sel + p) : -1 - lane;
-            const unsigned peers = __match_any_sync(0xffffffffu, e);
-            const int leader = __ffs(peers) - 1;
-            int b = 0;
-            if (valid && lane == leader) {
-                b = hist[warp * E + e];
-                hist[warp * E + e] = b + __popc(peers);
+        for (int base0 = p0; base0 < p1; base0 += 32 * GB) {
+            int ev[GB];
+#pragma unroll
+            for (int u = 0; u < GB; ++u) {
+                const int p = base0 + 32 * u + lane;
+                ev[u] = p < p1 ? __ldcg(a.sel + p) : -1 - lane;
             }
-            b = __shfl_sync(0xffffffffu, b, leader);
-            if (valid) {
-                const int pos = b + __popc(peers & lt);
-                a.pair_token[pos] = p / k;
-                a.pair_slot[pos] = p - (p / k) * k;
-                a.pair_of[p] = pos;
+#pragma unroll
+            for (int u = 0; u < GB; ++u) {
+                if (base0 + 32 * u >= p1) break;
+                const int p = base0 + 32 * u + lane;
+                const bool valid = p < p1;
+                const int e = ev[u];
+                const unsigned peers = __match_any_sync(0xffffffffu, e);
+                const int leader = __ffs(peers) - 1;
+                int b = 0;
+                if (valid && lane == leader) {
+                    b = hist[warp * E + e];
+                    hist[warp * E + e] = b + __popc(peers);
+                }
+                b = __shfl_sync(0xffffffffu, b, leader);
+                if (valid) {
+                    const int pos = b + __popc(peers & lt);
+                    a.pair_token[pos] = p / k;
+                    a.pair_slot[pos] = p - (p / k) * k;
+                    a.pair_of[p] = pos;
+                }
             }
         }
     }
@@ -696,8 +718,21 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(GroupedArgs a) {
 // Tensor-core path: per chunk, its pairs' quantized hidden states as the two
 // e4m3 planes, and per block the pairs' scales da and -4 bsum (as float) in
 // the chunk-aligned layout the contraction stages with one bulk copy.
+// The e4m3 planes of the tokens' quantized x, once per token (in token order;
+// the gather below copies them into pair order): one thread per 8 bytes.
+__global__ void __launch_bounds__(256) planes_tok_kernel(GroupedArgs a) {
+    const int64_t n8 = static_cast<int64_t>(a.T) * a.H / 8;
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (i >= n8) return;
+    uint2 hi, lo;
+    q_planes8(__ldcg(reinterpret_cast<const uint2 *>(a.qx) + i), hi, lo);
+    reinterpret_cast<uint2 *>(a.xqt)[i] = hi;
+    reinterpret_cast<uint2 *>(a.xqt + static_cast<int64_t>(a.T) * a.H)[i] = lo;
+}
+
 // CTA (c, y) handles pair columns 16 y .. 16 y + 15 of chunk c (chunks hold
-// 1..128 pairs, so a chunk is spread over several CTAs).
+// 1..128 pairs, so a chunk is spread over several CTAs): copies the pairs'
+// plane rows from token order and writes the chunk's scale columns.
 constexpr int GT_PAIRS = 16;
 static_assert(TC_CHUNK % GT_PAIRS == 0, "whole CTAs per chunk");
 
@@ -706,20 +741,18 @@ __global__ void __launch_bounds__(256) gather_tc_kernel(GroupedArgs a) {
     if (c >= __ldcg(a.n_chunks)) return;
     const int pb = __ldcg(a.chunk_begin + c), m = __ldcg(a.chunk_len + c);
     const int n0 = blockIdx.y * GT_PAIRS;
-    const int64_t plane = static_cast<int64_t>(a.P) * a.H;
+    const int64_t plane = static_cast<int64_t>(a.P) * a.H, tplane = static_cast<int64_t>(a.T) * a.H;
+    const int lane = threadIdx.x & 31, n16 = a.H / 16;
     for (int n = n0 + (threadIdx.x >> 5); n < m && n < n0 + GT_PAIRS; n += blockDim.x >> 5) {
         const int64_t pos = pb + n;
         const int64_t t = __ldcg(a.pair_token + pos);
-        const uint2 *src = reinterpret_cast<const uint2 *>(a.qx + t * a.H);
-        uint2 *dh = reinterpret_cast<uint2 *>(a.xq + pos * a.H);
-        uint2 *dl = reinterpret_cast<uint2 *>(a.xq + plane + pos * a.H);
-        for (int i = threadIdx.x & 31; i < a.H / 8; i += 32) {
-            uint2 hi, lo;
-            q_planes8(__ldcg(src + i), hi, lo);
-            dh[i] = hi;
-            dl[i] = lo;
+#pragma unroll
+        for (int pl = 0; pl < 2; ++pl) {
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.xqt + pl * tplane + t * a.H);
+            uint4 *dst = reinterpret_cast<uint4 *>(a.xq + pl * plane + pos * a.H);
+            for (int i = lane; i < n16; i += 32) dst[i] = __ldcg(src + i);
         }
-        if ((threadIdx.x & 31) == 0) a.pair_chunk[pos] = c;
+        if (lane == 0) a.pair_chunk[pos] = c;
     }
     for (int i = threadIdx.x; i < a.nbh * GT_PAIRS; i += blockDim.x) {
         const int b = i / GT_PAIRS, n = n0 + (i - b * GT_PAIRS);
@@ -936,6 +969,7 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
         a.chunk_len = reinterpret_cast<int *>(base + L.chunk_len);
         a.n_chunks = reinterpret_cast<int *>(base + L.n_chunks);
         a.xq = base + L.xq;
+        a.xqt = base + L.xqt;
         a.hq = base + L.hq;
         a.pair_chunk = reinterpret_cast<int *>(base + L.pair_chunk);
         a.xs = reinterpret_cast<float *>(base + L.xs);
@@ -991,6 +1025,11 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(3);
     if ((e = launch_quantize(a.X, a.T, a.H, a.qx, a.dx, a.bx, a.status, st)) != cudaSuccess) return e;
+    if (a.tc) {
+        const int64_t n8 = static_cast<int64_t>(a.T) * a.H / 8;
+        planes_tok_kernel<<<static_cast<unsigned>((n8 + 255) / 256), 256, 0, st>>>(a);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
     if (a.tc)
         gather_tc_kernel<<<dim3(static_cast<unsigned>(a.max_chunks), TC_CHUNK / GT_PAIRS), 256, 0, st>>>(a);
     else

@@ -24,6 +24,7 @@ struct MoeLayout {
     size_t dxg, bxg, dhp, bhp;  // [P][round4(nb)] (grouped only)
     size_t chunk_expert, chunk_begin, chunk_len, n_chunks;  // grouped GEMM work list
     size_t xq, hq;    // e4m3 activation planes [2][P][H], [2][P][I] for the tensor-core contraction (grouped only)
+    size_t xqt;       // the same planes of x in token order [2][T][H] (grouped only)
     size_t pair_chunk, xs, hs;  // tensor-core work list helpers (grouped only)
     size_t rnorm;     // fp32 [T + E]: Euclidean norms of the hidden states and router rows (grouped only)
     size_t rpart;     // fp32 [kScreenSplit][T][E]: partial router logits of the screening GEMM (grouped only)
@@ -95,6 +96,7 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.n_chunks = take(4);
         L.xq = take(2 * static_cast<size_t>(P * H));
         L.hq = take(2 * static_cast<size_t>(P * I));
+        L.xqt = take(2 * static_cast<size_t>(T * H));
         L.pair_chunk = take(4 * static_cast<size_t>(P));
         L.rnorm = take(4 * static_cast<size_t>(T + E));
         L.rpart = take(4 * static_cast<size_t>(kScreenSplit) * T * E);
@@ -104,7 +106,7 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = L.xg = SIZE_MAX;
         L.dxg = L.bxg = L.dhp = L.bhp = SIZE_MAX;
         L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
-        L.xq = L.hq = L.pair_chunk = L.xs = L.hs = L.rnorm = L.rpart = SIZE_MAX;
+        L.xq = L.hq = L.xqt = L.pair_chunk = L.xs = L.hs = L.rnorm = L.rpart = SIZE_MAX;
         L.max_chunks = 0;
     }
     L.total = off;
@@ -180,6 +182,7 @@ struct GroupedArgs {
     int chunk;            // pairs per chunk of the work list (GG_TOK, or TC_CHUNK on tensor cores)
     int max_chunks;       // capacity of the work list
     uint8_t *xq, *hq;     // [2][P][H], [2][P][I]: e4m3 planes 16 h and l of q = 16 h + l (tensor-core path)
+    uint8_t *xqt;         // [2][T][H]: the planes of the tokens' x, in token order (tensor-core path)
     int *pair_chunk;      // [P] chunk of each pair (tensor-core path)
     float *xs, *hs;       // [chunks][nb][2][TC_CHUNK]: per chunk and block, the pairs' scales da,
                           // then -4 bsum as float (tensor-core path)
