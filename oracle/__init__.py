@@ -41,6 +41,9 @@ def lib():
             "tqo_pack_trits": (i32, [vp, vp, vp, i64, i64, vp]),
             "tqo_pack_rtn": (i32, [vp, i64, i64, vp]),
             "tqo_pack_tied": (i32, [vp, i64, i64, i32, vp, vp]),
+            "tqo_mxfp4_bytes": (i64, [i64, i64]),
+            "tqo_mxfp4_dequant": (i32, [vp, i64, i64, vp]),
+            "tqo_mxfp4_gemv": (i32, [vp, i64, i64, vp, vp, vp, vp]),
             "tqo_unpack": (i32, [vp, i64, i64, vp, vp]),
             "tqo_dequant": (i32, [vp, i64, i64, vp]),
             "tqo_quantize_act": (i32, [vp, i64, i64, vp, vp, vp]),
@@ -137,6 +140,29 @@ def pack_tied(w, max_iter=64, with_iters=False):
     iters = np.empty((n, k // 256), np.int32)
     _check(lib().tqo_pack_tied(_p(w), n, k, int(max_iter), _p(out), _p(iters)), "pack_tied")
     return (out, iters) if with_iters else out
+
+
+def mxfp4_bytes(n: int, k: int) -> int:
+    return int(lib().tqo_mxfp4_bytes(n, k))
+
+
+def mxfp4_dequant(blocks, n: int, k: int) -> np.ndarray:
+    """fp64 W [n][k] of MXFP4 blocks (17 bytes per 32 elements)."""
+    blocks = _c(blocks, np.uint8)
+    w = np.empty((n, k), np.float64)
+    _check(lib().tqo_mxfp4_dequant(_p(blocks), n, k, _p(w)), "mxfp4_dequant")
+    return w
+
+
+def mxfp4_gemv(blocks, n: int, k: int, q, da):
+    """(y fp32 [n], S int32 [n][k/32]) of the MXFP4 dot pass."""
+    blocks = _c(blocks, np.uint8)
+    q = _c(q, np.int8)
+    da = _c(da, np.float32)
+    y = np.empty(n, np.float32)
+    S = np.empty((n, k // 32), np.int32)
+    _check(lib().tqo_mxfp4_gemv(_p(blocks), n, k, _p(q), _p(da), _p(y), _p(S)), "mxfp4_gemv")
+    return y, S
 
 
 def pack_trits(t1, t2, d_bits) -> np.ndarray:

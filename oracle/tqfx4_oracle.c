@@ -421,6 +421,80 @@ int tqo_gemv(const uint8_t *blocks, int64_t n, int64_t k, const int8_t *q, const
 }
 
 /* ------------------------------------------------------------------ */
+/* The MXFP4 arm (the released expert bytes the paper quantizes from,    */
+/* served directly): OCP microscaling blocks of 32 elements, one e8m0    */
+/* scale byte E (2^(E-127); E = 255 is NaN) and 32 e2m1 values (sign,    */
+/* two exponent bits, one mantissa bit: 0, 0.5, 1, 1.5, 2, 3, 4, 6), 17 */
+/* bytes per block, 4.25 bits/weight. Readings: the block stores E in    */
+/* byte 0 and the codes in bytes 1..16, element j (< 16) in the low      */
+/* nibble of byte 1 + j and element 16 + j in the high nibble (the       */
+/* interchange order of the released files); rows of k/32 blocks are     */
+/* contiguous. The dot pass uses the doubled codes c = 2 * e2m1 (the     */
+/* integers 0, 1, 2, 3, 4, 6, 8, 12 with a sign), so a block's sum       */
+/* S = sum c q is an exact int32 and the block's value is 2^(E-128) * S. */
+/* ------------------------------------------------------------------ */
+#define MX_K 32
+#define MX_BYTES 17
+
+int64_t tqo_mxfp4_bytes(int64_t n, int64_t k) {
+    if (n < 0 || k < 0 || k % MX_K) return -1;
+    return n * (k / MX_K) * MX_BYTES;
+}
+
+/* Doubled e2m1 code of a nibble: magnitudes 0, 1, 2, 3, 4, 6, 8, 12. */
+static int mx_code(int nib) {
+    static const int mag[8] = {0, 1, 2, 3, 4, 6, 8, 12};
+    int m = mag[nib & 7];
+    return (nib & 8) ? -m : m;
+}
+
+static int mx_nibble(const uint8_t *blk, int j) {
+    const uint8_t b = blk[1 + (j % 16)];
+    return (j < 16) ? (b & 0x0f) : (b >> 4);
+}
+
+/* Dequantized weights (fp64) W[n][k] = 2^(E-128) * c. Returns 0, -1 on a bad
+ * shape, -4 on a NaN scale (E = 255). */
+int tqo_mxfp4_dequant(const uint8_t *blocks, int64_t n, int64_t k, double *w) {
+    if (tqo_mxfp4_bytes(n, k) < 0) return -1;
+    int64_t nb = k / MX_K;
+    for (int64_t row = 0; row < n; row++)
+        for (int64_t b = 0; b < nb; b++) {
+            const uint8_t *blk = blocks + (row * nb + b) * MX_BYTES;
+            if (blk[0] == 255) return -4;
+            double sc = ldexp(1.0, (int)blk[0] - 128);
+            for (int j = 0; j < MX_K; j++) w[row * k + b * MX_K + j] = sc * mx_code(mx_nibble(blk, j));
+        }
+    return 0;
+}
+
+/* GEMV of MXFP4 blocks against per-256-block int8 activations (q, da as
+ * tqo_quantize_act writes them): per 32-block the exact sum S = sum c q,
+ * then the fixed float schedule acc = acc + (float)S * (2^(E-128) * da),
+ * blocks in ascending order (the power of two times da is exact). S_out
+ * (nullable) receives S [n][k/32]. Returns 0, -1 on a bad shape or k not a
+ * multiple of 256, -4 on a NaN scale, -5 on allocation failure. */
+int tqo_mxfp4_gemv(const uint8_t *blocks, int64_t n, int64_t k, const int8_t *q, const float *da, float *y,
+                   int32_t *S_out) {
+    if (tqo_mxfp4_bytes(n, k) < 0 || k % QK) return -1;
+    int64_t nb = k / MX_K;
+    for (int64_t row = 0; row < n; row++) {
+        float acc = 0.0f;
+        for (int64_t b = 0; b < nb; b++) {
+            const uint8_t *blk = blocks + (row * nb + b) * MX_BYTES;
+            if (blk[0] == 255) return -4;
+            int32_t s = 0;
+            for (int j = 0; j < MX_K; j++) s += (int32_t)mx_code(mx_nibble(blk, j)) * (int32_t)q[b * MX_K + j];
+            if (S_out) S_out[row * nb + b] = s;
+            float sc = ldexpf(1.0f, (int)blk[0] - 128) * da[(b * MX_K) / QK];
+            acc = acc + (float)s * sc;
+        }
+        y[row] = acc;
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
 /* exp in binary32 (used by SwiGLU). The paper does not fix how SwiGLU   */
 /* is evaluated; because its output is re-quantized to int8 (a rounding  */
 /* decision), both this oracle and the kernel evaluate it with the same  */

@@ -90,3 +90,19 @@ def log_uniform_scale_matrix(seed: int, n: int, k: int, device="cpu") -> torch.T
     sc = torch.pow(10.0, e).repeat_interleave(256, dim=1)[:, :k]
     return (w * sc).to(torch.float32)
 
+
+def mxfp4_matrix(seed: int, n: int, k: int, device="cpu") -> torch.Tensor:
+    """Random MXFP4 bytes for an n x k matrix (17 bytes per 32 elements: an
+    e8m0 scale byte, then 16 bytes of e2m1 nibbles), standing in for released
+    MXFP4 expert weights: scale bytes 119..124 (2^-8 .. 2^-3), magnitude codes
+    drawn with weights falling from 0 to 7 as in quantized heavy-tailed
+    weights, random signs. Random bytes only: no quantizer runs here."""
+    g = _gen((int(seed) << 24) + 23, device)
+    nb = n * (k // 32)
+    scale = torch.randint(119, 125, (nb, 1), generator=g, device=device, dtype=torch.int32)
+    probs = torch.tensor([0.22, 0.2, 0.16, 0.13, 0.1, 0.09, 0.06, 0.04], device=device)
+    mag = torch.multinomial(probs, nb * 32, replacement=True, generator=g).view(nb, 32)
+    sign = torch.randint(0, 2, (nb, 32), generator=g, device=device) * 8
+    nib = (mag + sign).to(torch.int32)
+    codes = nib[:, :16] | (nib[:, 16:] << 4)
+    return torch.cat([scale, codes], dim=1).to(torch.uint8).reshape(-1)
