@@ -13,7 +13,7 @@ router weights) per token / time per token; tokens/s per MoE layer is the
 same number divided by the bytes per token, reported beside it.
 
     python bench.py [--steps K] [--warmup W] [--gpus N] [--impl ours|reference]
-                    [--workload moe_decode|grouped_decode_64|prefill_2048]
+                    [--workload moe_decode|grouped_decode_64|prefill_2048|tiered_decode|mxfp4_gemv]
 
 The K timed steps are captured once into a CUDA graph and replayed inside
 the timed region (no host launch work in it); the other workloads time
@@ -477,6 +477,168 @@ def run_tiered(args, rank, world, local):
     if world > 1:
         dist.destroy_process_group()
 
+GEMV_N, GEMV_K, GEMV_POOL = 131072, 4096, 16
+
+
+def run_gemv(args, rank, world, local):
+    """The MXFP4 arm: one GEMV per step over a 131072 x 4096 matrix (64
+    experts' 2048 x 4096 gate projections stacked, 285 MB, larger than L2) in
+    MXFP4 blocks (the released bytes, 17 per 32 elements), a new activation
+    every step: tqfx4_quantize_act, then tqfx4_gemv_mxfp4. The tq2_0_fx4 GEMV
+    of a matrix of the same shape is timed beside it. Metric: effective MXFP4
+    GB/s (the matrix's bytes over the step time)."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_08910_gb300 import binding as B
+    from paper_2608_08910_gb300 import inputs, ops
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    assert args.warmup >= 3, "at least 3 warm-up steps"
+    dev = torch.device("cuda", local)
+    n, k = GEMV_N, GEMV_K
+    ws = ops.workspace(B.TQFX4_STATUS_BYTES, dev)
+    mx = inputs.mxfp4_matrix(SEED, n, k, dev)
+    mx_bytes = mx.numel()
+    fx = ops.pack_rtn(inputs.gemv_matrix(SEED, n, k, dev), ws)
+    fx_bytes = fx.numel()
+    torch.cuda.empty_cache()
+    X = inputs.hidden_states(SEED + rank, GEMV_POOL, k, dev)
+    q = torch.empty(k, dtype=torch.int8, device=dev)
+    da = torch.empty(k // 256, device=dev)
+    bs = torch.empty(k // 256, dtype=torch.int32, device=dev)
+    y = torch.empty(n, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i, fmt="mxfp4", st=stream, ev=None):
+        if ev:
+            ev[0].record(st)
+        B.tqfx4_quantize_act(X[i % GEMV_POOL], 1, k, q, da, bs, ws, st)
+        if ev:
+            ev[1].record(st)
+        if fmt == "mxfp4":
+            B.tqfx4_gemv_mxfp4(mx, n, k, q, da, y, None, ws, st)
+        else:
+            B.tqfx4_gemv(fx, n, k, q, da, bs, y, None, ws, st)
+        if ev:
+            ev[2].record(st)
+
+    def graph_of(fmt):
+        for i in range(args.warmup):
+            step(i, fmt)
+        torch.cuda.synchronize()
+        B.tqfx4_check(ws)
+        cap = torch.cuda.Stream(dev)
+        cap.wait_stream(stream)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(cap):
+            with torch.cuda.graph(g, stream=cap):
+                for i in range(args.steps):
+                    step(args.warmup + i, fmt, st=cap)
+        stream.wait_stream(cap)
+        g.replay()  # untimed
+        torch.cuda.synchronize()
+        return g
+
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(g):
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        g.replay()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        return max_over_ranks(ev0.elapsed_time(ev1) / 1e3, world, dev)
+
+    g_mx = graph_of("mxfp4")
+    with ClockSampler(local) as clk:
+        t = timed(g_mx)
+    B.tqfx4_check(ws)
+    t_fx = timed(graph_of("fx4"))
+    B.tqfx4_check(ws)
+
+    def stage_times(fmt):
+        reps = min(args.steps, 20)
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(reps)]
+        for i in range(reps):
+            step(i, fmt, ev=evs[i])
+        torch.cuda.synchronize()
+        return (sum(e[0].elapsed_time(e[1]) for e in evs) / reps / 1e3,
+                sum(e[1].elapsed_time(e[2]) for e in evs) / reps / 1e3)
+
+    q_mx, g_mx_s = stage_times("mxfp4")
+    _, g_fx_s = stage_times("fx4")
+    B.tqfx4_check(ws)
+
+    # end to end: the activation from pinned host memory, y back to it
+    Xh = X.cpu().pin_memory()
+    xin = torch.empty(k, device=dev)
+    yh = torch.empty(n, pin_memory=True)
+    for i in range(3):
+        xin.copy_(Xh[i], non_blocking=True)
+        B.tqfx4_quantize_act(xin, 1, k, q, da, bs, ws, stream)
+        B.tqfx4_gemv_mxfp4(mx, n, k, q, da, y, None, ws, stream)
+        yh.copy_(y, non_blocking=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for i in range(args.steps):
+        xin.copy_(Xh[i % GEMV_POOL], non_blocking=True)
+        B.tqfx4_quantize_act(xin, 1, k, q, da, bs, ws, stream)
+        B.tqfx4_gemv_mxfp4(mx, n, k, q, da, y, None, ws, stream)
+        yh.copy_(y, non_blocking=True)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
+    te = max_over_ranks(ev0.elapsed_time(ev1) / 1e3, world, dev)
+
+    peak, peak_kind = _peaks()
+    achieved = mx_bytes / g_mx_s / 1e9
+    line = {
+        "metric": "effective MXFP4 GB/s (GEMV, 131072 x 4096)",
+        "value": job_rate(mx_bytes * args.steps, world, t) / 1e9, "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "i8xe2m1-i32,f32",
+        "data": "synthetic",
+        "config": {"workload": "mxfp4_gemv", "n": n, "k": k, "matrix_bytes": mx_bytes,
+                   "l2": "inputs larger than L2 (285 MB matrix); a different activation per step"},
+        "fx4_same_shape": {"gbs": fx_bytes * args.steps / t_fx / 1e9, "ms_per_step": t_fx / args.steps * 1e3,
+                           "matrix_bytes": fx_bytes, "gemv_us": g_fx_s * 1e6,
+                           "gemv_gbs": fx_bytes / g_fx_s / 1e9},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None, "kernel": "mxfp4_gemv_kernel",
+                     "peak_source": peak_kind, "stage_us": {"quantize_act": q_mx * 1e6, "gemv": g_mx_s * 1e6}},
+        "e2e": {"value": job_rate(mx_bytes * args.steps, world, te) / 1e9, "unit": "GB/s",
+                "h2d_bytes_per_step": k * 4, "d2h_bytes_per_step": n * 4},
+        "gpu_launches": 2 * args.steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import numpy as np
+
+        import oracle
+        rows = 2048
+        sub = mx[:rows * (mx_bytes // n)].cpu().numpy()
+        qh, dah = q.cpu().numpy(), da.cpu().numpy()
+        done, el = 0, 0.0
+        while el < 10.0:
+            t0 = time.perf_counter()
+            oracle.mxfp4_gemv(sub, rows, k, qh, dah)
+            el += time.perf_counter() - t0
+            done += 1
+        line["cpu_baseline"] = {"value": done * sub.nbytes / el / 1e9, "unit": "GB/s", "cores": 1,
+                                "kind": "oracle", "sample": "%d GEMVs of the matrix's first %d rows" % (done, rows)}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 
 def main():
     ap = argparse.ArgumentParser()
@@ -490,10 +652,10 @@ def main():
     ap.add_argument("--tokens", type=int, default=0,
                     help="tokens per step of the grouped workloads (default: 64 or 2048; profiling only)")
     ap.add_argument("--workload", default="moe_decode",
-                    choices=["moe_decode", "grouped_decode_64", "prefill_2048", "tiered_decode"],
+                    choices=["moe_decode", "grouped_decode_64", "prefill_2048", "tiered_decode", "mxfp4_gemv"],
                     help="moe_decode (default): 1 token; grouped_decode_64: 64 tokens with Zipf(1.1) "
                          "routing; prefill_2048: 2048 tokens; tiered_decode: 1 token with the experts in "
-                         "host memory")
+                         "host memory; mxfp4_gemv: one GEMV over MXFP4 blocks")
     ap.add_argument("--slots", type=int, default=TOPK, help="device expert slots of tiered_decode")
     args = ap.parse_args()
     globals()["E"] = args.experts
@@ -507,6 +669,9 @@ def main():
         return
     if args.workload == "tiered_decode":
         run_tiered(args, rank, world, local)
+        return
+    if args.workload == "mxfp4_gemv":
+        run_gemv(args, rank, world, local)
         return
     if args.workload != "moe_decode":
         run_grouped(args, rank, world, local)

@@ -157,6 +157,33 @@ tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k,
                         void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * The MXFP4 arm: the released expert bytes the paper quantizes from (Sec.
+ * 2.1; the 4.25-bit row of Table 3), served by the integer dot pass with no
+ * transcode. Format (OCP microscaling): blocks of 32 consecutive elements of
+ * a row, 17 bytes each: byte 0 the e8m0 scale E (2^(E-127); E = 255 is NaN),
+ * bytes 1..16 the e2m1 codes (sign, two exponent bits, one mantissa bit:
+ * 0, 0.5, 1, 1.5, 2, 3, 4, 6), element j < 16 in the low nibble of byte
+ * 1 + j and element 16 + j in the high nibble. A row is k/32 consecutive
+ * blocks; rows are consecutive.
+ *   tqfx4_mxfp4_bytes: n * (k/32) * 17, or -1 if k is not a multiple of 32.
+ *   tqfx4_gemv_mxfp4: y = W x for such a matrix and x quantized by
+ *     tqfx4_quantize_act (q int8 [k], da fp32 [k/256]). Per 32-block the
+ *     exact int32 sum S = sum c q of the doubled codes c = 2 e2m1 (the
+ *     integers 0..12 with a sign) and q, then y[n] = the binary32 sum, in
+ *     ascending block order, of float(S) * (2^(E-128) * da) (every product
+ *     and sum one binary32 rounding; 2^(E-128) * da is exact unless it
+ *     falls below the normal range, with subnormals kept, not flushed).
+ *     block_sums: nullable int32 [n][k/32] (device) receives S. k must be a
+ *     multiple of 512 (rows 16-byte aligned), <= TQFX4_MAX_K; blocks and q
+ *     16-byte aligned. A NaN scale sets TQFX4_EDATA.
+ */
+int64_t tqfx4_mxfp4_bytes(int64_t n, int64_t k);
+tqfx4_status tqfx4_gemv_mxfp4(const void *blocks, int64_t n, int64_t k,
+                              const int8_t *q, const float *da,
+                              float *y, int32_t *block_sums,
+                              void *ws, size_t ws_bytes, void *stream);
+
+/*
  * Routed experts: gate and up are [n_experts] stacked matrices of shape
  * inter x hidden, down is [n_experts] stacked matrices of shape hidden x
  * inter, each expert's matrix at base + e * tqfx4_matrix_bytes(...) (one

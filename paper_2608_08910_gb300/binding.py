@@ -17,6 +17,7 @@ TQFX4_QK = 256
 TQFX4_ROWS = 4
 TQFX4_BLOCK_BYTES = 520
 TQFX4_STATUS_BYTES = 256
+TQFX4_MAX_K = 16384
 TQFX4_NOALLOC_SCRATCH_BYTES = 1 << 20
 TQFX4_SRC_TRITS = 0
 TQFX4_SRC_F32_RTN = 1
@@ -71,6 +72,8 @@ _SIGS = {
     "tqfx4_moe_workspace_views": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int, _int,
                                          C.POINTER(CMoeViews)]),
     "tqfx4_moe_ffn_noalloc": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp]),
+    "tqfx4_mxfp4_bytes": (_i64, [_i64, _i64]),
+    "tqfx4_gemv_mxfp4": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_route": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_experts": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_check": (_int, [_vp, _vp]),
@@ -177,6 +180,15 @@ def tqfx4_moe_ffn_noalloc(ex, rt, x, out, sel_idx, sel_w, stream=None):
     allocate device memory; see include/tqfx4.h)."""
     _check(lib().tqfx4_moe_ffn_noalloc(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w),
                                        _s(stream)), "tqfx4_moe_ffn_noalloc")
+
+
+def tqfx4_mxfp4_bytes(n: int, k: int) -> int:
+    return int(lib().tqfx4_mxfp4_bytes(n, k))
+
+
+def tqfx4_gemv_mxfp4(blocks, n, k, q, da, y, block_sums, ws, stream=None):
+    _check(lib().tqfx4_gemv_mxfp4(_p(blocks), n, k, _p(q), _p(da), _p(y), _p(block_sums), _p(ws), _nbytes(ws),
+                                  _s(stream)), "tqfx4_gemv_mxfp4")
 
 
 def tqfx4_moe_route(ex, rt, x, sel_idx, sel_w, ws, stream=None):

@@ -123,6 +123,26 @@ tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
 }
 
 
+int64_t tqfx4_mxfp4_bytes(int64_t n, int64_t k) { return tq::mxfp4_bytes(n, k); }
+
+tqfx4_status tqfx4_gemv_mxfp4(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da, float *y,
+                              int32_t *block_sums, void *ws, size_t ws_bytes, void *stream) {
+    const char *fn = "tqfx4_gemv_mxfp4";
+    if (n < 0 || k <= 0 || k % 512 || k > TQFX4_MAX_K)
+        return fail(TQFX4_ESHAPE, "%s: k=%lld must be a positive multiple of 512 <= %d", fn, (long long)k,
+                    TQFX4_MAX_K);
+    tqfx4_status s = check_ws(ws, ws_bytes, TQFX4_STATUS_BYTES, fn);
+    if (s) return s;
+    if (n == 0) return ok();
+    if (!blocks || !q || !da || !y) return fail(TQFX4_EINVAL, "%s: NULL input or output", fn);
+    if (!aligned(blocks, 16) || !aligned(q, 16) || !aligned(da, 4) || !aligned(y, 4) || !aligned(block_sums, 4))
+        return fail(TQFX4_EALIGN, "%s: blocks and q must be 16-byte aligned", fn);
+    cudaError_t e = tq::launch_mxfp4_gemv(blocks, n, k, q, da, y, block_sums, static_cast<int *>(ws),
+                                          static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
 // ---------------------------------------------------------------- MoE
 
 namespace {

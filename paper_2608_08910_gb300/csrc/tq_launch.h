@@ -28,6 +28,9 @@ bool moe_decode_args(const tqfx4_experts *ex, const tqfx4_router *rt, void *ws, 
 cudaError_t launch_moe_decode(const MoeArgs &a, const float *x, float *out, int32_t *sel_idx, float *sel_w,
                               cudaStream_t st, void *const *events);
 int gate_up_smem(const MoeArgs &a);
+int64_t mxfp4_bytes(int64_t n, int64_t k);
+cudaError_t launch_mxfp4_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da, float *y,
+                              int32_t *block_sums, int *status, cudaStream_t st);
 cudaError_t launch_moe_route(const MoeArgs &a, const float *x, int32_t *sel_idx, float *sel_w, cudaStream_t st);
 cudaError_t launch_moe_experts(const MoeArgs &a, const void *const *ptrs, float *out, cudaStream_t st);
 

@@ -59,3 +59,12 @@ def gemv(blocks, n: int, k: int, q, da, bsum, ws, block_sums: bool = False):
     S = torch.empty((n, k // 256), dtype=torch.int32, device=blocks.device) if block_sums else None
     B.tqfx4_gemv(blocks, n, k, q, da, bsum, y, S, ws)
     return (y, S) if block_sums else y
+
+
+def gemv_mxfp4(blocks, n: int, k: int, q, da, ws, block_sums: bool = False):
+    """y = W x for W in MXFP4 blocks (17 bytes per 32 elements) and x
+    quantized by quantize_act."""
+    y = torch.empty(n, dtype=torch.float32, device=blocks.device)
+    S = torch.empty((n, k // 32), dtype=torch.int32, device=blocks.device) if block_sums else None
+    B.tqfx4_gemv_mxfp4(blocks, n, k, q, da, y, S, ws)
+    return (y, S) if block_sums else y
