@@ -169,10 +169,12 @@ tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k,
  *   tqfx4_gemv_mxfp4: y = W x for such a matrix and x quantized by
  *     tqfx4_quantize_act (q int8 [k], da fp32 [k/256]). Per 32-block the
  *     exact int32 sum S = sum c q of the doubled codes c = 2 e2m1 (the
- *     integers 0..12 with a sign) and q, then y[n] = the binary32 sum, in
- *     ascending block order, of float(S) * (2^(E-128) * da) (every product
- *     and sum one binary32 rounding; 2^(E-128) * da is exact unless it
- *     falls below the normal range, with subnormals kept, not flushed).
+ *     integers 0..12 with a sign) and q, and its exact value
+ *     t = float(S) * 2^(E-128) (subnormals kept, inf past the range). Float
+ *     schedule, by the activation's 256-element scale unit g: G_g = the
+ *     binary32 sum of t over g's eight blocks in ascending order, then y[n]
+ *     = the binary32 sum of G_g * da[g] over g ascending (each product and
+ *     sum rounded once).
  *     block_sums: nullable int32 [n][k/32] (device) receives S. k must be a
  *     multiple of 512 (rows 16-byte aligned), <= TQFX4_MAX_K; blocks and q
  *     16-byte aligned. A NaN scale sets TQFX4_EDATA.

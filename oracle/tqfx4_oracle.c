@@ -469,25 +469,34 @@ int tqo_mxfp4_dequant(const uint8_t *blocks, int64_t n, int64_t k, double *w) {
 }
 
 /* GEMV of MXFP4 blocks against per-256-block int8 activations (q, da as
- * tqo_quantize_act writes them): per 32-block the exact sum S = sum c q,
- * then the fixed float schedule acc = acc + (float)S * (2^(E-128) * da),
- * blocks in ascending order (the power of two times da is exact). S_out
- * (nullable) receives S [n][k/32]. Returns 0, -1 on a bad shape or k not a
- * multiple of 256, -4 on a NaN scale, -5 on allocation failure. */
+ * tqo_quantize_act writes them): per 32-block the exact sum S = sum c q and
+ * its value t = (float)S * 2^(E-128) (exact: an integer below 2^16 times a
+ * power of two that binary32 holds, subnormals included; inf past the
+ * range). The float schedule follows the activation's scale unit: per
+ * 256-element block g (eight 32-blocks, one da[g]) G = G + t over its
+ * 32-blocks in ascending order, then acc = acc + G * da[g] over g in
+ * ascending order (each product and sum rounded once). S_out (nullable)
+ * receives S [n][k/32]. Returns 0, -1 on a bad shape or k not a multiple of
+ * 256, -4 on a NaN scale, -5 on allocation failure. */
 int tqo_mxfp4_gemv(const uint8_t *blocks, int64_t n, int64_t k, const int8_t *q, const float *da, float *y,
                    int32_t *S_out) {
     if (tqo_mxfp4_bytes(n, k) < 0 || k % QK) return -1;
     int64_t nb = k / MX_K;
+    const int per_g = QK / MX_K;
     for (int64_t row = 0; row < n; row++) {
         float acc = 0.0f;
-        for (int64_t b = 0; b < nb; b++) {
-            const uint8_t *blk = blocks + (row * nb + b) * MX_BYTES;
-            if (blk[0] == 255) return -4;
-            int32_t s = 0;
-            for (int j = 0; j < MX_K; j++) s += (int32_t)mx_code(mx_nibble(blk, j)) * (int32_t)q[b * MX_K + j];
-            if (S_out) S_out[row * nb + b] = s;
-            float sc = ldexpf(1.0f, (int)blk[0] - 128) * da[(b * MX_K) / QK];
-            acc = acc + (float)s * sc;
+        for (int64_t g = 0; g < k / QK; g++) {
+            float G = 0.0f;
+            for (int64_t b = g * per_g; b < (g + 1) * per_g; b++) {
+                const uint8_t *blk = blocks + (row * nb + b) * MX_BYTES;
+                if (blk[0] == 255) return -4;
+                int32_t s = 0;
+                for (int j = 0; j < MX_K; j++)
+                    s += (int32_t)mx_code(mx_nibble(blk, j)) * (int32_t)q[b * MX_K + j];
+                if (S_out) S_out[row * nb + b] = s;
+                G = G + (float)s * ldexpf(1.0f, (int)blk[0] - 128);
+            }
+            acc = acc + G * da[g];
         }
         y[row] = acc;
     }

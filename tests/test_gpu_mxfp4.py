@@ -1,8 +1,9 @@
 """GPU parity of tqfx4_gemv_mxfp4 (the MXFP4 arm: released expert bytes,
 17 bytes per 32 elements, served by the integer dot pass) against the CPU
 oracle, through the C ABI: int32 block sums bit-exact, fp32 outputs bit-exact
-(both sides run the same binary32 schedule: one block product per 32
-elements, added in ascending block order)."""
+(both sides run the same binary32 schedule: the exact block values of a
+256-element activation group added in block order, each group sum times its
+activation scale added in group order)."""
 import numpy as np
 import pytest
 import torch
