@@ -157,8 +157,8 @@ tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k,
                         void *ws, size_t ws_bytes, void *stream);
 
 /*
- * The MXFP4 arm: the released expert bytes the paper quantizes from (Sec.
- * 2.1; the 4.25-bit row of Table 3), served by the integer dot pass with no
+ * The MXFP4 arm (Sec. 2.3, the expert-lossless arm): the released expert
+ * bytes (4.25 bits/weight in Table 1), served by the integer dot pass with no
  * transcode. Format (OCP microscaling): blocks of 32 consecutive elements of
  * a row, 17 bytes each: byte 0 the e8m0 scale E (2^(E-127); E = 255 is NaN),
  * bytes 1..16 the e2m1 codes (sign, two exponent bits, one mantissa bit:

@@ -421,8 +421,8 @@ int tqo_gemv(const uint8_t *blocks, int64_t n, int64_t k, const int8_t *q, const
 }
 
 /* ------------------------------------------------------------------ */
-/* The MXFP4 arm (the released expert bytes the paper quantizes from,    */
-/* served directly): OCP microscaling blocks of 32 elements, one e8m0    */
+/* The MXFP4 arm (Sec. 2.3: the released expert bytes, served         */
+/* directly): OCP microscaling blocks of 32 elements, one e8m0          */
 /* scale byte E (2^(E-127); E = 255 is NaN) and 32 e2m1 values (sign,    */
 /* two exponent bits, one mantissa bit: 0, 0.5, 1, 1.5, 2, 3, 4, 6), 17 */
 /* bytes per block, 4.25 bits/weight. Readings: the block stores E in    */

@@ -1,4 +1,4 @@
-"""Pins of the oracle's MXFP4 arm (the released expert bytes, Table 3's
+"""Pins of the oracle's MXFP4 arm (the released expert bytes of Sec. 2.3, Table 1's
 4.25-bit format, served directly by an integer dot pass).
 
 Independent characterizations: the OCP microscaling definition of e2m1 from
@@ -35,7 +35,7 @@ def _ref_decode(blocks, n, k):
 
 
 def test_size_is_4_25_bits_per_weight():
-    # Table 3 lists the released MXFP4 bytes at 4.25 bits/weight
+    # Table 1 lists the released MXFP4 bytes at 4.25 bits/weight
     assert oracle.mxfp4_bytes(1024, 1024) * 8 / (1024 * 1024) == 4.25
     assert oracle.mxfp4_bytes(4, 100) < 0
 
