@@ -44,6 +44,8 @@ def lib():
             "tqo_mxfp4_bytes": (i64, [i64, i64]),
             "tqo_mxfp4_dequant": (i32, [vp, i64, i64, vp]),
             "tqo_mxfp4_gemv": (i32, [vp, i64, i64, vp, vp, vp, vp]),
+            "tqo_expert_ffn_mxfp4": (i32, [vp, vp, vp, i64, i64, vp, vp, vp, vp, vp, vp, vp, vp]),
+            "tqo_moe_tokens_fmt": (i32, [i32, vp, vp, vp, i64, i64, i64, vp, vp, i32, vp, i64, vp, vp, vp]),
             "tqo_unpack": (i32, [vp, i64, i64, vp, vp]),
             "tqo_dequant": (i32, [vp, i64, i64, vp]),
             "tqo_quantize_act": (i32, [vp, i64, i64, vp, vp, vp]),
@@ -243,8 +245,9 @@ def swiglu(g, u) -> np.ndarray:
     return h
 
 
-def expert_ffn(gate, up, down, hidden: int, inter: int, x):
-    """One SwiGLU expert; returns (out, debug dict of g, u, h, qh, dh, bh)."""
+def expert_ffn(gate, up, down, hidden: int, inter: int, x, fmt: str = "fx4"):
+    """One SwiGLU expert; returns (out, debug dict of g, u, h, qh, dh, bh).
+    fmt: the weight format of gate, up and down ("fx4" or "mxfp4")."""
     gate, up, down = (_c(a, np.uint8) for a in (gate, up, down))
     x = _c(x, np.float32)
     out = np.empty(hidden, np.float32)
@@ -254,8 +257,9 @@ def expert_ffn(gate, up, down, hidden: int, inter: int, x):
     qh = np.empty(inter, np.int8)
     dh = np.empty(inter // QK, np.float32)
     bh = np.empty(inter // QK, np.int32)
-    _check(lib().tqo_expert_ffn(_p(gate), _p(up), _p(down), hidden, inter, _p(x), _p(out),
-                                _p(g), _p(u), _p(h), _p(qh), _p(dh), _p(bh)), "expert_ffn")
+    fn = {"fx4": lib().tqo_expert_ffn, "mxfp4": lib().tqo_expert_ffn_mxfp4}[fmt]
+    _check(fn(_p(gate), _p(up), _p(down), hidden, inter, _p(x), _p(out),
+              _p(g), _p(u), _p(h), _p(qh), _p(dh), _p(bh)), "expert_ffn")
     return out, dict(g=g, u=u, h=h, qh=qh, dh=dh, bh=bh)
 
 
@@ -286,11 +290,11 @@ def _expert_ptrs(experts, E):
     return arrs, keep
 
 
-def moe_tokens(experts, E: int, hidden: int, inter: int, Wr, bias, top_k: int, X):
+def moe_tokens(experts, E: int, hidden: int, inter: int, Wr, bias, top_k: int, X, fmt: str = "fx4"):
     """Each token of X [T][hidden] through the MoE layer (per-token definition).
 
-    experts: dict expert id -> (gate, up, down) block arrays; experts a token
-    does not select may be absent."""
+    experts: dict expert id -> (gate, up, down) block arrays in format fmt
+    ("fx4" or "mxfp4"); experts a token does not select may be absent."""
     X = _c(X, np.float32)
     if X.ndim == 1:
         X = X[None, :]
@@ -301,8 +305,8 @@ def moe_tokens(experts, E: int, hidden: int, inter: int, Wr, bias, top_k: int, X
     OUT = np.empty((T, hidden), np.float32)
     idx = np.empty((T, top_k), np.int32)
     w = np.empty((T, top_k), np.float32)
-    rc = lib().tqo_moe_tokens(g, u, d, E, hidden, inter, _p(Wr), None if b is None else _p(b),
-                              top_k, _p(X), T, _p(OUT), _p(idx), _p(w))
+    rc = lib().tqo_moe_tokens_fmt({"fx4": 0, "mxfp4": 1}[fmt], g, u, d, E, hidden, inter, _p(Wr),
+                                  None if b is None else _p(b), top_k, _p(X), T, _p(OUT), _p(idx), _p(w))
     del keep
     _check(rc, "moe_tokens")
     return OUT, idx, w

@@ -550,10 +550,17 @@ void tqo_swiglu(const float *g, const float *u, int64_t n, float *h) {
 /* gate, up: [inter][hidden]; down: [hidden][inter]. Optional debug        */
 /* outputs (nullable): g, u, h [inter]; qh [inter]; dh, bh [inter/256].    */
 /* ------------------------------------------------------------------ */
-int tqo_expert_ffn(const uint8_t *gate, const uint8_t *up, const uint8_t *down,
-                   int64_t hidden, int64_t inter, const float *x, float *out,
-                   float *g_dbg, float *u_dbg, float *h_dbg, int8_t *qh_dbg,
-                   float *dh_dbg, int32_t *bh_dbg) {
+/* The dot pass of the expert's weight format: 0 = tq2_0_fx4 blocks,
+ * 1 = MXFP4 blocks (the expert-lossless arm of Sec. 2.3). */
+static int gemv_fmt(int fmt, const uint8_t *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
+                    float *y) {
+    return fmt ? tqo_mxfp4_gemv(blocks, n, k, q, da, y, NULL) : tqo_gemv(blocks, n, k, q, da, y, NULL);
+}
+
+static int expert_ffn_fmt(int fmt, const uint8_t *gate, const uint8_t *up, const uint8_t *down,
+                          int64_t hidden, int64_t inter, const float *x, float *out,
+                          float *g_dbg, float *u_dbg, float *h_dbg, int8_t *qh_dbg,
+                          float *dh_dbg, int32_t *bh_dbg) {
     if (hidden % QK || inter % QK || hidden <= 0 || inter <= 0) return -1;
     int64_t nbh = hidden / QK, nbi = inter / QK;
     int8_t *qx = (int8_t *)malloc((size_t)hidden);
@@ -568,13 +575,13 @@ int tqo_expert_ffn(const uint8_t *gate, const uint8_t *up, const uint8_t *down,
     int rc = -5;
     if (qx && dx && bx && g && u && h && qh && dh && bh) {
         rc = tqo_quantize_act(x, 1, hidden, qx, dx, bx);
-        if (!rc) rc = tqo_gemv(gate, inter, hidden, qx, dx, g, NULL);
-        if (!rc) rc = tqo_gemv(up, inter, hidden, qx, dx, u, NULL);
+        if (!rc) rc = gemv_fmt(fmt, gate, inter, hidden, qx, dx, g);
+        if (!rc) rc = gemv_fmt(fmt, up, inter, hidden, qx, dx, u);
         if (!rc) {
             tqo_swiglu(g, u, inter, h);
             rc = tqo_quantize_act(h, 1, inter, qh, dh, bh);
         }
-        if (!rc) rc = tqo_gemv(down, hidden, inter, qh, dh, out, NULL);
+        if (!rc) rc = gemv_fmt(fmt, down, hidden, inter, qh, dh, out);
         if (!rc) {
             if (g_dbg) memcpy(g_dbg, g, sizeof(float) * (size_t)inter);
             if (u_dbg) memcpy(u_dbg, u, sizeof(float) * (size_t)inter);
@@ -586,6 +593,21 @@ int tqo_expert_ffn(const uint8_t *gate, const uint8_t *up, const uint8_t *down,
     }
     free(qx); free(dx); free(bx); free(g); free(u); free(h); free(qh); free(dh); free(bh);
     return rc;
+}
+
+int tqo_expert_ffn(const uint8_t *gate, const uint8_t *up, const uint8_t *down,
+                   int64_t hidden, int64_t inter, const float *x, float *out,
+                   float *g_dbg, float *u_dbg, float *h_dbg, int8_t *qh_dbg,
+                   float *dh_dbg, int32_t *bh_dbg) {
+    return expert_ffn_fmt(0, gate, up, down, hidden, inter, x, out, g_dbg, u_dbg, h_dbg, qh_dbg, dh_dbg, bh_dbg);
+}
+
+/* The same expert with MXFP4 gate, up and down matrices. */
+int tqo_expert_ffn_mxfp4(const uint8_t *gate, const uint8_t *up, const uint8_t *down,
+                         int64_t hidden, int64_t inter, const float *x, float *out,
+                         float *g_dbg, float *u_dbg, float *h_dbg, int8_t *qh_dbg,
+                         float *dh_dbg, int32_t *bh_dbg) {
+    return expert_ffn_fmt(1, gate, up, down, hidden, inter, x, out, g_dbg, u_dbg, h_dbg, qh_dbg, dh_dbg, bh_dbg);
 }
 
 /* ------------------------------------------------------------------ */
@@ -633,9 +655,10 @@ int tqo_router(const float *Wr, const float *bias, int64_t E, int64_t H, const f
 /* Experts are given as per-expert pointer arrays; an entry may be NULL   */
 /* for an expert the token does not select (returns -6 if it does).       */
 /* ------------------------------------------------------------------ */
-int tqo_moe_token(const uint8_t *const *gate, const uint8_t *const *up, const uint8_t *const *down,
-                  int64_t E, int64_t hidden, int64_t inter, const float *Wr, const float *bias,
-                  int top_k, const float *x, float *out, int32_t *idx, float *w) {
+static int moe_token_fmt(int fmt, const uint8_t *const *gate, const uint8_t *const *up,
+                         const uint8_t *const *down, int64_t E, int64_t hidden, int64_t inter,
+                         const float *Wr, const float *bias, int top_k, const float *x, float *out,
+                         int32_t *idx, float *w) {
     int rc = tqo_router(Wr, bias, E, hidden, x, top_k, NULL, idx, w);
     if (rc) return rc;
     float *o = (float *)malloc(sizeof(float) * (size_t)hidden);
@@ -644,7 +667,7 @@ int tqo_moe_token(const uint8_t *const *gate, const uint8_t *const *up, const ui
     for (int j = 0; j < top_k; j++) {
         int32_t e = idx[j];
         if (!gate[e] || !up[e] || !down[e]) { free(o); return -6; }
-        rc = tqo_expert_ffn(gate[e], up[e], down[e], hidden, inter, x, o,
+        rc = expert_ffn_fmt(fmt, gate[e], up[e], down[e], hidden, inter, x, o,
                             NULL, NULL, NULL, NULL, NULL, NULL);
         if (rc) { free(o); return rc; }
         for (int64_t n = 0; n < hidden; n++) {
@@ -656,17 +679,32 @@ int tqo_moe_token(const uint8_t *const *gate, const uint8_t *const *up, const ui
     return 0;
 }
 
+int tqo_moe_token(const uint8_t *const *gate, const uint8_t *const *up, const uint8_t *const *down,
+                  int64_t E, int64_t hidden, int64_t inter, const float *Wr, const float *bias,
+                  int top_k, const float *x, float *out, int32_t *idx, float *w) {
+    return moe_token_fmt(0, gate, up, down, E, hidden, inter, Wr, bias, top_k, x, out, idx, w);
+}
+
 /* Batched MoE: by definition, each of the T tokens independently through
- * tqo_moe_token. X, OUT: [T][hidden]; idx, w: [T][top_k]. */
-int tqo_moe_tokens(const uint8_t *const *gate, const uint8_t *const *up, const uint8_t *const *down,
-                   int64_t E, int64_t hidden, int64_t inter, const float *Wr, const float *bias,
-                   int top_k, const float *X, int64_t T, float *OUT, int32_t *idx, float *w) {
+ * the one-token layer. X, OUT: [T][hidden]; idx, w: [T][top_k]. fmt: the
+ * experts' weight format (0 tq2_0_fx4, 1 MXFP4). */
+int tqo_moe_tokens_fmt(int fmt, const uint8_t *const *gate, const uint8_t *const *up,
+                       const uint8_t *const *down, int64_t E, int64_t hidden, int64_t inter,
+                       const float *Wr, const float *bias, int top_k, const float *X, int64_t T,
+                       float *OUT, int32_t *idx, float *w) {
+    if (fmt != 0 && fmt != 1) return -1;
     for (int64_t t = 0; t < T; t++) {
-        int rc = tqo_moe_token(gate, up, down, E, hidden, inter, Wr, bias, top_k,
+        int rc = moe_token_fmt(fmt, gate, up, down, E, hidden, inter, Wr, bias, top_k,
                                X + t * hidden, OUT + t * hidden, idx + t * top_k, w + t * top_k);
         if (rc) return rc;
     }
     return 0;
+}
+
+int tqo_moe_tokens(const uint8_t *const *gate, const uint8_t *const *up, const uint8_t *const *down,
+                   int64_t E, int64_t hidden, int64_t inter, const float *Wr, const float *bias,
+                   int top_k, const float *X, int64_t T, float *OUT, int32_t *idx, float *w) {
+    return tqo_moe_tokens_fmt(0, gate, up, down, E, hidden, inter, Wr, bias, top_k, X, T, OUT, idx, w);
 }
 
 /* Token gather per expert (the grouping step of batched decode/prefill):

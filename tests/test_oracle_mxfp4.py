@@ -83,3 +83,61 @@ def test_gemv_against_brute_force(n, k):
     exact = terms.sum(axis=1)
     bound = 2 * (k // 32 + 1) * 2.0 ** -24 * np.abs(terms).sum(axis=1)
     assert np.all(np.abs(y.astype(np.float64) - exact) <= bound)
+
+
+def _mx_expert(seed, hidden, inter):
+    return tuple(inputs.mxfp4_matrix(seed * 3 + p, *shape).numpy()
+                 for p, shape in enumerate(((inter, hidden), (inter, hidden), (hidden, inter))))
+
+
+def test_mxfp4_expert_ffn_tracks_fp64_reference():
+    # the SwiGLU expert over MXFP4 projections, against fp64 on the OCP-decoded weights
+    hidden, inter = 512, 768
+    g, u, d = _mx_expert(3, hidden, inter)
+    x = inputs.hidden_states(4, 1, hidden)[0].numpy()
+    out, dbg = oracle.expert_ffn(g, u, d, hidden, inter, x, fmt="mxfp4")
+    G, _ = _ref_decode(g, inter, hidden)
+    U, _ = _ref_decode(u, inter, hidden)
+    D, _ = _ref_decode(d, hidden, inter)
+    xd = x.astype(np.float64)
+    gg, uu = G @ xd, U @ xd
+    ref = D @ (gg / (1 + np.exp(-gg)) * uu)
+    assert np.abs(out - ref).max() < 0.03 * np.abs(ref).max()
+    bad = D @ (uu / (1 + np.exp(-uu)) * gg)  # gate and up swapped
+    assert np.abs(bad - ref).max() > 0.1 * np.abs(ref).max()
+    # the projections are the MXFP4 dot pass
+    q, da, _ = oracle.quantize_act(x)
+    assert np.array_equal(dbg["g"], oracle.mxfp4_gemv(g, inter, hidden, q, da)[0])
+
+
+def test_mxfp4_moe_tracks_fp64_reference():
+    hidden, inter, E, k = 512, 512, 8, 3
+    ex = {e: _mx_expert(10 + e, hidden, inter) for e in range(E)}
+    Wr = inputs.router_weight(5, E, hidden).numpy()
+    X = inputs.hidden_states(6, 3, hidden).numpy()
+    out, idx, w = oracle.moe_tokens(ex, E, hidden, inter, Wr, None, k, X, fmt="mxfp4")
+    for t in range(3):
+        l = Wr.astype(np.float64) @ X[t].astype(np.float64)
+        sel = np.lexsort((np.arange(E), -l))[:k]
+        assert np.array_equal(idx[t], sel)
+        p = np.exp(l[sel] - l[sel].max())
+        p /= p.sum()
+        ref = np.zeros(hidden)
+        for j, e in enumerate(sel):
+            G, _ = _ref_decode(ex[e][0], inter, hidden)
+            U, _ = _ref_decode(ex[e][1], inter, hidden)
+            D, _ = _ref_decode(ex[e][2], hidden, inter)
+            gg, uu = G @ X[t], U @ X[t]
+            ref += p[j] * (D @ (gg / (1 + np.exp(-gg)) * uu))
+        assert np.abs(out[t] - ref).max() < 0.03 * np.abs(ref).max()
+
+
+def test_mxfp4_moe_single_expert_reduces_to_the_ffn():
+    hidden, inter = 512, 512
+    ex = {0: _mx_expert(30, hidden, inter)}
+    Wr = np.zeros((1, hidden), np.float32)
+    x = inputs.hidden_states(31, 1, hidden)[0].numpy()
+    out, idx, w = oracle.moe_tokens(ex, 1, hidden, inter, Wr, None, 1, x, fmt="mxfp4")
+    ffn, _ = oracle.expert_ffn(*ex[0], hidden, inter, x, fmt="mxfp4")
+    assert idx[0, 0] == 0 and w[0, 0] == 1.0
+    assert np.array_equal(out[0], ffn)
