@@ -13,7 +13,8 @@ router weights) per token / time per token; tokens/s per MoE layer is the
 same number divided by the bytes per token, reported beside it.
 
     python bench.py [--steps K] [--warmup W] [--gpus N] [--impl ours|reference]
-                    [--workload moe_decode|grouped_decode_64|prefill_2048|tiered_decode|mxfp4_gemv]
+                    [--workload moe_decode|grouped_decode_64|prefill_2048|tiered_decode|mxfp4_gemv|
+                                moe_decode_mxfp4]
 
 The K timed steps are captured once into a CUDA graph and replayed inside
 the timed region (no host launch work in it); the other workloads time
@@ -42,6 +43,8 @@ SEED = 0
 POOL = 256  # distinct hidden states cycled through the steps
 WORKLOAD = "moe_decode_t1_e256_h4096_i2048_top8"
 METRIC = "effective tq2_0_fx4 GB/s (MoE-layer decode)"
+WORKLOAD_MX = "moe_decode_mxfp4_t1_e256_h4096_i2048_top8"
+METRIC_MX = "effective MXFP4 GB/s (MoE-layer decode)"
 
 
 def _peaks():
@@ -89,10 +92,13 @@ def _tensor_peak():
         return 1700.0, "fallback 1.7 PFLOP/s sustained"
 
 
-def bytes_per_token():
+def bytes_per_token(layer=None):
+    """(bytes one token reads: the selected experts' blocks and the router;
+    gate/up bytes; down bytes), tq2_0_fx4 unless a layer says otherwise."""
     from paper_2608_08910_gb300 import binding as B
-    mb = B.tqfx4_matrix_bytes(I, H)  # gate = up = down size
-    return TOPK * 3 * mb + E * H * 4, TOPK * 2 * mb, TOPK * mb
+    mg = layer.mb_gu if layer is not None else B.tqfx4_matrix_bytes(I, H)
+    md = layer.mb_d if layer is not None else B.tqfx4_matrix_bytes(H, I)
+    return TOPK * (2 * mg + md) + E * H * 4, TOPK * 2 * mg, TOPK * md
 
 
 class ClockSampler:
@@ -147,10 +153,11 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(self.samples)}
 
 
-def cpu_baseline(seconds_budget=20.0, tokens=None):
+def cpu_baseline(seconds_budget=20.0, tokens=None, layer=None):
     """The oracle (plain single-threaded C) on a bounded sample of the same
     workload: whole tokens through the MoE layer, packing of the experts they
-    select excluded from the time. Returns (GB/s, tokens, seconds)."""
+    select excluded from the time (layer: an MXFP4 layer whose expert bytes
+    the oracle reads instead). Returns (GB/s, tokens, seconds)."""
     import numpy as np
     import torch
 
@@ -160,15 +167,18 @@ def cpu_baseline(seconds_budget=20.0, tokens=None):
     dev = "cuda" if torch.cuda.is_available() else "cpu"
     Wr = inputs.router_weight(SEED, E, H, dev).cpu().numpy()
     X = inputs.hidden_states(SEED, POOL, H, dev).cpu().numpy()
-    per_token, _, _ = bytes_per_token()
+    per_token, _, _ = bytes_per_token(layer)
     total_t, done = 0.0, 0
     n_max = tokens if tokens else POOL
     for t in range(n_max):
         _, idx, _ = oracle.router(Wr, None, X[t], TOPK)
-        ex = {int(e): tuple(oracle.pack_rtn(inputs.expert_matrix(SEED, int(e), p, H, I, dev).cpu().numpy())
-                            for p in (0, 1, 2)) for e in idx}
+        if layer is not None:
+            ex = {int(e): tuple(b.cpu().numpy() for b in layer.expert_blocks(int(e))) for e in idx}
+        else:
+            ex = {int(e): tuple(oracle.pack_rtn(inputs.expert_matrix(SEED, int(e), p, H, I, dev).cpu().numpy())
+                                for p in (0, 1, 2)) for e in idx}
         t0 = time.perf_counter()
-        oracle.moe_tokens(ex, E, H, I, Wr, None, TOPK, X[t])
+        oracle.moe_tokens(ex, E, H, I, Wr, None, TOPK, X[t], fmt="mxfp4" if layer is not None else "fx4")
         total_t += time.perf_counter() - t0
         done += 1
         if tokens is None and total_t >= seconds_budget:
@@ -652,10 +662,12 @@ def main():
     ap.add_argument("--tokens", type=int, default=0,
                     help="tokens per step of the grouped workloads (default: 64 or 2048; profiling only)")
     ap.add_argument("--workload", default="moe_decode",
-                    choices=["moe_decode", "grouped_decode_64", "prefill_2048", "tiered_decode", "mxfp4_gemv"],
+                    choices=["moe_decode", "grouped_decode_64", "prefill_2048", "tiered_decode", "mxfp4_gemv",
+                             "moe_decode_mxfp4"],
                     help="moe_decode (default): 1 token; grouped_decode_64: 64 tokens with Zipf(1.1) "
                          "routing; prefill_2048: 2048 tokens; tiered_decode: 1 token with the experts in "
-                         "host memory; mxfp4_gemv: one GEMV over MXFP4 blocks")
+                         "host memory; mxfp4_gemv: one GEMV over MXFP4 blocks; moe_decode_mxfp4: moe_decode with "
+                         "MXFP4 experts")
     ap.add_argument("--slots", type=int, default=TOPK, help="device expert slots of tiered_decode")
     args = ap.parse_args()
     globals()["E"] = args.experts
@@ -673,9 +685,10 @@ def main():
     if args.workload == "mxfp4_gemv":
         run_gemv(args, rank, world, local)
         return
-    if args.workload != "moe_decode":
+    if args.workload not in ("moe_decode", "moe_decode_mxfp4"):
         run_grouped(args, rank, world, local)
         return
+    mx = args.workload == "moe_decode_mxfp4"
 
     import torch
     import torch.distributed as dist
@@ -690,14 +703,14 @@ def main():
 
     assert args.warmup >= 3, "at least 3 warm-up steps"
     dev = torch.device("cuda", local)
-    layer = MoeLayer.synthetic(SEED, E, H, I, TOPK, 0.0, dev)
+    layer = (MoeLayer.synthetic_mxfp4 if mx else MoeLayer.synthetic)(SEED, E, H, I, TOPK, 0.0, dev)
     ws = layer.workspace(1)
     X = inputs.hidden_states(SEED + rank, POOL, H, dev)
     out = torch.empty(H, device=dev)
     sel = torch.empty(TOPK, dtype=torch.int32, device=dev)
     selw = torch.empty(TOPK, device=dev)
     stream = torch.cuda.current_stream(dev)
-    per_token, gu_bytes, dn_bytes = bytes_per_token()
+    per_token, gu_bytes, dn_bytes = bytes_per_token(layer)
 
     def step(i, events=None, st=stream):
         layer.ffn(X[i % POOL], ws, out, sel, selw, stream=st, events=events)
@@ -742,8 +755,9 @@ def main():
     # ---- dominant kernel: CUDA events around every stage of every step, on
     # the launching stream (a second graph of the same K steps; the stage
     # launches are plain stream-ordered here) ----
-    n_st = B.tqfx4_moe_stage_count(0, 0)
-    names = [B.tqfx4_moe_stage_name(0, 0, s) for s in range(n_st)]
+    kind = 2 if mx else 0
+    n_st = B.tqfx4_moe_stage_count(kind, 0)
+    names = [B.tqfx4_moe_stage_name(kind, 0, s) for s in range(n_st)]
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_st + 1)] for _ in range(args.steps)]
     for row in evs:
         for e_ in row:
@@ -791,28 +805,32 @@ def main():
     e2e = per_token * tokens / te / 1e9
 
     line = {
-        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "metric": METRIC_MX if mx else METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "i8xi4-i32,f32", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "experts": E, "hidden": H, "inter": I, "top_k": TOPK,
-                   "tokens_per_step": 1, "bytes_per_token": per_token,
-                   "l2": "inputs larger than L2: 3.27 GB expert pool, a different hidden state per step",
+        "scaling": "weak", "vs_baseline": None, "dtype": "i8xe2m1-i32,f32" if mx else "i8xi4-i32,f32",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD_MX if mx else WORKLOAD, "experts": E, "hidden": H, "inter": I,
+                   "top_k": TOPK, "tokens_per_step": 1, "bytes_per_token": per_token,
+                   "l2": "inputs larger than L2: %.2f GB expert pool, a different hidden state per step"
+                         % ((2 * layer.mb_gu + layer.mb_d) * E / 1e9),
                    "parallelism": "replicas" if world > 1 else "single"},
         "tokens_per_s": tokens / t,
         "pct_of_hbm_peak": 100.0 * value / peak,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": GATE_UP_TRAFFIC, "kernel": dom,
+                     "frac": achieved / peak, "traffic": None if mx else GATE_UP_TRAFFIC,
+                     "kernel": "mxfp4_gemv_kernel (gate_up)" if mx else dom,
                      "traffic_source": "ncu capture (dram__bytes_read + write) of one gate_up_kernel launch",
                      "peak_source": peak_kind + " (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
                      else "fallback 6.8 TB/s",
                      "stage_us": {k: v * 1e6 for k, v in stage_s.items()}},
         "e2e": {"value": e2e, "unit": "GB/s", "h2d_bytes_per_step": H * 4,
                 "d2h_bytes_per_step": H * 4 + TOPK * 4},
-        "gpu_launches": 3 * args.steps,
+        # router, gate_up, down (tq2_0_fx4); router, gate_up, down, combine (MXFP4)
+        "gpu_launches": (4 if mx else 3) * args.steps,
         "clocks": clk.summary(),
     }
     if rank == 0 and not args.no_cpu_baseline:
-        v, n, secs = cpu_baseline()
+        v, n, secs = cpu_baseline(layer=layer if mx else None)
         line["cpu_baseline"] = {"value": v, "unit": "GB/s", "cores": 1, "kind": "oracle",
                                 "sample": "%d tokens through the layer (%.1f s), expert packing excluded" % (n, secs)}
     if rank == 0:

@@ -241,6 +241,28 @@ tqfx4_status tqfx4_moe_ffn(const tqfx4_experts *ex, const tqfx4_router *rt,
                            void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * tqfx4_moe_ffn_mxfp4 -- tqfx4_moe_ffn with MXFP4 experts (the
+ * expert-lossless arm, Sec. 2.3: the released expert bytes served by the
+ * same engine): ex->gate, up and down hold the stacked experts in the MXFP4
+ * layout of tqfx4_gemv_mxfp4, each expert projection
+ * tqfx4_mxfp4_bytes(rows, cols) contiguous bytes at base + e * that size.
+ * Routing, the activation quantizer, SwiGLU and the rank-order combine are
+ * tqfx4_moe_ffn's; each projection is tqfx4_gemv_mxfp4's dot pass. hidden
+ * and inter must be multiples of 512. Workspace: tqfx4_moe_workspace_bytes
+ * with tokens == 1. A NaN scale in a selected expert sets TQFX4_EDATA.
+ */
+tqfx4_status tqfx4_moe_ffn_mxfp4(const tqfx4_experts *ex, const tqfx4_router *rt,
+                                 const float *x, float *out, int32_t *sel_idx, float *sel_w,
+                                 void *ws, size_t ws_bytes, void *stream);
+/* The same, recording events[0..4] around its stages (router, gate_up,
+ * down with SwiGLU and the quantization of h in its prologue, combine:
+ * tqfx4_moe_stage_count(2, 0) == 4 and tqfx4_moe_stage_name(2, 0, i)); the
+ * stages then run without programmatic dependent launch. */
+tqfx4_status tqfx4_moe_ffn_mxfp4_traced(const tqfx4_experts *ex, const tqfx4_router *rt,
+                                        const float *x, float *out, int32_t *sel_idx, float *sel_w,
+                                        void *ws, size_t ws_bytes, void *stream, void *const *events);
+
+/*
  * tqfx4_moe_route and tqfx4_moe_experts -- tqfx4_moe_ffn in two calls, for
  * callers that place the selected experts' blocks themselves between the
  * routing decision and the expert projections: an expert tier that keeps

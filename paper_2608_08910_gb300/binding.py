@@ -61,6 +61,9 @@ _SIGS = {
     "tqfx4_gemv": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int]),
     "tqfx4_moe_ffn": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_moe_ffn_mxfp4": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_moe_ffn_mxfp4_traced": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz,
+                                          _vp, C.POINTER(_vp)]),
     "tqfx4_moe_grouped": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _i64, _vp, _vp, _vp, _int,
                                  _vp, _sz, _vp]),
     "tqfx4_moe_stage_count": (_int, [_int, _int]),
@@ -173,6 +176,17 @@ def tqfx4_moe_ffn(ex, rt, x, out, sel_idx, sel_w, ws, stream=None, events=None):
         rc = lib().tqfx4_moe_ffn_traced(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w),
                                         _p(ws), _nbytes(ws), _s(stream), arr)
     _check(rc, "tqfx4_moe_ffn")
+
+
+def tqfx4_moe_ffn_mxfp4(ex, rt, x, out, sel_idx, sel_w, ws, stream=None, events=None):
+    if events is None:
+        rc = lib().tqfx4_moe_ffn_mxfp4(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w), _p(ws),
+                                       _nbytes(ws), _s(stream))
+    else:
+        arr = (_vp * len(events))(*[e.cuda_event if hasattr(e, "cuda_event") else e for e in events])
+        rc = lib().tqfx4_moe_ffn_mxfp4_traced(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w),
+                                              _p(ws), _nbytes(ws), _s(stream), arr)
+    _check(rc, "tqfx4_moe_ffn_mxfp4")
 
 
 def tqfx4_moe_ffn_noalloc(ex, rt, x, out, sel_idx, sel_w, stream=None):

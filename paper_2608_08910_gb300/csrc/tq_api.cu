@@ -182,12 +182,15 @@ size_t tqfx4_moe_workspace_bytes(const tqfx4_experts *ex, const tqfx4_router *rt
 
 int tqfx4_moe_stage_count(int grouped, int path) {
     (void)path;
+    if (grouped == 2) return 4;
     return grouped ? tq::grouped_stage_count() : 3;
 }
 
 const char *tqfx4_moe_stage_name(int grouped, int path, int stage) {
     (void)path;
     static const char *dec[] = {"router", "gate_up", "down"};
+    static const char *mx[] = {"router", "gate_up", "down", "combine"};
+    if (grouped == 2) return (stage >= 0 && stage < 4) ? mx[stage] : "";
     if (grouped) return tq::grouped_stage_name(stage);
     if (stage >= 0 && stage < 3) return dec[stage];
     return "";
@@ -247,6 +250,50 @@ tqfx4_status tqfx4_moe_route(const tqfx4_experts *ex, const tqfx4_router *rt, co
     cudaError_t e = tq::launch_moe_route(a, x, sel_idx, sel_w, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, fn);
     return ok();
+}
+
+static tqfx4_status moe_ffn_mxfp4_impl(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x,
+                                       float *out, int32_t *sel_idx, float *sel_w, void *ws, size_t ws_bytes,
+                                       void *stream, void *const *events) {
+    const char *fn = "tqfx4_moe_ffn_mxfp4";
+    tqfx4_status s = check_moe_shapes(ex, rt, fn);
+    if (s) return s;
+    if (ex->hidden % 512 || ex->inter % 512)
+        return fail(TQFX4_ESHAPE, "%s: hidden and inter must be multiples of 512", fn);
+    if (!ex->gate || !ex->up || !ex->down || !rt->weight) return fail(TQFX4_EINVAL, "%s: NULL expert or router weights", fn);
+    if (!x || !out || !sel_idx || !sel_w) return fail(TQFX4_EINVAL, "%s: NULL input or output", fn);
+    if (!aligned(ex->gate, 16) || !aligned(ex->up, 16) || !aligned(ex->down, 16) || !aligned(rt->weight, 16) ||
+        !aligned(rt->bias, 4) || !aligned(x, 16) || !aligned(out, 4) || !aligned(sel_idx, 4) || !aligned(sel_w, 4))
+        return fail(TQFX4_EALIGN, "%s: expert blocks, router weights and x must be 16-byte aligned", fn);
+    tq::MoeArgs a;
+    tq::MoeLayout L;
+    if (!tq::moe_decode_args(ex, rt, nullptr, a, L))
+        return fail(TQFX4_ESHAPE, "%s: too many row ranges for the counter area", fn);
+    if ((s = check_ws(ws, ws_bytes, L.total, fn))) return s;
+    if (tq::mxfp4_gemv_smem(ex->hidden, 1) > tq::max_smem_optin() ||
+        tq::mxfp4_gemv_smem(ex->inter, rt->top_k) > tq::max_smem_optin())
+        return fail(TQFX4_ESHAPE, "%s: top_k x inter too large for the kernels' shared memory", fn);
+    tq::moe_decode_args(ex, rt, ws, a, L);
+    a.mb_gu = tq::mxfp4_bytes(ex->inter, ex->hidden);
+    a.mb_d = tq::mxfp4_bytes(ex->hidden, ex->inter);
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaEvent_t const *ev = reinterpret_cast<cudaEvent_t const *>(events);
+    cudaError_t e = ev ? tq::record_stage_event(ev[0], st) : cudaSuccess;
+    if (e == cudaSuccess) e = tq::launch_moe_route(a, x, sel_idx, sel_w, st);
+    if (e == cudaSuccess) e = tq::launch_moe_mxfp4_experts(a, out, st, ev ? ev + 1 : nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
+tqfx4_status tqfx4_moe_ffn_mxfp4(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, float *out,
+                                 int32_t *sel_idx, float *sel_w, void *ws, size_t ws_bytes, void *stream) {
+    return moe_ffn_mxfp4_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, nullptr);
+}
+
+tqfx4_status tqfx4_moe_ffn_mxfp4_traced(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x,
+                                        float *out, int32_t *sel_idx, float *sel_w, void *ws, size_t ws_bytes,
+                                        void *stream, void *const *events) {
+    return moe_ffn_mxfp4_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, events);
 }
 
 tqfx4_status tqfx4_moe_experts(const tqfx4_experts *ex, const tqfx4_router *rt, const void *const *ptrs, float *out,

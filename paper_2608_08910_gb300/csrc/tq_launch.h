@@ -31,6 +31,16 @@ int gate_up_smem(const MoeArgs &a);
 int64_t mxfp4_bytes(int64_t n, int64_t k);
 cudaError_t launch_mxfp4_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da, float *y,
                               int32_t *block_sums, int *status, cudaStream_t st);
+// Records a stage event on `st`; inside a stream capture it becomes an
+// external event node, so that the event keeps its timing meaning on replay.
+inline cudaError_t record_stage_event(cudaEvent_t ev, cudaStream_t st) {
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    cudaStreamIsCapturing(st, &cap);
+    return cudaEventRecordWithFlags(ev, st, cap == cudaStreamCaptureStatusActive ? cudaEventRecordExternal
+                                                                                  : cudaEventRecordDefault);
+}
+int mxfp4_gemv_smem(int64_t k, int acts);
+cudaError_t launch_moe_mxfp4_experts(const MoeArgs &a, float *out, cudaStream_t st, const cudaEvent_t *ev);
 cudaError_t launch_moe_route(const MoeArgs &a, const float *x, int32_t *sel_idx, float *sel_w, cudaStream_t st);
 cudaError_t launch_moe_experts(const MoeArgs &a, const void *const *ptrs, float *out, cudaStream_t st);
 

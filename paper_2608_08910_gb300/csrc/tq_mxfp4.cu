@@ -32,6 +32,7 @@
 // tile is decoded.
 #include "tq_common.cuh"
 #include "tq_launch.h"
+#include "tq_moe_common.cuh"
 
 namespace tq {
 
@@ -51,11 +52,35 @@ struct MxGeo {
     int slot;       // ring slot bytes (a tile, a multiple of 16)
 };
 
-// activation region: q interleaved (k bytes), -128 * sum q per block (8 L
-// ints), da (L floats), then 2^(E-128) for E = 0..255
-__host__ __device__ inline int mx_act_bytes(const MxGeo &g) {
-    return static_cast<int>(((g.k + 36 * g.L + 127) / 128) * 128) + 1024;
+// activation region: per activation q interleaved (k bytes), -128 * sum q
+// per block (8 L ints) and da (L floats); then 2^(E-128) for E = 0..255
+__host__ __device__ inline int mx_act_unit(const MxGeo &g) { return static_cast<int>(((g.k + 36 * g.L + 15) / 16) * 16); }
+__host__ __device__ inline int mx_act_bytes(const MxGeo &g, int acts) {
+    return ((acts * mx_act_unit(g) + 127) / 128) * 128 + 1024;
 }
+
+// The matrices of one launch, all n x k: matrix m (of n_mat <= 2K) is
+// base[m / K] + sel[m % K] * mat_bytes (sel null: base[m / K]), takes
+// activation m % K when acts > 1 (else the only one), and writes y[m / K] +
+// (m % K) * n. One matrix: K = 1, n_mat = 1 (block sums only then).
+struct MxJob {
+    const uint8_t *base[2];
+    int64_t mat_bytes;
+    const int32_t *sel;
+    int K, n_mat, acts;
+    const int8_t *q;  // [acts][k]
+    const float *da;  // [acts][k / 256]
+    float *y[2];
+    int32_t *S;  // nullable block sums [n_mat * n][k / 32]
+    // per-matrix mode: CTA c serves matrix c % K only, and builds its
+    // activation as the int8 quantization of h = silu(g_j) * u_j from these
+    // ([K][k] fp32 each) instead of reading q and da
+    const float *g, *u;
+};
+
+// Kernel modes: one matrix; several matrices sharing the CTAs; several
+// matrices with the CTAs split among them (activation from g and u).
+enum { MX_ONE = 0, MX_SHARED = 1, MX_PER_MAT = 2 };
 constexpr int MX_SLOTS = 3;
 __host__ __device__ inline int mx_warp_bytes(const MxGeo &g) { return MX_SLOTS * g.slot + 4 * 32 * g.J + 32; }
 
@@ -142,38 +167,21 @@ __device__ __forceinline__ bool mx_wait(uint64_t *bar, uint32_t parity) {
     }
 }
 
-template <bool kSums>
-__global__ void __launch_bounds__(MX_WARPS * 32) mxfp4_gemv_kernel(const uint8_t *__restrict__ blocks, MxGeo g,
-                                                                   const int8_t *__restrict__ q,
-                                                                   const float *__restrict__ da, float *__restrict__ y,
-                                                                   int32_t *__restrict__ S_out, int *status) {
-    extern __shared__ __align__(128) uint8_t smem[];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+// Stages activation `a` (q [k] int8, da [k/256]) into the interleaved layout.
+__device__ __forceinline__ void mx_stage_act(uint8_t *dst, const MxGeo &g, const int8_t *q, const float *da) {
     const int L = g.L;
-    uint4 *qv = reinterpret_cast<uint4 *>(smem);  // [8 blocks][2 halves][L groups]
-    int *qc = reinterpret_cast<int *>(smem + g.k);  // [8 blocks][L groups]
-    float *das = reinterpret_cast<float *>(smem + g.k + 32 * L);
-    float *p2 = reinterpret_cast<float *>(smem + mx_act_bytes(g) - 1024);
-    uint8_t *wbase = smem + mx_act_bytes(g) + warp * mx_warp_bytes(g);
-    uint8_t *slots = wbase;
-    float *tb = reinterpret_cast<float *>(wbase + MX_SLOTS * g.slot);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(wbase + MX_SLOTS * g.slot + 4 * 32 * g.J);
-    if (lane == 0)
-        for (int i = 0; i < MX_SLOTS; ++i) mbar_init(&bars[i], 1);
-    fence_barrier_init();
-    // the activation, interleaved per 16-element half block: bytes
-    // q[8h + e] and q[16 + 8h + e] alternate
-    for (int idx = threadIdx.x; idx < 16 * L; idx += blockDim.x) {
-        const int grp = idx % L, jh = idx / L;
-        const int8_t *src = q + static_cast<int64_t>(grp) * QK + (jh >> 1) * MX_K + (jh & 1) * 8;
-        const uint2 a = __ldg(reinterpret_cast<const uint2 *>(src));
-        const uint2 b = __ldg(reinterpret_cast<const uint2 *>(src + 16));
-        qv[idx] = make_uint4(__byte_perm(a.x, b.x, 0x5140), __byte_perm(a.x, b.x, 0x7362),
-                             __byte_perm(a.y, b.y, 0x5140), __byte_perm(a.y, b.y, 0x7362));
+    for (int r = threadIdx.x; r < 16 * L; r += blockDim.x) {
+        const int grp = r % L, jh = r / L;
+        const int8_t *src = q + grp * QK + (jh >> 1) * MX_K + (jh & 1) * 8;
+        const uint2 x0 = __ldg(reinterpret_cast<const uint2 *>(src));
+        const uint2 x1 = __ldg(reinterpret_cast<const uint2 *>(src + 16));
+        reinterpret_cast<uint4 *>(dst)[r] =
+            make_uint4(__byte_perm(x0.x, x1.x, 0x5140), __byte_perm(x0.x, x1.x, 0x7362),
+                       __byte_perm(x0.y, x1.y, 0x5140), __byte_perm(x0.y, x1.y, 0x7362));
     }
-    for (int idx = threadIdx.x; idx < 8 * L; idx += blockDim.x) {
-        const int grp = idx % L, j = idx / L;
-        const uint4 *src = reinterpret_cast<const uint4 *>(q + static_cast<int64_t>(grp) * QK + j * MX_K);
+    for (int r = threadIdx.x; r < 8 * L; r += blockDim.x) {
+        const int grp = r % L, j = r / L;
+        const uint4 *src = reinterpret_cast<const uint4 *>(q + grp * QK + j * MX_K);
         int sum = 0;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
@@ -183,31 +191,115 @@ __global__ void __launch_bounds__(MX_WARPS * 32) mxfp4_gemv_kernel(const uint8_t
             sum = __dp4a(static_cast<int>(v.z), 0x01010101, sum);
             sum = __dp4a(static_cast<int>(v.w), 0x01010101, sum);
         }
-        qc[idx] = -128 * sum;
+        reinterpret_cast<int *>(dst + g.k)[r] = -128 * sum;
     }
-    for (int i = threadIdx.x; i < L; i += blockDim.x) das[i] = __ldg(da + i);
+    for (int r = threadIdx.x; r < L; r += blockDim.x) reinterpret_cast<float *>(dst + g.k + 32 * L)[r] = __ldg(da + r);
+}
+
+// Builds the activation from h = silu(g) * u (k elements, fp32): one warp
+// per 256-element block, the decode path's SwiGLU and quantizer, written
+// straight into the interleaved layout. Returns false if h is not finite.
+__device__ __forceinline__ bool mx_stage_swiglu(uint8_t *dst, const MxGeo &g, const float *gv, const float *uv) {
+    const int L = g.L, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    bool ok = true;
+    for (int b = warp; b < L; b += MX_WARPS) {
+        const int o = b * QK + 8 * lane;
+        const float4 g0 = __ldcg(reinterpret_cast<const float4 *>(gv + o));
+        const float4 g1 = __ldcg(reinterpret_cast<const float4 *>(gv + o) + 1);
+        const float4 u0 = __ldcg(reinterpret_cast<const float4 *>(uv + o));
+        const float4 u1 = __ldcg(reinterpret_cast<const float4 *>(uv + o) + 1);
+        const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+        const float uu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+        float hv[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) hv[i] = tq_swiglu(gg[i], uu[i]);
+        uint2 pk;
+        float d;
+        int bsum;
+        ok &= quant_block_warp(hv, pk, d, bsum);
+        // lane holds elements 8 (lane % 4) .. + 7 of 32-block lane / 4: the
+        // half-block words pair lanes l and l + 2 (elements e and 16 + e)
+        const uint2 hi = make_uint2(__shfl_down_sync(0xffffffffu, pk.x, 2), __shfl_down_sync(0xffffffffu, pk.y, 2));
+        const int jb = lane >> 2, part = lane & 3;
+        if (part < 2)
+            reinterpret_cast<uint4 *>(dst)[(2 * jb + part) * L + b] =
+                make_uint4(__byte_perm(pk.x, hi.x, 0x5140), __byte_perm(pk.x, hi.x, 0x7362),
+                           __byte_perm(pk.y, hi.y, 0x5140), __byte_perm(pk.y, hi.y, 0x7362));
+        int sum = __dp4a(static_cast<int>(pk.x), 0x01010101, __dp4a(static_cast<int>(pk.y), 0x01010101, 0));
+        sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+        sum += __shfl_xor_sync(0xffffffffu, sum, 2);
+        if (part == 0) reinterpret_cast<int *>(dst + g.k)[jb * L + b] = -128 * sum;
+        if (lane == 0) reinterpret_cast<float *>(dst + g.k + 32 * L)[b] = d;
+    }
+    return ok;
+}
+
+template <bool kSums, int kMode>
+__global__ void __launch_bounds__(MX_WARPS * 32) mxfp4_gemv_kernel(MxGeo g, MxJob job, int *status) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int L = g.L, AU = mx_act_unit(g);
+    const int acts = kMode == MX_SHARED ? job.acts : 1;
+    const int act_bytes = mx_act_bytes(g, acts);
+    float *p2 = reinterpret_cast<float *>(smem + act_bytes - 1024);
+    uint8_t *wbase = smem + act_bytes + warp * mx_warp_bytes(g);
+    uint8_t *slots = wbase;
+    float *tb = reinterpret_cast<float *>(wbase + MX_SLOTS * g.slot);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(wbase + MX_SLOTS * g.slot + 4 * 32 * g.J);
+    if (lane == 0)
+        for (int i = 0; i < MX_SLOTS; ++i) mbar_init(&bars[i], 1);
+    fence_barrier_init();
     // 2^(E-128) for E = 0..254 (0 and 1 subnormal); E = 255 is flagged, its entry unused
     for (int E = threadIdx.x; E < 256; E += blockDim.x)
         p2[E] = __int_as_float(E >= 2 ? (E - 1) << 23 : 0x00200000 << E);
-    __syncthreads();
+    // everything below may read the previous kernel's results
+    grid_dependency_wait();
 
-    const int64_t tiles = (g.n + g.R - 1) / g.R;
-    const int64_t NW = static_cast<int64_t>(gridDim.x) * MX_WARPS;
-    const int64_t first = static_cast<int64_t>(blockIdx.x) * MX_WARPS + warp;
+    const int tpm = static_cast<int>((g.n + g.R - 1) / g.R);  // tiles per matrix
+    // the CTA's matrix (per-matrix mode) and the tiles its warps take
+    const int cta_m = kMode == MX_PER_MAT ? static_cast<int>(blockIdx.x) % job.K : 0;
+    const int cta_p = kMode == MX_PER_MAT ? static_cast<int>(blockIdx.x) / job.K : static_cast<int>(blockIdx.x);
+    const int n_cta = kMode == MX_PER_MAT ? static_cast<int>(gridDim.x) / job.K : static_cast<int>(gridDim.x);
+    const int tiles = kMode == MX_SHARED ? tpm * job.n_mat : tpm;
+    const int NW = n_cta * MX_WARPS;
+    const int first = cta_p * MX_WARPS + warp;
     const uint64_t policy = l2_policy_evict_first();
-    auto rows_of = [&](int64_t tile) {
-        const int64_t left = g.n - tile * g.R;
+    auto locate = [&](int tile, int &m, int &t) {
+        m = kMode == MX_SHARED ? tile / tpm : cta_m;
+        t = tile - (kMode == MX_SHARED ? m * tpm : 0);
+    };
+    auto rows_of = [&](int t) {
+        const int64_t left = g.n - static_cast<int64_t>(t) * g.R;
         return static_cast<int>(left < g.R ? left : g.R);
     };
-    auto issue = [&](int64_t tile, int s) {
+    auto issue = [&](int tile, int s) {
         if (lane == 0) {
-            const uint32_t bytes = static_cast<uint32_t>(rows_of(tile) * g.row_bytes);
+            int m, t;
+            locate(tile, m, t);
+            const uint8_t *mat = job.base[0];
+            if (kMode != MX_ONE)
+                mat = (m >= job.K ? job.base[1] : job.base[0]) + (job.sel ? job.sel[m % job.K] : 0) * job.mat_bytes;
+            const uint32_t bytes = static_cast<uint32_t>(rows_of(t) * g.row_bytes);
             mbar_arrive_expect_tx(&bars[s], bytes);
-            bulk_g2s_hint(slots + s * g.slot, blocks + tile * g.R * g.row_bytes, bytes, &bars[s], policy);
+            bulk_g2s_hint(slots + s * g.slot, mat + static_cast<int64_t>(t) * g.R * g.row_bytes, bytes, &bars[s],
+                          policy);
         }
     };
+    // the first weight tiles go out before the activation is staged
     if (first < tiles) issue(first, 0);
     if (first + NW < tiles) issue(first + NW, 1);
+    if (kMode == MX_PER_MAT) {
+        if (!mx_stage_swiglu(smem, g, job.g + static_cast<int64_t>(cta_m) * g.k,
+                             job.u + static_cast<int64_t>(cta_m) * g.k) &&
+            lane == 0)
+            report(status, TQFX4_EDATA, K_DOWN, cta_m);
+    } else {
+        for (int a = 0; a < acts; ++a)
+            mx_stage_act(smem + a * AU, g, job.q + static_cast<int64_t>(a) * g.k, job.da + static_cast<int64_t>(a) * L);
+    }
+    __syncthreads();
+    grid_dependents_launch();
+
     const int nb = L * (QK / MX_K);
     // this lane's groups of a tile: row gr[jj] (R when the lane has none), group gg[jj] of the row
     int gr[2], gg[2];
@@ -219,9 +311,9 @@ __global__ void __launch_bounds__(MX_WARPS * 32) mxfp4_gemv_kernel(const uint8_t
     }
     uint32_t emax = 0;
     int s = 0, ph = 0;  // slot of this tile, and the parity of its barrier
-    for (int64_t tile = first; tile < tiles; tile += NW) {
+    for (int tile = first; tile < tiles; tile += NW) {
         if (!__all_sync(0xffffffffu, mx_wait(&bars[s], static_cast<uint32_t>(ph)))) {
-            if (lane == 0) report(status, TQFX4_ETIMEOUT, K_GEMV, static_cast<int>(tile));
+            if (lane == 0) report(status, TQFX4_ETIMEOUT, K_GEMV, tile);
             break;
         }
         // the slot that held the previous tile (read by every lane before
@@ -231,7 +323,15 @@ __global__ void __launch_bounds__(MX_WARPS * 32) mxfp4_gemv_kernel(const uint8_t
             fence_proxy_async_smem();
             issue(tile + 2 * NW, s2);
         }
-        const int rows = rows_of(tile);
+        int m, t;
+        locate(tile, m, t);
+        const int jm = kMode == MX_ONE ? 0 : m % job.K;
+        const uint8_t *act = smem + (kMode == MX_SHARED && acts > 1 ? jm : 0) * AU;
+        const uint4 *qv = reinterpret_cast<const uint4 *>(act);
+        const int *qc = reinterpret_cast<const int *>(act + g.k);
+        const float *das = reinterpret_cast<const float *>(act + g.k + 32 * L);
+        const int rows = rows_of(t);
+        const int64_t row0 = static_cast<int64_t>(m) * g.n + static_cast<int64_t>(t) * g.R;
         const uint8_t *tp = slots + s * g.slot;
 #pragma unroll
         for (int jj = 0; jj < 2; ++jj) {
@@ -247,7 +347,7 @@ __global__ void __launch_bounds__(MX_WARPS * 32) mxfp4_gemv_kernel(const uint8_t
             }
             W[34] = 0u;
             float G = 0.0f;
-            int32_t *S_g = kSums ? S_out + (tile * g.R + gr[jj]) * nb + gg[jj] * (QK / MX_K) : nullptr;
+            int32_t *S_g = kSums ? job.S + (row0 + gr[jj]) * nb + gg[jj] * (QK / MX_K) : nullptr;
             mx_blocks<kSums, 0>(W, qv + gg[jj], qc + gg[jj], L, p2, G, S_g, emax);
             tb[tg] = __fmul_rn(G, das[gg[jj]]);
         }
@@ -260,7 +360,8 @@ __global__ void __launch_bounds__(MX_WARPS * 32) mxfp4_gemv_kernel(const uint8_t
                 const float2 v = t2[i];
                 acc = __fadd_rn(__fadd_rn(acc, v.x), v.y);
             }
-            y[tile * g.R + lane] = acc;
+            float *yb = kMode == MX_SHARED && m >= job.K ? job.y[1] : job.y[0];
+            yb[static_cast<int64_t>(jm) * g.n + static_cast<int64_t>(t) * g.R + lane] = acc;
         }
         __syncwarp();
         if (++s == MX_SLOTS) {
@@ -271,6 +372,17 @@ __global__ void __launch_bounds__(MX_WARPS * 32) mxfp4_gemv_kernel(const uint8_t
     if (__any_sync(0xffffffffu, emax == 255u) && lane == 0) report(status, TQFX4_EDATA, K_GEMV, -1);
 }
 
+// out[n] = sum over j in rank order of w_j * o_j[n] (binary32, no fused multiply-add).
+__global__ void __launch_bounds__(256) mx_combine_kernel(const float *__restrict__ o, const float *__restrict__ w,
+                                                         int K, int H, float *__restrict__ out) {
+    grid_dependency_wait();  // o of the down projections
+    const int n = blockIdx.x * blockDim.x + threadIdx.x;
+    if (n >= H) return;
+    float acc = 0.0f;
+    for (int j = 0; j < K; ++j) acc = __fadd_rn(acc, __fmul_rn(__ldg(w + j), __ldg(o + static_cast<int64_t>(j) * H + n)));
+    out[n] = acc;
+}
+
 }  // namespace
 
 int64_t mxfp4_bytes(int64_t n, int64_t k) {
@@ -278,9 +390,7 @@ int64_t mxfp4_bytes(int64_t n, int64_t k) {
     return n * (k / MX_K) * MX_BYTES;
 }
 
-cudaError_t launch_mxfp4_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da, float *y,
-                              int32_t *block_sums, int *status, cudaStream_t st) {
-    if (n == 0) return cudaSuccess;
+static MxGeo mx_geo(int64_t n, int64_t k) {
     MxGeo g;
     g.n = n;
     g.k = k;
@@ -289,25 +399,123 @@ cudaError_t launch_mxfp4_gemv(const void *blocks, int64_t n, int64_t k, const in
     g.J = (g.L + 31) / 32;
     g.row_bytes = g.L * MX_GB;
     g.slot = ((g.R * g.row_bytes + 15) / 16) * 16;
-    const int smem = mx_act_bytes(g) + MX_WARPS * mx_warp_bytes(g);
-    static unsigned char set[64];
-    const void *fn = block_sums ? reinterpret_cast<const void *>(mxfp4_gemv_kernel<true>)
-                                : reinterpret_cast<const void *>(mxfp4_gemv_kernel<false>);
-    cudaError_t e = allow_max_smem(fn, block_sums ? set : set + 32);
+    return g;
+}
+
+int mxfp4_gemv_smem(int64_t k, int acts) {
+    const MxGeo g = mx_geo(1, k);
+    return mx_act_bytes(g, acts) + MX_WARPS * mx_warp_bytes(g);
+}
+
+// One launch of the kernel in `mode`; `pdl`: as a programmatic dependent of
+// the previous kernel in the stream. Per-matrix mode: `ctas_per_mat` CTAs
+// per matrix.
+static cudaError_t launch_job(const MxGeo &g, const MxJob &job, int mode, bool pdl, int *status, cudaStream_t st) {
+    const int smem = mx_act_bytes(g, mode == MX_SHARED ? job.acts : 1) + MX_WARPS * mx_warp_bytes(g);
+    static unsigned char set[4][64];
+    const bool sums = job.S != nullptr;
+    const int v = mode == MX_ONE ? (sums ? 1 : 0) : mode + 1;
+    const void *fns[4] = {reinterpret_cast<const void *>(mxfp4_gemv_kernel<false, MX_ONE>),
+                          reinterpret_cast<const void *>(mxfp4_gemv_kernel<true, MX_ONE>),
+                          reinterpret_cast<const void *>(mxfp4_gemv_kernel<false, MX_SHARED>),
+                          reinterpret_cast<const void *>(mxfp4_gemv_kernel<false, MX_PER_MAT>)};
+    cudaError_t e = allow_max_smem(fns[v], set[v]);
     if (e != cudaSuccess) return e;
     if (smem > max_smem_optin()) return cudaErrorInvalidValue;
-    const int64_t tiles = (n + g.R - 1) / g.R;
-    int64_t grid = (tiles + 2 * MX_WARPS - 1) / (2 * MX_WARPS);  // at least two tiles per warp
+    const int64_t tpm = (g.n + g.R - 1) / g.R;
     const int64_t per_sm = max_smem_optin() / (smem + 1024);
     const int64_t cap = static_cast<int64_t>(num_sms()) * (per_sm > 0 ? per_sm : 1);
-    if (grid > cap) grid = cap;
-    if (block_sums)
-        mxfp4_gemv_kernel<true><<<static_cast<unsigned>(grid), MX_WARPS * 32, smem, st>>>(
-            static_cast<const uint8_t *>(blocks), g, q, da, y, block_sums, status);
-    else
-        mxfp4_gemv_kernel<false><<<static_cast<unsigned>(grid), MX_WARPS * 32, smem, st>>>(
-            static_cast<const uint8_t *>(blocks), g, q, da, y, nullptr, status);
-    return cudaGetLastError();
+    int64_t grid;
+    if (mode == MX_PER_MAT) {
+        // the CTAs that fit, split evenly among the matrices (at least two tiles per warp)
+        int64_t per = cap / job.K;
+        const int64_t need = (tpm + 2 * MX_WARPS - 1) / (2 * MX_WARPS);
+        if (per > need) per = need;
+        if (per < 1) per = 1;
+        grid = per * job.K;
+    } else {
+        grid = (tpm * (mode == MX_SHARED ? job.n_mat : 1) + 2 * MX_WARPS - 1) / (2 * MX_WARPS);
+        if (grid > cap) grid = cap;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(MX_WARPS * 32);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    MxGeo ga = g;
+    MxJob ja = job;
+    void *args[] = {&ga, &ja, &status};
+    return cudaLaunchKernelExC(&cfg, fns[v], args);
+}
+
+cudaError_t launch_mxfp4_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da, float *y,
+                              int32_t *block_sums, int *status, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    MxJob job{};
+    job.base[0] = job.base[1] = static_cast<const uint8_t *>(blocks);
+    job.K = job.n_mat = job.acts = 1;
+    job.q = q;
+    job.da = da;
+    job.y[0] = job.y[1] = y;
+    job.S = block_sums;
+    return launch_job(mx_geo(n, k), job, MX_ONE, false, status, st);
+}
+
+// ev (nullable): events recorded before gate/up, down (SwiGLU and the
+// quantization of h run in its prologue) and combine, and after combine.
+cudaError_t launch_moe_mxfp4_experts(const MoeArgs &a, float *out, cudaStream_t st, const cudaEvent_t *ev) {
+    const int K = a.top_k;
+    if (ev) record_stage_event(ev[0], st);
+    // gate and up of the selected experts: 2K matrices of I x H, one activation
+    MxJob gu{};
+    gu.base[0] = a.gate;
+    gu.base[1] = a.up;
+    gu.mat_bytes = a.mb_gu;
+    gu.sel = a.sel;
+    gu.K = K;
+    gu.n_mat = 2 * K;
+    gu.acts = 1;
+    gu.q = a.qx;
+    gu.da = a.dx;
+    gu.y[0] = a.g;
+    gu.y[1] = a.u;
+    cudaError_t e = launch_job(mx_geo(a.I, a.H), gu, MX_SHARED, ev == nullptr, a.status, st);
+    if (e != cudaSuccess) return e;
+    if (ev) record_stage_event(ev[1], st);
+    // down: K matrices of H x I, the CTAs split among the experts, each
+    // forming its expert's activation from g and u
+    MxJob dn{};
+    dn.base[0] = dn.base[1] = a.down;
+    dn.mat_bytes = a.mb_d;
+    dn.sel = a.sel;
+    dn.K = K;
+    dn.n_mat = K;
+    dn.acts = 1;
+    dn.g = a.g;
+    dn.u = a.u;
+    dn.y[0] = dn.y[1] = a.o;
+    if ((e = launch_job(mx_geo(a.H, a.I), dn, MX_PER_MAT, ev == nullptr, a.status, st)) != cudaSuccess) return e;
+    if (ev) record_stage_event(ev[2], st);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((a.H + 255) / 256);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = ev ? 0 : 1;
+    const float *o = a.o, *w = a.selw;
+    int Kk = K, H = a.H;
+    void *args[] = {&o, &w, &Kk, &H, &out};
+    e = cudaLaunchKernelExC(&cfg, reinterpret_cast<const void *>(mx_combine_kernel), args);
+    if (ev) record_stage_event(ev[3], st);
+    return e;
 }
 
 }  // namespace tq

@@ -1,4 +1,5 @@
-"""A routed-expert MoE layer held in device memory as tq2_0_fx4 blocks.
+"""A routed-expert MoE layer held in device memory as tq2_0_fx4 blocks (or,
+for the expert-lossless arm, as MXFP4 blocks).
 
 Plumbing only: it allocates the stacked expert matrices and the router with
 torch, fills them through tqfx4_pack, and calls tqfx4_moe_ffn /
@@ -13,14 +14,18 @@ from . import inputs
 
 
 class MoeLayer:
-    def __init__(self, gate, up, down, router_w, router_b, n_experts, hidden, inter, top_k):
+    def __init__(self, gate, up, down, router_w, router_b, n_experts, hidden, inter, top_k, fmt="fx4"):
+        """fmt: the experts' weight format, "fx4" (tq2_0_fx4 blocks) or
+        "mxfp4" (MXFP4 blocks, served by tqfx4_moe_ffn_mxfp4)."""
         self.gate, self.up, self.down = gate, up, down
         self.router_w, self.router_b = router_w, router_b
         self.n_experts, self.hidden, self.inter, self.top_k = n_experts, hidden, inter, top_k
+        self.fmt = fmt
         self.ex = B.c_experts(gate, up, down, n_experts, hidden, inter)
         self.rt = B.c_router(router_w, router_b, top_k)
-        self.mb_gu = B.tqfx4_matrix_bytes(inter, hidden)
-        self.mb_d = B.tqfx4_matrix_bytes(hidden, inter)
+        size = B.tqfx4_mxfp4_bytes if fmt == "mxfp4" else B.tqfx4_matrix_bytes
+        self.mb_gu = size(inter, hidden)
+        self.mb_d = size(hidden, inter)
 
     @classmethod
     def synthetic(cls, seed: int, n_experts: int, hidden: int, inter: int, top_k: int, zipf: float = 0.0,
@@ -44,6 +49,22 @@ class MoeLayer:
         rb = inputs.zipf_bias(n_experts, zipf).to(device) if zipf > 0 else None
         return cls(gate, up, down, rw, rb, n_experts, hidden, inter, top_k)
 
+    @classmethod
+    def synthetic_mxfp4(cls, seed: int, n_experts: int, hidden: int, inter: int, top_k: int, zipf: float = 0.0,
+                        device="cuda"):
+        """MXFP4 experts (random released-style bytes, inputs.mxfp4_matrix,
+        one seed per expert projection) and the router of synthetic()."""
+        mb_gu = B.tqfx4_mxfp4_bytes(inter, hidden)
+        mb_d = B.tqfx4_mxfp4_bytes(hidden, inter)
+        bufs = []
+        for proj, (n, k) in ((inputs.PROJ_GATE, (inter, hidden)), (inputs.PROJ_UP, (inter, hidden)),
+                             (inputs.PROJ_DOWN, (hidden, inter))):
+            bufs.append(torch.cat([inputs.mxfp4_matrix(inputs.expert_seed(seed, e, proj), n, k, device)
+                                   for e in range(n_experts)]))
+        rw = inputs.router_weight(seed, n_experts, hidden, device)
+        rb = inputs.zipf_bias(n_experts, zipf).to(device) if zipf > 0 else None
+        return cls(*bufs, rw, rb, n_experts, hidden, inter, top_k, fmt="mxfp4")
+
     def expert_blocks(self, e: int):
         """The (gate, up, down) byte ranges of expert e."""
         return (self.gate[e * self.mb_gu:(e + 1) * self.mb_gu], self.up[e * self.mb_gu:(e + 1) * self.mb_gu],
@@ -60,10 +81,15 @@ class MoeLayer:
         out = torch.empty(self.hidden, dtype=torch.float32, device=dev) if out is None else out
         sel_idx = torch.empty(self.top_k, dtype=torch.int32, device=dev) if sel_idx is None else sel_idx
         sel_w = torch.empty(self.top_k, dtype=torch.float32, device=dev) if sel_w is None else sel_w
-        B.tqfx4_moe_ffn(self.ex, self.rt, x, out, sel_idx, sel_w, ws, stream, events)
+        if self.fmt == "mxfp4":
+            B.tqfx4_moe_ffn_mxfp4(self.ex, self.rt, x, out, sel_idx, sel_w, ws, stream, events)
+        else:
+            B.tqfx4_moe_ffn(self.ex, self.rt, x, out, sel_idx, sel_w, ws, stream, events)
         return out, sel_idx, sel_w
 
     def grouped(self, X, ws, path=0, OUT=None, sel_idx=None, sel_w=None, stream=None, events=None):
+        if self.fmt != "fx4":
+            raise ValueError("the grouped path serves tq2_0_fx4 experts")
         T = X.shape[0]
         dev = X.device
         OUT = torch.empty((T, self.hidden), dtype=torch.float32, device=dev) if OUT is None else OUT
