@@ -44,6 +44,10 @@ def lib():
             "tqo_mxfp4_bytes": (i64, [i64, i64]),
             "tqo_mxfp4_dequant": (i32, [vp, i64, i64, vp]),
             "tqo_mxfp4_gemv": (i32, [vp, i64, i64, vp, vp, vp, vp]),
+            "tqo_free_bytes": (i64, [i64, i64]),
+            "tqo_pack_free": (i32, [vp, vp, vp, vp, i64, i64, vp]),
+            "tqo_free_dequant": (i32, [vp, i64, i64, vp]),
+            "tqo_free_gemv": (i32, [vp, i64, i64, vp, vp, vp, vp, vp]),
             "tqo_expert_ffn_mxfp4": (i32, [vp, vp, vp, i64, i64, vp, vp, vp, vp, vp, vp, vp, vp]),
             "tqo_moe_tokens_fmt": (i32, [i32, vp, vp, vp, i64, i64, i64, vp, vp, i32, vp, i64, vp, vp, vp]),
             "tqo_unpack": (i32, [vp, i64, i64, vp, vp]),
@@ -165,6 +169,44 @@ def mxfp4_gemv(blocks, n: int, k: int, q, da):
     S = np.empty((n, k // 32), np.int32)
     _check(lib().tqo_mxfp4_gemv(_p(blocks), n, k, _p(q), _p(da), _p(y), _p(S)), "mxfp4_gemv")
     return y, S
+
+
+# ---- the free-scale two-plane format (Table 1, 4.125 bits/weight) ------------
+
+def free_bytes(n: int, k: int) -> int:
+    return int(lib().tqo_free_bytes(n, k))
+
+
+def pack_free(t1, t2, a1_bits, a2_bits) -> np.ndarray:
+    """Two trit planes int8 [n][k] and their f16 scale bits [n][k/256] ->
+    528-byte blocks."""
+    t1, t2 = _c(t1, np.int8), _c(t2, np.int8)
+    a1_bits, a2_bits = _c(a1_bits, np.uint16), _c(a2_bits, np.uint16)
+    n, k = t1.shape
+    nbytes = free_bytes(n, k)
+    if nbytes < 0:
+        raise OracleError("bad shape %r" % (t1.shape,))
+    out = np.empty(nbytes, np.uint8)
+    _check(lib().tqo_pack_free(_p(t1), _p(t2), _p(a1_bits), _p(a2_bits), n, k, _p(out)), "pack_free")
+    return out
+
+
+def free_dequant(blocks, n: int, k: int) -> np.ndarray:
+    blocks = _c(blocks, np.uint8)
+    w = np.empty((n, k), np.float64)
+    _check(lib().tqo_free_dequant(_p(blocks), n, k, _p(w)), "free_dequant")
+    return w
+
+
+def free_gemv(blocks, n: int, k: int, q, da):
+    """(y fp32 [n], S1, S2 int32 [n][k/256]) of the two-plane dot pass."""
+    blocks = _c(blocks, np.uint8)
+    q, da = _c(q, np.int8), _c(da, np.float32)
+    y = np.empty(n, np.float32)
+    S1 = np.empty((n, k // QK), np.int32)
+    S2 = np.empty((n, k // QK), np.int32)
+    _check(lib().tqo_free_gemv(_p(blocks), n, k, _p(q), _p(da), _p(y), _p(S1), _p(S2)), "free_gemv")
+    return y, S1, S2
 
 
 def pack_trits(t1, t2, d_bits) -> np.ndarray:

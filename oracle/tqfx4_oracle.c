@@ -504,6 +504,119 @@ int tqo_mxfp4_gemv(const uint8_t *blocks, int64_t n, int64_t k, const int8_t *q,
 }
 
 /* ------------------------------------------------------------------ */
+/* The free-scale two-plane format (Table 1's free-scale K=2 row, 4.125   */
+/* bits/weight: the pair with two independent scales does not fold, so   */
+/* the two trit planes are stored apart): W = a1 t1 + a2 t2 per row and   */
+/* 256 columns, t1, t2 in {-1, 0, 1}, a1, a2 f16. Reading of the bytes     */
+/* (the paper gives only the size): blocks of 4 rows x 256 columns, 528   */
+/* bytes, ordered [N/4 row groups][K/256 blocks] like the 520-byte block; */
+/* bytes 0..7 hold a1 of rows 0..3 and bytes 8..15 a2 (f16, little        */
+/* endian); bytes 16 + 128 r .. + 63 hold row r's plane t1 and the next 64 */
+/* bytes its plane t2, element j in bits 2 (j % 4) of byte j / 4 as       */
+/* u = t + 1 in 0..2 (3 is invalid).                                      */
+/* ------------------------------------------------------------------ */
+#define FREE_BLOCK_BYTES 528
+#define FREE_PLANE_OFS 16
+#define FREE_ROW_BYTES 128
+
+int64_t tqo_free_bytes(int64_t n, int64_t k) {
+    if (n < 0 || k < 0 || n % ROWS || k % QK) return -1;
+    return (n / ROWS) * (k / QK) * FREE_BLOCK_BYTES;
+}
+
+static const uint8_t *free_block(const uint8_t *blocks, int64_t k, int64_t row, int64_t b) {
+    return blocks + ((row / ROWS) * (k / QK) + b) * FREE_BLOCK_BYTES;
+}
+
+/* Trit of plane p (0: t1, 1: t2) of row r, element j of a block; -9 if invalid. */
+static int free_trit(const uint8_t *blk, int r, int p, int j) {
+    const uint8_t byte = blk[FREE_PLANE_OFS + FREE_ROW_BYTES * r + 64 * p + j / 4];
+    const int u = (byte >> (2 * (j % 4))) & 3;
+    return u == 3 ? -9 : u - 1;
+}
+
+/* Pack two trit planes with their scales. t1, t2: int8 [n][k]; a1, a2: f16
+ * bits [n][k/256]. Returns 0, -1 on a bad shape, -2 on a trit outside
+ * {-1, 0, 1}. */
+int tqo_pack_free(const int8_t *t1, const int8_t *t2, const uint16_t *a1, const uint16_t *a2,
+                  int64_t n, int64_t k, uint8_t *out) {
+    if (tqo_free_bytes(n, k) < 0) return -1;
+    int64_t nb = k / QK;
+    memset(out, 0, (size_t)tqo_free_bytes(n, k));
+    for (int64_t row = 0; row < n; row++)
+        for (int64_t b = 0; b < nb; b++) {
+            uint8_t *blk = out + ((row / ROWS) * nb + b) * FREE_BLOCK_BYTES;
+            const int r = (int)(row % ROWS);
+            const uint16_t s1 = a1[row * nb + b], s2 = a2[row * nb + b];
+            blk[2 * r] = (uint8_t)(s1 & 0xff);
+            blk[2 * r + 1] = (uint8_t)(s1 >> 8);
+            blk[8 + 2 * r] = (uint8_t)(s2 & 0xff);
+            blk[8 + 2 * r + 1] = (uint8_t)(s2 >> 8);
+            for (int j = 0; j < QK; j++)
+                for (int p = 0; p < 2; p++) {
+                    const int t = (p ? t2 : t1)[row * k + b * QK + j];
+                    if (t < -1 || t > 1) return -2;
+                    blk[FREE_PLANE_OFS + FREE_ROW_BYTES * r + 64 * p + j / 4] |= (uint8_t)((t + 1) << (2 * (j % 4)));
+                }
+        }
+    return 0;
+}
+
+/* W = a1 t1 + a2 t2 in fp64. Returns 0, -1 on a bad shape, -3 on an
+ * invalid trit. */
+int tqo_free_dequant(const uint8_t *blocks, int64_t n, int64_t k, double *w) {
+    if (tqo_free_bytes(n, k) < 0) return -1;
+    for (int64_t row = 0; row < n; row++)
+        for (int64_t b = 0; b < k / QK; b++) {
+            const uint8_t *blk = free_block(blocks, k, row, b);
+            const int r = (int)(row % ROWS);
+            const double s1 = tqo_f16_to_f32((uint16_t)(blk[2 * r] | (blk[2 * r + 1] << 8)));
+            const double s2 = tqo_f16_to_f32((uint16_t)(blk[8 + 2 * r] | (blk[8 + 2 * r + 1] << 8)));
+            for (int j = 0; j < QK; j++) {
+                const int x1 = free_trit(blk, r, 0, j), x2 = free_trit(blk, r, 1, j);
+                if (x1 < -1 || x2 < -1) return -3;
+                w[row * k + b * QK + j] = s1 * x1 + s2 * x2;
+            }
+        }
+    return 0;
+}
+
+/* The two-plane dot pass: per (row, 256-block) the exact int32 sums
+ * S1 = sum t1 q and S2 = sum t2 q, then the fixed float schedule
+ * acc = acc + (float(S1) * (a1 * da) + float(S2) * (a2 * da)), blocks in
+ * ascending order, every product and sum rounded once. S1, S2 (nullable):
+ * [n][k/256]. Returns 0, -1 on a bad shape, -3 on an invalid trit. */
+int tqo_free_gemv(const uint8_t *blocks, int64_t n, int64_t k, const int8_t *q, const float *da, float *y,
+                  int32_t *S1_out, int32_t *S2_out) {
+    if (tqo_free_bytes(n, k) < 0) return -1;
+    int64_t nb = k / QK;
+    for (int64_t row = 0; row < n; row++) {
+        float acc = 0.0f;
+        for (int64_t b = 0; b < nb; b++) {
+            const uint8_t *blk = free_block(blocks, k, row, b);
+            const int r = (int)(row % ROWS);
+            int32_t s1 = 0, s2 = 0;
+            for (int j = 0; j < QK; j++) {
+                const int x1 = free_trit(blk, r, 0, j), x2 = free_trit(blk, r, 1, j);
+                if (x1 < -1 || x2 < -1) return -3;
+                s1 += x1 * (int32_t)q[b * QK + j];
+                s2 += x2 * (int32_t)q[b * QK + j];
+            }
+            if (S1_out) S1_out[row * nb + b] = s1;
+            if (S2_out) S2_out[row * nb + b] = s2;
+            const float a1 = tqo_f16_to_f32((uint16_t)(blk[2 * r] | (blk[2 * r + 1] << 8)));
+            const float a2 = tqo_f16_to_f32((uint16_t)(blk[8 + 2 * r] | (blk[8 + 2 * r + 1] << 8)));
+            const float p1 = (float)s1 * (a1 * da[b]);
+            const float p2 = (float)s2 * (a2 * da[b]);
+            const float t = p1 + p2;
+            acc = acc + t;
+        }
+        y[row] = acc;
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
 /* exp in binary32 (used by SwiGLU). The paper does not fix how SwiGLU   */
 /* is evaluated; because its output is re-quantized to int8 (a rounding  */
 /* decision), both this oracle and the kernel evaluate it with the same  */
