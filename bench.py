@@ -14,7 +14,7 @@ same number divided by the bytes per token, reported beside it.
 
     python bench.py [--steps K] [--warmup W] [--gpus N] [--impl ours|reference]
                     [--workload moe_decode|grouped_decode_64|prefill_2048|tiered_decode|mxfp4_gemv|
-                                moe_decode_mxfp4]
+                                moe_decode_mxfp4|free_gemv]
 
 The K timed steps are captured once into a CUDA graph and replayed inside
 the timed region (no host launch work in it); the other workloads time
@@ -491,12 +491,15 @@ GEMV_N, GEMV_K, GEMV_POOL = 131072, 4096, 16
 
 
 def run_gemv(args, rank, world, local):
-    """The MXFP4 arm: one GEMV per step over a 131072 x 4096 matrix (64
-    experts' 2048 x 4096 gate projections stacked, 285 MB, larger than L2) in
-    MXFP4 blocks (the released bytes, 17 per 32 elements), a new activation
-    every step: tqfx4_quantize_act, then tqfx4_gemv_mxfp4. The tq2_0_fx4 GEMV
-    of a matrix of the same shape is timed beside it. Metric: effective MXFP4
-    GB/s (the matrix's bytes over the step time)."""
+    """One GEMV per step over a 131072 x 4096 matrix (64 experts' 2048 x 4096
+    gate projections stacked, larger than L2) in a second weight format, a new
+    activation every step: tqfx4_quantize_act, then the format's dot pass.
+    mxfp4_gemv: MXFP4 blocks (the released bytes, 17 per 32 elements, 285 MB)
+    through tqfx4_gemv_mxfp4; free_gemv: the free-scale two-plane blocks
+    (528 bytes per 4 x 256, 277 MB) through tqfx4_gemv_free. The tq2_0_fx4
+    GEMV of a matrix of the same shape is timed beside it (for free_gemv this
+    is the paper's fold-versus-planes speed ablation). Metric: effective GB/s
+    of the format's bytes over the step time."""
     import torch
     import torch.distributed as dist
 
@@ -510,7 +513,14 @@ def run_gemv(args, rank, world, local):
     dev = torch.device("cuda", local)
     n, k = GEMV_N, GEMV_K
     ws = ops.workspace(B.TQFX4_STATUS_BYTES, dev)
-    mx = inputs.mxfp4_matrix(SEED, n, k, dev)
+    free = args.workload == "free_gemv"
+    if free:
+        t1, t2, s1 = inputs.trit_planes(SEED, n, k, dev)
+        s2 = inputs.trit_planes(SEED + 1, n, k, dev)[2]
+        mx = ops.pack_free(t1, t2, s1.view(torch.int16), s2.view(torch.int16), ws)
+        del t1, t2
+    else:
+        mx = inputs.mxfp4_matrix(SEED, n, k, dev)
     mx_bytes = mx.numel()
     fx = ops.pack_rtn(inputs.gemv_matrix(SEED, n, k, dev), ws)
     fx_bytes = fx.numel()
@@ -530,6 +540,8 @@ def run_gemv(args, rank, world, local):
             ev[1].record(st)
         if fmt == "mxfp4":
             B.tqfx4_gemv_mxfp4(mx, n, k, q, da, y, None, ws, st)
+        elif fmt == "free":
+            B.tqfx4_gemv_free(mx, n, k, q, da, bs, y, None, None, ws, st)
         else:
             B.tqfx4_gemv(fx, n, k, q, da, bs, y, None, ws, st)
         if ev:
@@ -566,7 +578,8 @@ def run_gemv(args, rank, world, local):
             dist.barrier()
         return max_over_ranks(ev0.elapsed_time(ev1) / 1e3, world, dev)
 
-    g_mx = graph_of("mxfp4")
+    fmt = "free" if free else "mxfp4"
+    g_mx = graph_of(fmt)
     with ClockSampler(local) as clk:
         t = timed(g_mx)
     B.tqfx4_check(ws)
@@ -582,7 +595,7 @@ def run_gemv(args, rank, world, local):
         return (sum(e[0].elapsed_time(e[1]) for e in evs) / reps / 1e3,
                 sum(e[1].elapsed_time(e[2]) for e in evs) / reps / 1e3)
 
-    q_mx, g_mx_s = stage_times("mxfp4")
+    q_mx, g_mx_s = stage_times(fmt)
     _, g_fx_s = stage_times("fx4")
     B.tqfx4_check(ws)
 
@@ -590,18 +603,23 @@ def run_gemv(args, rank, world, local):
     Xh = X.cpu().pin_memory()
     xin = torch.empty(k, device=dev)
     yh = torch.empty(n, pin_memory=True)
+
+    def step_e2e():
+        B.tqfx4_quantize_act(xin, 1, k, q, da, bs, ws, stream)
+        if free:
+            B.tqfx4_gemv_free(mx, n, k, q, da, bs, y, None, None, ws, stream)
+        else:
+            B.tqfx4_gemv_mxfp4(mx, n, k, q, da, y, None, ws, stream)
+        yh.copy_(y, non_blocking=True)
+
     for i in range(3):
         xin.copy_(Xh[i], non_blocking=True)
-        B.tqfx4_quantize_act(xin, 1, k, q, da, bs, ws, stream)
-        B.tqfx4_gemv_mxfp4(mx, n, k, q, da, y, None, ws, stream)
-        yh.copy_(y, non_blocking=True)
+        step_e2e()
     torch.cuda.synchronize()
     ev0.record(stream)
     for i in range(args.steps):
         xin.copy_(Xh[i % GEMV_POOL], non_blocking=True)
-        B.tqfx4_quantize_act(xin, 1, k, q, da, bs, ws, stream)
-        B.tqfx4_gemv_mxfp4(mx, n, k, q, da, y, None, ws, stream)
-        yh.copy_(y, non_blocking=True)
+        step_e2e()
     ev1.record(stream)
     torch.cuda.synchronize()
     B.tqfx4_check(ws)
@@ -610,18 +628,20 @@ def run_gemv(args, rank, world, local):
     peak, peak_kind = _peaks()
     achieved = mx_bytes / g_mx_s / 1e9
     line = {
-        "metric": "effective MXFP4 GB/s (GEMV, 131072 x 4096)",
+        "metric": ("effective free-scale two-plane GB/s (GEMV, 131072 x 4096)" if free
+                   else "effective MXFP4 GB/s (GEMV, 131072 x 4096)"),
         "value": job_rate(mx_bytes * args.steps, world, t) / 1e9, "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "i8xe2m1-i32,f32",
-        "data": "synthetic",
-        "config": {"workload": "mxfp4_gemv", "n": n, "k": k, "matrix_bytes": mx_bytes,
-                   "l2": "inputs larger than L2 (285 MB matrix); a different activation per step"},
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "i8xi2-i32,f32" if free else "i8xe2m1-i32,f32", "data": "synthetic",
+        "config": {"workload": args.workload, "n": n, "k": k, "matrix_bytes": mx_bytes,
+                   "l2": "inputs larger than L2 (%d MB matrix); a different activation per step" % (mx_bytes >> 20)},
         "fx4_same_shape": {"gbs": fx_bytes * args.steps / t_fx / 1e9, "ms_per_step": t_fx / args.steps * 1e3,
                            "matrix_bytes": fx_bytes, "gemv_us": g_fx_s * 1e6,
                            "gemv_gbs": fx_bytes / g_fx_s / 1e9},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": None, "kernel": "mxfp4_gemv_kernel",
+                     "frac": achieved / peak, "traffic": None,
+                     "kernel": "gemv_free_kernel" if free else "mxfp4_gemv_kernel",
                      "peak_source": peak_kind, "stage_us": {"quantize_act": q_mx * 1e6, "gemv": g_mx_s * 1e6}},
         "e2e": {"value": job_rate(mx_bytes * args.steps, world, te) / 1e9, "unit": "GB/s",
                 "h2d_bytes_per_step": k * 4, "d2h_bytes_per_step": n * 4},
@@ -638,7 +658,7 @@ def run_gemv(args, rank, world, local):
         done, el = 0, 0.0
         while el < 10.0:
             t0 = time.perf_counter()
-            oracle.mxfp4_gemv(sub, rows, k, qh, dah)
+            (oracle.free_gemv if free else oracle.mxfp4_gemv)(sub, rows, k, qh, dah)
             el += time.perf_counter() - t0
             done += 1
         line["cpu_baseline"] = {"value": done * sub.nbytes / el / 1e9, "unit": "GB/s", "cores": 1,
@@ -663,11 +683,11 @@ def main():
                     help="tokens per step of the grouped workloads (default: 64 or 2048; profiling only)")
     ap.add_argument("--workload", default="moe_decode",
                     choices=["moe_decode", "grouped_decode_64", "prefill_2048", "tiered_decode", "mxfp4_gemv",
-                             "moe_decode_mxfp4"],
+                             "moe_decode_mxfp4", "free_gemv"],
                     help="moe_decode (default): 1 token; grouped_decode_64: 64 tokens with Zipf(1.1) "
                          "routing; prefill_2048: 2048 tokens; tiered_decode: 1 token with the experts in "
-                         "host memory; mxfp4_gemv: one GEMV over MXFP4 blocks; moe_decode_mxfp4: moe_decode with "
-                         "MXFP4 experts")
+                         "host memory; mxfp4_gemv / free_gemv: one GEMV over MXFP4 / free-scale two-plane blocks; "
+                         "moe_decode_mxfp4: moe_decode with MXFP4 experts")
     ap.add_argument("--slots", type=int, default=TOPK, help="device expert slots of tiered_decode")
     args = ap.parse_args()
     globals()["E"] = args.experts
@@ -682,7 +702,7 @@ def main():
     if args.workload == "tiered_decode":
         run_tiered(args, rank, world, local)
         return
-    if args.workload == "mxfp4_gemv":
+    if args.workload in ("mxfp4_gemv", "free_gemv"):
         run_gemv(args, rank, world, local)
         return
     if args.workload not in ("moe_decode", "moe_decode_mxfp4"):

@@ -157,6 +157,36 @@ tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k,
                         void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * The free-scale two-plane format (Table 1's free-scale K=2 row, 4.125
+ * bits/weight; the ablation of the tie of Sec. 2.1): W = a1 t1 + a2 t2 per
+ * row and 256 columns, t1, t2 in {-1, 0, 1}, two independent f16 scales.
+ * The pair does not fold, so both trit planes are stored: blocks of 4 rows x
+ * 256 columns, 528 bytes, ordered [N/4 row groups][K/256 blocks] like the
+ * 520-byte block. Bytes 0..7: a1 of rows 0..3; bytes 8..15: a2 (f16, little
+ * endian); row r's plane t1 at bytes 16 + 128 r .. + 63 and plane t2 at the
+ * next 64 bytes, element j in bits 2 (j % 4) of byte j / 4 as u = t + 1
+ * (u = 3 is invalid). (The paper gives the size, not the byte order.)
+ *   tqfx4_free_bytes: (n/4)(k/256) * 528, or -1 unless n % 4 == 0 and
+ *     k % 256 == 0.
+ *   tqfx4_pack_free: t1, t2 int8 [n][k] (device, 16-byte aligned), a1, a2
+ *     f16 bits [n][k/256] (device) -> blocks (device, 16-byte aligned,
+ *     caller-allocated). A trit outside {-1, 0, 1} sets TQFX4_EDATA.
+ *   tqfx4_gemv_free: y = W x for x quantized by tqfx4_quantize_act (q, da,
+ *     bsum). Per (row, 256-block) the exact int32 sums S1 = sum t1 q and
+ *     S2 = sum t2 q; y[n] = the binary32 sum in ascending block order of
+ *     float(S1) * (a1 * da) + float(S2) * (a2 * da) (each product and sum
+ *     rounded once). S1, S2: both NULL or both int32 [n][k/256] (device).
+ *     k <= TQFX4_MAX_K.
+ */
+int64_t tqfx4_free_bytes(int64_t n, int64_t k);
+tqfx4_status tqfx4_pack_free(const int8_t *t1, const int8_t *t2, const uint16_t *a1_f16,
+                             const uint16_t *a2_f16, int64_t n, int64_t k, void *blocks,
+                             void *ws, size_t ws_bytes, void *stream);
+tqfx4_status tqfx4_gemv_free(const void *blocks, int64_t n, int64_t k, const int8_t *q,
+                             const float *da, const int32_t *bsum, float *y, int32_t *S1,
+                             int32_t *S2, void *ws, size_t ws_bytes, void *stream);
+
+/*
  * The MXFP4 arm (Sec. 2.3, the expert-lossless arm): the released expert
  * bytes (4.25 bits/weight in Table 1), served by the integer dot pass with no
  * transcode. Format (OCP microscaling): blocks of 32 consecutive elements of

@@ -75,6 +75,9 @@ _SIGS = {
     "tqfx4_moe_workspace_views": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int, _int,
                                          C.POINTER(CMoeViews)]),
     "tqfx4_moe_ffn_noalloc": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp]),
+    "tqfx4_free_bytes": (_i64, [_i64, _i64]),
+    "tqfx4_pack_free": (_int, [_vp, _vp, _vp, _vp, _i64, _i64, _vp, _vp, _sz, _vp]),
+    "tqfx4_gemv_free": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_mxfp4_bytes": (_i64, [_i64, _i64]),
     "tqfx4_gemv_mxfp4": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_route": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _sz, _vp]),
@@ -194,6 +197,20 @@ def tqfx4_moe_ffn_noalloc(ex, rt, x, out, sel_idx, sel_w, stream=None):
     allocate device memory; see include/tqfx4.h)."""
     _check(lib().tqfx4_moe_ffn_noalloc(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w),
                                        _s(stream)), "tqfx4_moe_ffn_noalloc")
+
+
+def tqfx4_free_bytes(n: int, k: int) -> int:
+    return int(lib().tqfx4_free_bytes(n, k))
+
+
+def tqfx4_pack_free(t1, t2, a1, a2, n, k, blocks, ws, stream=None):
+    _check(lib().tqfx4_pack_free(_p(t1), _p(t2), _p(a1), _p(a2), n, k, _p(blocks), _p(ws), _nbytes(ws),
+                                 _s(stream)), "tqfx4_pack_free")
+
+
+def tqfx4_gemv_free(blocks, n, k, q, da, bsum, y, S1, S2, ws, stream=None):
+    _check(lib().tqfx4_gemv_free(_p(blocks), n, k, _p(q), _p(da), _p(bsum), _p(y), _p(S1), _p(S2), _p(ws),
+                                 _nbytes(ws), _s(stream)), "tqfx4_gemv_free")
 
 
 def tqfx4_mxfp4_bytes(n: int, k: int) -> int:

@@ -123,6 +123,46 @@ tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
 }
 
 
+int64_t tqfx4_free_bytes(int64_t n, int64_t k) { return tq::free_bytes(n, k); }
+
+tqfx4_status tqfx4_pack_free(const int8_t *t1, const int8_t *t2, const uint16_t *a1_f16, const uint16_t *a2_f16,
+                             int64_t n, int64_t k, void *blocks, void *ws, size_t ws_bytes, void *stream) {
+    const char *fn = "tqfx4_pack_free";
+    tqfx4_status s = check_nk(n, k, fn);
+    if (s) return s;
+    if ((s = check_ws(ws, ws_bytes, TQFX4_STATUS_BYTES, fn))) return s;
+    if (n == 0 || k == 0) return ok();
+    if (!t1 || !t2 || !a1_f16 || !a2_f16 || !blocks) return fail(TQFX4_EINVAL, "%s: NULL input or output", fn);
+    if (!aligned(t1, 16) || !aligned(t2, 16) || !aligned(a1_f16, 2) || !aligned(a2_f16, 2) || !aligned(blocks, 16))
+        return fail(TQFX4_EALIGN, "%s: t1, t2 and blocks must be 16-byte aligned", fn);
+    cudaError_t e = tq::launch_pack_free(t1, t2, a1_f16, a2_f16, n, k, blocks, static_cast<int *>(ws),
+                                         static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
+tqfx4_status tqfx4_gemv_free(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
+                             const int32_t *bsum, float *y, int32_t *S1, int32_t *S2, void *ws, size_t ws_bytes,
+                             void *stream) {
+    const char *fn = "tqfx4_gemv_free";
+    tqfx4_status s = check_nk(n, k, fn);
+    if (s) return s;
+    if (k == 0 || k > TQFX4_MAX_K) return fail(TQFX4_ESHAPE, "%s: k=%lld must be in 256..%d", fn, (long long)k,
+                                               TQFX4_MAX_K);
+    if ((s = check_ws(ws, ws_bytes, TQFX4_STATUS_BYTES, fn))) return s;
+    if (n == 0) return ok();
+    if (!blocks || !q || !da || !bsum || !y) return fail(TQFX4_EINVAL, "%s: NULL input or output", fn);
+    if ((S1 == nullptr) != (S2 == nullptr)) return fail(TQFX4_EINVAL, "%s: S1 and S2 both or neither", fn);
+    if (!aligned(blocks, 16) || !aligned(q, 16) || !aligned(da, 4) || !aligned(bsum, 4) || !aligned(y, 4) ||
+        !aligned(S1, 4) || !aligned(S2, 4))
+        return fail(TQFX4_EALIGN, "%s: blocks and q must be 16-byte aligned", fn);
+    if (tq::gemv_free_smem(k, nullptr) < 0) return fail(TQFX4_ESHAPE, "%s: k too large for shared memory", fn);
+    cudaError_t e = tq::launch_gemv_free(blocks, n, k, q, da, bsum, y, S1, S2, static_cast<int *>(ws),
+                                         static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
 int64_t tqfx4_mxfp4_bytes(int64_t n, int64_t k) { return tq::mxfp4_bytes(n, k); }
 
 tqfx4_status tqfx4_gemv_mxfp4(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da, float *y,

@@ -1,0 +1,264 @@
+// The free-scale two-plane format (Table 1's free-scale K=2 row, 4.125
+// bits/weight): W = a1 t1 + a2 t2 per row and 256 columns with two
+// independent f16 scales, the two trit planes stored apart because the pair
+// does not fold. Blocks of 4 rows x 256 columns, 528 bytes, ordered
+// [N/4 row groups][K/256 blocks]: bytes 0..7 a1 of rows 0..3, 8..15 a2,
+// then per row r at 16 + 128 r the plane t1 (64 bytes) and the plane t2 (64
+// bytes), element j in bits 2 (j % 4) of byte j / 4 as u = t + 1 (3 is
+// invalid).
+//
+// tqfx4_pack_free: one warp per (row, 256-block), lane l packs elements
+// 8l .. 8l + 7 of both planes.
+//
+// tqfx4_gemv_free: the two-plane dot pass. Exact sums S = sum t q per plane
+// and block, then per block float(S1) * (a1 * da) + float(S2) * (a2 * da)
+// added to the row's sum in block order (the oracle's schedule). A warp
+// takes one row group (4 rows, all of k) per tile through a ring of bulk
+// copies; lane l takes the (row, block) pairs l, l + 32, ... . A plane word
+// holds 16 trits; its four 2-bit fields per byte are masked in place
+// (x & (0x03030303 << 2i), no shift) so that the unsigned x signed dp4a
+// sums 4^i u q into accumulator i; the four accumulators are shifted back
+// exactly (each is a multiple of 4^i) and sum u q - sum q = sum t q. The
+// activation is staged once per CTA with the four bytes of each dp4a word
+// transposed to match the fields (elements 4b + i of a 16-element word).
+#include "tq_common.cuh"
+#include "tq_launch.h"
+
+namespace tq {
+
+namespace {
+
+constexpr int FR_BLOCK = 528, FR_PLANE_OFS = 16, FR_ROW = 128;
+constexpr int FR_SLOTS = 2;
+
+__global__ void __launch_bounds__(256) pack_free_kernel(const int8_t *__restrict__ t1, const int8_t *__restrict__ t2,
+                                                        const uint16_t *__restrict__ a1,
+                                                        const uint16_t *__restrict__ a2, int64_t n, int64_t k,
+                                                        uint8_t *__restrict__ out, int *status) {
+    const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t L = k / QK;
+    if (w >= n * L) return;
+    const int64_t row = w / L, b = w - row * L;
+    const int r = static_cast<int>(row & 3);
+    uint8_t *blk = out + ((row >> 2) * L + b) * FR_BLOCK;
+    const int64_t src = row * k + b * QK + 8 * lane;
+    bool bad = false;
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+        const uint2 v = __ldg(reinterpret_cast<const uint2 *>((p ? t2 : t1) + src));
+        const uint32_t words[2] = {v.x, v.y};
+        uint32_t packed = 0;
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int t = static_cast<int8_t>((words[h] >> (8 * e)) & 0xffu);
+                bad |= t < -1 || t > 1;
+                packed |= static_cast<uint32_t>((t + 1) & 3) << (8 * h + 2 * e);
+            }
+        *reinterpret_cast<uint16_t *>(blk + FR_PLANE_OFS + FR_ROW * r + 64 * p + 2 * lane) =
+            static_cast<uint16_t>(packed);
+    }
+    if (lane == 0) {
+        reinterpret_cast<uint16_t *>(blk)[r] = a1[row * L + b];
+        reinterpret_cast<uint16_t *>(blk + 8)[r] = a2[row * L + b];
+    }
+    if (__any_sync(0xffffffffu, bad) && lane == 0) report(status, TQFX4_EDATA, K_PACK, static_cast<int>(w));
+}
+
+__device__ __forceinline__ int dp4a_us(uint32_t a, uint32_t b, int c) {
+    int d;
+    asm("dp4a.u32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+
+// sum u q over one plane of one (row, block): 16 words, each with its
+// transposed activation word group; acc[i] collects 4^i u q.
+__device__ __forceinline__ int free_plane_sum(const uint4 *pw, const uint4 *qv, int L) {
+    int acc[4] = {0, 0, 0, 0};
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        const uint4 x4 = pw[c];
+        const uint32_t xs[4] = {x4.x, x4.y, x4.z, x4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const uint4 qq = qv[(4 * c + e) * L];
+            const uint32_t x = xs[e];
+            acc[0] = dp4a_us(x & 0x03030303u, qq.x, acc[0]);
+            acc[1] = dp4a_us(x & 0x0c0c0c0cu, qq.y, acc[1]);
+            acc[2] = dp4a_us(x & 0x30303030u, qq.z, acc[2]);
+            acc[3] = dp4a_us(x & 0xc0c0c0c0u, qq.w, acc[3]);
+        }
+    }
+    return acc[0] + (acc[1] >> 2) + (acc[2] >> 4) + (acc[3] >> 6);
+}
+
+__device__ __forceinline__ bool free_wait(uint64_t *bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    return mbar_wait(bar, parity);
+}
+
+struct FreeGeo {
+    int64_t n, k;
+    int L;          // 256-blocks per row
+    int tile;       // bytes of a row group (L * 528)
+    int warps;
+};
+
+__host__ __device__ inline int free_act_bytes(int L) { return ((L * (QK + 8) + 127) / 128) * 128; }
+__host__ __device__ inline int free_warp_bytes(const FreeGeo &g) {
+    return FR_SLOTS * g.tile + 4 * 4 * g.L + 32;
+}
+
+// The fields of plane word w of a block: byte b of transposed word i is
+// element 16 w + 4 b + i.
+__device__ __forceinline__ uint4 free_transpose(uint4 v) {
+    const uint32_t t01l = __byte_perm(v.x, v.y, 0x5140), t23l = __byte_perm(v.z, v.w, 0x5140);
+    const uint32_t t01h = __byte_perm(v.x, v.y, 0x7362), t23h = __byte_perm(v.z, v.w, 0x7362);
+    return make_uint4(__byte_perm(t01l, t23l, 0x5410), __byte_perm(t01l, t23l, 0x7632),
+                      __byte_perm(t01h, t23h, 0x5410), __byte_perm(t01h, t23h, 0x7632));
+}
+
+template <bool kSums>
+__global__ void __launch_bounds__(256) gemv_free_kernel(const uint8_t *__restrict__ blocks, FreeGeo g,
+                                                        const int8_t *__restrict__ q, const float *__restrict__ da,
+                                                        const int32_t *__restrict__ bsum, float *__restrict__ y,
+                                                        int32_t *__restrict__ S1o, int32_t *__restrict__ S2o,
+                                                        int *status) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int L = g.L;
+    uint4 *qv = reinterpret_cast<uint4 *>(smem);  // [16 words][L blocks]
+    float *das = reinterpret_cast<float *>(smem + L * QK);
+    int *bss = reinterpret_cast<int *>(smem + L * QK + 4 * L);
+    uint8_t *wbase = smem + free_act_bytes(L) + warp * free_warp_bytes(g);
+    uint8_t *slots = wbase;
+    float *tb = reinterpret_cast<float *>(wbase + FR_SLOTS * g.tile);  // [4 rows][L]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(wbase + FR_SLOTS * g.tile + 16 * L);
+    if (lane == 0)
+        for (int i = 0; i < FR_SLOTS; ++i) mbar_init(&bars[i], 1);
+    fence_barrier_init();
+
+    const int64_t tiles = g.n / ROWS;
+    const int64_t NW = static_cast<int64_t>(gridDim.x) * g.warps;
+    const int64_t first = static_cast<int64_t>(blockIdx.x) * g.warps + warp;
+    const uint64_t policy = l2_policy_evict_first();
+    auto issue = [&](int64_t tile, int s) {
+        if (lane == 0) {
+            mbar_arrive_expect_tx(&bars[s], static_cast<uint32_t>(g.tile));
+            bulk_g2s_hint(slots + s * g.tile, blocks + tile * g.tile, static_cast<uint32_t>(g.tile), &bars[s],
+                          policy);
+        }
+    };
+    if (first < tiles) issue(first, 0);
+    if (first + NW < tiles) issue(first + NW, 1);
+    for (int idx = threadIdx.x; idx < 16 * L; idx += blockDim.x) {
+        const int b = idx % L, wd = idx / L;
+        qv[idx] = free_transpose(__ldg(reinterpret_cast<const uint4 *>(q + b * QK + 16 * wd)));
+    }
+    for (int i = threadIdx.x; i < L; i += blockDim.x) {
+        das[i] = __ldg(da + i);
+        bss[i] = __ldg(bsum + i);
+    }
+    __syncthreads();
+
+    const int pairs = ROWS * L;
+    int it = 0;
+    for (int64_t tile = first; tile < tiles; tile += NW, ++it) {
+        const int s = it & 1;
+        if (!__all_sync(0xffffffffu, free_wait(&bars[s], static_cast<uint32_t>((it >> 1) & 1)))) {
+            if (lane == 0) report(status, TQFX4_ETIMEOUT, K_GEMV, static_cast<int>(tile));
+            break;
+        }
+        const uint8_t *tp = slots + s * g.tile;
+        for (int p = lane; p < pairs; p += 32) {
+            const int r = p / L, b = p - r * L;
+            const uint8_t *blk = tp + b * FR_BLOCK;
+            const uint4 *pl = reinterpret_cast<const uint4 *>(blk + FR_PLANE_OFS + FR_ROW * r);
+            const int S1 = free_plane_sum(pl, qv + b, L) - bss[b];
+            const int S2 = free_plane_sum(pl + 4, qv + b, L) - bss[b];
+            const float a1 = __half2float(reinterpret_cast<const __half *>(blk)[r]);
+            const float a2 = __half2float(reinterpret_cast<const __half *>(blk + 8)[r]);
+            const float p1 = __fmul_rn(static_cast<float>(S1), __fmul_rn(a1, das[b]));
+            const float p2 = __fmul_rn(static_cast<float>(S2), __fmul_rn(a2, das[b]));
+            tb[p] = __fadd_rn(p1, p2);
+            if (kSums) {
+                const int64_t o = (tile * ROWS + r) * L + b;
+                S1o[o] = S1;
+                S2o[o] = S2;
+            }
+        }
+        __syncwarp();
+        if (tile + 2 * NW < tiles) {
+            fence_proxy_async_smem();
+            issue(tile + 2 * NW, s);
+        }
+        if (lane < ROWS) {
+            float acc = 0.0f;
+            for (int b = 0; b < L; ++b) acc = __fadd_rn(acc, tb[lane * L + b]);
+            y[tile * ROWS + lane] = acc;
+        }
+        __syncwarp();
+    }
+}
+
+}  // namespace
+
+int64_t free_bytes(int64_t n, int64_t k) {
+    if (n < 0 || k < 0 || n % ROWS || k % QK) return -1;
+    return (n / ROWS) * (k / QK) * FR_BLOCK;
+}
+
+cudaError_t launch_pack_free(const int8_t *t1, const int8_t *t2, const uint16_t *a1, const uint16_t *a2, int64_t n,
+                             int64_t k, void *out, int *status, cudaStream_t st) {
+    const int64_t warps = n * (k / QK);
+    if (warps == 0) return cudaSuccess;
+    pack_free_kernel<<<static_cast<unsigned>((warps * 32 + 255) / 256), 256, 0, st>>>(
+        t1, t2, a1, a2, n, k, static_cast<uint8_t *>(out), status);
+    return cudaGetLastError();
+}
+
+int gemv_free_smem(int64_t k, int *warps_out) {
+    FreeGeo g{};
+    g.L = static_cast<int>(k / QK);
+    g.tile = g.L * FR_BLOCK;
+    const int budget = max_smem_optin() - free_act_bytes(g.L);
+    int w = budget / free_warp_bytes(g);
+    if (w > 8) w = 8;
+    if (warps_out) *warps_out = w;
+    return w > 0 ? free_act_bytes(g.L) + w * free_warp_bytes(g) : -1;
+}
+
+cudaError_t launch_gemv_free(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
+                             const int32_t *bsum, float *y, int32_t *S1, int32_t *S2, int *status,
+                             cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    FreeGeo g{};
+    g.n = n;
+    g.k = k;
+    g.L = static_cast<int>(k / QK);
+    g.tile = g.L * FR_BLOCK;
+    const int smem = gemv_free_smem(k, &g.warps);
+    if (smem < 0) return cudaErrorInvalidValue;
+    static unsigned char set[2][64];
+    const bool sums = S1 != nullptr;
+    const void *fn = sums ? reinterpret_cast<const void *>(gemv_free_kernel<true>)
+                          : reinterpret_cast<const void *>(gemv_free_kernel<false>);
+    cudaError_t e = allow_max_smem(fn, set[sums ? 1 : 0]);
+    if (e != cudaSuccess) return e;
+    const int64_t tiles = n / ROWS;
+    int64_t grid = (tiles + 2 * g.warps - 1) / (2 * g.warps);
+    const int64_t per_sm = max_smem_optin() / (smem + 1024);
+    const int64_t cap = static_cast<int64_t>(num_sms()) * (per_sm > 0 ? per_sm : 1);
+    if (grid > cap) grid = cap;
+    const unsigned gr = static_cast<unsigned>(grid);
+    const uint8_t *b = static_cast<const uint8_t *>(blocks);
+    if (sums)
+        gemv_free_kernel<true><<<gr, g.warps * 32, smem, st>>>(b, g, q, da, bsum, y, S1, S2, status);
+    else
+        gemv_free_kernel<false><<<gr, g.warps * 32, smem, st>>>(b, g, q, da, bsum, y, nullptr, nullptr, status);
+    return cudaGetLastError();
+}
+
+}  // namespace tq

@@ -40,6 +40,12 @@ inline cudaError_t record_stage_event(cudaEvent_t ev, cudaStream_t st) {
                                                                                   : cudaEventRecordDefault);
 }
 int mxfp4_gemv_smem(int64_t k, int acts);
+int64_t free_bytes(int64_t n, int64_t k);
+int gemv_free_smem(int64_t k, int *warps_out);
+cudaError_t launch_pack_free(const int8_t *t1, const int8_t *t2, const uint16_t *a1, const uint16_t *a2, int64_t n,
+                             int64_t k, void *out, int *status, cudaStream_t st);
+cudaError_t launch_gemv_free(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
+                             const int32_t *bsum, float *y, int32_t *S1, int32_t *S2, int *status, cudaStream_t st);
 cudaError_t launch_moe_mxfp4_experts(const MoeArgs &a, float *out, cudaStream_t st, const cudaEvent_t *ev);
 cudaError_t launch_moe_route(const MoeArgs &a, const float *x, int32_t *sel_idx, float *sel_w, cudaStream_t st);
 cudaError_t launch_moe_experts(const MoeArgs &a, const void *const *ptrs, float *out, cudaStream_t st);

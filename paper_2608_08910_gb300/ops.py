@@ -68,3 +68,22 @@ def gemv_mxfp4(blocks, n: int, k: int, q, da, ws, block_sums: bool = False):
     S = torch.empty((n, k // 32), dtype=torch.int32, device=blocks.device) if block_sums else None
     B.tqfx4_gemv_mxfp4(blocks, n, k, q, da, y, S, ws)
     return (y, S) if block_sums else y
+
+
+def pack_free(t1, t2, a1, a2, ws):
+    """Two trit planes int8 [n][k] and their f16 scales [n][k/256] -> blocks
+    of the free-scale two-plane format."""
+    n, k = t1.shape
+    out = torch.empty(B.tqfx4_free_bytes(n, k), dtype=torch.uint8, device=t1.device)
+    B.tqfx4_pack_free(t1, t2, a1, a2, n, k, out, ws)
+    return out
+
+
+def gemv_free(blocks, n: int, k: int, q, da, bsum, ws, block_sums: bool = False):
+    y = torch.empty(n, dtype=torch.float32, device=blocks.device)
+    S1 = S2 = None
+    if block_sums:
+        S1 = torch.empty((n, k // 256), dtype=torch.int32, device=blocks.device)
+        S2 = torch.empty((n, k // 256), dtype=torch.int32, device=blocks.device)
+    B.tqfx4_gemv_free(blocks, n, k, q, da, bsum, y, S1, S2, ws)
+    return (y, S1, S2) if block_sums else y
