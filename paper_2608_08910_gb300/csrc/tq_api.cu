@@ -156,7 +156,8 @@ tqfx4_status tqfx4_gemv_free(const void *blocks, int64_t n, int64_t k, const int
     if (!aligned(blocks, 16) || !aligned(q, 16) || !aligned(da, 4) || !aligned(bsum, 4) || !aligned(y, 4) ||
         !aligned(S1, 4) || !aligned(S2, 4))
         return fail(TQFX4_EALIGN, "%s: blocks and q must be 16-byte aligned", fn);
-    if (tq::gemv_free_smem(k, nullptr) < 0) return fail(TQFX4_ESHAPE, "%s: k too large for shared memory", fn);
+    if (tq::gemv_free_smem(k) > tq::max_smem_optin())
+        return fail(TQFX4_ESHAPE, "%s: k too large for shared memory", fn);
     cudaError_t e = tq::launch_gemv_free(blocks, n, k, q, da, bsum, y, S1, S2, static_cast<int *>(ws),
                                          static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, fn);

@@ -13,8 +13,10 @@
 // tqfx4_gemv_free: the two-plane dot pass. Exact sums S = sum t q per plane
 // and block, then per block float(S1) * (a1 * da) + float(S2) * (a2 * da)
 // added to the row's sum in block order (the oracle's schedule). A warp
-// takes one row group (4 rows, all of k) per tile through a ring of bulk
-// copies; lane l takes the (row, block) pairs l, l + 32, ... . A plane word
+// takes row groups (4 rows) and streams each as chunks of up to 8 blocks
+// (4224 bytes) through a three-slot ring of bulk copies; in a chunk lane l
+// takes the (row, block) pair l, and lanes 0..3 carry the row sums from
+// chunk to chunk. A plane word
 // holds 16 trits; its four 2-bit fields per byte are masked in place
 // (x & (0x03030303 << 2i), no shift) so that the unsigned x signed dp4a
 // sums 4^i u q into accumulator i; the four accumulators are shifted back
@@ -29,7 +31,9 @@ namespace tq {
 namespace {
 
 constexpr int FR_BLOCK = 528, FR_PLANE_OFS = 16, FR_ROW = 128;
-constexpr int FR_SLOTS = 2;
+constexpr int FR_SLOTS = 3;
+constexpr int FR_WARPS = 8;
+constexpr int FR_CHUNK = 8;  // blocks of a row group per copy: 4 rows x 8 blocks = one pair per lane
 
 __global__ void __launch_bounds__(256) pack_free_kernel(const int8_t *__restrict__ t1, const int8_t *__restrict__ t2,
                                                         const uint16_t *__restrict__ a1,
@@ -101,14 +105,14 @@ __device__ __forceinline__ bool free_wait(uint64_t *bar, uint32_t parity) {
 
 struct FreeGeo {
     int64_t n, k;
-    int L;          // 256-blocks per row
-    int tile;       // bytes of a row group (L * 528)
-    int warps;
+    int L;  // 256-blocks per row
+    int C;  // blocks per chunk (one bulk copy): min(8, L)
+    int Q;  // chunks per row group
 };
 
 __host__ __device__ inline int free_act_bytes(int L) { return ((L * (QK + 8) + 127) / 128) * 128; }
 __host__ __device__ inline int free_warp_bytes(const FreeGeo &g) {
-    return FR_SLOTS * g.tile + 4 * 4 * g.L + 32;
+    return FR_SLOTS * g.C * FR_BLOCK + 4 * ROWS * g.C + 32;
 }
 
 // The fields of plane word w of a block: byte b of transposed word i is
@@ -121,38 +125,48 @@ __device__ __forceinline__ uint4 free_transpose(uint4 v) {
 }
 
 template <bool kSums>
-__global__ void __launch_bounds__(256) gemv_free_kernel(const uint8_t *__restrict__ blocks, FreeGeo g,
-                                                        const int8_t *__restrict__ q, const float *__restrict__ da,
-                                                        const int32_t *__restrict__ bsum, float *__restrict__ y,
-                                                        int32_t *__restrict__ S1o, int32_t *__restrict__ S2o,
-                                                        int *status) {
+__global__ void __launch_bounds__(FR_WARPS * 32) gemv_free_kernel(const uint8_t *__restrict__ blocks, FreeGeo g,
+                                                                  const int8_t *__restrict__ q,
+                                                                  const float *__restrict__ da,
+                                                                  const int32_t *__restrict__ bsum,
+                                                                  float *__restrict__ y, int32_t *__restrict__ S1o,
+                                                                  int32_t *__restrict__ S2o, int *status) {
     extern __shared__ __align__(128) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int L = g.L;
+    const int L = g.L, C = g.C, Q = g.Q;
     uint4 *qv = reinterpret_cast<uint4 *>(smem);  // [16 words][L blocks]
     float *das = reinterpret_cast<float *>(smem + L * QK);
     int *bss = reinterpret_cast<int *>(smem + L * QK + 4 * L);
     uint8_t *wbase = smem + free_act_bytes(L) + warp * free_warp_bytes(g);
     uint8_t *slots = wbase;
-    float *tb = reinterpret_cast<float *>(wbase + FR_SLOTS * g.tile);  // [4 rows][L]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(wbase + FR_SLOTS * g.tile + 16 * L);
+    const int slot = C * FR_BLOCK;
+    float *tb = reinterpret_cast<float *>(wbase + FR_SLOTS * slot);  // [4 rows][C]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(wbase + FR_SLOTS * slot + 4 * ROWS * C);
     if (lane == 0)
         for (int i = 0; i < FR_SLOTS; ++i) mbar_init(&bars[i], 1);
     fence_barrier_init();
 
-    const int64_t tiles = g.n / ROWS;
-    const int64_t NW = static_cast<int64_t>(gridDim.x) * g.warps;
-    const int64_t first = static_cast<int64_t>(blockIdx.x) * g.warps + warp;
+    // a warp's work: row groups first, first + NW, ..., each as Q chunks in
+    // order; u numbers the warp's chunks
+    const int64_t groups = g.n / ROWS;
+    const int64_t NW = static_cast<int64_t>(gridDim.x) * FR_WARPS;
+    const int64_t first = static_cast<int64_t>(blockIdx.x) * FR_WARPS + warp;
+    const int64_t my_groups = first < groups ? (groups - first + NW - 1) / NW : 0;
+    const int64_t units = my_groups * Q;
     const uint64_t policy = l2_policy_evict_first();
-    auto issue = [&](int64_t tile, int s) {
+    auto chunk_blocks = [&](int qi) { return qi == Q - 1 ? L - qi * C : C; };
+    auto issue = [&](int64_t u, int s) {
         if (lane == 0) {
-            mbar_arrive_expect_tx(&bars[s], static_cast<uint32_t>(g.tile));
-            bulk_g2s_hint(slots + s * g.tile, blocks + tile * g.tile, static_cast<uint32_t>(g.tile), &bars[s],
-                          policy);
+            const int64_t rg = first + (u / Q) * NW;
+            const int qi = static_cast<int>(u % Q);
+            const uint32_t bytes = static_cast<uint32_t>(chunk_blocks(qi) * FR_BLOCK);
+            mbar_arrive_expect_tx(&bars[s], bytes);
+            bulk_g2s_hint(slots + s * slot, blocks + (rg * L + static_cast<int64_t>(qi) * C) * FR_BLOCK, bytes,
+                          &bars[s], policy);
         }
     };
-    if (first < tiles) issue(first, 0);
-    if (first + NW < tiles) issue(first + NW, 1);
+    if (units > 0) issue(0, 0);
+    if (units > 1) issue(1, 1);
     for (int idx = threadIdx.x; idx < 16 * L; idx += blockDim.x) {
         const int b = idx % L, wd = idx / L;
         qv[idx] = free_transpose(__ldg(reinterpret_cast<const uint4 *>(q + b * QK + 16 * wd)));
@@ -163,18 +177,26 @@ __global__ void __launch_bounds__(256) gemv_free_kernel(const uint8_t *__restric
     }
     __syncthreads();
 
-    const int pairs = ROWS * L;
-    int it = 0;
-    for (int64_t tile = first; tile < tiles; tile += NW, ++it) {
-        const int s = it & 1;
-        if (!__all_sync(0xffffffffu, free_wait(&bars[s], static_cast<uint32_t>((it >> 1) & 1)))) {
-            if (lane == 0) report(status, TQFX4_ETIMEOUT, K_GEMV, static_cast<int>(tile));
+    float acc = 0.0f;  // lanes 0..3: the running sum of row `lane` of the current group
+    int s = 0, ph = 0;
+    for (int64_t u = 0; u < units; ++u) {
+        if (!__all_sync(0xffffffffu, free_wait(&bars[s], static_cast<uint32_t>(ph)))) {
+            if (lane == 0) report(status, TQFX4_ETIMEOUT, K_GEMV, static_cast<int>(u));
             break;
         }
-        const uint8_t *tp = slots + s * g.tile;
-        for (int p = lane; p < pairs; p += 32) {
-            const int r = p / L, b = p - r * L;
-            const uint8_t *blk = tp + b * FR_BLOCK;
+        // the slot of the previous chunk (read before the last __syncwarp)
+        // takes the chunk two ahead
+        if (u + 2 < units) {
+            fence_proxy_async_smem();
+            issue(u + 2, s == 0 ? FR_SLOTS - 1 : s - 1);
+        }
+        const int64_t rg = first + (u / Q) * NW;
+        const int qi = static_cast<int>(u % Q);
+        const int cb = chunk_blocks(qi);
+        const uint8_t *tp = slots + s * slot;
+        for (int p = lane; p < ROWS * cb; p += 32) {
+            const int r = p / cb, bl = p - r * cb, b = qi * C + bl;
+            const uint8_t *blk = tp + bl * FR_BLOCK;
             const uint4 *pl = reinterpret_cast<const uint4 *>(blk + FR_PLANE_OFS + FR_ROW * r);
             const int S1 = free_plane_sum(pl, qv + b, L) - bss[b];
             const int S2 = free_plane_sum(pl + 4, qv + b, L) - bss[b];
@@ -182,24 +204,24 @@ __global__ void __launch_bounds__(256) gemv_free_kernel(const uint8_t *__restric
             const float a2 = __half2float(reinterpret_cast<const __half *>(blk + 8)[r]);
             const float p1 = __fmul_rn(static_cast<float>(S1), __fmul_rn(a1, das[b]));
             const float p2 = __fmul_rn(static_cast<float>(S2), __fmul_rn(a2, das[b]));
-            tb[p] = __fadd_rn(p1, p2);
+            tb[r * C + bl] = __fadd_rn(p1, p2);
             if (kSums) {
-                const int64_t o = (tile * ROWS + r) * L + b;
+                const int64_t o = (rg * ROWS + r) * L + b;
                 S1o[o] = S1;
                 S2o[o] = S2;
             }
         }
         __syncwarp();
-        if (tile + 2 * NW < tiles) {
-            fence_proxy_async_smem();
-            issue(tile + 2 * NW, s);
-        }
         if (lane < ROWS) {
-            float acc = 0.0f;
-            for (int b = 0; b < L; ++b) acc = __fadd_rn(acc, tb[lane * L + b]);
-            y[tile * ROWS + lane] = acc;
+            if (qi == 0) acc = 0.0f;
+            for (int bl = 0; bl < cb; ++bl) acc = __fadd_rn(acc, tb[lane * C + bl]);
+            if (qi == Q - 1) y[rg * ROWS + lane] = acc;
         }
         __syncwarp();
+        if (++s == FR_SLOTS) {
+            s = 0;
+            ph ^= 1;
+        }
     }
 }
 
@@ -219,15 +241,11 @@ cudaError_t launch_pack_free(const int8_t *t1, const int8_t *t2, const uint16_t 
     return cudaGetLastError();
 }
 
-int gemv_free_smem(int64_t k, int *warps_out) {
+int gemv_free_smem(int64_t k) {
     FreeGeo g{};
     g.L = static_cast<int>(k / QK);
-    g.tile = g.L * FR_BLOCK;
-    const int budget = max_smem_optin() - free_act_bytes(g.L);
-    int w = budget / free_warp_bytes(g);
-    if (w > 8) w = 8;
-    if (warps_out) *warps_out = w;
-    return w > 0 ? free_act_bytes(g.L) + w * free_warp_bytes(g) : -1;
+    g.C = g.L < FR_CHUNK ? g.L : FR_CHUNK;
+    return free_act_bytes(g.L) + FR_WARPS * free_warp_bytes(g);
 }
 
 cudaError_t launch_gemv_free(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
@@ -238,26 +256,27 @@ cudaError_t launch_gemv_free(const void *blocks, int64_t n, int64_t k, const int
     g.n = n;
     g.k = k;
     g.L = static_cast<int>(k / QK);
-    g.tile = g.L * FR_BLOCK;
-    const int smem = gemv_free_smem(k, &g.warps);
-    if (smem < 0) return cudaErrorInvalidValue;
+    g.C = g.L < FR_CHUNK ? g.L : FR_CHUNK;
+    g.Q = (g.L + g.C - 1) / g.C;
+    const int smem = gemv_free_smem(k);
+    if (smem > max_smem_optin()) return cudaErrorInvalidValue;
     static unsigned char set[2][64];
     const bool sums = S1 != nullptr;
     const void *fn = sums ? reinterpret_cast<const void *>(gemv_free_kernel<true>)
                           : reinterpret_cast<const void *>(gemv_free_kernel<false>);
     cudaError_t e = allow_max_smem(fn, set[sums ? 1 : 0]);
     if (e != cudaSuccess) return e;
-    const int64_t tiles = n / ROWS;
-    int64_t grid = (tiles + 2 * g.warps - 1) / (2 * g.warps);
+    const int64_t groups = n / ROWS;
+    int64_t grid = (groups + FR_WARPS - 1) / FR_WARPS;
     const int64_t per_sm = max_smem_optin() / (smem + 1024);
     const int64_t cap = static_cast<int64_t>(num_sms()) * (per_sm > 0 ? per_sm : 1);
     if (grid > cap) grid = cap;
     const unsigned gr = static_cast<unsigned>(grid);
     const uint8_t *b = static_cast<const uint8_t *>(blocks);
     if (sums)
-        gemv_free_kernel<true><<<gr, g.warps * 32, smem, st>>>(b, g, q, da, bsum, y, S1, S2, status);
+        gemv_free_kernel<true><<<gr, FR_WARPS * 32, smem, st>>>(b, g, q, da, bsum, y, S1, S2, status);
     else
-        gemv_free_kernel<false><<<gr, g.warps * 32, smem, st>>>(b, g, q, da, bsum, y, nullptr, nullptr, status);
+        gemv_free_kernel<false><<<gr, FR_WARPS * 32, smem, st>>>(b, g, q, da, bsum, y, nullptr, nullptr, status);
     return cudaGetLastError();
 }
 

@@ -41,7 +41,7 @@ inline cudaError_t record_stage_event(cudaEvent_t ev, cudaStream_t st) {
 }
 int mxfp4_gemv_smem(int64_t k, int acts);
 int64_t free_bytes(int64_t n, int64_t k);
-int gemv_free_smem(int64_t k, int *warps_out);
+int gemv_free_smem(int64_t k);
 cudaError_t launch_pack_free(const int8_t *t1, const int8_t *t2, const uint16_t *a1, const uint16_t *a2, int64_t n,
                              int64_t k, void *out, int *status, cudaStream_t st);
 cudaError_t launch_gemv_free(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
