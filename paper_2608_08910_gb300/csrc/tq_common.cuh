@@ -378,4 +378,37 @@ __device__ __forceinline__ bool quant_block_warp(const float v[8], uint2 &packed
     return __all_sync(0xffffffffu, finite);
 }
 
+// e4m3 byte of the integer a in 0..8 (exact): 0, 1 -> 0x38 (2^0), 2 -> 0x40,
+// 3 -> 0x44, 4 -> 0x48, 5 -> 0x4A, 6 -> 0x4C, 7 -> 0x4E, 8 -> 0x50, by a
+// byte permute over the first eight.
+__device__ __forceinline__ uint32_t e4m3_mag(uint32_t a) {
+    const uint32_t t = __byte_perm(0x44403800u, 0x4E4C4A48u, a & 7u) & 0xFFu;
+    return a == 8u ? 0x50u : t;
+}
+
+// Eight int8 activations q as the two e4m3 planes of q = 16 h + l, with
+// h = floor((q + 8) / 16) in -8..8 and l in -8..7: bytes of 16 h and of l.
+__device__ __forceinline__ void q_planes8(uint2 v, uint2 &hi, uint2 &lo) {
+    uint32_t hw[2], lw[2];
+#pragma unroll
+    for (int w = 0; w < 2; ++w) {
+        const uint32_t word = w ? v.y : v.x;
+        hw[w] = lw[w] = 0u;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int q = static_cast<int>(word << (24 - 8 * i)) >> 24;  // signed byte i
+            const int h = (q + 8) >> 4;                                  // arithmetic shift: floor
+            const int l = q - 16 * h;
+            const uint32_t ah = static_cast<uint32_t>(h < 0 ? -h : h), al = static_cast<uint32_t>(l < 0 ? -l : l);
+            // 16 h: four more in the exponent than h
+            const uint32_t hb = ah ? ((e4m3_mag(ah) + 0x20u) | (h < 0 ? 0x80u : 0u)) : 0u;
+            const uint32_t lb = e4m3_mag(al) | (l < 0 ? 0x80u : 0u);
+            hw[w] |= hb << (8 * i);
+            lw[w] |= lb << (8 * i);
+        }
+    }
+    hi = make_uint2(hw[0], hw[1]);
+    lo = make_uint2(lw[0], lw[1]);
+}
+
 }  // namespace tq

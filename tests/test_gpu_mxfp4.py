@@ -48,6 +48,21 @@ def test_gemv_mxfp4_bit_exact(n, k, ws):
     assert rel_err(got, ry) <= FP32_TOL
 
 
+# without block sums (the kernel variant that skips them): rows not a
+# multiple of the 16 rows a CTA starts with, k from one to 32 units of 512,
+# and the largest k
+TC_SHAPES = [(1, 512), (128, 512), (300, 1536), (2048, 4096), (4096, 2048), (1000, 8192), (5, 16384)]
+
+
+@pytest.mark.parametrize("n,k", TC_SHAPES)
+def test_gemv_mxfp4_without_sums_bit_exact(n, k, ws):
+    blocks, q, da = _case(n, k, 7 * n + k)
+    ry, _ = oracle.mxfp4_gemv(blocks.numpy(), n, k, q, da)
+    y = ops.gemv_mxfp4(blocks.to(DEV), n, k, torch.from_numpy(q).to(DEV), torch.from_numpy(da).to(DEV), ws)
+    B.tqfx4_check(ws)
+    assert np.array_equal(y.cpu().numpy().view(np.uint32), ry.view(np.uint32))
+
+
 def test_gemv_mxfp4_uses_device_quantized_activation(ws):
     # the activation from the library's own quantizer, as the decode path feeds it
     n, k = 512, 4096
