@@ -488,6 +488,10 @@ def run_tiered(args, rank, world, local):
         dist.destroy_process_group()
 
 GEMV_N, GEMV_K, GEMV_POOL = 131072, 4096, 16
+# DRAM bytes (read + write) of one launch of the GEMV kernels on the 131072 x
+# 4096 workload, from ncu --set full captures (profiles/); None once a kernel
+# changes until it is captured again.
+GEMV_TRAFFIC = {"mxfp4_gemv": 285286144 + 3272960, "free_gemv": 276862976 + 3671296}
 
 
 def run_gemv(args, rank, world, local):
@@ -640,7 +644,7 @@ def run_gemv(args, rank, world, local):
                            "matrix_bytes": fx_bytes, "gemv_us": g_fx_s * 1e6,
                            "gemv_gbs": fx_bytes / g_fx_s / 1e9},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": None,
+                     "frac": achieved / peak, "traffic": GEMV_TRAFFIC[args.workload],
                      "kernel": "gemv_free_kernel" if free else "mxfp4_gemv_kernel",
                      "peak_source": peak_kind, "stage_us": {"quantize_act": q_mx * 1e6, "gemv": g_mx_s * 1e6}},
         "e2e": {"value": job_rate(mx_bytes * args.steps, world, te) / 1e9, "unit": "GB/s",

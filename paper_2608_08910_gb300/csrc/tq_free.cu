@@ -155,18 +155,23 @@ __global__ void __launch_bounds__(FR_WARPS * 32) gemv_free_kernel(const uint8_t 
     const int64_t units = my_groups * Q;
     const uint64_t policy = l2_policy_evict_first();
     auto chunk_blocks = [&](int qi) { return qi == Q - 1 ? L - qi * C : C; };
-    auto issue = [&](int64_t u, int s) {
+    // the next chunk to copy (row group, chunk), advanced by every lane alike
+    int64_t rg_n = first;
+    int qi_n = 0;
+    auto issue_next = [&](int s) {
         if (lane == 0) {
-            const int64_t rg = first + (u / Q) * NW;
-            const int qi = static_cast<int>(u % Q);
-            const uint32_t bytes = static_cast<uint32_t>(chunk_blocks(qi) * FR_BLOCK);
+            const uint32_t bytes = static_cast<uint32_t>(chunk_blocks(qi_n) * FR_BLOCK);
             mbar_arrive_expect_tx(&bars[s], bytes);
-            bulk_g2s_hint(slots + s * slot, blocks + (rg * L + static_cast<int64_t>(qi) * C) * FR_BLOCK, bytes,
+            bulk_g2s_hint(slots + s * slot, blocks + (rg_n * L + static_cast<int64_t>(qi_n) * C) * FR_BLOCK, bytes,
                           &bars[s], policy);
         }
+        if (++qi_n == Q) {
+            qi_n = 0;
+            rg_n += NW;
+        }
     };
-    if (units > 0) issue(0, 0);
-    if (units > 1) issue(1, 1);
+    if (units > 0) issue_next(0);
+    if (units > 1) issue_next(1);
     for (int idx = threadIdx.x; idx < 16 * L; idx += blockDim.x) {
         const int b = idx % L, wd = idx / L;
         qv[idx] = free_transpose(__ldg(reinterpret_cast<const uint4 *>(q + b * QK + 16 * wd)));
@@ -179,6 +184,8 @@ __global__ void __launch_bounds__(FR_WARPS * 32) gemv_free_kernel(const uint8_t 
 
     float acc = 0.0f;  // lanes 0..3: the running sum of row `lane` of the current group
     int s = 0, ph = 0;
+    int64_t rg = first;  // the current chunk (row group, chunk)
+    int qi = 0;
     for (int64_t u = 0; u < units; ++u) {
         if (!__all_sync(0xffffffffu, free_wait(&bars[s], static_cast<uint32_t>(ph)))) {
             if (lane == 0) report(status, TQFX4_ETIMEOUT, K_GEMV, static_cast<int>(u));
@@ -188,14 +195,12 @@ __global__ void __launch_bounds__(FR_WARPS * 32) gemv_free_kernel(const uint8_t 
         // takes the chunk two ahead
         if (u + 2 < units) {
             fence_proxy_async_smem();
-            issue(u + 2, s == 0 ? FR_SLOTS - 1 : s - 1);
+            issue_next(s == 0 ? FR_SLOTS - 1 : s - 1);
         }
-        const int64_t rg = first + (u / Q) * NW;
-        const int qi = static_cast<int>(u % Q);
         const int cb = chunk_blocks(qi);
         const uint8_t *tp = slots + s * slot;
-        for (int p = lane; p < ROWS * cb; p += 32) {
-            const int r = p / cb, bl = p - r * cb, b = qi * C + bl;
+        auto pair = [&](int r, int bl) {
+            const int b = qi * C + bl;
             const uint8_t *blk = tp + bl * FR_BLOCK;
             const uint4 *pl = reinterpret_cast<const uint4 *>(blk + FR_PLANE_OFS + FR_ROW * r);
             const int S1 = free_plane_sum(pl, qv + b, L) - bss[b];
@@ -210,6 +215,14 @@ __global__ void __launch_bounds__(FR_WARPS * 32) gemv_free_kernel(const uint8_t 
                 S1o[o] = S1;
                 S2o[o] = S2;
             }
+        };
+        if (cb == FR_CHUNK) {
+            pair(lane >> 3, lane & 7);  // a full chunk: one pair per lane
+        } else {
+            for (int p = lane; p < ROWS * cb; p += 32) {
+                const int r = p / cb;
+                pair(r, p - r * cb);
+            }
         }
         __syncwarp();
         if (lane < ROWS) {
@@ -218,6 +231,10 @@ __global__ void __launch_bounds__(FR_WARPS * 32) gemv_free_kernel(const uint8_t 
             if (qi == Q - 1) y[rg * ROWS + lane] = acc;
         }
         __syncwarp();
+        if (++qi == Q) {
+            qi = 0;
+            rg += NW;
+        }
         if (++s == FR_SLOTS) {
             s = 0;
             ph ^= 1;
