@@ -50,10 +50,10 @@ __global__ void __launch_bounds__(256, 1) gemv_kernel(const uint8_t *__restrict_
     job.das = das;
     job.bss = bss;
     job.nb = nb;
-    if (job.rg_begin < job.rg_end) warp_stream_prefetch(ring, &job, 1, g.rpu, warp, g.warps);
+    if (job.rg_begin < job.rg_end) warp_stream_prefetch(ring, job, g.rpu, warp, g.warps);
     load_act_smem(q, da, bsum, nb, qs, das, bss);
     __syncthreads();
-    if (job.rg_begin < job.rg_end) warp_stream_run(ring, &job, 1, g.rpu, warp, g.warps, status, K_GEMV);
+    if (job.rg_begin < job.rg_end) warp_stream_run(ring, job, g.rpu, warp, g.warps, status, K_GEMV);
 }
 
 __global__ void zero_kernel(float *y, int64_t n) {

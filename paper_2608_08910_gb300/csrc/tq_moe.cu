@@ -146,11 +146,13 @@ __global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
     q.dyn_ctr = a.ctr + kCtrGateUp;
     q.dyn_base = static_cast<int64_t>(gridDim.x) * a.static_gu;
     q.total = total;
+    const int upm32 = static_cast<int>(upm);  // units are few: 32-bit index arithmetic
     auto map = [&](int64_t u) {
-        const int j = static_cast<int>(u / (2 * upm));
-        const int64_t rem = u - static_cast<int64_t>(j) * 2 * upm;
-        const int qq = rem >= upm;
-        const int64_t r = rem - qq * upm;
+        const int u32 = static_cast<int>(u);
+        const int j = u32 / (2 * upm32);
+        const int rem = u32 - j * 2 * upm32;
+        const int qq = rem >= upm32;
+        const int64_t r = rem - qq * upm32;
         UnitRef U;
         U.mat = a.ptrs ? ptr_s[qq * a.top_k + j] : (qq ? a.up : a.gate) + static_cast<int64_t>(sel_s[j]) * a.mb_gu;
         U.rg0 = r * a.rpu_gu;
@@ -198,7 +200,7 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
     job.bss = bss;
     job.nb = nbi;
     const bool any = job.rg_begin < job.rg_end;
-    if (any) warp_stream_prefetch(ring, &job, 1, a.rpu_d, warp, a.warps_d, 1);
+    if (any) warp_stream_prefetch(ring, job, a.rpu_d, warp, a.warps_d, 1);
     if (warp == a.warps_d - 1) {
         // the routing weights (needed by the combine at the end); the router
         // has completed, so this runs while gate/up drains
@@ -261,10 +263,10 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
             }
         }
     }
-    if (any) warp_stream_prefetch_from(ring, &job, 1, a.rpu_d, warp, a.warps_d, 1);
+    if (any) warp_stream_prefetch_from(ring, job, a.rpu_d, warp, a.warps_d, 1);
     __syncthreads();
     TQ_STAMP(2, 3);
-    if (any) warp_stream_run(ring, &job, 1, a.rpu_d, warp, a.warps_d, a.status, K_DOWN);
+    if (any) warp_stream_run(ring, job, a.rpu_d, warp, a.warps_d, a.status, K_DOWN);
     __syncthreads();
     TQ_STAMP(2, 4);
     if (threadIdx.x == 0) last = (atomic_add_acq_rel(&a.ctr[kCtrDown + p], 1) == K - 1);

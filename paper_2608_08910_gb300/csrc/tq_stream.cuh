@@ -63,86 +63,73 @@ __device__ __forceinline__ void ring_init(const WarpRing &r) {
         for (int s = 0; s < r.stages; ++s) mbar_init(&r.bars[s], 1);
 }
 
-// Locate global unit u of the concatenated jobs.
-__device__ __forceinline__ void unit_locate(const MatJob *jobs, int njobs, int rpu, int64_t u, int &q,
-                                            int64_t &rg0, int &rgs) {
-    q = 0;
-    int64_t n0 = job_units(jobs[0], rpu);
-    while (q + 1 < njobs && u >= n0) {
-        u -= n0;
-        ++q;
-        n0 = job_units(jobs[q], rpu);
-    }
-    rg0 = jobs[q].rg_begin + u * rpu;
-    rgs = static_cast<int>(imin64(rpu, jobs[q].rg_end - rg0));
+// Unit u of a job: rgs row groups from rg0 (a multiplication, no division).
+__device__ __forceinline__ void unit_locate(const MatJob &j, int rpu, int64_t u, int64_t &rg0, int &rgs) {
+    rg0 = j.rg_begin + u * rpu;
+    rgs = static_cast<int>(imin64(rpu, j.rg_end - rg0));
 }
 
-__device__ __forceinline__ void unit_issue(const WarpRing &r, const MatJob *jobs, int njobs, int rpu, int64_t u,
-                                           int slot) {
-    int q, rgs;
+__device__ __forceinline__ void unit_issue(const WarpRing &r, const MatJob &j, int rpu, int64_t u, int slot) {
+    int rgs;
     int64_t rg0;
-    unit_locate(jobs, njobs, rpu, u, q, rg0, rgs);
-    const int64_t stripe = static_cast<int64_t>(jobs[q].nb) * BLOCK_BYTES;
+    unit_locate(j, rpu, u, rg0, rgs);
+    const int64_t stripe = static_cast<int64_t>(j.nb) * BLOCK_BYTES;
     uint8_t *dst[2] = {r.slots + slot * r.slot_bytes, nullptr};
-    const uint8_t *src[2] = {jobs[q].mat + rg0 * stripe, nullptr};
+    const uint8_t *src[2] = {j.mat + rg0 * stripe, nullptr};
     const uint32_t bytes[2] = {static_cast<uint32_t>(rgs * stripe), 0u};
     uint32_t ofs[2];
     stage_ranges(threadIdx.x & 31, 1, dst, src, bytes, &r.bars[slot], ofs);
 }
 
-__device__ __forceinline__ int64_t jobs_total_units(const MatJob *jobs, int njobs, int rpu) {
-    int64_t total = 0;
-    for (int q = 0; q < njobs; ++q) total += job_units(jobs[q], rpu);
-    return total;
-}
-
 // Issue the first `stages` units of this warp's share (units first, first +
-// step, ...). Only the matrix pointers and row ranges of the jobs are used,
-// so this may run before the activations are in shared memory.
-__device__ __forceinline__ void warp_stream_prefetch(const WarpRing &r, const MatJob *jobs, int njobs, int rpu,
-                                                     int64_t first, int64_t step, int max_stages = 1 << 30) {
-    const int64_t total = jobs_total_units(jobs, njobs, rpu);
+// step, ...) of the job. Only its matrix pointer and row range are used, so
+// this may run before the activations are in shared memory.
+__device__ __forceinline__ void warp_stream_prefetch(const WarpRing &r, const MatJob &j, int rpu, int64_t first,
+                                                     int64_t step, int max_stages = 1 << 30) {
+    const int64_t total = job_units(j, rpu);
     int64_t nx = first;
     for (int s = 0; s < r.stages && s < max_stages; ++s, nx += step)
-        if (nx < total) unit_issue(r, jobs, njobs, rpu, nx, s);
+        if (nx < total) unit_issue(r, j, rpu, nx, s);
 }
 
 // Issue the remaining prefetch slots [from, stages) after a partial
 // warp_stream_prefetch(..., from).
-__device__ __forceinline__ void warp_stream_prefetch_from(const WarpRing &r, const MatJob *jobs, int njobs,
-                                                          int rpu, int64_t first, int64_t step, int from) {
-    const int64_t total = jobs_total_units(jobs, njobs, rpu);
+__device__ __forceinline__ void warp_stream_prefetch_from(const WarpRing &r, const MatJob &j, int rpu,
+                                                          int64_t first, int64_t step, int from) {
+    const int64_t total = job_units(j, rpu);
     int64_t nx = first + from * step;
     for (int s = from; s < r.stages; ++s, nx += step)
-        if (nx < total) unit_issue(r, jobs, njobs, rpu, nx, s);
+        if (nx < total) unit_issue(r, j, rpu, nx, s);
 }
 
 // Consume this warp's units (prefetched by warp_stream_prefetch), refilling
 // each slot with the unit `stages` steps ahead. Returns false if a copy
 // never arrived (status recorded).
-__device__ __forceinline__ bool warp_stream_run(const WarpRing &r, const MatJob *jobs, int njobs, int rpu,
-                                                int64_t first, int64_t step, int *status, int kernel_id) {
+__device__ __forceinline__ bool warp_stream_run(const WarpRing &r, const MatJob &J, int rpu, int64_t first,
+                                                int64_t step, int *status, int kernel_id) {
     const int lane = threadIdx.x & 31;
-    const int64_t total = jobs_total_units(jobs, njobs, rpu);
-    int it = 0;
-    for (int64_t u = first; u < total; u += step, ++it) {
-        const int slot = it % r.stages;
-        const uint32_t parity = static_cast<uint32_t>((it / r.stages) & 1);
+    const int64_t total = job_units(J, rpu);
+    const int nb = J.nb;
+    const int64_t stripe = static_cast<int64_t>(nb) * BLOCK_BYTES;
+    const int rgl0 = lane / nb, b00 = lane - rgl0 * nb;  // the lane's first block of a unit
+    int slot = 0;
+    uint32_t parity = 0;
+    for (int64_t u = first; u < total; u += step) {
         if (!__all_sync(0xffffffffu, mbar_wait(&r.bars[slot], parity))) {
             if (lane == 0) report(status, TQFX4_ETIMEOUT, kernel_id, static_cast<int>(u));
             return false;
         }
         __syncwarp();
-        int q, rgs;
+        int rgs;
         int64_t rg0;
-        unit_locate(jobs, njobs, rpu, u, q, rg0, rgs);
-        const MatJob &J = jobs[q];
-        const int nb = J.nb;
-        const int64_t stripe = static_cast<int64_t>(nb) * BLOCK_BYTES;
+        unit_locate(J, rpu, u, rg0, rgs);
         const uint8_t *data = r.slots + slot * r.slot_bytes + src_ofs(J.mat + rg0 * stripe);
         const int nblk = rgs * nb;
-        for (int i = lane; i < nblk; i += 32) {
-            const int rgl = i / nb, b = i - rgl * nb;
+        for (int i = lane, rgl = rgl0, b = b00; i < nblk; i += 32) {
+            if (i != lane) {
+                rgl = i / nb;
+                b = i - rgl * nb;
+            }
             const uint8_t *blk = data + i * BLOCK_BYTES;
             int S[4];
             block_dot(blk + CODE_OFS, J.qs + b * QS_STRIDE, J.bss[b], S);
@@ -168,7 +155,11 @@ __device__ __forceinline__ bool warp_stream_run(const WarpRing &r, const MatJob 
         const int64_t nu = u + static_cast<int64_t>(r.stages) * step;
         if (nu < total) {
             fence_proxy_async_smem();
-            unit_issue(r, jobs, njobs, rpu, nu, slot);
+            unit_issue(r, J, rpu, nu, slot);
+        }
+        if (++slot == r.stages) {
+            slot = 0;
+            parity ^= 1u;
         }
     }
     return true;
@@ -246,14 +237,15 @@ __device__ __forceinline__ bool warp_units_run(const WarpRing &r, UnitQueue &q, 
                                                int64_t (&slot_u)[MAXST], int *status, int kernel_id) {
     const int lane = threadIdx.x & 31;
     const int64_t stripe = static_cast<int64_t>(nb) * BLOCK_BYTES;
-    for (int it = 0;; ++it) {
-        const int slot = it % r.stages;
+    const int rgl0 = lane / nb, b00 = lane - rgl0 * nb;  // the lane's first block of a unit
+    int slot = 0;
+    uint32_t parity = 0;
+    for (;; slot = (slot + 1 == r.stages) ? 0 : slot + 1, parity ^= (slot == 0) ? 1u : 0u) {
         int64_t u = -1;
 #pragma unroll
         for (int s = 0; s < MAXST; ++s)
             if (s == slot) u = slot_u[s];
         if (u < 0) break;
-        const uint32_t parity = static_cast<uint32_t>((it / r.stages) & 1);
         if (!__all_sync(0xffffffffu, mbar_wait(&r.bars[slot], parity))) {
             if (lane == 0) report(status, TQFX4_ETIMEOUT, kernel_id, static_cast<int>(u));
             return false;
@@ -262,8 +254,11 @@ __device__ __forceinline__ bool warp_units_run(const WarpRing &r, UnitQueue &q, 
         const UnitRef U = map(u);
         const uint8_t *data = r.slots + slot * r.slot_bytes + src_ofs(U.mat + U.rg0 * stripe);
         const int nblk = U.rgs * nb;
-        for (int i = lane; i < nblk; i += 32) {
-            const int rgl = i / nb, b = i - rgl * nb;
+        for (int i = lane, rgl = rgl0, b = b00; i < nblk; i += 32) {
+            if (i != lane) {
+                rgl = i / nb;
+                b = i - rgl * nb;
+            }
             const uint8_t *blk = data + i * BLOCK_BYTES;
             int S[4];
             block_dot(blk + CODE_OFS, qs + b * QS_STRIDE, bss[b], S);
