@@ -1,10 +1,12 @@
 // tqfx4_gemv: the integer dot pass of Tied Trit-Planes Sec. 2.2 on GB300.
 //
-// Data path: a matrix is one contiguous stream of 520-byte blocks. The grid
-// splits it into one contiguous range of row groups per CTA; each warp of a
-// CTA streams units of that range through its own shared-memory ring with
-// cp.async.bulk (tq_stream.cuh) and applies the fixed float schedule
-// acc = acc + float(S) * (d * da) over the blocks in ascending order.
+// Data path: a matrix is one contiguous stream of 520-byte blocks, and the
+// fixed float schedule acc = acc + float(S) * (d * da) runs over the blocks
+// of a row in ascending order. For k a multiple of 512 the chunked pass
+// below streams row groups in 8-block chunks, one (row, block) per lane;
+// otherwise (rows 8-byte aligned) the grid splits the matrix into one
+// contiguous range of row groups per CTA and each warp streams units of it
+// through the engine of tq_stream.cuh.
 #include "tq_launch.h"
 #include "tq_stream.cuh"
 
@@ -54,6 +56,152 @@ __global__ void __launch_bounds__(256, 1) gemv_kernel(const uint8_t *__restrict_
     load_act_smem(q, da, bsum, nb, qs, das, bss);
     __syncthreads();
     if (job.rg_begin < job.rg_end) warp_stream_run(ring, job, g.rpu, warp, g.warps, status, K_GEMV);
+}
+
+// ---- the chunked pass (k a multiple of 512) ----------------------------
+//
+// A warp takes row groups (first, first + NW, ...) and streams each as
+// chunks of up to 8 blocks (4160 bytes) through a three-slot ring of bulk
+// copies, 16 warps per SM. In a full chunk lane l takes row l / 8 of block
+// l % 8: the 128 code bytes of its row (element j in the low nibble of
+// byte j, element 128 + j in the high one), with the activation laid out
+// [16-byte word][block] in shared memory so that lanes on different blocks
+// read different banks. Lanes 0..3 carry their row's sum from chunk to
+// chunk; the float schedule is the one above.
+constexpr int FX_SLOTS = 3, FX_WARPS = 8, FX_CHUNK = 8;
+
+struct FxGeo {
+    int64_t n;
+    int L, C, Q;  // blocks per row group, per chunk (min(8, L)), chunks per row group
+};
+
+__host__ __device__ inline int fx_act_bytes(int L) { return ((L * (QK + 8) + 127) / 128) * 128; }
+__host__ __device__ inline int fx_warp_bytes(const FxGeo &g) {
+    return FX_SLOTS * g.C * BLOCK_BYTES + 4 * ROWS * g.C + 32;
+}
+
+// Exact S of one row of a block: 32 code words against the activation
+// words w (low nibbles) and 32 + w (high nibbles, kept at 16 u and divided
+// out), S = sum u q - 4 bsum.
+__device__ __forceinline__ int fx_row_dot(const uint2 *codes, const uint4 *qv, int L, int bsum) {
+    int lo = 0, hi = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const uint4 ql = qv[i * L], qh = qv[(8 + i) * L];  // activation words 4i..4i+3 and 32+4i..
+        const uint2 c0 = codes[2 * i], c1 = codes[2 * i + 1];
+        lo = dp4a_us(c0.x & 0x0f0f0f0fu, ql.x, lo);
+        lo = dp4a_us(c0.y & 0x0f0f0f0fu, ql.y, lo);
+        lo = dp4a_us(c1.x & 0x0f0f0f0fu, ql.z, lo);
+        lo = dp4a_us(c1.y & 0x0f0f0f0fu, ql.w, lo);
+        hi = dp4a_us(c0.x & 0xf0f0f0f0u, qh.x, hi);
+        hi = dp4a_us(c0.y & 0xf0f0f0f0u, qh.y, hi);
+        hi = dp4a_us(c1.x & 0xf0f0f0f0u, qh.z, hi);
+        hi = dp4a_us(c1.y & 0xf0f0f0f0u, qh.w, hi);
+    }
+    return lo + (hi >> 4) - 4 * bsum;
+}
+
+template <bool kSums>
+__global__ void __launch_bounds__(FX_WARPS * 32) gemv_chunk_kernel(const uint8_t *__restrict__ blocks, FxGeo g,
+                                                                   const int8_t *__restrict__ q,
+                                                                   const float *__restrict__ da,
+                                                                   const int32_t *__restrict__ bsum,
+                                                                   float *__restrict__ y,
+                                                                   int32_t *__restrict__ s_out, int *status) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int L = g.L, C = g.C, Q = g.Q;
+    uint4 *qv = reinterpret_cast<uint4 *>(smem);  // [16 words][L blocks]
+    float *das = reinterpret_cast<float *>(smem + L * QK);
+    int *bss = reinterpret_cast<int *>(smem + L * QK + 4 * L);
+    uint8_t *wbase = smem + fx_act_bytes(L) + warp * fx_warp_bytes(g);
+    const int slot = C * BLOCK_BYTES;
+    uint8_t *slots = wbase;
+    float *tb = reinterpret_cast<float *>(wbase + FX_SLOTS * slot);  // [4 rows][C]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(wbase + FX_SLOTS * slot + 4 * ROWS * C);
+    if (lane == 0)
+        for (int i = 0; i < FX_SLOTS; ++i) mbar_init(&bars[i], 1);
+    fence_barrier_init();
+
+    const int64_t groups = g.n / ROWS;
+    const int64_t NW = static_cast<int64_t>(gridDim.x) * FX_WARPS;
+    const int64_t first = static_cast<int64_t>(blockIdx.x) * FX_WARPS + warp;
+    const int64_t units = first < groups ? (groups - first + NW - 1) / NW * Q : 0;
+    const uint64_t policy = l2_policy_evict_first();
+    auto chunk_blocks = [&](int qi) { return qi == Q - 1 ? L - qi * C : C; };
+    int64_t rg_n = first;  // the next chunk to copy
+    int qi_n = 0;
+    auto issue_next = [&](int s) {
+        if (lane == 0) {
+            const uint32_t bytes = static_cast<uint32_t>(chunk_blocks(qi_n) * BLOCK_BYTES);
+            mbar_arrive_expect_tx(&bars[s], bytes);
+            bulk_g2s_hint(slots + s * slot, blocks + (rg_n * L + static_cast<int64_t>(qi_n) * C) * BLOCK_BYTES,
+                          bytes, &bars[s], policy);
+        }
+        if (++qi_n == Q) {
+            qi_n = 0;
+            rg_n += NW;
+        }
+    };
+    if (units > 0) issue_next(0);
+    if (units > 1) issue_next(1);
+    for (int idx = threadIdx.x; idx < 16 * L; idx += blockDim.x) {
+        const int b = idx % L, wd = idx / L;
+        qv[idx] = __ldg(reinterpret_cast<const uint4 *>(q + b * QK + 16 * wd));
+    }
+    for (int i = threadIdx.x; i < L; i += blockDim.x) {
+        das[i] = __ldg(da + i);
+        bss[i] = __ldg(bsum + i);
+    }
+    __syncthreads();
+
+    float acc = 0.0f;  // lanes 0..3: the running sum of row `lane` of the current group
+    int s = 0, ph = 0;
+    int64_t rg = first;
+    int qi = 0;
+    for (int64_t u = 0; u < units; ++u) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&bars[s], static_cast<uint32_t>(ph)))) {
+            if (lane == 0) report(status, TQFX4_ETIMEOUT, K_GEMV, static_cast<int>(u));
+            break;
+        }
+        if (u + 2 < units) {  // the slot of the previous chunk takes the chunk two ahead
+            fence_proxy_async_smem();
+            issue_next(s == 0 ? FX_SLOTS - 1 : s - 1);
+        }
+        const int cb = chunk_blocks(qi);
+        const uint8_t *tp = slots + s * slot;
+        auto pair = [&](int r, int bl) {
+            const int b = qi * C + bl;
+            const uint8_t *blk = tp + bl * BLOCK_BYTES;
+            const int S = fx_row_dot(reinterpret_cast<const uint2 *>(blk + CODE_OFS + 128 * r), qv + b, L, bss[b]);
+            const float sc = __fmul_rn(block_scale(blk, r), das[b]);
+            tb[r * C + bl] = __fmul_rn(static_cast<float>(S), sc);
+            if (kSums) s_out[(rg * ROWS + r) * L + b] = S;
+        };
+        if (cb == FX_CHUNK) {
+            pair(lane >> 3, lane & 7);
+        } else {
+            for (int p = lane; p < ROWS * cb; p += 32) {
+                const int r = p / cb;
+                pair(r, p - r * cb);
+            }
+        }
+        __syncwarp();
+        if (lane < ROWS) {
+            if (qi == 0) acc = 0.0f;
+            for (int bl = 0; bl < cb; ++bl) acc = __fadd_rn(acc, tb[lane * C + bl]);
+            if (qi == Q - 1) y[rg * ROWS + lane] = acc;
+        }
+        __syncwarp();
+        if (++qi == Q) {
+            qi = 0;
+            rg += NW;
+        }
+        if (++s == FX_SLOTS) {
+            s = 0;
+            ph ^= 1;
+        }
+    }
 }
 
 __global__ void zero_kernel(float *y, int64_t n) {
@@ -131,6 +279,34 @@ cudaError_t launch_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
     if (n == 0) return cudaSuccess;
     if (k == 0) {
         zero_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(y, n);
+        return cudaGetLastError();
+    }
+    if (k % 512 == 0) {  // the chunked pass (row groups start 16-byte aligned)
+        FxGeo f{};
+        f.n = n;
+        f.L = static_cast<int>(k / QK);
+        f.C = f.L < FX_CHUNK ? f.L : FX_CHUNK;
+        f.Q = (f.L + f.C - 1) / f.C;
+        const int smem = fx_act_bytes(f.L) + FX_WARPS * fx_warp_bytes(f);
+        static unsigned char set[2][64];
+        const bool sums = block_sums != nullptr;
+        const void *fn = sums ? reinterpret_cast<const void *>(gemv_chunk_kernel<true>)
+                              : reinterpret_cast<const void *>(gemv_chunk_kernel<false>);
+        cudaError_t e = allow_max_smem(fn, set[sums ? 1 : 0]);
+        if (e != cudaSuccess) return e;
+        if (smem > max_smem_optin()) return cudaErrorInvalidValue;
+        const int64_t groups = n / ROWS;
+        const int64_t per_sm = max_smem_optin() / (smem + 1024);
+        int64_t grid = (groups + FX_WARPS - 1) / FX_WARPS;
+        const int64_t cap = static_cast<int64_t>(num_sms()) * (per_sm > 0 ? per_sm : 1);
+        if (grid > cap) grid = cap;
+        const uint8_t *b = static_cast<const uint8_t *>(blocks);
+        if (sums)
+            gemv_chunk_kernel<true><<<static_cast<unsigned>(grid), FX_WARPS * 32, smem, st>>>(b, f, q, da, bsum, y,
+                                                                                              block_sums, status);
+        else
+            gemv_chunk_kernel<false><<<static_cast<unsigned>(grid), FX_WARPS * 32, smem, st>>>(b, f, q, da, bsum, y,
+                                                                                               nullptr, status);
         return cudaGetLastError();
     }
     const GemvGeom g = gemv_geom(n, k);
