@@ -61,14 +61,14 @@ __global__ void __launch_bounds__(256, 1) gemv_kernel(const uint8_t *__restrict_
 // ---- the chunked pass (k a multiple of 512) ----------------------------
 //
 // A warp takes row groups (first, first + NW, ...) and streams each as
-// chunks of up to 8 blocks (4160 bytes) through a three-slot ring of bulk
-// copies, 16 warps per SM. In a full chunk lane l takes row l / 8 of block
-// l % 8: the 128 code bytes of its row (element j in the low nibble of
-// byte j, element 128 + j in the high one), with the activation laid out
-// [16-byte word][block] in shared memory so that lanes on different blocks
-// read different banks. Lanes 0..3 carry their row's sum from chunk to
+// chunks of up to 16 blocks (8320 bytes) through a three-slot ring of bulk
+// copies. In a full chunk lane l takes rows 2 (l / 16), 2 (l / 16) + 1 of
+// block l % 16: 128 code bytes a row (element j in the low nibble of byte j,
+// element 128 + j in the high one), the two rows sharing the activation
+// loads, with the activation laid out [16-byte word][block] in shared
+// memory so that lanes on different blocks read different banks. Lanes 0..3 carry their row's sum from chunk to
 // chunk; the float schedule is the one above.
-constexpr int FX_SLOTS = 3, FX_WARPS = 8, FX_CHUNK = 8;
+constexpr int FX_SLOTS = 3, FX_WARPS = 8, FX_CHUNK = 16;
 
 struct FxGeo {
     int64_t n;
@@ -80,25 +80,31 @@ __host__ __device__ inline int fx_warp_bytes(const FxGeo &g) {
     return FX_SLOTS * g.C * BLOCK_BYTES + 4 * ROWS * g.C + 32;
 }
 
-// Exact S of one row of a block: 32 code words against the activation
+// Exact S of two rows of a block (codes: the first row's 128 bytes, the
+// second row 128 bytes on): 32 code words a row against the activation
 // words w (low nibbles) and 32 + w (high nibbles, kept at 16 u and divided
-// out), S = sum u q - 4 bsum.
-__device__ __forceinline__ int fx_row_dot(const uint2 *codes, const uint4 *qv, int L, int bsum) {
-    int lo = 0, hi = 0;
+// out), S = sum u q - 4 bsum; the activation words are loaded once for both.
+__device__ __forceinline__ void fx_row2_dot(const uint2 *codes, const uint4 *qv, int L, int bsum, int &S0,
+                                            int &S1) {
+    int lo[2] = {0, 0}, hi[2] = {0, 0};
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
         const uint4 ql = qv[i * L], qh = qv[(8 + i) * L];  // activation words 4i..4i+3 and 32+4i..
-        const uint2 c0 = codes[2 * i], c1 = codes[2 * i + 1];
-        lo = dp4a_us(c0.x & 0x0f0f0f0fu, ql.x, lo);
-        lo = dp4a_us(c0.y & 0x0f0f0f0fu, ql.y, lo);
-        lo = dp4a_us(c1.x & 0x0f0f0f0fu, ql.z, lo);
-        lo = dp4a_us(c1.y & 0x0f0f0f0fu, ql.w, lo);
-        hi = dp4a_us(c0.x & 0xf0f0f0f0u, qh.x, hi);
-        hi = dp4a_us(c0.y & 0xf0f0f0f0u, qh.y, hi);
-        hi = dp4a_us(c1.x & 0xf0f0f0f0u, qh.z, hi);
-        hi = dp4a_us(c1.y & 0xf0f0f0f0u, qh.w, hi);
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+            const uint2 c0 = codes[16 * r + 2 * i], c1 = codes[16 * r + 2 * i + 1];
+            lo[r] = dp4a_us(c0.x & 0x0f0f0f0fu, ql.x, lo[r]);
+            lo[r] = dp4a_us(c0.y & 0x0f0f0f0fu, ql.y, lo[r]);
+            lo[r] = dp4a_us(c1.x & 0x0f0f0f0fu, ql.z, lo[r]);
+            lo[r] = dp4a_us(c1.y & 0x0f0f0f0fu, ql.w, lo[r]);
+            hi[r] = dp4a_us(c0.x & 0xf0f0f0f0u, qh.x, hi[r]);
+            hi[r] = dp4a_us(c0.y & 0xf0f0f0f0u, qh.y, hi[r]);
+            hi[r] = dp4a_us(c1.x & 0xf0f0f0f0u, qh.z, hi[r]);
+            hi[r] = dp4a_us(c1.y & 0xf0f0f0f0u, qh.w, hi[r]);
+        }
     }
-    return lo + (hi >> 4) - 4 * bsum;
+    S0 = lo[0] + (hi[0] >> 4) - 4 * bsum;
+    S1 = lo[1] + (hi[1] >> 4) - 4 * bsum;
 }
 
 template <bool kSums>
@@ -170,20 +176,26 @@ __global__ void __launch_bounds__(FX_WARPS * 32) gemv_chunk_kernel(const uint8_t
         }
         const int cb = chunk_blocks(qi);
         const uint8_t *tp = slots + s * slot;
-        auto pair = [&](int r, int bl) {
+        // rows 2 rp and 2 rp + 1 of block bl of the chunk
+        auto pair = [&](int rp, int bl) {
             const int b = qi * C + bl;
             const uint8_t *blk = tp + bl * BLOCK_BYTES;
-            const int S = fx_row_dot(reinterpret_cast<const uint2 *>(blk + CODE_OFS + 128 * r), qv + b, L, bss[b]);
-            const float sc = __fmul_rn(block_scale(blk, r), das[b]);
-            tb[r * C + bl] = __fmul_rn(static_cast<float>(S), sc);
-            if (kSums) s_out[(rg * ROWS + r) * L + b] = S;
+            int S[2];
+            fx_row2_dot(reinterpret_cast<const uint2 *>(blk + CODE_OFS + 256 * rp), qv + b, L, bss[b], S[0], S[1]);
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                const int r = 2 * rp + i;
+                const float sc = __fmul_rn(block_scale(blk, r), das[b]);
+                tb[r * C + bl] = __fmul_rn(static_cast<float>(S[i]), sc);
+                if (kSums) s_out[(rg * ROWS + r) * L + b] = S[i];
+            }
         };
         if (cb == FX_CHUNK) {
-            pair(lane >> 3, lane & 7);
+            pair(lane >> 4, lane & 15);
         } else {
-            for (int p = lane; p < ROWS * cb; p += 32) {
-                const int r = p / cb;
-                pair(r, p - r * cb);
+            for (int p = lane; p < 2 * cb; p += 32) {
+                const int rp = p / cb;
+                pair(rp, p - rp * cb);
             }
         }
         __syncwarp();
