@@ -77,25 +77,29 @@ __device__ __forceinline__ int dp4a_us(uint32_t a, uint32_t b, int c) {
     return d;
 }
 
-// sum u q over one plane of one (row, block): 16 words, each with its
-// transposed activation word group; acc[i] collects 4^i u q.
-__device__ __forceinline__ int free_plane_sum(const uint4 *pw, const uint4 *qv, int L) {
-    int acc[4] = {0, 0, 0, 0};
+// sum u q over both planes of one (row, block): 16 words a plane, each
+// with its transposed activation word group (loaded once for the two
+// planes); acc[p][i] collects 4^i u q of plane p.
+__device__ __forceinline__ void free_pair_sums(const uint4 *pw, const uint4 *qv, int L, int &U1, int &U2) {
+    int acc[2][4] = {{0, 0, 0, 0}, {0, 0, 0, 0}};
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
-        const uint4 x4 = pw[c];
-        const uint32_t xs[4] = {x4.x, x4.y, x4.z, x4.w};
+        const uint4 x4[2] = {pw[c], pw[4 + c]};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const uint4 qq = qv[(4 * c + e) * L];
-            const uint32_t x = xs[e];
-            acc[0] = dp4a_us(x & 0x03030303u, qq.x, acc[0]);
-            acc[1] = dp4a_us(x & 0x0c0c0c0cu, qq.y, acc[1]);
-            acc[2] = dp4a_us(x & 0x30303030u, qq.z, acc[2]);
-            acc[3] = dp4a_us(x & 0xc0c0c0c0u, qq.w, acc[3]);
+#pragma unroll
+            for (int p = 0; p < 2; ++p) {
+                const uint32_t x = e == 0 ? x4[p].x : e == 1 ? x4[p].y : e == 2 ? x4[p].z : x4[p].w;
+                acc[p][0] = dp4a_us(x & 0x03030303u, qq.x, acc[p][0]);
+                acc[p][1] = dp4a_us(x & 0x0c0c0c0cu, qq.y, acc[p][1]);
+                acc[p][2] = dp4a_us(x & 0x30303030u, qq.z, acc[p][2]);
+                acc[p][3] = dp4a_us(x & 0xc0c0c0c0u, qq.w, acc[p][3]);
+            }
         }
     }
-    return acc[0] + (acc[1] >> 2) + (acc[2] >> 4) + (acc[3] >> 6);
+    U1 = acc[0][0] + (acc[0][1] >> 2) + (acc[0][2] >> 4) + (acc[0][3] >> 6);
+    U2 = acc[1][0] + (acc[1][1] >> 2) + (acc[1][2] >> 4) + (acc[1][3] >> 6);
 }
 
 __device__ __forceinline__ bool free_wait(uint64_t *bar, uint32_t parity) {
@@ -203,8 +207,9 @@ __global__ void __launch_bounds__(FR_WARPS * 32) gemv_free_kernel(const uint8_t 
             const int b = qi * C + bl;
             const uint8_t *blk = tp + bl * FR_BLOCK;
             const uint4 *pl = reinterpret_cast<const uint4 *>(blk + FR_PLANE_OFS + FR_ROW * r);
-            const int S1 = free_plane_sum(pl, qv + b, L) - bss[b];
-            const int S2 = free_plane_sum(pl + 4, qv + b, L) - bss[b];
+            int U1, U2;
+            free_pair_sums(pl, qv + b, L, U1, U2);
+            const int S1 = U1 - bss[b], S2 = U2 - bss[b];
             const float a1 = __half2float(reinterpret_cast<const __half *>(blk)[r]);
             const float a2 = __half2float(reinterpret_cast<const __half *>(blk + 8)[r]);
             const float p1 = __fmul_rn(static_cast<float>(S1), __fmul_rn(a1, das[b]));
