@@ -14,7 +14,7 @@ same number divided by the bytes per token, reported beside it.
 
     python bench.py [--steps K] [--warmup W] [--gpus N] [--impl ours|reference]
                     [--workload moe_decode|grouped_decode_64|prefill_2048|tiered_decode|mxfp4_gemv|
-                                moe_decode_mxfp4|free_gemv]
+                                moe_decode_mxfp4|free_gemv|pack_tied]
 
 The K timed steps are captured once into a CUDA graph and replayed inside
 the timed region (no host launch work in it); the other workloads time
@@ -673,6 +673,131 @@ def run_gemv(args, rank, world, local):
         dist.destroy_process_group()
 
 
+PACK_MATS = 8  # distinct 2048 x 4096 fp32 expert matrices cycled (268 MB, larger than L2)
+
+
+def run_pack(args, rank, world, local):
+    """The tied alternating solver (Sec. 2.1) as a pack source: one step packs
+    one 2048 x 4096 fp32 expert projection (Student-t(5) x 0.02) into
+    tq2_0_fx4 blocks through tqfx4_pack(TQFX4_SRC_F32_TIED); eight matrices
+    are cycled. Round-to-nearest packing of the same matrices is timed
+    beside it. Metric: expert matrices packed per second."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_08910_gb300 import binding as B
+    from paper_2608_08910_gb300 import inputs, ops
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    assert args.warmup >= 3, "at least 3 warm-up steps"
+    dev = torch.device("cuda", local)
+    n, k = I, H  # a gate projection: 2048 x 4096
+    W = [inputs.expert_matrix(SEED, e, inputs.PROJ_GATE, H, I, dev) for e in range(PACK_MATS)]
+    ws = ops.workspace(B.TQFX4_STATUS_BYTES, dev)
+    out = ops.empty_blocks(n, k, dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i, src=B.TQFX4_SRC_F32_TIED, st=stream):
+        B.tqfx4_pack(src, W[i % PACK_MATS], None, None, n, k, out, ws, st)
+
+    def graph_of(src):
+        for i in range(args.warmup):
+            step(i, src)
+        torch.cuda.synchronize()
+        B.tqfx4_check(ws)
+        cap = torch.cuda.Stream(dev)
+        cap.wait_stream(stream)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(cap):
+            with torch.cuda.graph(g, stream=cap):
+                for i in range(args.steps):
+                    step(i, src, st=cap)
+        stream.wait_stream(cap)
+        g.replay()
+        torch.cuda.synchronize()
+        return g
+
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(g):
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        g.replay()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        return max_over_ranks(ev0.elapsed_time(ev1) / 1e3, world, dev)
+
+    g_tied = graph_of(B.TQFX4_SRC_F32_TIED)
+    with ClockSampler(local) as clk:
+        t = timed(g_tied)
+    B.tqfx4_check(ws)
+    t_rtn = timed(graph_of(B.TQFX4_SRC_F32_RTN))
+    B.tqfx4_check(ws)
+
+    # end to end: each matrix from pinned host memory, its blocks back to it
+    Wh = [w.cpu().pin_memory() for w in W]
+    win = torch.empty((n, k), device=dev)
+    outh = torch.empty(out.numel(), dtype=torch.uint8, pin_memory=True)
+    for i in range(3):
+        win.copy_(Wh[i % PACK_MATS], non_blocking=True)
+        B.tqfx4_pack(B.TQFX4_SRC_F32_TIED, win, None, None, n, k, out, ws, stream)
+        outh.copy_(out, non_blocking=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for i in range(args.steps):
+        win.copy_(Wh[i % PACK_MATS], non_blocking=True)
+        B.tqfx4_pack(B.TQFX4_SRC_F32_TIED, win, None, None, n, k, out, ws, stream)
+        outh.copy_(out, non_blocking=True)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
+    te = max_over_ranks(ev0.elapsed_time(ev1) / 1e3, world, dev)
+
+    peak, peak_kind = _peaks()
+    moved = n * k * 4 + out.numel()  # fp32 in, blocks out
+    achieved = moved * args.steps / t / 1e9
+    line = {
+        "metric": "expert matrices packed per second (tied solver, 2048 x 4096)",
+        "value": job_rate(args.steps, world, t), "unit": "matrices/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "pack_tied", "n": n, "k": k, "matrices_cycled": PACK_MATS,
+                   "l2": "inputs larger than L2 (%d MB of fp32 matrices cycled)" % (PACK_MATS * n * k * 4 >> 20)},
+        "rtn_same_shape": {"ms_per_step": t_rtn / args.steps * 1e3, "matrices_per_s": args.steps / t_rtn},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": None, "kernel": "pack_kernel (tied source)", "peak_source": peak_kind,
+                     "note": "fp32 in + blocks out per launch over its time; the solver (an average of 12.8 "
+                             "scale updates a block) is arithmetic-bound, so HBM stays mostly idle"},
+        "e2e": {"value": job_rate(args.steps, world, te), "unit": "matrices/s", "h2d_bytes_per_step": n * k * 4,
+                "d2h_bytes_per_step": out.numel()},
+        "gpu_launches": args.steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        rows = 32
+        sub = W[0][:rows].cpu().numpy()
+        done, el = 0, 0.0
+        while el < 10.0:
+            t0 = time.perf_counter()
+            oracle.pack_tied(sub)
+            el += time.perf_counter() - t0
+            done += 1
+        line["cpu_baseline"] = {"value": done * rows / n / el, "unit": "matrices/s", "cores": 1, "kind": "oracle",
+                                "sample": "%d tied packs of the first %d rows, scaled to whole matrices"
+                                          % (done, rows)}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 
 def main():
     ap = argparse.ArgumentParser()
@@ -687,11 +812,12 @@ def main():
                     help="tokens per step of the grouped workloads (default: 64 or 2048; profiling only)")
     ap.add_argument("--workload", default="moe_decode",
                     choices=["moe_decode", "grouped_decode_64", "prefill_2048", "tiered_decode", "mxfp4_gemv",
-                             "moe_decode_mxfp4", "free_gemv"],
+                             "moe_decode_mxfp4", "free_gemv", "pack_tied"],
                     help="moe_decode (default): 1 token; grouped_decode_64: 64 tokens with Zipf(1.1) "
                          "routing; prefill_2048: 2048 tokens; tiered_decode: 1 token with the experts in "
                          "host memory; mxfp4_gemv / free_gemv: one GEMV over MXFP4 / free-scale two-plane blocks; "
-                         "moe_decode_mxfp4: moe_decode with MXFP4 experts")
+                         "moe_decode_mxfp4: moe_decode with MXFP4 experts; pack_tied: the tied solver packing expert "
+                         "matrices")
     ap.add_argument("--slots", type=int, default=TOPK, help="device expert slots of tiered_decode")
     args = ap.parse_args()
     globals()["E"] = args.experts
@@ -708,6 +834,9 @@ def main():
         return
     if args.workload in ("mxfp4_gemv", "free_gemv"):
         run_gemv(args, rank, world, local)
+        return
+    if args.workload == "pack_tied":
+        run_pack(args, rank, world, local)
         return
     if args.workload not in ("moe_decode", "moe_decode_mxfp4"):
         run_grouped(args, rank, world, local)
