@@ -186,6 +186,43 @@ def cpu_baseline(seconds_budget=20.0, tokens=None, layer=None):
     return per_token * done / total_t / 1e9, done, total_t
 
 
+def cpu_baseline_all_cores(tokens_per_core=2):
+    """The same oracle on all host cores: one Python thread per core, each
+    running whole tokens through the MoE layer (the oracle's C calls release
+    the interpreter lock, so the threads run in parallel). The experts of
+    the sampled tokens are packed first, outside the timed region. Returns
+    (GB/s, tokens, seconds, threads)."""
+    import concurrent.futures
+
+    import torch
+
+    import oracle
+    from paper_2608_08910_gb300 import inputs
+
+    cores = os.cpu_count() or 1
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    Wr = inputs.router_weight(SEED, E, H, dev).cpu().numpy()
+    X = inputs.hidden_states(SEED, POOL, H, dev).cpu().numpy()
+    n_tok = min(POOL, cores * tokens_per_core)
+    per_token, _, _ = bytes_per_token()
+    ex = {}
+    for t in range(n_tok):
+        _, idx, _ = oracle.router(Wr, None, X[t], TOPK)
+        for e in idx:
+            if int(e) not in ex:
+                ex[int(e)] = tuple(oracle.pack_rtn(inputs.expert_matrix(SEED, int(e), p, H, I, dev).cpu().numpy())
+                                   for p in (0, 1, 2))
+
+    def work(t):
+        oracle.moe_tokens(ex, E, H, I, Wr, None, TOPK, X[t])
+
+    with concurrent.futures.ThreadPoolExecutor(max_workers=cores) as pool:
+        t0 = time.perf_counter()
+        list(pool.map(work, range(n_tok)))
+        el = time.perf_counter() - t0
+    return per_token * n_tok / el / 1e9, n_tok, el, cores
+
+
 def run_reference(args, rank, world):
     """--impl reference: the CPU oracle, as it stands, on this machine's host
     cores; each step is one expert FFN of a routed token (1/8 of a token)."""
@@ -269,9 +306,13 @@ def run_grouped(args, rank, world, local):
     B.tqfx4_check(ws)
     mb = B.tqfx4_matrix_bytes(I, H)
     touched = 0
+    hits = None  # (token, slot) pairs per expert of the first batch, descending
     for X in Xs:
         layer.grouped(X, ws, path, OUT, sel, selw, stream=stream)
-        touched += int((torch.bincount(sel.flatten().long(), minlength=E) > 0).sum())
+        counts = torch.bincount(sel.flatten().long(), minlength=E)
+        touched += int((counts > 0).sum())
+        if hits is None:
+            hits = sorted(counts.tolist(), reverse=True)
     bytes_per_step = touched / n_batches * 3 * mb + E * H * 4
     # The K steps are captured once into a CUDA graph (as a serving loop
     # would run them), so the timed region holds no host launch work.
@@ -363,7 +404,10 @@ def run_grouped(args, rank, world, local):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "i8xi4-i32,f32",
         "data": "synthetic",
         "config": {"workload": args.workload, "tokens": T, "experts": E, "hidden": H, "inter": I, "top_k": TOPK,
-                   "zipf": zipf, "touched_experts_avg": touched / n_batches,
+                   "zipf": zipf, "touched_experts_avg": touched / n_batches, "seed": SEED,
+                   "expert_hits_first_batch": {"top16": hits[:16], "experts_with_1": hits.count(1),
+                                               "experts_with_2_to_4": sum(1 for h in hits if 2 <= h <= 4),
+                                               "touched": sum(1 for h in hits if h > 0)},
                    "l2": "inputs larger than L2 (3.27 GB expert pool); 4 batches cycled"},
         "effective_gbs": bytes_per_step * args.steps * world / t / 1e9,
         "roofline": roof,
@@ -904,6 +948,15 @@ def main():
     t = max_over_ranks(t, world, dev)
     tokens = args.steps * world  # tokens of the whole job
     value = job_rate(per_token * args.steps, world, t) / 1e9
+    # band: five more replays of the same K steps (outside the reported timing)
+    reps_ms = []
+    for _ in range(5):
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        graph.replay()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        reps_ms.append(ev0.elapsed_time(ev1) / args.steps)
 
     # ---- dominant kernel: CUDA events around every stage of every step, on
     # the launching stream (a second graph of the same K steps; the stage
@@ -981,11 +1034,19 @@ def main():
         # router, gate_up, down (tq2_0_fx4); router, gate_up, down, combine (MXFP4)
         "gpu_launches": (4 if mx else 3) * args.steps,
         "clocks": clk.summary(),
+        "repeats_ms_per_step": {"min": min(reps_ms), "median": statistics.median(reps_ms), "max": max(reps_ms),
+                                "spread": (max(reps_ms) - min(reps_ms)) / statistics.median(reps_ms),
+                                "n": len(reps_ms), "note": "5 more replays of the timed graph"},
     }
     if rank == 0 and not args.no_cpu_baseline:
         v, n, secs = cpu_baseline(layer=layer if mx else None)
         line["cpu_baseline"] = {"value": v, "unit": "GB/s", "cores": 1, "kind": "oracle",
                                 "sample": "%d tokens through the layer (%.1f s), expert packing excluded" % (n, secs)}
+        if world == 1 and not mx:
+            va, na, sa, ca = cpu_baseline_all_cores()
+            line["cpu_baseline_all_cores"] = {
+                "value": va, "unit": "GB/s", "cores": ca, "kind": "oracle",
+                "sample": "%d tokens on %d threads (%.1f s wall), expert packing excluded" % (na, ca, sa)}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
