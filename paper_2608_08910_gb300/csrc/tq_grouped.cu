@@ -959,6 +959,7 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
                                cudaStream_t st, void *const *events) {
     GroupedArgs a = a0;
     a.chunk = a.tc ? TC_CHUNK : GG_TOK;
+    a.small_max = a.tc ? small_groups_max(a) : 0;
     a.X = X;
     a.OUT = OUT;
     a.sel_out = sel_idx;
@@ -1006,11 +1007,13 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
     const int64_t units = static_cast<int64_t>(a.P) * a.nbi;
     if (a.tc) {
         if ((e = launch_tc_gemm(a, false, st)) != cudaSuccess) return e;
+        if (a.small_max && (e = launch_small_groups(a, false, st)) != cudaSuccess) return e;
         rec(5);
         swiglu_quant_kernel<<<static_cast<unsigned>((units * 32 + 255) / 256), 256, 0, st>>>(a);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
         rec(6);
         if ((e = launch_tc_gemm(a, true, st)) != cudaSuccess) return e;
+        if (a.small_max && (e = launch_small_groups(a, true, st)) != cudaSuccess) return e;
     } else {
         CUtensorMap mg, mu, md, mx, mh, sdx, sbx, sdh, sbh;
         if ((e = scale_map(&sdx, a.dxg, a.P, a.nbhp, true)) != cudaSuccess) return e;

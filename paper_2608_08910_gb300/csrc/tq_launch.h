@@ -56,6 +56,11 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
 cudaError_t launch_moe_grouped(const GroupedArgs &a, const float *X, float *OUT, int32_t *sel_idx, float *sel_w,
                                cudaStream_t st, void *const *events);
 cudaError_t launch_tc_gemm(const GroupedArgs &a, bool down, cudaStream_t st);
+// Largest chunk (pairs) the streaming small-group pass takes for these
+// shapes and buffers, 0 if it takes none; the pass itself, run after the
+// tensor-core pass of the same projection.
+int small_groups_max(const GroupedArgs &a);
+cudaError_t launch_small_groups(const GroupedArgs &a, bool down, cudaStream_t st);
 int grouped_stage_count();
 const char *grouped_stage_name(int s);
 int down_smem(const MoeArgs &a);

@@ -181,6 +181,8 @@ struct GroupedArgs {
     int tc;               // contraction on tcgen05 tensor cores
     int chunk;            // pairs per chunk of the work list (GG_TOK, or TC_CHUNK on tensor cores)
     int max_chunks;       // capacity of the work list
+    int small_max;        // chunks of at most this many pairs take the streaming
+                          // small-group pass instead of the tensor cores (0: none)
     uint8_t *xq, *hq;     // [2][P][H], [2][P][I]: e4m3 planes 16 h and l of q = 16 h + l (tensor-core path)
     uint8_t *xqt;         // [2][T][H]: the planes of the tokens' x, in token order (tensor-core path)
     int *pair_chunk;      // [P] chunk of each pair (tensor-core path)

@@ -385,6 +385,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         const int e = __ldcg(a.chunk_expert + chunk);
         const int pb = __ldcg(a.chunk_begin + chunk);
         const int m = __ldcg(a.chunk_len + chunk);
+        if (m <= a.small_max) continue;  // the small-group pass's chunk (every role skips it alike)
         const int n_rg = J.N / 4;
         const int rg0 = static_cast<int>(tl) * TC_RG;
         const int nb = J.nb;
