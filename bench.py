@@ -413,9 +413,10 @@ def run_grouped(args, rank, world, local):
         "roofline": roof,
         "e2e": {"value": tokens / te, "unit": "tokens/s", "h2d_bytes_per_step": T * H * 4,
                 "d2h_bytes_per_step": T * H * 4 + T * TOPK * 4},
-        # router (screening GEMM, norms and refinement from 256 tokens, else one kernel), top-k, group,
-        # quantize, gather, gate/up, SwiGLU, down, combine
-        "gpu_launches": ((3 if T >= 256 else 1) + 8) * args.steps,
+        # router (norms, screening GEMM and refinement from 256 tokens, else one kernel), top-k, group,
+        # quantize, activation planes, gather, gate/up (tensor cores, then the small-group pass), SwiGLU,
+        # down (the same two), combine
+        "gpu_launches": ((3 if T >= 256 else 1) + 11) * args.steps,
         "clocks": clk.summary(),
     }
     if rank == 0:
