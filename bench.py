@@ -386,7 +386,8 @@ def run_grouped(args, rank, world, local):
         peak_tc, tc_kind = _tensor_peak()
         achieved = flops_gu / stage_s["gate_up"] / 1e12
         roof = {"bound": "tensor", "achieved": achieved, "peak": peak_tc, "unit": "TFLOP/s",
-                "frac": achieved / peak_tc, "kernel": "tc_gemm_kernel (gate_up)",
+                "frac": achieved / peak_tc,
+                "kernel": "gate_up stage: tc_gemm_kernel, then small_groups_kernel (chunks of <= 4 pairs, if any)",
                 "traffic": TC_GATE_UP_TRAFFIC if (T == 2048 and E == 256) else None,
                 "traffic_source": "ncu capture at 64 experts / 512 tokens, scaled x4",
                 "peak_source": tc_kind}
@@ -394,7 +395,8 @@ def run_grouped(args, rank, world, local):
         gu_bytes = touched / n_batches * 2 * mb
         achieved = gu_bytes / stage_s["gate_up"] / 1e9
         roof = {"bound": "hbm", "achieved": achieved, "peak": peak_hbm, "unit": "GB/s",
-                "frac": achieved / peak_hbm, "traffic": None, "kernel": "tc_gemm_kernel (gate_up)",
+                "frac": achieved / peak_hbm, "traffic": None,
+                "kernel": "gate_up stage: tc_gemm_kernel (chunks of > 4 pairs), then small_groups_kernel",
                 "peak_source": peak_kind}
     roof["stage_us"] = {k: v * 1e6 for k, v in stage_s.items()}
     line = {
