@@ -190,7 +190,7 @@ __global__ void __launch_bounds__(SG_WARPS * 32) small_groups_kernel(GroupedArgs
         for (int k = 0; k < my; ++k) {
             if (!__all_sync(0xffffffffu, mbar_wait(&bars[s], static_cast<uint32_t>(ph)))) {
                 if (lane == 0) {
-                    report(a.status, TQFX4_ETIMEOUT, K_GDOWN, c);
+                    report(a.status, TQFX4_ETIMEOUT, J.down ? K_GDOWN : K_GGATEUP, c);
                     abort_all = 1;
                 }
                 // the later copies of the range may still be in flight: wait for them (bounded) before leaving
