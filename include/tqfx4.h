@@ -93,7 +93,9 @@ typedef enum tqfx4_status {
 /* Paths for tqfx4_moe_grouped. */
 #define TQFX4_PATH_AUTO 0    /* the library's choice: PREFILL (measured faster at every batch size) */
 #define TQFX4_PATH_DECODE 1  /* per-expert grouped GEMM on integer MMA (weights read once) */
-#define TQFX4_PATH_PREFILL 2 /* per-expert grouped GEMM on tensor cores (tcgen05) */
+#define TQFX4_PATH_PREFILL 2 /* per-expert grouped GEMM on tensor cores (tcgen05); chunks of at most
+                                4 pairs stream through an integer (dp4a) pass instead; results
+                                are the same bit for bit on every path */
 
 /* Bytes of one N x K matrix: (N/4) * (K/256) * 520 (Sec. 2.2: 4.0625
  * bits/weight). Returns -1 if N % 4 or K % 256 or a size is negative. */
