@@ -7,8 +7,10 @@
 // fixed float schedule y = y + float(S) * (d * da) over the blocks in order,
 // so the outputs are the oracle's bit for bit, as on the other paths.
 //
-// Work: each CTA first lists the small chunks (so that the items spread
-// evenly over the CTAs), then takes items (chunk, matrix, range of units);
+// Work: each CTA first lists the small chunks in ascending chunk order (the
+// same list in every CTA, so that item numbers name the same work
+// everywhere and the items spread evenly over the CTAs), then takes items
+// (chunk, matrix, range of units);
 // a unit is 16 blocks (8320 bytes, 16 / L whole row groups for L = k / 256
 // blocks a row, L dividing 16). A CTA's warps issue their first copies of
 // the range, then stage the chunk's activations ([16-byte word][block] per
@@ -111,14 +113,22 @@ __global__ void __launch_bounds__(SG_WARPS * 32) small_groups_kernel(GroupedArgs
         for (int i = 0; i < SG_SLOTS; ++i) mbar_init(&bars[i], 1);
     fence_barrier_init();
     __syncthreads();
-    // the chunks this pass takes, in any order (each writes its own outputs)
+    // the chunks this pass takes, in ascending chunk order: every CTA must
+    // build the same list, since item w means the same (chunk, matrix,
+    // range) to all of them (warp 0 compacts 32 chunks at a time)
     const int n_chunks = __ldcg(a.n_chunks);
-    for (int c = threadIdx.x; c < n_chunks; c += blockDim.x) {
-        const int m = __ldcg(a.chunk_len + c);
-        if (m > 0 && m <= SG_MAX) {
-            const int i = atomicAdd(&n_small, 1);
-            if (i < SG_LIST) list[i] = c;
+    if (warp == 0) {
+        int base = 0;
+        for (int c0 = 0; c0 < n_chunks; c0 += 32) {
+            const int c = c0 + lane;
+            const int m = c < n_chunks ? __ldcg(a.chunk_len + c) : 0;
+            const bool small = m > 0 && m <= SG_MAX;
+            const uint32_t bal = __ballot_sync(0xffffffffu, small);
+            const int i = base + __popc(bal & ((1u << lane) - 1u));
+            if (small && i < SG_LIST) list[i] = c;
+            base += __popc(bal);
         }
+        if (lane == 0) n_small = base;
     }
     __syncthreads();
     const int ns = min(n_small, SG_LIST);

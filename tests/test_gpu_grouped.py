@@ -1,7 +1,9 @@
 """GPU parity of tqfx4_moe_grouped (T tokens grouped by expert: batched
-decode and prefill) against the CPU oracle, through the C ABI, on both
-contractions: the decode path (legacy integer MMA) and the prefill path
-(tcgen05 tensor cores on exact bf16 operands).
+decode and prefill) against the CPU oracle, through the C ABI, on every
+contraction: the decode path (legacy integer MMA), the prefill path (tcgen05
+tensor cores on exact e4m3 encodings of the codes and of the two activation
+planes; chunks of at most 4 pairs stream through the integer small-group
+pass) and the automatic choice (the prefill path).
 
 Per call: the routing of every token (bit-exact up to accepted near-ties),
 the grouping (counts, offsets and the stable expert-then-token order,
@@ -31,7 +33,12 @@ def run_grouped(layer, X, path=0):
     return ws, OUT.cpu().numpy(), sel.cpu().numpy(), selw.cpu().numpy()
 
 
-def check_grouped(layer, seed, X, sample, path=0, check_stages=True):
+def check_grouped(layer, seed, X, sample, path=0, check_stages=True, stage_tokens=None):
+    """Checks the call's routing and grouping for every token, the combined
+    output of the `sample` tokens against the oracle, and, for the
+    `stage_tokens` (default: the sample, if check_stages), every pair's g,
+    u, quantized h and expert output bit for bit. Returns (OUT, sel, selw,
+    near-tie count, the stage-checked (token, expert) pairs)."""
     H, I, E, k = layer.hidden, layer.inter, layer.n_experts, layer.top_k
     T = X.shape[0]
     P = T * k
@@ -55,24 +62,37 @@ def check_grouped(layer, seed, X, sample, path=0, check_stages=True):
     assert np.array_equal(g("pair_slot", torch.int32, (P,)), ps)
     pair_of = g("pair_of", torch.int32, (T, k))
     assert np.array_equal(pt[pair_of], np.repeat(np.arange(T), k).reshape(T, k))
-    if check_stages:
+    if stage_tokens is None:
+        stage_tokens = sample if check_stages else []
+    elif callable(stage_tokens):
+        stage_tokens = stage_tokens(sel)
+    if len(stage_tokens):
         gv, uv = g("g", torch.float32, (P, I)), g("u", torch.float32, (P, I))
         qh, ov = g("qh", torch.int8, (P, I)), g("o", torch.float32, (P, H))
-    for t in sample:
+    checked = []
+    hits = np.bincount(sel.ravel(), minlength=E)
+    for t in sorted(set(sample) | set(stage_tokens)):
         ex = oracle_experts(seed, sel[t], H, I)
-        ref, ridx, _ = oracle.moe_tokens(ex, E, H, I, Wr, bias, k, Xn[t])
-        if np.array_equal(ridx[0], sel[t]):
-            e_ = rel_err(OUT[t], ref[0])
-            assert e_ <= FP32_TOL, (t, e_)
-        if check_stages:
+        if t in stage_tokens:  # stage by stage first: a failure names the stage and the pair
             for j in range(k):
                 pos = pair_of[t, j]
-                ro, dbg = oracle.expert_ffn(*ex[int(sel[t, j])], H, I, Xn[t])
-                assert np.array_equal(gv[pos].view(np.uint32), dbg["g"].view(np.uint32))
-                assert np.array_equal(uv[pos].view(np.uint32), dbg["u"].view(np.uint32))
-                assert np.array_equal(qh[pos], dbg["qh"])
-                assert np.array_equal(ov[pos].view(np.uint32), ro.view(np.uint32))
-    return OUT, sel, selw, ties
+                e = int(sel[t, j])
+                ro, dbg = oracle.expert_ffn(*ex[e], H, I, Xn[t])
+                where = "token %d slot %d expert %d (%d pairs)" % (t, j, e, hits[e])
+                for name, got, want in (("g", gv[pos], dbg["g"]), ("u", uv[pos], dbg["u"]),
+                                        ("qh", qh[pos], dbg["qh"]), ("o", ov[pos], ro)):
+                    gb = got.view(np.uint32) if got.dtype == np.float32 else got
+                    wb = want.view(np.uint32) if want.dtype == np.float32 else want
+                    bad = np.flatnonzero(gb != wb)
+                    assert bad.size == 0, "%s: %s differs at %d of %d entries (first %s)" % (
+                        where, name, bad.size, got.size, bad[:8])
+                checked.append((t, e))
+        if t in sample:
+            ref, ridx, _ = oracle.moe_tokens(ex, E, H, I, Wr, bias, k, Xn[t])
+            if np.array_equal(ridx[0], sel[t]):
+                e_ = rel_err(OUT[t], ref[0])
+                assert e_ <= FP32_TOL, (t, e_)
+    return OUT, sel, selw, ties, checked
 
 
 @pytest.mark.parametrize("E,H,I,k,T,zipf", [
@@ -148,10 +168,34 @@ def zipf_layer():
 def test_grouped_decode_64_tokens_zipf_full_size(zipf_layer):
     # batched decode: 64 tokens, 256 experts, top-8, Zipf(1.1) router bias
     X = inputs.hidden_states(0, 64, 4096)
-    OUT, sel, selw, ties = check_grouped(zipf_layer, 0, X, sample=[0, 17, 63], path=B.TQFX4_PATH_DECODE)
+    OUT, sel, selw, ties, _ = check_grouped(zipf_layer, 0, X, sample=[0, 17, 63], path=B.TQFX4_PATH_DECODE)
     hits = np.bincount(sel.ravel(), minlength=256)
     assert hits.max() > 8 and (hits > 0).sum() < 256  # the skew is visible
 
+
+def test_grouped_decode_64_tokens_zipf_full_size_auto(zipf_layer):
+    # the batched-decode workload on the path the library chooses (AUTO):
+    # experts with at most 4 pairs go through the streaming small-group pass
+    # at K = 4096 (gate/up) and K = 2048 (down), the others through the
+    # tensor-core contraction. Every token's routing and the grouping are
+    # checked; 8 tokens' outputs against the oracle; every pair of 4 tokens
+    # stage by stage (g, u, quantized h, expert output), bit for bit.
+    X = inputs.hidden_states(0, 64, 4096)
+    sample = [0, 5, 17, 26, 31, 40, 52, 63]
+
+    def stage_tokens(sel):
+        # token 0 and the three tokens with the most pairs on experts of at
+        # most 4 pairs (the small-group pass)
+        hits = np.bincount(sel.ravel(), minlength=256)
+        n_small = (hits[sel] <= 4).sum(axis=1)
+        return sorted({0, *np.argsort(-n_small, kind="stable")[:3].tolist()})
+
+    OUT, sel, selw, ties, checked = check_grouped(zipf_layer, 0, X, sample=sample, path=B.TQFX4_PATH_AUTO,
+                                                  stage_tokens=stage_tokens)
+    hits = np.bincount(sel.ravel(), minlength=256)
+    small = [e for _, e in checked if hits[e] <= 4]
+    tensor = [e for _, e in checked if hits[e] > 4]
+    assert len(small) >= 4 and len(tensor) >= 4, (len(small), len(tensor))  # both contractions covered
 
 @pytest.fixture(scope="module")
 def prefill_layer():
@@ -159,5 +203,9 @@ def prefill_layer():
 
 
 def test_grouped_prefill_2048_tokens_full_size(prefill_layer):
+    # every token's routing and the grouping; 3 tokens' outputs, and every
+    # pair of 2 of them stage by stage, on the tensor-core contraction at
+    # K = 4096 / 2048 (about 64 pairs a chunk)
     X = inputs.hidden_states(1, 2048, 4096)
-    check_grouped(prefill_layer, 0, X, sample=[0, 1023, 2047], path=B.TQFX4_PATH_PREFILL, check_stages=False)
+    check_grouped(prefill_layer, 0, X, sample=[0, 1023, 2047], path=B.TQFX4_PATH_PREFILL,
+                  stage_tokens=[1023, 2047])
