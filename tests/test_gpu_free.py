@@ -66,10 +66,18 @@ def test_gemv_large_sampled(ws):
     B.tqfx4_check(ws)
     groups = np.unique(np.concatenate([np.arange(4), np.arange(n // 4 - 4, n // 4),
                                        np.random.default_rng(0).integers(0, n // 4, 100)]))
-    gb = B.tqfx4_free_bytes(4, k)
-    sub = blocks.view(n // 4, gb)[torch.from_numpy(groups).to(DEV)].cpu().numpy()
-    ry, _, _ = oracle.free_gemv(sub, 4 * len(groups), k, q.cpu().numpy(), da.cpu().numpy())
     rows = (groups[:, None] * 4 + np.arange(4)[None, :]).reshape(-1)
+    # the oracle packs the sampled rows itself, from the same generated planes
+    t1, t2, a1, a2 = _planes(5, n, k, DEV)
+    ri = torch.from_numpy(rows).to(DEV)
+    ref = oracle.pack_free(t1[ri].cpu().numpy(), t2[ri].cpu().numpy(), _np16(a1[ri]), _np16(a2[ri]))
+    del t1, t2
+    gb = B.tqfx4_free_bytes(4, k)
+    sub = blocks.view(n // 4, gb)[torch.from_numpy(groups).to(DEV)].cpu().numpy().reshape(-1)
+    assert np.array_equal(sub, ref)
+    rq, rda, _ = oracle.quantize_act(x.numpy())
+    assert np.array_equal(q.cpu().numpy(), rq)
+    ry, _, _ = oracle.free_gemv(ref, 4 * len(groups), k, rq, rda)
     assert np.array_equal(y.cpu().numpy()[rows].view(np.uint32), ry.view(np.uint32))
 
 

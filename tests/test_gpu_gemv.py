@@ -163,3 +163,50 @@ def test_host_side_argument_errors(ws):
         with pytest.raises(B.TqfxError) as e:
             fn()
         assert e.value.status == status
+
+
+def test_gemv_large_sampled(ws):
+    # 131072 x 4096 (272 MB of blocks, larger than L2): the chunked pass with
+    # many more row groups than warps, so each warp carries its ring across
+    # row groups. The oracle packs and multiplies sampled row groups (the
+    # first and last four and 100 random ones) from the same fp32 rows; the
+    # GPU's blocks of those row groups and their outputs must be bit-exact.
+    n, k = 131072, 4096
+    w = inputs.gemv_matrix(3, n, k, DEV)
+    blocks = ops.pack_rtn(w, ws)
+    x = inputs.hidden_states(4, 1, k)[0]
+    q, da, bs = ops.quantize_act(x.to(DEV), ws)
+    y = ops.gemv(blocks, n, k, q, da, bs, ws)
+    B.tqfx4_check(ws)
+    groups = np.unique(np.concatenate([np.arange(4), np.arange(n // 4 - 4, n // 4),
+                                       np.random.default_rng(1).integers(0, n // 4, 100)]))
+    rows = (groups[:, None] * 4 + np.arange(4)[None, :]).reshape(-1)
+    w_rows = w[torch.from_numpy(rows).to(DEV)].cpu().numpy()
+    del w
+    ref_blocks = oracle.pack_rtn(w_rows)
+    gb = B.tqfx4_matrix_bytes(4, k)
+    got_blocks = blocks.view(n // 4, gb)[torch.from_numpy(groups).to(DEV)].cpu().numpy().reshape(-1)
+    assert np.array_equal(got_blocks, ref_blocks)
+    rq, rda, rbs = oracle.quantize_act(x.numpy())
+    assert np.array_equal(q.cpu().numpy(), rq) and np.array_equal(bs.cpu().numpy(), rbs)
+    ry, _ = oracle.gemv(ref_blocks, len(rows), k, rq, rda)
+    assert np.array_equal(y.cpu().numpy()[rows].view(np.uint32), ry.view(np.uint32))
+
+
+def test_gemv_1024_benchmark_inputs(ws):
+    # the single-GEMV workload's own inputs: N(0, 0.02) weights, seed 0,
+    # round-to-nearest codes; an N(0, 1) vector quantized per block
+    n = k = 1024
+    w = inputs.gemv_matrix(0, n, k)
+    x = inputs.hidden_states(0, 1, k)[0]
+    rb = oracle.pack_rtn(w.numpy())
+    rq, rda, _ = oracle.quantize_act(x.numpy())
+    ry, rS = oracle.gemv(rb, n, k, rq, rda)
+    blocks = ops.pack_rtn(w.to(DEV), ws)
+    q, da, bs = ops.quantize_act(x.to(DEV), ws)
+    y, S = ops.gemv(blocks, n, k, q, da, bs, ws, block_sums=True)
+    B.tqfx4_check(ws)
+    assert np.array_equal(blocks.cpu().numpy(), rb)
+    assert np.array_equal(S.cpu().numpy(), rS)
+    assert np.array_equal(y.cpu().numpy().view(np.uint32), ry.view(np.uint32))
+    assert rel_err(y.cpu().numpy(), ry) <= FP32_TOL

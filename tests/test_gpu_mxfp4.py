@@ -71,7 +71,10 @@ def test_gemv_mxfp4_uses_device_quantized_activation(ws):
     q, da, _ = ops.quantize_act(x.to(DEV), ws)
     y = ops.gemv_mxfp4(blocks.to(DEV), n, k, q, da, ws)
     B.tqfx4_check(ws)
-    ry, _ = oracle.mxfp4_gemv(blocks.numpy(), n, k, q.cpu().numpy(), da.cpu().numpy())
+    rq, rda, _ = oracle.quantize_act(x.numpy())  # the oracle quantizes its own copy
+    assert np.array_equal(q.cpu().numpy(), rq) and np.array_equal(da.cpu().numpy().view(np.uint32),
+                                                                  rda.view(np.uint32))
+    ry, _ = oracle.mxfp4_gemv(blocks.numpy(), n, k, rq, rda)
     assert np.array_equal(y.cpu().numpy().view(np.uint32), ry.view(np.uint32))
 
 

@@ -7,17 +7,21 @@ the same bytes and the same kernels, so outputs do not depend on residency
 (Sec. 2.2, property iii). Here that is checked bit for bit: the tier's
 outputs, selections and weights equal the resident tqfx4_moe_ffn's for every
 token, also when the slab holds only top_k experts and evicts.
-The resident path itself is checked against the CPU oracle in
-test_gpu_moe.py.
+The two-call decode and the tier are also checked against the CPU oracle
+directly: their outputs within 1e-4 relative of the oracle's MoE (and bit for
+bit, since the float schedules are the same), on the small layer and on the
+256-expert benchmark layer.
 """
 import numpy as np
 import pytest
 import torch
 
+import oracle
 from paper_2608_08910_gb300 import binding as B
 from paper_2608_08910_gb300 import inputs
 from paper_2608_08910_gb300.moe import MoeLayer
 from paper_2608_08910_gb300.tier import ExpertTier
+from tests.parity import FP32_TOL, oracle_experts, rel_err
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
@@ -25,6 +29,20 @@ DEV = "cuda"
 
 def _bits(t):
     return t.cpu().numpy().view(np.uint32)
+
+
+def _oracle_out(L, seed, x, sel):
+    """The oracle's MoE output for token x, if its own routing equals `sel`
+    (else None: a near-tie, accepted by the selection tests)."""
+    Wr = L.router_w.cpu().numpy()
+    bias = None if L.router_b is None else L.router_b.cpu().numpy()
+    xn = x.cpu().numpy()
+    _, ridx, _ = oracle.router(Wr, bias, xn, L.top_k)
+    if not np.array_equal(ridx, sel):
+        return None
+    ex = oracle_experts(seed, ridx, L.hidden, L.inter)
+    ref, _, _ = oracle.moe_tokens(ex, L.n_experts, L.hidden, L.inter, Wr, bias, L.top_k, xn)
+    return ref[0]
 
 
 @pytest.fixture(scope="module")
@@ -51,6 +69,11 @@ def test_route_then_experts_equals_ffn(small):
         B.tqfx4_moe_experts(L.ex, L.rt, ptrs, out, ws)
         B.tqfx4_check(ws)
         assert np.array_equal(_bits(out), _bits(ref_out))
+        if t < 2:  # against the oracle itself
+            ref = _oracle_out(L, 41, X[t], sel.cpu().numpy())
+            if ref is not None:
+                assert rel_err(out.cpu().numpy(), ref) <= FP32_TOL
+                assert np.array_equal(_bits(out), ref.view(np.uint32))
 
 
 @pytest.mark.parametrize("slots", [6, 12])
@@ -80,12 +103,20 @@ def test_tier_full_size_layer():
     ws = L.workspace(1)
     tier = ExpertTier(L, 8)
     X = inputs.hidden_states(7, 2, 4096, DEV)
+    compared = 0
     for t in range(2):
         ref_out = L.ffn(X[t], ws)[0].clone()
         out = torch.empty(4096, device=DEV)
-        tier.ffn(X[t], ws, out, torch.empty(8, dtype=torch.int32, device=DEV), torch.empty(8, device=DEV))
+        sel = torch.empty(8, dtype=torch.int32, device=DEV)
+        tier.ffn(X[t], ws, out, sel, torch.empty(8, device=DEV))
         B.tqfx4_check(ws)
         assert np.array_equal(_bits(out), _bits(ref_out))
+        ref = _oracle_out(L, 0, X[t], sel.cpu().numpy())  # the tier against the oracle
+        if ref is not None:
+            assert rel_err(out.cpu().numpy(), ref) <= FP32_TOL
+            assert np.array_equal(_bits(out), ref.view(np.uint32))
+            compared += 1
+    assert compared >= 1
 
 
 def test_experts_argument_errors(small):
