@@ -83,6 +83,7 @@ _SIGS = {
     "tqfx4_moe_route": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_experts": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_check": (_int, [_vp, _vp]),
+    "tqfx4_selftest_wait_timeout": (_int, [_vp, _sz, _vp]),
     "tqfx4_last_error": (C.c_char_p, []),
     "tqfx4_status_string": (C.c_char_p, [_int]),
 }
@@ -262,6 +263,10 @@ def tqfx4_moe_workspace_views(ex, rt, tokens, grouped, path) -> dict:
 
 def tqfx4_check(ws, stream=None):
     _check(lib().tqfx4_check(_p(ws), _s(stream)), "tqfx4_check")
+
+
+def tqfx4_selftest_wait_timeout(ws, stream=None):
+    _check(lib().tqfx4_selftest_wait_timeout(_p(ws), _nbytes(ws), _s(stream)), "tqfx4_selftest_wait_timeout")
 
 
 def tqfx4_last_error() -> str:

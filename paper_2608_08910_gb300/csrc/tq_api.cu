@@ -436,13 +436,21 @@ tqfx4_status tqfx4_check(void *ws, void *stream) {
     if (st[0] == 0) return ok();
     e = cudaMemset(ws, 0, sizeof(st));
     if (e != cudaSuccess) return cuda_fail(e, "tqfx4_check: status clear");
-    static const char *kernels[] = {"?",      "pack",   "quantize", "gemv",   "router",  "gate_up",
-                                    "down",   "topk",   "group",    "g_gateup", "g_down", "combine",
-                                    "prefill"};
-    const char *kn = (st[1] >= 0 && st[1] < 13) ? kernels[st[1]] : "?";
+    static const char *kernels[] = {"?",      "pack",   "quantize", "gemv",     "router", "gate_up", "down",
+                                    "topk",   "group",  "g_gateup", "g_down",   "combine", "prefill", "selftest"};
+    const int nk = static_cast<int>(sizeof(kernels) / sizeof(kernels[0]));
+    const char *kn = (st[1] >= 0 && st[1] < nk) ? kernels[st[1]] : "?";
     if (st[0] == TQFX4_EDATA || st[0] == TQFX4_ETIMEOUT)
         return fail(static_cast<tqfx4_status>(st[0]), "device error %d in kernel %s (unit %d)", st[0], kn, st[2]);
     return fail(TQFX4_ECUDA, "unknown device status %d in kernel %s", st[0], kn);
+}
+
+tqfx4_status tqfx4_selftest_wait_timeout(void *ws, size_t ws_bytes, void *stream) {
+    tqfx4_status s = check_ws(ws, ws_bytes, TQFX4_STATUS_BYTES, "tqfx4_selftest_wait_timeout");
+    if (s) return s;
+    cudaError_t e = tq::launch_selftest_timeout(static_cast<int *>(ws), static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "tqfx4_selftest_wait_timeout");
+    return ok();
 }
 
 const char *tqfx4_last_error(void) { return g_err; }

@@ -50,6 +50,7 @@ constexpr int QS_STRIDE = 264;    // shared-memory stride of one 256-byte activa
 enum KernelId : int {
     K_PACK = 1, K_QUANT = 2, K_GEMV = 3, K_ROUTER = 4, K_GATEUP = 5, K_DOWN = 6,
     K_TOPK = 7, K_GROUP = 8, K_GGATEUP = 9, K_GDOWN = 10, K_COMBINE = 11, K_PREFILL = 12,
+    K_SELFTEST = 13,
 };
 
 // Roughly two seconds at the GB300's 2 GHz clock: any mbarrier wait longer
@@ -105,14 +106,14 @@ __device__ __forceinline__ uint32_t mbar_try_wait(uint64_t *bar, uint32_t parity
     return ok;
 }
 
-// Waits for phase `parity` of `bar` to complete; gives up after
-// kWaitBudgetCycles and returns false.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
+// Waits for phase `parity` of `bar` to complete; gives up after `budget`
+// cycles (kWaitBudgetCycles by default) and returns false.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, long long budget = kWaitBudgetCycles) {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     while (true) {
         if (mbar_try_wait(bar, parity)) return true;
-        if (clock64() - t0 > kWaitBudgetCycles) return false;
+        if (clock64() - t0 > budget) return false;
     }
 }
 

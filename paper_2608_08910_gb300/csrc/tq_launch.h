@@ -64,5 +64,6 @@ cudaError_t launch_small_groups(const GroupedArgs &a, bool down, cudaStream_t st
 int grouped_stage_count();
 const char *grouped_stage_name(int s);
 int down_smem(const MoeArgs &a);
+cudaError_t launch_selftest_timeout(int *status, cudaStream_t st);
 
 }  // namespace tq

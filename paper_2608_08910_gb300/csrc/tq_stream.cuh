@@ -45,6 +45,7 @@ struct WarpRing {
     uint64_t *bars;
     int stages;
     int slot_bytes;
+    long long budget;  // cycles a copy may take before it is reported lost
 };
 
 __device__ __forceinline__ WarpRing carve_ring(uint8_t *wbase, int stages, int slot_bytes, int rpu, int nb) {
@@ -54,6 +55,7 @@ __device__ __forceinline__ WarpRing carve_ring(uint8_t *wbase, int stages, int s
     r.bars = reinterpret_cast<uint64_t *>(wbase + stages * slot_bytes + stream_tbuf_bytes(rpu, nb));
     r.stages = stages;
     r.slot_bytes = slot_bytes;
+    r.budget = kWaitBudgetCycles;
     return r;
 }
 
@@ -115,7 +117,7 @@ __device__ __forceinline__ bool warp_stream_run(const WarpRing &r, const MatJob 
     int slot = 0;
     uint32_t parity = 0;
     for (int64_t u = first; u < total; u += step) {
-        if (!__all_sync(0xffffffffu, mbar_wait(&r.bars[slot], parity))) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&r.bars[slot], parity, r.budget))) {
             if (lane == 0) report(status, TQFX4_ETIMEOUT, kernel_id, static_cast<int>(u));
             return false;
         }
@@ -246,7 +248,7 @@ __device__ __forceinline__ bool warp_units_run(const WarpRing &r, UnitQueue &q, 
         for (int s = 0; s < MAXST; ++s)
             if (s == slot) u = slot_u[s];
         if (u < 0) break;
-        if (!__all_sync(0xffffffffu, mbar_wait(&r.bars[slot], parity))) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&r.bars[slot], parity, r.budget))) {
             if (lane == 0) report(status, TQFX4_ETIMEOUT, kernel_id, static_cast<int>(u));
             return false;
         }
