@@ -349,16 +349,19 @@ tqfx4_status tqfx4_moe_grouped(const tqfx4_experts *ex, const tqfx4_router *rt,
  *   Inputs, outputs and their rules are those of tqfx4_moe_ffn. The scratch
  *   is a device array of TQFX4_NOALLOC_SCRATCH_BYTES (1 MiB) inside the
  *   library, which every GPU that loads the library keeps until the process
- *   exits. Shapes whose tqfx4_moe_workspace_bytes exceeds that size are
- *   rejected with TQFX4_EWORKSPACE before anything is enqueued (the
- *   256-expert, hidden 4096, intermediate 2048, top-8 layer needs about
- *   0.35 MiB). The call allocates nothing: no cudaMalloc, no cudaFree.
- *   The first call on a device looks up the scratch's device address
- *   (cudaGetSymbolAddress) with that device current; make that first call
- *   before any stream capture. Each call clears the scratch's status word
- *   and counters on `stream` before its kernels; device-side error reports
- *   therefore are not kept between calls (use tqfx4_moe_ffn with a workspace
- *   and tqfx4_check to read them).
+ *   exits. Shapes whose one-token workspace (the layout tqfx4_moe_ffn uses)
+ *   exceeds that size are rejected with TQFX4_EWORKSPACE before anything is
+ *   enqueued (the 256-expert, hidden 4096, intermediate 2048, top-8 layer
+ *   needs 361 472 bytes, about 0.35 MiB). The call allocates nothing: no
+ *   cudaMalloc, no cudaFree.
+ *   Every call looks up the scratch's device address in the current context
+ *   (cudaGetSymbolAddress; nothing is cached, so a device reset or a
+ *   non-primary context is followed). The first call on a device may load
+ *   the library's device code there: make it before any stream capture.
+ *   Each call clears the scratch's status word and counters on `stream`
+ *   before its kernels; device-side error reports therefore are not kept
+ *   between calls (use tqfx4_moe_ffn with a workspace and tqfx4_check to
+ *   read them).
  *   All calls share the one scratch array, which keeps the last call's
  *   contents: calls whose work overlaps on the GPU (different streams, or
  *   different host threads without ordering) race on it and must not be
@@ -425,6 +428,19 @@ tqfx4_status tqfx4_moe_workspace_views(const tqfx4_experts *ex, const tqfx4_rout
  * stream reports a CUDA error.
  */
 tqfx4_status tqfx4_check(void *ws, void *stream);
+
+/*
+ * tqfx4_selftest_wait_timeout -- a check of the library's failure detection
+ * that faults nothing: one warp runs the streaming engine's consume loop
+ * (the loop under the GEMV and MoE kernels) on a ring whose copies were
+ * never issued, with a wait budget of 10^6 cycles instead of the production
+ * limit of about two seconds. Its wait gives up, the warp records
+ * TQFX4_ETIMEOUT in the status word of `ws` (kernel "selftest") and the
+ * kernel returns; no copy is in flight, so the context stays usable.
+ * tqfx4_check(ws, stream) then returns TQFX4_ETIMEOUT and clears the word.
+ * ws: device, at least TQFX4_STATUS_BYTES. Not part of the paper's method.
+ */
+tqfx4_status tqfx4_selftest_wait_timeout(void *ws, size_t ws_bytes, void *stream);
 
 /* Message for the last error returned on the calling host thread. */
 const char *tqfx4_last_error(void);

@@ -13,42 +13,33 @@ namespace {
 // loads the library holds these bytes until the process exits.
 __device__ __align__(256) unsigned char g_noalloc_scratch[TQFX4_NOALLOC_SCRATCH_BYTES];
 
-// Device address of g_noalloc_scratch, looked up once per device (in host
-// code the array's name is only a stand-in, not a device address).
-constexpr int kMaxDevices = 64;
-void *g_scratch_addr[kMaxDevices];
-
 }  // namespace
 
 extern "C" tqfx4_status tqfx4_moe_ffn_noalloc(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x,
                                               float *out, int32_t *sel_idx, float *sel_w, void *stream) {
-    const size_t need = tqfx4_moe_workspace_bytes(ex, rt, 1, TQFX4_PATH_AUTO);
-    if (need == 0)
+    if (tqfx4_moe_workspace_bytes(ex, rt, 1, TQFX4_PATH_AUTO) == 0)
         return tqfx4_moe_ffn(ex, rt, x, out, sel_idx, sel_w, nullptr, 0, stream);  // reports the shape error
-    if (need > TQFX4_NOALLOC_SCRATCH_BYTES) {
+    // the bound tqfx4_moe_ffn checks: the one-token (decode) layout
+    const tq::MoeLayout L = tq::moe_layout(ex->n_experts, ex->hidden, ex->inter, rt->top_k, 1, false, true);
+    if (L.total > TQFX4_NOALLOC_SCRATCH_BYTES) {
         char msg[200];
         snprintf(msg, sizeof(msg),
                  "tqfx4_moe_ffn_noalloc: these shapes need %zu bytes of scratch; the library holds %d "
                  "(use tqfx4_moe_ffn with a caller workspace)",
-                 need, TQFX4_NOALLOC_SCRATCH_BYTES);
+                 L.total, TQFX4_NOALLOC_SCRATCH_BYTES);
         return tq::api_fail(TQFX4_EWORKSPACE, msg);
     }
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices)
-        return tq::api_fail(TQFX4_ECUDA, "tqfx4_moe_ffn_noalloc: no usable current device");
-    if (!g_scratch_addr[dev]) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess || !p)
-            return tq::api_fail(TQFX4_ECUDA, "tqfx4_moe_ffn_noalloc: cudaGetSymbolAddress failed");
-        g_scratch_addr[dev] = p;
-    }
-    void *ws = g_scratch_addr[dev];
+    // In host code g_noalloc_scratch only names a host-side stand-in; the
+    // device address is looked up in the current context on every call (no
+    // cached copy), so it stays right after a device reset, which reloads
+    // the library's device code, and under a context other than the
+    // device's primary one.
+    void *ws = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&ws, g_noalloc_scratch);
+    if (e != cudaSuccess || !ws)
+        return tq::api_fail(TQFX4_ECUDA, "tqfx4_moe_ffn_noalloc: cudaGetSymbolAddress failed");
     // The status word and the counters must start every call at zero; the
     // rest of the scratch is fully rewritten by the call.
-    const tq::MoeLayout L =
-        tq::moe_layout(ex->n_experts, ex->hidden, ex->inter, rt->top_k, 1, false, true);
     e = cudaMemsetAsync(ws, 0, L.ctr + 4 * L.n_ctr, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return tq::api_fail(TQFX4_ECUDA, "tqfx4_moe_ffn_noalloc: clearing the scratch failed");
     return tqfx4_moe_ffn(ex, rt, x, out, sel_idx, sel_w, ws, TQFX4_NOALLOC_SCRATCH_BYTES, stream);

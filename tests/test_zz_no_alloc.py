@@ -48,7 +48,7 @@ def test_noalloc_matches_workspace_entry_point_twice(E, H, I, k):
 
 
 def test_noalloc_refuses_shapes_beyond_its_scratch():
-    # hidden = inter = 16384 with 1024 experts and top-16 needs more than 1 MiB
+    # hidden = inter = 16384 with 1024 experts and top-16: its one-token workspace exceeds 1 MiB
     ex = B.c_experts(None, None, None, 1024, 16384, 16384)
     rt = B.c_router(None, None, 16)
     assert B.tqfx4_moe_workspace_bytes(ex, rt, 1, 0) > B.TQFX4_NOALLOC_SCRATCH_BYTES
