@@ -3,7 +3,7 @@ pass and routed-expert MoE kernels, behind the C ABI of libtqfx4.
 
 The public calls have the names of include/tqfx4.h and live in `binding`;
 `ops` holds tensor-allocating conveniences built on them; `inputs` holds the
-seeded synthetic input generators; `workloads` the named benchmark shapes.
+seeded synthetic input generators.
 """
 from .binding import (  # noqa: F401
     TQFX4_BLOCK_BYTES, TQFX4_PATH_AUTO, TQFX4_PATH_DECODE, TQFX4_PATH_PREFILL, TQFX4_QK, TQFX4_ROWS,

@@ -3,7 +3,8 @@
 // Data path: a matrix is one contiguous stream of 520-byte blocks, and the
 // fixed float schedule acc = acc + float(S) * (d * da) runs over the blocks
 // of a row in ascending order. For k a multiple of 512 the chunked pass
-// below streams row groups in 8-block chunks, one (row, block) per lane;
+// below streams row groups in chunks of up to 16 blocks, two rows of a
+// block per lane;
 // otherwise (rows 8-byte aligned) the grid splits the matrix into one
 // contiguous range of row groups per CTA and each warp streams units of it
 // through the engine of tq_stream.cuh.
@@ -72,7 +73,7 @@ constexpr int FX_SLOTS = 3, FX_WARPS = 8, FX_CHUNK = 16;
 
 struct FxGeo {
     int64_t n;
-    int L, C, Q;  // blocks per row group, per chunk (min(8, L)), chunks per row group
+    int L, C, Q;  // blocks per row group, per chunk (min(FX_CHUNK, L)), chunks per row group
 };
 
 __host__ __device__ inline int fx_act_bytes(int L) { return ((L * (QK + 8) + 127) / 128) * 128; }

@@ -4,7 +4,7 @@
 // that expert.
 //
 // tcgen05.mma has no integer kind on sm_103a, so the integer block sums
-// S = sum_j c_j q_j (Eq. 5) are formed with kind::f8f6f4 on e4m3 operands
+// S = sum_j c_j q_j of the dot pass (Sec. 2.2) are formed with kind::f8f6f4 on e4m3 operands
 // that hold small dyadic numbers exactly:
 //   A  the nibble u = c + 4 (0..8) as the e4m3 byte 0x0u, which is exactly
 //      u * 2^-9 (subnormals, and 0x08 = 2^-6), so unpacking a 32-bit word of
