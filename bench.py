@@ -13,8 +13,8 @@ router weights) per token / time per token; tokens/s per MoE layer is the
 same number divided by the bytes per token, reported beside it.
 
     python bench.py [--steps K] [--warmup W] [--gpus N] [--impl ours|reference]
-                    [--workload moe_decode|grouped_decode_64|prefill_2048|tiered_decode|mxfp4_gemv|
-                                moe_decode_mxfp4|free_gemv|pack_tied]
+                    [--workload moe_decode|gemv_1024|expert_ffn|grouped_decode_64|prefill_2048|
+                                tiered_decode|mxfp4_gemv|moe_decode_mxfp4|free_gemv|pack_tied]
 
 The K timed steps are captured once into a CUDA graph and replayed inside
 the timed region (no host launch work in it); the other workloads time
@@ -720,6 +720,252 @@ def run_gemv(args, rank, world, local):
         dist.destroy_process_group()
 
 
+SMALL_POOL_BYTES = 256 << 20  # distinct weight bytes rotated through the steps of gemv_1024 / expert_ffn
+
+
+def run_small(args, rank, world, local):
+    """The two single-matrix workloads, each on a pool of distinct weights
+    larger than L2 (at least 256 MB), one pool entry per step, a new
+    activation every step:
+    gemv_1024: one 1024 x 1024 tq2_0_fx4 GEMV (round-to-nearest codes of
+      N(0, 0.02) weights) of an N(0, 1) vector: tqfx4_quantize_act, then
+      tqfx4_gemv; 512 matrices (273 MB) rotated.
+    expert_ffn: one SwiGLU expert, gate/up 4096 -> 2048, down 2048 -> 4096,
+      Student-t(5) x 0.02 weights: tqfx4_moe_ffn on a one-expert layer (its
+      router is a single 4096-element logit, its weight 1); 21 such experts
+      (268 MB) rotated.
+    Metric: effective GB/s of the matrices' blocks over the step time. The
+    same steps on one resident matrix (hot L2) are reported beside it."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_08910_gb300 import binding as B
+    from paper_2608_08910_gb300 import inputs, ops
+    from paper_2608_08910_gb300.moe import MoeLayer
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    assert args.warmup >= 3, "at least 3 warm-up steps"
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    gemv = args.workload == "gemv_1024"
+    xpool = 64
+    if gemv:
+        n = k = 1024
+        mat = B.tqfx4_matrix_bytes(n, k)
+        M = (SMALL_POOL_BYTES + mat - 1) // mat
+        ws = ops.workspace(B.TQFX4_STATUS_BYTES, dev)
+        # M matrices stacked as one (M n) x k matrix: matrix i is row groups [i n/4, (i+1) n/4)
+        pool = ops.pack_rtn(inputs.gemv_matrix(SEED, M * n, k, dev), ws)
+        torch.cuda.empty_cache()
+        X = inputs.hidden_states(SEED + rank, xpool, k, dev)
+        q = torch.empty(k, dtype=torch.int8, device=dev)
+        da = torch.empty(k // 256, device=dev)
+        bs = torch.empty(k // 256, dtype=torch.int32, device=dev)
+        y = torch.empty(n, device=dev)
+        step_bytes = mat
+
+        def step(i, st=stream, hot=False, ev=None, x=None):
+            if ev:
+                ev[0].record(st)
+            B.tqfx4_quantize_act(X[i % xpool] if x is None else x, 1, k, q, da, bs, ws, st)
+            if ev:
+                ev[1].record(st)
+            m = 0 if hot else i % M
+            B.tqfx4_gemv(pool[m * mat:(m + 1) * mat], n, k, q, da, bs, y, None, ws, st)
+            if ev:
+                ev[2].record(st)
+        launches = 2
+        kern = "gemv_chunk_kernel"
+        cfg = {"workload": "gemv_1024x1024", "n": n, "k": k, "matrix_bytes": mat, "pool_matrices": M,
+               "l2": "inputs larger than L2: %d distinct matrices (%d MB) rotated, a new activation per step"
+                     % (M, M * mat >> 20)}
+    else:
+        Hh, Ii = H, I
+        mat = 2 * B.tqfx4_matrix_bytes(Ii, Hh) + B.tqfx4_matrix_bytes(Hh, Ii)
+        M = (SMALL_POOL_BYTES + mat - 1) // mat
+        layers = [MoeLayer.synthetic(SEED + m, 1, Hh, Ii, 1, 0.0, dev) for m in range(M)]
+        torch.cuda.empty_cache()
+        ws = layers[0].workspace(1)
+        X = inputs.hidden_states(SEED + rank, xpool, Hh, dev)
+        out = torch.empty(Hh, device=dev)
+        sel = torch.empty(1, dtype=torch.int32, device=dev)
+        selw = torch.empty(1, device=dev)
+        step_bytes = mat
+        n_st = B.tqfx4_moe_stage_count(0, 0)
+
+        def step(i, st=stream, hot=False, ev=None, x=None):
+            L = layers[0 if hot else i % M]
+            L.ffn(X[i % xpool] if x is None else x, ws, out, sel, selw, stream=st, events=ev)
+        launches = n_st
+        kern = "gate_up"
+        cfg = {"workload": "expert_ffn_h4096_i2048", "hidden": Hh, "inter": Ii, "expert_bytes": mat,
+               "pool_experts": M, "router": "one expert (a single 4096-element logit, weight 1)",
+               "l2": "inputs larger than L2: %d distinct experts (%d MB) rotated, a new activation per step"
+                     % (M, M * mat >> 20)}
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
+
+    def graph_of(hot):
+        cap = torch.cuda.Stream(dev)
+        cap.wait_stream(stream)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(cap):
+            with torch.cuda.graph(g, stream=cap):
+                for i in range(args.steps):
+                    step(args.warmup + i, st=cap, hot=hot)
+        stream.wait_stream(cap)
+        g.replay()  # untimed
+        torch.cuda.synchronize()
+        return g
+
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(g):
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        g.replay()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        return max_over_ranks(ev0.elapsed_time(ev1) / 1e3, world, dev)
+
+    g_cold = graph_of(False)
+    with ClockSampler(local) as clk:
+        t = timed(g_cold)
+    B.tqfx4_check(ws)
+    reps = [timed(g_cold) for _ in range(3)]
+    t_hot = timed(graph_of(True))
+    B.tqfx4_check(ws)
+
+    # the dominant kernel's duration: CUDA events around each stage of every
+    # step, on the launching stream, in plain stream order (the library's
+    # traced call records its own stage events; the GEMV steps are not
+    # captured, since an event recorded by torch inside a capture does not time)
+    n_ev = 3 if gemv else launches + 1
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_ev)] for _ in range(args.steps)]
+    for row in evs:
+        for e_ in row:
+            e_.record(stream)
+    torch.cuda.synchronize()
+    if gemv:
+        for i in range(args.steps):
+            step(args.warmup + i, ev=evs[i])
+    else:
+        cap = torch.cuda.Stream(dev)
+        cap.wait_stream(stream)
+        g_ev = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(cap):
+            with torch.cuda.graph(g_ev, stream=cap):
+                for i in range(args.steps):
+                    step(args.warmup + i, st=cap, ev=evs[i])
+        stream.wait_stream(cap)
+        g_ev.replay()
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
+    stage = [sum(r[s].elapsed_time(r[s + 1]) for r in evs) / args.steps / 1e3 for s in range(n_ev - 1)]
+    if gemv:
+        names = ["quantize_act", "gemv"]
+        dom_s, dom_bytes = stage[1], mat
+    else:
+        names = [B.tqfx4_moe_stage_name(0, 0, s) for s in range(launches)]
+        dom_s, dom_bytes = stage[1], 2 * B.tqfx4_matrix_bytes(I, H)
+    stage_us = {names[s]: stage[s] * 1e6 for s in range(len(names))}
+
+    # end to end through the public API: x from pinned host memory, y (out)
+    # back to it, every step; plain calls, no graph
+    xpin = X.cpu().pin_memory()
+    xin = torch.empty(X.shape[1], device=dev)
+    res = y if gemv else out
+    resh = torch.empty(res.numel(), pin_memory=True)
+    for i in range(3):
+        xin.copy_(xpin[i], non_blocking=True)
+        step(i, x=xin)
+        resh.copy_(res, non_blocking=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for i in range(args.steps):
+        xin.copy_(xpin[i % xpool], non_blocking=True)
+        step(args.warmup + i, x=xin)
+        resh.copy_(res, non_blocking=True)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
+    te = max_over_ranks(ev0.elapsed_time(ev1) / 1e3, world, dev)
+
+    peak, peak_kind = _peaks()
+    achieved = dom_bytes / dom_s / 1e9
+    line = {
+        "metric": "effective tq2_0_fx4 GB/s (%s)" % ("GEMV 1024 x 1024" if gemv else "one expert SwiGLU FFN"),
+        "value": job_rate(step_bytes * args.steps, world, t) / 1e9, "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "i8xi4-i32,f32",
+        "data": "synthetic", "config": cfg,
+        "steps_per_s": job_rate(args.steps, world, t),
+        "repeats_ms_per_step": [r / args.steps * 1e3 for r in reps],
+        "hot_l2": {"value": step_bytes * args.steps / t_hot / 1e9, "unit": "GB/s",
+                   "ms_per_step": t_hot / args.steps * 1e3,
+                   "note": "the same steps on one resident matrix (L2-resident after the first step)"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": None, "kernel": kern,
+                     "peak_source": peak_kind + " (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
+                     else "fallback 6.8 TB/s",
+                     "stage_us": stage_us,
+                     "note": ("a single-wave launch of 32 CTAs: bound by latency (launch, one copy round trip), "
+                              "not by HBM" if gemv else "the gate and up projections of one expert")},
+        "e2e": {"value": job_rate(step_bytes * args.steps, world, te) / 1e9, "unit": "GB/s",
+                "h2d_bytes_per_step": X.shape[1] * 4, "d2h_bytes_per_step": res.numel() * 4},
+        "gpu_launches": launches * args.steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import concurrent.futures
+
+        import numpy as np
+
+        import oracle
+        xs = X[:8].cpu().numpy()
+        if gemv:
+            blocks = oracle.pack_rtn(inputs.gemv_matrix(SEED, n, k).numpy())
+
+            def one(i):
+                rq, rda, _ = oracle.quantize_act(xs[i % 8])
+                oracle.gemv(blocks, n, k, rq, rda)
+        else:
+            ex = tuple(oracle.pack_rtn(inputs.expert_matrix(SEED, 0, p, H, I, dev).cpu().numpy()) for p in (0, 1, 2))
+
+            def one(i):
+                oracle.expert_ffn(*ex, H, I, xs[i % 8])
+        done, el = 0, 0.0
+        while el < 10.0:
+            t0 = time.perf_counter()
+            one(done)
+            el += time.perf_counter() - t0
+            done += 1
+        line["cpu_baseline"] = {"value": done * step_bytes / el / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                "sample": "%d %s on one core (%.1f s)" % (done, "GEMVs" if gemv else "expert FFNs", el)}
+        cores = os.cpu_count() or 1
+        n_all = done * cores // 2 if gemv else 2 * cores
+        with concurrent.futures.ThreadPoolExecutor(max_workers=cores) as ex_:
+            t0 = time.perf_counter()
+            list(ex_.map(one, range(n_all)))
+            el_all = time.perf_counter() - t0
+        line["cpu_baseline_all_cores"] = {"value": n_all * step_bytes / el_all / 1e9, "unit": "GB/s", "cores": cores,
+                                          "kind": "oracle", "sample": "%d steps on %d threads (%.1f s wall)"
+                                          % (n_all, cores, el_all)}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 PACK_MATS = 8  # distinct 2048 x 4096 fp32 expert matrices cycled (268 MB, larger than L2)
 
 
@@ -858,9 +1104,10 @@ def main():
     ap.add_argument("--tokens", type=int, default=0,
                     help="tokens per step of the grouped workloads (default: 64 or 2048; profiling only)")
     ap.add_argument("--workload", default="moe_decode",
-                    choices=["moe_decode", "grouped_decode_64", "prefill_2048", "tiered_decode", "mxfp4_gemv",
-                             "moe_decode_mxfp4", "free_gemv", "pack_tied"],
-                    help="moe_decode (default): 1 token; grouped_decode_64: 64 tokens with Zipf(1.1) "
+                    choices=["moe_decode", "gemv_1024", "expert_ffn", "grouped_decode_64", "prefill_2048",
+                             "tiered_decode", "mxfp4_gemv", "moe_decode_mxfp4", "free_gemv", "pack_tied"],
+                    help="moe_decode (default): 1 token; gemv_1024: one 1024 x 1024 GEMV; expert_ffn: one "
+                         "SwiGLU expert FFN; grouped_decode_64: 64 tokens with Zipf(1.1) "
                          "routing; prefill_2048: 2048 tokens; tiered_decode: 1 token with the experts in "
                          "host memory; mxfp4_gemv / free_gemv: one GEMV over MXFP4 / free-scale two-plane blocks; "
                          "moe_decode_mxfp4: moe_decode with MXFP4 experts; pack_tied: the tied solver packing expert "
@@ -884,6 +1131,9 @@ def main():
         return
     if args.workload == "pack_tied":
         run_pack(args, rank, world, local)
+        return
+    if args.workload in ("gemv_1024", "expert_ffn"):
+        run_small(args, rank, world, local)
         return
     if args.workload not in ("moe_decode", "moe_decode_mxfp4"):
         run_grouped(args, rank, world, local)
