@@ -82,6 +82,20 @@ def test_moe_ffn_small_shapes(E, H, I, k, zipf):
     run_and_check(layer, seed, X)
 
 
+# shapes of the one-launch decode: 16-block slots of 1..8 row groups
+# (hidden 512..4096) or 16-block chunks of a row (8192), down slots of 1..8
+# experts (inter 512..4096) or chunks (8192); fewer experts than CTAs, more
+# experts than CTAs, top-k up to 16
+@pytest.mark.parametrize("E,H,I,k,zipf", [(64, 1024, 2048, 8, 0.0), (16, 2048, 512, 4, 1.1),
+                                          (1024, 512, 1024, 16, 0.5), (12, 4096, 4096, 7, 0.0),
+                                          (8, 8192, 1024, 3, 0.0), (8, 1024, 8192, 2, 0.0)])
+def test_moe_ffn_one_launch_shapes(E, H, I, k, zipf):
+    seed = E * 5 + H + 3 * I
+    layer = MoeLayer.synthetic(seed, E, H, I, k, zipf, DEV)
+    X = inputs.hidden_states(seed, 3, H)
+    run_and_check(layer, seed, X)
+
+
 def test_one_expert_ffn_full_size():
     # the batch-1 SwiGLU expert, gate/up 4096->2048 and down 2048->4096
     layer = MoeLayer.synthetic(1, 1, 4096, 2048, 1, 0.0, DEV)
@@ -117,6 +131,20 @@ def test_moe_decode_is_deterministic(full_layer):
     b = full_layer.ffn(x, ws)
     for p, q in zip(a, b):
         assert torch.equal(p, q)
+
+
+def test_moe_decode_many_calls_in_a_row(full_layer):
+    # the cross-CTA counters return to zero after every call: 50 calls on one
+    # workspace, alternating two tokens, each equal to the first call's result
+    X = inputs.hidden_states(6, 2, 4096).to(DEV)
+    ws = full_layer.workspace(1)
+    ref = [[t.clone() for t in full_layer.ffn(X[i], ws)] for i in range(2)]
+    outs = []
+    for c in range(50):
+        outs.append(full_layer.ffn(X[c % 2], ws)[0].clone())
+    B.tqfx4_check(ws)
+    for c, o in enumerate(outs):
+        assert torch.equal(o, ref[c % 2][0])
 
 
 def test_moe_top_k_equals_n_experts():
