@@ -56,9 +56,9 @@ def _peaks():
         return 6800.0, "fallback"
 
 
-# DRAM bytes (read + write) of one moe_fused_kernel launch (the whole one-token layer), from an
-# ncu capture; None until the current kernel has been captured.
-DECODE_TRAFFIC = None
+# DRAM bytes (read + write) of one gate_up_kernel launch of the 256-expert layer, from an ncu
+# capture; None until the current kernel has been captured.
+GATE_UP_TRAFFIC = None
 # The same for one tc_gemm_kernel gate/up launch of the 2048-token prefill: an ncu capture at 64
 # experts and 512 tokens (one chunk per expert, as in the full workload) scaled by the full
 # workload's 4x weight bytes and pairs.
@@ -798,7 +798,7 @@ def run_small(args, rank, world, local):
             L = layers[0 if hot else i % M]
             L.ffn(X[i % xpool] if x is None else x, ws, out, sel, selw, stream=st, events=ev)
         launches = n_st
-        kern = "moe_fused_kernel (the whole one-expert layer in one launch)"
+        kern = "gate_up"
         cfg = {"workload": "expert_ffn_h4096_i2048", "hidden": Hh, "inter": Ii, "expert_bytes": mat,
                "pool_experts": M, "router": "one expert (a single 4096-element logit, weight 1)",
                "l2": "inputs larger than L2: %d distinct experts (%d MB) rotated, a new activation per step"
@@ -875,7 +875,7 @@ def run_small(args, rank, world, local):
         dom_s, dom_bytes = stage[1], mat
     else:
         names = [B.tqfx4_moe_stage_name(0, 0, s) for s in range(launches)]
-        dom_s, dom_bytes = stage[0], mat
+        dom_s, dom_bytes = stage[1], 2 * B.tqfx4_matrix_bytes(I, H)
     stage_us = {names[s]: stage[s] * 1e6 for s in range(len(names))}
 
     # end to end through the public API: x from pinned host memory, y (out)
@@ -918,7 +918,7 @@ def run_small(args, rank, world, local):
                      else "fallback 6.8 TB/s",
                      "stage_us": stage_us,
                      "note": ("a single-wave launch of 32 CTAs: bound by latency (launch, one copy round trip), "
-                              "not by HBM" if gemv else "the expert's three matrices over the layer's launch")},
+                              "not by HBM" if gemv else "the gate and up projections of one expert")},
         "e2e": {"value": job_rate(step_bytes * args.steps, world, te) / 1e9, "unit": "GB/s",
                 "h2d_bytes_per_step": X.shape[1] * 4, "d2h_bytes_per_step": res.numel() * 4},
         "gpu_launches": launches * args.steps,
@@ -1235,9 +1235,9 @@ def main():
         for s in range(n_st):
             acc[s] += row[s].elapsed_time(row[s + 1]) / 1e3
     stage_s = {names[s]: acc[s] / args.steps for s in range(n_st)}
-    dom = "gate_up" if mx else "moe_layer"
+    dom = "gate_up"
     peak, peak_kind = _peaks()
-    achieved = (gu_bytes if mx else per_token) / stage_s[dom] / 1e9
+    achieved = gu_bytes / stage_s[dom] / 1e9
 
     # ---- end to end through the public API with host buffers ----
     Xh = X.cpu().pin_memory()
@@ -1275,18 +1275,17 @@ def main():
         "tokens_per_s": tokens / t,
         "pct_of_hbm_peak": 100.0 * value / peak,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": None if mx else DECODE_TRAFFIC,
-                     "kernel": "mxfp4_gemv_kernel (gate_up)" if mx else
-                               "moe_fused_kernel (router, gate/up, SwiGLU, down and combine in one launch)",
-                     "algorithmic_bytes": gu_bytes if mx else per_token,
-                     "traffic_source": "ncu capture (dram__bytes_read + write) of one launch",
+                     "frac": achieved / peak, "traffic": None if mx else GATE_UP_TRAFFIC,
+                     "kernel": "mxfp4_gemv_kernel (gate_up)" if mx else dom,
+                     "algorithmic_bytes": gu_bytes,
+                     "traffic_source": "ncu capture (dram__bytes_read + write) of one gate_up_kernel launch",
                      "peak_source": peak_kind + " (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
                      else "fallback 6.8 TB/s",
                      "stage_us": {k: v * 1e6 for k, v in stage_s.items()}},
         "e2e": {"value": e2e, "unit": "GB/s", "h2d_bytes_per_step": H * 4,
                 "d2h_bytes_per_step": H * 4 + TOPK * 4},
         # router, gate_up, down (tq2_0_fx4); router, gate_up, down, combine (MXFP4)
-        "gpu_launches": (4 if mx else 1) * args.steps,
+        "gpu_launches": (4 if mx else 3) * args.steps,
         "clocks": clk.summary(),
         "repeats_ms_per_step": {"min": min(reps_ms), "median": statistics.median(reps_ms), "max": max(reps_ms),
                                 "spread": (max(reps_ms) - min(reps_ms)) / statistics.median(reps_ms),

@@ -377,10 +377,7 @@ tqfx4_status tqfx4_moe_ffn_noalloc(const tqfx4_experts *ex, const tqfx4_router *
  * `events[i]` (cudaEvent_t, created by the caller) on the stream before
  * stage i, and events[n_stages] after the last stage, where n_stages is
  * given by tqfx4_moe_stage_count. Stage names come from
- * tqfx4_moe_stage_name. tqfx4_moe_ffn has one stage, "moe_layer" (its
- * router, gate/up, SwiGLU, down and combine run as one launch for hidden
- * and intermediate sizes of 512, 1024, 2048, 4096 or a multiple of 4096,
- * else as three launches that the two events bracket together).
+ * tqfx4_moe_stage_name.
  */
 int tqfx4_moe_stage_count(int grouped, int path);
 const char *tqfx4_moe_stage_name(int grouped, int path, int stage);

@@ -224,15 +224,17 @@ size_t tqfx4_moe_workspace_bytes(const tqfx4_experts *ex, const tqfx4_router *rt
 int tqfx4_moe_stage_count(int grouped, int path) {
     (void)path;
     if (grouped == 2) return 4;
-    return grouped ? tq::grouped_stage_count() : 1;
+    return grouped ? tq::grouped_stage_count() : 3;
 }
 
 const char *tqfx4_moe_stage_name(int grouped, int path, int stage) {
     (void)path;
+    static const char *dec[] = {"router", "gate_up", "down"};
     static const char *mx[] = {"router", "gate_up", "down", "combine"};
     if (grouped == 2) return (stage >= 0 && stage < 4) ? mx[stage] : "";
     if (grouped) return tq::grouped_stage_name(stage);
-    return stage == 0 ? "moe_layer" : "";
+    if (stage >= 0 && stage < 3) return dec[stage];
+    return "";
 }
 
 static tqfx4_status moe_ffn_impl(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, float *out,
@@ -250,20 +252,10 @@ static tqfx4_status moe_ffn_impl(const tqfx4_experts *ex, const tqfx4_router *rt
     if (!tq::moe_decode_args(ex, rt, nullptr, a, L))
         return fail(TQFX4_ESHAPE, "%s: too many row ranges for the counter area", fn);
     if ((s = check_ws(ws, ws_bytes, L.total, fn))) return s;
-    const bool fused = tq::moe_fused_applies(a);
-    if (!fused && (tq::gate_up_smem(a) > tq::max_smem_optin() || tq::down_smem(a) > tq::max_smem_optin()))
+    if (tq::gate_up_smem(a) > tq::max_smem_optin() || tq::down_smem(a) > tq::max_smem_optin())
         return fail(TQFX4_ESHAPE, "%s: top_k x inter too large for the decode kernels' shared memory", fn);
     tq::moe_decode_args(ex, rt, ws, a, L);
-    const cudaStream_t st = static_cast<cudaStream_t>(stream);
-    cudaError_t e;
-    if (fused) {
-        cudaEvent_t const *ev = reinterpret_cast<cudaEvent_t const *>(events);
-        e = ev ? tq::record_stage_event(ev[0], st) : cudaSuccess;
-        if (e == cudaSuccess) e = tq::launch_moe_fused(a, x, out, sel_idx, sel_w, st);
-        if (e == cudaSuccess && ev) e = tq::record_stage_event(ev[1], st);
-    } else {
-        e = tq::launch_moe_decode(a, x, out, sel_idx, sel_w, st, events);
-    }
+    cudaError_t e = tq::launch_moe_decode(a, x, out, sel_idx, sel_w, static_cast<cudaStream_t>(stream), events);
     if (e != cudaSuccess) return cuda_fail(e, fn);
     return ok();
 }

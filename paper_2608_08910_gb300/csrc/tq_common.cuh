@@ -219,33 +219,6 @@ __device__ __forceinline__ void block_dot(const uint8_t *codes, const uint8_t *q
     for (int r = 0; r < 4; ++r) S[r] = lo[r] + (hi[r] >> 4) - 4 * bsum;
 }
 
-// Exact S of two rows of a block (codes: the first row's 128 bytes, the
-// second row 128 bytes on): 32 code words a row against the activation
-// words w (low nibbles) and 32 + w (high nibbles, kept at 16 u and divided
-// out), S = sum u q - 4 bsum; the activation words are loaded once for both.
-__device__ __forceinline__ void fx_row2_dot(const uint2 *codes, const uint4 *qv, int L, int bsum, int &S0,
-                                            int &S1) {
-    int lo[2] = {0, 0}, hi[2] = {0, 0};
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        const uint4 ql = qv[i * L], qh = qv[(8 + i) * L];  // activation words 4i..4i+3 and 32+4i..
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-            const uint2 c0 = codes[16 * r + 2 * i], c1 = codes[16 * r + 2 * i + 1];
-            lo[r] = dp4a_us(c0.x & 0x0f0f0f0fu, ql.x, lo[r]);
-            lo[r] = dp4a_us(c0.y & 0x0f0f0f0fu, ql.y, lo[r]);
-            lo[r] = dp4a_us(c1.x & 0x0f0f0f0fu, ql.z, lo[r]);
-            lo[r] = dp4a_us(c1.y & 0x0f0f0f0fu, ql.w, lo[r]);
-            hi[r] = dp4a_us(c0.x & 0xf0f0f0f0u, qh.x, hi[r]);
-            hi[r] = dp4a_us(c0.y & 0xf0f0f0f0u, qh.y, hi[r]);
-            hi[r] = dp4a_us(c1.x & 0xf0f0f0f0u, qh.z, hi[r]);
-            hi[r] = dp4a_us(c1.y & 0xf0f0f0f0u, qh.w, hi[r]);
-        }
-    }
-    S0 = lo[0] + (hi[0] >> 4) - 4 * bsum;
-    S1 = lo[1] + (hi[1] >> 4) - 4 * bsum;
-}
-
 // Scale of row r (0..3) of the block at `blk` (shared memory), as fp32.
 __device__ __forceinline__ float block_scale(const uint8_t *blk, int r) {
     const __half h = *reinterpret_cast<const __half *>(blk + 2 * r);

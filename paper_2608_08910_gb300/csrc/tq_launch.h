@@ -65,10 +65,5 @@ int grouped_stage_count();
 const char *grouped_stage_name(int s);
 int down_smem(const MoeArgs &a);
 cudaError_t launch_selftest_timeout(int *status, cudaStream_t st);
-// The one-launch decode (tq_moe_fused.cu): whether it serves these shapes,
-// and its launch.
-bool moe_fused_applies(const MoeArgs &a);
-cudaError_t launch_moe_fused(const MoeArgs &a, const float *x, float *out, int32_t *sel_idx, float *sel_w,
-                             cudaStream_t st);
 
 }  // namespace tq

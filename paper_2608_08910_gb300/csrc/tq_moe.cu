@@ -1,9 +1,7 @@
 // tqfx4_moe_ffn: one token through a routed-expert MoE layer whose gate/up/
 // down projections are tq2_0_fx4 matrices (Tied Trit-Planes, Sec. 1 and 2.2).
 //
-// Three launches, reading only the selected experts' bytes (the path for
-// the shapes the one-launch decode of tq_moe_fused.cu does not take, and
-// the two halves of the expert tier's decode):
+// Three launches, reading only the selected experts' bytes:
 //   router   one CTA per expert: logit W_r[e] x + bias[e] by a compensated
 //            binary32 dot product kept as a double-binary32 pair; extra CTAs
 //            quantize x. The CTA that finishes last (one counter) selects
@@ -405,13 +403,15 @@ cudaError_t launch_moe_decode(const MoeArgs &a0, const float *x, float *out, int
     rec(0);
     router_kernel<<<a.E + (a.nbh + 3) / 4, 128, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    if ((e = launch_pdl(reinterpret_cast<const void *>(gate_up_kernel), a.top_k * a.parts_gu, a.warps_gu * 32,
-                        gate_up_smem(a), st, false, a)) != cudaSuccess)
-        return e;
-    if ((e = launch_pdl(reinterpret_cast<const void *>(down_kernel), a.top_k * a.parts_d, a.warps_d * 32,
-                        down_smem(a), st, false, a)) != cudaSuccess)
-        return e;
     rec(1);
+    if ((e = launch_pdl(reinterpret_cast<const void *>(gate_up_kernel), a.top_k * a.parts_gu, a.warps_gu * 32,
+                        gate_up_smem(a), st, events != nullptr, a)) != cudaSuccess)
+        return e;
+    rec(2);
+    if ((e = launch_pdl(reinterpret_cast<const void *>(down_kernel), a.top_k * a.parts_d, a.warps_d * 32,
+                        down_smem(a), st, events != nullptr, a)) != cudaSuccess)
+        return e;
+    rec(3);
     return cudaSuccess;
 }
 

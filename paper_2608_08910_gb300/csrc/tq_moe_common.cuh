@@ -319,9 +319,7 @@ __device__ __forceinline__ unsigned long long topk_key(float hi, float lo, int e
 // shifts its list. Keys are distinct (their low bits are the expert index),
 // so exactly one lane owns the maximum. Writes the selection, in rank order,
 // to res. All lanes of the warp must call.
-// kShared: the logits are in shared memory (plain loads) rather than in
-// global memory (read through L2).
-template <int KPL, bool kShared = false>
+template <int KPL>
 __device__ __forceinline__ void topk_warp_kpl(const float *lhi, const float *llo, int E, int k, int *res) {
     const int lane = threadIdx.x & 31;
     uint32_t kh[KPL], kl[KPL];  // (0, 0) is below every key
@@ -329,8 +327,8 @@ __device__ __forceinline__ void topk_warp_kpl(const float *lhi, const float *llo
 #pragma unroll
     for (int i = 0; i < KPL; ++i) {  // all loads in flight before the first use
         const int e = lane + 32 * i;
-        h[i] = e < E ? (kShared ? lhi[e] : __ldcg(lhi + e)) : 0.0f;
-        l[i] = e < E ? (kShared ? llo[e] : __ldcg(llo + e)) : 0.0f;
+        h[i] = e < E ? __ldcg(lhi + e) : 0.0f;
+        l[i] = e < E ? __ldcg(llo + e) : 0.0f;
     }
 #pragma unroll
     for (int i = 0; i < KPL; ++i) {
@@ -373,14 +371,13 @@ __device__ __forceinline__ void topk_warp_kpl(const float *lhi, const float *llo
 }
 
 // topk_warp_kpl with the register capacity chosen for E (<= 1024).
-template <bool kShared = false>
 __device__ __forceinline__ void topk_warp(const float *lhi, const float *llo, int E, int k, int *res) {
     if (E <= 256)
-        topk_warp_kpl<8, kShared>(lhi, llo, E, k, res);
+        topk_warp_kpl<8>(lhi, llo, E, k, res);
     else if (E <= 512)
-        topk_warp_kpl<16, kShared>(lhi, llo, E, k, res);
+        topk_warp_kpl<16>(lhi, llo, E, k, res);
     else
-        topk_warp_kpl<32, kShared>(lhi, llo, E, k, res);
+        topk_warp_kpl<32>(lhi, llo, E, k, res);
 }
 
 // ---- double-binary32 softmax ----------------------------------------------------
@@ -434,37 +431,6 @@ __device__ __forceinline__ void ff_exp_nonpos(float dh, float dl, float &eh, flo
     const int n = static_cast<int>(nf);
     eh = ldexpf(ph, n);
     el = ldexpf(pl, n);
-}
-
-// Softmax weights from the selected logits themselves, in rank order
-// (sh[j], sl[j]: the double-binary32 logit of the j-th selected expert, any
-// memory the warp can read): the arithmetic of softmax_ff_warp below, so
-// the weights are the same bits. Writes w[0..k) from lanes j < k.
-__device__ __forceinline__ void softmax_ff_sel(const float *sh, const float *sl, int k, float *w) {
-    const int lane = threadIdx.x & 31;
-    const float h0 = sh[0], l0 = sl[0];
-    float eh = 0.0f, el = 0.0f;
-    if (lane < k) {
-        float dh, dl;
-        ff_add(sh[lane], sl[lane], -h0, -l0, dh, dl);
-        ff_exp_nonpos(dh, dl, eh, el);
-    }
-    float s_h = eh, s_l = el;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float oh = __shfl_xor_sync(0xffffffffu, s_h, o), ol = __shfl_xor_sync(0xffffffffu, s_l, o);
-        ff_add(s_h, s_l, oh, ol, s_h, s_l);
-    }
-    if (lane < k) {
-        const float q = __fdiv_rn(eh, s_h);
-        float ph, pl;
-        ff_mul(q, 0.0f, s_h, s_l, ph, pl);
-        float rh, rl;
-        ff_add(eh, el, -ph, -pl, rh, rl);
-        const float q2 = __fdiv_rn(rh, s_h);
-        w[lane] = __fadd_rn(q, q2);
-    }
-    __syncwarp();
 }
 
 // Softmax weights of the selected logits sel[0..k) (k <= 32) by one warp:

@@ -84,9 +84,8 @@ def test_moe_workspace_layout(lib):
 
 
 def test_stage_names(lib):
-    assert lib.tqfx4_moe_stage_count(0, 0) == 1
-    assert lib.tqfx4_moe_stage_name(0, 0, 0).decode() == "moe_layer"
-    assert lib.tqfx4_moe_stage_name(0, 0, 1).decode() == ""
+    assert lib.tqfx4_moe_stage_count(0, 0) == 3
+    assert [lib.tqfx4_moe_stage_name(0, 0, s).decode() for s in range(3)] == ["router", "gate_up", "down"]
     n = lib.tqfx4_moe_stage_count(1, 0)
     names = [lib.tqfx4_moe_stage_name(1, 0, s).decode() for s in range(n)]
     assert names[0] == "router" and "gate_up" in names and "down" in names and names[-1] == "combine"

@@ -82,14 +82,13 @@ def test_moe_ffn_small_shapes(E, H, I, k, zipf):
     run_and_check(layer, seed, X)
 
 
-# shapes of the one-launch decode: 16-block slots of 1..8 row groups
-# (hidden 512..4096) or 16-block chunks of a row (8192), down slots of 1..8
-# experts (inter 512..4096) or chunks (8192); fewer experts than CTAs, more
-# experts than CTAs, top-k up to 16
+# hidden and intermediate sizes from 512 to 8192 (rows of 2 to 32 blocks),
+# fewer and more experts than SMs, top-k up to 16 and a top-k of 7 (row
+# ranges that do not divide evenly)
 @pytest.mark.parametrize("E,H,I,k,zipf", [(64, 1024, 2048, 8, 0.0), (16, 2048, 512, 4, 1.1),
                                           (1024, 512, 1024, 16, 0.5), (12, 4096, 4096, 7, 0.0),
                                           (8, 8192, 1024, 3, 0.0), (8, 1024, 8192, 2, 0.0)])
-def test_moe_ffn_one_launch_shapes(E, H, I, k, zipf):
+def test_moe_ffn_more_shapes(E, H, I, k, zipf):
     seed = E * 5 + H + 3 * I
     layer = MoeLayer.synthetic(seed, E, H, I, k, zipf, DEV)
     X = inputs.hidden_states(seed, 3, H)
