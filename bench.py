@@ -56,13 +56,14 @@ def _peaks():
         return 6800.0, "fallback"
 
 
-# DRAM bytes (read + write) of one gate_up_kernel launch of the 256-expert layer, from an ncu
-# capture; None until the current kernel has been captured.
-GATE_UP_TRAFFIC = None
+# DRAM bytes (read + write) of one gate_up_kernel launch, from an ncu --set full capture of the
+# 64-expert layer (one launch reads the 8 selected experts whatever the expert count). Set to None
+# when the kernel changes until it is captured again.
+GATE_UP_TRAFFIC = 68196864 + 982528
 # The same for one tc_gemm_kernel gate/up launch of the 2048-token prefill: an ncu capture at 64
 # experts and 512 tokens (one chunk per expert, as in the full workload) scaled by the full
 # workload's 4x weight bytes and pairs.
-TC_GATE_UP_TRAFFIC = 4 * (581043968 + 59059456)
+TC_GATE_UP_TRAFFIC = 4 * (580448000 + 58149632)
 
 
 def max_over_ranks(t, world, device):
@@ -537,7 +538,7 @@ GEMV_N, GEMV_K, GEMV_POOL = 131072, 4096, 16
 # DRAM bytes (read + write) of one launch of the GEMV kernels on the 131072 x
 # 4096 workload, from ncu --set full captures (profiles/); None once a kernel
 # changes until it is captured again.
-GEMV_TRAFFIC = {"mxfp4_gemv": 285286144 + 3272960, "free_gemv": 276862976 + 3671296}
+GEMV_TRAFFIC = {"mxfp4_gemv": 285286144 + 3272960, "free_gemv": 276858112 + 3605504}
 
 
 def run_gemv(args, rank, world, local):
