@@ -4,11 +4,24 @@
 #include <cstdio>
 #include <cstring>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "tq_launch.h"
 #include "tq_moe_common.cuh"
 #include "tqfx4.h"
 
 namespace {
+
+// One NVTX range per call that enqueues work, named after the entry point,
+// so that a profiler shows the library's calls on the host timeline (the
+// header-only NVTX API returns at once when no tool is attached).
+struct TqRange {
+    explicit TqRange(const char *name) { nvtxRangePushA(name); }
+    ~TqRange() { nvtxRangePop(); }
+    TqRange(const TqRange &) = delete;
+    TqRange &operator=(const TqRange &) = delete;
+};
+#define TQ_RANGE() TqRange tq_range_(__func__)
 
 thread_local char g_err[512] = "";
 
@@ -65,6 +78,7 @@ size_t tqfx4_basic_workspace_bytes(void) { return TQFX4_STATUS_BYTES; }
 
 tqfx4_status tqfx4_pack(int src, const void *a, const int8_t *t2, const uint16_t *scales_f16, int64_t n,
                         int64_t k, void *blocks, void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
     tqfx4_status s = check_nk(n, k, "tqfx4_pack");
     if (s) return s;
     if ((s = check_ws(ws, ws_bytes, TQFX4_STATUS_BYTES, "tqfx4_pack"))) return s;
@@ -89,6 +103,7 @@ tqfx4_status tqfx4_pack(int src, const void *a, const int8_t *t2, const uint16_t
 
 tqfx4_status tqfx4_quantize_act(const float *x, int64_t m, int64_t k, int8_t *q, float *da, int32_t *bsum,
                                 void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
     tqfx4_status s = check_nk(0, k, "tqfx4_quantize_act");
     if (s) return s;
     if (m < 0) return fail(TQFX4_EINVAL, "tqfx4_quantize_act: negative m");
@@ -106,6 +121,7 @@ tqfx4_status tqfx4_quantize_act(const float *x, int64_t m, int64_t k, int8_t *q,
 tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
                         const int32_t *bsum, float *y, int32_t *block_sums, void *ws, size_t ws_bytes,
                         void *stream) {
+    TQ_RANGE();
     tqfx4_status s = check_nk(n, k, "tqfx4_gemv");
     if (s) return s;
     if (k > TQFX4_MAX_K) return fail(TQFX4_ESHAPE, "tqfx4_gemv: k=%lld exceeds %d", (long long)k, TQFX4_MAX_K);
@@ -127,6 +143,7 @@ int64_t tqfx4_free_bytes(int64_t n, int64_t k) { return tq::free_bytes(n, k); }
 
 tqfx4_status tqfx4_pack_free(const int8_t *t1, const int8_t *t2, const uint16_t *a1_f16, const uint16_t *a2_f16,
                              int64_t n, int64_t k, void *blocks, void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
     const char *fn = "tqfx4_pack_free";
     tqfx4_status s = check_nk(n, k, fn);
     if (s) return s;
@@ -144,6 +161,7 @@ tqfx4_status tqfx4_pack_free(const int8_t *t1, const int8_t *t2, const uint16_t 
 tqfx4_status tqfx4_gemv_free(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
                              const int32_t *bsum, float *y, int32_t *S1, int32_t *S2, void *ws, size_t ws_bytes,
                              void *stream) {
+    TQ_RANGE();
     const char *fn = "tqfx4_gemv_free";
     tqfx4_status s = check_nk(n, k, fn);
     if (s) return s;
@@ -168,6 +186,7 @@ int64_t tqfx4_mxfp4_bytes(int64_t n, int64_t k) { return tq::mxfp4_bytes(n, k); 
 
 tqfx4_status tqfx4_gemv_mxfp4(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da, float *y,
                               int32_t *block_sums, void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
     const char *fn = "tqfx4_gemv_mxfp4";
     if (n < 0 || k <= 0 || k % 512 || k > TQFX4_MAX_K)
         return fail(TQFX4_ESHAPE, "%s: k=%lld must be a positive multiple of 512 <= %d", fn, (long long)k,
@@ -262,17 +281,20 @@ static tqfx4_status moe_ffn_impl(const tqfx4_experts *ex, const tqfx4_router *rt
 
 tqfx4_status tqfx4_moe_ffn(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, float *out,
                            int32_t *sel_idx, float *sel_w, void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
     return moe_ffn_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, nullptr);
 }
 
 tqfx4_status tqfx4_moe_ffn_traced(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, float *out,
                                   int32_t *sel_idx, float *sel_w, void *ws, size_t ws_bytes, void *stream,
                                   void *const *events) {
+    TQ_RANGE();
     return moe_ffn_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, events);
 }
 
 tqfx4_status tqfx4_moe_route(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, int32_t *sel_idx,
                              float *sel_w, void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
     const char *fn = "tqfx4_moe_route";
     tqfx4_status s = check_moe_shapes(ex, rt, fn);
     if (s) return s;
@@ -328,17 +350,20 @@ static tqfx4_status moe_ffn_mxfp4_impl(const tqfx4_experts *ex, const tqfx4_rout
 
 tqfx4_status tqfx4_moe_ffn_mxfp4(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, float *out,
                                  int32_t *sel_idx, float *sel_w, void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
     return moe_ffn_mxfp4_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, nullptr);
 }
 
 tqfx4_status tqfx4_moe_ffn_mxfp4_traced(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x,
                                         float *out, int32_t *sel_idx, float *sel_w, void *ws, size_t ws_bytes,
                                         void *stream, void *const *events) {
+    TQ_RANGE();
     return moe_ffn_mxfp4_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, events);
 }
 
 tqfx4_status tqfx4_moe_experts(const tqfx4_experts *ex, const tqfx4_router *rt, const void *const *ptrs, float *out,
                                void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
     const char *fn = "tqfx4_moe_experts";
     tqfx4_status s = check_moe_shapes(ex, rt, fn);
     if (s) return s;
@@ -388,12 +413,14 @@ static tqfx4_status moe_grouped_impl(const tqfx4_experts *ex, const tqfx4_router
 tqfx4_status tqfx4_moe_grouped(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X, int64_t T,
                                float *OUT, int32_t *sel_idx, float *sel_w, int path, void *ws, size_t ws_bytes,
                                void *stream) {
+    TQ_RANGE();
     return moe_grouped_impl(ex, rt, X, T, OUT, sel_idx, sel_w, path, ws, ws_bytes, stream, nullptr);
 }
 
 tqfx4_status tqfx4_moe_grouped_traced(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X, int64_t T,
                                       float *OUT, int32_t *sel_idx, float *sel_w, int path, void *ws,
                                       size_t ws_bytes, void *stream, void *const *events) {
+    TQ_RANGE();
     return moe_grouped_impl(ex, rt, X, T, OUT, sel_idx, sel_w, path, ws, ws_bytes, stream, events);
 }
 
@@ -427,6 +454,7 @@ tqfx4_status tqfx4_moe_workspace_views(const tqfx4_experts *ex, const tqfx4_rout
 }
 
 tqfx4_status tqfx4_check(void *ws, void *stream) {
+    TQ_RANGE();
     if (!ws) return fail(TQFX4_EINVAL, "tqfx4_check: workspace is NULL");
     cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "tqfx4_check: stream");
@@ -446,6 +474,7 @@ tqfx4_status tqfx4_check(void *ws, void *stream) {
 }
 
 tqfx4_status tqfx4_selftest_wait_timeout(void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
     tqfx4_status s = check_ws(ws, ws_bytes, TQFX4_STATUS_BYTES, "tqfx4_selftest_wait_timeout");
     if (s) return s;
     cudaError_t e = tq::launch_selftest_timeout(static_cast<int *>(ws), static_cast<cudaStream_t>(stream));

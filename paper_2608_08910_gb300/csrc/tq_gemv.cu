@@ -43,6 +43,8 @@ __global__ void __launch_bounds__(256, 1) gemv_kernel(const uint8_t *__restrict_
                                      g.stages, g.slot_bytes, g.rpu, nb);
     ring_init(ring);
     fence_barrier_init();
+    grid_dependency_wait();  // the blocks, q, da and bsum may come from the previous kernel
+    grid_dependents_launch();
     MatJob job;
     job.mat = blocks;
     job.rg_begin = static_cast<int64_t>(blockIdx.x) * g.rg_per_cta;
@@ -129,6 +131,8 @@ __global__ void __launch_bounds__(FX_WARPS * 32) gemv_chunk_kernel(const uint8_t
     if (lane == 0)
         for (int i = 0; i < FX_SLOTS; ++i) mbar_init(&bars[i], 1);
     fence_barrier_init();
+    grid_dependency_wait();  // the blocks, q, da and bsum may come from the previous kernel
+    grid_dependents_launch();
 
     const int64_t groups = g.n / ROWS;
     const int64_t NW = static_cast<int64_t>(gridDim.x) * FX_WARPS;
@@ -314,13 +318,10 @@ cudaError_t launch_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
         const int64_t cap = static_cast<int64_t>(num_sms()) * (per_sm > 0 ? per_sm : 1);
         if (grid > cap) grid = cap;
         const uint8_t *b = static_cast<const uint8_t *>(blocks);
-        if (sums)
-            gemv_chunk_kernel<true><<<static_cast<unsigned>(grid), FX_WARPS * 32, smem, st>>>(b, f, q, da, bsum, y,
-                                                                                              block_sums, status);
-        else
-            gemv_chunk_kernel<false><<<static_cast<unsigned>(grid), FX_WARPS * 32, smem, st>>>(b, f, q, da, bsum, y,
-                                                                                               nullptr, status);
-        return cudaGetLastError();
+        const dim3 gd(static_cast<unsigned>(grid)), bd(FX_WARPS * 32);
+        if (sums) return launch_dependent(gemv_chunk_kernel<true>, gd, bd, smem, st, b, f, q, da, bsum, y, block_sums, status);
+        return launch_dependent(gemv_chunk_kernel<false>, gd, bd, smem, st, b, f, q, da, bsum, y,
+                                static_cast<int32_t *>(nullptr), status);
     }
     const GemvGeom g = gemv_geom(n, k);
     const int smem = gemv_act_bytes(g.nb) + g.warps * stream_warp_bytes(g.stages, g.slot_bytes, g.rpu, g.nb);
@@ -328,9 +329,8 @@ cudaError_t launch_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
     cudaError_t e = allow_max_smem(reinterpret_cast<const void *>(gemv_kernel), smem_set);
     if (e != cudaSuccess) return e;
     const int grid = static_cast<int>((g.n_rg + g.rg_per_cta - 1) / g.rg_per_cta);
-    gemv_kernel<<<grid, g.warps * 32, smem, st>>>(static_cast<const uint8_t *>(blocks), g, q, da, bsum, y,
-                                                  block_sums, status);
-    return cudaGetLastError();
+    return launch_dependent(gemv_kernel, dim3(grid), dim3(g.warps * 32), smem, st, static_cast<const uint8_t *>(blocks),
+                            g, q, da, bsum, y, block_sums, status);
 }
 
 }  // namespace tq

@@ -66,4 +66,25 @@ const char *grouped_stage_name(int s);
 int down_smem(const MoeArgs &a);
 cudaError_t launch_selftest_timeout(int *status, cudaStream_t st);
 
+// kernel<<<grid, block, smem, st>>>(args...) as a programmatic dependent of
+// the previous kernel in the stream: its CTAs may become resident while that
+// kernel drains. Every kernel launched this way executes griddepcontrol.wait
+// before its first access to global memory, so the order of the stream
+// holds.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                                    Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
 }  // namespace tq

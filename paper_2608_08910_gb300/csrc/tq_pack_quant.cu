@@ -123,6 +123,8 @@ __global__ void __launch_bounds__(256) pack_kernel(const void *a, const int8_t *
 // One warp per (row, block) of the activations.
 __global__ void __launch_bounds__(256) quantize_kernel(const float *x, int64_t units, int nb, int64_t k,
                                                        int8_t *q, float *da, int32_t *bsum, int *status) {
+    grid_dependency_wait();  // x may come from the previous kernel
+    grid_dependents_launch();
     const int lane = threadIdx.x & 31;
     const int64_t unit = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     if (unit >= units) return;
@@ -169,8 +171,8 @@ cudaError_t launch_quantize(const float *x, int64_t m, int64_t k, int8_t *q, flo
     const int64_t units = m * nb;
     if (units == 0) return cudaSuccess;
     const int64_t grid = (units * 32 + 255) / 256;
-    quantize_kernel<<<static_cast<unsigned>(grid), 256, 0, st>>>(x, units, nb, k, q, da, bsum, status);
-    return cudaGetLastError();
+    return launch_dependent(quantize_kernel, dim3(static_cast<unsigned>(grid)), dim3(256), 0, st, x, units, nb, k, q,
+                            da, bsum, status);
 }
 
 }  // namespace tq
