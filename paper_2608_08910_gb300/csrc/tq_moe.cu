@@ -82,7 +82,8 @@ __global__ void __launch_bounds__(128) router_kernel(MoeArgs a) {
         if (a.bias) ff_add(hi, lo, __ldg(a.bias + e), 0.0f, hi, lo);
         a.logits[e] = hi;
         a.logits_lo[e] = lo;
-        last = (atomic_add_acq_rel(&a.ctr[kCtrRouter], 1) == a.E - 1);
+        // one expert: this CTA is the last (its logit is its own), no count
+        last = a.E == 1 || atomic_add_acq_rel(&a.ctr[kCtrRouter], 1) == a.E - 1;
     }
     __syncthreads();
     TQ_STAMP(0, 2);
@@ -269,7 +270,8 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
     if (any) warp_stream_run(ring, job, a.rpu_d, warp, a.warps_d, a.status, K_DOWN);
     __syncthreads();
     TQ_STAMP(2, 4);
-    if (threadIdx.x == 0) last = (atomic_add_acq_rel(&a.ctr[kCtrDown + p], 1) == K - 1);
+    // top-1: this CTA alone holds row range p (its rows are its own), no count
+    if (threadIdx.x == 0) last = K == 1 || atomic_add_acq_rel(&a.ctr[kCtrDown + p], 1) == K - 1;
     __syncthreads();
     if (!last) return;
     const int64_t r0 = job.rg_begin * 4, r1 = job.rg_end * 4;
