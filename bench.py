@@ -728,8 +728,9 @@ def run_small(args, rank, world, local):
     larger than L2 (at least 256 MB), one pool entry per step, a new
     activation every step:
     gemv_1024: one 1024 x 1024 tq2_0_fx4 GEMV (round-to-nearest codes of
-      N(0, 0.02) weights) of an N(0, 1) vector: tqfx4_quantize_act, then
-      tqfx4_gemv; 512 matrices (273 MB) rotated.
+      N(0, 0.02) weights) of an N(0, 1) vector quantized per block:
+      tqfx4_gemv_x (the quantization and the GEMV in one launch); 505
+      matrices (269 MB) rotated.
     expert_ffn: one SwiGLU expert, gate/up 4096 -> 2048, down 2048 -> 4096,
       Student-t(5) x 0.02 weights: tqfx4_moe_ffn on a one-expert layer (its
       router is a single 4096-element logit, its weight 1); 21 such experts
@@ -760,24 +761,19 @@ def run_small(args, rank, world, local):
         pool = ops.pack_rtn(inputs.gemv_matrix(SEED, M * n, k, dev), ws)
         torch.cuda.empty_cache()
         X = inputs.hidden_states(SEED + rank, xpool, k, dev)
-        q = torch.empty(k, dtype=torch.int8, device=dev)
-        da = torch.empty(k // 256, device=dev)
-        bs = torch.empty(k // 256, dtype=torch.int32, device=dev)
         y = torch.empty(n, device=dev)
         step_bytes = mat
 
         def step(i, st=stream, hot=False, ev=None, x=None):
             if ev:
                 ev[0].record(st)
-            B.tqfx4_quantize_act(X[i % xpool] if x is None else x, 1, k, q, da, bs, ws, st)
+            m = 0 if hot else i % M
+            B.tqfx4_gemv_x(pool[m * mat:(m + 1) * mat], n, k, X[i % xpool] if x is None else x, y, None, None,
+                           None, ws, st)
             if ev:
                 ev[1].record(st)
-            m = 0 if hot else i % M
-            B.tqfx4_gemv(pool[m * mat:(m + 1) * mat], n, k, q, da, bs, y, None, ws, st)
-            if ev:
-                ev[2].record(st)
-        launches = 2
-        kern = "gemv_chunk_kernel"
+        launches = 1
+        kern = "gemv_chunk_kernel (quantization inside)"
         cfg = {"workload": "gemv_1024x1024", "n": n, "k": k, "matrix_bytes": mat, "pool_matrices": M,
                "l2": "inputs larger than L2: %d distinct matrices (%d MB) rotated, a new activation per step"
                      % (M, M * mat >> 20)}
@@ -849,7 +845,7 @@ def run_small(args, rank, world, local):
     # step, on the launching stream, in plain stream order (the library's
     # traced call records its own stage events; the GEMV steps are not
     # captured, since an event recorded by torch inside a capture does not time)
-    n_ev = 3 if gemv else launches + 1
+    n_ev = launches + 1
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_ev)] for _ in range(args.steps)]
     for row in evs:
         for e_ in row:
@@ -872,8 +868,8 @@ def run_small(args, rank, world, local):
     B.tqfx4_check(ws)
     stage = [sum(r[s].elapsed_time(r[s + 1]) for r in evs) / args.steps / 1e3 for s in range(n_ev - 1)]
     if gemv:
-        names = ["quantize_act", "gemv"]
-        dom_s, dom_bytes = stage[1], mat
+        names = ["gemv_x"]
+        dom_s, dom_bytes = stage[0], mat
     else:
         names = [B.tqfx4_moe_stage_name(0, 0, s) for s in range(launches)]
         dom_s, dom_bytes = stage[1], 2 * B.tqfx4_matrix_bytes(I, H)

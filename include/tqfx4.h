@@ -159,6 +159,23 @@ tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k,
                         void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * tqfx4_gemv_x -- tqfx4_quantize_act and tqfx4_gemv in one launch (Sec. 2.2):
+ * y = W x for one fp32 vector x, quantized per 256-block inside the kernel
+ * with the quantizer of tqfx4_quantize_act, then dotted as tqfx4_gemv does;
+ * q, da, bsum and y are the two calls' results bit for bit.
+ *   blocks: device, the N x K matrix (16-byte aligned). x: fp32 [k]
+ *   (device, 16-byte aligned). y: fp32 [n] (device).
+ *   q, da, bsum: all NULL, or device outputs for the quantized vector (k
+ *   bytes 16-byte aligned, k/256 and k/256 entries).
+ *   k must be a positive multiple of 512 up to TQFX4_MAX_K (the chunked
+ *   pass), else TQFX4_ESHAPE; n == 0 does nothing. A non-finite x sets
+ *   TQFX4_EDATA.
+ */
+tqfx4_status tqfx4_gemv_x(const void *blocks, int64_t n, int64_t k, const float *x, float *y,
+                          int8_t *q, float *da, int32_t *bsum,
+                          void *ws, size_t ws_bytes, void *stream);
+
+/*
  * The free-scale two-plane format (Table 1's free-scale K=2 row, 4.125
  * bits/weight; the ablation of the tie of Sec. 2.1): W = a1 t1 + a2 t2 per
  * row and 256 columns, t1, t2 in {-1, 0, 1}, two independent f16 scales.

@@ -59,6 +59,7 @@ _SIGS = {
     "tqfx4_pack": (_int, [_int, _vp, _vp, _vp, _i64, _i64, _vp, _vp, _sz, _vp]),
     "tqfx4_quantize_act": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_gemv": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_gemv_x": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int]),
     "tqfx4_moe_ffn": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_ffn_mxfp4": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
@@ -155,6 +156,11 @@ def tqfx4_quantize_act(x, m, k, q, da, bsum, ws, stream=None):
 def tqfx4_gemv(blocks, n, k, q, da, bsum, y, block_sums, ws, stream=None):
     _check(lib().tqfx4_gemv(_p(blocks), n, k, _p(q), _p(da), _p(bsum), _p(y), _p(block_sums), _p(ws),
                             _nbytes(ws), _s(stream)), "tqfx4_gemv")
+
+
+def tqfx4_gemv_x(blocks, n, k, x, y, q, da, bsum, ws, stream=None):
+    _check(lib().tqfx4_gemv_x(_p(blocks), n, k, _p(x), _p(y), _p(q), _p(da), _p(bsum), _p(ws), _nbytes(ws),
+                              _s(stream)), "tqfx4_gemv_x")
 
 
 # ---------------------------------------------------------------- MoE

@@ -138,6 +138,27 @@ tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
     return ok();
 }
 
+tqfx4_status tqfx4_gemv_x(const void *blocks, int64_t n, int64_t k, const float *x, float *y, int8_t *q, float *da,
+                          int32_t *bsum, void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
+    const char *fn = "tqfx4_gemv_x";
+    tqfx4_status s = check_nk(n, k, fn);
+    if (s) return s;
+    if (k == 0 || k % 512 || k > TQFX4_MAX_K)
+        return fail(TQFX4_ESHAPE, "%s: k=%lld must be a multiple of 512 in 512..%d", fn, (long long)k, TQFX4_MAX_K);
+    if ((s = check_ws(ws, ws_bytes, TQFX4_STATUS_BYTES, fn))) return s;
+    if (n == 0) return ok();
+    if (!blocks || !x || !y) return fail(TQFX4_EINVAL, "%s: NULL input or output", fn);
+    if ((q == nullptr) != (da == nullptr) || (q == nullptr) != (bsum == nullptr))
+        return fail(TQFX4_EINVAL, "%s: q, da and bsum all or none", fn);
+    if (!aligned(blocks, 16) || !aligned(x, 16) || !aligned(y, 4) || !aligned(q, 16) || !aligned(da, 4) ||
+        !aligned(bsum, 4))
+        return fail(TQFX4_EALIGN, "%s: blocks, x and q must be 16-byte aligned", fn);
+    cudaError_t e = tq::launch_gemv_x(blocks, n, k, x, q, da, bsum, y, static_cast<int *>(ws),
+                                      static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
 
 int64_t tqfx4_free_bytes(int64_t n, int64_t k) { return tq::free_bytes(n, k); }
 

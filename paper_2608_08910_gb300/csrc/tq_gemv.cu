@@ -110,13 +110,19 @@ __device__ __forceinline__ void fx_row2_dot(const uint2 *codes, const uint4 *qv,
     S1 = lo[1] + (hi[1] >> 4) - 4 * bsum;
 }
 
-template <bool kSums>
+// kFromX: the activation is the fp32 vector x, quantized per 256-block by
+// each CTA into its shared memory with the quantizer of tqfx4_quantize_act
+// (CTA 0 also writes q, da and bsum where given); otherwise it is the
+// quantized vector (q, da, bsum).
+template <bool kSums, bool kFromX>
 __global__ void __launch_bounds__(FX_WARPS * 32) gemv_chunk_kernel(const uint8_t *__restrict__ blocks, FxGeo g,
                                                                    const int8_t *__restrict__ q,
                                                                    const float *__restrict__ da,
                                                                    const int32_t *__restrict__ bsum,
                                                                    float *__restrict__ y,
-                                                                   int32_t *__restrict__ s_out, int *status) {
+                                                                   int32_t *__restrict__ s_out, int *status,
+                                                                   const float *__restrict__ x, int8_t *q_out,
+                                                                   float *da_out, int32_t *bsum_out) {
     extern __shared__ __align__(128) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int L = g.L, C = g.C, Q = g.Q;
@@ -156,13 +162,42 @@ __global__ void __launch_bounds__(FX_WARPS * 32) gemv_chunk_kernel(const uint8_t
     };
     if (units > 0) issue_next(0);
     if (units > 1) issue_next(1);
-    for (int idx = threadIdx.x; idx < 16 * L; idx += blockDim.x) {
-        const int b = idx % L, wd = idx / L;
-        qv[idx] = __ldg(reinterpret_cast<const uint4 *>(q + b * QK + 16 * wd));
-    }
-    for (int i = threadIdx.x; i < L; i += blockDim.x) {
-        das[i] = __ldg(da + i);
-        bss[i] = __ldg(bsum + i);
+    if constexpr (kFromX) {
+        // one warp per 256-block while the first copies fly; lane l's eight
+        // codes are bytes 8 l .. 8 l + 7 of the block: half l % 2 of word l / 2
+        bool finite = true;
+        for (int b = warp; b < L; b += FX_WARPS) {
+            const float4 *src = reinterpret_cast<const float4 *>(x + b * QK + 8 * lane);
+            const float4 v0 = __ldg(src), v1 = __ldg(src + 1);
+            const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+            uint2 packed;
+            float d;
+            int sum;
+            finite &= quant_block_warp(v, packed, d, sum);
+            reinterpret_cast<uint2 *>(qv + (lane >> 1) * L + b)[lane & 1] = packed;
+            if (lane == 0) {
+                das[b] = d;
+                bss[b] = sum;
+            }
+            if (blockIdx.x == 0 && q_out) {
+                *reinterpret_cast<uint2 *>(q_out + b * QK + 8 * lane) = packed;
+                if (lane == 0) {
+                    da_out[b] = d;
+                    bsum_out[b] = sum;
+                }
+            }
+        }
+        if (!finite && blockIdx.x == 0 && lane == 0) report(status, TQFX4_EDATA, K_QUANT, -1);
+        __syncwarp();
+    } else {
+        for (int idx = threadIdx.x; idx < 16 * L; idx += blockDim.x) {
+            const int b = idx % L, wd = idx / L;
+            qv[idx] = __ldg(reinterpret_cast<const uint4 *>(q + b * QK + 16 * wd));
+        }
+        for (int i = threadIdx.x; i < L; i += blockDim.x) {
+            das[i] = __ldg(da + i);
+            bss[i] = __ldg(bsum + i);
+        }
     }
     __syncthreads();
 
@@ -307,8 +342,8 @@ cudaError_t launch_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
         const int smem = fx_act_bytes(f.L) + FX_WARPS * fx_warp_bytes(f);
         static unsigned char set[2][64];
         const bool sums = block_sums != nullptr;
-        const void *fn = sums ? reinterpret_cast<const void *>(gemv_chunk_kernel<true>)
-                              : reinterpret_cast<const void *>(gemv_chunk_kernel<false>);
+        const void *fn = sums ? reinterpret_cast<const void *>(gemv_chunk_kernel<true, false>)
+                              : reinterpret_cast<const void *>(gemv_chunk_kernel<false, false>);
         cudaError_t e = allow_max_smem(fn, set[sums ? 1 : 0]);
         if (e != cudaSuccess) return e;
         if (smem > max_smem_optin()) return cudaErrorInvalidValue;
@@ -319,9 +354,15 @@ cudaError_t launch_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
         if (grid > cap) grid = cap;
         const uint8_t *b = static_cast<const uint8_t *>(blocks);
         const dim3 gd(static_cast<unsigned>(grid)), bd(FX_WARPS * 32);
-        if (sums) return launch_dependent(gemv_chunk_kernel<true>, gd, bd, smem, st, b, f, q, da, bsum, y, block_sums, status);
-        return launch_dependent(gemv_chunk_kernel<false>, gd, bd, smem, st, b, f, q, da, bsum, y,
-                                static_cast<int32_t *>(nullptr), status);
+        const float *nx = nullptr;
+        int8_t *nq = nullptr;
+        float *nd = nullptr;
+        int32_t *ns = nullptr;
+        if (sums)
+            return launch_dependent(gemv_chunk_kernel<true, false>, gd, bd, smem, st, b, f, q, da, bsum, y, block_sums,
+                                    status, nx, nq, nd, ns);
+        return launch_dependent(gemv_chunk_kernel<false, false>, gd, bd, smem, st, b, f, q, da, bsum, y,
+                                static_cast<int32_t *>(nullptr), status, nx, nq, nd, ns);
     }
     const GemvGeom g = gemv_geom(n, k);
     const int smem = gemv_act_bytes(g.nb) + g.warps * stream_warp_bytes(g.stages, g.slot_bytes, g.rpu, g.nb);
@@ -331,6 +372,34 @@ cudaError_t launch_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
     const int grid = static_cast<int>((g.n_rg + g.rg_per_cta - 1) / g.rg_per_cta);
     return launch_dependent(gemv_kernel, dim3(grid), dim3(g.warps * 32), smem, st, static_cast<const uint8_t *>(blocks),
                             g, q, da, bsum, y, block_sums, status);
+}
+
+// The chunked pass with the activation quantized inside (kFromX): k a
+// multiple of 512 (the caller checks).
+cudaError_t launch_gemv_x(const void *blocks, int64_t n, int64_t k, const float *x, int8_t *q, float *da,
+                          int32_t *bsum, float *y, int *status, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    FxGeo f{};
+    f.n = n;
+    f.L = static_cast<int>(k / QK);
+    f.C = f.L < FX_CHUNK ? f.L : FX_CHUNK;
+    f.Q = (f.L + f.C - 1) / f.C;
+    const int smem = fx_act_bytes(f.L) + FX_WARPS * fx_warp_bytes(f);
+    static unsigned char set[64];
+    cudaError_t e = allow_max_smem(reinterpret_cast<const void *>(gemv_chunk_kernel<false, true>), set);
+    if (e != cudaSuccess) return e;
+    if (smem > max_smem_optin()) return cudaErrorInvalidValue;
+    const int64_t groups = n / ROWS;
+    const int64_t per_sm = max_smem_optin() / (smem + 1024);
+    int64_t grid = (groups + FX_WARPS - 1) / FX_WARPS;
+    const int64_t cap = static_cast<int64_t>(num_sms()) * (per_sm > 0 ? per_sm : 1);
+    if (grid > cap) grid = cap;
+    const int8_t *nq = nullptr;
+    const float *nd = nullptr;
+    const int32_t *ns = nullptr;
+    return launch_dependent(gemv_chunk_kernel<false, true>, dim3(static_cast<unsigned>(grid)), dim3(FX_WARPS * 32),
+                            smem, st, static_cast<const uint8_t *>(blocks), f, nq, nd, ns, y,
+                            static_cast<int32_t *>(nullptr), status, x, q, da, bsum);
 }
 
 }  // namespace tq

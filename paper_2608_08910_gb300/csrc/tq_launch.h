@@ -17,6 +17,8 @@ cudaError_t launch_pack(int src, const void *a, const int8_t *t2, const uint16_t
                         void *blocks, int *status, cudaStream_t st);
 cudaError_t launch_quantize(const float *x, int64_t m, int64_t k, int8_t *q, float *da, int32_t *bsum,
                             int *status, cudaStream_t st);
+cudaError_t launch_gemv_x(const void *blocks, int64_t n, int64_t k, const float *x, int8_t *q, float *da,
+                          int32_t *bsum, float *y, int *status, cudaStream_t st);
 cudaError_t launch_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *q, const float *da,
                         const int32_t *bsum, float *y, int32_t *block_sums, int *status, cudaStream_t st);
 

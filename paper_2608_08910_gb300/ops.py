@@ -61,6 +61,19 @@ def gemv(blocks, n: int, k: int, q, da, bsum, ws, block_sums: bool = False):
     return (y, S) if block_sums else y
 
 
+def gemv_x(blocks, n: int, k: int, x, ws, quantized: bool = False):
+    """y = W x for an fp32 x, quantized inside the same launch; with
+    quantized=True also returns the quantized vector (q, da, bsum)."""
+    y = torch.empty(n, dtype=torch.float32, device=blocks.device)
+    q = da = bsum = None
+    if quantized:
+        q = torch.empty(k, dtype=torch.int8, device=blocks.device)
+        da = torch.empty(k // 256, dtype=torch.float32, device=blocks.device)
+        bsum = torch.empty(k // 256, dtype=torch.int32, device=blocks.device)
+    B.tqfx4_gemv_x(blocks, n, k, x, y, q, da, bsum, ws)
+    return (y, q, da, bsum) if quantized else y
+
+
 def gemv_mxfp4(blocks, n: int, k: int, q, da, ws, block_sums: bool = False):
     """y = W x for W in MXFP4 blocks (17 bytes per 32 elements) and x
     quantized by quantize_act."""

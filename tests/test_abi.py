@@ -98,6 +98,10 @@ def test_host_validation_rejects_bad_arguments(lib):
     assert lib.tqfx4_gemv(None, 1024, 1000, None, None, None, None, None, None, 0, None) == 2
     assert lib.tqfx4_gemv(None, 1024, 1024, None, None, None, None, None, None, 0, None) == 1
     assert lib.tqfx4_quantize_act(None, 1, 100, None, None, None, None, 0, None) == 2
+    # the one-launch GEMV takes the chunked pass only: k a multiple of 512
+    assert lib.tqfx4_gemv_x(None, 1024, 256, None, None, None, None, None, None, 0, None) == 2
+    assert lib.tqfx4_gemv_x(None, 1024, 1280, None, None, None, None, None, None, 0, None) == 2
+    assert lib.tqfx4_gemv_x(None, 1024, 1024, None, None, None, None, None, None, 0, None) == 1
     assert lib.tqfx4_pack(7, None, None, None, 4, 256, None, None, 0, None) == 1  # unknown source kind
     ex, rt = shapes()
     assert lib.tqfx4_moe_ffn(C.byref(ex), C.byref(rt), None, None, None, None, None, 0, None) == 1

@@ -210,3 +210,54 @@ def test_gemv_1024_benchmark_inputs(ws):
     assert np.array_equal(S.cpu().numpy(), rS)
     assert np.array_equal(y.cpu().numpy().view(np.uint32), ry.view(np.uint32))
     assert rel_err(y.cpu().numpy(), ry) <= FP32_TOL
+
+
+# the one-launch GEMV (quantization inside): shapes of the chunked pass with
+# ragged row counts, 2 to 64 blocks a row, more row groups than warps
+SHAPES_X = [(4, 512), (1024, 1024), (260, 4096), (2048, 4096), (4096, 2048), (12, 8192), (1204, 512),
+            (8, 16384), (16388, 1024)]
+
+
+@pytest.mark.parametrize("n,k", SHAPES_X)
+def test_gemv_x_equals_quantize_then_gemv(n, k, ws):
+    w = _w(n, k, 3 * n + k)
+    x = inputs.hidden_states(n + k, 1, k)[0].to(DEV)
+    blocks = ops.pack_rtn(w.to(DEV), ws)
+    q, da, bs = ops.quantize_act(x, ws)
+    y = ops.gemv(blocks, n, k, q, da, bs, ws)
+    y2, q2, da2, bs2 = ops.gemv_x(blocks, n, k, x, ws, quantized=True)
+    y3 = ops.gemv_x(blocks, n, k, x, ws)
+    B.tqfx4_check(ws)
+    assert torch.equal(q2, q) and torch.equal(bs2, bs)
+    assert torch.equal(da2.view(torch.int32), da.view(torch.int32))
+    assert torch.equal(y2.view(torch.int32), y.view(torch.int32))
+    assert torch.equal(y3.view(torch.int32), y.view(torch.int32))
+
+
+def test_gemv_x_1024_benchmark_inputs(ws):
+    # the single-GEMV workload in one launch, against the oracle
+    n = k = 1024
+    w = inputs.gemv_matrix(0, n, k)
+    x = inputs.hidden_states(0, 1, k)[0]
+    rb = oracle.pack_rtn(w.numpy())
+    rq, rda, rbs = oracle.quantize_act(x.numpy())
+    ry, _ = oracle.gemv(rb, n, k, rq, rda)
+    blocks = ops.pack_rtn(w.to(DEV), ws)
+    y, q, da, bs = ops.gemv_x(blocks, n, k, x.to(DEV), ws, quantized=True)
+    B.tqfx4_check(ws)
+    assert np.array_equal(q.cpu().numpy(), rq.reshape(-1))
+    assert np.array_equal(da.cpu().numpy().view(np.uint32), rda.reshape(-1).view(np.uint32))
+    assert np.array_equal(bs.cpu().numpy(), rbs.reshape(-1))
+    assert np.array_equal(y.cpu().numpy().view(np.uint32), ry.view(np.uint32))
+    assert rel_err(y.cpu().numpy(), ry) <= FP32_TOL
+
+
+def test_gemv_x_reports_nonfinite_activation(ws):
+    n, k = 64, 1024
+    blocks = ops.pack_rtn(_w(n, k, 1).to(DEV), ws)
+    x = inputs.hidden_states(1, 1, k)[0]
+    x[700] = float("inf")
+    ops.gemv_x(blocks, n, k, x.to(DEV), ws)
+    with pytest.raises(B.TqfxError) as e:
+        B.tqfx4_check(ws)
+    assert e.value.status == 7
