@@ -732,9 +732,9 @@ def run_small(args, rank, world, local):
       tqfx4_gemv_x (the quantization and the GEMV in one launch); 505
       matrices (269 MB) rotated.
     expert_ffn: one SwiGLU expert, gate/up 4096 -> 2048, down 2048 -> 4096,
-      Student-t(5) x 0.02 weights: tqfx4_moe_ffn on a one-expert layer (its
-      router is a single 4096-element logit, its weight 1); 21 such experts
-      (268 MB) rotated.
+      Student-t(5) x 0.02 weights: tqfx4_expert_ffn (the expert alone, no
+      router: gate/up with the quantization of x inside, then down); 21
+      such experts (268 MB) rotated.
     Metric: effective GB/s of the matrices' blocks over the step time. The
     same steps on one resident matrix (hot L2) are reported beside it."""
     import torch
@@ -783,21 +783,18 @@ def run_small(args, rank, world, local):
         M = (SMALL_POOL_BYTES + mat - 1) // mat
         layers = [MoeLayer.synthetic(SEED + m, 1, Hh, Ii, 1, 0.0, dev) for m in range(M)]
         torch.cuda.empty_cache()
-        ws = layers[0].workspace(1)
+        ws = layers[0].expert_workspace()
         X = inputs.hidden_states(SEED + rank, xpool, Hh, dev)
         out = torch.empty(Hh, device=dev)
-        sel = torch.empty(1, dtype=torch.int32, device=dev)
-        selw = torch.empty(1, device=dev)
         step_bytes = mat
-        n_st = B.tqfx4_moe_stage_count(0, 0)
 
         def step(i, st=stream, hot=False, ev=None, x=None):
             L = layers[0 if hot else i % M]
-            L.ffn(X[i % xpool] if x is None else x, ws, out, sel, selw, stream=st, events=ev)
-        launches = n_st
+            L.expert_ffn(0, X[i % xpool] if x is None else x, ws, out, stream=st, events=ev)
+        launches = 2
         kern = "gate_up"
         cfg = {"workload": "expert_ffn_h4096_i2048", "hidden": Hh, "inter": Ii, "expert_bytes": mat,
-               "pool_experts": M, "router": "one expert (a single 4096-element logit, weight 1)",
+               "pool_experts": M, "call": "tqfx4_expert_ffn (no router)",
                "l2": "inputs larger than L2: %d distinct experts (%d MB) rotated, a new activation per step"
                      % (M, M * mat >> 20)}
 
@@ -871,8 +868,8 @@ def run_small(args, rank, world, local):
         names = ["gemv_x"]
         dom_s, dom_bytes = stage[0], mat
     else:
-        names = [B.tqfx4_moe_stage_name(0, 0, s) for s in range(launches)]
-        dom_s, dom_bytes = stage[1], 2 * B.tqfx4_matrix_bytes(I, H)
+        names = ["gate_up", "down"]
+        dom_s, dom_bytes = stage[0], 2 * B.tqfx4_matrix_bytes(I, H)
     stage_us = {names[s]: stage[s] * 1e6 for s in range(len(names))}
 
     # end to end through the public API: x from pinned host memory, y (out)

@@ -390,6 +390,31 @@ tqfx4_status tqfx4_moe_ffn_noalloc(const tqfx4_experts *ex, const tqfx4_router *
                                    void *stream);
 
 /*
+ * tqfx4_expert_ffn -- one expert's SwiGLU FFN for one token (Sec. 1 and
+ * 2.2; the expert FFN of tqfx4_moe_ffn, without a router): g = W_gate x and
+ * u = W_up x through the integer dot pass with x quantized per 256-block,
+ * h = silu(g) u quantized per 256-block, out = W_down h. The output, and
+ * the intermediates left in the workspace, are bit for bit those of
+ * tqfx4_moe_ffn on a one-expert layer (whose routing weight is 1).
+ *   gate, up: inter x hidden matrices; down: hidden x inter (device,
+ *   16-byte aligned, tqfx4_matrix_bytes each). x: fp32 [hidden] (device,
+ *   16-byte aligned); out: fp32 [hidden] (device).
+ *   ws: at least tqfx4_expert_ffn_workspace_bytes(hidden, inter) bytes,
+ *   zeroed once before its first use (0 for invalid shapes: hidden and
+ *   inter positive multiples of 256 up to TQFX4_MAX_K). Two launches
+ *   (gate/up with the quantization of x inside, then down); a non-finite x
+ *   or h sets TQFX4_EDATA. tqfx4_expert_ffn_traced records events[0..2]
+ *   before, between and after the two (stages "gate_up", "down").
+ */
+size_t tqfx4_expert_ffn_workspace_bytes(int64_t hidden, int64_t inter);
+tqfx4_status tqfx4_expert_ffn(const void *gate, const void *up, const void *down,
+                              int64_t hidden, int64_t inter, const float *x, float *out,
+                              void *ws, size_t ws_bytes, void *stream);
+tqfx4_status tqfx4_expert_ffn_traced(const void *gate, const void *up, const void *down,
+                                     int64_t hidden, int64_t inter, const float *x, float *out,
+                                     void *ws, size_t ws_bytes, void *stream, void *const *events);
+
+/*
  * Profiling variants: identical to the calls above, and additionally record
  * `events[i]` (cudaEvent_t, created by the caller) on the stream before
  * stage i, and events[n_stages] after the last stage, where n_stages is

@@ -60,6 +60,9 @@ _SIGS = {
     "tqfx4_quantize_act": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_gemv": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_gemv_x": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_expert_ffn_workspace_bytes": (_sz, [_i64, _i64]),
+    "tqfx4_expert_ffn": (_int, [_vp, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_expert_ffn_traced": (_int, [_vp, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp, _vp]),
     "tqfx4_moe_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int]),
     "tqfx4_moe_ffn": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_ffn_mxfp4": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
@@ -156,6 +159,21 @@ def tqfx4_quantize_act(x, m, k, q, da, bsum, ws, stream=None):
 def tqfx4_gemv(blocks, n, k, q, da, bsum, y, block_sums, ws, stream=None):
     _check(lib().tqfx4_gemv(_p(blocks), n, k, _p(q), _p(da), _p(bsum), _p(y), _p(block_sums), _p(ws),
                             _nbytes(ws), _s(stream)), "tqfx4_gemv")
+
+
+def tqfx4_expert_ffn_workspace_bytes(hidden, inter):
+    return lib().tqfx4_expert_ffn_workspace_bytes(hidden, inter)
+
+
+def tqfx4_expert_ffn(gate, up, down, hidden, inter, x, out, ws, stream=None, events=None):
+    if events is None:
+        rc = lib().tqfx4_expert_ffn(_p(gate), _p(up), _p(down), hidden, inter, _p(x), _p(out), _p(ws), _nbytes(ws),
+                                    _s(stream))
+    else:
+        arr = (_vp * len(events))(*[e.cuda_event if hasattr(e, "cuda_event") else e for e in events])
+        rc = lib().tqfx4_expert_ffn_traced(_p(gate), _p(up), _p(down), hidden, inter, _p(x), _p(out), _p(ws),
+                                           _nbytes(ws), _s(stream), arr)
+    _check(rc, "tqfx4_expert_ffn")
 
 
 def tqfx4_gemv_x(blocks, n, k, x, y, q, da, bsum, ws, stream=None):

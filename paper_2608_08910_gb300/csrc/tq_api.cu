@@ -313,6 +313,50 @@ tqfx4_status tqfx4_moe_ffn_traced(const tqfx4_experts *ex, const tqfx4_router *r
     return moe_ffn_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, events);
 }
 
+size_t tqfx4_expert_ffn_workspace_bytes(int64_t hidden, int64_t inter) {
+    if (hidden <= 0 || inter <= 0 || hidden % 256 || inter % 256 || hidden > TQFX4_MAX_K || inter > TQFX4_MAX_K)
+        return 0;
+    return tq::moe_layout(1, hidden, inter, 1, 1, false, true).total;
+}
+
+static tqfx4_status expert_ffn_impl(const void *gate, const void *up, const void *down, int64_t hidden,
+                                    int64_t inter, const float *x, float *out, void *ws, size_t ws_bytes,
+                                    void *stream, void *const *events) {
+    const char *fn = "tqfx4_expert_ffn";
+    const tqfx4_experts ex{gate, up, down, 1, hidden, inter};
+    tqfx4_router rt{};
+    rt.top_k = 1;
+    tqfx4_status s = check_moe_shapes(&ex, &rt, fn);
+    if (s) return s;
+    if (!gate || !up || !down || !x || !out) return fail(TQFX4_EINVAL, "%s: NULL matrix, input or output", fn);
+    if (!aligned(gate, 16) || !aligned(up, 16) || !aligned(down, 16) || !aligned(x, 16) || !aligned(out, 4))
+        return fail(TQFX4_EALIGN, "%s: matrices and x must be 16-byte aligned", fn);
+    tq::MoeArgs a;
+    tq::MoeLayout L;
+    if (!tq::moe_decode_args(&ex, &rt, nullptr, a, L))
+        return fail(TQFX4_ESHAPE, "%s: too many row ranges for the counter area", fn);
+    if ((s = check_ws(ws, ws_bytes, L.total, fn))) return s;
+    if (tq::gate_up_smem(a) > tq::max_smem_optin() || tq::down_smem(a) > tq::max_smem_optin())
+        return fail(TQFX4_ESHAPE, "%s: inter too large for the decode kernels' shared memory", fn);
+    tq::moe_decode_args(&ex, &rt, ws, a, L);
+    cudaError_t e = tq::launch_expert_ffn(a, x, out, static_cast<cudaStream_t>(stream), events);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
+tqfx4_status tqfx4_expert_ffn(const void *gate, const void *up, const void *down, int64_t hidden, int64_t inter,
+                              const float *x, float *out, void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
+    return expert_ffn_impl(gate, up, down, hidden, inter, x, out, ws, ws_bytes, stream, nullptr);
+}
+
+tqfx4_status tqfx4_expert_ffn_traced(const void *gate, const void *up, const void *down, int64_t hidden,
+                                     int64_t inter, const float *x, float *out, void *ws, size_t ws_bytes,
+                                     void *stream, void *const *events) {
+    TQ_RANGE();
+    return expert_ffn_impl(gate, up, down, hidden, inter, x, out, ws, ws_bytes, stream, events);
+}
+
 tqfx4_status tqfx4_moe_route(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, int32_t *sel_idx,
                              float *sel_w, void *ws, size_t ws_bytes, void *stream) {
     TQ_RANGE();

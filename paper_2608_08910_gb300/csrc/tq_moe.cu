@@ -115,7 +115,7 @@ __global__ void __launch_bounds__(128) router_kernel(MoeArgs a) {
 __global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     TQ_STAMP(1, 0);
-    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nbh = a.nbh;
     __shared__ int sel_s[TQFX4_MAX_TOP_K];
     __shared__ const uint8_t *ptr_s[2 * TQFX4_MAX_TOP_K];
@@ -133,8 +133,8 @@ __global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
     // issue the activation loads first: weight copies issued before them
     // would queue ahead in the memory system
     ActRegs act;
-    act_load(a.qx, a.dx, a.bx, nbh, act);
-    if (threadIdx.x < a.top_k) sel_s[threadIdx.x] = __ldcg(a.sel + threadIdx.x);
+    if (!a.single) act_load(a.qx, a.dx, a.bx, nbh, act);
+    if (threadIdx.x < a.top_k) sel_s[threadIdx.x] = a.single ? 0 : __ldcg(a.sel + threadIdx.x);
     if (a.ptrs && threadIdx.x < 2 * a.top_k) ptr_s[threadIdx.x] = a.ptrs[threadIdx.x];
     __syncthreads();
     const int64_t n_rg = a.I / 4;
@@ -163,7 +163,37 @@ __global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
     };
     int64_t slot_u[kMaxStages];
     warp_units_prefetch(ring, q, nbh, map, slot_u);
-    act_store(act, nbh, qs, das, bss);
+    if (a.single) {
+        // x quantized here while the first copies fly (the quantizer of
+        // tqfx4_quantize_act, one warp per 256-block); CTA 0 keeps it in the
+        // workspace for inspection
+        bool finite = true;
+        for (int b = warp; b < nbh; b += a.warps_gu) {
+            const float4 *src = reinterpret_cast<const float4 *>(a.x + b * QK + 8 * lane);
+            const float4 v0 = __ldg(src), v1 = __ldg(src + 1);
+            const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+            uint2 packed;
+            float d;
+            int sum;
+            finite &= quant_block_warp(v, packed, d, sum);
+            *reinterpret_cast<uint2 *>(qs + b * QS_STRIDE + 8 * lane) = packed;
+            if (lane == 0) {
+                das[b] = d;
+                bss[b] = sum;
+            }
+            if (blockIdx.x == 0) {
+                *reinterpret_cast<uint2 *>(a.qx + b * QK + 8 * lane) = packed;
+                if (lane == 0) {
+                    a.dx[b] = d;
+                    a.bx[b] = sum;
+                }
+            }
+        }
+        if (!finite && blockIdx.x == 0 && lane == 0) report(a.status, TQFX4_EDATA, K_GATEUP, -1);
+        __syncwarp();
+    } else {
+        act_store(act, nbh, qs, das, bss);
+    }
     __syncthreads();
     TQ_STAMP(1, 2);
     warp_units_run(ring, q, nbh, qs, das, bss, map, [](int64_t) {}, slot_u, a.status, K_GATEUP);
@@ -188,7 +218,7 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
     ring_init(ring);
     fence_barrier_init();
     const int j = blockIdx.x / a.parts_d, p = blockIdx.x - j * a.parts_d;
-    const int64_t e = a.ptrs ? 0 : __ldcg(a.sel + j);
+    const int64_t e = (a.ptrs || a.single) ? 0 : __ldcg(a.sel + j);
     const int64_t n_rg = a.H / 4;
     MatJob job;
     job.mat = a.ptrs ? a.ptrs[2 * K + j] : a.down + e * a.mb_d;
@@ -202,7 +232,9 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
     job.nb = nbi;
     const bool any = job.rg_begin < job.rg_end;
     if (any) warp_stream_prefetch(ring, job, a.rpu_d, warp, a.warps_d, 1);
-    if (warp == a.warps_d - 1) {
+    if (a.single) {
+        if (threadIdx.x == 0) selw_s[0] = 1.0f;  // the one expert's weight
+    } else if (warp == a.warps_d - 1) {
         // the routing weights (needed by the combine at the end); the router
         // has completed, so this runs while gate/up drains
         int sel_l[TQFX4_MAX_TOP_K];
@@ -216,7 +248,10 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
     TQ_STAMP(2, 1);
     grid_dependency_wait();  // g and u of the gate/up kernel
     TQ_STAMP(2, 2);
-    if (blockIdx.x == 0 && threadIdx.x == 0) a.ctr[kCtrRouter] = 0;  // for the next call
+    if (blockIdx.x == 0 && threadIdx.x == 0) {  // for the next call
+        a.ctr[kCtrRouter] = 0;
+        if (a.single) a.ctr[kCtrGateUp] = 0;  // no router zeroes it
+    }
     // h_j = silu(g_j) u_j and its int8 quantization, one 256-block per warp;
     // the g/u loads go out before the rest of the weight prefetch
     const float *gj = a.g + static_cast<int64_t>(j) * a.I;
@@ -429,6 +464,40 @@ cudaError_t launch_moe_route(const MoeArgs &a0, const float *x, int32_t *sel_idx
     a.route_only = 1;
     router_kernel<<<a.E + (a.nbh + 3) / 4, 128, 0, st>>>(a);
     return cudaGetLastError();
+}
+
+// One expert's FFN without a router: gate/up (x quantized inside) and down
+// as programmatic dependents, events[0..2] (optional) around the two.
+cudaError_t launch_expert_ffn(const MoeArgs &a0, const float *x, float *out, cudaStream_t st,
+                              void *const *events) {
+    MoeArgs a = a0;
+    a.x = x;
+    a.out = out;
+    a.sel_out = nullptr;
+    a.selw_out = nullptr;
+    a.single = 1;
+    static unsigned char set_gu[64], set_dn[64];
+    cudaError_t e = allow_max_smem(reinterpret_cast<const void *>(gate_up_kernel), set_gu);
+    if (e == cudaSuccess) e = allow_max_smem(reinterpret_cast<const void *>(down_kernel), set_dn);
+    if (e != cudaSuccess) return e;
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (events) cudaStreamIsCapturing(st, &cap);
+    auto rec = [&](int i) {
+        if (events && events[i])
+            cudaEventRecordWithFlags(static_cast<cudaEvent_t>(events[i]), st,
+                                     cap == cudaStreamCaptureStatusActive ? cudaEventRecordExternal
+                                                                          : cudaEventRecordDefault);
+    };
+    rec(0);
+    if ((e = launch_pdl(reinterpret_cast<const void *>(gate_up_kernel), a.top_k * a.parts_gu, a.warps_gu * 32,
+                        gate_up_smem(a), st, events != nullptr, a)) != cudaSuccess)
+        return e;
+    rec(1);
+    if ((e = launch_pdl(reinterpret_cast<const void *>(down_kernel), a.top_k * a.parts_d, a.warps_d * 32,
+                        down_smem(a), st, events != nullptr, a)) != cudaSuccess)
+        return e;
+    rec(2);
+    return cudaSuccess;
 }
 
 cudaError_t launch_moe_experts(const MoeArgs &a0, const void *const *ptrs, float *out, cudaStream_t st) {

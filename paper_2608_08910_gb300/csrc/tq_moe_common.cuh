@@ -147,6 +147,10 @@ struct MoeArgs {
     // for the stacked layout (base + expert * matrix bytes)
     const uint8_t *const *ptrs;
     int route_only;  // the router also forms the routing weights, and no expert kernels follow
+    // one expert's FFN without a router (tqfx4_expert_ffn): the expert is
+    // expert 0 of the stacked matrices, its weight 1; gate/up quantizes x
+    // itself and down resets gate/up's unit counter for the next call
+    int single;
 };
 
 // Arguments of the grouped (T-token) kernels.

@@ -76,6 +76,22 @@ class MoeLayer:
             raise ValueError("invalid MoE shapes")
         return torch.zeros(((n + 255) // 256) * 256, dtype=torch.uint8, device=self.gate.device)
 
+    def expert_workspace(self) -> torch.Tensor:
+        """A zeroed workspace for expert_ffn."""
+        n = B.tqfx4_expert_ffn_workspace_bytes(self.hidden, self.inter)
+        if n == 0:
+            raise ValueError("invalid expert shapes")
+        return torch.zeros(((n + 255) // 256) * 256, dtype=torch.uint8, device=self.gate.device)
+
+    def expert_ffn(self, e: int, x, ws, out=None, stream=None, events=None):
+        """Expert e's SwiGLU FFN alone (tqfx4_expert_ffn: no router, weight 1)."""
+        if self.fmt != "fx4":
+            raise ValueError("expert_ffn serves tq2_0_fx4 experts")
+        out = torch.empty(self.hidden, dtype=torch.float32, device=x.device) if out is None else out
+        g, u, d = self.expert_blocks(e)
+        B.tqfx4_expert_ffn(g, u, d, self.hidden, self.inter, x, out, ws, stream, events)
+        return out
+
     def ffn(self, x, ws, out=None, sel_idx=None, sel_w=None, stream=None, events=None):
         dev = x.device
         out = torch.empty(self.hidden, dtype=torch.float32, device=dev) if out is None else out

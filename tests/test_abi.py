@@ -98,6 +98,13 @@ def test_host_validation_rejects_bad_arguments(lib):
     assert lib.tqfx4_gemv(None, 1024, 1000, None, None, None, None, None, None, 0, None) == 2
     assert lib.tqfx4_gemv(None, 1024, 1024, None, None, None, None, None, None, 0, None) == 1
     assert lib.tqfx4_quantize_act(None, 1, 100, None, None, None, None, 0, None) == 2
+    # the expert FFN's workspace: the one-expert, top-1 decode layout (at most
+    # the MoE call's, which also covers the grouped layout); 0 for bad shapes
+    ex1, rt1 = shapes(E=1, k=1)
+    n1 = lib.tqfx4_expert_ffn_workspace_bytes(4096, 2048)
+    assert 0 < n1 <= lib.tqfx4_moe_workspace_bytes(C.byref(ex1), C.byref(rt1), 1, 0)
+    assert lib.tqfx4_expert_ffn_workspace_bytes(4000, 2048) == 0
+    assert lib.tqfx4_expert_ffn_workspace_bytes(4096, 0) == 0
     # the one-launch GEMV takes the chunked pass only: k a multiple of 512
     assert lib.tqfx4_gemv_x(None, 1024, 256, None, None, None, None, None, None, 0, None) == 2
     assert lib.tqfx4_gemv_x(None, 1024, 1280, None, None, None, None, None, None, 0, None) == 2

@@ -165,3 +165,54 @@ def test_moe_argument_errors(full_layer):
     with pytest.raises(B.TqfxError) as e:
         full_layer.ffn(x[1:], ws)
     assert e.value.status == 3
+
+
+def test_expert_ffn_equals_the_one_expert_layer():
+    # tqfx4_expert_ffn (no router) against tqfx4_moe_ffn on the same expert as
+    # a one-expert layer, and against the oracle: output and intermediates
+    layer = MoeLayer.synthetic(2, 1, 4096, 2048, 1, 0.0, DEV)
+    X = inputs.hidden_states(2, 3, 4096)
+    ws_moe = layer.workspace(1)
+    ws_exp = layer.expert_workspace()
+    ex = oracle_experts(2, [0], 4096, 2048)
+    for t in range(3):
+        x = X[t].to(DEV)
+        out_moe = layer.ffn(x, ws_moe)[0].clone()
+        out_exp = layer.expert_ffn(0, x, ws_exp)
+        B.tqfx4_check(ws_moe)
+        B.tqfx4_check(ws_exp)
+        assert torch.equal(out_exp.view(torch.int32), out_moe.view(torch.int32))
+        for name, dt, shape in (("qx", torch.int8, (4096,)), ("g", torch.float32, (2048,)),
+                                ("u", torch.float32, (2048,)), ("h", torch.float32, (2048,)),
+                                ("qh", torch.int8, (2048,)), ("o", torch.float32, (4096,))):
+            a_ = layer.view(ws_moe, name, dt, shape)
+            b_ = layer.view(ws_exp, name, dt, shape)
+            assert torch.equal(a_.view(torch.uint8), b_.view(torch.uint8)), name
+        ref, _ = oracle.expert_ffn(*ex[0], 4096, 2048, X[t].numpy())
+        assert np.array_equal(out_exp.cpu().numpy().view(np.uint32), ref.view(np.uint32))
+
+
+@pytest.mark.parametrize("H,I", [(1024, 512), (2048, 4096), (768, 1280)])
+def test_expert_ffn_of_one_expert_of_a_layer(H, I):
+    # expert 5 of an 8-expert layer, ragged block counts, 20 calls in a row
+    # on one workspace (gate/up's unit counter is reset by every call)
+    layer = MoeLayer.synthetic(H + I, 8, H, I, 2, 0.0, DEV)
+    ws = layer.expert_workspace()
+    ex = oracle_experts(H + I, [5], H, I)
+    X = inputs.hidden_states(H, 2, H)
+    refs = [oracle.expert_ffn(*ex[5], H, I, X[t].numpy())[0] for t in range(2)]
+    for c in range(20):
+        out = layer.expert_ffn(5, X[c % 2].to(DEV), ws)
+        B.tqfx4_check(ws)
+        assert np.array_equal(out.cpu().numpy().view(np.uint32), refs[c % 2].view(np.uint32))
+
+
+def test_expert_ffn_reports_nonfinite_input():
+    layer = MoeLayer.synthetic(4, 1, 1024, 512, 1, 0.0, DEV)
+    ws = layer.expert_workspace()
+    x = inputs.hidden_states(4, 1, 1024)[0]
+    x[5] = float("nan")
+    layer.expert_ffn(0, x.to(DEV), ws)
+    with pytest.raises(B.TqfxError) as e:
+        B.tqfx4_check(ws)
+    assert e.value.status == 7
