@@ -63,7 +63,7 @@ GATE_UP_TRAFFIC = 68196864 + 982528
 # The same for one tc_gemm_kernel gate/up launch of the 2048-token prefill: an ncu capture at 64
 # experts and 512 tokens (one chunk per expert, as in the full workload) scaled by the full
 # workload's 4x weight bytes and pairs.
-TC_GATE_UP_TRAFFIC = 4 * (580448000 + 58149632)
+TC_GATE_UP_TRAFFIC = 4 * (580200448 + 58917376)
 
 
 def max_over_ranks(t, world, device):

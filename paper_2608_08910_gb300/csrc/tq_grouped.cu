@@ -698,7 +698,7 @@ __global__ void __launch_bounds__(256) planes_tok_kernel(GroupedArgs a) {
 }
 
 // CTA (c, y) handles pair columns 16 y .. 16 y + 15 of chunk c (chunks hold
-// 1..128 pairs, so a chunk is spread over several CTAs): copies the pairs'
+// 1..TC_CHUNK pairs, so a chunk is spread over several CTAs): copies the pairs'
 // plane rows from token order and writes the chunk's scale columns.
 constexpr int GT_PAIRS = 16;
 static_assert(TC_CHUNK % GT_PAIRS == 0, "whole CTAs per chunk");

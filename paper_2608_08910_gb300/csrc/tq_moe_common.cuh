@@ -40,8 +40,9 @@ constexpr int GG_TOK = 64;
 constexpr int64_t kTcMinPairs = 1;
 // Slices of the hidden dimension the router's screening GEMM sums separately.
 constexpr int kScreenSplit = 4;
-// Pairs per chunk on the tensor-core path (the largest MMA N used).
-constexpr int TC_CHUNK = 128;
+// Pairs per chunk on the tensor-core path: both activation planes of a
+// chunk side by side make the MMA's N = 2 x 96 = 192.
+constexpr int TC_CHUNK = 96;
 
 inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 

@@ -1,6 +1,6 @@
 // Grouped expert GEMM on the 5th-generation tensor cores (tcgen05), the
 // contraction of the prefill path: one work item is 128 weight rows (32 row
-// groups) of one expert times one chunk of <= 128 (token, slot) pairs of
+// groups) of one expert times one chunk of <= TC_CHUNK (token, slot) pairs of
 // that expert.
 //
 // tcgen05.mma has no integer kind on sm_103a, so the integer block sums
@@ -36,11 +36,11 @@
 //              r4 = w) and writes their codes into A, into the buffer of
 //              block b - 2 once that block's MMAs are complete;
 //   warps 4-11 epilogue. Warp w serves TMEM lanes 32 (w % 4) .. + 31 and
-//              the 32-column chunks (pairs) e and e + 2, e = (w - 4) / 4: per
-//              block it reads the accumulator (with the planes side by side:
-//              both halves, then hands the buffer back to the MMAs at once)
-//              and the running output y (kept in TMEM), adds
-//              float(S) * (d * da) and writes y back; at the end of the item
+//              the 16-column pieces (pairs) q, q + 2 and q + 4 of the chunk,
+//              q = (w - 4) / 4: per block it reads both plane halves of its
+//              pieces of the accumulator, hands the buffer back to the MMAs
+//              after its last read, and adds float(S) * (d * da) to the
+//              running outputs y, kept in registers; at the end of the item
 //              it stores y;
 //   warp 12    producer: TMA copies of the raw weight blocks (one box per
 //              two blocks of the tile), of the activation planes (one 4-D
@@ -48,15 +48,16 @@
 //              chunk's pairs rounded up to 16, times 512 bytes) and a bulk
 //              copy of the chunk's block scales;
 //   warp 13    TMEM allocation; one thread issues the MMAs (M = 128, K = 32)
-//              and two commits per block. Chunks of up to 64 pairs take one
-//              MMA of N = 128 per K-step with both planes side by side (the
-//              two 64-column halves of the accumulator are added by the
-//              epilogue, exactly); larger chunks one MMA per plane, N = the
-//              pairs rounded up to 16. Each shared-memory access the thread
-//              makes stalls its issue, and the tensor pipe with it, so it
-//              reads the abort flag only when it actually has to wait.
-// TMEM: A in columns [0, 128) (two blocks of 64), y in [128, 256),
-// accumulators in [256, 512).
+//              and two commits per block: one MMA of N = 2 x (pairs rounded up
+//              to 16) per K-step, with both planes side by side (the two halves
+//              of the accumulator are added by the epilogue, exactly). An MMA
+//              takes about the same issue time whatever N, so the chunk
+//              (TC_CHUNK pairs) is as wide as two accumulator buffers allow.
+//              Each shared-memory access the thread makes stalls its issue,
+//              and the tensor pipe with it, so it reads the abort flag only
+//              when it actually has to wait.
+// TMEM: A in columns [0, 128) (two blocks of 64), two accumulator buffers of
+// TC_DCOLS columns from column 128.
 // The epilogue uses scalar fp32 operations: the packed f32x2 forms were
 // measured to give results that differ from them.
 // Every wait is bounded. On a timeout the CTA records the error, all roles
@@ -82,11 +83,11 @@ constexpr int TC_THREADS = (TC_MATH_WARPS + 2) * 32;
 constexpr int TC_RAW_ROW = 2 * BLOCK_BYTES;    // two blocks of one row group: 1040 bytes
 constexpr int TC_RAW_BYTES = 33 * 1024;        // 32 x 1040 bytes, padded
 // B, the activation planes of a block: four regions (k-stage ks, plane pl)
-// of R rows (pairs) x 128 bytes, R = 64 for chunks of up to 64 pairs, else
-// the pairs rounded up to 16, so a block takes R * 512 bytes (32 KB for 64
-// pairs, 64 KB for 128), loaded by one 4-D TMA copy. Blocks are placed one after another in a byte ring
-// (never split at its end), which keeps more small blocks in flight than
-// fixed slots sized for 128 pairs.
+// of R rows (pairs) x 128 bytes, R = the chunk's pairs rounded up to 16, so a
+// block takes R * 512 bytes (32 KB for 64 pairs), loaded by one 4-D TMA copy.
+// Blocks are placed one after another in a byte ring (never split at its
+// end), which keeps more small blocks in flight than fixed slots sized for
+// the largest chunk.
 constexpr int TC_B_ROW = 128;                  // one pair's 128 elements of one plane
 constexpr int TC_B_RING = 144 * 1024;          // ring bytes
 constexpr int TC_B_SLOTS = 8;                  // full / empty barrier pairs: blocks in flight at most
@@ -100,15 +101,18 @@ constexpr int TC_NBAR = 11 + 2 * TC_B_SLOTS + 2 * TC_SC_STAGES + 2 * TC_DW_STAGE
 constexpr int TC_OFF_BSTART = TC_OFF_BAR + TC_NBAR * 8;  // [TC_B_SLOTS] int64: producer's ring history
 constexpr int TC_SMEM = TC_OFF_BSTART + TC_B_SLOTS * 8 + 16 + 1024;  // + TMEM address, abort flag, alignment slack
 constexpr int TC_TMEM_COLS = 512;
-constexpr uint32_t TC_TMEM_Y = 128;            // the running output y (128 columns: pairs)
-constexpr uint32_t TC_TMEM_D = 256;            // first accumulator column
+constexpr uint32_t TC_TMEM_D = 128;            // first accumulator column
+constexpr int TC_DCOLS = 192;                  // columns of one accumulator buffer
+constexpr int TC_SIDE_MAX = TC_DCOLS / 2;      // pairs up to which both planes go side by side
 constexpr int TC_A_COLS = 64;                  // TMEM columns of one block of A (256 bytes per row)
 
 static_assert(TC_OFF_B % 1024 == 0, "swizzled tiles need 1024-byte alignment");
-static_assert(TC_B_RING % 2048 == 0 && TC_B_RING >= 2 * TC_CHUNK * 4 * TC_B_ROW, "ring: two blocks of 128 pairs");
+static_assert(TC_B_RING % 2048 == 0 && TC_B_RING >= 2 * TC_CHUNK * 4 * TC_B_ROW, "ring: two blocks of a full chunk");
 static_assert(TC_SMEM <= 227 * 1024, "shared memory per CTA");
 static_assert(TC_RG * TC_RAW_ROW <= TC_RAW_BYTES, "raw stage too small");
-static_assert(TC_CHUNK == 128, "four 32-column epilogue chunks");
+static_assert(TC_CHUNK <= TC_SIDE_MAX && TC_CHUNK % 16 == 0 && TC_CHUNK / 16 <= 6,
+              "both planes side by side; at most three 16-column pieces per epilogue warp");
+static_assert(TC_TMEM_D + 2 * TC_DCOLS <= TC_TMEM_COLS, "accumulators within the allocation");
 
 // Instruction descriptor of tcgen05.mma kind::f8f6f4: D fp32 (bits 4-5 = 1),
 // A and B e4m3 (bits 7-9 = 0, 10-12 = 0), both K-major (bits 15, 16 = 0),
@@ -167,6 +171,13 @@ __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::
 // taddr .. taddr + 31.
 __device__ __forceinline__ void tc_ld32(uint32_t taddr, uint32_t (&r)[32]) {
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 " TC_LIST32 ", [%32];" : TC_W32(r) : "r"(taddr));
+}
+__device__ __forceinline__ void tc_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
 }
 __device__ __forceinline__ void tc_st32(uint32_t taddr, const uint32_t (&r)[32]) {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%32], " TC_LIST32 ";" ::TC_R32(r), "r"(taddr) : "memory");
@@ -370,11 +381,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
     // All roles walk the same items and blocks, so each keeps identical
     // counts of raw stages and blocks used so far (the ring positions).
-    int64_t nraw = 0, nblk = 0;
+    int nraw = 0, nblk = 0;  // a CTA's blocks stay far below 2^31
     BRing bring;
     // Producer: uses issued on each raw stage's full barrier, and the last
     // block of B and of scales issued (for the drain).
-    int64_t n_rf0 = 0, n_rf1 = 0, last_b = -1, last_sc = -1;
+    int n_rf0 = 0, n_rf1 = 0, last_b = -1, last_sc = -1;
     for (int64_t w = blockIdx.x; w < items; w += gridDim.x) {
         if (*reinterpret_cast<volatile int *>(abort)) break;
         const int chunk = static_cast<int>(w / per_chunk);
@@ -390,11 +401,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         const int rg0 = static_cast<int>(tl) * TC_RG;
         const int nb = J.nb;
         const int nmma = (m + 15) & ~15;          // pairs rounded up to 16
-        // Up to 64 pairs: both planes side by side in one MMA of N = 128
-        // (B rows 0..63 the high plane, 64..127 the low one; the epilogue adds
-        // the two halves of the accumulator), else one MMA per plane, N = nmma.
-        const bool side = nmma <= 64;
-        const int brows = side ? 64 : nmma;       // B rows per (k-stage, plane)
+        // Both planes side by side in one MMA of N = 2 nmma (B rows 0..nmma-1
+        // the high plane, then the low one; the epilogue adds the two halves
+        // of the accumulator, exactly).
+        const int brows = nmma;                   // B rows per (k-stage, plane)
         const int bbytes = 4 * brows * TC_B_ROW;  // one block of B
 
         if (warp == TC_MATH_WARPS) {
@@ -403,9 +413,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                 const CUtensorMap *wmap = second ? &wmap1 : &wmap0;
                 const float *sc = scales + static_cast<int64_t>(chunk) * nb * (2 * TC_CHUNK);
                 for (int b = 0; b < nb; ++b) {
-                    const int64_t bb = nblk + b;
+                    const int bb = nblk + b;
                     if ((b & 1) == 0) {
-                        const int64_t rb = nraw + b / 2;
+                        const int rb = nraw + b / 2;
                         const int rs = static_cast<int>(rb & 1);
                         if (!tc_wait(&raw_empty[rs], static_cast<uint32_t>(((rb >> 1) & 1) ^ 1), abort, a.status, 1))
                             break;
@@ -420,8 +430,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     // user of this barrier pair (in-order consumption makes
                     // the latest of them sufficient)
                     const int64_t v = bring.place(bbytes);
-                    int64_t need = bb - TC_B_SLOTS;
-                    for (int64_t j = bb - 1; j > need && j >= 0; --j)
+                    int need = bb - TC_B_SLOTS;
+                    for (int j = bb - 1; j > need && j >= 0; --j)
                         if (b_start[j % TC_B_SLOTS] < v + bbytes - TC_B_RING) {
                             need = j;
                             break;
@@ -447,13 +457,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         } else if (warp == TC_MATH_WARPS + 1) {
             // ---------------- MMA issuer ----------------
             if (lane == 0) {
-                const uint32_t idesc = tc_idesc(side ? 128 : nmma);
+                const uint32_t idesc = tc_idesc(2 * nmma);
                 // B descriptors: ring start; the others differ by constant
                 // byte offsets (>> 4) in the start-address field
                 const uint64_t bdesc0 = umma_desc(smem_u32(smem + TC_OFF_B));
                 const int region = brows * TC_B_ROW;  // one (k-stage, plane) of B
                 for (int b = 0; b < nb; ++b) {
-                    const int64_t bb = nblk + b;
+                    const int bb = nblk + b;
                     const int bs = static_cast<int>(bb & 1);
                     const int64_t v = bring.place(bbytes);
                     const int slot = static_cast<int>(bb % TC_B_SLOTS);
@@ -464,23 +474,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                                   static_cast<uint32_t>((bb / TC_B_SLOTS) & 1), abort, a.status, 4))
                         break;
                     tc_fence_after();
-                    const uint32_t d_tmem = tmem + TC_TMEM_D + bs * TC_CHUNK;
+                    const uint32_t d_tmem = tmem + TC_TMEM_D + bs * TC_DCOLS;
                     const uint32_t a_tmem = tmem + bs * TC_A_COLS;
                     const uint64_t bd = bdesc0 + static_cast<uint64_t>((v % TC_B_RING) >> 4);
-                    if (side) {
 #pragma unroll
-                        for (int kk = 0; kk < 8; ++kk)  // 32-element step: A columns 8 kk .. 8 kk + 7
-                            tc_mma_ts(d_tmem, a_tmem + 8 * kk, bd + (((kk >> 2) * 2 * region + (kk & 3) * 32) >> 4),
-                                      idesc, kk != 0 ? 1u : 0u);
-                    } else {
-#pragma unroll
-                        for (int kk = 0; kk < 8; ++kk)
-#pragma unroll
-                            for (int pl = 0; pl < 2; ++pl)
-                                tc_mma_ts(d_tmem, a_tmem + 8 * kk,
-                                          bd + ((((kk >> 2) * 2 + pl) * region + (kk & 3) * 32) >> 4), idesc,
-                                          (kk | pl) != 0 ? 1u : 0u);
-                    }
+                    for (int kk = 0; kk < 8; ++kk)  // 32-element step: A columns 8 kk .. 8 kk + 7
+                        tc_mma_ts(d_tmem, a_tmem + 8 * kk, bd + (((kk >> 2) * 2 * region + (kk & 3) * 32) >> 4),
+                                  idesc, kk != 0 ? 1u : 0u);
                     tc_commit(&b_empty[slot]);
                     tc_commit(&d_full[bs]);
                 }
@@ -495,9 +495,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             if (warp < TC_CONV_WARPS) {
                 // ---- unpacking: codes of row (rgl, r4) into A, one block at a time
                 for (int b = 0; b < nb && ok; ++b) {
-                    const int64_t bb = nblk + b;
+                    const int bb = nblk + b;
                     const int as = static_cast<int>(bb & 1);
-                    const int64_t rb = nraw + b / 2;
+                    const int rb = nraw + b / 2;
                     const int rs = static_cast<int>(rb & 1);
                     // the raw blocks (for odd b the phase its even partner already
                     // waited for), a free slot of the weight-scale ring, and the A
@@ -558,12 +558,19 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     }
                 }
             } else {
-                // ---- epilogue: y (in TMEM) += float(S) * (d * da), block after block;
-                // two warps per lane quadrant, 32-column chunks (pairs) eh and eh + 2
-                const int eh = (warp - TC_CONV_WARPS) >> 2;
-                const uint32_t ycol = tmem + lane_base + TC_TMEM_Y;
+                // ---- epilogue: y (registers) += float(S) * (d * da), block after
+                // block; two warps per lane quadrant, warp q2 takes the 16-column
+                // pieces (pairs) q2, q2 + 2 and q2 + 4
+                const int q2 = (warp - TC_CONV_WARPS) >> 2;
+                const int npc = (m + 15) >> 4;  // pieces of the chunk (at most 6)
+                const int mine = npc > q2 ? (npc - q2 + 1) / 2 : 0;  // this warp's pieces (0..3)
+                float y[3][16];
+#pragma unroll
+                for (int k = 0; k < 3; ++k)
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) y[k][i] = 0.0f;
                 for (int b = 0; b < nb && ok; ++b) {
-                    const int64_t bb = nblk + b;
+                    const int bb = nblk + b;
                     const int bs = static_cast<int>(bb & 1);
                     const int ss = static_cast<int>(bb % TC_SC_STAGES);
                     const int ds = static_cast<int>(bb % TC_DW_STAGES);
@@ -576,67 +583,60 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     tc_fence_after();
                     const float dw = dw_ring[ds * TC_ROWS + r4 * 32 + rgl];
                     const float *sc = reinterpret_cast<const float *>(smem + TC_OFF_SC + ss * TC_SC_BYTES);
-                    const uint32_t dcol = tmem + lane_base + TC_TMEM_D + bs * TC_CHUNK;
-                    // With the planes side by side a warp has one chunk: once both
-                    // accumulator halves are in registers the buffer goes back to
-                    // the MMAs, before the y update.
-                    bool released = false;
-#pragma unroll 1
-                    for (int c = eh; c < TC_CHUNK / 32; c += 2) {
-                        if (32 * c >= m) break;
-                        uint32_t d[32], yv[32];
-                        tc_ld32(dcol + 32 * c, d);
-                        if (side) {  // D = high-plane half + low-plane half (exact)
-                            tc_ld32(dcol + 64 + 32 * c, yv);
-                            tc_wait_ld();
+                    const uint32_t dcol = tmem + lane_base + TC_TMEM_D + bs * TC_DCOLS;
+                    if (mine == 0) {  // nothing to read: hand the buffer back at once
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&d_empty[bs]);
+                    }
+#pragma unroll
+                    for (int k = 0; k < 3; ++k) {
+                        if (k >= mine) break;
+                        const int pc = q2 + 2 * k;
+                        // piece pc's accumulator columns, both plane halves; after
+                        // the warp's last read of the buffer it goes back to the MMAs
+                        uint32_t hv[16], lv[16];
+                        tc_ld16(dcol + 16 * pc, hv);
+                        tc_ld16(dcol + nmma + 16 * pc, lv);
+                        tc_wait_ld();
+                        if (k == mine - 1) {
                             tc_fence_before();
                             __syncwarp();
                             if (lane == 0) mbar_arrive(&d_empty[bs]);
-                            released = true;
-#pragma unroll
-                            for (int i = 0; i < 32; ++i)
-                                d[i] = __float_as_uint(__fadd_rn(__uint_as_float(d[i]), __uint_as_float(yv[i])));
                         }
-                        if (b > 0) tc_ld32(ycol + 32 * c, yv);
-                        tc_wait_ld();
 #pragma unroll
-                        for (int n4 = 0; n4 < 8; ++n4) {
-                            const float4 da = *reinterpret_cast<const float4 *>(sc + 32 * c + 4 * n4);
-                            const float4 bi = *reinterpret_cast<const float4 *>(sc + TC_CHUNK + 32 * c + 4 * n4);
+                        for (int n4 = 0; n4 < 4; ++n4) {
+                            const float4 da = *reinterpret_cast<const float4 *>(sc + 16 * pc + 4 * n4);
+                            const float4 bi = *reinterpret_cast<const float4 *>(sc + TC_CHUNK + 16 * pc + 4 * n4);
                             const float dav[4] = {da.x, da.y, da.z, da.w}, biv[4] = {bi.x, bi.y, bi.z, bi.w};
 #pragma unroll
                             for (int q = 0; q < 4; ++q) {
                                 const int i = 4 * n4 + q;
-                                // S = 512 D - 4 bsum, exact (integers below 2^18)
-                                const float S = __fmaf_rn(512.0f, __uint_as_float(d[i]), biv[q]);
-                                const float yo = b > 0 ? __uint_as_float(yv[i]) : 0.0f;
-                                yv[i] = __float_as_uint(__fadd_rn(yo, __fmul_rn(S, __fmul_rn(dw, dav[q]))));
+                                // D = high-plane half + low-plane half (exact); S = 512 D - 4 bsum,
+                                // exact (integers below 2^18)
+                                const float D = __fadd_rn(__uint_as_float(hv[i]), __uint_as_float(lv[i]));
+                                const float S = __fmaf_rn(512.0f, D, biv[q]);
+                                y[k][i] = __fadd_rn(y[k][i], __fmul_rn(S, __fmul_rn(dw, dav[q])));
                             }
                         }
-                        tc_st32(ycol + 32 * c, yv);
                     }
-                    tc_wait_st();
-                    tc_fence_before();
                     __syncwarp();
                     if (lane == 0) {
-                        if (!released) mbar_arrive(&d_empty[bs]);
                         mbar_arrive(&sc_empty[ss]);
                         mbar_arrive(&dw_empty[ds]);
                     }
                 }
                 if (ok && rg0 + rgl < n_rg) {
-                    const int64_t grow = static_cast<int64_t>(rg0 + rgl) * 4 + r4;
-#pragma unroll 1
-                    for (int c = eh; c < TC_CHUNK / 32; c += 2) {
-                        const int n0 = 32 * c;
-                        if (n0 >= m) break;
-                        uint32_t yv[32];
-                        tc_ld32(ycol + 32 * c, yv);
-                        tc_wait_ld();
+                    // row (rg0 + rgl, r4) of the pairs' outputs: pair n at yr[n N]
+                    float *yr = J.Y + static_cast<int64_t>(pb) * J.N + (static_cast<int64_t>(rg0 + rgl) * 4 + r4);
+                    const int N = J.N;
 #pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            if (n0 + i < m)
-                                J.Y[static_cast<int64_t>(pb + n0 + i) * J.N + grow] = __uint_as_float(yv[i]);
+                    for (int k = 0; k < 3; ++k) {
+                        if (k >= mine) break;
+                        const int n0 = 16 * (q2 + 2 * k);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i)
+                            if (n0 + i < m) yr[(n0 + i) * N] = y[k][i];
                     }
                 }
             }
@@ -651,10 +651,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (n_rf0 > 0) mbar_wait(&raw_full[0], static_cast<uint32_t>((n_rf0 - 1) & 1));
         if (n_rf1 > 0) mbar_wait(&raw_full[1], static_cast<uint32_t>((n_rf1 - 1) & 1));
         // the last TC_B_SLOTS blocks of B, oldest first
-        for (int64_t u = imax64(0, last_b - TC_B_SLOTS + 1); u <= last_b; ++u)
+        for (int u = max(0, last_b - TC_B_SLOTS + 1); u <= last_b; ++u)
             mbar_wait(&b_full[u % TC_B_SLOTS], static_cast<uint32_t>((u / TC_B_SLOTS) & 1));
         // the last TC_SC_STAGES scale copies, oldest first
-        for (int64_t u = imax64(0, last_sc - TC_SC_STAGES + 1); u <= last_sc; ++u)
+        for (int u = max(0, last_sc - TC_SC_STAGES + 1); u <= last_sc; ++u)
             mbar_wait(&sc_full[u % TC_SC_STAGES], static_cast<uint32_t>((u / TC_SC_STAGES) & 1));
     }
     if (warp == TC_MATH_WARPS + 1 && lane == 0) {
