@@ -314,6 +314,22 @@ __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
         }
     }
     if (tid == blockDim.x - 1) *a.n_chunks = cincl;
+    // The tensor-core launches' share of the list: the chunks of more than
+    // small_max pairs, in chunk order, so that those launches deal their items
+    // out over these alone (the small-group pass takes the others). An entry
+    // carries the chunk's fields too: one load per item.
+    int ntc = 0;
+    for (int i = 0; i < nc; ++i) ntc += min(CH, c - i * CH) > a.small_max;
+    const int tincl = block_scan_1024(ntc, warp_tot);
+    if (tid < E) {
+        const int base = cincl - nc;
+        int pos = tincl - ntc;
+        for (int i = 0; i < nc; ++i) {
+            const int len = min(CH, c - i * CH);
+            if (len > a.small_max) a.tc_list[pos++] = make_int4(base + i, tid, incl - c + i * CH, len);
+        }
+    }
+    if (tid == blockDim.x - 1) *a.n_tc = tincl;
     // Stable placement: W warps take consecutive ranges of the pairs; each
     // counts its hits per expert, the counts are turned into per-warp start
     // positions (expert offset + hits of the earlier ranges), and each warp
@@ -935,6 +951,8 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
         a.chunk_begin = reinterpret_cast<int *>(base + L.chunk_begin);
         a.chunk_len = reinterpret_cast<int *>(base + L.chunk_len);
         a.n_chunks = reinterpret_cast<int *>(base + L.n_chunks);
+        a.tc_list = reinterpret_cast<int4 *>(base + L.tc_list);
+        a.n_tc = reinterpret_cast<int *>(base + L.n_tc);
         a.xq = base + L.xq;
         a.xqt = base + L.xqt;
         a.hq = base + L.hq;

@@ -23,6 +23,7 @@ struct MoeLayout {
     size_t xg;  // int8 [P][H] (grouped only)
     size_t dxg, bxg, dhp, bhp;  // [P][round4(nb)] (grouped only)
     size_t chunk_expert, chunk_begin, chunk_len, n_chunks;  // grouped GEMM work list
+    size_t tc_list, n_tc;  // int4 [max_chunks] (chunk, expert, begin, pairs) of the tensor-core launches' chunks, and their count (grouped only)
     size_t xq, hq;    // e4m3 activation planes [2][P][H], [2][P][I] for the tensor-core contraction (grouped only)
     size_t xqt;       // the same planes of x in token order [2][T][H] (grouped only)
     size_t pair_chunk, xs, hs;  // tensor-core work list helpers (grouped only)
@@ -95,6 +96,8 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.chunk_begin = take(4 * static_cast<size_t>(L.max_chunks));
         L.chunk_len = take(4 * static_cast<size_t>(L.max_chunks));
         L.n_chunks = take(4);
+        L.tc_list = take(16 * static_cast<size_t>(L.max_chunks));
+        L.n_tc = take(4);
         L.xq = take(2 * static_cast<size_t>(P * H));
         L.hq = take(2 * static_cast<size_t>(P * I));
         L.xqt = take(2 * static_cast<size_t>(T * H));
@@ -107,6 +110,7 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.counts = L.offsets = L.pair_token = L.pair_slot = L.pair_of = L.xg = SIZE_MAX;
         L.dxg = L.bxg = L.dhp = L.bhp = SIZE_MAX;
         L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
+        L.tc_list = L.n_tc = SIZE_MAX;
         L.xq = L.hq = L.xqt = L.pair_chunk = L.xs = L.hs = L.rnorm = L.rpart = SIZE_MAX;
         L.max_chunks = 0;
     }
@@ -182,6 +186,8 @@ struct GroupedArgs {
     float *o;
     int *counts, *offsets, *pair_token, *pair_slot, *pair_of;
     int *chunk_expert, *chunk_begin, *chunk_len, *n_chunks;
+    int4 *tc_list;        // chunks of more than small_max pairs, in chunk order: (chunk, expert, first pair, pairs)
+    int *n_tc;            // their count
     int keep_h;
     int tc;               // contraction on tcgen05 tensor cores
     int chunk;            // pairs per chunk of the work list (GG_TOK, or TC_CHUNK on tensor cores)

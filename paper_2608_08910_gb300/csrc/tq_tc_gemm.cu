@@ -373,11 +373,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(tmem_slot);
 
-    const int n_chunks = __ldcg(a.n_chunks);
+    // Items are dealt out over the chunks of more than small_max pairs alone
+    // (the work list's tensor-core share, in chunk order), so every CTA gets
+    // the same number to within one.
+    const int n_tc = __ldcg(a.n_tc);
     const int64_t tiles0 = (j0.N / 4 + TC_RG - 1) / TC_RG;
     const int64_t tiles1 = njobs > 1 ? (j1.N / 4 + TC_RG - 1) / TC_RG : 0;
     const int64_t per_chunk = tiles0 + tiles1;
-    const int64_t items = static_cast<int64_t>(n_chunks) * per_chunk;
+    const int64_t items = static_cast<int64_t>(n_tc) * per_chunk;
 
     // All roles walk the same items and blocks, so each keeps identical
     // counts of raw stages and blocks used so far (the ring positions).
@@ -388,15 +391,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     int n_rf0 = 0, n_rf1 = 0, last_b = -1, last_sc = -1;
     for (int64_t w = blockIdx.x; w < items; w += gridDim.x) {
         if (*reinterpret_cast<volatile int *>(abort)) break;
-        const int chunk = static_cast<int>(w / per_chunk);
-        int64_t tl = w - chunk * per_chunk;
+        const int ci = static_cast<int>(w / per_chunk);
+        const int4 t = __ldcg(a.tc_list + ci);  // (chunk, expert, first pair, pairs)
+        const int chunk = t.x;
+        int64_t tl = w - ci * per_chunk;
         const bool second = tl >= tiles0;
         if (second) tl -= tiles0;
         const TcJob &J = second ? j1 : j0;
-        const int e = __ldcg(a.chunk_expert + chunk);
-        const int pb = __ldcg(a.chunk_begin + chunk);
-        const int m = __ldcg(a.chunk_len + chunk);
-        if (m <= a.small_max) continue;  // the small-group pass's chunk (every role skips it alike)
+        const int e = t.y;
+        const int pb = t.z;
+        const int m = t.w;
         const int n_rg = J.N / 4;
         const int rg0 = static_cast<int>(tl) * TC_RG;
         const int nb = J.nb;
