@@ -278,30 +278,80 @@ __device__ __forceinline__ int block_scan_1024(int v, int *warp_tot) {
     return r;
 }
 
+// The lanes whose expert equals this lane's (valid lanes only; an invalid
+// lane's mask holds the invalid lanes): one ballot per bit of the expert
+// index and one for validity. Deterministic, and far cheaper than
+// __match_any_sync with many distinct values in the warp.
+template <int BITS>
+__device__ __forceinline__ unsigned expert_peers_t(int e, bool valid) {
+    unsigned m = __ballot_sync(0xffffffffu, valid);
+    if (!valid) m = ~m;
+#pragma unroll
+    for (int b = 0; b < BITS; ++b) {
+        const bool set = (e >> b) & 1;
+        const unsigned bal = __ballot_sync(0xffffffffu, set);
+        m &= set ? bal : ~bal;
+    }
+    return m;
+}
+__device__ __forceinline__ unsigned expert_peers(int e, bool valid, int bits) {
+    return bits <= 8 ? expert_peers_t<8>(e, valid) : expert_peers_t<10>(e, valid);
+}
+
+// Work lists of at least this many pairs leave the scattered (token, slot)
+// stores to scatter_pairs_kernel; smaller ones take them in the grouping kernel.
+constexpr int kScatterMinPairs = 4096;
+
 __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
     // counts, offsets, the chunk list and the stable (token, slot) order of
-    // the pairs inside each expert's range
+    // the pairs inside each expert's range. W warps take consecutive ranges
+    // of the pairs; each counts its hits per expert (the experts' totals are
+    // the sums over warps), the counts are turned into per-warp start
+    // positions (expert offset + hits of the earlier ranges), and each warp
+    // places its pairs in order, ranking equal experts by lane.
     constexpr int HIST = 8192;  // per-warp counts: warps x experts
-    __shared__ int cnt[TQFX4_MAX_EXPERTS], off[TQFX4_MAX_EXPERTS + 1];
     __shared__ int hist[HIST];
     __shared__ int warp_tot[32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int E = a.E, P = a.P, k = a.top_k, CH = a.chunk;
-    if (tid < E) cnt[tid] = 0;
+    const int W = min(32, HIST / E);
+    const int ebits = E > 256 ? 10 : 8;  // bits of an expert index (at most TQFX4_MAX_EXPERTS = 1024)
+    const int R = (P + W - 1) / W;
+    const unsigned lt = (1u << lane) - 1u;
+    // the selections are read 8 rounds of 32 at a time (all loads in flight
+    // before the first use), then processed round by round in order
+    constexpr int GB = 8;
+    for (int i = tid; i < W * E; i += blockDim.x) hist[i] = 0;
     __syncthreads();
-    for (int p = tid; p < P; p += blockDim.x) atomicAdd(&cnt[__ldcg(a.sel + p)], 1);
+    if (warp < W) {
+        const int p0 = warp * R, p1 = min(P, p0 + R);
+        for (int base0 = p0; base0 < p1; base0 += 32 * GB) {
+            int ev[GB];
+#pragma unroll
+            for (int u = 0; u < GB; ++u) {
+                const int p = base0 + 32 * u + lane;
+                ev[u] = p < p1 ? __ldcg(a.sel + p) : -1 - lane;
+            }
+#pragma unroll
+            for (int u = 0; u < GB; ++u) {
+                if (base0 + 32 * u >= p1) break;
+                const int e = ev[u];
+                const bool valid = base0 + 32 * u + lane < p1;
+                const unsigned peers = expert_peers(e, valid, ebits);
+                if (valid && lane == __ffs(peers) - 1) hist[warp * E + e] += __popc(peers);
+            }
+        }
+    }
     __syncthreads();
-    const int c = tid < E ? cnt[tid] : 0;
+    int c = 0;
+    if (tid < E)
+        for (int w = 0; w < W; ++w) c += hist[w * E + tid];
     const int incl = block_scan_1024(c, warp_tot);
     if (tid < E) {
-        off[tid + 1] = incl;
         a.counts[tid] = c;
         a.offsets[tid + 1] = incl;
     }
-    if (tid == 0) {
-        off[0] = 0;
-        a.offsets[0] = 0;
-    }
+    if (tid == 0) a.offsets[0] = 0;
     // chunk list: ceil(count / CH) chunks per expert
     const int nc = (c + CH - 1) / CH;
     const int cincl = block_scan_1024(nc, warp_tot);
@@ -330,40 +380,9 @@ __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
         }
     }
     if (tid == blockDim.x - 1) *a.n_tc = tincl;
-    // Stable placement: W warps take consecutive ranges of the pairs; each
-    // counts its hits per expert, the counts are turned into per-warp start
-    // positions (expert offset + hits of the earlier ranges), and each warp
-    // places its pairs in order, ranking equal experts by lane.
-    const int W = min(32, HIST / E);
-    const int R = (P + W - 1) / W;
-    for (int i = tid; i < W * E; i += blockDim.x) hist[i] = 0;
-    __syncthreads();
-    const unsigned lt = (1u << lane) - 1u;
-    // the selections are read 8 rounds of 32 at a time (all loads in flight
-    // before the first use), then processed round by round in order
-    constexpr int GB = 8;
-    if (warp < W) {
-        const int p0 = warp * R, p1 = min(P, p0 + R);
-        for (int base0 = p0; base0 < p1; base0 += 32 * GB) {
-            int ev[GB];
-#pragma unroll
-            for (int u = 0; u < GB; ++u) {
-                const int p = base0 + 32 * u + lane;
-                ev[u] = p < p1 ? __ldcg(a.sel + p) : -1 - lane;
-            }
-#pragma unroll
-            for (int u = 0; u < GB; ++u) {
-                if (base0 + 32 * u >= p1) break;
-                const int e = ev[u];
-                const bool valid = base0 + 32 * u + lane < p1;
-                const unsigned peers = __match_any_sync(0xffffffffu, e);
-                if (valid && lane == __ffs(peers) - 1) hist[warp * E + e] += __popc(peers);
-            }
-        }
-    }
-    __syncthreads();
+    // per-warp start positions
     if (tid < E) {
-        int run = off[tid];
+        int run = incl - c;
         for (int w = 0; w < W; ++w) {
             const int h = hist[w * E + tid];
             hist[w * E + tid] = run;
@@ -371,6 +390,7 @@ __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
         }
     }
     __syncthreads();
+    const bool inline_scatter = P < kScatterMinPairs;
     if (warp < W) {
         const int p0 = warp * R, p1 = min(P, p0 + R);
         for (int base0 = p0; base0 < p1; base0 += 32 * GB) {
@@ -386,7 +406,7 @@ __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
                 const int p = base0 + 32 * u + lane;
                 const bool valid = p < p1;
                 const int e = ev[u];
-                const unsigned peers = __match_any_sync(0xffffffffu, e);
+                const unsigned peers = expert_peers(e, valid, ebits);
                 const int leader = __ffs(peers) - 1;
                 int b = 0;
                 if (valid && lane == leader) {
@@ -396,13 +416,27 @@ __global__ void __launch_bounds__(1024) group_kernel(GroupedArgs a) {
                 b = __shfl_sync(0xffffffffu, b, leader);
                 if (valid) {
                     const int pos = b + __popc(peers & lt);
-                    a.pair_token[pos] = p / k;
-                    a.pair_slot[pos] = p - (p / k) * k;
                     a.pair_of[p] = pos;
+                    if (inline_scatter) {
+                        a.pair_token[pos] = p / k;
+                        a.pair_slot[pos] = p - (p / k) * k;
+                    }
                 }
             }
         }
     }
+}
+
+// The inverse of pair_of (each pair's token and slot at its place in expert
+// order): scattered stores, spread over many CTAs rather than the grouping
+// kernel's one.
+__global__ void __launch_bounds__(256) scatter_pairs_kernel(GroupedArgs a) {
+    const int p = blockIdx.x * blockDim.x + threadIdx.x;
+    if (p >= a.P) return;
+    const int pos = __ldcg(a.pair_of + p);
+    const int t = p / a.top_k;
+    a.pair_token[pos] = t;
+    a.pair_slot[pos] = p - t * a.top_k;
 }
 
 // ---------------------------------------------------------------- grouped GEMM
@@ -1008,6 +1042,7 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(2);
     group_kernel<<<1, 1024, 0, st>>>(a);
+    if (a.P >= kScatterMinPairs) scatter_pairs_kernel<<<(a.P + 255) / 256, 256, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     rec(3);
     if ((e = launch_quantize(a.X, a.T, a.H, a.qx, a.dx, a.bx, a.status, st)) != cudaSuccess) return e;
