@@ -73,7 +73,7 @@ __global__ void __launch_bounds__(128) router_batch_kernel(GroupedArgs a) {
 // Cauchy-Schwarz), gamma_H = H u / (1 - H u), u = 2^-24. The bias add and
 // the bound arithmetic add a few units of roundoff relative to |logit|; the
 // bound below covers them with margin.
-constexpr int RG_T = 64, RG_E = 64, RG_BK = 32;
+constexpr int RG_T = 128, RG_E = 128, RG_BK = 8;
 
 __global__ void __launch_bounds__(256) router_norm_kernel(GroupedArgs a) {
     const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
@@ -90,39 +90,32 @@ __global__ void __launch_bounds__(256) router_norm_kernel(GroupedArgs a) {
 }
 
 // part[s][t][e] = fl(sum over slice s of x[t][h] w[e][h]), h ascending, one
-// thread per output; tiles of 64 tokens x 64 experts, 4 x 4 outputs per
-// thread, grid z = slice.
-__global__ void __launch_bounds__(256) router_gemm_kernel(GroupedArgs a) {
+// thread per output; tiles of 128 tokens x 128 experts, 8 x 8 outputs per
+// thread (rows 4 ty .. + 3 and 64 + 4 ty .. + 3, columns likewise with tx),
+// k-steps of 8 staged through shared memory, grid z = slice.
+__global__ void __launch_bounds__(256, 2) router_gemm_kernel(GroupedArgs a) {
     __shared__ __align__(16) float xs[2][RG_BK][RG_T + 4];
     __shared__ __align__(16) float wsm[2][RG_BK][RG_E + 4];
     const int e0 = blockIdx.x * RG_E, t0 = blockIdx.y * RG_T;
     const int hs = a.H / kScreenSplit, h0 = blockIdx.z * hs;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-    float acc[4][4];
+    float acc[8][8];
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
-    float4 xr[2], wr[2];
+        for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
+    // staging: thread i loads 4 consecutive k of row i / 2 of each tile
+    const int sr = threadIdx.x >> 1, sc = 4 * (threadIdx.x & 1);
+    const float *xrow = t0 + sr < a.T ? a.X + static_cast<int64_t>(t0 + sr) * a.H : nullptr;
+    const float *wrow = e0 + sr < a.E ? a.wr + static_cast<int64_t>(e0 + sr) * a.H : nullptr;
+    float4 xr, wr;
     auto fetch = [&](int k0) {
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const int i = threadIdx.x + 256 * u, r = i >> 3, c4 = i & 7;
-            xr[u] = t0 + r < a.T ? __ldg(reinterpret_cast<const float4 *>(a.X + static_cast<int64_t>(t0 + r) * a.H + k0) + c4)
-                                 : make_float4(0.f, 0.f, 0.f, 0.f);
-            wr[u] = e0 + r < a.E ? __ldg(reinterpret_cast<const float4 *>(a.wr + static_cast<int64_t>(e0 + r) * a.H + k0) + c4)
-                                 : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
+        xr = xrow ? __ldg(reinterpret_cast<const float4 *>(xrow + k0 + sc)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        wr = wrow ? __ldg(reinterpret_cast<const float4 *>(wrow + k0 + sc)) : make_float4(0.f, 0.f, 0.f, 0.f);
     };
     auto stash = [&](int buf) {
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const int i = threadIdx.x + 256 * u, r = i >> 3, c4 = i & 7;
-            xs[buf][4 * c4][r] = xr[u].x, xs[buf][4 * c4 + 1][r] = xr[u].y;
-            xs[buf][4 * c4 + 2][r] = xr[u].z, xs[buf][4 * c4 + 3][r] = xr[u].w;
-            wsm[buf][4 * c4][r] = wr[u].x, wsm[buf][4 * c4 + 1][r] = wr[u].y;
-            wsm[buf][4 * c4 + 2][r] = wr[u].z, wsm[buf][4 * c4 + 3][r] = wr[u].w;
-        }
+        xs[buf][sc][sr] = xr.x, xs[buf][sc + 1][sr] = xr.y, xs[buf][sc + 2][sr] = xr.z, xs[buf][sc + 3][sr] = xr.w;
+        wsm[buf][sc][sr] = wr.x, wsm[buf][sc + 1][sr] = wr.y, wsm[buf][sc + 2][sr] = wr.z, wsm[buf][sc + 3][sr] = wr.w;
     };
     fetch(h0);
     stash(0);
@@ -131,25 +124,29 @@ __global__ void __launch_bounds__(256) router_gemm_kernel(GroupedArgs a) {
     for (int it = 0; it < nk; ++it) {
         const int buf = it & 1;
         if (it + 1 < nk) fetch(h0 + (it + 1) * RG_BK);
-#pragma unroll 8
+#pragma unroll
         for (int k = 0; k < RG_BK; ++k) {
-            const float4 xv = *reinterpret_cast<const float4 *>(&xs[buf][k][4 * ty]);
-            const float4 wv = *reinterpret_cast<const float4 *>(&wsm[buf][k][4 * tx]);
-            const float xx[4] = {xv.x, xv.y, xv.z, xv.w}, ww[4] = {wv.x, wv.y, wv.z, wv.w};
+            const float4 x0 = *reinterpret_cast<const float4 *>(&xs[buf][k][4 * ty]);
+            const float4 x1 = *reinterpret_cast<const float4 *>(&xs[buf][k][64 + 4 * ty]);
+            const float4 w0 = *reinterpret_cast<const float4 *>(&wsm[buf][k][4 * tx]);
+            const float4 w1 = *reinterpret_cast<const float4 *>(&wsm[buf][k][64 + 4 * tx]);
+            const float xx[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+            const float ww[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
+            for (int i = 0; i < 8; ++i)
 #pragma unroll
-                for (int j = 0; j < 4; ++j) acc[i][j] = __fmaf_rn(xx[i], ww[j], acc[i][j]);
+                for (int j = 0; j < 8; ++j) acc[i][j] = __fmaf_rn(xx[i], ww[j], acc[i][j]);
         }
         if (it + 1 < nk) stash(buf ^ 1);
         __syncthreads();
     }
     float *part = a.rpart + static_cast<int64_t>(blockIdx.z) * a.T * a.E;
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const int t = t0 + 4 * ty + i, e = e0 + 4 * tx + j;
+        for (int j = 0; j < 8; ++j) {
+            const int t = t0 + (i < 4 ? 4 * ty + i : 60 + 4 * ty + i);
+            const int e = e0 + (j < 4 ? 4 * tx + j : 60 + 4 * tx + j);
             if (t < a.T && e < a.E) part[static_cast<int64_t>(t) * a.E + e] = acc[i][j];
         }
 }

@@ -40,7 +40,7 @@ constexpr int GG_TOK = 64;
 // from 4 tokens (top-8) up, so the automatic choice always takes it.
 constexpr int64_t kTcMinPairs = 1;
 // Slices of the hidden dimension the router's screening GEMM sums separately.
-constexpr int kScreenSplit = 4;
+constexpr int kScreenSplit = 8;
 // Pairs per chunk on the tensor-core path: both activation planes of a
 // chunk side by side make the MMA's N = 2 x 96 = 192.
 constexpr int TC_CHUNK = 96;
