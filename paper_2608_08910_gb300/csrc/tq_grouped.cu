@@ -152,13 +152,12 @@ __global__ void __launch_bounds__(256, 2) router_gemm_kernel(GroupedArgs a) {
 }
 
 // One CTA per token: the slice sums and the bounds, the k-th largest lower
-// bound (warp 0), then the compensated logits of the candidates, spread over
-// the CTA's warps.
+// bound (warp 0), then the list of candidates (the experts whose upper bound
+// reaches it), whose compensated logits router_cand_kernel forms.
 constexpr int RF_WARPS = 4;
 
 __global__ void __launch_bounds__(RF_WARPS * 32) router_refine_kernel(GroupedArgs a) {
     extern __shared__ float lower[];  // [E]
-    __shared__ int cand[TQFX4_MAX_EXPERTS];
     __shared__ int n_cand;
     __shared__ float kth_s;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -206,14 +205,30 @@ __global__ void __launch_bounds__(RF_WARPS * 32) router_refine_kernel(GroupedArg
     }
     __syncthreads();
     const float kth = kth_s;
+    int *cand = a.rcand + static_cast<int64_t>(t) * a.E;
     for (int e = threadIdx.x; e < a.E; e += blockDim.x) {
         const float v = lg[e];
         if (v + bound(e, v) >= kth) cand[atomicAdd(&n_cand, 1)] = e;
     }
     __syncthreads();
+    if (threadIdx.x == 0) a.rcount[t] = n_cand;
+}
+
+// The candidates' compensated logits, one warp per (token, candidate): CTA
+// (t, y) takes candidates y * RC_WARPS + w, then every RC_Y * RC_WARPS-th,
+// so the work is spread over the whole grid whatever each token's count.
+constexpr int RC_WARPS = 8, RC_Y = 2;
+
+__global__ void __launch_bounds__(RC_WARPS * 32) router_cand_kernel(GroupedArgs a) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int t = blockIdx.x;
+    const int n = __ldcg(a.rcount + t);
+    const int *cand = a.rcand + static_cast<int64_t>(t) * a.E;
     const float *x = a.X + static_cast<int64_t>(t) * a.H;
-    for (int i = warp; i < n_cand; i += RF_WARPS) {
-        const int c = cand[i];
+    float *lg = a.logits + static_cast<int64_t>(t) * a.E;
+    float *ll = a.logits_lo + static_cast<int64_t>(t) * a.E;
+    for (int i = blockIdx.y * RC_WARPS + warp; i < n; i += RC_Y * RC_WARPS) {
+        const int c = __ldcg(cand + i);
         float hi, lo;
         router_logit_warp(a.wr + static_cast<int64_t>(c) * a.H, x, a.H, hi, lo);
         if (lane == 0) {
@@ -992,6 +1007,8 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
         a.hs = reinterpret_cast<float *>(base + L.hs);
         a.rnorm = reinterpret_cast<float *>(base + L.rnorm);
         a.rpart = reinterpret_cast<float *>(base + L.rpart);
+        a.rcand = reinterpret_cast<int *>(base + L.rcand);
+        a.rcount = reinterpret_cast<int *>(base + L.rcount);
     }
     return true;
 }
@@ -1030,6 +1047,7 @@ cudaError_t launch_moe_grouped(const GroupedArgs &a0, const float *X, float *OUT
         router_norm_kernel<<<(a.T + a.E + 7) / 8, 256, 0, st>>>(a);
         router_gemm_kernel<<<dim3((a.E + RG_E - 1) / RG_E, (a.T + RG_T - 1) / RG_T, kScreenSplit), 256, 0, st>>>(a);
         router_refine_kernel<<<a.T, RF_WARPS * 32, a.E * sizeof(float), st>>>(a);
+        router_cand_kernel<<<dim3(a.T, RC_Y), RC_WARPS * 32, 0, st>>>(a);
     } else {
         router_batch_kernel<<<dim3(a.E, (a.T + RB_TOK - 1) / RB_TOK), 128, 0, st>>>(a);
     }

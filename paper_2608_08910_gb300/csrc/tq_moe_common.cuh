@@ -29,6 +29,7 @@ struct MoeLayout {
     size_t pair_chunk, xs, hs;  // tensor-core work list helpers (grouped only)
     size_t rnorm;     // fp32 [T + E]: Euclidean norms of the hidden states and router rows (grouped only)
     size_t rpart;     // fp32 [kScreenSplit][T][E]: partial router logits of the screening GEMM (grouped only)
+    size_t rcand, rcount;  // int [T][E], [T]: each token's screened-in experts and their count (grouped only)
     int64_t max_chunks;
     size_t total;
 };
@@ -104,6 +105,8 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.pair_chunk = take(4 * static_cast<size_t>(P));
         L.rnorm = take(4 * static_cast<size_t>(T + E));
         L.rpart = take(4 * static_cast<size_t>(kScreenSplit) * T * E);
+        L.rcand = take(4 * static_cast<size_t>(T) * E);
+        L.rcount = take(4 * static_cast<size_t>(T));
         L.xs = take(static_cast<size_t>(L.max_chunks) * nbh * 2 * TC_CHUNK * 4);
         L.hs = take(static_cast<size_t>(L.max_chunks) * nbi * 2 * TC_CHUNK * 4);
     } else {
@@ -112,6 +115,7 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
         L.tc_list = L.n_tc = SIZE_MAX;
         L.xq = L.hq = L.xqt = L.pair_chunk = L.xs = L.hs = L.rnorm = L.rpart = SIZE_MAX;
+        L.rcand = L.rcount = SIZE_MAX;
         L.max_chunks = 0;
     }
     L.total = off;
@@ -201,6 +205,7 @@ struct GroupedArgs {
                           // then -4 bsum as float (tensor-core path)
     float *rnorm;         // [T + E] norms for the screened router
     float *rpart;         // [kScreenSplit][T][E] partial logits of the screening GEMM
+    int *rcand, *rcount;  // [T][E], [T]: the experts each token's compensated logits are formed for
 };
 
 // Shared-memory bytes of one quantized activation vector of nb blocks
