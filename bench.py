@@ -59,11 +59,11 @@ def _peaks():
 # DRAM bytes (read + write) of one gate_up_kernel launch, from an ncu --set full capture of the
 # 64-expert layer (one launch reads the 8 selected experts whatever the expert count). Set to None
 # when the kernel changes until it is captured again.
-GATE_UP_TRAFFIC = 68196864 + 982528
+GATE_UP_TRAFFIC = 68200448 + 936704
 # The same for one tc_gemm_kernel gate/up launch of the 2048-token prefill: an ncu capture at 64
 # experts and 512 tokens (one chunk per expert, as in the full workload) scaled by the full
 # workload's 4x weight bytes and pairs.
-TC_GATE_UP_TRAFFIC = 4 * (580200448 + 58917376)
+TC_GATE_UP_TRAFFIC = 4 * (580347392 + 58900992)
 
 
 def max_over_ranks(t, world, device):
