@@ -101,6 +101,7 @@ def check_grouped(layer, seed, X, sample, path=0, check_stages=True, stage_token
     (32, 1024, 512, 6, 33, 1.1),     # skewed routing
     (4, 512, 512, 4, 3, 0.0),        # top_k = n_experts
     (64, 2048, 1536, 8, 1, 0.0),     # a single token; inter not a multiple of 1024
+    (512, 512, 512, 8, 600, 1.1),    # 10-bit expert indices; 4800 pairs: the wide (token, slot) scatter
 ])
 @pytest.mark.parametrize("path", [B.TQFX4_PATH_DECODE, B.TQFX4_PATH_PREFILL])
 def test_grouped_small(E, H, I, k, T, zipf, path):
