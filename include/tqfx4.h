@@ -289,6 +289,27 @@ tqfx4_status tqfx4_moe_ffn(const tqfx4_experts *ex, const tqfx4_router *rt,
                            const float *x, float *out, int32_t *sel_idx, float *sel_w,
                            void *ws, size_t ws_bytes, void *stream);
 
+/* Workspace bytes for tqfx4_moe_ffn_host: tqfx4_moe_ffn's layout followed by
+ * device staging for x, out and the selection. 0 if the shapes are invalid. */
+size_t tqfx4_moe_ffn_host_workspace_bytes(const tqfx4_experts *ex, const tqfx4_router *rt);
+
+/*
+ * tqfx4_moe_ffn_host -- tqfx4_moe_ffn for a token in host memory (Sec. 2.2,
+ * the serving call with its copies): x_host (fp32 [hidden]) is copied into
+ * the workspace's staging, the layer runs, and out (fp32 [hidden]) and, when
+ * their pointers are not NULL, sel_idx (int32 [top_k]) and sel_w (fp32
+ * [top_k]) are copied back, all ordered on `stream` with one copy each. The
+ * call returns once the work is enqueued: the host buffers must stay valid,
+ * and the outputs are complete only after the stream has passed them
+ * (synchronize before reading). Page-locked host buffers make the copies
+ * asynchronous; pageable ones make the call wait for them. The results equal
+ * tqfx4_moe_ffn's bit for bit. Workspace: tqfx4_moe_ffn_host_workspace_bytes.
+ * Errors: as tqfx4_moe_ffn, and TQFX4_EINVAL for a NULL x_host or out_host.
+ */
+tqfx4_status tqfx4_moe_ffn_host(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x_host,
+                                float *out_host, int32_t *sel_idx_host, float *sel_w_host, void *ws,
+                                size_t ws_bytes, void *stream);
+
 /*
  * tqfx4_moe_ffn_mxfp4 -- tqfx4_moe_ffn with MXFP4 experts (the
  * expert-lossless arm, Sec. 2.3: the released expert bytes served by the

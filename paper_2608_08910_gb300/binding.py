@@ -65,6 +65,8 @@ _SIGS = {
     "tqfx4_expert_ffn_traced": (_int, [_vp, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp, _vp]),
     "tqfx4_moe_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int]),
     "tqfx4_moe_ffn": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_moe_ffn_host": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_moe_ffn_host_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter)]),
     "tqfx4_moe_ffn_mxfp4": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_ffn_mxfp4_traced": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz,
                                           _vp, C.POINTER(_vp)]),
@@ -204,6 +206,18 @@ def tqfx4_moe_ffn(ex, rt, x, out, sel_idx, sel_w, ws, stream=None, events=None):
         rc = lib().tqfx4_moe_ffn_traced(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w),
                                         _p(ws), _nbytes(ws), _s(stream), arr)
     _check(rc, "tqfx4_moe_ffn")
+
+
+def tqfx4_moe_ffn_host_workspace_bytes(ex: CExperts, rt: CRouter) -> int:
+    return int(lib().tqfx4_moe_ffn_host_workspace_bytes(C.byref(ex), C.byref(rt)))
+
+
+def tqfx4_moe_ffn_host(ex, rt, x, out, sel_idx, sel_w, ws, stream=None):
+    """x, out, sel_idx, sel_w: CPU tensors (page-locked for asynchronous copies);
+    sel_idx and sel_w may be None. The outputs are complete once `stream` has
+    passed the call."""
+    _check(lib().tqfx4_moe_ffn_host(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w), _p(ws),
+                                    _nbytes(ws), _s(stream)), "tqfx4_moe_ffn_host")
 
 
 def tqfx4_moe_ffn_mxfp4(ex, rt, x, out, sel_idx, sel_w, ws, stream=None, events=None):

@@ -313,6 +313,56 @@ tqfx4_status tqfx4_moe_ffn_traced(const tqfx4_experts *ex, const tqfx4_router *r
     return moe_ffn_impl(ex, rt, x, out, sel_idx, sel_w, ws, ws_bytes, stream, events);
 }
 
+// Staging of tqfx4_moe_ffn_host after the decode layout: x, out, the selection.
+struct HostStaging {
+    size_t x, out, sel, selw, total;
+};
+static HostStaging host_staging(const tqfx4_experts *ex, const tqfx4_router *rt) {
+    HostStaging h;
+    size_t off = tq::align256(tq::moe_layout(ex->n_experts, ex->hidden, ex->inter, rt->top_k, 1, false, true).total);
+    h.x = off;
+    off = tq::align256(off + 4 * static_cast<size_t>(ex->hidden));
+    h.out = off;
+    off = tq::align256(off + 4 * static_cast<size_t>(ex->hidden));
+    h.sel = off;
+    off = tq::align256(off + 4 * static_cast<size_t>(rt->top_k));
+    h.selw = off;
+    h.total = tq::align256(off + 4 * static_cast<size_t>(rt->top_k));
+    return h;
+}
+
+size_t tqfx4_moe_ffn_host_workspace_bytes(const tqfx4_experts *ex, const tqfx4_router *rt) {
+    if (check_moe_shapes(ex, rt, "tqfx4_moe_ffn_host_workspace_bytes")) return 0;
+    return host_staging(ex, rt).total;
+}
+
+tqfx4_status tqfx4_moe_ffn_host(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x_host,
+                                float *out_host, int32_t *sel_idx_host, float *sel_w_host, void *ws, size_t ws_bytes,
+                                void *stream) {
+    TQ_RANGE();
+    const char *fn = "tqfx4_moe_ffn_host";
+    tqfx4_status s = check_moe_shapes(ex, rt, fn);
+    if (s) return s;
+    if ((s = check_moe_ptrs(ex, rt, fn))) return s;
+    if (!x_host || !out_host) return fail(TQFX4_EINVAL, "%s: NULL x or out", fn);
+    const HostStaging h = host_staging(ex, rt);
+    if ((s = check_ws(ws, ws_bytes, h.total, fn))) return s;
+    uint8_t *base = static_cast<uint8_t *>(ws);
+    float *xd = reinterpret_cast<float *>(base + h.x), *od = reinterpret_cast<float *>(base + h.out);
+    int32_t *sd = reinterpret_cast<int32_t *>(base + h.sel);
+    float *wd = reinterpret_cast<float *>(base + h.selw);
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t xb = 4 * static_cast<size_t>(ex->hidden), kb = 4 * static_cast<size_t>(rt->top_k);
+    cudaError_t e = cudaMemcpyAsync(xd, x_host, xb, cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    if ((s = moe_ffn_impl(ex, rt, xd, od, sd, wd, ws, ws_bytes, stream, nullptr))) return s;
+    e = cudaMemcpyAsync(out_host, od, xb, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && sel_idx_host) e = cudaMemcpyAsync(sel_idx_host, sd, kb, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && sel_w_host) e = cudaMemcpyAsync(sel_w_host, wd, kb, cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
 size_t tqfx4_expert_ffn_workspace_bytes(int64_t hidden, int64_t inter) {
     if (hidden <= 0 || inter <= 0 || hidden % 256 || inter % 256 || hidden > TQFX4_MAX_K || inter > TQFX4_MAX_K)
         return 0;

@@ -103,6 +103,22 @@ class MoeLayer:
             B.tqfx4_moe_ffn(self.ex, self.rt, x, out, sel_idx, sel_w, ws, stream, events)
         return out, sel_idx, sel_w
 
+    def host_workspace(self):
+        """The workspace of ffn_host (device memory)."""
+        n = B.tqfx4_moe_ffn_host_workspace_bytes(self.ex, self.rt)
+        if n == 0:
+            raise ValueError("invalid MoE shapes")
+        return torch.zeros(n, dtype=torch.uint8, device=self.gate.device)
+
+    def ffn_host(self, x, ws, out, sel_idx=None, sel_w=None, stream=None):
+        """One token with x and the outputs in host memory (CPU tensors,
+        page-locked for asynchronous copies); ordered on `stream`, complete
+        once the stream has passed it."""
+        if self.fmt != "fx4":
+            raise ValueError("ffn_host serves tq2_0_fx4 experts")
+        B.tqfx4_moe_ffn_host(self.ex, self.rt, x, out, sel_idx, sel_w, ws, stream)
+        return out, sel_idx, sel_w
+
     def grouped(self, X, ws, path=0, OUT=None, sel_idx=None, sel_w=None, stream=None, events=None):
         if self.fmt != "fx4":
             raise ValueError("the grouped path serves tq2_0_fx4 experts")

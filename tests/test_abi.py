@@ -109,6 +109,14 @@ def test_host_validation_rejects_bad_arguments(lib):
     assert lib.tqfx4_gemv_x(None, 1024, 256, None, None, None, None, None, None, 0, None) == 2
     assert lib.tqfx4_gemv_x(None, 1024, 1280, None, None, None, None, None, None, 0, None) == 2
     assert lib.tqfx4_gemv_x(None, 1024, 1024, None, None, None, None, None, None, 0, None) == 1
+    # the host-buffer MoE call: staging after the decode layout; NULL host
+    # buffers and bad shapes are refused before any copy
+    exh, rth = shapes()
+    nh = lib.tqfx4_moe_ffn_host_workspace_bytes(C.byref(exh), C.byref(rth))
+    assert nh >= 2 * 4 * 4096 + 2 * 4 * 8 and nh % 256 == 0
+    assert lib.tqfx4_moe_ffn_host_workspace_bytes(C.byref(ex_bad_h := shapes(H=4000)[0]), C.byref(rth)) == 0
+    assert lib.tqfx4_moe_ffn_host(C.byref(exh), C.byref(rth), None, None, None, None, None, 0, None) == 1
+    assert lib.tqfx4_moe_ffn_host(C.byref(ex_bad_h), C.byref(rth), None, None, None, None, None, 0, None) == 2
     assert lib.tqfx4_pack(7, None, None, None, 4, 256, None, None, 0, None) == 1  # unknown source kind
     ex, rt = shapes()
     assert lib.tqfx4_moe_ffn(C.byref(ex), C.byref(rt), None, None, None, None, None, 0, None) == 1

@@ -146,6 +146,35 @@ def test_moe_decode_many_calls_in_a_row(full_layer):
         assert torch.equal(o, ref[c % 2][0])
 
 
+@pytest.mark.parametrize("pinned", [True, False])
+def test_moe_ffn_host_equals_the_device_call(full_layer, pinned):
+    # the host-buffer entry point copies x in and out, sel_idx and sel_w back
+    # on the stream: the same bits as the device call, token after token on one
+    # workspace, with page-locked and with pageable host buffers
+    X = inputs.hidden_states(7, 4, 4096)
+    ws = full_layer.workspace(1)
+    wsh = full_layer.host_workspace()
+    stream = torch.cuda.current_stream()
+    for t in range(X.shape[0]):
+        ref = [v.cpu() for v in full_layer.ffn(X[t].to(DEV), ws)]
+        xh = X[t].clone().pin_memory() if pinned else X[t].clone()
+        outh = torch.empty(4096).pin_memory() if pinned else torch.empty(4096)
+        selh = torch.empty(8, dtype=torch.int32)
+        wh = torch.empty(8)
+        full_layer.ffn_host(xh, wsh, outh, selh, wh, stream=stream)
+        stream.synchronize()
+        B.tqfx4_check(wsh)
+        assert torch.equal(outh.view(torch.int32), ref[0].view(torch.int32)), t
+        assert torch.equal(selh, ref[1]), t
+        assert torch.equal(wh.view(torch.int32), ref[2].view(torch.int32)), t
+    # the selection outputs are optional
+    outh = torch.empty(4096).pin_memory()
+    full_layer.ffn_host(X[0].clone().pin_memory(), wsh, outh, None, None, stream=stream)
+    stream.synchronize()
+    ref0 = full_layer.ffn(X[0].to(DEV), ws)[0].cpu()
+    assert torch.equal(outh.view(torch.int32), ref0.view(torch.int32))
+
+
 def test_moe_top_k_equals_n_experts():
     layer = MoeLayer.synthetic(3, 4, 256, 256, 4, 0.0, DEV)
     run_and_check(layer, 3, inputs.hidden_states(3, 2, 256))
