@@ -295,15 +295,19 @@ size_t tqfx4_moe_ffn_host_workspace_bytes(const tqfx4_experts *ex, const tqfx4_r
 
 /*
  * tqfx4_moe_ffn_host -- tqfx4_moe_ffn for a token in host memory (Sec. 2.2,
- * the serving call with its copies): x_host (fp32 [hidden]) is copied into
- * the workspace's staging, the layer runs, and out (fp32 [hidden]) and, when
+ * the serving call with its transfers): x_host (fp32 [hidden]) reaches the
+ * workspace's staging, the layer runs, and out (fp32 [hidden]) and, when
  * their pointers are not NULL, sel_idx (int32 [top_k]) and sel_w (fp32
- * [top_k]) are copied back, all ordered on `stream` with one copy each. The
- * call returns once the work is enqueued: the host buffers must stay valid,
- * and the outputs are complete only after the stream has passed them
- * (synchronize before reading). Page-locked host buffers make the copies
- * asynchronous; pageable ones make the call wait for them. The results equal
- * tqfx4_moe_ffn's bit for bit. Workspace: tqfx4_moe_ffn_host_workspace_bytes.
+ * [top_k]) reach host memory, all ordered on `stream`. Page-locked host
+ * buffers (16-byte aligned x, 4-byte aligned outputs) are used in place
+ * through their device addresses: a small kernel reads x and the layer
+ * writes out and the selection directly, with no copy-engine transfer.
+ * Pageable or unaligned ones go through the staging with one
+ * cudaMemcpyAsync each (which makes the call wait for them). The call
+ * returns once the work is enqueued: the host buffers must stay valid, and
+ * the outputs are complete only after the stream has passed them
+ * (synchronize before reading). The results equal tqfx4_moe_ffn's bit for
+ * bit. Workspace: tqfx4_moe_ffn_host_workspace_bytes.
  * Errors: as tqfx4_moe_ffn, and TQFX4_EINVAL for a NULL x_host or out_host.
  */
 tqfx4_status tqfx4_moe_ffn_host(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x_host,

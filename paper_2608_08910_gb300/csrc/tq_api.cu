@@ -336,6 +336,18 @@ size_t tqfx4_moe_ffn_host_workspace_bytes(const tqfx4_experts *ex, const tqfx4_r
     return host_staging(ex, rt).total;
 }
 
+// The device address of page-locked host memory (the same pointer under
+// unified addressing), or null for pageable memory or an unaligned pointer.
+static void *mapped(const void *host, size_t align) {
+    if (!host || reinterpret_cast<uintptr_t>(host) % align) return nullptr;
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, host) != cudaSuccess) {
+        cudaGetLastError();  // not sticky: clear it for the launches that follow
+        return nullptr;
+    }
+    return at.type == cudaMemoryTypeHost ? at.devicePointer : nullptr;
+}
+
 tqfx4_status tqfx4_moe_ffn_host(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x_host,
                                 float *out_host, int32_t *sel_idx_host, float *sel_w_host, void *ws, size_t ws_bytes,
                                 void *stream) {
@@ -353,12 +365,22 @@ tqfx4_status tqfx4_moe_ffn_host(const tqfx4_experts *ex, const tqfx4_router *rt,
     float *wd = reinterpret_cast<float *>(base + h.selw);
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const size_t xb = 4 * static_cast<size_t>(ex->hidden), kb = 4 * static_cast<size_t>(rt->top_k);
-    cudaError_t e = cudaMemcpyAsync(xd, x_host, xb, cudaMemcpyHostToDevice, st);
+    // Page-locked host buffers are used in place: x is read into the staging
+    // by a small kernel and the layer writes out and the selection straight
+    // into host memory, with no copy engine round trip. Pageable ones go
+    // through the staging with cudaMemcpyAsync.
+    const float *xm = static_cast<const float *>(mapped(x_host, 16));
+    float *om = static_cast<float *>(mapped(out_host, 4));
+    int32_t *sm = static_cast<int32_t *>(mapped(sel_idx_host, 4));
+    float *wm = static_cast<float *>(mapped(sel_w_host, 4));
+    cudaError_t e = xm ? tq::launch_copy_f32(xd, xm, ex->hidden, st)
+                       : cudaMemcpyAsync(xd, x_host, xb, cudaMemcpyHostToDevice, st);
     if (e != cudaSuccess) return cuda_fail(e, fn);
-    if ((s = moe_ffn_impl(ex, rt, xd, od, sd, wd, ws, ws_bytes, stream, nullptr))) return s;
-    e = cudaMemcpyAsync(out_host, od, xb, cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess && sel_idx_host) e = cudaMemcpyAsync(sel_idx_host, sd, kb, cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess && sel_w_host) e = cudaMemcpyAsync(sel_w_host, wd, kb, cudaMemcpyDeviceToHost, st);
+    if ((s = moe_ffn_impl(ex, rt, xd, om ? om : od, sm ? sm : sd, wm ? wm : wd, ws, ws_bytes, stream, nullptr)))
+        return s;
+    if (!om) e = cudaMemcpyAsync(out_host, od, xb, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && sel_idx_host && !sm) e = cudaMemcpyAsync(sel_idx_host, sd, kb, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && sel_w_host && !wm) e = cudaMemcpyAsync(sel_w_host, wd, kb, cudaMemcpyDeviceToHost, st);
     if (e != cudaSuccess) return cuda_fail(e, fn);
     return ok();
 }

@@ -27,6 +27,7 @@ tqfx4_status api_fail(tqfx4_status s, const char *msg);
 struct MoeArgs;
 struct MoeLayout;
 bool moe_decode_args(const tqfx4_experts *ex, const tqfx4_router *rt, void *ws, MoeArgs &a, MoeLayout &L);
+cudaError_t launch_copy_f32(float *dst, const float *src, int64_t n, cudaStream_t st);
 cudaError_t launch_moe_decode(const MoeArgs &a, const float *x, float *out, int32_t *sel_idx, float *sel_w,
                               cudaStream_t st, void *const *events);
 int gate_up_smem(const MoeArgs &a);

@@ -452,6 +452,20 @@ cudaError_t launch_moe_decode(const MoeArgs &a0, const float *x, float *out, int
     return cudaSuccess;
 }
 
+// n fp32 values (both ends 16-byte aligned, n a multiple of 4) from src to
+// dst; src may be page-locked host memory seen through its device address.
+__global__ void __launch_bounds__(256) copy_f32_kernel(float4 *dst, const float4 *__restrict__ src, int n4) {
+    const int i = blockIdx.x * 256 + threadIdx.x;
+    if (i < n4) dst[i] = src[i];
+}
+
+cudaError_t launch_copy_f32(float *dst, const float *src, int64_t n, cudaStream_t st) {
+    const int n4 = static_cast<int>(n / 4);
+    copy_f32_kernel<<<(n4 + 255) / 256, 256, 0, st>>>(reinterpret_cast<float4 *>(dst),
+                                                       reinterpret_cast<const float4 *>(src), n4);
+    return cudaGetLastError();
+}
+
 // The two halves of launch_moe_decode for callers that place the selected
 // experts' blocks themselves between routing and the expert projections
 // (an expert tier): the router alone (selection and routing weights), then

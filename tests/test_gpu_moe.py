@@ -146,21 +146,34 @@ def test_moe_decode_many_calls_in_a_row(full_layer):
         assert torch.equal(o, ref[c % 2][0])
 
 
-@pytest.mark.parametrize("pinned", [True, False])
-def test_moe_ffn_host_equals_the_device_call(full_layer, pinned):
-    # the host-buffer entry point copies x in and out, sel_idx and sel_w back
-    # on the stream: the same bits as the device call, token after token on one
-    # workspace, with page-locked and with pageable host buffers
+def host_buffer(v, kind):
+    """v in host memory: page-locked, pageable, or page-locked 4 bytes off
+    16-byte alignment."""
+    if kind == "pinned":
+        return v.clone().pin_memory()
+    if kind == "pageable":
+        return v.clone()
+    buf = torch.empty(v.numel() + 1, dtype=v.dtype).pin_memory()
+    buf[1:] = v
+    return buf[1:]
+
+
+@pytest.mark.parametrize("kind", ["pinned", "pageable", "pinned_unaligned"])
+def test_moe_ffn_host_equals_the_device_call(full_layer, kind):
+    # the host-buffer entry point brings x in and out, sel_idx and sel_w back
+    # on the stream (page-locked buffers in place, the others through staging
+    # copies): the same bits as the device call, token after token on one
+    # workspace
     X = inputs.hidden_states(7, 4, 4096)
     ws = full_layer.workspace(1)
     wsh = full_layer.host_workspace()
     stream = torch.cuda.current_stream()
     for t in range(X.shape[0]):
         ref = [v.cpu() for v in full_layer.ffn(X[t].to(DEV), ws)]
-        xh = X[t].clone().pin_memory() if pinned else X[t].clone()
-        outh = torch.empty(4096).pin_memory() if pinned else torch.empty(4096)
-        selh = torch.empty(8, dtype=torch.int32)
-        wh = torch.empty(8)
+        xh = host_buffer(X[t], kind)
+        outh = host_buffer(torch.zeros(4096), kind)
+        selh = host_buffer(torch.zeros(8, dtype=torch.int32), kind)
+        wh = host_buffer(torch.zeros(8), kind)
         full_layer.ffn_host(xh, wsh, outh, selh, wh, stream=stream)
         stream.synchronize()
         B.tqfx4_check(wsh)
