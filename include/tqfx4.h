@@ -175,6 +175,22 @@ tqfx4_status tqfx4_gemv_x(const void *blocks, int64_t n, int64_t k, const float 
                           int8_t *q, float *da, int32_t *bsum,
                           void *ws, size_t ws_bytes, void *stream);
 
+/* Workspace bytes for tqfx4_gemv_x_host: the status word, then staging for x
+ * and y. 0 for shapes tqfx4_gemv_x refuses. */
+size_t tqfx4_gemv_x_host_workspace_bytes(int64_t n, int64_t k);
+
+/*
+ * tqfx4_gemv_x_host -- tqfx4_gemv_x with x (fp32 [k]) and y (fp32 [n]) in
+ * host memory, ordered on `stream` (Sec. 2.2). Page-locked buffers (x 16-byte
+ * and y 4-byte aligned) are used in place through their device addresses:
+ * the kernel reads x and writes y directly. Pageable or unaligned ones go
+ * through the workspace's staging with one cudaMemcpyAsync each. Returns once
+ * enqueued; y is complete after the stream has passed the call. y equals
+ * tqfx4_gemv_x's bit for bit. Errors: as tqfx4_gemv_x.
+ */
+tqfx4_status tqfx4_gemv_x_host(const void *blocks, int64_t n, int64_t k, const float *x_host, float *y_host,
+                               void *ws, size_t ws_bytes, void *stream);
+
 /*
  * The free-scale two-plane format (Table 1's free-scale K=2 row, 4.125
  * bits/weight; the ablation of the tie of Sec. 2.1): W = a1 t1 + a2 t2 per
@@ -435,6 +451,23 @@ size_t tqfx4_expert_ffn_workspace_bytes(int64_t hidden, int64_t inter);
 tqfx4_status tqfx4_expert_ffn(const void *gate, const void *up, const void *down,
                               int64_t hidden, int64_t inter, const float *x, float *out,
                               void *ws, size_t ws_bytes, void *stream);
+
+/* Workspace bytes for tqfx4_expert_ffn_host: tqfx4_expert_ffn's, then
+ * staging for x and out. 0 if the shapes are invalid. */
+size_t tqfx4_expert_ffn_host_workspace_bytes(int64_t hidden, int64_t inter);
+
+/*
+ * tqfx4_expert_ffn_host -- tqfx4_expert_ffn with x and out (fp32 [hidden])
+ * in host memory, ordered on `stream`. A page-locked x (16-byte aligned) is
+ * read into the staging by a small kernel and a page-locked out (4-byte
+ * aligned) is written in place by the down kernel; pageable or unaligned
+ * buffers go through the staging with one cudaMemcpyAsync each. Returns once
+ * enqueued; out is complete after the stream has passed the call. out equals
+ * tqfx4_expert_ffn's bit for bit. Errors: as tqfx4_expert_ffn.
+ */
+tqfx4_status tqfx4_expert_ffn_host(const void *gate, const void *up, const void *down, int64_t hidden,
+                                   int64_t inter, const float *x_host, float *out_host, void *ws, size_t ws_bytes,
+                                   void *stream);
 tqfx4_status tqfx4_expert_ffn_traced(const void *gate, const void *up, const void *down,
                                      int64_t hidden, int64_t inter, const float *x, float *out,
                                      void *ws, size_t ws_bytes, void *stream, void *const *events);

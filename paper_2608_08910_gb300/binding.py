@@ -66,6 +66,10 @@ _SIGS = {
     "tqfx4_moe_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int]),
     "tqfx4_moe_ffn": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_ffn_host": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_gemv_x_host": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_gemv_x_host_workspace_bytes": (_sz, [_i64, _i64]),
+    "tqfx4_expert_ffn_host": (_int, [_vp, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_expert_ffn_host_workspace_bytes": (_sz, [_i64, _i64]),
     "tqfx4_moe_ffn_host_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter)]),
     "tqfx4_moe_ffn_mxfp4": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_moe_ffn_mxfp4_traced": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz,
@@ -206,6 +210,28 @@ def tqfx4_moe_ffn(ex, rt, x, out, sel_idx, sel_w, ws, stream=None, events=None):
         rc = lib().tqfx4_moe_ffn_traced(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w),
                                         _p(ws), _nbytes(ws), _s(stream), arr)
     _check(rc, "tqfx4_moe_ffn")
+
+
+def tqfx4_gemv_x_host_workspace_bytes(n: int, k: int) -> int:
+    return int(lib().tqfx4_gemv_x_host_workspace_bytes(n, k))
+
+
+def tqfx4_gemv_x_host(blocks, n, k, x, y, ws, stream=None):
+    """x, y: CPU tensors (page-locked: used in place); y is complete once
+    `stream` has passed the call."""
+    _check(lib().tqfx4_gemv_x_host(_p(blocks), n, k, _p(x), _p(y), _p(ws), _nbytes(ws), _s(stream)),
+           "tqfx4_gemv_x_host")
+
+
+def tqfx4_expert_ffn_host_workspace_bytes(hidden: int, inter: int) -> int:
+    return int(lib().tqfx4_expert_ffn_host_workspace_bytes(hidden, inter))
+
+
+def tqfx4_expert_ffn_host(gate, up, down, hidden, inter, x, out, ws, stream=None):
+    """x, out: CPU tensors (page-locked: used in place); out is complete once
+    `stream` has passed the call."""
+    _check(lib().tqfx4_expert_ffn_host(_p(gate), _p(up), _p(down), hidden, inter, _p(x), _p(out), _p(ws),
+                                       _nbytes(ws), _s(stream)), "tqfx4_expert_ffn_host")
 
 
 def tqfx4_moe_ffn_host_workspace_bytes(ex: CExperts, rt: CRouter) -> int:

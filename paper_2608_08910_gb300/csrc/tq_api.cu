@@ -40,6 +40,19 @@ tqfx4_status ok() {
 
 bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+// The device address of page-locked host memory (the same pointer under
+// unified addressing), or null for pageable memory or an unaligned pointer.
+static void *mapped(const void *host, size_t align) {
+    if (!host || reinterpret_cast<uintptr_t>(host) % align) return nullptr;
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, host) != cudaSuccess) {
+        cudaGetLastError();  // not sticky: clear it for the launches that follow
+        return nullptr;
+    }
+    return at.type == cudaMemoryTypeHost ? at.devicePointer : nullptr;
+}
+
+
 tqfx4_status cuda_fail(cudaError_t e, const char *what) {
     return fail(TQFX4_ECUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
 }
@@ -156,6 +169,42 @@ tqfx4_status tqfx4_gemv_x(const void *blocks, int64_t n, int64_t k, const float 
         return fail(TQFX4_EALIGN, "%s: blocks, x and q must be 16-byte aligned", fn);
     cudaError_t e = tq::launch_gemv_x(blocks, n, k, x, q, da, bsum, y, static_cast<int *>(ws),
                                       static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
+size_t tqfx4_gemv_x_host_workspace_bytes(int64_t n, int64_t k) {
+    if (n < 0 || k <= 0 || k % 512 || k > TQFX4_MAX_K || n % 4) return 0;
+    return tq::align256(tq::align256(TQFX4_STATUS_BYTES + 4 * static_cast<size_t>(k)) + 4 * static_cast<size_t>(n));
+}
+
+tqfx4_status tqfx4_gemv_x_host(const void *blocks, int64_t n, int64_t k, const float *x_host, float *y_host,
+                               void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
+    const char *fn = "tqfx4_gemv_x_host";
+    tqfx4_status s = check_nk(n, k, fn);
+    if (s) return s;
+    const size_t need = tqfx4_gemv_x_host_workspace_bytes(n, k);
+    if (need == 0)
+        return fail(TQFX4_ESHAPE, "%s: k=%lld must be a multiple of 512 in 512..%d", fn, (long long)k, TQFX4_MAX_K);
+    if ((s = check_ws(ws, ws_bytes, need, fn))) return s;
+    if (n == 0) return ok();
+    if (!blocks || !x_host || !y_host) return fail(TQFX4_EINVAL, "%s: NULL input or output", fn);
+    // page-locked buffers in place (the kernel reads x and writes y through
+    // their device addresses); others through staging after the status word
+    uint8_t *base = static_cast<uint8_t *>(ws);
+    float *xd = reinterpret_cast<float *>(base + TQFX4_STATUS_BYTES);
+    float *yd = reinterpret_cast<float *>(base + tq::align256(TQFX4_STATUS_BYTES + 4 * static_cast<size_t>(k)));
+    const float *xm = static_cast<const float *>(mapped(x_host, 16));
+    float *ym = static_cast<float *>(mapped(y_host, 4));
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaSuccess;
+    if (!xm) e = cudaMemcpyAsync(xd, x_host, 4 * static_cast<size_t>(k), cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    if ((s = tqfx4_gemv_x(blocks, n, k, xm ? xm : xd, ym ? ym : yd, nullptr, nullptr, nullptr, ws, ws_bytes,
+                          stream)))
+        return s;
+    if (!ym) e = cudaMemcpyAsync(y_host, yd, 4 * static_cast<size_t>(n), cudaMemcpyDeviceToHost, st);
     if (e != cudaSuccess) return cuda_fail(e, fn);
     return ok();
 }
@@ -336,18 +385,6 @@ size_t tqfx4_moe_ffn_host_workspace_bytes(const tqfx4_experts *ex, const tqfx4_r
     return host_staging(ex, rt).total;
 }
 
-// The device address of page-locked host memory (the same pointer under
-// unified addressing), or null for pageable memory or an unaligned pointer.
-static void *mapped(const void *host, size_t align) {
-    if (!host || reinterpret_cast<uintptr_t>(host) % align) return nullptr;
-    cudaPointerAttributes at;
-    if (cudaPointerGetAttributes(&at, host) != cudaSuccess) {
-        cudaGetLastError();  // not sticky: clear it for the launches that follow
-        return nullptr;
-    }
-    return at.type == cudaMemoryTypeHost ? at.devicePointer : nullptr;
-}
-
 tqfx4_status tqfx4_moe_ffn_host(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x_host,
                                 float *out_host, int32_t *sel_idx_host, float *sel_w_host, void *ws, size_t ws_bytes,
                                 void *stream) {
@@ -427,6 +464,43 @@ tqfx4_status tqfx4_expert_ffn_traced(const void *gate, const void *up, const voi
                                      void *stream, void *const *events) {
     TQ_RANGE();
     return expert_ffn_impl(gate, up, down, hidden, inter, x, out, ws, ws_bytes, stream, events);
+}
+
+size_t tqfx4_expert_ffn_host_workspace_bytes(int64_t hidden, int64_t inter) {
+    const size_t base = tqfx4_expert_ffn_workspace_bytes(hidden, inter);
+    if (base == 0) return 0;
+    return tq::align256(tq::align256(tq::align256(base) + 4 * static_cast<size_t>(hidden)) +
+                        4 * static_cast<size_t>(hidden));
+}
+
+tqfx4_status tqfx4_expert_ffn_host(const void *gate, const void *up, const void *down, int64_t hidden,
+                                   int64_t inter, const float *x_host, float *out_host, void *ws, size_t ws_bytes,
+                                   void *stream) {
+    TQ_RANGE();
+    const char *fn = "tqfx4_expert_ffn_host";
+    const size_t base = tqfx4_expert_ffn_workspace_bytes(hidden, inter);
+    if (base == 0) return fail(TQFX4_ESHAPE, "%s: hidden and inter must be positive multiples of 256", fn);
+    const size_t need = tqfx4_expert_ffn_host_workspace_bytes(hidden, inter);
+    if (!gate || !up || !down || !x_host || !out_host)
+        return fail(TQFX4_EINVAL, "%s: NULL matrix, input or output", fn);
+    tqfx4_status s = check_ws(ws, ws_bytes, need, fn);
+    if (s) return s;
+    uint8_t *b = static_cast<uint8_t *>(ws);
+    const size_t xo = tq::align256(base), oo = tq::align256(xo + 4 * static_cast<size_t>(hidden));
+    float *xd = reinterpret_cast<float *>(b + xo), *od = reinterpret_cast<float *>(b + oo);
+    // page-locked buffers in place: a small kernel reads x into the staging
+    // and the down kernel writes out straight into host memory
+    const float *xm = static_cast<const float *>(mapped(x_host, 16));
+    float *om = static_cast<float *>(mapped(out_host, 4));
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t hb = 4 * static_cast<size_t>(hidden);
+    cudaError_t e = xm ? tq::launch_copy_f32(xd, xm, hidden, st) : cudaMemcpyAsync(xd, x_host, hb, cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    if ((s = expert_ffn_impl(gate, up, down, hidden, inter, xd, om ? om : od, ws, ws_bytes, stream, nullptr)))
+        return s;
+    if (!om) e = cudaMemcpyAsync(out_host, od, hb, cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
 }
 
 tqfx4_status tqfx4_moe_route(const tqfx4_experts *ex, const tqfx4_router *rt, const float *x, int32_t *sel_idx,

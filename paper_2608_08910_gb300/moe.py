@@ -92,6 +92,22 @@ class MoeLayer:
         B.tqfx4_expert_ffn(g, u, d, self.hidden, self.inter, x, out, ws, stream, events)
         return out
 
+    def expert_host_workspace(self) -> torch.Tensor:
+        """A zeroed workspace for expert_ffn_host."""
+        n = B.tqfx4_expert_ffn_host_workspace_bytes(self.hidden, self.inter)
+        if n == 0:
+            raise ValueError("invalid expert shapes")
+        return torch.zeros(n, dtype=torch.uint8, device=self.gate.device)
+
+    def expert_ffn_host(self, e: int, x, ws, out, stream=None):
+        """expert_ffn with x and out in host memory (CPU tensors, page-locked
+        ones used in place); out is complete once `stream` has passed it."""
+        if self.fmt != "fx4":
+            raise ValueError("expert_ffn serves tq2_0_fx4 experts")
+        g, u, d = self.expert_blocks(e)
+        B.tqfx4_expert_ffn_host(g, u, d, self.hidden, self.inter, x, out, ws, stream)
+        return out
+
     def ffn(self, x, ws, out=None, sel_idx=None, sel_w=None, stream=None, events=None):
         dev = x.device
         out = torch.empty(self.hidden, dtype=torch.float32, device=dev) if out is None else out

@@ -61,6 +61,21 @@ def gemv(blocks, n: int, k: int, q, da, bsum, ws, block_sums: bool = False):
     return (y, S) if block_sums else y
 
 
+def gemv_x_host_workspace(n: int, k: int, device="cuda"):
+    """The workspace of gemv_x_host (device memory)."""
+    nb = B.tqfx4_gemv_x_host_workspace_bytes(n, k)
+    if nb == 0:
+        raise ValueError("gemv_x_host: k must be a positive multiple of 512 and n of 4")
+    return torch.zeros(nb, dtype=torch.uint8, device=device)
+
+
+def gemv_x_host(blocks, n: int, k: int, x, y, ws, stream=None):
+    """y = W x with x and y in host memory (CPU tensors; page-locked ones are
+    used in place); y is complete once `stream` has passed the call."""
+    B.tqfx4_gemv_x_host(blocks, n, k, x, y, ws, stream)
+    return y
+
+
 def gemv_x(blocks, n: int, k: int, x, ws, quantized: bool = False):
     """y = W x for an fp32 x, quantized inside the same launch; with
     quantized=True also returns the quantized vector (q, da, bsum)."""

@@ -117,6 +117,17 @@ def test_host_validation_rejects_bad_arguments(lib):
     assert lib.tqfx4_moe_ffn_host_workspace_bytes(C.byref(ex_bad_h := shapes(H=4000)[0]), C.byref(rth)) == 0
     assert lib.tqfx4_moe_ffn_host(C.byref(exh), C.byref(rth), None, None, None, None, None, 0, None) == 1
     assert lib.tqfx4_moe_ffn_host(C.byref(ex_bad_h), C.byref(rth), None, None, None, None, None, 0, None) == 2
+    # the host-buffer GEMV and expert FFN: status word and staging; shape and
+    # NULL errors before any copy
+    assert lib.tqfx4_gemv_x_host_workspace_bytes(1024, 1024) >= B.TQFX4_STATUS_BYTES + 8 * 1024
+    assert lib.tqfx4_gemv_x_host_workspace_bytes(1024, 256) == 0
+    assert lib.tqfx4_gemv_x_host(None, 1024, 256, None, None, None, 0, None) == 2
+    assert lib.tqfx4_gemv_x_host(None, 1024, 1024, None, None, None, 0, None) == 1  # workspace first
+    ne = lib.tqfx4_expert_ffn_host_workspace_bytes(4096, 2048)
+    assert ne >= lib.tqfx4_expert_ffn_workspace_bytes(4096, 2048) + 2 * 4 * 4096
+    assert lib.tqfx4_expert_ffn_host_workspace_bytes(4000, 2048) == 0
+    assert lib.tqfx4_expert_ffn_host(None, None, None, 4000, 2048, None, None, None, 0, None) == 2
+    assert lib.tqfx4_expert_ffn_host(None, None, None, 4096, 2048, None, None, None, 0, None) == 1
     assert lib.tqfx4_pack(7, None, None, None, 4, 256, None, None, 0, None) == 1  # unknown source kind
     ex, rt = shapes()
     assert lib.tqfx4_moe_ffn(C.byref(ex), C.byref(rt), None, None, None, None, None, 0, None) == 1

@@ -252,6 +252,36 @@ def test_gemv_x_1024_benchmark_inputs(ws):
     assert rel_err(y.cpu().numpy(), ry) <= FP32_TOL
 
 
+def _host(v, kind):
+    """v in host memory: page-locked, pageable, or page-locked 4 bytes off
+    16-byte alignment."""
+    if kind == "pinned":
+        return v.clone().pin_memory()
+    if kind == "pageable":
+        return v.clone()
+    buf = torch.empty(v.numel() + 1, dtype=v.dtype).pin_memory()
+    buf[1:] = v
+    return buf[1:]
+
+
+@pytest.mark.parametrize("kind", ["pinned", "pageable", "pinned_unaligned"])
+@pytest.mark.parametrize("n,k", [(1024, 1024), (2048, 4096), (36, 512)])
+def test_gemv_x_host_equals_the_device_call(n, k, kind, ws):
+    # x and y in host memory (page-locked ones used in place by the kernel,
+    # the others through staging copies): y bit-identical to gemv_x's
+    blocks = ops.pack_rtn(_w(n, k, 5 * n + k).to(DEV), ws)
+    wsh = ops.gemv_x_host_workspace(n, k)
+    stream = torch.cuda.current_stream()
+    for t in range(3):
+        x = inputs.hidden_states(n + k + t, 1, k)[0]
+        ref = ops.gemv_x(blocks, n, k, x.to(DEV), ws).cpu()
+        xh, yh = _host(x, kind), _host(torch.zeros(n), kind)
+        ops.gemv_x_host(blocks, n, k, xh, yh, wsh, stream)
+        stream.synchronize()
+        B.tqfx4_check(wsh)
+        assert torch.equal(yh.view(torch.int32), ref.view(torch.int32)), t
+
+
 def test_gemv_x_reports_nonfinite_activation(ws):
     n, k = 64, 1024
     blocks = ops.pack_rtn(_w(n, k, 1).to(DEV), ws)

@@ -188,6 +188,25 @@ def test_moe_ffn_host_equals_the_device_call(full_layer, kind):
     assert torch.equal(outh.view(torch.int32), ref0.view(torch.int32))
 
 
+@pytest.mark.parametrize("kind", ["pinned", "pageable", "pinned_unaligned"])
+def test_expert_ffn_host_equals_the_device_call(kind):
+    # x and out in host memory (page-locked: x read by a small kernel, out
+    # written in place by the down kernel; others through staging copies):
+    # out bit-identical to expert_ffn's, 4 tokens on one workspace
+    layer = MoeLayer.synthetic(31, 1, 4096, 2048, 1, 0.0, DEV)
+    ws = layer.expert_workspace()
+    wsh = layer.expert_host_workspace()
+    stream = torch.cuda.current_stream()
+    X = inputs.hidden_states(31, 4, 4096)
+    for t in range(X.shape[0]):
+        ref = layer.expert_ffn(0, X[t].to(DEV), ws).cpu()
+        xh, oh = host_buffer(X[t], kind), host_buffer(torch.zeros(4096), kind)
+        layer.expert_ffn_host(0, xh, wsh, oh, stream=stream)
+        stream.synchronize()
+        B.tqfx4_check(wsh)
+        assert torch.equal(oh.view(torch.int32), ref.view(torch.int32)), t
+
+
 def test_moe_top_k_equals_n_experts():
     layer = MoeLayer.synthetic(3, 4, 256, 256, 4, 0.0, DEV)
     run_and_check(layer, 3, inputs.hidden_states(3, 2, 256))
