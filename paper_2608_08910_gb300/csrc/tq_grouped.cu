@@ -781,7 +781,7 @@ __global__ void __launch_bounds__(256) gather_tc_kernel(GroupedArgs a) {
             uint4 *dst = reinterpret_cast<uint4 *>(a.xq + pl * plane + pos * a.H);
             for (int i = lane; i < n16; i += 32) dst[i] = __ldcg(src + i);
         }
-        if (lane == 0) a.pair_chunk[pos] = c;
+        if (lane == 0) a.pair_hs[pos] = c * a.nbi * 2 * TC_CHUNK + n;
     }
     for (int i = threadIdx.x; i < a.nbh * GT_PAIRS; i += blockDim.x) {
         const int b = i / GT_PAIRS, n = n0 + (i - b * GT_PAIRS);
@@ -806,6 +806,8 @@ __global__ void __launch_bounds__(256) swiglu_quant_kernel(GroupedArgs a) {
     const int64_t p = unit / a.nbi;
     const int b = static_cast<int>(unit - p * a.nbi);
     const int64_t o = p * a.I + b * QK + 8 * lane;
+    // the pair's scale slot, loaded with g and u (used at the end)
+    const int hsb = (a.tc && lane == 0) ? __ldcg(a.pair_hs + p) : 0;
     const float4 g0 = __ldcg(reinterpret_cast<const float4 *>(a.g + o));
     const float4 g1 = __ldcg(reinterpret_cast<const float4 *>(a.g + o) + 1);
     const float4 u0 = __ldcg(reinterpret_cast<const float4 *>(a.u + o));
@@ -826,11 +828,9 @@ __global__ void __launch_bounds__(256) swiglu_quant_kernel(GroupedArgs a) {
         *reinterpret_cast<uint2 *>(a.hq + o) = hi;
         *reinterpret_cast<uint2 *>(a.hq + static_cast<int64_t>(a.P) * a.I + o) = lo;
         if (lane == 0) {
-            const int c = __ldcg(a.pair_chunk + p);
-            const int n = static_cast<int>(p - __ldcg(a.chunk_begin + c));
-            float *hs = a.hs + (static_cast<int64_t>(c) * a.nbi + b) * 2 * TC_CHUNK;
-            hs[n] = d;
-            hs[TC_CHUNK + n] = static_cast<float>(-4 * sum);
+            float *hs = a.hs + hsb + static_cast<int64_t>(b) * 2 * TC_CHUNK;
+            hs[0] = d;
+            hs[TC_CHUNK] = static_cast<float>(-4 * sum);
         }
     }
     if (a.keep_h) {
@@ -1002,7 +1002,7 @@ bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, vo
         a.xq = base + L.xq;
         a.xqt = base + L.xqt;
         a.hq = base + L.hq;
-        a.pair_chunk = reinterpret_cast<int *>(base + L.pair_chunk);
+        a.pair_hs = reinterpret_cast<int *>(base + L.pair_hs);
         a.xs = reinterpret_cast<float *>(base + L.xs);
         a.hs = reinterpret_cast<float *>(base + L.hs);
         a.rnorm = reinterpret_cast<float *>(base + L.rnorm);

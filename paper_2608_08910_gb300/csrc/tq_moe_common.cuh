@@ -26,7 +26,7 @@ struct MoeLayout {
     size_t tc_list, n_tc;  // int4 [max_chunks] (chunk, expert, begin, pairs) of the tensor-core launches' chunks, and their count (grouped only)
     size_t xq, hq;    // e4m3 activation planes [2][P][H], [2][P][I] for the tensor-core contraction (grouped only)
     size_t xqt;       // the same planes of x in token order [2][T][H] (grouped only)
-    size_t pair_chunk, xs, hs;  // tensor-core work list helpers (grouped only)
+    size_t pair_hs, xs, hs;  // tensor-core work list helpers (grouped only)
     size_t rnorm;     // fp32 [T + E]: Euclidean norms of the hidden states and router rows (grouped only)
     size_t rpart;     // fp32 [kScreenSplit][T][E]: partial router logits of the screening GEMM (grouped only)
     size_t rcand, rcount;  // int [T][E], [T]: each token's screened-in experts and their count (grouped only)
@@ -102,7 +102,7 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.xq = take(2 * static_cast<size_t>(P * H));
         L.hq = take(2 * static_cast<size_t>(P * I));
         L.xqt = take(2 * static_cast<size_t>(T * H));
-        L.pair_chunk = take(4 * static_cast<size_t>(P));
+        L.pair_hs = take(4 * static_cast<size_t>(P));
         L.rnorm = take(4 * static_cast<size_t>(T + E));
         L.rpart = take(4 * static_cast<size_t>(kScreenSplit) * T * E);
         L.rcand = take(4 * static_cast<size_t>(T) * E);
@@ -114,7 +114,7 @@ inline MoeLayout moe_layout(int64_t E, int64_t H, int64_t I, int64_t top_k, int6
         L.dxg = L.bxg = L.dhp = L.bhp = SIZE_MAX;
         L.chunk_expert = L.chunk_begin = L.chunk_len = L.n_chunks = SIZE_MAX;
         L.tc_list = L.n_tc = SIZE_MAX;
-        L.xq = L.hq = L.xqt = L.pair_chunk = L.xs = L.hs = L.rnorm = L.rpart = SIZE_MAX;
+        L.xq = L.hq = L.xqt = L.pair_hs = L.xs = L.hs = L.rnorm = L.rpart = SIZE_MAX;
         L.rcand = L.rcount = SIZE_MAX;
         L.max_chunks = 0;
     }
@@ -200,7 +200,7 @@ struct GroupedArgs {
                           // small-group pass instead of the tensor cores (0: none)
     uint8_t *xq, *hq;     // [2][P][H], [2][P][I]: e4m3 planes 16 h and l of q = 16 h + l (tensor-core path)
     uint8_t *xqt;         // [2][T][H]: the planes of the tokens' x, in token order (tensor-core path)
-    int *pair_chunk;      // [P] chunk of each pair (tensor-core path)
+    int *pair_hs;         // [P] each pair's block-0 scale slot in hs: chunk * nbi * 2 TC_CHUNK + place (tensor-core path)
     float *xs, *hs;       // [chunks][nb][2][TC_CHUNK]: per chunk and block, the pairs' scales da,
                           // then -4 bsum as float (tensor-core path)
     float *rnorm;         // [T + E] norms for the screened router
