@@ -145,6 +145,19 @@ tqfx4_status tqfx4_quantize_act(const float *x, int64_t m, int64_t k,
                                 void *ws, size_t ws_bytes, void *stream);
 
 /*
+ * tqfx4_validate_blocks -- checks an N x K tq2_0_fx4 matrix against the
+ * format (Sec. 2.2): every code nibble u is 0..8 (the nine levels c = u - 4)
+ * and every f16 row scale is finite. A violation records TQFX4_EDATA in the
+ * status word (tqfx4_check; the detail names a bad block), so a matrix from
+ * an outside source can be checked before it is served. The debug build
+ * (libtqfx4_debug.so, compiled with TQFX4_DEBUG) runs this check on every
+ * matrix the dot-pass entry points read, and checks data-dependent indices
+ * inside the kernels. blocks: device, 16-byte aligned.
+ */
+tqfx4_status tqfx4_validate_blocks(const void *blocks, int64_t n, int64_t k, void *ws, size_t ws_bytes,
+                                   void *stream);
+
+/*
  * tqfx4_gemv -- the integer dot pass (Sec. 2.2): y = W x for one activation
  * vector already quantized by tqfx4_quantize_act.
  *   blocks: device, the N x K matrix. q, da, bsum: device, one vector

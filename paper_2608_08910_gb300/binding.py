@@ -12,6 +12,7 @@ import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libtqfx4.so")
+DEBUG_LIB_PATH = os.path.join(_HERE, "libtqfx4_debug.so")  # the TQFX4_DEBUG build (build.build(debug=True))
 
 TQFX4_QK = 256
 TQFX4_ROWS = 4
@@ -65,6 +66,7 @@ _SIGS = {
     "tqfx4_expert_ffn_traced": (_int, [_vp, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp, _vp]),
     "tqfx4_moe_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int]),
     "tqfx4_moe_ffn": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "tqfx4_validate_blocks": (_int, [_vp, _i64, _i64, _vp, _sz, _vp]),
     "tqfx4_moe_ffn_host": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_gemv_x_host": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_gemv_x_host_workspace_bytes": (_sz, [_i64, _i64]),
@@ -101,18 +103,23 @@ _SIGS = {
 _lib = None
 
 
+def load(path: str):
+    """A library of this ABI at `path`, with every declared signature set."""
+    if not os.path.exists(path):
+        raise RuntimeError("%s is not built; run __graft_entry__.build()" % path)
+    L = C.CDLL(path)
+    for name, (res, args) in _SIGS.items():
+        f = getattr(L, name)  # a missing export is a build error: raise here
+        f.restype = res
+        f.argtypes = args
+    return L
+
+
 def lib():
     """Load libtqfx4.so (built in-tree by __graft_entry__.build())."""
     global _lib
     if _lib is None:
-        if not os.path.exists(LIB_PATH):
-            raise RuntimeError("libtqfx4.so is not built (%s); run __graft_entry__.build()" % LIB_PATH)
-        L = C.CDLL(LIB_PATH)
-        for name, (res, args) in _SIGS.items():
-            f = getattr(L, name)  # a missing export is a build error: raise here
-            f.restype = res
-            f.argtypes = args
-        _lib = L
+        _lib = load(LIB_PATH)
     return _lib
 
 
@@ -210,6 +217,12 @@ def tqfx4_moe_ffn(ex, rt, x, out, sel_idx, sel_w, ws, stream=None, events=None):
         rc = lib().tqfx4_moe_ffn_traced(C.byref(ex), C.byref(rt), _p(x), _p(out), _p(sel_idx), _p(sel_w),
                                         _p(ws), _nbytes(ws), _s(stream), arr)
     _check(rc, "tqfx4_moe_ffn")
+
+
+def tqfx4_validate_blocks(blocks, n, k, ws, stream=None):
+    """Checks the format of an n x k matrix (nibbles 0..8, finite scales); a
+    violation shows in tqfx4_check(ws) as TQFX4_EDATA."""
+    _check(lib().tqfx4_validate_blocks(_p(blocks), n, k, _p(ws), _nbytes(ws), _s(stream)), "tqfx4_validate_blocks")
 
 
 def tqfx4_gemv_x_host_workspace_bytes(n: int, k: int) -> int:

@@ -1,5 +1,8 @@
 """Build libtqfx4.so in-tree: every csrc/*.cu compiled for sm_103a with nvcc
-(in parallel), then linked into one shared library next to this file."""
+(in parallel), then linked into one shared library next to this file.
+build(debug=True) builds the debug variant libtqfx4_debug.so (TQFX4_DEBUG:
+format validation of every matrix an entry point reads, and checks of
+data-dependent indices inside the kernels)."""
 import concurrent.futures as cf
 import glob
 import os
@@ -13,6 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libtqfx4.so")
+LIB_DEBUG = os.path.join(PKG, "libtqfx4_debug.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -30,24 +34,25 @@ def _deps():
         [os.path.join(INCLUDE, "tqfx4.h"), os.path.abspath(__file__)]
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+def up_to_date(lib: str = LIB) -> bool:
+    if not os.path.exists(lib):
         return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(p) <= t for p in _deps())
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    if not force and up_to_date():
-        return LIB
-    os.makedirs(BUILD, exist_ok=True)
+def build(force: bool = False, verbose: bool = False, extra_flags=(), debug: bool = False) -> str:
+    lib, build_dir = (LIB_DEBUG, os.path.join(BUILD, "debug")) if debug else (LIB, BUILD)
+    if not force and up_to_date(lib):
+        return lib
+    os.makedirs(build_dir, exist_ok=True)
     nvcc = _nvcc()
     common = ["-std=c++17", "-O3", "-lineinfo", *ARCH, "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC,
-              "--expt-relaxed-constexpr", *extra_flags]
+              "--expt-relaxed-constexpr", *(["-DTQFX4_DEBUG"] if debug else []), *extra_flags]
     objs = []
 
     def compile_one(src):
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(build_dir, os.path.basename(src)[:-3] + ".o")
         cmd = [nvcc, *common, "-c", src, "-o", obj]
         if verbose:
             print(" ".join(cmd), flush=True)
@@ -61,16 +66,16 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
     srcs = _sources()
     with cf.ThreadPoolExecutor(max_workers=min(len(srcs), os.cpu_count() or 4)) as ex:
         objs = list(ex.map(compile_one, srcs))
-    tmp = LIB + ".tmp%d" % os.getpid()
+    tmp = lib + ".tmp%d" % os.getpid()
     cuda_lib = os.path.join(os.path.dirname(os.path.dirname(nvcc)), "lib64")
     cmd = [nvcc, "-shared", *ARCH, "-cudart", "shared", "-o", tmp, *objs,
            "-Xlinker", "-rpath," + cuda_lib]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError("link failed:\n%s%s" % (r.stdout, r.stderr))
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose="-v" in sys.argv))
+    print(build(force="--force" in sys.argv, verbose="-v" in sys.argv, debug="--debug" in sys.argv))

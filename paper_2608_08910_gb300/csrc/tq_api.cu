@@ -40,6 +40,19 @@ tqfx4_status ok() {
 
 bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+// The debug build (TQFX4_DEBUG) checks every tq2_0_fx4 matrix an entry point
+// reads against the format before its kernels run; the release build does
+// nothing here.
+cudaError_t debug_validate(const void *blocks, int64_t n, int64_t k, void *ws, void *stream) {
+#ifdef TQFX4_DEBUG
+    if (!blocks || n <= 0 || k <= 0) return cudaSuccess;
+    return tq::launch_validate(blocks, n, k, static_cast<int *>(ws), static_cast<cudaStream_t>(stream));
+#else
+    (void)blocks, (void)n, (void)k, (void)ws, (void)stream;
+    return cudaSuccess;
+#endif
+}
+
 // The device address of page-locked host memory (the same pointer under
 // unified addressing), or null for pageable memory or an unaligned pointer.
 static void *mapped(const void *host, size_t align) {
@@ -145,8 +158,10 @@ tqfx4_status tqfx4_gemv(const void *blocks, int64_t n, int64_t k, const int8_t *
     if (k > 0 && (!aligned(blocks, 16) || !aligned(q, 16) || !aligned(da, 4) || !aligned(bsum, 4)))
         return fail(TQFX4_EALIGN, "tqfx4_gemv: blocks and q must be 16-byte aligned");
     if (!aligned(y, 4) || !aligned(block_sums, 4)) return fail(TQFX4_EALIGN, "tqfx4_gemv: misaligned output");
-    cudaError_t e = tq::launch_gemv(blocks, n, k, q, da, bsum, y, block_sums, static_cast<int *>(ws),
-                                    static_cast<cudaStream_t>(stream));
+    cudaError_t e = debug_validate(blocks, n, k, ws, stream);
+    if (e == cudaSuccess)
+        e = tq::launch_gemv(blocks, n, k, q, da, bsum, y, block_sums, static_cast<int *>(ws),
+                            static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "tqfx4_gemv");
     return ok();
 }
@@ -167,8 +182,10 @@ tqfx4_status tqfx4_gemv_x(const void *blocks, int64_t n, int64_t k, const float 
     if (!aligned(blocks, 16) || !aligned(x, 16) || !aligned(y, 4) || !aligned(q, 16) || !aligned(da, 4) ||
         !aligned(bsum, 4))
         return fail(TQFX4_EALIGN, "%s: blocks, x and q must be 16-byte aligned", fn);
-    cudaError_t e = tq::launch_gemv_x(blocks, n, k, x, q, da, bsum, y, static_cast<int *>(ws),
-                                      static_cast<cudaStream_t>(stream));
+    cudaError_t e = debug_validate(blocks, n, k, ws, stream);
+    if (e == cudaSuccess)
+        e = tq::launch_gemv_x(blocks, n, k, x, q, da, bsum, y, static_cast<int *>(ws),
+                              static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, fn);
     return ok();
 }
@@ -205,6 +222,21 @@ tqfx4_status tqfx4_gemv_x_host(const void *blocks, int64_t n, int64_t k, const f
                           stream)))
         return s;
     if (!ym) e = cudaMemcpyAsync(y_host, yd, 4 * static_cast<size_t>(n), cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
+tqfx4_status tqfx4_validate_blocks(const void *blocks, int64_t n, int64_t k, void *ws, size_t ws_bytes,
+                                   void *stream) {
+    TQ_RANGE();
+    const char *fn = "tqfx4_validate_blocks";
+    tqfx4_status s = check_nk(n, k, fn);
+    if (s) return s;
+    if ((s = check_ws(ws, ws_bytes, TQFX4_STATUS_BYTES, fn))) return s;
+    if (n == 0 || k == 0) return ok();
+    if (!blocks) return fail(TQFX4_EINVAL, "%s: NULL blocks", fn);
+    if (!aligned(blocks, 16)) return fail(TQFX4_EALIGN, "%s: blocks must be 16-byte aligned", fn);
+    cudaError_t e = tq::launch_validate(blocks, n, k, static_cast<int *>(ws), static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, fn);
     return ok();
 }
@@ -344,7 +376,12 @@ static tqfx4_status moe_ffn_impl(const tqfx4_experts *ex, const tqfx4_router *rt
     if (tq::gate_up_smem(a) > tq::max_smem_optin() || tq::down_smem(a) > tq::max_smem_optin())
         return fail(TQFX4_ESHAPE, "%s: top_k x inter too large for the decode kernels' shared memory", fn);
     tq::moe_decode_args(ex, rt, ws, a, L);
-    cudaError_t e = tq::launch_moe_decode(a, x, out, sel_idx, sel_w, static_cast<cudaStream_t>(stream), events);
+    // (debug build) the stacked experts: E x inter rows of gate and of up, E x hidden rows of down
+    cudaError_t e = debug_validate(ex->gate, ex->n_experts * ex->inter, ex->hidden, ws, stream);
+    if (e == cudaSuccess) e = debug_validate(ex->up, ex->n_experts * ex->inter, ex->hidden, ws, stream);
+    if (e == cudaSuccess) e = debug_validate(ex->down, ex->n_experts * ex->hidden, ex->inter, ws, stream);
+    if (e == cudaSuccess)
+        e = tq::launch_moe_decode(a, x, out, sel_idx, sel_w, static_cast<cudaStream_t>(stream), events);
     if (e != cudaSuccess) return cuda_fail(e, fn);
     return ok();
 }
@@ -448,7 +485,10 @@ static tqfx4_status expert_ffn_impl(const void *gate, const void *up, const void
     if (tq::gate_up_smem(a) > tq::max_smem_optin() || tq::down_smem(a) > tq::max_smem_optin())
         return fail(TQFX4_ESHAPE, "%s: inter too large for the decode kernels' shared memory", fn);
     tq::moe_decode_args(&ex, &rt, ws, a, L);
-    cudaError_t e = tq::launch_expert_ffn(a, x, out, static_cast<cudaStream_t>(stream), events);
+    cudaError_t e = debug_validate(gate, inter, hidden, ws, stream);
+    if (e == cudaSuccess) e = debug_validate(up, inter, hidden, ws, stream);
+    if (e == cudaSuccess) e = debug_validate(down, hidden, inter, ws, stream);
+    if (e == cudaSuccess) e = tq::launch_expert_ffn(a, x, out, static_cast<cudaStream_t>(stream), events);
     if (e != cudaSuccess) return cuda_fail(e, fn);
     return ok();
 }
@@ -616,7 +656,11 @@ static tqfx4_status moe_grouped_impl(const tqfx4_experts *ex, const tqfx4_router
     tq::grouped_args(ex, rt, T, ws, a, L);
     // The tensor-core contraction pays off once the chunks are mostly full.
     a.tc = path == TQFX4_PATH_PREFILL || (path == TQFX4_PATH_AUTO && T * rt->top_k >= tq::kTcMinPairs);
-    cudaError_t e = tq::launch_moe_grouped(a, X, OUT, sel_idx, sel_w, static_cast<cudaStream_t>(stream), events);
+    cudaError_t e = debug_validate(ex->gate, ex->n_experts * ex->inter, ex->hidden, ws, stream);
+    if (e == cudaSuccess) e = debug_validate(ex->up, ex->n_experts * ex->inter, ex->hidden, ws, stream);
+    if (e == cudaSuccess) e = debug_validate(ex->down, ex->n_experts * ex->hidden, ex->inter, ws, stream);
+    if (e == cudaSuccess)
+        e = tq::launch_moe_grouped(a, X, OUT, sel_idx, sel_w, static_cast<cudaStream_t>(stream), events);
     if (e != cudaSuccess) return cuda_fail(e, fn);
     return ok();
 }

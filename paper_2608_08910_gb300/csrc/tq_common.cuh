@@ -50,8 +50,19 @@ constexpr int QS_STRIDE = 264;    // shared-memory stride of one 256-byte activa
 enum KernelId : int {
     K_PACK = 1, K_QUANT = 2, K_GEMV = 3, K_ROUTER = 4, K_GATEUP = 5, K_DOWN = 6,
     K_TOPK = 7, K_GROUP = 8, K_GGATEUP = 9, K_GDOWN = 10, K_COMBINE = 11, K_PREFILL = 12,
-    K_SELFTEST = 13,
+    K_SELFTEST = 13, K_VALIDATE = 14,
 };
+
+// Checks of data-dependent indices inside the kernels, compiled in by the
+// debug build (-DTQFX4_DEBUG, libtqfx4_debug.so): a failed check records
+// TQFX4_EDATA with the kernel and `detail`, and the caller then keeps its
+// access in bounds instead of faulting. The release build compiles them out.
+#ifdef TQFX4_DEBUG
+#define TQ_DEBUG_CHECK(cond, status, kernel, detail) \
+    ((cond) ? true : (::tq::report((status), TQFX4_EDATA, (kernel), (detail)), false))
+#else
+#define TQ_DEBUG_CHECK(cond, status, kernel, detail) true
+#endif
 
 // Roughly two seconds at the GB300's 2 GHz clock: any mbarrier wait longer
 // than this is treated as lost, reported, and abandoned.

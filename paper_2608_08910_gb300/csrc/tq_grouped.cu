@@ -734,7 +734,8 @@ __global__ void __launch_bounds__((GG_CW + 1) * 32, 1)
 // Gather the quantized hidden state of each pair's token into pair order.
 __global__ void __launch_bounds__(256) gather_rows_kernel(GroupedArgs a) {
     const int64_t pos = blockIdx.x;
-    const int64_t t = __ldcg(a.pair_token + pos);
+    int64_t t = __ldcg(a.pair_token + pos);
+    if (!TQ_DEBUG_CHECK(t >= 0 && t < a.T, a.status, K_GROUP, static_cast<int>(pos))) t = 0;
     const uint4 *src = reinterpret_cast<const uint4 *>(a.qx + t * a.H);
     uint4 *dst = reinterpret_cast<uint4 *>(a.xg + pos * a.H);
     for (int i = threadIdx.x; i < a.H / 16; i += blockDim.x) dst[i] = __ldcg(src + i);
@@ -774,7 +775,8 @@ __global__ void __launch_bounds__(256) gather_tc_kernel(GroupedArgs a) {
     const int lane = threadIdx.x & 31, n16 = a.H / 16;
     for (int n = n0 + (threadIdx.x >> 5); n < m && n < n0 + GT_PAIRS; n += blockDim.x >> 5) {
         const int64_t pos = pb + n;
-        const int64_t t = __ldcg(a.pair_token + pos);
+        int64_t t = __ldcg(a.pair_token + pos);
+        if (!TQ_DEBUG_CHECK(t >= 0 && t < a.T, a.status, K_GROUP, static_cast<int>(pos))) t = 0;
 #pragma unroll
         for (int pl = 0; pl < 2; ++pl) {
             const uint4 *src = reinterpret_cast<const uint4 *>(a.xqt + pl * tplane + t * a.H);
@@ -859,7 +861,9 @@ __global__ void __launch_bounds__(256) combine_kernel(GroupedArgs a) {
     __shared__ int pos[TQFX4_MAX_TOP_K];
     __shared__ float w[TQFX4_MAX_TOP_K];
     if (threadIdx.x < k) {
-        pos[threadIdx.x] = __ldcg(a.pair_of + static_cast<int64_t>(t) * k + threadIdx.x);
+        int p = __ldcg(a.pair_of + static_cast<int64_t>(t) * k + threadIdx.x);
+        if (!TQ_DEBUG_CHECK(p >= 0 && p < a.P, a.status, K_COMBINE, t)) p = 0;
+        pos[threadIdx.x] = p;
         w[threadIdx.x] = __ldcg(a.selw + static_cast<int64_t>(t) * k + threadIdx.x);
     }
     __syncthreads();

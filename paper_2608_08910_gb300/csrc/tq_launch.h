@@ -15,6 +15,7 @@ cudaError_t allow_max_smem(const void *kernel, unsigned char *flags);
 
 cudaError_t launch_pack(int src, const void *a, const int8_t *t2, const uint16_t *scales, int64_t n, int64_t k,
                         void *blocks, int *status, cudaStream_t st);
+cudaError_t launch_validate(const void *blocks, int64_t n, int64_t k, int *status, cudaStream_t st);
 cudaError_t launch_quantize(const float *x, int64_t m, int64_t k, int8_t *q, float *da, int32_t *bsum,
                             int *status, cudaStream_t st);
 cudaError_t launch_gemv_x(const void *blocks, int64_t n, int64_t k, const float *x, int8_t *q, float *da,

@@ -134,7 +134,11 @@ __global__ void __launch_bounds__(256, 1) gate_up_kernel(MoeArgs a) {
     // would queue ahead in the memory system
     ActRegs act;
     if (!a.single) act_load(a.qx, a.dx, a.bx, nbh, act);
-    if (threadIdx.x < a.top_k) sel_s[threadIdx.x] = a.single ? 0 : __ldcg(a.sel + threadIdx.x);
+    if (threadIdx.x < a.top_k) {
+        int e = a.single ? 0 : __ldcg(a.sel + threadIdx.x);
+        if (!TQ_DEBUG_CHECK(e >= 0 && e < a.E, a.status, K_GATEUP, -2)) e = 0;
+        sel_s[threadIdx.x] = e;
+    }
     if (a.ptrs && threadIdx.x < 2 * a.top_k) ptr_s[threadIdx.x] = a.ptrs[threadIdx.x];
     __syncthreads();
     const int64_t n_rg = a.I / 4;
@@ -218,7 +222,8 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
     ring_init(ring);
     fence_barrier_init();
     const int j = blockIdx.x / a.parts_d, p = blockIdx.x - j * a.parts_d;
-    const int64_t e = (a.ptrs || a.single) ? 0 : __ldcg(a.sel + j);
+    int64_t e = (a.ptrs || a.single) ? 0 : __ldcg(a.sel + j);
+    if (!TQ_DEBUG_CHECK(e >= 0 && e < a.E, a.status, K_DOWN, -2)) e = 0;
     const int64_t n_rg = a.H / 4;
     MatJob job;
     job.mat = a.ptrs ? a.ptrs[2 * K + j] : a.down + e * a.mb_d;

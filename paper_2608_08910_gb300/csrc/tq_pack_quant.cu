@@ -165,6 +165,40 @@ cudaError_t launch_pack(int src, const void *a, const int8_t *t2, const uint16_t
     return cudaGetLastError();
 }
 
+// One warp per block of the matrix: its 512 code bytes (16 a lane, four
+// 32-bit words at 4-byte alignment) must hold nibbles 0..8, and lanes 0-3
+// check the four f16 row scales are finite. A bad block records TQFX4_EDATA
+// with its index.
+__global__ void __launch_bounds__(256) validate_kernel(const uint8_t *__restrict__ blocks, int64_t nblocks,
+                                                       int *status) {
+    const int64_t blk = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (blk >= nblocks) return;  // whole warps
+    const uint8_t *b = blocks + blk * BLOCK_BYTES;
+    const uint32_t *w = reinterpret_cast<const uint32_t *>(b + CODE_OFS + 16 * lane);
+    uint32_t bad = 0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        // per byte, u + 0x77 reaches bit 7 exactly when the nibble u is 9..15
+        const uint32_t x = __ldg(w + i);
+        bad |= ((x & 0x0f0f0f0fu) + 0x77777777u | ((x >> 4) & 0x0f0f0f0fu) + 0x77777777u) & 0x80808080u;
+    }
+    if (lane < ROWS) {  // f16 exponent all ones: infinity or NaN
+        const uint16_t h = __ldg(reinterpret_cast<const unsigned short *>(b) + lane);
+        bad |= (h & 0x7C00u) == 0x7C00u;
+    }
+    if (__any_sync(0xffffffffu, bad != 0) && lane == 0)
+        report(status, TQFX4_EDATA, K_VALIDATE, static_cast<int>(imin64(blk, 0x7fffffff)));
+}
+
+cudaError_t launch_validate(const void *blocks, int64_t n, int64_t k, int *status, cudaStream_t st) {
+    const int64_t nblocks = (n / ROWS) * (k / QK);
+    if (nblocks == 0) return cudaSuccess;
+    const int64_t grid = (nblocks * 32 + 255) / 256;
+    validate_kernel<<<static_cast<unsigned>(grid), 256, 0, st>>>(static_cast<const uint8_t *>(blocks), nblocks, status);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_quantize(const float *x, int64_t m, int64_t k, int8_t *q, float *da, int32_t *bsum,
                             int *status, cudaStream_t st) {
     const int nb = static_cast<int>(k / QK);

@@ -158,20 +158,12 @@ __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::
         "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]),   \
         "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]),   \
         "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
-#define TC_W32(r)                                                                                                    \
-    "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),      \
-        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),       \
-        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),      \
-        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
 #define TC_LIST32                                                                                                    \
     "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,"  \
     "%30,%31}"
 
-// 32 TMEM lanes x 32 columns of 32 bits: the calling thread's lane, columns
-// taddr .. taddr + 31.
-__device__ __forceinline__ void tc_ld32(uint32_t taddr, uint32_t (&r)[32]) {
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 " TC_LIST32 ", [%32];" : TC_W32(r) : "r"(taddr));
-}
+// TMEM loads and stores of 32 lanes x 16 or 32 columns of 32 bits: each
+// thread of the warp its own lane, columns taddr .. taddr + 15 (or 31).
 __device__ __forceinline__ void tc_ld16(uint32_t taddr, uint32_t (&r)[16]) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
@@ -401,6 +393,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         const int e = t.y;
         const int pb = t.z;
         const int m = t.w;
+        // every role reads the same record, so all skip a bad one alike
+        if (!TQ_DEBUG_CHECK(e >= 0 && e < a.E && m >= 1 && m <= TC_CHUNK && pb >= 0 && pb + m <= a.P, a.status,
+                            K_PREFILL, ci))
+            continue;
         const int n_rg = J.N / 4;
         const int rg0 = static_cast<int>(tl) * TC_RG;
         const int nb = J.nb;

@@ -55,6 +55,16 @@ def test_matrix_bytes_match_the_format(lib):
     assert lib.tqfx4_matrix_bytes(4, 100) < 0  # k not a multiple of 256
 
 
+def test_debug_library_builds_and_exports_the_same_functions():
+    # the TQFX4_DEBUG variant (format validation in the entry points, index
+    # checks in the kernels) compiles for sm_103a and carries the whole ABI
+    from paper_2608_08910_gb300 import build
+    path = build.build(debug=True)
+    raw = C.CDLL(path)
+    missing = [n for n in declared_functions() if not hasattr(raw, n)]
+    assert not missing, missing
+
+
 def test_status_strings(lib):
     for code, name in B.STATUS_NAMES.items():
         assert lib.tqfx4_status_string(code).decode() == name
@@ -128,6 +138,9 @@ def test_host_validation_rejects_bad_arguments(lib):
     assert lib.tqfx4_expert_ffn_host_workspace_bytes(4000, 2048) == 0
     assert lib.tqfx4_expert_ffn_host(None, None, None, 4000, 2048, None, None, None, 0, None) == 2
     assert lib.tqfx4_expert_ffn_host(None, None, None, 4096, 2048, None, None, None, 0, None) == 1
+    # the format check: shapes, then the workspace, then NULL blocks
+    assert lib.tqfx4_validate_blocks(None, 6, 256, None, 0, None) == 2
+    assert lib.tqfx4_validate_blocks(None, 4, 256, None, 0, None) == 1
     assert lib.tqfx4_pack(7, None, None, None, 4, 256, None, None, 0, None) == 1  # unknown source kind
     ex, rt = shapes()
     assert lib.tqfx4_moe_ffn(C.byref(ex), C.byref(rt), None, None, None, None, None, 0, None) == 1
