@@ -410,6 +410,29 @@ tqfx4_status tqfx4_moe_grouped(const tqfx4_experts *ex, const tqfx4_router *rt,
                                int32_t *sel_idx, float *sel_w, int path,
                                void *ws, size_t ws_bytes, void *stream);
 
+/* Workspace bytes for tqfx4_moe_grouped_host with `tokens` tokens on `path`:
+ * tqfx4_moe_grouped's layout followed by staging for X, OUT and the
+ * selection. 0 if the shapes are invalid or tokens < 1. */
+size_t tqfx4_moe_grouped_host_workspace_bytes(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t tokens,
+                                              int path);
+
+/*
+ * tqfx4_moe_grouped_host -- tqfx4_moe_grouped with X, OUT (fp32 [T][hidden])
+ * and, when their pointers are not NULL, sel_idx (int32 [T][top_k]) and
+ * sel_w (fp32 [T][top_k]) in host memory, ordered on `stream`. Page-locked
+ * buffers (X and OUT 16-byte aligned, the selection 4-byte aligned) are used
+ * in place: a copy kernel reads X into the workspace's staging, and the
+ * combine and the top-k write OUT and the selection straight into host
+ * memory; pageable or unaligned buffers go through the staging with one
+ * cudaMemcpyAsync each. Returns once enqueued; the outputs are complete after
+ * the stream has passed the call. Results equal tqfx4_moe_grouped's bit for
+ * bit. Workspace: tqfx4_moe_grouped_host_workspace_bytes. T == 0 does
+ * nothing.
+ */
+tqfx4_status tqfx4_moe_grouped_host(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X_host,
+                                    int64_t T, float *OUT_host, int32_t *sel_idx_host, float *sel_w_host, int path,
+                                    void *ws, size_t ws_bytes, void *stream);
+
 /*
  * tqfx4_moe_ffn_noalloc -- tqfx4_moe_ffn without a caller workspace, for
  * callers that cannot allocate device memory: for example a plug-in whose

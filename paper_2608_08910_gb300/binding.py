@@ -67,6 +67,9 @@ _SIGS = {
     "tqfx4_moe_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int]),
     "tqfx4_moe_ffn": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_validate_blocks": (_int, [_vp, _i64, _i64, _vp, _sz, _vp]),
+    "tqfx4_moe_grouped_host": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _i64, _vp, _vp, _vp, _int,
+                                      _vp, _sz, _vp]),
+    "tqfx4_moe_grouped_host_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int]),
     "tqfx4_moe_ffn_host": (_int, [C.POINTER(CExperts), C.POINTER(CRouter), _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_gemv_x_host": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_gemv_x_host_workspace_bytes": (_sz, [_i64, _i64]),
@@ -223,6 +226,17 @@ def tqfx4_validate_blocks(blocks, n, k, ws, stream=None):
     """Checks the format of an n x k matrix (nibbles 0..8, finite scales); a
     violation shows in tqfx4_check(ws) as TQFX4_EDATA."""
     _check(lib().tqfx4_validate_blocks(_p(blocks), n, k, _p(ws), _nbytes(ws), _s(stream)), "tqfx4_validate_blocks")
+
+
+def tqfx4_moe_grouped_host_workspace_bytes(ex: CExperts, rt: CRouter, tokens: int, path: int = 0) -> int:
+    return int(lib().tqfx4_moe_grouped_host_workspace_bytes(C.byref(ex), C.byref(rt), tokens, path))
+
+
+def tqfx4_moe_grouped_host(ex, rt, X, T, OUT, sel_idx, sel_w, path, ws, stream=None):
+    """X, OUT, sel_idx, sel_w: CPU tensors (page-locked: used in place);
+    sel_idx and sel_w may be None. Complete once `stream` has passed the call."""
+    _check(lib().tqfx4_moe_grouped_host(C.byref(ex), C.byref(rt), _p(X), T, _p(OUT), _p(sel_idx), _p(sel_w), path,
+                                        _p(ws), _nbytes(ws), _s(stream)), "tqfx4_moe_grouped_host")
 
 
 def tqfx4_gemv_x_host_workspace_bytes(n: int, k: int) -> int:

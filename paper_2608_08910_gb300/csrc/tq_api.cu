@@ -672,6 +672,71 @@ tqfx4_status tqfx4_moe_grouped(const tqfx4_experts *ex, const tqfx4_router *rt, 
     return moe_grouped_impl(ex, rt, X, T, OUT, sel_idx, sel_w, path, ws, ws_bytes, stream, nullptr);
 }
 
+// Staging of tqfx4_moe_grouped_host after the grouped layout: X, OUT, the selection.
+struct GroupedStaging {
+    size_t x, out, sel, selw, total;
+};
+static GroupedStaging grouped_staging(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T) {
+    GroupedStaging g;
+    const size_t th = 4 * static_cast<size_t>(T) * ex->hidden, tk = 4 * static_cast<size_t>(T) * rt->top_k;
+    size_t off = tq::align256(tq::moe_layout(ex->n_experts, ex->hidden, ex->inter, rt->top_k, T, true, true).total);
+    g.x = off;
+    off = tq::align256(off + th);
+    g.out = off;
+    off = tq::align256(off + th);
+    g.sel = off;
+    off = tq::align256(off + tk);
+    g.selw = off;
+    g.total = tq::align256(off + tk);
+    return g;
+}
+
+size_t tqfx4_moe_grouped_host_workspace_bytes(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t tokens,
+                                              int path) {
+    (void)path;
+    if (check_moe_shapes(ex, rt, "tqfx4_moe_grouped_host_workspace_bytes") || tokens < 1) return 0;
+    return grouped_staging(ex, rt, tokens).total;
+}
+
+tqfx4_status tqfx4_moe_grouped_host(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X_host,
+                                    int64_t T, float *OUT_host, int32_t *sel_idx_host, float *sel_w_host, int path,
+                                    void *ws, size_t ws_bytes, void *stream) {
+    TQ_RANGE();
+    const char *fn = "tqfx4_moe_grouped_host";
+    tqfx4_status s = check_moe_shapes(ex, rt, fn);
+    if (s) return s;
+    if (T < 0) return fail(TQFX4_EINVAL, "%s: negative token count", fn);
+    if (T == 0) return ok();
+    if ((s = check_moe_ptrs(ex, rt, fn))) return s;
+    if (!X_host || !OUT_host) return fail(TQFX4_EINVAL, "%s: NULL X or OUT", fn);
+    const GroupedStaging g = grouped_staging(ex, rt, T);
+    if ((s = check_ws(ws, ws_bytes, g.total, fn))) return s;
+    uint8_t *b = static_cast<uint8_t *>(ws);
+    float *xd = reinterpret_cast<float *>(b + g.x), *od = reinterpret_cast<float *>(b + g.out);
+    int32_t *sd = reinterpret_cast<int32_t *>(b + g.sel);
+    float *wd = reinterpret_cast<float *>(b + g.selw);
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t th = 4 * static_cast<size_t>(T) * ex->hidden, tk = 4 * static_cast<size_t>(T) * rt->top_k;
+    // page-locked buffers in place: a copy kernel reads X into the staging
+    // (every router and gather CTA reads it), and the combine and the top-k
+    // write OUT and the selection straight into host memory
+    const float *xm = static_cast<const float *>(mapped(X_host, 16));
+    float *om = static_cast<float *>(mapped(OUT_host, 16));
+    int32_t *sm = static_cast<int32_t *>(mapped(sel_idx_host, 4));
+    float *wm = static_cast<float *>(mapped(sel_w_host, 4));
+    cudaError_t e = xm ? tq::launch_copy_f32(xd, xm, T * ex->hidden, st)
+                       : cudaMemcpyAsync(xd, X_host, th, cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    if ((s = moe_grouped_impl(ex, rt, xd, T, om ? om : od, sm ? sm : sd, wm ? wm : wd, path, ws, ws_bytes, stream,
+                              nullptr)))
+        return s;
+    if (!om) e = cudaMemcpyAsync(OUT_host, od, th, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && sel_idx_host && !sm) e = cudaMemcpyAsync(sel_idx_host, sd, tk, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && sel_w_host && !wm) e = cudaMemcpyAsync(sel_w_host, wd, tk, cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
 tqfx4_status tqfx4_moe_grouped_traced(const tqfx4_experts *ex, const tqfx4_router *rt, const float *X, int64_t T,
                                       float *OUT, int32_t *sel_idx, float *sel_w, int path, void *ws,
                                       size_t ws_bytes, void *stream, void *const *events) {

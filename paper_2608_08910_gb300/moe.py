@@ -146,6 +146,21 @@ class MoeLayer:
         B.tqfx4_moe_grouped(self.ex, self.rt, X, T, OUT, sel_idx, sel_w, path, ws, stream, events)
         return OUT, sel_idx, sel_w
 
+    def grouped_host_workspace(self, tokens: int, path: int = 0) -> torch.Tensor:
+        """The workspace of grouped_host (device memory)."""
+        n = B.tqfx4_moe_grouped_host_workspace_bytes(self.ex, self.rt, tokens, path)
+        if n == 0:
+            raise ValueError("invalid MoE shapes")
+        return torch.zeros(n, dtype=torch.uint8, device=self.gate.device)
+
+    def grouped_host(self, X, ws, OUT, sel_idx=None, sel_w=None, path=0, stream=None):
+        """grouped with X and the outputs in host memory (CPU tensors,
+        page-locked ones used in place); complete once `stream` has passed it."""
+        if self.fmt != "fx4":
+            raise ValueError("the grouped path serves tq2_0_fx4 experts")
+        B.tqfx4_moe_grouped_host(self.ex, self.rt, X, X.shape[0], OUT, sel_idx, sel_w, path, ws, stream)
+        return OUT, sel_idx, sel_w
+
     def view(self, ws, name, dtype, shape, tokens=1, grouped=0, path=0):
         """A typed view of one intermediate the last call left in `ws`."""
         off = B.tqfx4_moe_workspace_views(self.ex, self.rt, tokens, grouped, path)[name]

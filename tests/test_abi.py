@@ -138,6 +138,15 @@ def test_host_validation_rejects_bad_arguments(lib):
     assert lib.tqfx4_expert_ffn_host_workspace_bytes(4000, 2048) == 0
     assert lib.tqfx4_expert_ffn_host(None, None, None, 4000, 2048, None, None, None, 0, None) == 2
     assert lib.tqfx4_expert_ffn_host(None, None, None, 4096, 2048, None, None, None, 0, None) == 1
+    # the host-buffer grouped call
+    exg, rtg = shapes()
+    ng = lib.tqfx4_moe_grouped_host_workspace_bytes(C.byref(exg), C.byref(rtg), 64, 0)
+    assert ng >= lib.tqfx4_moe_workspace_bytes(C.byref(exg), C.byref(rtg), 64, 0) + 2 * 64 * 4096 * 4
+    assert lib.tqfx4_moe_grouped_host_workspace_bytes(C.byref(exg), C.byref(rtg), 0, 0) == 0
+    assert lib.tqfx4_moe_grouped_host(C.byref(exg), C.byref(rtg), None, 0, None, None, None, 0, None, 0,
+                                      None) == 0  # no tokens: nothing to do
+    assert lib.tqfx4_moe_grouped_host(C.byref(exg), C.byref(rtg), None, -1, None, None, None, 0, None, 0,
+                                      None) == 1
     # the format check: shapes, then the workspace, then NULL blocks
     assert lib.tqfx4_validate_blocks(None, 6, 256, None, 0, None) == 2
     assert lib.tqfx4_validate_blocks(None, 4, 256, None, 0, None) == 1

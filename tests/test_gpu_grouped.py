@@ -142,6 +142,31 @@ def test_tensor_core_path_equals_integer_mma_path():
         assert np.array_equal(a.view(np.uint8), b.view(np.uint8))
 
 
+@pytest.mark.parametrize("kind", ["pinned", "pageable"])
+@pytest.mark.parametrize("path", [B.TQFX4_PATH_DECODE, B.TQFX4_PATH_PREFILL])
+def test_grouped_host_equals_the_device_call(kind, path):
+    # X, OUT and the selection in host memory (page-locked ones used in place:
+    # a copy kernel reads X, the combine and the top-k write into host memory;
+    # pageable ones through staging copies): the device call's bits
+    layer = MoeLayer.synthetic(12, 32, 1024, 512, 6, 1.1, DEV)
+    T = 40
+    X = inputs.hidden_states(12, T, 1024)
+    ws = layer.workspace(T, path)
+    OUT, sel, selw = layer.grouped(X.to(DEV), ws, path)
+    wsh = layer.grouped_host_workspace(T, path)
+    host = (lambda t: t.pin_memory()) if kind == "pinned" else (lambda t: t)
+    Xh = host(X.clone())
+    OUTh = host(torch.zeros(T, 1024))
+    selh, selwh = host(torch.zeros(T, 6, dtype=torch.int32)), host(torch.zeros(T, 6))
+    stream = torch.cuda.current_stream()
+    layer.grouped_host(Xh, wsh, OUTh, selh, selwh, path, stream=stream)
+    stream.synchronize()
+    B.tqfx4_check(wsh)
+    assert torch.equal(OUTh.view(torch.int32), OUT.cpu().view(torch.int32))
+    assert torch.equal(selh, sel.cpu())
+    assert torch.equal(selwh.view(torch.int32), selw.cpu().view(torch.int32))
+
+
 def test_grouped_empty_batch():
     layer = MoeLayer.synthetic(6, 8, 512, 512, 2, 0.0, DEV)
     ws = layer.workspace(1)
