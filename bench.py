@@ -729,8 +729,8 @@ def run_small(args, rank, world, local):
       matrices (269 MB) rotated.
     expert_ffn: one SwiGLU expert, gate/up 4096 -> 2048, down 2048 -> 4096,
       Student-t(5) x 0.02 weights: tqfx4_expert_ffn (the expert alone, no
-      router: gate/up with the quantization of x inside, then down); 21
-      such experts (268 MB) rotated.
+      router: one cooperative launch that holds the expert on chip, with
+      the quantization of x inside); 21 such experts (268 MB) rotated.
     Metric: effective GB/s of the matrices' blocks over the step time. The
     same steps on one resident matrix (hot L2) are reported beside it."""
     import torch
@@ -787,8 +787,8 @@ def run_small(args, rank, world, local):
         def step(i, st=stream, hot=False, ev=None, x=None):
             L = layers[0 if hot else i % M]
             L.expert_ffn(0, X[i % xpool] if x is None else x, ws, out, stream=st, events=ev)
-        launches = 2
-        kern = "gate_up"
+        launches = B.tqfx4_expert_ffn_launches(Hh, Ii)
+        kern = "expert_ffn_kernel (one cooperative launch)" if launches == 1 else "gate_up"
         cfg = {"workload": "expert_ffn_h4096_i2048", "hidden": Hh, "inter": Ii, "expert_bytes": mat,
                "pool_experts": M, "call": "tqfx4_expert_ffn (no router)",
                "l2": "inputs larger than L2: %d distinct experts (%d MB) rotated, a new activation per step"
@@ -838,7 +838,7 @@ def run_small(args, rank, world, local):
     # step, on the launching stream, in plain stream order (the library's
     # traced call records its own stage events; the GEMV steps are not
     # captured, since an event recorded by torch inside a capture does not time)
-    n_ev = launches + 1
+    n_ev = 2 if gemv else 3  # the traced expert call records three events either way
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_ev)] for _ in range(args.steps)]
     for row in evs:
         for e_ in row:
@@ -862,6 +862,9 @@ def run_small(args, rank, world, local):
     stage = [sum(r[s].elapsed_time(r[s + 1]) for r in evs) / args.steps / 1e3 for s in range(n_ev - 1)]
     if gemv:
         names = ["gemv_x"]
+        dom_s, dom_bytes = stage[0], mat
+    elif launches == 1:
+        names = ["expert_ffn"]
         dom_s, dom_bytes = stage[0], mat
     else:
         names = ["gate_up", "down"]
@@ -914,7 +917,10 @@ def run_small(args, rank, world, local):
                      else "fallback 6.8 TB/s",
                      "stage_us": stage_us,
                      "note": ("a single-wave launch of 32 CTAs: bound by latency (launch, one copy round trip), "
-                              "not by HBM" if gemv else "the gate and up projections of one expert")},
+                              "not by HBM" if gemv else
+                              "all three matrices of the expert in one launch: bound by the chain of copy, "
+                              "grid barrier and the two dot passes, not by HBM" if launches == 1
+                              else "the gate and up projections of one expert")},
         "e2e": {"value": job_rate(step_bytes * args.steps, world, te) / 1e9, "unit": "GB/s",
                 "h2d_bytes_per_step": X.shape[1] * 4, "d2h_bytes_per_step": resh.numel() * 4},
         "gpu_launches": launches * args.steps,

@@ -478,12 +478,26 @@ tqfx4_status tqfx4_moe_ffn_noalloc(const tqfx4_experts *ex, const tqfx4_router *
  *   16-byte aligned); out: fp32 [hidden] (device).
  *   ws: at least tqfx4_expert_ffn_workspace_bytes(hidden, inter) bytes,
  *   zeroed once before its first use (0 for invalid shapes: hidden and
- *   inter positive multiples of 256 up to TQFX4_MAX_K). Two launches
- *   (gate/up with the quantization of x inside, then down); a non-finite x
- *   or h sets TQFX4_EDATA. tqfx4_expert_ffn_traced records events[0..2]
- *   before, between and after the two (stages "gate_up", "down").
+ *   inter positive multiples of 256 up to TQFX4_MAX_K), and zeroed again
+ *   after a call that reported TQFX4_ETIMEOUT. A non-finite x or h sets
+ *   TQFX4_EDATA.
+ *   Launches (tqfx4_expert_ffn_launches tells which): one cooperative
+ *   launch of one CTA per SM where the expert fits the SMs' shared memory
+ *   and hidden and inter are multiples of 512 (the 4096 x 2048 expert does):
+ *   each CTA copies its share of all three matrices on chip at its start,
+ *   forms its g, u and h rows, meets the others at a grid-wide barrier
+ *   (bounded wait, TQFX4_ETIMEOUT when it runs out), quantizes h and forms
+ *   its down rows. Otherwise two launches: gate/up with the quantization
+ *   of x inside, then down. tqfx4_expert_ffn_traced records events[0..2]
+ *   before, between and after the two (stages "gate_up", "down"); around
+ *   the one launch it records events[0] before and events[1] and events[2]
+ *   after it.
  */
 size_t tqfx4_expert_ffn_workspace_bytes(int64_t hidden, int64_t inter);
+
+/* Kernel launches tqfx4_expert_ffn makes for these shapes on the current
+ * device: 1 (the cooperative one-launch kernel) or 2; 0 for invalid shapes. */
+int tqfx4_expert_ffn_launches(int64_t hidden, int64_t inter);
 tqfx4_status tqfx4_expert_ffn(const void *gate, const void *up, const void *down,
                               int64_t hidden, int64_t inter, const float *x, float *out,
                               void *ws, size_t ws_bytes, void *stream);

@@ -62,6 +62,7 @@ _SIGS = {
     "tqfx4_gemv": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_gemv_x": (_int, [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_expert_ffn_workspace_bytes": (_sz, [_i64, _i64]),
+    "tqfx4_expert_ffn_launches": (_int, [_i64, _i64]),
     "tqfx4_expert_ffn": (_int, [_vp, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp]),
     "tqfx4_expert_ffn_traced": (_int, [_vp, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _sz, _vp, _vp]),
     "tqfx4_moe_workspace_bytes": (_sz, [C.POINTER(CExperts), C.POINTER(CRouter), _i64, _int]),
@@ -179,6 +180,10 @@ def tqfx4_gemv(blocks, n, k, q, da, bsum, y, block_sums, ws, stream=None):
 
 def tqfx4_expert_ffn_workspace_bytes(hidden, inter):
     return lib().tqfx4_expert_ffn_workspace_bytes(hidden, inter)
+
+
+def tqfx4_expert_ffn_launches(hidden, inter):
+    return int(lib().tqfx4_expert_ffn_launches(hidden, inter))
 
 
 def tqfx4_expert_ffn(gate, up, down, hidden, inter, x, out, ws, stream=None, events=None):

@@ -465,6 +465,17 @@ size_t tqfx4_expert_ffn_workspace_bytes(int64_t hidden, int64_t inter) {
     return tq::moe_layout(1, hidden, inter, 1, 1, false, true).total;
 }
 
+int tqfx4_expert_ffn_launches(int64_t hidden, int64_t inter) {
+    if (tqfx4_expert_ffn_workspace_bytes(hidden, inter) == 0) return 0;
+    const tqfx4_experts ex{nullptr, nullptr, nullptr, 1, hidden, inter};
+    tqfx4_router rt{};
+    rt.top_k = 1;
+    tq::MoeArgs a;
+    tq::MoeLayout L;
+    if (!tq::moe_decode_args(&ex, &rt, nullptr, a, L)) return 0;
+    return tq::expert_ffn_one_launch(a) ? 1 : 2;
+}
+
 static tqfx4_status expert_ffn_impl(const void *gate, const void *up, const void *down, int64_t hidden,
                                     int64_t inter, const float *x, float *out, void *ws, size_t ws_bytes,
                                     void *stream, void *const *events) {

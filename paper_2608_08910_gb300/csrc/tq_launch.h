@@ -54,6 +54,7 @@ cudaError_t launch_moe_mxfp4_experts(const MoeArgs &a, float *out, cudaStream_t 
 cudaError_t launch_moe_route(const MoeArgs &a, const float *x, int32_t *sel_idx, float *sel_w, cudaStream_t st);
 cudaError_t launch_moe_experts(const MoeArgs &a, const void *const *ptrs, float *out, cudaStream_t st);
 cudaError_t launch_expert_ffn(const MoeArgs &a, const float *x, float *out, cudaStream_t st, void *const *events);
+bool expert_ffn_one_launch(const MoeArgs &a);  // launch_expert_ffn takes the one-launch kernel
 
 struct GroupedArgs;
 bool grouped_args(const tqfx4_experts *ex, const tqfx4_router *rt, int64_t T, void *ws, GroupedArgs &a,

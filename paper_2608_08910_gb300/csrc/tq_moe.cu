@@ -324,6 +324,256 @@ __global__ void __launch_bounds__(256, 1) down_kernel(MoeArgs a) {
     TQ_STAMP(2, 5);
 }
 
+// ---------------------------------------------------------------- one expert, one launch
+
+// tqfx4_expert_ffn in one cooperative launch of G CTAs (one per SM, all
+// resident at once). The expert's bytes fit the SMs' shared memory, so
+// every CTA requests its whole share of gate, up and down at its start, one
+// bulk copy and one mbarrier per row group: CTA c owns row groups
+// [c T / G, (c + 1) T / G) of gate and the same of up (T = I / 4), so it
+// forms h = silu(g) u for its rows itself, and [c T' / G, (c + 1) T' / G) of
+// down (T' = H / 4). While the copies fly it quantizes x (every CTA the
+// whole vector); after its g, u and h rows, a grid-wide barrier (bounded)
+// precedes the quantization of h, which every CTA forms for itself from
+// the h rows of all, and the down rows follow from bytes already on chip.
+// Arithmetic, intermediates in the workspace and output are those of the
+// two-launch path (gate_up_kernel, down_kernel with `single`), bit for bit.
+struct FfnGeo {
+    int G;               // CTAs
+    int rg_i, rg_d;      // row groups of gate (= of up), I / 4, and of down, H / 4
+    int max_i, max_d;    // most row groups of gate (= of up) and of down a CTA owns
+    int tb_bytes;        // block terms [row][block] (padded stride), then the row sums
+    int smem;            // dynamic shared memory
+    unsigned long long *arrived;  // grid barrier: CTAs arrived over all calls (8-byte aligned word of the counters)
+};
+
+__device__ __forceinline__ unsigned long long ld_acquire_gpu(const unsigned long long *p) {
+    unsigned long long v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void red_release_gpu(unsigned long long *p, unsigned long long v) {
+    asm volatile("red.release.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+// Grid-wide barrier of G resident CTAs over a 64-bit count of arrivals that
+// only grows (G a call; it never wraps in practice). Every call starts with
+// the count a multiple of G, and a CTA reads it before its own arrival, so
+// target = (count / G + 1) G is this call's full count whatever the other
+// CTAs have done by then. Arrival: one thread, after a CTA barrier, adds 1
+// with release semantics (the CTA's writes before it) and polls with
+// acquire loads until the target; gives up after kWaitBudgetCycles.
+__device__ __forceinline__ unsigned long long grid_barrier_target(const unsigned long long *arrived, int G) {
+    return (ld_acquire_gpu(arrived) / G + 1) * G;
+}
+__device__ __forceinline__ bool grid_barrier(unsigned long long *arrived, unsigned long long target) {
+    red_release_gpu(arrived, 1ull);
+    const long long t0 = clock64();
+    while (ld_acquire_gpu(arrived) < target)
+        if (clock64() - t0 > kWaitBudgetCycles) return false;
+    return true;
+}
+
+// Exact sum S of one row of a block (the row's 128 code bytes at `codes`)
+// against the activation block `qb` with sum `bsum`: block_dot's arithmetic
+// for a single row.
+__device__ __forceinline__ int row_dot(const uint8_t *codes, const uint8_t *qb, int bsum) {
+    const uint2 *c2 = reinterpret_cast<const uint2 *>(codes);
+    const uint2 *q2 = reinterpret_cast<const uint2 *>(qb);
+    int lo0 = 0, lo1 = 0, hi0 = 0, hi1 = 0;  // four chains: integer sums, exact in any order
+#pragma unroll 4
+    for (int w = 0; w < 16; ++w) {
+        const uint2 qa = q2[w], qh = q2[16 + w], c = c2[w];
+        lo0 = dp4a_us(c.x & 0x0f0f0f0fu, qa.x, lo0);
+        lo1 = dp4a_us(c.y & 0x0f0f0f0fu, qa.y, lo1);
+        hi0 = dp4a_us(c.x & 0xf0f0f0f0u, qh.x, hi0);
+        hi1 = dp4a_us(c.y & 0xf0f0f0f0u, qh.y, hi1);
+    }
+    return (lo0 + lo1) + ((hi0 + hi1) >> 4) - 4 * bsum;
+}
+
+// Terms t = float(S) * (d * da) of every (row, block) of the n_rg row
+// groups at `w` into tb[(4 r + row) (nb + 1) + b], one item a thread (the
+// row slowest, so that neighbouring threads read neighbouring blocks); each
+// thread waits for its row group's copy. False if a copy never arrived.
+__device__ __forceinline__ bool ffn_terms(const uint8_t *w, uint64_t *bars, int n_rg, int nb, const uint8_t *qs,
+                                          const float *das, const int *bss, float *tb) {
+    bool ok = true;
+    const int per_row = n_rg * nb, rg_bytes = nb * BLOCK_BYTES;
+    for (int i = threadIdx.x; i < 4 * per_row; i += blockDim.x) {
+        const int rr = i / per_row, rem = i - rr * per_row;
+        const int r = rem / nb, b = rem - r * nb;
+        if (!mbar_wait(&bars[r], 0)) {
+            ok = false;
+            continue;
+        }
+        const uint8_t *blk = w + r * rg_bytes + b * BLOCK_BYTES;
+        const int S = row_dot(blk + CODE_OFS + rr * ROW_BYTES, qs + b * QS_STRIDE, bss[b]);
+        const float sc = __fmul_rn(block_scale(blk, rr), das[b]);
+        tb[(r * 4 + rr) * (nb + 1) + b] = __fmul_rn(static_cast<float>(S), sc);
+    }
+    return ok;
+}
+
+constexpr int FFN_THREADS = 256;  // 512 measured 1.6 % slower at 4096 x 2048 (the copies bind, not the arithmetic)
+
+__global__ void __launch_bounds__(FFN_THREADS, 1) expert_ffn_kernel(MoeArgs a, FfnGeo f) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+    const int nbh = a.nbh, nbi = a.nbi, c = blockIdx.x;
+    const int gu_bytes = nbh * BLOCK_BYTES, d_bytes = nbi * BLOCK_BYTES;  // one row group's
+    uint8_t *wgu = smem;  // this CTA's gate row groups, then the same row groups of up
+    uint8_t *wd = wgu + 2 * f.max_i * gu_bytes;
+    uint8_t *qx = wd + f.max_d * d_bytes;
+    float *dxs = reinterpret_cast<float *>(qx + nbh * QS_STRIDE);
+    int *bxs = reinterpret_cast<int *>(dxs + nbh);
+    uint8_t *qh = qx + act_bytes(nbh);
+    float *dhs = reinterpret_cast<float *>(qh + nbi * QS_STRIDE);
+    int *bhs = reinterpret_cast<int *>(dhs + nbi);
+    float *tb = reinterpret_cast<float *>(qh + act_bytes(nbi));
+    float *ys = tb + (f.tb_bytes / 4 - 8 * f.max_i);  // the g rows, then the u rows
+    uint64_t *bars = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(tb) + f.tb_bytes);
+    __shared__ int ok_s;
+    unsigned long long target = 0;
+    if (tid == 0) target = grid_barrier_target(f.arrived, f.G);
+    const int i0 = static_cast<int>(static_cast<int64_t>(c) * f.rg_i / f.G);
+    const int i1 = static_cast<int>(static_cast<int64_t>(c + 1) * f.rg_i / f.G);
+    const int d0 = static_cast<int>(static_cast<int64_t>(c) * f.rg_d / f.G);
+    const int d1 = static_cast<int>(static_cast<int64_t>(c + 1) * f.rg_d / f.G);
+    const int ni = i1 - i0, ngu = 2 * ni, nd = d1 - d0;
+    if (tid < ngu + nd) mbar_init(&bars[tid], 1);
+    fence_barrier_init();
+    __syncthreads();
+    // x first (its loads would queue behind the weight copies), then every
+    // weight byte of this CTA, one row group a thread: gate/up now, down
+    // once the g and u terms are formed (gate/up's bytes are needed first;
+    // down's still arrive before the grid barrier ends)
+    float4 xv[2][2];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+        const int b = warp + j * nw;
+        if (b < nbh) {
+            const float4 *src = reinterpret_cast<const float4 *>(a.x + b * QK + 8 * lane);
+            xv[j][0] = __ldg(src);
+            xv[j][1] = __ldg(src + 1);
+        }
+    }
+    auto issue = [&](int i) {  // row-group copy i of this CTA: gate, up, then down
+        const uint64_t policy = l2_policy_evict_first();
+        const uint8_t *src;
+        uint8_t *dst;
+        int bytes;
+        if (i < ngu) {
+            const int64_t rg = i0 + (i < ni ? i : i - ni);
+            src = (i < ni ? a.gate : a.up) + rg * gu_bytes;
+            dst = wgu + i * gu_bytes;
+            bytes = gu_bytes;
+        } else {
+            src = a.down + static_cast<int64_t>(d0 + i - ngu) * d_bytes;
+            dst = wd + (i - ngu) * d_bytes;
+            bytes = d_bytes;
+        }
+        mbar_arrive_expect_tx(&bars[i], static_cast<uint32_t>(bytes));
+        bulk_g2s_hint(dst, src, static_cast<uint32_t>(bytes), &bars[i], policy);
+    };
+    if (tid < ngu) issue(tid);
+    __syncwarp();
+    // x quantized per 256-block while the copies fly (the quantizer of
+    // tqfx4_quantize_act); CTA 0 leaves it in the workspace
+    bool finite = true;
+    for (int b = warp, j = 0; b < nbh; b += nw, ++j) {
+        float4 v0, v1;
+        if (j < 2) {
+            v0 = j == 0 ? xv[0][0] : xv[1][0];
+            v1 = j == 0 ? xv[0][1] : xv[1][1];
+        } else {
+            const float4 *src = reinterpret_cast<const float4 *>(a.x + b * QK + 8 * lane);
+            v0 = __ldg(src);
+            v1 = __ldg(src + 1);
+        }
+        const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+        uint2 packed;
+        float d;
+        int sum;
+        finite &= quant_block_warp(v, packed, d, sum);
+        *reinterpret_cast<uint2 *>(qx + b * QS_STRIDE + 8 * lane) = packed;
+        if (lane == 0) {
+            dxs[b] = d;
+            bxs[b] = sum;
+        }
+        if (c == 0) {
+            *reinterpret_cast<uint2 *>(a.qx + b * QK + 8 * lane) = packed;
+            if (lane == 0) {
+                a.dx[b] = d;
+                a.bx[b] = sum;
+            }
+        }
+    }
+    if (!finite && c == 0 && lane == 0) report(a.status, TQFX4_EDATA, K_GATEUP, -1);
+    __syncwarp();
+    __syncthreads();
+    // g and u rows (the terms, then one thread per row adds its blocks in
+    // order), then h = silu(g) u of the same rows
+    bool ok = ffn_terms(wgu, bars, ngu, nbh, qx, dxs, bxs, tb);
+    if (!__syncthreads_and(ok) && tid == 0) report(a.status, TQFX4_ETIMEOUT, K_GATEUP, c);
+    if (tid >= ngu && tid < ngu + nd) issue(tid);
+    __syncwarp();
+    for (int t = tid; t < ngu * 4; t += blockDim.x) {
+        const float *row = tb + t * (nbh + 1);
+        float acc = 0.0f;
+        for (int b = 0; b < nbh; ++b) acc = __fadd_rn(acc, row[b]);
+        ys[t] = acc;
+        const int up = t >= ni * 4;
+        (up ? a.u : a.g)[i0 * 4 + t - up * ni * 4] = acc;
+    }
+    __syncthreads();
+    for (int t = tid; t < ni * 4; t += blockDim.x) a.h[i0 * 4 + t] = tq_swiglu(ys[t], ys[ni * 4 + t]);
+    __syncthreads();
+    if (tid == 0) {
+        ok_s = grid_barrier(f.arrived, target);
+        if (!ok_s) report(a.status, TQFX4_ETIMEOUT, K_DOWN, -3);
+    }
+    __syncthreads();
+    // the quantization of h, one 256-block per warp, in every CTA (its down
+    // rows need all of it); CTA 0 leaves it in the workspace
+    for (int b = warp; b < nbi; b += nw) {
+        const int o = b * QK + 8 * lane;
+        const float4 h0 = __ldcg(reinterpret_cast<const float4 *>(a.h + o));
+        const float4 h1 = __ldcg(reinterpret_cast<const float4 *>(a.h + o) + 1);
+        const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+        uint2 packed;
+        float d;
+        int sum;
+        const bool hok = quant_block_warp(hv, packed, d, sum);
+        *reinterpret_cast<uint2 *>(qh + b * QS_STRIDE + 8 * lane) = packed;
+        if (lane == 0) {
+            dhs[b] = d;
+            bhs[b] = sum;
+        }
+        if (c == 0) {
+            *reinterpret_cast<uint2 *>(a.qh + o) = packed;
+            if (lane == 0) {
+                a.dh[b] = d;
+                a.bh[b] = sum;
+                if (!hok) report(a.status, TQFX4_EDATA, K_DOWN, b);
+            }
+        }
+    }
+    __syncwarp();
+    __syncthreads();
+    // down rows, then out = 0 + 1 * o (the combine of a top-1 layer)
+    ok = ffn_terms(wd, bars + ngu, nd, nbi, qh, dhs, bhs, tb);
+    if (!__syncthreads_and(ok) && tid == 0) report(a.status, TQFX4_ETIMEOUT, K_DOWN, c);
+    for (int t = tid; t < nd * 4; t += blockDim.x) {
+        const float *row = tb + t * (nbi + 1);
+        float acc = 0.0f;
+        for (int b = 0; b < nbi; ++b) acc = __fadd_rn(acc, row[b]);
+        const int n = d0 * 4 + t;
+        a.o[n] = acc;
+        a.out[n] = __fadd_rn(0.0f, __fmul_rn(1.0f, acc));
+    }
+}
+
 // ---------------------------------------------------------------- host side
 
 namespace {
@@ -485,8 +735,47 @@ cudaError_t launch_moe_route(const MoeArgs &a0, const float *x, int32_t *sel_idx
     return cudaGetLastError();
 }
 
-// One expert's FFN without a router: gate/up (x quantized inside) and down
-// as programmatic dependents, events[0..2] (optional) around the two.
+// Geometry of expert_ffn_kernel, or false where it does not apply (the two
+// launches serve the call then): row-group copies 16-byte aligned (an even
+// number of blocks a row), one copy per thread, every share in shared
+// memory. The grid barrier's count takes two of the counter area's last
+// three words, which no other kernel of the one-expert call uses.
+static bool expert_ffn_geo(const MoeArgs &a, FfnGeo &f) {
+    if (a.nbh % 2 != 0 || a.nbi % 2 != 0 || a.n_ctr < kCtrDown + a.parts_d + 3) return false;
+    f.G = num_sms();
+    f.rg_i = a.I / 4;
+    f.rg_d = a.H / 4;
+    f.max_i = (f.rg_i + f.G - 1) / f.G;
+    f.max_d = (f.rg_d + f.G - 1) / f.G;
+    if (2 * f.max_i + f.max_d > FFN_THREADS) return false;
+    const int64_t tb = 4 * (imax64(static_cast<int64_t>(2 * f.max_i) * 4 * (a.nbh + 1),
+                                   static_cast<int64_t>(f.max_d) * 4 * (a.nbi + 1)) +
+                            8 * f.max_i);
+    f.tb_bytes = static_cast<int>((tb + 15) / 16 * 16);
+    const int64_t smem = static_cast<int64_t>(2 * f.max_i) * a.nbh * BLOCK_BYTES +
+                         static_cast<int64_t>(f.max_d) * a.nbi * BLOCK_BYTES + act_bytes(a.nbh) + act_bytes(a.nbi) +
+                         f.tb_bytes + 8 * (2 * f.max_i + f.max_d);
+    if (smem > max_smem_optin() - 1024) return false;  // room for the static shared memory
+    f.smem = static_cast<int>(smem);
+    f.arrived = nullptr;
+    if (a.ctr) {
+        int *w = a.ctr + a.n_ctr - 2;  // the last two counters, or the two before them: 8-byte aligned
+        if (reinterpret_cast<uintptr_t>(w) % 8 != 0) --w;
+        f.arrived = reinterpret_cast<unsigned long long *>(w);
+    }
+    return true;
+}
+
+bool expert_ffn_one_launch(const MoeArgs &a) {
+    FfnGeo f;
+    return expert_ffn_geo(a, f);
+}
+
+// One expert's FFN without a router: one cooperative launch of
+// expert_ffn_kernel where its geometry applies, else gate/up (x quantized
+// inside) and down as programmatic dependents; events[0..2] (optional)
+// before, between and after the two (after the one launch: events[1] and
+// events[2] together).
 cudaError_t launch_expert_ffn(const MoeArgs &a0, const float *x, float *out, cudaStream_t st,
                               void *const *events) {
     MoeArgs a = a0;
@@ -495,10 +784,6 @@ cudaError_t launch_expert_ffn(const MoeArgs &a0, const float *x, float *out, cud
     a.sel_out = nullptr;
     a.selw_out = nullptr;
     a.single = 1;
-    static unsigned char set_gu[64], set_dn[64];
-    cudaError_t e = allow_max_smem(reinterpret_cast<const void *>(gate_up_kernel), set_gu);
-    if (e == cudaSuccess) e = allow_max_smem(reinterpret_cast<const void *>(down_kernel), set_dn);
-    if (e != cudaSuccess) return e;
     cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
     if (events) cudaStreamIsCapturing(st, &cap);
     auto rec = [&](int i) {
@@ -507,6 +792,34 @@ cudaError_t launch_expert_ffn(const MoeArgs &a0, const float *x, float *out, cud
                                      cap == cudaStreamCaptureStatusActive ? cudaEventRecordExternal
                                                                           : cudaEventRecordDefault);
     };
+    cudaError_t e;
+    FfnGeo f;
+    if (expert_ffn_geo(a, f)) {
+        static unsigned char set_ffn[64];
+        if ((e = allow_max_smem(reinterpret_cast<const void *>(expert_ffn_kernel), set_ffn)) != cudaSuccess)
+            return e;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(f.G);
+        cfg.blockDim = dim3(FFN_THREADS);
+        cfg.dynamicSmemBytes = f.smem;
+        cfg.stream = st;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeCooperative;
+        attr[0].val.cooperative = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        void *args[] = {&a, &f};
+        rec(0);
+        if ((e = cudaLaunchKernelExC(&cfg, reinterpret_cast<const void *>(expert_ffn_kernel), args)) != cudaSuccess)
+            return e;
+        rec(1);
+        rec(2);
+        return cudaSuccess;
+    }
+    static unsigned char set_gu[64], set_dn[64];
+    e = allow_max_smem(reinterpret_cast<const void *>(gate_up_kernel), set_gu);
+    if (e == cudaSuccess) e = allow_max_smem(reinterpret_cast<const void *>(down_kernel), set_dn);
+    if (e != cudaSuccess) return e;
     rec(0);
     if ((e = launch_pdl(reinterpret_cast<const void *>(gate_up_kernel), a.top_k * a.parts_gu, a.warps_gu * 32,
                         gate_up_smem(a), st, events != nullptr, a)) != cudaSuccess)

@@ -115,6 +115,12 @@ def test_host_validation_rejects_bad_arguments(lib):
     assert 0 < n1 <= lib.tqfx4_moe_workspace_bytes(C.byref(ex1), C.byref(rt1), 1, 0)
     assert lib.tqfx4_expert_ffn_workspace_bytes(4000, 2048) == 0
     assert lib.tqfx4_expert_ffn_workspace_bytes(4096, 0) == 0
+    # one cooperative launch where the expert fits on chip with even block
+    # counts, else two; 0 for bad shapes
+    assert lib.tqfx4_expert_ffn_launches(4096, 2048) == 1
+    assert lib.tqfx4_expert_ffn_launches(768, 1280) == 2
+    assert lib.tqfx4_expert_ffn_launches(4096, 8192) == 2
+    assert lib.tqfx4_expert_ffn_launches(4000, 2048) == 0
     # the one-launch GEMV takes the chunked pass only: k a multiple of 512
     assert lib.tqfx4_gemv_x(None, 1024, 256, None, None, None, None, None, None, 0, None) == 2
     assert lib.tqfx4_gemv_x(None, 1024, 1280, None, None, None, None, None, None, 0, None) == 2
