@@ -268,6 +268,26 @@ def test_expert_ffn_of_one_expert_of_a_layer(H, I):
         assert np.array_equal(out.cpu().numpy().view(np.uint32), refs[c % 2].view(np.uint32))
 
 
+@pytest.mark.parametrize("H,I,launches", [(4096, 2048, 1), (768, 1280, 2)])
+def test_expert_ffn_traced_and_its_launch_count(H, I, launches):
+    # the traced call (three events on the stream) gives the untraced call's
+    # bits on both paths, and the launch-count query names the path
+    assert B.tqfx4_expert_ffn_launches(H, I) == launches
+    layer = MoeLayer.synthetic(H + 7, 1, H, I, 1, 0.0, DEV)
+    ws = layer.expert_workspace()
+    x = inputs.hidden_states(H + 7, 1, H)[0].to(DEV)
+    ref = layer.expert_ffn(0, x, ws).clone()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    for e in ev:  # torch creates an event's handle at its first record
+        e.record()
+    torch.cuda.synchronize()
+    out = layer.expert_ffn(0, x, ws, events=ev)
+    torch.cuda.synchronize()
+    B.tqfx4_check(ws)
+    assert torch.equal(out.view(torch.int32), ref.view(torch.int32))
+    assert ev[0].elapsed_time(ev[1]) > 0.0 and ev[1].elapsed_time(ev[2]) >= 0.0
+
+
 def test_expert_ffn_reports_nonfinite_input():
     layer = MoeLayer.synthetic(4, 1, 1024, 512, 1, 0.0, DEV)
     ws = layer.expert_workspace()
