@@ -510,7 +510,8 @@ size_t tqfx4_expert_ffn_host_workspace_bytes(int64_t hidden, int64_t inter);
  * tqfx4_expert_ffn_host -- tqfx4_expert_ffn with x and out (fp32 [hidden])
  * in host memory, ordered on `stream`. A page-locked x (16-byte aligned) is
  * read into the staging by a small kernel and a page-locked out (4-byte
- * aligned) is written in place by the down kernel; pageable or unaligned
+ * aligned) is written in place by the kernel that forms the down rows (the
+ * one-launch kernel, or the down kernel of the two); pageable or unaligned
  * buffers go through the staging with one cudaMemcpyAsync each. Returns once
  * enqueued; out is complete after the stream has passed the call. out equals
  * tqfx4_expert_ffn's bit for bit. Errors: as tqfx4_expert_ffn.

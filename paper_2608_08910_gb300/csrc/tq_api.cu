@@ -540,7 +540,8 @@ tqfx4_status tqfx4_expert_ffn_host(const void *gate, const void *up, const void 
     const size_t xo = tq::align256(base), oo = tq::align256(xo + 4 * static_cast<size_t>(hidden));
     float *xd = reinterpret_cast<float *>(b + xo), *od = reinterpret_cast<float *>(b + oo);
     // page-locked buffers in place: a small kernel reads x into the staging
-    // and the down kernel writes out straight into host memory
+    // (once, not by every CTA of the FFN over the host link) and the kernel
+    // that forms the down rows writes out straight into host memory
     const float *xm = static_cast<const float *>(mapped(x_host, 16));
     float *om = static_cast<float *>(mapped(out_host, 4));
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
