@@ -64,6 +64,8 @@ GATE_UP_TRAFFIC = 68200448 + 936704
 # experts and 512 tokens (one chunk per expert, as in the full workload) scaled by the full
 # workload's 4x weight bytes and pairs.
 TC_GATE_UP_TRAFFIC = 4 * (580347392 + 58900992)
+# The same for one expert_ffn_kernel launch (the 4096 -> 2048 -> 4096 expert, one launch).
+EXPERT_FFN_TRAFFIC = 12829440 + 0
 
 
 def max_over_ranks(t, world, device):
@@ -912,7 +914,7 @@ def run_small(args, rank, world, local):
                    "ms_per_step": t_hot / args.steps * 1e3,
                    "note": "the same steps on one resident matrix (L2-resident after the first step)"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                     "traffic": None, "kernel": kern,
+                     "traffic": EXPERT_FFN_TRAFFIC if (not gemv and launches == 1) else None, "kernel": kern,
                      "peak_source": peak_kind + " (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
                      else "fallback 6.8 TB/s",
                      "stage_us": stage_us,
